@@ -1,0 +1,331 @@
+/*
+ * CPU oracle for the trainer -> rollout weight-synchronisation hot path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the tests, the smoke check and the CPU
+ * baseline / reference arm of the benchmark may load this file.  It shares no
+ * code with the CUDA library and is written to be read against its definition,
+ * not to be fast: single thread, scalar, one element at a time.
+ *
+ * What it computes (RobustRL, Section 5.2.1, "UCX-based Weight Update"):
+ *   (1) reshard: the trainer's parameters, held as flat FSDP-style shards, are
+ *       re-laid into the rollout engine's layout (step 1 of that section);
+ *   (2) the rollout holds 16-bit weights (Section 7.4 speaks of the model "in
+ *       FP16 precision"); here the cast is float32 -> bfloat16,
+ *       round-to-nearest-even;
+ *   (3) the model is placed layer by layer into a transfer buffer (step 2);
+ *       here that buffer is a sequence of fixed-size buckets;
+ *   (4) each bucket carries a 64-bit word-sum so that a rollout that
+ *       reconnects after a failure (Section 5.2.2, "Relay server failure
+ *       during pulling", "Trainer failure during pulling") can check what it
+ *       pulled;
+ *   (5) unpack: buckets back to the rollout's tensors; (6) verify.
+ *
+ * The paper prints no layout, byte format or checksum; the definitions below
+ * are the readings this build takes, stated once here:
+ *
+ *  Source.  Parameters are concatenated in manifest order into one flat byte
+ *  buffer; each starts at a multiple of max(align_bytes, element size); gap
+ *  bytes are zero.  The total is padded up to a multiple of 16 * n_shards and
+ *  cut into n_shards equal shards of S bytes: flat byte f lives in shard f / S
+ *  at offset f % S.  A parameter of shape [d0, d1, ...] is viewed as a matrix
+ *  [rows = d0, cols = d1 * d2 * ...] (cols = 1 for a vector).
+ *
+ *  Destination.  A destination tensor is a list of blocks (param, row0, nrows,
+ *  col0, ncols); its elements are the blocks' elements taken block by block,
+ *  each block row by row: element j of a block is the parameter element at
+ *  row row0 + j / ncols, column col0 + j % ncols.
+ *
+ *  Cast.  float32 bits b -> bfloat16: a NaN (|b| > 0x7F800000) keeps its sign
+ *  and top payload with the quiet bit forced, (b >> 16) | 0x0040; any other
+ *  value rounds to nearest, ties to even: (b + 0x7FFF + ((b >> 16) & 1)) >> 16
+ *  (so +-0 and subnormals are kept, overflow carries into +-inf and +-inf map
+ *  to themselves).  A bfloat16 source is copied bit for bit.
+ *
+ *  Stream and buckets.  Each rollout rank r has a byte stream holding its
+ *  destination tensors in the given order, each starting at the next multiple
+ *  of tensor_align; elements are little-endian.  The stream is cut every
+ *  bucket_bytes; the last bucket and all alignment gaps are zero.  Buckets are
+ *  numbered rank-major.
+ *
+ *  Checksum.  cs[b] = sum over k of the little-endian 64-bit word at bytes
+ *  [8k, 8k + 8) of bucket b, modulo 2^64 (bucket_bytes % 8 == 0).
+ */
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+typedef struct {
+    int64_t rows;
+    int64_t cols;
+    int32_t elem_bytes; /* 4: float32, 2: bfloat16 */
+    int32_t pad_;
+} orc_param;
+
+typedef struct {
+    int32_t param;
+    int32_t pad_;
+    int64_t row0, nrows, col0, ncols;
+} orc_block;
+
+typedef struct {
+    int32_t rank;
+    int32_t n_blocks;
+    const orc_block* blocks;
+} orc_tensor;
+
+typedef struct {
+    /* description */
+    int32_t n_params;
+    int32_t n_shards;
+    const orc_param* params;
+    int64_t align_bytes;
+    int32_t n_tensors;
+    int32_t tp;
+    const orc_tensor* tensors;
+    int64_t tensor_align;
+    int64_t bucket_bytes;
+    /* derived by orc_layout_compute(), arrays owned by the caller */
+    int64_t* param_offset;      /* [n_params] flat byte offset of each parameter   */
+    int64_t* tensor_numel;      /* [n_tensors]                                      */
+    int64_t* tensor_offset;     /* [n_tensors] byte offset in its rank's stream     */
+    int64_t* rank_stream_bytes; /* [tp]                                             */
+    int64_t* rank_first_bucket; /* [tp + 1]; rank_first_bucket[tp] = bucket count   */
+    int64_t flat_bytes;         /* end of the last parameter                        */
+    int64_t shard_bytes;        /* S                                                */
+} orc_layout;
+
+/* Where source values come from: real shard buffers, or a generator that maps
+ * an element index (flat byte offset / element size) to its bits. */
+typedef uint32_t (*orc_value_fn)(const void* ctx, int64_t elem_index, int32_t elem_bytes);
+
+typedef struct {
+    const uint8_t* const* shards; /* n_shards host buffers of shard_bytes, or NULL */
+    orc_value_fn gen;             /* used when shards == NULL                       */
+    const void* gen_ctx;
+} orc_source;
+
+enum { ORC_OK = 0, ORC_EINVAL = -1, ORC_ENOMEM = -2, ORC_ESOURCE = -3 };
+
+static int64_t align_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+/* ---------------------------------------------------------------- layout */
+
+int orc_layout_compute(orc_layout* L) {
+    if (L->n_params < 0 || L->n_shards < 1 || L->align_bytes < 1 || L->tp < 1 ||
+        L->n_tensors < 0 || L->tensor_align < 2 || L->tensor_align % 2 != 0 ||
+        L->bucket_bytes < 8 || L->bucket_bytes % 8 != 0)
+        return ORC_EINVAL;
+
+    /* Source: parameters one after another, each aligned. */
+    int64_t off = 0;
+    for (int32_t p = 0; p < L->n_params; ++p) {
+        const orc_param* P = &L->params[p];
+        if (P->rows < 0 || P->cols < 0 || (P->elem_bytes != 2 && P->elem_bytes != 4))
+            return ORC_EINVAL;
+        int64_t a = L->align_bytes > P->elem_bytes ? L->align_bytes : P->elem_bytes;
+        off = align_up(off, a);
+        L->param_offset[p] = off;
+        off += P->rows * P->cols * P->elem_bytes;
+    }
+    L->flat_bytes = off;
+    L->shard_bytes = align_up(off, 16 * (int64_t)L->n_shards) / L->n_shards;
+
+    /* Destination: per-rank streams. */
+    for (int32_t r = 0; r < L->tp; ++r) L->rank_stream_bytes[r] = 0;
+    for (int32_t t = 0; t < L->n_tensors; ++t) {
+        const orc_tensor* T = &L->tensors[t];
+        if (T->rank < 0 || T->rank >= L->tp || T->n_blocks < 0) return ORC_EINVAL;
+        int64_t numel = 0;
+        for (int32_t k = 0; k < T->n_blocks; ++k) {
+            const orc_block* B = &T->blocks[k];
+            if (B->param < 0 || B->param >= L->n_params) return ORC_EINVAL;
+            const orc_param* P = &L->params[B->param];
+            if (B->row0 < 0 || B->nrows < 0 || B->row0 + B->nrows > P->rows) return ORC_EINVAL;
+            if (B->col0 < 0 || B->ncols < 0 || B->col0 + B->ncols > P->cols) return ORC_EINVAL;
+            numel += B->nrows * B->ncols;
+        }
+        int64_t start = align_up(L->rank_stream_bytes[T->rank], L->tensor_align);
+        L->tensor_numel[t] = numel;
+        L->tensor_offset[t] = start;
+        L->rank_stream_bytes[T->rank] = start + 2 * numel;
+    }
+    L->rank_first_bucket[0] = 0;
+    for (int32_t r = 0; r < L->tp; ++r) {
+        int64_t nb = (L->rank_stream_bytes[r] + L->bucket_bytes - 1) / L->bucket_bytes;
+        L->rank_first_bucket[r + 1] = L->rank_first_bucket[r] + nb;
+    }
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------ cast */
+
+uint16_t orc_rne_bf16(uint32_t b) {
+    if ((b & 0x7FFFFFFFu) > 0x7F800000u) return (uint16_t)((b >> 16) | 0x0040u);
+    return (uint16_t)((b + 0x7FFFu + ((b >> 16) & 1u)) >> 16);
+}
+
+void orc_rne_bf16_array(const uint32_t* in, uint16_t* out, int64_t n) {
+    for (int64_t i = 0; i < n; ++i) out[i] = orc_rne_bf16(in[i]);
+}
+
+static uint16_t cast_to_bf16(uint32_t bits, int32_t elem_bytes) {
+    return elem_bytes == 4 ? orc_rne_bf16(bits) : (uint16_t)bits;
+}
+
+/* ---------------------------------------------------------------- source */
+
+static int source_byte(const orc_layout* L, const orc_source* S, int64_t f, uint8_t* out) {
+    int64_t s = f / L->shard_bytes;
+    if (s >= L->n_shards || S->shards[s] == NULL) return ORC_ESOURCE;
+    *out = S->shards[s][f % L->shard_bytes];
+    return ORC_OK;
+}
+
+/* Bits of the element at flat byte offset f (little-endian). */
+static int source_bits(const orc_layout* L, const orc_source* S, int64_t f, int32_t es,
+                       uint32_t* bits) {
+    if (S->shards == NULL) {
+        *bits = S->gen(S->gen_ctx, f / es, es);
+        return ORC_OK;
+    }
+    uint32_t v = 0;
+    for (int32_t i = 0; i < es; ++i) {
+        uint8_t byte;
+        int rc = source_byte(L, S, f + i, &byte);
+        if (rc) return rc;
+        v |= (uint32_t)byte << (8 * i);
+    }
+    *bits = v;
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------- reshard */
+
+/* Elements j0 .. j1-1 of destination tensor t, cast to bfloat16. */
+int orc_tensor_elements(const orc_layout* L, const orc_source* S, int32_t t, int64_t j0,
+                        int64_t j1, uint16_t* out) {
+    const orc_tensor* T = &L->tensors[t];
+    int64_t base = 0; /* index in the tensor of the current block's first element */
+    for (int32_t k = 0; k < T->n_blocks; ++k) {
+        const orc_block* B = &T->blocks[k];
+        const orc_param* P = &L->params[B->param];
+        int64_t n = B->nrows * B->ncols;
+        int64_t lo = j0 > base ? j0 : base;
+        int64_t hi = j1 < base + n ? j1 : base + n;
+        for (int64_t j = lo; j < hi; ++j) {
+            int64_t jj = j - base;
+            int64_t row = B->row0 + jj / B->ncols;
+            int64_t col = B->col0 + jj % B->ncols;
+            int64_t f = L->param_offset[B->param] + (row * P->cols + col) * P->elem_bytes;
+            uint32_t bits;
+            int rc = source_bits(L, S, f, P->elem_bytes, &bits);
+            if (rc) return rc;
+            out[j - j0] = cast_to_bf16(bits, P->elem_bytes);
+        }
+        base += n;
+    }
+    return ORC_OK;
+}
+
+/* The whole of destination tensor t, straight from the source (no buckets). */
+int orc_reshard_tensor(const orc_layout* L, const orc_source* S, int32_t t, uint16_t* out) {
+    return orc_tensor_elements(L, S, t, 0, L->tensor_numel[t], out);
+}
+
+/* ----------------------------------------------------------------- pack */
+
+static int32_t rank_of_bucket(const orc_layout* L, int64_t b) {
+    for (int32_t r = 0; r < L->tp; ++r)
+        if (b < L->rank_first_bucket[r + 1]) return r;
+    return -1;
+}
+
+/* Bucket b's bytes (bucket_bytes of them). */
+int orc_pack_bucket(const orc_layout* L, const orc_source* S, int64_t b, uint8_t* out) {
+    int32_t r = rank_of_bucket(L, b);
+    if (b < 0 || r < 0) return ORC_EINVAL;
+    int64_t lo = (b - L->rank_first_bucket[r]) * L->bucket_bytes;
+    int64_t hi = lo + L->bucket_bytes;
+    memset(out, 0, (size_t)L->bucket_bytes);
+    for (int32_t t = 0; t < L->n_tensors; ++t) {
+        if (L->tensors[t].rank != r) continue;
+        int64_t t_lo = L->tensor_offset[t];
+        int64_t t_hi = t_lo + 2 * L->tensor_numel[t];
+        int64_t a = lo > t_lo ? lo : t_lo;
+        int64_t z = hi < t_hi ? hi : t_hi;
+        if (a >= z) continue;
+        int64_t j0 = (a - t_lo) / 2, j1 = (z - t_lo) / 2;
+        uint16_t* tmp = (uint16_t*)malloc((size_t)(j1 - j0) * 2);
+        if (!tmp) return ORC_ENOMEM;
+        int rc = orc_tensor_elements(L, S, t, j0, j1, tmp);
+        if (rc) {
+            free(tmp);
+            return rc;
+        }
+        for (int64_t j = j0; j < j1; ++j) {
+            int64_t pos = t_lo + 2 * j - lo;
+            out[pos] = (uint8_t)(tmp[j - j0] & 0xFF);
+            out[pos + 1] = (uint8_t)(tmp[j - j0] >> 8);
+        }
+        free(tmp);
+    }
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------- checksum */
+
+uint64_t orc_checksum(const uint8_t* bytes, int64_t n) {
+    uint64_t sum = 0;
+    for (int64_t k = 0; k + 8 <= n; k += 8) {
+        uint64_t word = 0;
+        for (int i = 0; i < 8; ++i) word |= (uint64_t)bytes[k + i] << (8 * i);
+        sum += word;
+    }
+    return sum;
+}
+
+/* Buckets first .. first+count-1 and their checksums, into out (count * bucket_bytes). */
+int orc_pack_range(const orc_layout* L, const orc_source* S, int64_t first, int64_t count,
+                   uint8_t* out, uint64_t* checksums) {
+    for (int64_t i = 0; i < count; ++i) {
+        uint8_t* bucket = out + i * L->bucket_bytes;
+        int rc = orc_pack_bucket(L, S, first + i, bucket);
+        if (rc) return rc;
+        checksums[i] = orc_checksum(bucket, L->bucket_bytes);
+    }
+    return ORC_OK;
+}
+
+/* --------------------------------------------------------------- unpack */
+
+/* Destination tensor t read back out of the buckets (buckets[b] = bucket b's bytes). */
+int orc_unpack_tensor(const orc_layout* L, const uint8_t* const* buckets, int32_t t,
+                      uint16_t* out) {
+    const orc_tensor* T = &L->tensors[t];
+    int64_t first = L->rank_first_bucket[T->rank];
+    for (int64_t j = 0; j < L->tensor_numel[t]; ++j) {
+        int64_t pos = L->tensor_offset[t] + 2 * j;
+        const uint8_t* bucket = buckets[first + pos / L->bucket_bytes];
+        if (bucket == NULL) return ORC_ESOURCE;
+        int64_t o = pos % L->bucket_bytes;
+        out[j] = (uint16_t)(bucket[o] | (bucket[o + 1] << 8));
+    }
+    return ORC_OK;
+}
+
+/* --------------------------------------------------------------- verify */
+
+/* Number of buckets whose recomputed checksum differs from checksums[b]; the
+ * first such index in *first_bad (-1 if none). */
+int64_t orc_verify(const orc_layout* L, const uint8_t* const* buckets, const uint64_t* checksums,
+                   int64_t first, int64_t count, int64_t* first_bad) {
+    int64_t bad = 0;
+    *first_bad = -1;
+    for (int64_t b = first; b < first + count; ++b) {
+        if (orc_checksum(buckets[b], L->bucket_bytes) != checksums[b]) {
+            if (bad == 0) *first_bad = b;
+            ++bad;
+        }
+    }
+    return bad;
+}

@@ -1,0 +1,295 @@
+"""Pins for the oracle's source addressing, reshard, stream/bucket cut, checksum,
+unpack and verify (RobustRL Section 5.2.1 steps 1-2 and Section 5.2.2).
+
+The paper prints no worked example for this path, so the oracle is pinned by:
+* a hand-worked example (tests/golden/layout_worked_example.json);
+* a PyTorch restatement of the rollout layout (vLLM-style cat/chunk/stack on
+  whole parameter tensors, then byte-level concatenation into streams and
+  buckets) on scaled-down workloads of every family;
+* invariants: shard-count invariance, coverage counts, unpack(pack) = reshard,
+  checksum linearity, numpy's wrapping uint64 sum.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from oracle import qwen3
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "layout_worked_example.json")
+
+
+def _int(x):
+    return int(x, 16) if isinstance(x, str) else int(x)
+
+
+# ---------------------------------------------------------------------------
+# Hand-worked example
+# ---------------------------------------------------------------------------
+
+def _golden_layout():
+    g = json.load(open(GOLDEN))
+    params = [(p["name"], tuple(p["dims"]), p["elem_bytes"]) for p in g["params"]]
+    tensors = [(t["name"], t["rank"], [tuple(b) for b in t["blocks"]]) for t in g["tensors"]]
+    L = oracle.Layout(params, tensors, n_shards=g["n_shards"], tp=g["tp"],
+                      bucket_bytes=g["bucket_bytes"], align_bytes=g["align_bytes"],
+                      tensor_align=g["tensor_align"])
+    # Build the flat source by hand from the expected offsets, then cut it.
+    e = g["expect"]
+    flat = bytearray(e["shard_bytes"] * g["n_shards"])
+    for p, off in zip(g["params"], e["param_offset"]):
+        for k, v in enumerate(p["bits"]):
+            flat[off + k * p["elem_bytes"]: off + (k + 1) * p["elem_bytes"]] = \
+                _int(v).to_bytes(p["elem_bytes"], "little")
+    S = e["shard_bytes"]
+    shards = [np.frombuffer(bytes(flat[s * S:(s + 1) * S]), np.uint8)
+              for s in range(g["n_shards"])]
+    return g, L, shards
+
+
+def test_golden_layout_numbers():
+    g, L, _ = _golden_layout()
+    e = g["expect"]
+    assert list(L.param_offset) == e["param_offset"]
+    assert L.flat_bytes == e["flat_bytes"]
+    assert L.shard_bytes == e["shard_bytes"]
+    assert list(L.tensor_numel) == e["tensor_numel"]
+    assert list(L.tensor_offset) == e["tensor_offset"]
+    assert list(L.rank_stream_bytes) == e["rank_stream_bytes"]
+    assert list(L.rank_first_bucket) == e["rank_first_bucket"]
+
+
+def test_golden_values():
+    g, L, shards = _golden_layout()
+    e = g["expect"]
+    src = oracle.Source(shards=shards)
+    for t, want in enumerate(e["tensors_bf16"]):
+        np.testing.assert_array_equal(L.reshard_tensor(src, t),
+                                      np.array([_int(x) for x in want], np.uint16))
+    buckets, cs = L.pack(src)
+    for b, hx in enumerate(e["buckets_hex"]):
+        assert buckets[b].tobytes().hex() == hx
+    assert [int(c) for c in cs] == [_int(c) for c in e["checksums"]]
+
+
+# ---------------------------------------------------------------------------
+# PyTorch restatement of the rollout layout
+# ---------------------------------------------------------------------------
+
+def _param_tensors(params, flat_offsets, seed, specials):
+    """Whole parameter tensors (as integer bit patterns) for the generator's values."""
+    out = {}
+    for (name, dims, es), off in zip(params, flat_offsets):
+        n = int(np.prod(dims))
+        vals = synth.values_host(n, es, seed, first_idx=off // es, specials=specials)
+        t = torch.from_numpy(vals.view(np.int32 if es == 4 else np.int16).copy())
+        out[name] = t.view(*dims)
+    return out
+
+
+def _flat_offsets(params, align=16):
+    offs, off = [], 0
+    for _, dims, es in params:
+        a = max(align, es)
+        off = (off + a - 1) // a * a
+        offs.append(off)
+        off += int(np.prod(dims)) * es
+    return offs
+
+
+def _to_bf16_bits(t: torch.Tensor) -> torch.Tensor:
+    """fp32 bit patterns -> bf16 bit patterns: PyTorch's conversion for numbers, the
+    stated NaN rule for NaNs; a bf16 source passes through."""
+    if t.dtype == torch.int16:
+        return t
+    conv = t.view(torch.float32).to(torch.bfloat16).view(torch.int16)
+    u = t.to(torch.int64) & 0xFFFFFFFF
+    nan = (u & 0x7FFFFFFF) > 0x7F800000
+    nan_bits = ((u >> 16) | 0x40).to(torch.int32).to(torch.int16)
+    return torch.where(nan, nan_bits, conv)
+
+
+def restate_rollout(shape, P, tp):
+    """Per rank, the rollout tensors built the way an inference engine's loader would."""
+    H = shape.hidden
+    ranks = []
+    for r in range(tp):
+        ts = [P["model.embed_tokens.weight"].chunk(tp, 0)[r]]
+        for i in range(shape.layers):
+            pre = f"model.layers.{i}."
+            a = pre + "self_attn."
+            ts.append(torch.cat([P[a + "q_proj.weight"].chunk(tp, 0)[r],
+                                 P[a + "k_proj.weight"].chunk(tp, 0)[r],
+                                 P[a + "v_proj.weight"].chunk(tp, 0)[r]], 0))
+            ts.append(P[a + "o_proj.weight"].chunk(tp, 1)[r])
+            ts.append(P[a + "q_norm.weight"])
+            ts.append(P[a + "k_norm.weight"])
+            ts.append(P[pre + "input_layernorm.weight"])
+            ts.append(P[pre + "post_attention_layernorm.weight"])
+            if shape.n_experts:
+                ex = pre + "mlp.experts."
+                ts.append(P[pre + "mlp.gate.weight"])
+                ts.append(torch.stack([
+                    torch.cat([P[f"{ex}{e}.gate_proj.weight"].chunk(tp, 0)[r],
+                               P[f"{ex}{e}.up_proj.weight"].chunk(tp, 0)[r]], 0)
+                    for e in range(shape.n_experts)]))
+                ts.append(torch.stack([P[f"{ex}{e}.down_proj.weight"].chunk(tp, 1)[r]
+                                       for e in range(shape.n_experts)]))
+            else:
+                m = pre + "mlp."
+                ts.append(torch.cat([P[m + "gate_proj.weight"].chunk(tp, 0)[r],
+                                     P[m + "up_proj.weight"].chunk(tp, 0)[r]], 0))
+                ts.append(P[m + "down_proj.weight"].chunk(tp, 1)[r])
+        ts.append(P["model.norm.weight"])
+        if not shape.tied:
+            ts.append(P["lm_head.weight"].chunk(tp, 0)[r])
+        assert all(t.shape[-1] in (H, t.shape[-1]) for t in ts)
+        ranks.append([_to_bf16_bits(t.contiguous()) for t in ts])
+    return ranks
+
+
+def restate_buckets(ranks, bucket_bytes, tensor_align=256):
+    out = []
+    for tensors in ranks:
+        stream = bytearray()
+        for t in tensors:
+            stream += bytes((-len(stream)) % tensor_align)
+            stream += t.numpy().tobytes()
+        stream += bytes((-len(stream)) % bucket_bytes)
+        out += [bytes(stream[i:i + bucket_bytes]) for i in range(0, len(stream), bucket_bytes)]
+    return out
+
+
+RESTATE = ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2", "tiny-moe-f32"]
+
+
+def _workload(name):
+    return synth.WORKLOADS.get(name) or synth.TEST_WORKLOADS[name]
+
+
+@pytest.mark.parametrize("name", RESTATE)
+def test_oracle_matches_restatement(name):
+    w = _workload(name)
+    L = oracle.workload_layout(w)
+    P = _param_tensors(L.params, _flat_offsets(L.params), w.seed, w.specials)
+    ranks = restate_rollout(w.shape, P, w.tp)
+    # Per-tensor reshard, straight from the materialised shards.
+    src = oracle.Source(shards=L.host_shards(w.seed, w.specials))
+    flat_t = [t for rank in ranks for t in rank]
+    order = [i for r in range(w.tp) for i, (_, rk, _) in enumerate(L.tensors) if rk == r]
+    assert len(order) == len(flat_t)
+    for t_idx, want in zip(order, flat_t):
+        got = L.reshard_tensor(src, t_idx)
+        np.testing.assert_array_equal(got, want.reshape(-1).numpy().view(np.uint16),
+                                      err_msg=L.tensors[t_idx][0])
+    # Buckets and checksums.
+    want_b = restate_buckets(ranks, w.bucket_bytes)
+    buckets, cs = L.pack(src)
+    assert buckets.shape[0] == len(want_b)
+    for b, wb in enumerate(want_b):
+        assert buckets[b].tobytes() == wb, f"bucket {b}"
+        assert int(cs[b]) == int(np.frombuffer(wb, "<u8").sum(dtype=np.uint64))
+
+
+# ---------------------------------------------------------------------------
+# Invariants
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n_shards", [1, 2, 3, 7, 8, 13])
+def test_shard_count_invariance(n_shards):
+    w = synth.TEST_WORKLOADS["tiny-tp4"]
+    ref_L = oracle.workload_layout(w.with_(n_shards=1))
+    ref, ref_cs = ref_L.pack(oracle.Source(shards=ref_L.host_shards(w.seed, w.specials)))
+    L = oracle.workload_layout(w.with_(n_shards=n_shards))
+    got, cs = L.pack(oracle.Source(shards=L.host_shards(w.seed, w.specials)))
+    np.testing.assert_array_equal(got, ref)
+    np.testing.assert_array_equal(cs, ref_cs)
+
+
+def test_generator_mode_matches_buffer_mode():
+    w = synth.TEST_WORKLOADS["tiny-moe-f32"]
+    L = oracle.workload_layout(w)
+    a, ca = L.pack(oracle.Source(shards=L.host_shards(w.seed, w.specials)))
+    b, cb = L.pack(oracle.Source(seed=w.seed, specials=w.specials))
+    np.testing.assert_array_equal(a, b)
+    np.testing.assert_array_equal(ca, cb)
+
+
+@pytest.mark.parametrize("name", ["qwen3-0.6b", "qwen3-8b", "qwen3-8b-tp4", "qwen3-30b-a3b",
+                                  "tiny-moe-tp2"])
+def test_coverage_counts(name):
+    """Every parameter element is read tp times if replicated, once otherwise, and
+    within one rank no parameter element is read twice (metadata only: full sizes)."""
+    w = _workload(name)
+    params = qwen3.manifest(w.shape, w.src_elem_bytes)
+    tensors = qwen3.rollout_tensors(w.shape, params, w.tp)
+    area = np.zeros(len(params), np.int64)
+    per_rank = {}
+    for _, r, blocks in tensors:
+        for (p, r0, nr, c0, nc) in blocks:
+            area[p] += nr * nc
+            per_rank.setdefault((r, p), []).append((r0, nr, c0, nc))
+    for p, (pname, dims, _) in enumerate(params):
+        numel = int(np.prod(dims))
+        replicated = len(dims) == 1 or pname.endswith("mlp.gate.weight")
+        assert area[p] == numel * (w.tp if replicated else 1), pname
+    for (r, p), rects in per_rank.items():
+        # Rectangles of one rank on one parameter must not overlap.
+        for i in range(len(rects)):
+            for j in range(i + 1, len(rects)):
+                a, b = rects[i], rects[j]
+                rows = a[0] < b[0] + b[1] and b[0] < a[0] + a[1]
+                cols = a[2] < b[2] + b[3] and b[2] < a[2] + a[3]
+                assert not (rows and cols), (r, params[p][0])
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-moe-tp2"])
+def test_unpack_of_pack_is_reshard(name):
+    w = _workload(name)
+    L = oracle.workload_layout(w)
+    src = oracle.Source(shards=L.host_shards(w.seed, w.specials))
+    buckets, _ = L.pack(src)
+    for t in range(len(L.tensors)):
+        np.testing.assert_array_equal(L.unpack_tensor(buckets, t), L.reshard_tensor(src, t))
+
+
+def test_checksum_against_numpy_and_linearity():
+    rng = np.random.default_rng(5)
+    for n in (8, 64, 4096, 1 << 20):
+        buf = rng.integers(0, 256, size=n, dtype=np.uint8)
+        assert oracle.checksum(buf) == int(buf.view("<u8").sum(dtype=np.uint64))
+    allff = np.full(1 << 12, 0xFF, np.uint8)
+    assert oracle.checksum(allff) == ((1 << 64) - 1) * (len(allff) // 8) % (1 << 64)
+    for off in range(0, 64, 2):
+        buf = np.zeros(64, np.uint8)
+        buf[off:off + 2] = [0x34, 0x12]
+        assert oracle.checksum(buf) == 0x1234 << (8 * (off % 8))
+
+
+def test_verify_flags_damage():
+    w = synth.WORKLOADS["tiny"]
+    L = oracle.workload_layout(w)
+    buckets, cs = L.pack(oracle.Source(seed=w.seed, specials=w.specials))
+    assert L.verify(buckets, cs) == (0, -1)
+    bad = buckets.copy()
+    bad[5, 1234] ^= 0x10
+    assert L.verify(bad, cs) == (1, 5)
+    bad[11] = 0
+    assert L.verify(bad, cs) == (2, 5)
+    swapped = buckets.copy()
+    swapped[[2, 3]] = swapped[[3, 2]]
+    assert L.verify(swapped, cs) == (2, 2)
+
+
+def test_layout_rejects_bad_input():
+    params = [("a", (4, 4), 4)]
+    with pytest.raises(RuntimeError):
+        oracle.Layout(params, [("t", 0, [(0, 2, 3, 0, 4)])], 1, 1, 64)   # rows out of range
+    with pytest.raises(RuntimeError):
+        oracle.Layout(params, [("t", 1, [(0, 0, 1, 0, 4)])], 1, 1, 64)   # rank out of range
+    with pytest.raises(RuntimeError):
+        oracle.Layout(params, [("t", 0, [(0, 0, 1, 0, 4)])], 1, 1, 12)   # bucket % 8 != 0
