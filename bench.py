@@ -1,0 +1,406 @@
+"""Benchmark: one full trainer -> rollout weight sync per step on GB300.
+
+A step is the whole hot path once (RobustRL Section 5.2.1 steps 1-2 and the
+Section 5.2.2 check): rr_pack (reshard + bf16 cast + bucket pack + checksum),
+rr_unpack (buckets -> rollout tensors) and rr_verify (recompute and compare
+every checksum).  Default workload: Qwen3-8B-shaped fp32 weights in 8 flat
+FSDP-style shards -> TP=1 bf16 rollout layout with fused QKV / gate_up,
+128 MiB buckets, seeded synthetic values ~N(0, 0.02).
+
+Metric: GB/s of algorithmic bytes (every byte read once, every byte written
+once: pack = source bytes + bucket bytes, unpack = 2 x tensor bytes, verify =
+bucket bytes), plus ms per full model sync (pack + unpack).  Inputs (33 GB of
+source) are far larger than L2, so no flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
+
+Under torchrun each rank runs an independent replica on its own GPU (the
+path does not shard: replicas only); the value is the bytes of all replicas
+over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "weight-sync reshard+pack GB/s and ms per full model sync; % of HBM roofline"
+UNIT = "GB/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--workload", default="qwen3-8b")
+    ap.add_argument("--bucket-mib", type=int, default=0, help="override the bucket size")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-buckets", type=int, default=2,
+                    help="buckets in the oracle's CPU sample")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# Distributed plumbing (replicas only)
+# ---------------------------------------------------------------------------
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# Clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.rows = []
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.gpu)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                self.rows.append(parts)
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=2)
+
+    def summary(self):
+        if not self.rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in self.rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in self.rows for n, v in zip(names, r[5:9])
+                          if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.rows)}
+
+
+def visible_gpu_index(local_rank: int) -> int:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [v for v in vis.split(",") if v.strip()]
+        if local_rank < len(ids) and ids[local_rank].strip().isdigit():
+            return int(ids[local_rank])
+    return local_rank
+
+
+# ---------------------------------------------------------------------------
+# Peaks and profile summaries
+# ---------------------------------------------------------------------------
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    path = os.path.join(ROOT, "paper_2512_22492_gb300", "csrc", "rr_device.cu")
+    return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per pack launch from the committed ncu summary, if it was taken
+    on the current kernel source; else None."""
+    path = os.path.join(ROOT, "profiles", f"rr_pack_{workload}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
+    m_bytes = re.search(r"dram_bytes_per_launch_full:\s*([0-9]+)", text)
+    if not (m_hash and m_bytes) or m_hash.group(1) != kernel_source_hash():
+        return None
+    return int(m_bytes.group(1))
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (baseline leg and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_sample_setup(w, bucket_bytes):
+    """Oracle layout and host shards whose leading bytes (enough for the first
+    buckets' sources) hold the seeded values; the rest are lazily zeroed."""
+    import numpy as np
+    import oracle
+    import synth
+    L = oracle.workload_layout(w, bucket_bytes=bucket_bytes)
+    need = 8 * bucket_bytes          # covers a few buckets' fp32 sources
+    flat = np.zeros(L.shard_bytes * L.n_shards, np.uint8)
+    for p, (_, _, es) in enumerate(L.params):
+        off = int(L.param_offset[p])
+        if off >= need:
+            break
+        n = min(L.param_numel(p), (need - off) // es)
+        flat[off:off + n * es] = synth.values_host(n, es, w.seed, off // es, w.specials).view(
+            np.uint8)
+    shards = [flat[s * L.shard_bytes:(s + 1) * L.shard_bytes] for s in range(L.n_shards)]
+    return L, oracle.Source(shards=shards), shards
+
+
+def oracle_time(L, src, first, count):
+    t0 = time.perf_counter()
+    moved = L.sync_sample(src, first, count)
+    return moved, time.perf_counter() - t0
+
+
+def cpu_baseline(w, bucket_bytes, n_buckets_sample):
+    L, src, _keep = oracle_sample_setup(w, bucket_bytes)
+    moved, dt = oracle_time(L, src, 0, n_buckets_sample)
+    return {"value": round(moved / dt / 1e9, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"buckets 0..{n_buckets_sample - 1} of {L.n_buckets} "
+                      f"({n_buckets_sample} x {bucket_bytes >> 20} MiB): pack, unpack of their "
+                      f"elements, verify; single-threaded C oracle; {moved / 1e9:.3f} GB in "
+                      f"{dt:.2f} s; host cores available {os.cpu_count()}"}
+
+
+def run_reference(args, w, bucket_bytes, world, rank):
+    if rank != 0:
+        return
+    L, src, _keep = oracle_sample_setup(w, bucket_bytes)
+    count = 1
+    for _ in range(args.warmup):
+        oracle_time(L, src, 0, count)
+    moved_total, t_total = 0, 0.0
+    for _ in range(args.steps):
+        moved, dt = oracle_time(L, src, 0, count)
+        moved_total += moved
+        t_total += dt
+    value = moved_total / t_total / 1e9
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(t_total / args.steps * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u16", "data": "synthetic",
+        "config": {"workload": w.name, "bucket_bytes": bucket_bytes,
+                   "step": f"oracle sync of bucket 0 of {L.n_buckets} (bounded sample)"},
+        "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"bucket 0 of {L.n_buckets} ({bucket_bytes >> 20} MiB): "
+                                   "pack, unpack of its elements, verify per step"},
+        "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def run_native(args, w, bucket_bytes, world, rank, local):
+    import torch
+    import paper_2512_22492_gb300 as rr
+    from tests import gpu_harness as H
+
+    torch.cuda.set_device(local)
+    stream = torch.cuda.current_stream()
+    m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp)
+    plan = rr.rr_plan_create(m, s, d, bucket_bytes)
+    st = plan.stats()
+    buf = H.alloc(plan, poison=None)
+    H.fill_with_generator(buf, m, w.seed, w.specials)
+    torch.cuda.synchronize()
+
+    pack_bytes = st["pack_bytes_read"] + st["pack_bytes_written"]
+    unpack_bytes = st["unpack_bytes_read"] + st["unpack_bytes_written"]
+    verify_bytes = st["verify_bytes_read"]
+    step_bytes = pack_bytes + unpack_bytes + verify_bytes
+
+    def step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        H.pack(buf, stream)
+        if ev:
+            ev[1].record(stream)
+        H.unpack(buf, stream)
+        if ev:
+            ev[2].record(stream)
+        n_bad, _ = H.verify(buf, stream)
+        if ev:
+            ev[3].record(stream)
+        if n_bad:
+            raise RuntimeError(f"verify found {n_bad} bad buckets")
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(visible_gpu_index(local)) as clk:
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for k in range(args.steps):
+            step(evs[k])
+        t1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    total_ms = max_over_ranks(t0.elapsed_time(t1), world)
+    pack_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    unpack_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    verify_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
+    ms_per_step = total_ms / args.steps
+    value = world * step_bytes / (ms_per_step * 1e-3) / 1e9
+
+    # End to end through the public API with host buffers: every step copies the
+    # trainer's shards from pinned host memory, syncs, and reads back the checksums.
+    e2e = None
+    if not args.no_e2e:
+        host_src = torch.empty(buf.flat.numel(), dtype=torch.uint8, pin_memory=True)
+        host_src.copy_(buf.flat)
+        host_cs = torch.empty(buf.checksums.numel(), dtype=torch.int64, pin_memory=True)
+        h2d, d2h = host_src.numel(), host_cs.numel() * 8 + 32
+
+        def e2e_step():
+            buf.flat.copy_(host_src, non_blocking=True)
+            step()
+            host_cs.copy_(buf.checksums, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(a.elapsed_time(b), world) / args.steps
+        e2e = {"value": round(world * step_bytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": round(e2e_ms, 3)}
+        del host_src
+
+    peak, peak_kind = hbm_peak()
+    pack_gbs = pack_bytes / (pack_ms * 1e-3) / 1e9
+    traffic = profiled_traffic(w.name) if bucket_bytes == w.bucket_bytes else None
+    clocks = clk.summary()
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u16",
+        "data": "synthetic",
+        "config": {"workload": w.name, "src_dtype": w.src_dtype, "n_shards": w.n_shards,
+                   "tp": w.tp, "bucket_bytes": bucket_bytes, "n_buckets": plan.n_buckets,
+                   "step": "rr_pack + rr_unpack + rr_verify",
+                   "step_bytes": step_bytes, "l2": "inputs > L2 (no flush needed)",
+                   "parallelism": f"replicas{world}"},
+        "ms_per_full_model_sync": round(pack_ms + unpack_ms, 3),
+        "ops": {
+            "pack": {"ms": round(pack_ms, 3), "bytes": pack_bytes,
+                     "GB/s": round(pack_gbs, 1), "frac_of_peak": round(pack_gbs / peak, 4)},
+            "unpack": {"ms": round(unpack_ms, 3), "bytes": unpack_bytes,
+                       "GB/s": round(unpack_bytes / (unpack_ms * 1e-3) / 1e9, 1),
+                       "frac_of_peak": round(unpack_bytes / (unpack_ms * 1e-3) / 1e9 / peak, 4)},
+            "verify": {"ms": round(verify_ms, 3), "bytes": verify_bytes,
+                       "GB/s": round(verify_bytes / (verify_ms * 1e-3) / 1e9, 1),
+                       "frac_of_peak": round(verify_bytes / (verify_ms * 1e-3) / 1e9 / peak, 4)},
+        },
+        "roofline": {"bound": "hbm", "kernel": "rr_pack_kernel", "achieved": round(pack_gbs, 1),
+                     "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
+                     "frac": round(pack_gbs / peak, 4), "traffic": traffic,
+                     "algorithmic_bytes": pack_bytes},
+        "clocks": clocks,
+        "gpu_launches": 3 * args.steps,
+        "e2e": e2e,
+    }
+    del buf
+    torch.cuda.empty_cache()
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, bucket_bytes, args.cpu_buckets)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    import synth
+    w = synth.WORKLOADS.get(args.workload) or synth.TEST_WORKLOADS[args.workload]
+    bucket_bytes = args.bucket_mib * (1 << 20) if args.bucket_mib else w.bucket_bytes
+    world, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, w, bucket_bytes, world, rank)
+    else:
+        run_native(args, w, bucket_bytes, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,260 @@
+/*
+ * rr.h - C ABI of the trainer -> rollout weight-synchronisation hot path.
+ *
+ * RobustRL (arXiv 2512.22492), Section 5.2.1 "UCX-based Weight Update":
+ * after a training step the trainer's weights are (1) resharded to the
+ * rollout's sharding and (2) placed layer by layer into a transfer buffer
+ * that the transport moves to the rollout; Section 5.2.2 has a recovered or
+ * resumed rollout pull (part of) that buffer again.  This library is the
+ * on-GPU part of that route, for one GPU: gather from flat FSDP-style shards,
+ * cast to bfloat16, pack into fixed-size buckets with a 64-bit checksum each,
+ * and unpack buckets into the rollout's tensors.  The transport is not here.
+ *
+ * Definitions (the paper fixes none of these; they are this library's):
+ *
+ *  Source layout.  Parameters are concatenated in manifest order into one
+ *  flat byte buffer, each starting at a multiple of max(align_bytes, element
+ *  size) (or at the caller's explicit offsets); the total is padded to a
+ *  multiple of 16 * n_shards and cut into n_shards shards of equal size S.
+ *  Flat byte f is byte f % S of shard f / S.  A parameter of shape
+ *  [d0, d1, ...] is viewed as a matrix [d0, d1 * d2 * ...]; a vector [d0] is
+ *  [d0, 1].
+ *
+ *  Destination.  A destination tensor is a list of blocks; its elements are
+ *  the blocks' elements, block after block, each block row-major.  Block
+ *  (param, row0, nrows, col0, ncols) covers rows [row0, row0 + nrows) and
+ *  columns [col0, col0 + ncols) of the parameter's matrix view.  Fused QKV,
+ *  fused gate_up, stacked experts and tensor-parallel slices are all block
+ *  lists; the library knows nothing about any model.
+ *
+ *  Cast.  float32 -> bfloat16 rounds to nearest, ties to even, in integer
+ *  arithmetic: +-0, subnormals and +-inf are kept, overflow goes to +-inf,
+ *  and a NaN keeps its sign and upper payload with the quiet bit set
+ *  ((bits >> 16) | 0x0040).  A bfloat16 source is copied bit for bit.
+ *
+ *  Stream and buckets.  Each destination rank r has a byte stream holding
+ *  its tensors in the order given, each starting at the next multiple of
+ *  tensor_align_bytes, elements little-endian.  The stream is cut into
+ *  buckets of exactly bucket_bytes; alignment gaps and the last bucket's
+ *  tail are zero.  Buckets are numbered rank-major: rank 0's first.
+ *
+ *  Checksum.  checksums[b] = sum of the little-endian 64-bit words of
+ *  bucket b, modulo 2^64.  The sum is order-independent, so the GPU may
+ *  accumulate in any grouping and still match exactly.
+ *
+ * Memory.  Every pointer argument named "device" is CUDA device memory of
+ * the device the plan was created on, owned by the caller; every device
+ * pointer must be 16-byte aligned.  The plan owns its device segment tables
+ * and a small verify scratch area; rr_pack and rr_unpack allocate nothing.
+ *
+ * Errors.  Every call returns rr_status.  Argument and layout errors are
+ * reported synchronously and leave outputs untouched; RR_ECUDA means a CUDA
+ * call failed (rr_last_error() has the CUDA message).  rr_last_error()
+ * returns a per-thread description of the most recent failure.
+ *
+ * Threads and streams.  A plan is immutable after creation; rr_pack and
+ * rr_unpack may run on it concurrently on different streams as long as
+ * their outputs are distinct.  rr_verify serialises on the plan.
+ */
+#ifndef RR_H
+#define RR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    RR_OK = 0,
+    RR_EINVAL = 1,    /* bad argument: null pointer, bad size, misaligned pointer        */
+    RR_ENOMEM = 2,    /* host or device allocation failed (plan creation only)           */
+    RR_ECUDA = 3,     /* a CUDA call failed                                              */
+    RR_ELAYOUT = 4,   /* the layout description is inconsistent or out of range          */
+    RR_EMISMATCH = 5  /* rr_verify: at least one bucket's checksum differs               */
+} rr_status;
+
+typedef enum { RR_F32 = 0, RR_BF16 = 1 } rr_dtype;
+
+/* One trainer parameter (manifest entry). */
+typedef struct {
+    const char* name;   /* informational, may be NULL                              */
+    int32_t ndim;       /* 0..4                                                    */
+    int64_t shape[4];   /* sizes of the first ndim dimensions                      */
+    rr_dtype dtype;     /* dtype of the trainer's copy: RR_F32 or RR_BF16          */
+} rr_param;
+
+/* Trainer side: flat FSDP-style shards. */
+typedef struct {
+    int32_t n_shards;                 /* 1..65535                                      */
+    int64_t align_bytes;              /* parameter start alignment, >= 1 (16 typical)  */
+    const int64_t* param_flat_offset; /* optional [n_params] explicit flat byte
+                                         offsets (each a multiple of the element size,
+                                         non-overlapping); NULL = computed as above    */
+} rr_src_layout;
+
+/* A 2-D block of a parameter's matrix view. */
+typedef struct {
+    int32_t param;
+    int64_t row0, nrows, col0, ncols;
+} rr_block;
+
+/* One rollout tensor. */
+typedef struct {
+    const char* name;        /* informational, may be NULL                          */
+    int32_t rank;            /* destination rank, 0 .. tp-1                         */
+    int64_t numel;           /* must equal the sum of the blocks' nrows * ncols     */
+    int32_t n_blocks;
+    const rr_block* blocks;
+} rr_dst_tensor;
+
+/* Rollout side. */
+typedef struct {
+    int32_t tp;                   /* number of destination ranks (tensor parallel)     */
+    int32_t n_tensors;
+    const rr_dst_tensor* tensors; /* order within a rank = order in its stream         */
+    int64_t tensor_align_bytes;   /* power of two >= 2; 256 typical                    */
+} rr_dst_layout;
+
+typedef struct rr_plan rr_plan;
+
+/* Tuning / inspection options for rr_plan_create_ex.  Zero means default. */
+typedef struct {
+    int32_t host_only;   /* 1: build the tables on the host only and touch no GPU; such
+                            a plan can be queried and exported but not executed       */
+    int32_t grid_blocks; /* persistent grid size; default: SMs x resident blocks      */
+    int64_t chunk_bytes; /* largest destination bytes per work item; default 32 KiB   */
+} rr_plan_options;
+
+/* Compiles manifest + source layout + destination layout + bucket size into
+ * device-resident segment tables (Section 5.2.1 step 1: "reshard ... to align
+ * with the sharding of the rollout").  bucket_bytes: a multiple of 8, at most
+ * 2^32 - 16.  Uses the current CUDA device.  *out is valid only on RR_OK. */
+rr_status rr_plan_create(const rr_param* manifest, int32_t n_params, const rr_src_layout* src,
+                         const rr_dst_layout* dst, size_t bucket_bytes, rr_plan** out);
+rr_status rr_plan_create_ex(const rr_param* manifest, int32_t n_params,
+                            const rr_src_layout* src, const rr_dst_layout* dst,
+                            size_t bucket_bytes, const rr_plan_options* opts, rr_plan** out);
+void rr_plan_destroy(rr_plan* plan);
+
+/* Bucket geometry.  Any output pointer may be NULL.  stream_bytes_per_rank has
+ * tp entries; first_bucket_of_rank has tp + 1 (the last is n_buckets). */
+rr_status rr_plan_query(const rr_plan* plan, int32_t* n_buckets, int64_t* stream_bytes_per_rank,
+                        int32_t* first_bucket_of_rank);
+
+/* Source geometry: shard size S, end of the last parameter, per-parameter flat
+ * offsets ([n_params]).  Any output pointer may be NULL. */
+rr_status rr_plan_source(const rr_plan* plan, int64_t* shard_bytes, int64_t* flat_bytes,
+                         int64_t* param_flat_offset);
+
+/* Destination geometry: per tensor numel and byte offset within its rank's
+ * stream ([n_tensors] each).  Any output pointer may be NULL. */
+rr_status rr_plan_tensors(const rr_plan* plan, int64_t* tensor_numel,
+                          int64_t* tensor_stream_offset);
+
+typedef struct {
+    int64_t n_pack_items;
+    int64_t n_unpack_items;
+    int32_t grid_blocks;         /* pack kernel grid (blocks)                          */
+    int32_t unpack_grid_blocks;
+    int32_t verify_grid_blocks;
+    int32_t n_buckets;
+    int32_t n_shards;
+    int32_t n_tensors;
+    int64_t bucket_bytes;
+    int64_t pack_bytes_read;     /* source bytes read by one rr_pack                    */
+    int64_t pack_bytes_written;  /* bucket bytes written by one rr_pack (all buckets)   */
+    int64_t unpack_bytes_read;   /* bucket bytes read by one rr_unpack                  */
+    int64_t unpack_bytes_written;/* destination bytes written by one rr_unpack          */
+    int64_t verify_bytes_read;   /* bucket bytes read by one rr_verify                  */
+} rr_plan_stats;
+
+rr_status rr_plan_get_stats(const rr_plan* plan, rr_plan_stats* stats);
+
+/* Work items of the segment tables, as the kernels read them (exported for
+ * inspection and host-side tests). */
+enum {
+    RR_ITEM_F32_VEC = 0,    /* fp32 -> bf16, 8 elements per 16-byte store            */
+    RR_ITEM_F32_SCALAR = 1, /* fp32 -> bf16, one element at a time (ragged/misaligned)*/
+    RR_ITEM_BF16_VEC = 2,   /* bf16 -> bf16                                          */
+    RR_ITEM_BF16_SCALAR = 3,
+    RR_ITEM_ZERO_VEC = 4,   /* zero fill of alignment gaps / bucket tails            */
+    RR_ITEM_ZERO_SCALAR = 5,
+    RR_ITEM_COPY_VEC = 6,   /* unpack: 16-byte copies                                */
+    RR_ITEM_COPY_SCALAR = 7 /* unpack: 2-byte copies                                 */
+};
+
+/* Pack work item: n_rows rows of row_len elements; row i starts at source
+ * element offset i * src_stride from the first; the destination is the
+ * contiguous range [dst_off, dst_off + 2 * n_rows * row_len) of one bucket. */
+typedef struct {
+    uint64_t src;        /* bits 0..47: byte offset in the shard; bits 48..63: shard   */
+    uint32_t dst_off;    /* byte offset in the bucket                                   */
+    uint32_t bucket;     /* global bucket index                                         */
+    uint32_t row_len;    /* elements per row                                            */
+    uint32_t n_rows;
+    uint32_t src_stride; /* elements between consecutive row starts                     */
+    uint16_t kind;       /* RR_ITEM_F32_* / BF16_* / ZERO_*                            */
+    uint16_t reserved;
+} rr_pack_item;
+
+/* Unpack work item: copy nbytes from bucket `bucket` at src_off to tensor
+ * `tensor` at dst_off. */
+typedef struct {
+    uint64_t dst_off;
+    uint32_t src_off;
+    uint32_t bucket;
+    uint32_t tensor;
+    uint32_t nbytes;
+    uint32_t kind;       /* RR_ITEM_COPY_*                                             */
+    uint32_t reserved;
+} rr_unpack_item;
+
+/* Copies up to cap items (and, if block_first is not NULL, the per-block item
+ * ranges: grid_blocks + 1 entries for pack, unpack_grid_blocks + 1 for
+ * unpack) into caller memory. */
+rr_status rr_plan_export_pack(const rr_plan* plan, rr_pack_item* items, int64_t cap,
+                              uint32_t* block_first);
+rr_status rr_plan_export_unpack(const rr_plan* plan, rr_unpack_item* items, int64_t cap,
+                                uint32_t* block_first);
+
+/* Reshard + cast + pack + checksum, fused in one persistent kernel launch
+ * (Section 5.2.1 steps 1-2: the model is placed "layer by layer into a
+ * buffer for transmission"; the checksums serve Section 5.2.2's reconnect).
+ *   src_shards: host array of n_shards device pointers, S bytes each.
+ *   buckets:    host array of n_buckets device pointers, bucket_bytes each;
+ *               equally spaced pointers (one allocation cut into buckets)
+ *               lift the limit on how many buckets a launch can address.
+ *   checksums:  device array of n_buckets uint64, overwritten.
+ * Stream-ordered and asynchronous: returns after enqueueing a memset of the
+ * checksums and one kernel on `stream`. */
+rr_status rr_pack(const rr_plan* plan, const void* const* src_shards, void* const* buckets,
+                  uint64_t* checksums, cudaStream_t stream);
+
+/* Buckets -> rollout tensors (Section 5.2.1: the receiving rollout
+ * "finishes the weight update").
+ *   buckets: host array of n_buckets device pointers;
+ *   dst:     host array of n_tensors device pointers, numel * 2 bytes each.
+ * Stream-ordered and asynchronous (one kernel launch). */
+rr_status rr_unpack(const rr_plan* plan, const void* const* buckets, void* const* dst,
+                    cudaStream_t stream);
+
+/* Recomputes every bucket's checksum on the GPU and compares it with
+ * checksums (device, n_buckets).  Blocks the calling thread until `stream`
+ * has finished the check.  *n_bad = number of mismatching buckets, *first_bad
+ * = lowest such index or -1 (either pointer may be NULL).  Returns
+ * RR_EMISMATCH when n_bad > 0. */
+rr_status rr_verify(const rr_plan* plan, const void* const* buckets, const uint64_t* checksums,
+                    int64_t* n_bad, int64_t* first_bad, cudaStream_t stream);
+
+const char* rr_status_str(rr_status status);
+const char* rr_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RR_H */

@@ -102,6 +102,9 @@ def lib() -> ctypes.CDLL:
         L.orc_checksum.restype = ctypes.c_uint64
         L.orc_unpack_tensor.argtypes = [LP, ctypes.POINTER(vp), ctypes.c_int32, vp]
         L.orc_unpack_tensor.restype = ctypes.c_int
+        L.orc_unpack_elements.argtypes = [LP, ctypes.POINTER(vp), ctypes.c_int32, ctypes.c_int64,
+                                          ctypes.c_int64, vp]
+        L.orc_unpack_elements.restype = ctypes.c_int
         L.orc_verify.argtypes = [LP, ctypes.POINTER(vp), vp, ctypes.c_int64, ctypes.c_int64,
                                  _P64]
         L.orc_verify.restype = ctypes.c_int64
@@ -283,6 +286,45 @@ class Layout:
                "unpack_tensor")
         del keep
         return out
+
+    def unpack_elements(self, buckets, t: int, j0: int, j1: int) -> np.ndarray:
+        ptrs, keep = self._bucket_ptrs(buckets)
+        out = np.empty(j1 - j0, np.uint16)
+        _check(lib().orc_unpack_elements(ctypes.byref(self.c), ptrs, t, j0, j1, out.ctypes.data),
+               "unpack_elements")
+        del keep
+        return out
+
+    def sync_sample(self, src: "Source", first: int, count: int) -> int:
+        """One CPU weight sync restricted to buckets [first, first+count): pack
+        them, unpack every tensor element that lies in them, verify them.
+        Returns the algorithmic bytes moved: pack reads the source elements and
+        writes the buckets, unpack reads and writes each element's two bytes,
+        verify reads the buckets."""
+        packed, cs = self.pack(src, first, count)
+        buckets = [None] * self.n_buckets
+        for i in range(count):
+            buckets[first + i] = packed[i]
+        moved = 0
+        for t, (_, rank, blocks) in enumerate(self.tensors):
+            fb = int(self.rank_first_bucket[rank])
+            lo = (first - fb) * self.bucket_bytes
+            hi = (first + count - fb) * self.bucket_bytes
+            t_lo = int(self.tensor_offset[t])
+            t_hi = t_lo + 2 * int(self.tensor_numel[t])
+            a, z = max(lo, t_lo), min(hi, t_hi)
+            if a < z:
+                self.unpack_elements(buckets, t, (a - t_lo) // 2, (z - t_lo) // 2)
+                es = self.params[blocks[0][0]][2]
+                moved += (z - a) // 2 * es      # pack: source bytes read
+                moved += 2 * (z - a)             # unpack: read + write
+        full_cs = np.zeros(self.n_buckets, np.uint64)
+        full_cs[first:first + count] = cs
+        n_bad, _ = self.verify(buckets, full_cs, first, count)
+        if n_bad:
+            raise RuntimeError("oracle verify failed on its own buckets")
+        moved += 2 * count * self.bucket_bytes   # pack writes + verify reads
+        return moved
 
     def verify(self, buckets, checksums, first: int = 0, count: Optional[int] = None):
         """(number of bad buckets, first bad index or -1)."""

@@ -298,19 +298,26 @@ int orc_pack_range(const orc_layout* L, const orc_source* S, int64_t first, int6
 
 /* --------------------------------------------------------------- unpack */
 
-/* Destination tensor t read back out of the buckets (buckets[b] = bucket b's bytes). */
-int orc_unpack_tensor(const orc_layout* L, const uint8_t* const* buckets, int32_t t,
-                      uint16_t* out) {
+/* Elements j0 .. j1-1 of destination tensor t read back out of the buckets
+ * (buckets[b] = bucket b's bytes; buckets not needed may be NULL). */
+int orc_unpack_elements(const orc_layout* L, const uint8_t* const* buckets, int32_t t,
+                        int64_t j0, int64_t j1, uint16_t* out) {
     const orc_tensor* T = &L->tensors[t];
     int64_t first = L->rank_first_bucket[T->rank];
-    for (int64_t j = 0; j < L->tensor_numel[t]; ++j) {
+    for (int64_t j = j0; j < j1; ++j) {
         int64_t pos = L->tensor_offset[t] + 2 * j;
         const uint8_t* bucket = buckets[first + pos / L->bucket_bytes];
         if (bucket == NULL) return ORC_ESOURCE;
         int64_t o = pos % L->bucket_bytes;
-        out[j] = (uint16_t)(bucket[o] | (bucket[o + 1] << 8));
+        out[j - j0] = (uint16_t)(bucket[o] | (bucket[o + 1] << 8));
     }
     return ORC_OK;
+}
+
+/* The whole of destination tensor t read back out of the buckets. */
+int orc_unpack_tensor(const orc_layout* L, const uint8_t* const* buckets, int32_t t,
+                      uint16_t* out) {
+    return orc_unpack_elements(L, buckets, t, 0, L->tensor_numel[t], out);
 }
 
 /* --------------------------------------------------------------- verify */

@@ -1,0 +1,15 @@
+"""GB300-native trainer -> rollout weight synchronisation hot path.
+
+RobustRL (arXiv 2512.22492) Section 5.2.1: reshard the trainer's weights to
+the rollout's sharding and place them layer by layer into a transfer buffer;
+Section 5.2.2: a rollout that reconnects after a failure pulls (part of) that
+buffer again.  This package is the on-GPU part of that route for one GB300:
+a C-ABI CUDA library (``include/rr.h``, ``csrc/``) and its Python binding.
+"""
+from .rr import (Block, DstLayout, DstTensor, Param, Plan, PlanOptions, RRError, SrcLayout,
+                 rr_pack, rr_plan_create, rr_status_str, rr_unpack, rr_verify)
+from .layouts import qwen3_manifest, qwen3_rollout, qwen3_sync
+
+__all__ = ["Block", "DstLayout", "DstTensor", "Param", "Plan", "PlanOptions", "RRError",
+           "SrcLayout", "rr_pack", "rr_plan_create", "rr_status_str", "rr_unpack", "rr_verify",
+           "qwen3_manifest", "qwen3_rollout", "qwen3_sync"]

@@ -1,0 +1,594 @@
+// Device side of the weight-sync hot path for GB300 (sm_103a): the pack
+// (gather + bf16 cast + bucket write + checksum), unpack and verify kernels,
+// and the C-ABI entry points that launch them.
+//
+// RobustRL Section 5.2.1 (steps 1-2: reshard, then place the model layer by
+// layer into a transfer buffer) and Section 5.2.2 (a rollout that resumes or
+// restarts a pull must know which parts of the buffer it holds intact).
+//
+// All three kernels are persistent: one launch of `grid_blocks` blocks walks
+// the whole work table, each block a contiguous, weight-balanced range of it.
+// The work is pure data movement bound by HBM bandwidth: 16-byte coalesced
+// loads and stores, several vectors in flight per thread, the cast done in
+// integer arithmetic in registers, the checksum accumulated per warp in
+// registers and flushed with one 64-bit atomic per warp per bucket change.
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstring>
+
+#include "rr_internal.h"
+
+namespace {
+
+constexpr int kThreads = 256;       // threads per block, all three kernels
+constexpr int kUnroll = 4;          // 16-byte vectors in flight per thread
+constexpr int kSmallPtrs = 64;      // pointer-table sizes of the two launch shapes
+constexpr int kLargePtrs = 3968;    // keeps the kernel parameters under 32 KB
+constexpr int64_t kVerifyChunk = 64 * 1024;
+
+// ---------------------------------------------------------------------------
+// Launch arguments (passed by value in the kernel parameter space, so that a
+// plan can run concurrently on several streams with different buffers).
+// ---------------------------------------------------------------------------
+
+template <int NPTR>
+struct PackArgs {
+    const rr_pack_item* items;
+    const uint32_t* block_first;
+    unsigned long long* checksums;
+    char* bucket_base;        // equally spaced buckets: base + b * stride
+    uint64_t bucket_stride;   // 0: bucket b is ptr[n_shards + b]
+    int32_t n_shards;
+    int32_t pad;
+    const void* ptr[NPTR];    // shards, then (table mode) buckets
+};
+
+template <int NPTR>
+struct UnpackArgs {
+    const rr_unpack_item* items;
+    const uint32_t* block_first;
+    const char* bucket_base;
+    uint64_t bucket_stride;
+    int32_t dst_base;         // index in ptr[] of destination tensor 0
+    int32_t pad;
+    const void* ptr[NPTR];    // (table mode) buckets, then destination tensors
+};
+
+template <int NPTR>
+struct VerifyArgs {
+    unsigned long long* sums;       // [n_buckets], zeroed
+    unsigned long long* counters;   // [4]: blocks done, n_bad, max(ULLONG_MAX - bad index)
+    const unsigned long long* expected;
+    const char* bucket_base;
+    uint64_t bucket_stride;
+    uint64_t bucket_bytes;
+    uint64_t chunk_bytes;
+    uint64_t chunks_per_bucket;
+    uint64_t total_chunks;
+    int32_t n_buckets;
+    int32_t pad;
+    const void* ptr[NPTR];          // (table mode) buckets
+};
+
+// ---------------------------------------------------------------------------
+// Small device helpers
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+    uint4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
+    return r;
+}
+
+__device__ __forceinline__ void st_stream(void* p, uint4 v) {
+    asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+// float32 bits -> value whose upper half is the bfloat16 result: round to
+// nearest even by adding 0x7FFF plus the lowest kept bit; a NaN instead
+// keeps its upper half with the quiet bit set (no rounding, so it can never
+// carry into the exponent and become an infinity).
+__device__ __forceinline__ uint32_t round_hi(uint32_t x) {
+    const uint32_t r = x + 0x7FFFu + ((x >> 16) & 1u);
+    return (x & 0x7FFFFFFFu) > 0x7F800000u ? (x | 0x00400000u) : r;
+}
+
+// Two float32 -> two bfloat16 packed little-endian in one word.
+__device__ __forceinline__ uint32_t cast2(uint32_t a, uint32_t b) {
+    return __byte_perm(round_hi(a), round_hi(b), 0x7632);
+}
+
+__device__ __forceinline__ uint16_t cast1(uint32_t a) { return uint16_t(round_hi(a) >> 16); }
+
+__device__ __forceinline__ unsigned long long words(uint4 v) {
+    return ((unsigned long long)v.y << 32 | v.x) + ((unsigned long long)v.w << 32 | v.z);
+}
+
+__device__ __forceinline__ unsigned long long warp_sum(unsigned long long v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    return v;
+}
+
+__device__ __forceinline__ void flush(unsigned long long* dst, unsigned long long acc) {
+    acc = warp_sum(acc);
+    if ((threadIdx.x & 31) == 0 && acc != 0ull) atomicAdd(dst, acc);
+}
+
+template <int NPTR>
+__device__ __forceinline__ char* bucket_of(const PackArgs<NPTR>& a, uint32_t b) {
+    return a.bucket_stride ? a.bucket_base + (uint64_t)b * a.bucket_stride
+                           : (char*)a.ptr[a.n_shards + b];
+}
+
+// ---------------------------------------------------------------------------
+// Pack
+// ---------------------------------------------------------------------------
+
+// Vector item: n_rows rows of row_len (multiple of 8) elements, 16-byte
+// aligned source rows and destination.  One "vector" is 8 elements: 32 (fp32)
+// or 16 (bf16) source bytes, 16 destination bytes.  Thread t handles vectors
+// t, t + T, t + 2T, ...; (row, vector-in-row) is advanced incrementally.
+template <int ES>
+__device__ __forceinline__ unsigned long long pack_vec(const char* src, char* dst,
+                                                       const rr_pack_item& d) {
+    const uint32_t vpr = d.row_len >> 3;
+    const uint32_t nvec = vpr * d.n_rows;
+    const uint64_t stride = (uint64_t)d.src_stride * ES;
+    const uint32_t dq = kThreads / vpr, dr = kThreads - dq * vpr;
+    uint32_t v = threadIdx.x;
+    uint32_t r = v / vpr, c = v - r * vpr;
+    unsigned long long acc = 0;
+    while (v < nvec) {
+        uint4 x[kUnroll][ES / 2];
+        uint32_t vv[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            vv[u] = v;
+            if (v < nvec) {
+                const char* p = src + r * stride + (uint64_t)c * (8 * ES);
+                x[u][0] = ld_stream(p);
+                if (ES == 4) x[u][ES / 2 - 1] = ld_stream(p + 16);
+            }
+            v += kThreads;
+            c += dr;
+            r += dq;
+            if (c >= vpr) {
+                c -= vpr;
+                ++r;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            if (vv[u] < nvec) {
+                uint4 o;
+                if (ES == 4) {
+                    o.x = cast2(x[u][0].x, x[u][0].y);
+                    o.y = cast2(x[u][0].z, x[u][0].w);
+                    o.z = cast2(x[u][ES / 2 - 1].x, x[u][ES / 2 - 1].y);
+                    o.w = cast2(x[u][ES / 2 - 1].z, x[u][ES / 2 - 1].w);
+                } else {
+                    o = x[u][0];
+                }
+                st_stream(dst + (uint64_t)vv[u] * 16, o);
+                acc += words(o);
+            }
+        }
+    }
+    return acc;
+}
+
+// Scalar item: any alignment and row length; one element per thread-step.
+// Each element's checksum contribution is its bits shifted to its byte
+// position within the 64-bit word it lands in.
+template <int ES>
+__device__ __forceinline__ unsigned long long pack_scalar(const char* src, char* dst,
+                                                          const rr_pack_item& d) {
+    const uint32_t L = d.row_len;
+    const uint32_t n = L * d.n_rows;
+    const uint64_t stride = (uint64_t)d.src_stride * ES;
+    const uint32_t dq = kThreads / L, dr = kThreads - dq * L;
+    uint32_t e = threadIdx.x;
+    uint32_t r = e / L, c = e - r * L;
+    unsigned long long acc = 0;
+    for (; e < n; e += kThreads) {
+        const char* p = src + r * stride + (uint64_t)c * ES;
+        uint16_t h;
+        if (ES == 4)
+            h = cast1(*(const uint32_t*)p);
+        else
+            h = *(const uint16_t*)p;
+        *(uint16_t*)(dst + 2ull * e) = h;
+        acc += (unsigned long long)h << (8 * ((d.dst_off + 2 * e) & 7));
+        c += dr;
+        r += dq;
+        if (c >= L) {
+            c -= L;
+            ++r;
+        }
+    }
+    return acc;
+}
+
+template <int NPTR>
+__global__ void __launch_bounds__(kThreads, 2) rr_pack_kernel(const __grid_constant__ PackArgs<NPTR> a) {
+    const uint32_t i1 = a.block_first[blockIdx.x + 1];
+    unsigned long long acc = 0;
+    uint32_t cur = 0xFFFFFFFFu;
+    for (uint32_t it = a.block_first[blockIdx.x]; it < i1; ++it) {
+        const rr_pack_item d = a.items[it];
+        if (d.bucket != cur) {
+            if (cur != 0xFFFFFFFFu) flush(a.checksums + cur, acc);
+            cur = d.bucket;
+            acc = 0;
+        }
+        char* dst = bucket_of(a, d.bucket) + d.dst_off;
+        const char* src = (const char*)a.ptr[d.src >> 48] + (d.src & 0xFFFFFFFFFFFFull);
+        switch (d.kind) {
+            case RR_ITEM_F32_VEC: acc += pack_vec<4>(src, dst, d); break;
+            case RR_ITEM_BF16_VEC: acc += pack_vec<2>(src, dst, d); break;
+            case RR_ITEM_F32_SCALAR: acc += pack_scalar<4>(src, dst, d); break;
+            case RR_ITEM_BF16_SCALAR: acc += pack_scalar<2>(src, dst, d); break;
+            case RR_ITEM_ZERO_VEC:
+                for (uint32_t v = threadIdx.x; v < (d.row_len >> 3); v += kThreads)
+                    st_stream(dst + 16ull * v, make_uint4(0, 0, 0, 0));
+                break;
+            default:  // RR_ITEM_ZERO_SCALAR
+                for (uint32_t e = threadIdx.x; e < d.row_len; e += kThreads)
+                    *(uint16_t*)(dst + 2ull * e) = 0;
+                break;
+        }
+    }
+    if (cur != 0xFFFFFFFFu) flush(a.checksums + cur, acc);
+}
+
+// ---------------------------------------------------------------------------
+// Unpack
+// ---------------------------------------------------------------------------
+
+template <int NPTR>
+__global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
+    const uint32_t i1 = a.block_first[blockIdx.x + 1];
+    for (uint32_t it = a.block_first[blockIdx.x]; it < i1; ++it) {
+        const rr_unpack_item d = a.items[it];
+        const char* src = (a.bucket_stride ? a.bucket_base + (uint64_t)d.bucket * a.bucket_stride
+                                           : (const char*)a.ptr[d.bucket]) + d.src_off;
+        char* dst = (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off;
+        if (d.kind == RR_ITEM_COPY_VEC) {
+            const uint32_t nvec = d.nbytes >> 4;
+            for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * kUnroll) {
+                uint4 x[kUnroll];
+#pragma unroll
+                for (int u = 0; u < kUnroll; ++u)
+                    if (v + u * kThreads < nvec) x[u] = ld_stream(src + 16ull * (v + u * kThreads));
+#pragma unroll
+                for (int u = 0; u < kUnroll; ++u)
+                    if (v + u * kThreads < nvec) st_stream(dst + 16ull * (v + u * kThreads), x[u]);
+            }
+        } else {
+            for (uint32_t e = threadIdx.x; e < (d.nbytes >> 1); e += kThreads)
+                *(uint16_t*)(dst + 2ull * e) = *(const uint16_t*)(src + 2ull * e);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Verify
+// ---------------------------------------------------------------------------
+
+template <int NPTR>
+__global__ void __launch_bounds__(kThreads, 4) rr_verify_kernel(const __grid_constant__ VerifyArgs<NPTR> a) {
+    const uint64_t c0 = a.total_chunks * blockIdx.x / gridDim.x;
+    const uint64_t c1 = a.total_chunks * (blockIdx.x + 1) / gridDim.x;
+    unsigned long long acc = 0;
+    uint32_t cur = 0xFFFFFFFFu;
+    for (uint64_t ch = c0; ch < c1; ++ch) {
+        const uint32_t b = (uint32_t)(ch / a.chunks_per_bucket);
+        const uint64_t off = (ch - (uint64_t)b * a.chunks_per_bucket) * a.chunk_bytes;
+        const uint64_t len = min(a.chunk_bytes, a.bucket_bytes - off);
+        if (b != cur) {
+            if (cur != 0xFFFFFFFFu) flush(a.sums + cur, acc);
+            cur = b;
+            acc = 0;
+        }
+        const char* p = (a.bucket_stride ? a.bucket_base + (uint64_t)b * a.bucket_stride
+                                         : (const char*)a.ptr[b]) + off;
+        const uint32_t nvec = (uint32_t)(len >> 4);
+        for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * kUnroll) {
+            uint4 x[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u)
+                if (v + u * kThreads < nvec) x[u] = ld_stream(p + 16ull * (v + u * kThreads));
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u)
+                if (v + u * kThreads < nvec) acc += words(x[u]);
+        }
+        if ((len & 15) && threadIdx.x == 0)   // a trailing 8-byte word
+            acc += *(const unsigned long long*)(p + (len & ~15ull));
+    }
+    if (cur != 0xFFFFFFFFu) flush(a.sums + cur, acc);
+
+    // The last block to finish compares all sums (no block waits for another).
+    __shared__ bool last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        last = atomicAdd(&a.counters[0], 1ull) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    for (int32_t b = threadIdx.x; b < a.n_buckets; b += kThreads) {
+        if (__ldcg(a.sums + b) != a.expected[b]) {
+            atomicAdd(&a.counters[1], 1ull);
+            atomicMax(&a.counters[2], ULLONG_MAX - (unsigned long long)b);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Host helpers
+// ---------------------------------------------------------------------------
+
+rr_status cuda_fail(cudaError_t e, const char* what) {
+    return rr_fail(RR_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define RR_CUDA(call)                                   \
+    do {                                                \
+        cudaError_t e_ = (call);                        \
+        if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
+    } while (0)
+
+bool aligned16(const void* p) { return p && ((uintptr_t)p & 15u) == 0; }
+
+// Equally spaced bucket pointers (one allocation cut into buckets)?
+bool uniform(const void* const* ptrs, int32_t n, int64_t min_stride, uint64_t* stride) {
+    if (n <= 1) {
+        *stride = (uint64_t)min_stride;
+        return true;
+    }
+    const intptr_t s = (const char*)ptrs[1] - (const char*)ptrs[0];
+    if (s < min_stride) return false;
+    for (int32_t i = 2; i < n; ++i)
+        if ((const char*)ptrs[i] - (const char*)ptrs[i - 1] != s) return false;
+    *stride = (uint64_t)s;
+    return true;
+}
+
+rr_status check_plan(const rr_plan* P) {
+    if (!P) return rr_fail(RR_EINVAL, "plan is NULL");
+    if (P->host_only) return rr_fail(RR_EINVAL, "plan was created host-only");
+    int dev = -1;
+    RR_CUDA(cudaGetDevice(&dev));
+    if (dev != P->device)
+        return rr_fail(RR_EINVAL, "plan belongs to device %d, current device is %d", P->device, dev);
+    return RR_OK;
+}
+
+rr_status check_ptrs(const void* const* ptrs, int32_t n, const char* what) {
+    if (n > 0 && !ptrs) return rr_fail(RR_EINVAL, "%s array is NULL", what);
+    for (int32_t i = 0; i < n; ++i)
+        if (!aligned16(ptrs[i]))
+            return rr_fail(RR_EINVAL, "%s[%d] is NULL or not 16-byte aligned", what, i);
+    return RR_OK;
+}
+
+template <int NPTR>
+rr_status launch_pack(const rr_plan* P, const void* const* src, void* const* buckets,
+                      uint64_t* checksums, bool table, uint64_t stride, cudaStream_t s) {
+    PackArgs<NPTR> a;
+    std::memset(&a, 0, sizeof a);
+    a.items = P->d_pack_items;
+    a.block_first = P->d_pack_block_first;
+    a.checksums = (unsigned long long*)checksums;
+    a.n_shards = P->n_shards;
+    for (int32_t i = 0; i < P->n_shards; ++i) a.ptr[i] = src[i];
+    if (table) {
+        for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[P->n_shards + b] = buckets[b];
+    } else {
+        a.bucket_base = (char*)buckets[0];
+        a.bucket_stride = stride;
+    }
+    rr_pack_kernel<NPTR><<<P->grid_blocks, kThreads, 0, s>>>(a);
+    RR_CUDA(cudaGetLastError());
+    return RR_OK;
+}
+
+template <int NPTR>
+rr_status launch_unpack(const rr_plan* P, const void* const* buckets, void* const* dst, bool table,
+                        uint64_t stride, cudaStream_t s) {
+    UnpackArgs<NPTR> a;
+    std::memset(&a, 0, sizeof a);
+    a.items = P->d_unpack_items;
+    a.block_first = P->d_unpack_block_first;
+    int32_t k = 0;
+    if (table) {
+        for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[k++] = buckets[b];
+    } else {
+        a.bucket_base = (const char*)buckets[0];
+        a.bucket_stride = stride;
+    }
+    a.dst_base = k;
+    for (int32_t t = 0; t < P->n_tensors; ++t) a.ptr[k++] = dst[t];
+    rr_unpack_kernel<NPTR><<<P->unpack_grid_blocks, kThreads, 0, s>>>(a);
+    RR_CUDA(cudaGetLastError());
+    return RR_OK;
+}
+
+template <int NPTR>
+rr_status launch_verify(const rr_plan* P, const void* const* buckets, const uint64_t* checksums,
+                        bool table, uint64_t stride, cudaStream_t s) {
+    VerifyArgs<NPTR> a;
+    std::memset(&a, 0, sizeof a);
+    a.sums = P->d_verify_scratch;
+    a.counters = P->d_verify_scratch + P->n_buckets;
+    a.expected = (const unsigned long long*)checksums;
+    a.bucket_bytes = (uint64_t)P->bucket_bytes;
+    a.chunk_bytes = (uint64_t)std::min<int64_t>(kVerifyChunk, P->bucket_bytes);
+    a.chunks_per_bucket = (a.bucket_bytes + a.chunk_bytes - 1) / a.chunk_bytes;
+    a.total_chunks = a.chunks_per_bucket * (uint64_t)P->n_buckets;
+    a.n_buckets = P->n_buckets;
+    if (table) {
+        for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[b] = buckets[b];
+    } else {
+        a.bucket_base = (const char*)buckets[0];
+        a.bucket_stride = stride;
+    }
+    rr_verify_kernel<NPTR><<<P->verify_grid_blocks, kThreads, 0, s>>>(a);
+    RR_CUDA(cudaGetLastError());
+    return RR_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Plan device state
+// ---------------------------------------------------------------------------
+
+rr_status rr_device_default_grid(int32_t* pack, int32_t* unpack, int32_t* verify) {
+    int dev = 0, sms = 0, p = 0, u = 0, v = 0;
+    RR_CUDA(cudaGetDevice(&dev));
+    RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, rr_verify_kernel<kLargePtrs>, kThreads, 0));
+    *pack = sms * (p > 0 ? p : 1);
+    *unpack = sms * (u > 0 ? u : 1);
+    *verify = sms * (v > 0 ? v : 1);
+    return RR_OK;
+}
+
+rr_status rr_device_upload(rr_plan* P) {
+    RR_CUDA(cudaGetDevice(&P->device));
+    auto up = [](void** d, const void* h, size_t bytes) -> cudaError_t {
+        cudaError_t e = cudaMalloc(d, bytes ? bytes : 16);
+        if (e != cudaSuccess) return e;
+        return bytes ? cudaMemcpy(*d, h, bytes, cudaMemcpyHostToDevice) : cudaSuccess;
+    };
+    cudaError_t e;
+    if ((e = up((void**)&P->d_pack_items, P->pack_items.data(),
+                P->pack_items.size() * sizeof(rr_pack_item))) != cudaSuccess ||
+        (e = up((void**)&P->d_pack_block_first, P->pack_block_first.data(),
+                P->pack_block_first.size() * sizeof(uint32_t))) != cudaSuccess ||
+        (e = up((void**)&P->d_unpack_items, P->unpack_items.data(),
+                P->unpack_items.size() * sizeof(rr_unpack_item))) != cudaSuccess ||
+        (e = up((void**)&P->d_unpack_block_first, P->unpack_block_first.data(),
+                P->unpack_block_first.size() * sizeof(uint32_t))) != cudaSuccess ||
+        (e = cudaMalloc((void**)&P->d_verify_scratch,
+                        (size_t(P->n_buckets) + 4) * sizeof(unsigned long long))) != cudaSuccess ||
+        (e = cudaHostAlloc((void**)&P->h_verify_result, 4 * sizeof(unsigned long long),
+                           cudaHostAllocDefault)) != cudaSuccess)
+        return e == cudaErrorMemoryAllocation ? rr_fail(RR_ENOMEM, "device allocation failed")
+                                              : cuda_fail(e, "plan upload");
+    return RR_OK;
+}
+
+void rr_device_release(rr_plan* P) {
+    if (!P || P->device < 0) return;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    if (prev != P->device) cudaSetDevice(P->device);
+    cudaFree(P->d_pack_items);
+    cudaFree(P->d_pack_block_first);
+    cudaFree(P->d_unpack_items);
+    cudaFree(P->d_unpack_block_first);
+    cudaFree(P->d_verify_scratch);
+    cudaFreeHost(P->h_verify_result);
+    P->d_pack_items = nullptr;
+    P->d_pack_block_first = nullptr;
+    P->d_unpack_items = nullptr;
+    P->d_unpack_block_first = nullptr;
+    P->d_verify_scratch = nullptr;
+    P->h_verify_result = nullptr;
+    if (prev >= 0 && prev != P->device) cudaSetDevice(prev);
+    P->device = -1;
+}
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+
+extern "C" rr_status rr_pack(const rr_plan* P, const void* const* src_shards,
+                             void* const* buckets, uint64_t* checksums, cudaStream_t stream) {
+    rr_clear_error();
+    rr_status st = check_plan(P);
+    if (st) return st;
+    if ((st = check_ptrs(src_shards, P->n_shards, "src_shards"))) return st;
+    if ((st = check_ptrs((const void* const*)buckets, P->n_buckets, "buckets"))) return st;
+    if (P->n_buckets == 0) return RR_OK;
+    if (!aligned16(checksums)) return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    uint64_t stride = 0;
+    const bool table = !uniform((const void* const*)buckets, P->n_buckets, P->bucket_bytes, &stride);
+    RR_CUDA(cudaMemsetAsync(checksums, 0, size_t(P->n_buckets) * 8, stream));
+    if (P->pack_items.empty()) return RR_OK;
+    const int32_t need = P->n_shards + (table ? P->n_buckets : 0);
+    if (need <= kSmallPtrs)
+        return launch_pack<kSmallPtrs>(P, src_shards, buckets, checksums, table, stride, stream);
+    if (need <= kLargePtrs)
+        return launch_pack<kLargePtrs>(P, src_shards, buckets, checksums, table, stride, stream);
+    return rr_fail(RR_EINVAL,
+                   "%d shards + %d separately allocated buckets exceed %d pointers; allocate the "
+                   "buckets as one equally spaced block",
+                   P->n_shards, P->n_buckets, kLargePtrs);
+}
+
+extern "C" rr_status rr_unpack(const rr_plan* P, const void* const* buckets, void* const* dst,
+                               cudaStream_t stream) {
+    rr_clear_error();
+    rr_status st = check_plan(P);
+    if (st) return st;
+    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if (P->n_tensors > 0 && !dst) return rr_fail(RR_EINVAL, "dst array is NULL");
+    for (int32_t t = 0; t < P->n_tensors; ++t)
+        if (P->tensor_numel[t] > 0 && !aligned16(dst[t]))
+            return rr_fail(RR_EINVAL, "dst[%d] is NULL or not 16-byte aligned", t);
+    if (P->unpack_items.empty()) return RR_OK;
+    uint64_t stride = 0;
+    const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
+    const int32_t need = P->n_tensors + (table ? P->n_buckets : 0);
+    if (need <= kSmallPtrs) return launch_unpack<kSmallPtrs>(P, buckets, dst, table, stride, stream);
+    if (need <= kLargePtrs) return launch_unpack<kLargePtrs>(P, buckets, dst, table, stride, stream);
+    return rr_fail(RR_EINVAL, "%d tensors + %d separately allocated buckets exceed %d pointers",
+                   P->n_tensors, P->n_buckets, kLargePtrs);
+}
+
+extern "C" rr_status rr_verify(const rr_plan* P, const void* const* buckets,
+                               const uint64_t* checksums, int64_t* n_bad, int64_t* first_bad,
+                               cudaStream_t stream) {
+    rr_clear_error();
+    rr_status st = check_plan(P);
+    if (st) return st;
+    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if (P->n_buckets > 0 && !aligned16(checksums))
+        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    if (n_bad) *n_bad = 0;
+    if (first_bad) *first_bad = -1;
+    if (P->n_buckets == 0) return RR_OK;
+    uint64_t stride = 0;
+    const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
+    if (table && P->n_buckets > kLargePtrs)
+        return rr_fail(RR_EINVAL, "%d separately allocated buckets exceed %d pointers",
+                       P->n_buckets, kLargePtrs);
+
+    rr_plan* M = const_cast<rr_plan*>(P);   // the scratch area is the only mutable state
+    std::lock_guard<std::mutex> lock(M->verify_mutex);
+    RR_CUDA(cudaMemsetAsync(P->d_verify_scratch, 0,
+                            (size_t(P->n_buckets) + 4) * sizeof(unsigned long long), stream));
+    st = (!table || P->n_buckets <= kSmallPtrs)
+             ? launch_verify<kSmallPtrs>(P, buckets, checksums, table, stride, stream)
+             : launch_verify<kLargePtrs>(P, buckets, checksums, table, stride, stream);
+    if (st) return st;
+    RR_CUDA(cudaMemcpyAsync(P->h_verify_result, P->d_verify_scratch + P->n_buckets,
+                            4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, stream));
+    RR_CUDA(cudaStreamSynchronize(stream));
+    const unsigned long long bad = P->h_verify_result[1];
+    if (n_bad) *n_bad = (int64_t)bad;
+    if (first_bad) *first_bad = bad ? (int64_t)(ULLONG_MAX - P->h_verify_result[2]) : -1;
+    return bad ? RR_EMISMATCH : RR_OK;
+}

@@ -1,0 +1,63 @@
+// Internal plan representation shared by the host planner (rr_plan.cpp) and
+// the device code (rr_device.cu).  Not part of the public ABI.
+#pragma once
+
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "rr.h"
+
+struct rr_plan {
+    // ---- source ---------------------------------------------------------
+    int32_t n_params = 0;
+    std::vector<int64_t> rows, cols;   // matrix view of each parameter
+    std::vector<int32_t> es;           // element bytes (4 or 2)
+    std::vector<int64_t> param_off;    // flat byte offsets
+    int32_t n_shards = 0;
+    int64_t shard_bytes = 0;           // S
+    int64_t flat_bytes = 0;
+
+    // ---- destination ----------------------------------------------------
+    int32_t tp = 0;
+    int32_t n_tensors = 0;
+    std::vector<int32_t> tensor_rank;
+    std::vector<int64_t> tensor_numel;
+    std::vector<int64_t> tensor_off;   // byte offset in its rank's stream
+    int64_t tensor_align = 0;
+    int64_t bucket_bytes = 0;
+    std::vector<int64_t> rank_stream_bytes;
+    std::vector<int32_t> rank_first_bucket;  // tp + 1
+    int32_t n_buckets = 0;
+
+    // ---- work tables ----------------------------------------------------
+    int32_t grid_blocks = 0;          // pack kernel grid
+    int32_t unpack_grid_blocks = 0;
+    int32_t verify_grid_blocks = 0;
+    int64_t chunk_bytes = 0;
+    bool host_only = false;
+    std::vector<rr_pack_item> pack_items;
+    std::vector<uint32_t> pack_block_first;     // grid_blocks + 1
+    std::vector<rr_unpack_item> unpack_items;
+    std::vector<uint32_t> unpack_block_first;   // grid_blocks + 1
+    rr_plan_stats stats{};
+
+    // ---- device state (owned) -------------------------------------------
+    int device = -1;
+    rr_pack_item* d_pack_items = nullptr;
+    uint32_t* d_pack_block_first = nullptr;
+    rr_unpack_item* d_unpack_items = nullptr;
+    uint32_t* d_unpack_block_first = nullptr;
+    unsigned long long* d_verify_scratch = nullptr;  // n_buckets sums + 4 counters
+    unsigned long long* h_verify_result = nullptr;   // pinned, 4 words
+    std::mutex verify_mutex;
+};
+
+// Records a per-thread error message and returns s.
+rr_status rr_fail(rr_status s, const char* fmt, ...);
+void rr_clear_error();
+
+// Device side (rr_device.cu).
+rr_status rr_device_default_grid(int32_t* pack, int32_t* unpack, int32_t* verify);
+rr_status rr_device_upload(rr_plan* p);
+void rr_device_release(rr_plan* p);

@@ -1,0 +1,536 @@
+// Host planner: compiles a manifest, a source shard layout, a destination
+// (rollout) layout and a bucket size into the work tables that the pack and
+// unpack kernels walk.
+//
+// RobustRL Section 5.2.1, step 1 ("reshard the model to align with the
+// sharding of the rollout") and step 2 ("placing the model layer by layer
+// into a buffer for transmission"): the plan is the reshard expressed as a
+// table of strided gathers, each landing in one fixed-size bucket.
+//
+// A work item never crosses a source shard, a bucket, or `chunk_bytes` of
+// destination; items are emitted rank by rank in stream order, so the table
+// is sorted by (bucket, offset).  Items whose addresses and lengths allow it
+// are 16-byte vector items; the rest (ragged heads and tails, misaligned
+// sources, odd row lengths) are scalar items.
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "rr_internal.h"
+
+namespace {
+
+thread_local std::string g_error;
+
+constexpr int64_t kDefaultChunkBytes = 32 * 1024;
+constexpr int64_t kItemOverhead = 1024;   // balancing weight of one item, in bytes
+constexpr int64_t kMaxShardOffset = (int64_t(1) << 48) - 1;
+
+int64_t align_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
+
+class Builder {
+public:
+    explicit Builder(rr_plan* p) : P(p), chunk_elems(p->chunk_bytes / 2) {}
+
+    // ---- pack ------------------------------------------------------------
+
+    // Emits the items of one strided run of parameter p: n rows of l elements,
+    // row i starting at parameter element first + i * st, landing contiguously
+    // in rank `rank`'s stream at byte `pos0`.
+    void pack_run(int32_t p, int64_t first, int64_t l, int64_t n, int64_t st, int32_t rank,
+                  int64_t pos0) {
+        if (l == 0 || n == 0) return;
+        const int32_t es = P->es[p];
+        const int64_t S = P->shard_bytes, B = P->bucket_bytes;
+        const int64_t fb = P->rank_first_bucket[rank];
+        int64_t i = 0, c = 0;
+        while (i < n) {
+            const int64_t pos = pos0 + 2 * (i * l + c);
+            const int64_t bl = pos / B, boff = pos - bl * B;
+            const int64_t brem = (B - boff) / 2;                      // elements left in bucket
+            const int64_t f = P->param_off[p] + (first + i * st + c) * es;
+            const int64_t sh = f / S, soff = f - sh * S;
+            const int64_t srem = (S - soff) / es;                     // elements left in shard
+            if (c == 0 && n - i > 1 && l <= chunk_elems) {
+                int64_t k = std::min({n - i, chunk_elems / l, brem / l});
+                const int64_t room = S - soff;
+                const int64_t kshard = room >= l * es ? (room - l * es) / (st * es) + 1 : 0;
+                k = std::min(k, kshard);
+                if (k >= 2) {
+                    pack_rows(es, sh, soff, fb + bl, boff, l, k, st);
+                    i += k;
+                    continue;
+                }
+            }
+            const int64_t len = std::min({l - c, chunk_elems, brem, srem});
+            pack_piece(es, sh, soff, fb + bl, boff, len);
+            c += len;
+            if (c == l) {
+                c = 0;
+                ++i;
+            }
+        }
+    }
+
+    // Zero fill of stream bytes [a, b) of rank `rank` (alignment gaps, last bucket's tail).
+    void zero_range(int32_t rank, int64_t a, int64_t b) {
+        const int64_t B = P->bucket_bytes;
+        const int64_t fb = P->rank_first_bucket[rank];
+        while (a < b) {
+            const int64_t bl = a / B, boff = a - bl * B;
+            const int64_t len = std::min({(b - a) / 2, (B - boff) / 2, chunk_elems});
+            split3(RR_ITEM_ZERO_VEC, RR_ITEM_ZERO_SCALAR, 2, 0, 0, fb + bl, boff, len, true);
+            a += 2 * len;
+        }
+    }
+
+    // ---- unpack ----------------------------------------------------------
+
+    void unpack_tensor(int32_t t) {
+        const int64_t B = P->bucket_bytes;
+        const int64_t fb = P->rank_first_bucket[P->tensor_rank[t]];
+        const int64_t nbytes = 2 * P->tensor_numel[t];
+        int64_t x = 0;
+        while (x < nbytes) {
+            const int64_t pos = P->tensor_off[t] + x;
+            const int64_t bl = pos / B, boff = pos - bl * B;
+            int64_t len = std::min({nbytes - x, B - boff, P->chunk_bytes});
+            copy_piece(fb + bl, boff, t, x, len);
+            x += len;
+        }
+    }
+
+    int64_t pack_read = 0;
+
+private:
+    rr_plan* P;
+    int64_t chunk_elems;
+
+    void emit_pack(int kind, int64_t shard, int64_t soff, int64_t bucket, int64_t boff,
+                   int64_t row_len, int64_t n_rows, int64_t stride) {
+        rr_pack_item it;
+        it.src = (uint64_t(shard) << 48) | uint64_t(soff);
+        it.dst_off = uint32_t(boff);
+        it.bucket = uint32_t(bucket);
+        it.row_len = uint32_t(row_len);
+        it.n_rows = uint32_t(n_rows);
+        it.src_stride = uint32_t(stride);
+        it.kind = uint16_t(kind);
+        it.reserved = 0;
+        P->pack_items.push_back(it);
+        if (kind <= RR_ITEM_BF16_SCALAR)
+            pack_read += row_len * n_rows * (kind <= RR_ITEM_F32_SCALAR ? 4 : 2);
+    }
+
+    // One row piece: scalar head up to 16-byte destination alignment, vector
+    // body when the source is then 16-byte aligned too, scalar tail.
+    void split3(int vec_kind, int sc_kind, int32_t es, int64_t shard, int64_t soff,
+                int64_t bucket, int64_t boff, int64_t len, bool src_free) {
+        int64_t h = ((16 - boff % 16) % 16) / 2;
+        h = std::min(h, len);
+        if (h) {
+            emit_pack(sc_kind, shard, soff, bucket, boff, h, 1, h);
+            soff += h * es;
+            boff += 2 * h;
+            len -= h;
+        }
+        const int64_t body = len / 8 * 8;
+        if (body && (src_free || soff % 16 == 0)) {
+            emit_pack(vec_kind, shard, soff, bucket, boff, body, 1, body);
+            soff += body * es;
+            boff += 2 * body;
+            len -= body;
+        }
+        if (len) emit_pack(sc_kind, shard, soff, bucket, boff, len, 1, len);
+    }
+
+    void pack_piece(int32_t es, int64_t shard, int64_t soff, int64_t bucket, int64_t boff,
+                    int64_t len) {
+        if (es == 4)
+            split3(RR_ITEM_F32_VEC, RR_ITEM_F32_SCALAR, 4, shard, soff, bucket, boff, len, false);
+        else
+            split3(RR_ITEM_BF16_VEC, RR_ITEM_BF16_SCALAR, 2, shard, soff, bucket, boff, len,
+                   false);
+    }
+
+    void pack_rows(int32_t es, int64_t shard, int64_t soff, int64_t bucket, int64_t boff,
+                   int64_t l, int64_t k, int64_t st) {
+        const bool vec = boff % 16 == 0 && l % 8 == 0 && soff % 16 == 0 && (st * es) % 16 == 0;
+        const int kind = es == 4 ? (vec ? RR_ITEM_F32_VEC : RR_ITEM_F32_SCALAR)
+                                 : (vec ? RR_ITEM_BF16_VEC : RR_ITEM_BF16_SCALAR);
+        emit_pack(kind, shard, soff, bucket, boff, l, k, st);
+    }
+
+    void emit_copy(int kind, int64_t bucket, int64_t boff, int32_t t, int64_t x, int64_t len) {
+        rr_unpack_item it;
+        it.dst_off = uint64_t(x);
+        it.src_off = uint32_t(boff);
+        it.bucket = uint32_t(bucket);
+        it.tensor = uint32_t(t);
+        it.nbytes = uint32_t(len);
+        it.kind = uint32_t(kind);
+        it.reserved = 0;
+        P->unpack_items.push_back(it);
+    }
+
+    void copy_piece(int64_t bucket, int64_t boff, int32_t t, int64_t x, int64_t len) {
+        if ((boff - x) % 16 != 0) {   // source and destination phases differ
+            emit_copy(RR_ITEM_COPY_SCALAR, bucket, boff, t, x, len);
+            return;
+        }
+        int64_t h = std::min((16 - boff % 16) % 16, len);
+        if (h) {
+            emit_copy(RR_ITEM_COPY_SCALAR, bucket, boff, t, x, h);
+            boff += h;
+            x += h;
+            len -= h;
+        }
+        const int64_t body = len / 16 * 16;
+        if (body) {
+            emit_copy(RR_ITEM_COPY_VEC, bucket, boff, t, x, body);
+            boff += body;
+            x += body;
+            len -= body;
+        }
+        if (len) emit_copy(RR_ITEM_COPY_SCALAR, bucket, boff, t, x, len);
+    }
+};
+
+int64_t pack_weight(const rr_pack_item& it) {
+    const int64_t n = int64_t(it.row_len) * it.n_rows;
+    switch (it.kind) {
+        case RR_ITEM_F32_VEC: return 6 * n + kItemOverhead;
+        case RR_ITEM_F32_SCALAR: return 12 * n + kItemOverhead;
+        case RR_ITEM_BF16_VEC: return 4 * n + kItemOverhead;
+        case RR_ITEM_BF16_SCALAR: return 8 * n + kItemOverhead;
+        default: return 2 * n + kItemOverhead;
+    }
+}
+
+int64_t unpack_weight(const rr_unpack_item& it) {
+    return (it.kind == RR_ITEM_COPY_VEC ? 2 : 4) * int64_t(it.nbytes) + kItemOverhead;
+}
+
+// Cuts items [0, n) into `grid` contiguous ranges of roughly equal weight.
+template <class Item, class W>
+void partition(const std::vector<Item>& items, int32_t grid, std::vector<uint32_t>& first, W w) {
+    first.assign(size_t(grid) + 1, uint32_t(items.size()));
+    first[0] = 0;
+    int64_t total = 0;
+    for (const Item& it : items) total += w(it);
+    int64_t cum = 0;
+    int32_t g = 1;
+    for (size_t i = 0; i < items.size() && g < grid; ++i) {
+        cum += w(items[i]);
+        while (g < grid && cum * grid >= total * g) first[g++] = uint32_t(i + 1);
+    }
+}
+
+rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_params,
+                                const rr_src_layout* src, const rr_dst_layout* dst,
+                                size_t bucket_bytes) {
+    if (n_params < 0 || (n_params > 0 && !manifest) || !src || !dst)
+        return rr_fail(RR_EINVAL, "null manifest / layout pointer or negative n_params");
+    if (bucket_bytes < 8 || bucket_bytes % 8 != 0 || bucket_bytes > (size_t(1) << 32) - 16)
+        return rr_fail(RR_EINVAL, "bucket_bytes must be a multiple of 8 in [8, 2^32 - 16]");
+    if (src->n_shards < 1 || src->n_shards > 65535)
+        return rr_fail(RR_EINVAL, "n_shards must be in [1, 65535]");
+    if (src->align_bytes < 1) return rr_fail(RR_EINVAL, "align_bytes must be >= 1");
+    if (dst->tp < 1) return rr_fail(RR_EINVAL, "tp must be >= 1");
+    if (dst->n_tensors < 0 || (dst->n_tensors > 0 && !dst->tensors))
+        return rr_fail(RR_EINVAL, "bad destination tensor list");
+    if (!is_pow2(dst->tensor_align_bytes) || dst->tensor_align_bytes < 2)
+        return rr_fail(RR_EINVAL, "tensor_align_bytes must be a power of two >= 2");
+
+    P->n_params = n_params;
+    P->rows.resize(n_params);
+    P->cols.resize(n_params);
+    P->es.resize(n_params);
+    P->param_off.resize(n_params);
+    for (int32_t p = 0; p < n_params; ++p) {
+        const rr_param& m = manifest[p];
+        if (m.ndim < 0 || m.ndim > 4) return rr_fail(RR_EINVAL, "param %d: ndim %d", p, m.ndim);
+        if (m.dtype != RR_F32 && m.dtype != RR_BF16)
+            return rr_fail(RR_EINVAL, "param %d: bad dtype", p);
+        int64_t rows = m.ndim ? m.shape[0] : 1, cols = 1;
+        for (int32_t d = 0; d < m.ndim; ++d)
+            if (m.shape[d] < 0) return rr_fail(RR_EINVAL, "param %d: negative dim", p);
+        for (int32_t d = 1; d < m.ndim; ++d) cols *= m.shape[d];
+        if (cols > 0xFFFFFFFFll) return rr_fail(RR_ELAYOUT, "param %d: row too long", p);
+        P->rows[p] = rows;
+        P->cols[p] = cols;
+        P->es[p] = m.dtype == RR_F32 ? 4 : 2;
+    }
+
+    // Source offsets.
+    int64_t end = 0;
+    if (src->param_flat_offset) {
+        std::vector<std::pair<int64_t, int64_t>> spans;
+        for (int32_t p = 0; p < n_params; ++p) {
+            const int64_t o = src->param_flat_offset[p];
+            const int64_t sz = P->rows[p] * P->cols[p] * P->es[p];
+            if (o < 0 || o % P->es[p] != 0)
+                return rr_fail(RR_ELAYOUT, "param %d: flat offset %lld not a multiple of %d", p,
+                               (long long)o, P->es[p]);
+            P->param_off[p] = o;
+            if (sz) spans.emplace_back(o, o + sz);
+            end = std::max(end, o + sz);
+        }
+        std::sort(spans.begin(), spans.end());
+        for (size_t i = 1; i < spans.size(); ++i)
+            if (spans[i].first < spans[i - 1].second)
+                return rr_fail(RR_ELAYOUT, "explicit parameter offsets overlap");
+    } else {
+        for (int32_t p = 0; p < n_params; ++p) {
+            end = align_up(end, std::max<int64_t>(src->align_bytes, P->es[p]));
+            P->param_off[p] = end;
+            end += P->rows[p] * P->cols[p] * P->es[p];
+        }
+    }
+    P->flat_bytes = end;
+    P->n_shards = src->n_shards;
+    P->shard_bytes = align_up(end, 16 * int64_t(src->n_shards)) / src->n_shards;
+    if (P->shard_bytes > kMaxShardOffset) return rr_fail(RR_ELAYOUT, "shards too large");
+
+    // Destination streams.
+    P->tp = dst->tp;
+    P->n_tensors = dst->n_tensors;
+    P->tensor_align = dst->tensor_align_bytes;
+    P->bucket_bytes = int64_t(bucket_bytes);
+    P->tensor_rank.resize(dst->n_tensors);
+    P->tensor_numel.resize(dst->n_tensors);
+    P->tensor_off.resize(dst->n_tensors);
+    P->rank_stream_bytes.assign(dst->tp, 0);
+    for (int32_t t = 0; t < dst->n_tensors; ++t) {
+        const rr_dst_tensor& T = dst->tensors[t];
+        if (T.rank < 0 || T.rank >= dst->tp)
+            return rr_fail(RR_ELAYOUT, "tensor %d: rank %d outside [0, %d)", t, T.rank, dst->tp);
+        if (T.n_blocks < 0 || (T.n_blocks > 0 && !T.blocks))
+            return rr_fail(RR_EINVAL, "tensor %d: bad block list", t);
+        int64_t numel = 0;
+        for (int32_t k = 0; k < T.n_blocks; ++k) {
+            const rr_block& b = T.blocks[k];
+            if (b.param < 0 || b.param >= n_params)
+                return rr_fail(RR_ELAYOUT, "tensor %d block %d: param %d out of range", t, k,
+                               b.param);
+            const int64_t R = P->rows[b.param], C = P->cols[b.param];
+            if (b.row0 < 0 || b.nrows < 0 || b.row0 + b.nrows > R || b.col0 < 0 || b.ncols < 0 ||
+                b.col0 + b.ncols > C)
+                return rr_fail(RR_ELAYOUT,
+                               "tensor %d block %d: rows [%lld,+%lld) cols [%lld,+%lld) outside "
+                               "param %d's [%lld, %lld]",
+                               t, k, (long long)b.row0, (long long)b.nrows, (long long)b.col0,
+                               (long long)b.ncols, b.param, (long long)R, (long long)C);
+            numel += b.nrows * b.ncols;
+        }
+        if (T.numel != numel)
+            return rr_fail(RR_ELAYOUT, "tensor %d: numel %lld but blocks cover %lld", t,
+                           (long long)T.numel, (long long)numel);
+        const int64_t start = align_up(P->rank_stream_bytes[T.rank], P->tensor_align);
+        P->tensor_rank[t] = T.rank;
+        P->tensor_numel[t] = numel;
+        P->tensor_off[t] = start;
+        P->rank_stream_bytes[T.rank] = start + 2 * numel;
+    }
+    P->rank_first_bucket.assign(size_t(dst->tp) + 1, 0);
+    int64_t nb = 0;
+    for (int32_t r = 0; r < dst->tp; ++r) {
+        nb += (P->rank_stream_bytes[r] + P->bucket_bytes - 1) / P->bucket_bytes;
+        if (nb > 0x7FFFFFFF) return rr_fail(RR_ELAYOUT, "too many buckets");
+        P->rank_first_bucket[r + 1] = int32_t(nb);
+    }
+    P->n_buckets = int32_t(nb);
+    return RR_OK;
+}
+
+void build_tables(rr_plan* P, const rr_dst_layout* dst) {
+    Builder b(P);
+    for (int32_t r = 0; r < P->tp; ++r) {
+        int64_t cursor = 0;   // end of the previous tensor in the stream
+        for (int32_t t = 0; t < P->n_tensors; ++t) {
+            if (P->tensor_rank[t] != r) continue;
+            b.zero_range(r, cursor, P->tensor_off[t]);
+            int64_t pos = P->tensor_off[t];
+            const rr_dst_tensor& T = dst->tensors[t];
+            for (int32_t k = 0; k < T.n_blocks; ++k) {
+                const rr_block& bl = T.blocks[k];
+                const int64_t C = P->cols[bl.param];
+                if (bl.ncols == C)   // whole rows: one contiguous run
+                    b.pack_run(bl.param, bl.row0 * C, bl.nrows * bl.ncols, 1, bl.nrows * bl.ncols,
+                               r, pos);
+                else
+                    b.pack_run(bl.param, bl.row0 * C + bl.col0, bl.ncols, bl.nrows, C, r, pos);
+                pos += 2 * bl.nrows * bl.ncols;
+            }
+            cursor = pos;
+        }
+        const int64_t nb = P->rank_first_bucket[r + 1] - P->rank_first_bucket[r];
+        b.zero_range(r, cursor, nb * P->bucket_bytes);
+        for (int32_t t = 0; t < P->n_tensors; ++t)
+            if (P->tensor_rank[t] == r) b.unpack_tensor(t);
+    }
+    partition(P->pack_items, P->grid_blocks, P->pack_block_first, pack_weight);
+    partition(P->unpack_items, P->unpack_grid_blocks, P->unpack_block_first, unpack_weight);
+
+    rr_plan_stats& s = P->stats;
+    s.n_pack_items = int64_t(P->pack_items.size());
+    s.n_unpack_items = int64_t(P->unpack_items.size());
+    s.grid_blocks = P->grid_blocks;
+    s.unpack_grid_blocks = P->unpack_grid_blocks;
+    s.verify_grid_blocks = P->verify_grid_blocks;
+    s.n_buckets = P->n_buckets;
+    s.n_shards = P->n_shards;
+    s.n_tensors = P->n_tensors;
+    s.bucket_bytes = P->bucket_bytes;
+    s.pack_bytes_read = b.pack_read;
+    s.pack_bytes_written = int64_t(P->n_buckets) * P->bucket_bytes;
+    int64_t dst_bytes = 0;
+    for (int32_t t = 0; t < P->n_tensors; ++t) dst_bytes += 2 * P->tensor_numel[t];
+    s.unpack_bytes_read = dst_bytes;
+    s.unpack_bytes_written = dst_bytes;
+    s.verify_bytes_read = int64_t(P->n_buckets) * P->bucket_bytes;
+}
+
+}  // namespace
+
+rr_status rr_fail(rr_status s, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_error = buf;
+    return s;
+}
+
+void rr_clear_error() { g_error.clear(); }
+
+extern "C" {
+
+rr_status rr_plan_create_ex(const rr_param* manifest, int32_t n_params,
+                            const rr_src_layout* src, const rr_dst_layout* dst,
+                            size_t bucket_bytes, const rr_plan_options* opts, rr_plan** out) {
+    rr_clear_error();
+    if (!out) return rr_fail(RR_EINVAL, "out is NULL");
+    *out = nullptr;
+    rr_plan* P = new (std::nothrow) rr_plan();
+    if (!P) return rr_fail(RR_ENOMEM, "host allocation failed");
+    rr_status st = RR_OK;
+    try {
+        st = validate_and_describe(P, manifest, n_params, src, dst, bucket_bytes);
+        if (st == RR_OK) {
+            P->host_only = opts && opts->host_only;
+            P->chunk_bytes = opts && opts->chunk_bytes ? opts->chunk_bytes : kDefaultChunkBytes;
+            if (P->chunk_bytes < 16 || P->chunk_bytes % 16 != 0 || P->chunk_bytes > (1 << 30))
+                st = rr_fail(RR_EINVAL, "chunk_bytes must be a multiple of 16 in [16, 2^30]");
+        }
+        if (st == RR_OK) {
+            if (opts && opts->grid_blocks > 0)
+                P->grid_blocks = P->unpack_grid_blocks = P->verify_grid_blocks = opts->grid_blocks;
+            else if (P->host_only)
+                P->grid_blocks = P->unpack_grid_blocks = P->verify_grid_blocks = 152 * 2;
+            else
+                st = rr_device_default_grid(&P->grid_blocks, &P->unpack_grid_blocks,
+                                            &P->verify_grid_blocks);
+        }
+        if (st == RR_OK) {
+            build_tables(P, dst);
+            if (P->pack_items.size() >= 0xFFFFFFFFull || P->unpack_items.size() >= 0xFFFFFFFFull)
+                st = rr_fail(RR_ELAYOUT, "too many work items; raise chunk_bytes");
+        }
+        if (st == RR_OK && !P->host_only) st = rr_device_upload(P);
+    } catch (const std::bad_alloc&) {
+        st = rr_fail(RR_ENOMEM, "host allocation failed while planning");
+    }
+    if (st != RR_OK) {
+        rr_device_release(P);
+        delete P;
+        return st;
+    }
+    *out = P;
+    return RR_OK;
+}
+
+rr_status rr_plan_create(const rr_param* manifest, int32_t n_params, const rr_src_layout* src,
+                         const rr_dst_layout* dst, size_t bucket_bytes, rr_plan** out) {
+    return rr_plan_create_ex(manifest, n_params, src, dst, bucket_bytes, nullptr, out);
+}
+
+void rr_plan_destroy(rr_plan* plan) {
+    if (!plan) return;
+    rr_device_release(plan);
+    delete plan;
+}
+
+rr_status rr_plan_query(const rr_plan* P, int32_t* n_buckets, int64_t* stream_bytes_per_rank,
+                        int32_t* first_bucket_of_rank) {
+    if (!P) return rr_fail(RR_EINVAL, "plan is NULL");
+    if (n_buckets) *n_buckets = P->n_buckets;
+    if (stream_bytes_per_rank)
+        std::copy(P->rank_stream_bytes.begin(), P->rank_stream_bytes.end(), stream_bytes_per_rank);
+    if (first_bucket_of_rank)
+        std::copy(P->rank_first_bucket.begin(), P->rank_first_bucket.end(), first_bucket_of_rank);
+    return RR_OK;
+}
+
+rr_status rr_plan_source(const rr_plan* P, int64_t* shard_bytes, int64_t* flat_bytes,
+                         int64_t* param_flat_offset) {
+    if (!P) return rr_fail(RR_EINVAL, "plan is NULL");
+    if (shard_bytes) *shard_bytes = P->shard_bytes;
+    if (flat_bytes) *flat_bytes = P->flat_bytes;
+    if (param_flat_offset) std::copy(P->param_off.begin(), P->param_off.end(), param_flat_offset);
+    return RR_OK;
+}
+
+rr_status rr_plan_tensors(const rr_plan* P, int64_t* tensor_numel, int64_t* tensor_stream_offset) {
+    if (!P) return rr_fail(RR_EINVAL, "plan is NULL");
+    if (tensor_numel) std::copy(P->tensor_numel.begin(), P->tensor_numel.end(), tensor_numel);
+    if (tensor_stream_offset)
+        std::copy(P->tensor_off.begin(), P->tensor_off.end(), tensor_stream_offset);
+    return RR_OK;
+}
+
+rr_status rr_plan_get_stats(const rr_plan* P, rr_plan_stats* stats) {
+    if (!P || !stats) return rr_fail(RR_EINVAL, "NULL argument");
+    *stats = P->stats;
+    return RR_OK;
+}
+
+rr_status rr_plan_export_pack(const rr_plan* P, rr_pack_item* items, int64_t cap,
+                              uint32_t* block_first) {
+    if (!P || (cap > 0 && !items)) return rr_fail(RR_EINVAL, "NULL argument");
+    const int64_t n = std::min<int64_t>(cap, int64_t(P->pack_items.size()));
+    if (n > 0) std::memcpy(items, P->pack_items.data(), size_t(n) * sizeof(rr_pack_item));
+    if (block_first)
+        std::copy(P->pack_block_first.begin(), P->pack_block_first.end(), block_first);
+    return RR_OK;
+}
+
+rr_status rr_plan_export_unpack(const rr_plan* P, rr_unpack_item* items, int64_t cap,
+                                uint32_t* block_first) {
+    if (!P || (cap > 0 && !items)) return rr_fail(RR_EINVAL, "NULL argument");
+    const int64_t n = std::min<int64_t>(cap, int64_t(P->unpack_items.size()));
+    if (n > 0) std::memcpy(items, P->unpack_items.data(), size_t(n) * sizeof(rr_unpack_item));
+    if (block_first)
+        std::copy(P->unpack_block_first.begin(), P->unpack_block_first.end(), block_first);
+    return RR_OK;
+}
+
+const char* rr_status_str(rr_status s) {
+    switch (s) {
+        case RR_OK: return "RR_OK";
+        case RR_EINVAL: return "RR_EINVAL: invalid argument";
+        case RR_ENOMEM: return "RR_ENOMEM: out of memory";
+        case RR_ECUDA: return "RR_ECUDA: CUDA error";
+        case RR_ELAYOUT: return "RR_ELAYOUT: inconsistent layout";
+        case RR_EMISMATCH: return "RR_EMISMATCH: checksum mismatch";
+    }
+    return "unknown rr_status";
+}
+
+const char* rr_last_error(void) { return g_error.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,141 @@
+"""Layout descriptions for Qwen3-family models: trainer manifest -> rollout tensors.
+
+The C library knows nothing about models; a weight sync is described to it
+as a parameter manifest plus, per rollout tensor, a list of 2-D blocks of
+those parameters.  This module writes those descriptions for Qwen3 dense and
+MoE decoders, as the paper's system uses them (RobustRL Section 7.1: FSDP
+trainer, vLLM rollout with tensor parallelism; Section 5.2.1 step 1: reshard
+"to align with the sharding of the rollout").
+
+Trainer manifest: module-registration order of the Hugging Face Qwen3 model.
+Rollout tensors, per rank r of TP = t, in this order:
+  embed_tokens        rows r of t of the embedding
+  per layer:          qkv_proj = [q; k; v] (row slices), o_proj (column slice),
+                      q_norm, k_norm, input_layernorm, post_attention_layernorm
+                      (replicated), then
+                      dense: gate_up_proj = [gate; up] (row slices), down_proj
+                             (column slice)
+                      MoE:   router (replicated), experts.w13 = stacked
+                             [gate_e; up_e] (row slices), experts.w2 = stacked
+                             down_e (column slices)
+  norm                replicated
+  lm_head             rows r of t, unless tied to the embedding
+"""
+from __future__ import annotations
+
+from typing import Dict, List, Tuple
+
+from .rr import Block, DstLayout, DstTensor, Param, SrcLayout
+
+
+def qwen3_manifest(shape, dtype: str = "f32") -> List[Param]:
+    """Trainer parameters of a Qwen3 decoder (``shape`` has layers, hidden, n_q,
+    n_kv, head_dim, intermediate, vocab, tied, n_experts, moe_intermediate)."""
+    h, d = shape.hidden, shape.head_dim
+    out = [Param("model.embed_tokens.weight", (shape.vocab, h), dtype)]
+    for i in range(shape.layers):
+        L = f"model.layers.{i}"
+        out += [Param(f"{L}.self_attn.q_proj.weight", (shape.n_q * d, h), dtype),
+                Param(f"{L}.self_attn.k_proj.weight", (shape.n_kv * d, h), dtype),
+                Param(f"{L}.self_attn.v_proj.weight", (shape.n_kv * d, h), dtype),
+                Param(f"{L}.self_attn.o_proj.weight", (h, shape.n_q * d), dtype),
+                Param(f"{L}.self_attn.q_norm.weight", (d,), dtype),
+                Param(f"{L}.self_attn.k_norm.weight", (d,), dtype)]
+        if getattr(shape, "n_experts", 0):
+            m = shape.moe_intermediate
+            out.append(Param(f"{L}.mlp.gate.weight", (shape.n_experts, h), dtype))
+            for e in range(shape.n_experts):
+                out += [Param(f"{L}.mlp.experts.{e}.gate_proj.weight", (m, h), dtype),
+                        Param(f"{L}.mlp.experts.{e}.up_proj.weight", (m, h), dtype),
+                        Param(f"{L}.mlp.experts.{e}.down_proj.weight", (h, m), dtype)]
+        else:
+            m = shape.intermediate
+            out += [Param(f"{L}.mlp.gate_proj.weight", (m, h), dtype),
+                    Param(f"{L}.mlp.up_proj.weight", (m, h), dtype),
+                    Param(f"{L}.mlp.down_proj.weight", (h, m), dtype)]
+        out += [Param(f"{L}.input_layernorm.weight", (h,), dtype),
+                Param(f"{L}.post_attention_layernorm.weight", (h,), dtype)]
+    out.append(Param("model.norm.weight", (h,), dtype))
+    if not shape.tied:
+        out.append(Param("lm_head.weight", (shape.vocab, h), dtype))
+    return out
+
+
+class _Slicer:
+    """Blocks of named parameters: whole, r-th row range, r-th column range."""
+
+    def __init__(self, manifest: List[Param], tp: int):
+        self.idx: Dict[str, int] = {p.name: i for i, p in enumerate(manifest)}
+        self.mat: Dict[str, Tuple[int, int]] = {}
+        for p in manifest:
+            rows = p.shape[0] if len(p.shape) else 1
+            cols = 1
+            for s in p.shape[1:]:
+                cols *= s
+            self.mat[p.name] = (rows, cols)
+        self.tp = tp
+
+    def whole(self, name: str) -> Block:
+        rows, cols = self.mat[name]
+        return Block(self.idx[name], 0, rows, 0, cols)
+
+    def rows(self, name: str, r: int) -> Block:
+        rows, cols = self.mat[name]
+        if rows % self.tp:
+            raise ValueError(f"{name}: {rows} rows do not divide over TP={self.tp}")
+        n = rows // self.tp
+        return Block(self.idx[name], r * n, n, 0, cols)
+
+    def cols(self, name: str, r: int) -> Block:
+        rows, cols = self.mat[name]
+        if cols % self.tp:
+            raise ValueError(f"{name}: {cols} columns do not divide over TP={self.tp}")
+        n = cols // self.tp
+        return Block(self.idx[name], 0, rows, r * n, n)
+
+
+def qwen3_rollout(shape, manifest: List[Param], tp: int = 1,
+                  tensor_align_bytes: int = 256) -> DstLayout:
+    """Rollout (inference-engine) tensors for TP = tp, rank-major."""
+    s = _Slicer(manifest, tp)
+    tensors: List[DstTensor] = []
+    for r in range(tp):
+        def add(name, blocks):
+            tensors.append(DstTensor(name, r, blocks))
+
+        add("embed_tokens", [s.rows("model.embed_tokens.weight", r)])
+        for i in range(shape.layers):
+            L = f"model.layers.{i}"
+            a = f"{L}.self_attn"
+            add(f"layers.{i}.qkv_proj", [s.rows(f"{a}.q_proj.weight", r),
+                                         s.rows(f"{a}.k_proj.weight", r),
+                                         s.rows(f"{a}.v_proj.weight", r)])
+            add(f"layers.{i}.o_proj", [s.cols(f"{a}.o_proj.weight", r)])
+            add(f"layers.{i}.q_norm", [s.whole(f"{a}.q_norm.weight")])
+            add(f"layers.{i}.k_norm", [s.whole(f"{a}.k_norm.weight")])
+            add(f"layers.{i}.input_layernorm", [s.whole(f"{L}.input_layernorm.weight")])
+            add(f"layers.{i}.post_attention_layernorm",
+                [s.whole(f"{L}.post_attention_layernorm.weight")])
+            if getattr(shape, "n_experts", 0):
+                E = shape.n_experts
+                x = f"{L}.mlp.experts"
+                add(f"layers.{i}.router", [s.whole(f"{L}.mlp.gate.weight")])
+                add(f"layers.{i}.experts.w13",
+                    [b for e in range(E) for b in (s.rows(f"{x}.{e}.gate_proj.weight", r),
+                                                   s.rows(f"{x}.{e}.up_proj.weight", r))])
+                add(f"layers.{i}.experts.w2",
+                    [s.cols(f"{x}.{e}.down_proj.weight", r) for e in range(E)])
+            else:
+                add(f"layers.{i}.gate_up_proj", [s.rows(f"{L}.mlp.gate_proj.weight", r),
+                                                 s.rows(f"{L}.mlp.up_proj.weight", r)])
+                add(f"layers.{i}.down_proj", [s.cols(f"{L}.mlp.down_proj.weight", r)])
+        add("norm", [s.whole("model.norm.weight")])
+        if not shape.tied:
+            add("lm_head", [s.rows("lm_head.weight", r)])
+    return DstLayout(tp=tp, tensors=tensors, tensor_align_bytes=tensor_align_bytes)
+
+
+def qwen3_sync(shape, dtype: str, n_shards: int, tp: int):
+    """(manifest, source layout, destination layout) for one Qwen3 weight sync."""
+    manifest = qwen3_manifest(shape, dtype)
+    return manifest, SrcLayout(n_shards=n_shards, align_bytes=16), qwen3_rollout(shape, manifest, tp)

@@ -1,0 +1,400 @@
+"""Python binding of the weight-sync C ABI (include/rr.h): argument marshalling only.
+
+Every step of the path runs in the CUDA library ``librr.so``; this module
+turns Python descriptions and torch tensors into the plain structs, pointers
+and sizes that the ABI takes.  There is no fallback: if the library cannot be
+loaded, importing this module raises.
+
+Functions carry the ABI's names: ``rr_plan_create``, ``rr_pack``,
+``rr_unpack``, ``rr_verify`` (RobustRL Section 5.2.1 steps 1-2 and
+Section 5.2.2), plus the plan queries.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import List, Optional, Sequence
+
+from . import build as _build
+
+# ---------------------------------------------------------------------------
+# Library
+# ---------------------------------------------------------------------------
+
+if not os.path.exists(_build.LIB):
+    raise ImportError(
+        f"{_build.LIB} is missing: build it with `python -m paper_2512_22492_gb300.build` "
+        "(needs nvcc); there is no CPU fallback")
+_lib = ctypes.CDLL(_build.LIB)
+
+RR_OK, RR_EINVAL, RR_ENOMEM, RR_ECUDA, RR_ELAYOUT, RR_EMISMATCH = range(6)
+RR_F32, RR_BF16 = 0, 1
+(RR_ITEM_F32_VEC, RR_ITEM_F32_SCALAR, RR_ITEM_BF16_VEC, RR_ITEM_BF16_SCALAR, RR_ITEM_ZERO_VEC,
+ RR_ITEM_ZERO_SCALAR, RR_ITEM_COPY_VEC, RR_ITEM_COPY_SCALAR) = range(8)
+
+
+class _Param(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char_p), ("ndim", ctypes.c_int32),
+                ("shape", ctypes.c_int64 * 4), ("dtype", ctypes.c_int)]
+
+
+class _SrcLayout(ctypes.Structure):
+    _fields_ = [("n_shards", ctypes.c_int32), ("align_bytes", ctypes.c_int64),
+                ("param_flat_offset", ctypes.POINTER(ctypes.c_int64))]
+
+
+class _Block(ctypes.Structure):
+    _fields_ = [("param", ctypes.c_int32), ("row0", ctypes.c_int64), ("nrows", ctypes.c_int64),
+                ("col0", ctypes.c_int64), ("ncols", ctypes.c_int64)]
+
+
+class _DstTensor(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char_p), ("rank", ctypes.c_int32), ("numel", ctypes.c_int64),
+                ("n_blocks", ctypes.c_int32), ("blocks", ctypes.POINTER(_Block))]
+
+
+class _DstLayout(ctypes.Structure):
+    _fields_ = [("tp", ctypes.c_int32), ("n_tensors", ctypes.c_int32),
+                ("tensors", ctypes.POINTER(_DstTensor)), ("tensor_align_bytes", ctypes.c_int64)]
+
+
+class _Options(ctypes.Structure):
+    _fields_ = [("host_only", ctypes.c_int32), ("grid_blocks", ctypes.c_int32),
+                ("chunk_bytes", ctypes.c_int64)]
+
+
+class _Stats(ctypes.Structure):
+    _fields_ = [("n_pack_items", ctypes.c_int64), ("n_unpack_items", ctypes.c_int64),
+                ("grid_blocks", ctypes.c_int32), ("unpack_grid_blocks", ctypes.c_int32),
+                ("verify_grid_blocks", ctypes.c_int32), ("n_buckets", ctypes.c_int32),
+                ("n_shards", ctypes.c_int32), ("n_tensors", ctypes.c_int32),
+                ("bucket_bytes", ctypes.c_int64),
+                ("pack_bytes_read", ctypes.c_int64), ("pack_bytes_written", ctypes.c_int64),
+                ("unpack_bytes_read", ctypes.c_int64), ("unpack_bytes_written", ctypes.c_int64),
+                ("verify_bytes_read", ctypes.c_int64)]
+
+
+class PackItem(ctypes.Structure):
+    _fields_ = [("src", ctypes.c_uint64), ("dst_off", ctypes.c_uint32),
+                ("bucket", ctypes.c_uint32), ("row_len", ctypes.c_uint32),
+                ("n_rows", ctypes.c_uint32), ("src_stride", ctypes.c_uint32),
+                ("kind", ctypes.c_uint16), ("reserved", ctypes.c_uint16)]
+
+
+class UnpackItem(ctypes.Structure):
+    _fields_ = [("dst_off", ctypes.c_uint64), ("src_off", ctypes.c_uint32),
+                ("bucket", ctypes.c_uint32), ("tensor", ctypes.c_uint32),
+                ("nbytes", ctypes.c_uint32), ("kind", ctypes.c_uint32),
+                ("reserved", ctypes.c_uint32)]
+
+
+def _np_dtype(struct):
+    import numpy as np
+    m = {ctypes.c_uint64: "<u8", ctypes.c_uint32: "<u4", ctypes.c_uint16: "<u2"}
+    return np.dtype({"names": [f for f, _ in struct._fields_],
+                     "formats": [m[t] for _, t in struct._fields_],
+                     "offsets": [getattr(struct, f).offset for f, _ in struct._fields_],
+                     "itemsize": ctypes.sizeof(struct)})
+
+
+PACK_ITEM_DTYPE = _np_dtype(PackItem)
+UNPACK_ITEM_DTYPE = _np_dtype(UnpackItem)
+
+_vp = ctypes.c_void_p
+_P64 = ctypes.POINTER(ctypes.c_int64)
+_P32 = ctypes.POINTER(ctypes.c_int32)
+
+
+def _sig(name, args, res=ctypes.c_int):
+    f = getattr(_lib, name)
+    f.argtypes = args
+    f.restype = res
+    return f
+
+
+_sig("rr_plan_create_ex", [ctypes.POINTER(_Param), ctypes.c_int32, ctypes.POINTER(_SrcLayout),
+                           ctypes.POINTER(_DstLayout), ctypes.c_size_t, ctypes.POINTER(_Options),
+                           ctypes.POINTER(_vp)])
+_sig("rr_plan_create", [ctypes.POINTER(_Param), ctypes.c_int32, ctypes.POINTER(_SrcLayout),
+                        ctypes.POINTER(_DstLayout), ctypes.c_size_t, ctypes.POINTER(_vp)])
+_sig("rr_plan_destroy", [_vp], None)
+_sig("rr_plan_query", [_vp, _P32, _P64, _P32])
+_sig("rr_plan_source", [_vp, _P64, _P64, _P64])
+_sig("rr_plan_tensors", [_vp, _P64, _P64])
+_sig("rr_plan_get_stats", [_vp, ctypes.POINTER(_Stats)])
+_sig("rr_plan_export_pack", [_vp, ctypes.POINTER(PackItem), ctypes.c_int64,
+                             ctypes.POINTER(ctypes.c_uint32)])
+_sig("rr_plan_export_unpack", [_vp, ctypes.POINTER(UnpackItem), ctypes.c_int64,
+                               ctypes.POINTER(ctypes.c_uint32)])
+_sig("rr_pack", [_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _vp])
+_sig("rr_unpack", [_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp])
+_sig("rr_verify", [_vp, ctypes.POINTER(_vp), _vp, _P64, _P64, _vp])
+_sig("rr_status_str", [ctypes.c_int], ctypes.c_char_p)
+_sig("rr_last_error", [], ctypes.c_char_p)
+
+LIBRARY_PATH = _build.LIB
+EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_query",
+            "rr_plan_source", "rr_plan_tensors", "rr_plan_get_stats", "rr_plan_export_pack",
+            "rr_plan_export_unpack", "rr_pack", "rr_unpack", "rr_verify", "rr_status_str",
+            "rr_last_error")
+
+
+class RRError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        detail = _lib.rr_last_error().decode()
+        super().__init__(f"{what}: {_lib.rr_status_str(status).decode()}"
+                         + (f" ({detail})" if detail else ""))
+
+
+def _check(status: int, what: str) -> None:
+    if status != RR_OK:
+        raise RRError(status, what)
+
+
+def rr_status_str(status: int) -> str:
+    return _lib.rr_status_str(status).decode()
+
+
+# ---------------------------------------------------------------------------
+# Descriptions
+# ---------------------------------------------------------------------------
+
+@dataclass
+class Param:
+    name: str
+    shape: Sequence[int]
+    dtype: str = "f32"    # "f32" or "bf16"
+
+
+@dataclass
+class SrcLayout:
+    n_shards: int
+    align_bytes: int = 16
+    param_flat_offset: Optional[Sequence[int]] = None
+
+
+@dataclass
+class Block:
+    param: int
+    row0: int
+    nrows: int
+    col0: int
+    ncols: int
+
+
+@dataclass
+class DstTensor:
+    name: str
+    rank: int
+    blocks: List[Block]
+    numel: Optional[int] = None   # default: sum of the blocks
+
+    def size(self) -> int:
+        return sum(b.nrows * b.ncols for b in self.blocks) if self.numel is None else self.numel
+
+
+@dataclass
+class DstLayout:
+    tp: int
+    tensors: List[DstTensor]
+    tensor_align_bytes: int = 256
+
+
+@dataclass
+class PlanOptions:
+    host_only: bool = False
+    grid_blocks: int = 0
+    chunk_bytes: int = 0
+
+
+# ---------------------------------------------------------------------------
+# Plan
+# ---------------------------------------------------------------------------
+
+class Plan:
+    """Owns an rr_plan; exposes its geometry."""
+
+    def __init__(self, handle: int, n_params: int, dst: DstLayout):
+        self._h = ctypes.c_void_p(handle)
+        self.n_params = n_params
+        self.tp = dst.tp
+        self.n_tensors = len(dst.tensors)
+        self.tensor_names = [t.name for t in dst.tensors]
+        self.tensor_ranks = [t.rank for t in dst.tensors]
+        st = self.stats()
+        self.n_buckets = st["n_buckets"]
+        self.bucket_bytes = st["bucket_bytes"]
+        self.n_shards = st["n_shards"]
+        self.grid_blocks = st["grid_blocks"]
+        self._unpack_grid = st["unpack_grid_blocks"]
+        sb = (ctypes.c_int64 * self.tp)()
+        fb = (ctypes.c_int32 * (self.tp + 1))()
+        nb = ctypes.c_int32()
+        _check(_lib.rr_plan_query(self._h, ctypes.byref(nb), sb, fb), "rr_plan_query")
+        self.stream_bytes_per_rank = list(sb)
+        self.first_bucket_of_rank = list(fb)
+        shard = ctypes.c_int64()
+        flat = ctypes.c_int64()
+        offs = (ctypes.c_int64 * max(1, n_params))()
+        _check(_lib.rr_plan_source(self._h, ctypes.byref(shard), ctypes.byref(flat), offs),
+               "rr_plan_source")
+        self.shard_bytes = shard.value
+        self.flat_bytes = flat.value
+        self.param_flat_offset = list(offs)[:n_params]
+        numel = (ctypes.c_int64 * max(1, self.n_tensors))()
+        toff = (ctypes.c_int64 * max(1, self.n_tensors))()
+        _check(_lib.rr_plan_tensors(self._h, numel, toff), "rr_plan_tensors")
+        self.tensor_numel = list(numel)[:self.n_tensors]
+        self.tensor_stream_offset = list(toff)[:self.n_tensors]
+
+    @property
+    def handle(self) -> ctypes.c_void_p:
+        if not self._h:
+            raise ValueError("plan destroyed")
+        return self._h
+
+    def stats(self) -> dict:
+        s = _Stats()
+        _check(_lib.rr_plan_get_stats(self._h, ctypes.byref(s)), "rr_plan_get_stats")
+        return {k: getattr(s, k) for k, _ in _Stats._fields_}
+
+    def export_pack(self):
+        """(items as a numpy structured array, per-block first item)."""
+        import numpy as np
+        n = self.stats()["n_pack_items"]
+        items = np.zeros(max(1, n), dtype=PACK_ITEM_DTYPE)
+        first = np.zeros(self.stats()["grid_blocks"] + 1, dtype=np.uint32)
+        _check(_lib.rr_plan_export_pack(self._h, items.ctypes.data_as(ctypes.POINTER(PackItem)),
+                                        n, first.ctypes.data_as(ctypes.POINTER(ctypes.c_uint32))),
+               "rr_plan_export_pack")
+        return items[:n], first
+
+    def export_unpack(self):
+        import numpy as np
+        n = self.stats()["n_unpack_items"]
+        items = np.zeros(max(1, n), dtype=UNPACK_ITEM_DTYPE)
+        # The unpack table is cut for the unpack kernel's own grid.
+        first = np.zeros(self._unpack_grid + 1, dtype=np.uint32)
+        _check(_lib.rr_plan_export_unpack(self._h,
+                                          items.ctypes.data_as(ctypes.POINTER(UnpackItem)), n,
+                                          first.ctypes.data_as(ctypes.POINTER(ctypes.c_uint32))),
+               "rr_plan_export_unpack")
+        return items[:n], first
+
+    def destroy(self) -> None:
+        if self._h:
+            _lib.rr_plan_destroy(self._h)
+            self._h = ctypes.c_void_p(0)
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
+                   bucket_bytes: int, options: Optional[PlanOptions] = None) -> Plan:
+    n = len(manifest)
+    cp = (_Param * max(1, n))()
+    names = []
+    for i, p in enumerate(manifest):
+        nm = p.name.encode()
+        names.append(nm)
+        cp[i].name = nm
+        cp[i].ndim = len(p.shape)
+        for d, s in enumerate(p.shape):
+            cp[i].shape[d] = s
+        cp[i].dtype = RR_F32 if p.dtype == "f32" else RR_BF16
+    cs = _SrcLayout(n_shards=src.n_shards, align_bytes=src.align_bytes)
+    offs = None
+    if src.param_flat_offset is not None:
+        offs = (ctypes.c_int64 * max(1, n))(*src.param_flat_offset)
+        cs.param_flat_offset = offs
+    keep = []
+    ct = (_DstTensor * max(1, len(dst.tensors)))()
+    for i, t in enumerate(dst.tensors):
+        cb = (_Block * max(1, len(t.blocks)))()
+        for k, b in enumerate(t.blocks):
+            cb[k].param, cb[k].row0, cb[k].nrows, cb[k].col0, cb[k].ncols = \
+                b.param, b.row0, b.nrows, b.col0, b.ncols
+        nm = t.name.encode()
+        keep += [cb, nm]
+        ct[i].name = nm
+        ct[i].rank = t.rank
+        ct[i].numel = t.size()
+        ct[i].n_blocks = len(t.blocks)
+        ct[i].blocks = ctypes.cast(cb, ctypes.POINTER(_Block))
+    cd = _DstLayout(tp=dst.tp, n_tensors=len(dst.tensors),
+                    tensors=ctypes.cast(ct, ctypes.POINTER(_DstTensor)),
+                    tensor_align_bytes=dst.tensor_align_bytes)
+    out = ctypes.c_void_p()
+    if options is None:
+        st = _lib.rr_plan_create(cp, n, ctypes.byref(cs), ctypes.byref(cd), bucket_bytes,
+                                 ctypes.byref(out))
+    else:
+        co = _Options(host_only=int(options.host_only), grid_blocks=options.grid_blocks,
+                      chunk_bytes=options.chunk_bytes)
+        st = _lib.rr_plan_create_ex(cp, n, ctypes.byref(cs), ctypes.byref(cd), bucket_bytes,
+                                    ctypes.byref(co), ctypes.byref(out))
+    _check(st, "rr_plan_create")
+    return Plan(out.value, n, dst)
+
+
+# ---------------------------------------------------------------------------
+# Pointers and streams
+# ---------------------------------------------------------------------------
+
+def _ptr(x) -> int:
+    if isinstance(x, int):
+        return x
+    return int(x.data_ptr())
+
+
+def _ptr_array(xs) -> ctypes.Array:
+    """Host array of device pointers from tensors / ints, or the rows of a 2-D tensor."""
+    if hasattr(xs, "dim") and xs.dim() == 2:
+        base = xs.data_ptr()
+        step = xs.stride(0) * xs.element_size()
+        ptrs = [base + i * step for i in range(xs.shape[0])]
+    else:
+        ptrs = [_ptr(x) for x in xs]
+    return (ctypes.c_void_p * max(1, len(ptrs)))(*ptrs)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return int(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return stream
+    return int(stream.cuda_stream)
+
+
+# ---------------------------------------------------------------------------
+# Hot path
+# ---------------------------------------------------------------------------
+
+def rr_pack(plan: Plan, src_shards, buckets, checksums, stream=None) -> None:
+    """Reshard + cast + pack + checksum (asynchronous on `stream`)."""
+    _check(_lib.rr_pack(plan.handle, _ptr_array(src_shards), _ptr_array(buckets),
+                        _ptr(checksums), _stream(stream)), "rr_pack")
+
+
+def rr_unpack(plan: Plan, buckets, dst, stream=None) -> None:
+    """Buckets -> destination tensors (asynchronous on `stream`)."""
+    _check(_lib.rr_unpack(plan.handle, _ptr_array(buckets), _ptr_array(dst), _stream(stream)),
+           "rr_unpack")
+
+
+def rr_verify(plan: Plan, buckets, checksums, stream=None):
+    """Recompute and compare checksums; returns (n_bad, first_bad).  Synchronous."""
+    n_bad = ctypes.c_int64()
+    first = ctypes.c_int64()
+    st = _lib.rr_verify(plan.handle, _ptr_array(buckets), _ptr(checksums), ctypes.byref(n_bad),
+                        ctypes.byref(first), _stream(stream))
+    if st not in (RR_OK, RR_EMISMATCH):
+        _check(st, "rr_verify")
+    return n_bad.value, first.value

@@ -1,0 +1,150 @@
+"""Shared test helpers: layout descriptions handed to both sides, and a numpy
+interpreter of the library's exported work tables (host-side planner checks).
+
+A description is plain data (params, tensors, sizes); ``to_oracle`` and
+``to_product`` turn the same description into the oracle's and the library's
+inputs, so neither side's code reaches the other.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle
+import synth
+
+ITEM_F32_VEC, ITEM_F32_SCALAR, ITEM_BF16_VEC, ITEM_BF16_SCALAR, ITEM_ZERO_VEC, \
+    ITEM_ZERO_SCALAR, ITEM_COPY_VEC, ITEM_COPY_SCALAR = range(8)
+
+
+def workload(name):
+    return synth.WORKLOADS.get(name) or synth.TEST_WORKLOADS[name]
+
+
+# ---------------------------------------------------------------------------
+# Random adversarial layouts
+# ---------------------------------------------------------------------------
+
+def random_layout(seed: int, max_params: int = 7, bucket_choices=(8, 24, 40, 64, 200, 4096, 65536)):
+    """Odd shapes, mixed dtypes, mid-row shard cuts, tiny buckets, ragged blocks."""
+    rng = np.random.default_rng(seed)
+    n_params = int(rng.integers(1, max_params + 1))
+    params = []
+    for i in range(n_params):
+        es = int(rng.choice([2, 4]))
+        nd = int(rng.integers(1, 4))
+        dims = tuple(int(rng.integers(1, 70)) for _ in range(nd))
+        params.append((f"p{i}", dims, es))
+    tp = int(rng.integers(1, 4))
+    tensors = []
+    for t in range(int(rng.integers(1, 9))):
+        blocks = []
+        for _ in range(int(rng.integers(1, 4))):
+            p = int(rng.integers(0, n_params))
+            dims = params[p][1]
+            rows = dims[0]
+            cols = int(np.prod(dims[1:])) if len(dims) > 1 else 1
+            r0 = int(rng.integers(0, rows))
+            nr = int(rng.integers(0, rows - r0 + 1))
+            if rng.random() < 0.4:
+                c0, nc = 0, cols
+            else:
+                c0 = int(rng.integers(0, cols))
+                nc = int(rng.integers(0, cols - c0 + 1))
+            blocks.append((p, r0, nr, c0, nc))
+        tensors.append((f"t{t}", int(rng.integers(0, tp)), blocks))
+    return dict(params=params, tensors=tensors, tp=tp,
+                n_shards=int(rng.integers(1, 6)),
+                bucket_bytes=int(rng.choice(bucket_choices)),
+                align_bytes=int(rng.choice([1, 2, 4, 8, 16, 32])),
+                tensor_align=int(rng.choice([2, 4, 16, 256])),
+                seed=int(rng.integers(1, 1 << 20)), specials=bool(rng.random() < 0.5))
+
+
+def workload_desc(name, bucket_bytes=None):
+    w = workload(name)
+    from oracle import qwen3
+    params = qwen3.manifest(w.shape, w.src_elem_bytes)
+    return dict(params=params, tensors=None, workload=w, tp=w.tp, n_shards=w.n_shards,
+                bucket_bytes=bucket_bytes or w.bucket_bytes, align_bytes=16, tensor_align=256,
+                seed=w.seed, specials=w.specials)
+
+
+def to_oracle(desc) -> "oracle.Layout":
+    if desc.get("workload") is not None:
+        return oracle.workload_layout(desc["workload"], bucket_bytes=desc["bucket_bytes"])
+    return oracle.Layout(desc["params"], desc["tensors"], n_shards=desc["n_shards"],
+                         tp=desc["tp"], bucket_bytes=desc["bucket_bytes"],
+                         align_bytes=desc["align_bytes"], tensor_align=desc["tensor_align"])
+
+
+def to_product(desc):
+    import paper_2512_22492_gb300 as rr
+    if desc.get("workload") is not None:
+        w = desc["workload"]
+        return rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp)
+    manifest = [rr.Param(n, d, "f32" if es == 4 else "bf16") for n, d, es in desc["params"]]
+    src = rr.SrcLayout(n_shards=desc["n_shards"], align_bytes=desc["align_bytes"])
+    dst = rr.DstLayout(tp=desc["tp"], tensor_align_bytes=desc["tensor_align"],
+                       tensors=[rr.DstTensor(n, r, [rr.Block(*b) for b in blocks])
+                                for n, r, blocks in desc["tensors"]])
+    return manifest, src, dst
+
+
+# ---------------------------------------------------------------------------
+# Work-table interpreter (what the kernels are specified to do with each item)
+# ---------------------------------------------------------------------------
+
+def check_and_run_pack(items, shards, n_buckets, bucket_bytes, shard_bytes):
+    """Applies pack items to host shards; asserts every item's preconditions and
+    that every bucket byte is written exactly once.  Returns the buckets."""
+    out = np.zeros((n_buckets, bucket_bytes), np.uint8)
+    hits = np.zeros((n_buckets, bucket_bytes), np.uint16)
+    for it in items:
+        kind, b, off = int(it["kind"]), int(it["bucket"]), int(it["dst_off"])
+        L, R, st = int(it["row_len"]), int(it["n_rows"]), int(it["src_stride"])
+        n = L * R
+        assert 0 <= b < n_buckets and off % 2 == 0 and off + 2 * n <= bucket_bytes
+        hits[b, off:off + 2 * n] += 1
+        if kind in (ITEM_ZERO_VEC, ITEM_ZERO_SCALAR):
+            assert R == 1
+            if kind == ITEM_ZERO_VEC:
+                assert off % 16 == 0 and L % 8 == 0
+            out[b, off:off + 2 * n] = 0
+            continue
+        es = 4 if kind in (ITEM_F32_VEC, ITEM_F32_SCALAR) else 2
+        shard, soff = int(it["src"]) >> 48, int(it["src"]) & ((1 << 48) - 1)
+        if kind in (ITEM_F32_VEC, ITEM_BF16_VEC):
+            assert off % 16 == 0 and L % 8 == 0 and soff % 16 == 0
+            assert R == 1 or (st * es) % 16 == 0
+        assert soff + ((R - 1) * st + L) * es <= shard_bytes
+        idx = soff + (np.arange(R, dtype=np.int64)[:, None] * st * es
+                      + np.arange(L, dtype=np.int64)[None, :] * es).ravel()
+        raw = np.zeros(idx.size, np.uint32)
+        for k in range(es):
+            raw |= shards[shard][idx + k].astype(np.uint32) << (8 * k)
+        vals = oracle.rne_bf16(raw) if es == 4 else raw.astype(np.uint16)
+        out[b, off:off + 2 * n] = vals.astype("<u2").view(np.uint8)
+    assert hits.min() == 1 and hits.max() == 1, "bucket bytes not written exactly once"
+    return out
+
+
+def check_and_run_unpack(items, buckets, tensor_numel):
+    dst = [np.zeros(2 * n, np.uint8) for n in tensor_numel]
+    hits = [np.zeros(2 * n, np.uint16) for n in tensor_numel]
+    for it in items:
+        kind, b, so = int(it["kind"]), int(it["bucket"]), int(it["src_off"])
+        t, do, nb = int(it["tensor"]), int(it["dst_off"]), int(it["nbytes"])
+        assert nb % 2 == 0 and so + nb <= buckets.shape[1] and do + nb <= dst[t].size
+        if kind == ITEM_COPY_VEC:
+            assert so % 16 == 0 and do % 16 == 0 and nb % 16 == 0
+        dst[t][do:do + nb] = buckets[b, so:so + nb]
+        hits[t][do:do + nb] += 1
+    for h in hits:
+        assert h.size == 0 or (h.min() == 1 and h.max() == 1), "dst bytes not written once"
+    return [d.view("<u2") for d in dst]
+
+
+def check_partition(first, n_items):
+    first = np.asarray(first, np.int64)
+    assert first[0] == 0 and first[-1] == n_items
+    assert np.all(np.diff(first) >= 0)

@@ -1,0 +1,125 @@
+"""GPU-side test/bench harness: device buffers for one weight sync, filled from
+host shards or by the device generator, and runs of the library's calls.
+
+Used by the -m gpu tests, the smoke check and the benchmark.  It imports the
+library (the product) and ``synth`` (inputs), never the oracle.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+from typing import List, Optional
+
+import numpy as np
+import torch
+
+import synth
+import paper_2512_22492_gb300 as rr
+
+
+@dataclass
+class SyncBuffers:
+    plan: "rr.Plan"
+    flat: torch.Tensor                 # n_shards * shard_bytes, uint8
+    shards: List[int]                  # device pointers into flat
+    bucket_store: torch.Tensor         # [n_buckets, bucket_bytes] uint8 (uniform layout)
+    buckets: list                      # what is passed as the bucket array
+    checksums: torch.Tensor            # [n_buckets] int64 (uint64 bits)
+    dst: List[torch.Tensor]            # one int16 tensor per destination tensor
+
+
+def make_plan(manifest, src, dst, bucket_bytes, **opts):
+    options = rr.PlanOptions(**opts) if opts else None
+    return rr.rr_plan_create(manifest, src, dst, bucket_bytes, options)
+
+
+def alloc(plan, separate_buckets: bool = False, poison: Optional[int] = 0xAB,
+          with_dst: bool = True, flat: Optional[torch.Tensor] = None) -> SyncBuffers:
+    dev = torch.device("cuda")
+    if flat is None:
+        flat = torch.zeros(plan.n_shards * plan.shard_bytes, dtype=torch.uint8, device=dev)
+    assert flat.numel() == plan.n_shards * plan.shard_bytes
+    base = flat.data_ptr()
+    shards = [base + s * plan.shard_bytes for s in range(plan.n_shards)]
+    if separate_buckets:
+        # Separately allocated buckets (pointer-table launch shape).
+        # Shuffled so that the pointers are not equally spaced.
+        bl = [torch.empty(plan.bucket_bytes, dtype=torch.uint8, device=dev)
+              for _ in range(plan.n_buckets)]
+        if poison is not None:
+            for b in bl:
+                b.fill_(poison)
+        order = np.random.default_rng(plan.n_buckets).permutation(len(bl))
+        bl = [bl[i] for i in order]
+        buckets = bl
+        bucket_store = bl
+    else:
+        bucket_store = torch.empty((plan.n_buckets, plan.bucket_bytes), dtype=torch.uint8,
+                                   device=dev)
+        if poison is not None:
+            bucket_store.fill_(poison)
+        buckets = bucket_store
+    checksums = torch.zeros(max(1, plan.n_buckets), dtype=torch.int64, device=dev)
+    dst = [torch.empty(max(1, n), dtype=torch.int16, device=dev)
+           for n in plan.tensor_numel] if with_dst else []
+    if poison is not None:
+        for d in dst:
+            d.fill_(0x5A5A)
+    return SyncBuffers(plan, flat, shards, bucket_store, buckets, checksums, dst)
+
+
+def fill_from_host(buf: SyncBuffers, host_shards) -> None:
+    host = np.concatenate([np.asarray(s, np.uint8) for s in host_shards])
+    assert host.size == buf.flat.numel()
+    buf.flat.copy_(torch.from_numpy(host))
+
+
+def fill_with_generator(buf: SyncBuffers, manifest, seed: int, specials: bool,
+                        stream: int = 0) -> None:
+    """Device generator, one launch per parameter at the library's flat offsets."""
+    base = buf.flat.data_ptr()
+    for p, off in zip(manifest, buf.plan.param_flat_offset):
+        es = 4 if p.dtype == "f32" else 2
+        n = int(np.prod(p.shape)) if len(p.shape) else 1
+        synth.fill_dev(base + off, n, es, seed, first_idx=off // es, specials=specials,
+                       stream=stream)
+
+
+def bucket_list(buf: SyncBuffers):
+    if isinstance(buf.buckets, torch.Tensor):
+        return [buf.buckets[i] for i in range(buf.buckets.shape[0])]
+    return list(buf.buckets)
+
+
+def pack(buf: SyncBuffers, stream=None):
+    rr.rr_pack(buf.plan, buf.shards, buf.buckets, buf.checksums, stream)
+
+
+def unpack(buf: SyncBuffers, stream=None):
+    rr.rr_unpack(buf.plan, buf.buckets, buf.dst, stream)
+
+
+def verify(buf: SyncBuffers, stream=None):
+    return rr.rr_verify(buf.plan, buf.buckets, buf.checksums, stream)
+
+
+def buckets_host(buf: SyncBuffers, idx=None) -> np.ndarray:
+    bl = bucket_list(buf)
+    idx = range(len(bl)) if idx is None else idx
+    return np.stack([bl[i].cpu().numpy() for i in idx]) if len(idx) else \
+        np.zeros((0, buf.plan.bucket_bytes), np.uint8)
+
+
+def checksums_host(buf: SyncBuffers) -> np.ndarray:
+    return buf.checksums.cpu().numpy().view(np.uint64)[:buf.plan.n_buckets]
+
+
+def tensor_host(buf: SyncBuffers, t: int) -> np.ndarray:
+    return buf.dst[t][:buf.plan.tensor_numel[t]].cpu().numpy().view(np.uint16)
+
+
+def device_word_sums(buf: SyncBuffers) -> np.ndarray:
+    """Per-bucket 64-bit word sums computed with torch (wrapping int64 adds)."""
+    out = []
+    for b in bucket_list(buf):
+        out.append(int(b.view(torch.int64).sum().item()) & ((1 << 64) - 1))
+    return np.array(out, dtype=np.uint64)

@@ -1,0 +1,186 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle, bit for bit.
+
+Buckets, checksums and unpacked tensors are integer / bit-pattern data, so the
+bar is exact equality (RobustRL Section 5.2.1 steps 1-2; Section 5.2.2 for
+the checksums).  Small workloads are compared in full; the full-size
+workloads (Qwen3-8B, its TP=4 bucket sweep, Qwen3-30B-A3B) on sampled
+buckets and tensors that the oracle computes one by one, plus properties that
+hold at any size (every checksum equals a word sum taken by torch; verify
+finds nothing; unpack(pack) equals the sampled tensors).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from tests import _util as U
+from tests import gpu_harness as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.init()
+    yield
+    torch.cuda.synchronize()
+
+
+def full_parity(desc, separate_buckets=False, **opts):
+    L = U.to_oracle(desc)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"], **opts)
+    buf = H.alloc(plan, separate_buckets=separate_buckets)
+    shards = L.host_shards(desc["seed"], desc["specials"])
+    H.fill_from_host(buf, shards)
+    H.pack(buf)
+    H.unpack(buf)
+    n_bad, first = H.verify(buf)
+    torch.cuda.synchronize()
+    want, want_cs = L.pack(oracle.Source(shards=shards))
+    got = H.buckets_host(buf)
+    np.testing.assert_array_equal(got, want)
+    np.testing.assert_array_equal(H.checksums_host(buf), want_cs)
+    for t in range(len(L.tensors)):
+        np.testing.assert_array_equal(H.tensor_host(buf, t), L.reshard_tensor(
+            oracle.Source(shards=shards), t), err_msg=f"tensor {t}")
+    assert (n_bad, first) == (0, -1)
+    return buf, L, shards
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2",
+                                  "tiny-moe-f32"])
+def test_small_workloads(name):
+    full_parity(U.workload_desc(name))
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-tp4"])
+def test_separately_allocated_buckets(name):
+    full_parity(U.workload_desc(name), separate_buckets=True)
+
+
+@pytest.mark.parametrize("chunk", [16, 1040, 4096])
+def test_small_chunks_and_buckets(chunk):
+    full_parity(U.workload_desc("tiny-tp4", bucket_bytes=8 * 1024), chunk_bytes=chunk)
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_random_layouts(seed):
+    full_parity(U.random_layout(seed), separate_buckets=bool(seed % 2))
+
+
+@pytest.mark.parametrize("grid", [1, 3, 1000])
+def test_grid_sizes(grid):
+    full_parity(U.workload_desc("tiny-moe-tp2"), grid_blocks=grid)
+
+
+def test_qwen3_0_6b_full():
+    """Qwen3-0.6B, 8 fp32 shards -> TP=1, 32 MiB buckets: every byte compared."""
+    full_parity(U.workload_desc("qwen3-0.6b"))
+
+
+def test_device_generator_matches_host():
+    n = 5_000_001
+    for es, specials in ((4, True), (4, False), (2, False)):
+        t = torch.empty(n * es, dtype=torch.uint8, device="cuda")
+        synth.fill_dev(t.data_ptr(), n, es, seed=77, first_idx=123456789, specials=specials)
+        torch.cuda.synchronize()
+        got = t.cpu().numpy().view(np.uint32 if es == 4 else np.uint16)
+        np.testing.assert_array_equal(got, synth.values_host(n, es, 77, 123456789, specials))
+
+
+# ---------------------------------------------------------------------------
+# Full-size workloads, sampled
+# ---------------------------------------------------------------------------
+
+def sampled_parity(name, bucket_sizes=None, tensors=("norm",), n_random_buckets=3):
+    w = U.workload(name)
+    desc = U.workload_desc(name)
+    m, s, d = U.to_product(desc)
+    gen = oracle.Source(seed=w.seed, specials=w.specials)
+    flat = None
+    for bb in bucket_sizes or [w.bucket_bytes]:
+        plan = H.make_plan(m, s, d, bb)
+        buf = H.alloc(plan, poison=None, with_dst=False, flat=flat)
+        if flat is None:
+            H.fill_with_generator(buf, m, w.seed, w.specials)
+            flat = buf.flat
+        L = oracle.workload_layout(w, bucket_bytes=bb)
+        assert L.n_buckets == plan.n_buckets
+        H.pack(buf)
+        n_bad, first = H.verify(buf)
+        assert (n_bad, first) == (0, -1)
+        torch.cuda.synchronize()
+        # Property at any size: every checksum equals torch's word sum of its bucket.
+        np.testing.assert_array_equal(H.checksums_host(buf), H.device_word_sums(buf))
+        rng = np.random.default_rng(bb)
+        fr = plan.first_bucket_of_rank
+        pick = sorted({0, plan.n_buckets - 1, *[fr[r] for r in range(plan.tp)],
+                       *[fr[r + 1] - 1 for r in range(plan.tp)],
+                       *rng.integers(0, plan.n_buckets, n_random_buckets).tolist()})
+        cs = H.checksums_host(buf)
+        for b in pick:
+            want, want_cs = L.pack(gen, first=b, count=1)
+            np.testing.assert_array_equal(H.buckets_host(buf, [b])[0], want[0],
+                                          err_msg=f"bucket {b} (bucket_bytes {bb})")
+            assert cs[b] == want_cs[0]
+        buf = None
+
+
+def _unpack_sampled(name, names):
+    w = U.workload(name)
+    desc = U.workload_desc(name)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, w.bucket_bytes)
+    buf = H.alloc(plan, poison=None)
+    H.fill_with_generator(buf, m, w.seed, w.specials)
+    H.pack(buf)
+    H.unpack(buf)
+    assert H.verify(buf) == (0, -1)
+    torch.cuda.synchronize()
+    L = oracle.workload_layout(w)
+    gen = oracle.Source(seed=w.seed, specials=w.specials)
+    for nm, rank in names:
+        t = L.tensor_index(nm, rank)
+        assert plan.tensor_names[t] == nm and plan.tensor_ranks[t] == rank
+        np.testing.assert_array_equal(H.tensor_host(buf, t), L.reshard_tensor(gen, t),
+                                      err_msg=f"{nm} rank {rank}")
+    # Every other tensor, against its own bytes read straight out of the
+    # buckets by torch (unpack must be the exact inverse of the stream cut).
+    B = plan.bucket_bytes
+    store = buf.bucket_store.view(-1)
+    for t in range(plan.n_tensors):
+        r = plan.tensor_ranks[t]
+        start = plan.first_bucket_of_rank[r] * B + plan.tensor_stream_offset[t]
+        n = 2 * plan.tensor_numel[t]
+        want = store[start:start + n].view(torch.int16)
+        assert torch.equal(buf.dst[t][:plan.tensor_numel[t]], want), plan.tensor_names[t]
+
+
+def test_qwen3_8b_sampled():
+    sampled_parity("qwen3-8b", n_random_buckets=4)
+    torch.cuda.empty_cache()
+    _unpack_sampled("qwen3-8b", [("layers.0.qkv_proj", 0), ("layers.17.o_proj", 0),
+                                 ("layers.35.down_proj", 0), ("layers.35.post_attention_layernorm",
+                                                              0), ("norm", 0)])
+    torch.cuda.empty_cache()
+
+
+def test_qwen3_8b_tp4_bucket_sweep_sampled():
+    sampled_parity("qwen3-8b-tp4", bucket_sizes=synth.TP4_BUCKET_SWEEP, n_random_buckets=1)
+    torch.cuda.empty_cache()
+    _unpack_sampled("qwen3-8b-tp4", [("layers.3.qkv_proj", 1), ("layers.20.o_proj", 2),
+                                     ("layers.35.down_proj", 3), ("layers.7.gate_up_proj", 0),
+                                     ("norm", 3)])
+    torch.cuda.empty_cache()
+
+
+def test_qwen3_30b_a3b_sampled():
+    sampled_parity("qwen3-30b-a3b", n_random_buckets=2)
+    torch.cuda.empty_cache()
+    _unpack_sampled("qwen3-30b-a3b", [("layers.0.router", 0), ("layers.47.experts.w2", 0),
+                                      ("layers.5.qkv_proj", 0), ("norm", 0)])
+    torch.cuda.empty_cache()

@@ -1,0 +1,152 @@
+"""Host-side checks of the library's planner (no GPU): the C ABI loads and
+exports what include/rr.h declares; host-only plans agree with the oracle on
+geometry; their work tables, interpreted item by item, reproduce the oracle's
+buckets and tensors; bad descriptions are rejected with the right status."""
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+import paper_2512_22492_gb300 as rr
+from paper_2512_22492_gb300 import rr as rrmod
+from tests import _util as U
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "rr.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(rr_[a-z_]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol():
+    import ctypes
+    lib = ctypes.CDLL(rrmod.LIBRARY_PATH)
+    names = declared_functions()
+    assert "rr_pack" in names and "rr_plan_create" in names
+    for name in names:
+        assert hasattr(lib, name), f"{name} declared in rr.h but not exported"
+
+
+def host_plan(desc, **opt):
+    m, s, d = U.to_product(desc)
+    return rr.rr_plan_create(m, s, d, desc["bucket_bytes"], rr.PlanOptions(host_only=True, **opt))
+
+
+@pytest.mark.parametrize("name", ["tiny", "qwen3-0.6b", "qwen3-8b", "qwen3-8b-tp4",
+                                  "qwen3-30b-a3b", "tiny-moe-tp2"])
+def test_geometry_matches_oracle(name):
+    desc = U.workload_desc(name)
+    L = U.to_oracle(desc)
+    p = host_plan(desc)
+    assert p.n_buckets == L.n_buckets
+    assert p.shard_bytes == L.shard_bytes and p.flat_bytes == L.flat_bytes
+    assert p.param_flat_offset == list(L.param_offset)
+    assert p.first_bucket_of_rank == list(L.rank_first_bucket)
+    assert p.stream_bytes_per_rank == list(L.rank_stream_bytes)
+    assert p.tensor_numel == list(L.tensor_numel)
+    assert p.tensor_stream_offset == list(L.tensor_offset)
+
+
+def run_and_compare(desc, **opt):
+    L = U.to_oracle(desc)
+    p = host_plan(desc, **opt)
+    shards = L.host_shards(desc["seed"], desc["specials"])
+    want, want_cs = L.pack(oracle.Source(shards=shards))
+    items, first = p.export_pack()
+    U.check_partition(first, len(items))
+    got = U.check_and_run_pack(items, shards, p.n_buckets, p.bucket_bytes, p.shard_bytes)
+    np.testing.assert_array_equal(got, want)
+    uitems, ufirst = p.export_unpack()
+    U.check_partition(ufirst, len(uitems))
+    tensors = U.check_and_run_unpack(uitems, want, p.tensor_numel)
+    for t, arr in enumerate(tensors):
+        np.testing.assert_array_equal(arr, L.unpack_tensor(want, t))
+    return p, items
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2",
+                                  "tiny-moe-f32"])
+def test_tables_reproduce_oracle_workloads(name):
+    run_and_compare(U.workload_desc(name))
+
+
+@pytest.mark.parametrize("chunk", [16, 48, 4096])
+def test_tables_small_chunks(chunk):
+    run_and_compare(U.workload_desc("tiny-tp4", bucket_bytes=8 * 1024), chunk_bytes=chunk)
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_tables_random_layouts(seed):
+    run_and_compare(U.random_layout(seed), grid_blocks=7)
+
+
+def test_vector_items_dominate_on_aligned_workloads():
+    p, items = run_and_compare(U.workload_desc("tiny"))
+    data = items[items["kind"] <= U.ITEM_BF16_SCALAR]
+    elems = data["row_len"].astype(np.int64) * data["n_rows"]
+    vec = elems[data["kind"] == U.ITEM_F32_VEC].sum()
+    assert vec == elems.sum(), "an aligned fp32 workload should need no scalar items"
+
+
+def test_full_size_tables_are_consistent():
+    """Qwen3-8B TP=4: metadata-only checks over ~0.5M items."""
+    desc = U.workload_desc("qwen3-8b-tp4")
+    p = host_plan(desc)
+    items, first = p.export_pack()
+    U.check_partition(first, len(items))
+    n = items["row_len"].astype(np.int64) * items["n_rows"]
+    bucket_bytes = np.zeros(p.n_buckets, np.int64)
+    np.add.at(bucket_bytes, items["bucket"].astype(np.int64), 2 * n)
+    assert np.all(bucket_bytes == p.bucket_bytes)
+    assert np.all(items["dst_off"].astype(np.int64) + 2 * n <= p.bucket_bytes)
+    assert np.all(2 * n <= 32 * 1024)
+    st = p.stats()
+    data = items["kind"] <= U.ITEM_BF16_SCALAR
+    assert (n[data] * 4).sum() == st["pack_bytes_read"]
+    assert np.all(items["kind"][data] == U.ITEM_F32_VEC)
+
+
+def test_rejections():
+    params = [rr.Param("a", (4, 6), "f32"), rr.Param("b", (5,), "bf16")]
+    src = rr.SrcLayout(n_shards=2)
+    good = rr.DstLayout(tp=1, tensors=[rr.DstTensor("t", 0, [rr.Block(0, 0, 4, 0, 6)])])
+    opts = rr.PlanOptions(host_only=True)
+    rr.rr_plan_create(params, src, good, 64, opts)
+
+    def status(params=params, src=src, dst=good, bucket=64):
+        with pytest.raises(rr.RRError) as e:
+            rr.rr_plan_create(params, src, dst, bucket, opts)
+        return e.value.status
+
+    bad_rows = rr.DstLayout(tp=1, tensors=[rr.DstTensor("t", 0, [rr.Block(0, 2, 3, 0, 6)])])
+    bad_cols = rr.DstLayout(tp=1, tensors=[rr.DstTensor("t", 0, [rr.Block(0, 0, 1, 5, 2)])])
+    bad_param = rr.DstLayout(tp=1, tensors=[rr.DstTensor("t", 0, [rr.Block(2, 0, 1, 0, 1)])])
+    bad_rank = rr.DstLayout(tp=1, tensors=[rr.DstTensor("t", 1, [rr.Block(0, 0, 1, 0, 6)])])
+    bad_numel = rr.DstLayout(tp=1, tensors=[rr.DstTensor("t", 0, [rr.Block(0, 0, 1, 0, 6)],
+                                                         numel=7)])
+    assert status(dst=bad_rows) == rrmod.RR_ELAYOUT
+    assert status(dst=bad_cols) == rrmod.RR_ELAYOUT
+    assert status(dst=bad_param) == rrmod.RR_ELAYOUT
+    assert status(dst=bad_rank) == rrmod.RR_ELAYOUT
+    assert status(dst=bad_numel) == rrmod.RR_ELAYOUT
+    assert status(bucket=12) == rrmod.RR_EINVAL
+    assert status(bucket=0) == rrmod.RR_EINVAL
+    assert status(src=rr.SrcLayout(n_shards=0)) == rrmod.RR_EINVAL
+    overlap = rr.SrcLayout(n_shards=1, param_flat_offset=[0, 64])
+    assert status(src=overlap) == rrmod.RR_ELAYOUT
+    misaligned = rr.SrcLayout(n_shards=1, param_flat_offset=[2, 200])
+    assert status(src=misaligned) == rrmod.RR_ELAYOUT
+    assert status(dst=rr.DstLayout(tp=1, tensors=good.tensors, tensor_align_bytes=3)) \
+        == rrmod.RR_EINVAL
+
+
+def test_host_only_plan_refuses_to_run():
+    desc = U.workload_desc("tiny")
+    p = host_plan(desc)
+    with pytest.raises(rr.RRError) as e:
+        rr.rr_pack(p, [16] * p.n_shards, [16] * p.n_buckets, 16, stream=0)
+    assert e.value.status == rrmod.RR_EINVAL
