@@ -24,7 +24,7 @@ from . import build as _build
 
 if not os.path.exists(_build.LIB):
     raise ImportError(
-        f"{_build.LIB} is missing: build it with `python -m paper_2512_22492_gb300.build` "
+        f"{_build.LIB} is missing: build it with `python paper_2512_22492_gb300/build.py` "
         "(needs nvcc); there is no CPU fallback")
 _lib = ctypes.CDLL(_build.LIB)
 

@@ -21,7 +21,7 @@ class SyncBuffers:
     plan: "rr.Plan"
     flat: torch.Tensor                 # n_shards * shard_bytes, uint8
     shards: List[int]                  # device pointers into flat
-    bucket_store: torch.Tensor         # [n_buckets, bucket_bytes] uint8 (uniform layout)
+    bucket_store: torch.Tensor         # [n_buckets, row >= bucket_bytes] uint8 (uniform layout)
     buckets: list                      # what is passed as the bucket array
     checksums: torch.Tensor            # [n_buckets] int64 (uint64 bits)
     dst: List[torch.Tensor]            # one int16 tensor per destination tensor
@@ -53,11 +53,12 @@ def alloc(plan, separate_buckets: bool = False, poison: Optional[int] = 0xAB,
         buckets = bl
         bucket_store = bl
     else:
-        bucket_store = torch.empty((plan.n_buckets, plan.bucket_bytes), dtype=torch.uint8,
-                                   device=dev)
+        # One allocation; rows padded to 16 bytes so every bucket is 16-byte aligned.
+        row = (plan.bucket_bytes + 15) // 16 * 16
+        bucket_store = torch.empty((plan.n_buckets, row), dtype=torch.uint8, device=dev)
         if poison is not None:
             bucket_store.fill_(poison)
-        buckets = bucket_store
+        buckets = bucket_store[:, :plan.bucket_bytes]
     checksums = torch.zeros(max(1, plan.n_buckets), dtype=torch.int64, device=dev)
     dst = [torch.empty(max(1, n), dtype=torch.int16, device=dev)
            for n in plan.tensor_numel] if with_dst else []

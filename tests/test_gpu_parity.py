@@ -13,7 +13,9 @@ import pytest
 import torch
 
 import oracle
+import paper_2512_22492_gb300 as rr
 import synth
+from paper_2512_22492_gb300 import rr as rrmod
 from tests import _util as U
 from tests import gpu_harness as H
 
@@ -33,6 +35,14 @@ def full_parity(desc, separate_buckets=False, **opts):
     L = U.to_oracle(desc)
     m, s, d = U.to_product(desc)
     plan = H.make_plan(m, s, d, desc["bucket_bytes"], **opts)
+    if separate_buckets and plan.n_shards + plan.n_buckets > 3968:
+        # Beyond the pointer table of one launch: the library must refuse
+        # separately allocated buckets and accept one equally spaced block.
+        buf = H.alloc(plan, separate_buckets=True, with_dst=False)
+        with pytest.raises(rr.RRError) as e:
+            H.pack(buf)
+        assert e.value.status == rrmod.RR_EINVAL
+        separate_buckets = False
     buf = H.alloc(plan, separate_buckets=separate_buckets)
     shards = L.host_shards(desc["seed"], desc["specials"])
     H.fill_from_host(buf, shards)
@@ -151,6 +161,7 @@ def _unpack_sampled(name, names):
     # Every other tensor, against its own bytes read straight out of the
     # buckets by torch (unpack must be the exact inverse of the stream cut).
     B = plan.bucket_bytes
+    assert buf.bucket_store.shape[1] == B
     store = buf.bucket_store.view(-1)
     for t in range(plan.n_tensors):
         r = plan.tensor_ranks[t]
