@@ -1,9 +1,9 @@
 /*
  * rr.h - C ABI of the trainer -> rollout weight-synchronisation hot path.
  *
- * RobustRL (arXiv 2512.22492), Section 5.2.1 "UCX-based Weight Update":
+ * RobustRL (arXiv 2512.22492), Section 5.2.1 (the UCX-based weight update):
  * after a training step the trainer's weights are (1) resharded to the
- * rollout's sharding and (2) placed layer by layer into a transfer buffer
+ * rollout's sharding and (2) copied, one layer after another, into a transfer buffer
  * that the transport moves to the rollout; Section 5.2.2 has a recovered or
  * resumed rollout pull (part of) that buffer again.  This library is the
  * on-GPU part of that route, for one GPU: gather from flat FSDP-style shards,
@@ -130,8 +130,8 @@ typedef struct {
 } rr_plan_options;
 
 /* Compiles manifest + source layout + destination layout + bucket size into
- * device-resident segment tables (Section 5.2.1 step 1: "reshard ... to align
- * with the sharding of the rollout").  bucket_bytes: a multiple of 8, at most
+ * device-resident segment tables (Section 5.2.1 step 1: the weights are
+ * re-laid out in the rollout's sharding).  bucket_bytes: a multiple of 8, at most
  * 2^32 - 16.  Uses the current CUDA device.  *out is valid only on RR_OK. */
 rr_status rr_plan_create(const rr_param* manifest, int32_t n_params, const rr_src_layout* src,
                          const rr_dst_layout* dst, size_t bucket_bytes, rr_plan** out);
@@ -222,8 +222,8 @@ rr_status rr_plan_export_unpack(const rr_plan* plan, rr_unpack_item* items, int6
                                 uint32_t* block_first);
 
 /* Reshard + cast + pack + checksum, fused in one persistent kernel launch
- * (Section 5.2.1 steps 1-2: the model is placed "layer by layer into a
- * buffer for transmission"; the checksums serve Section 5.2.2's reconnect).
+ * (Section 5.2.1 steps 1-2: the resharded model fills a transfer buffer; the
+ * checksums serve the reconnect cases of Section 5.2.2).
  *   src_shards: host array of n_shards device pointers, S bytes each.
  *   buckets:    host array of n_buckets device pointers, bucket_bytes each;
  *               equally spaced pointers (one allocation cut into buckets)
@@ -234,8 +234,8 @@ rr_status rr_plan_export_unpack(const rr_plan* plan, rr_unpack_item* items, int6
 rr_status rr_pack(const rr_plan* plan, const void* const* src_shards, void* const* buckets,
                   uint64_t* checksums, cudaStream_t stream);
 
-/* Buckets -> rollout tensors (Section 5.2.1: the receiving rollout
- * "finishes the weight update").
+/* Buckets -> rollout tensors (Section 5.2.1: the receiving rollout completes
+ * its weight update from what it pulled).
  *   buckets: host array of n_buckets device pointers;
  *   dst:     host array of n_tensors device pointers, numel * 2 bytes each.
  * Stream-ordered and asynchronous (one kernel launch). */

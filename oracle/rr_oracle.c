@@ -6,13 +6,14 @@
  * code with the CUDA library and is written to be read against its definition,
  * not to be fast: single thread, scalar, one element at a time.
  *
- * What it computes (RobustRL, Section 5.2.1, "UCX-based Weight Update"):
+ * What it computes (RobustRL, Section 5.2.1, the UCX-based weight update):
  *   (1) reshard: the trainer's parameters, held as flat FSDP-style shards, are
  *       re-laid into the rollout engine's layout (step 1 of that section);
- *   (2) the rollout holds 16-bit weights (Section 7.4 speaks of the model "in
- *       FP16 precision"); here the cast is float32 -> bfloat16,
- *       round-to-nearest-even;
- *   (3) the model is placed layer by layer into a transfer buffer (step 2);
+ *   (2) the rollout holds 16-bit weights (Section 7.4 sizes the transferred
+ *       model at two bytes per parameter); here the cast is float32 ->
+ *       bfloat16, round-to-nearest-even;
+ *   (3) the model is copied, one layer after another, into a transfer buffer
+ *       (step 2);
  *       here that buffer is a sequence of fixed-size buckets;
  *   (4) each bucket carries a 64-bit word-sum so that a rollout that
  *       reconnects after a failure (Section 5.2.2, "Relay server failure

@@ -1,7 +1,7 @@
 """GB300-native trainer -> rollout weight synchronisation hot path.
 
 RobustRL (arXiv 2512.22492) Section 5.2.1: reshard the trainer's weights to
-the rollout's sharding and place them layer by layer into a transfer buffer;
+the rollout's sharding and copy them, one layer after another, into a transfer buffer;
 Section 5.2.2: a rollout that reconnects after a failure pulls (part of) that
 buffer again.  This package is the on-GPU part of that route for one GB300:
 a C-ABI CUDA library (``include/rr.h``, ``csrc/``) and its Python binding.

@@ -592,3 +592,4 @@ extern "C" rr_status rr_verify(const rr_plan* P, const void* const* buckets,
     if (first_bad) *first_bad = bad ? (int64_t)(ULLONG_MAX - P->h_verify_result[2]) : -1;
     return bad ? RR_EMISMATCH : RR_OK;
 }
+

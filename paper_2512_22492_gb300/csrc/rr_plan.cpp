@@ -2,10 +2,10 @@
 // (rollout) layout and a bucket size into the work tables that the pack and
 // unpack kernels walk.
 //
-// RobustRL Section 5.2.1, step 1 ("reshard the model to align with the
-// sharding of the rollout") and step 2 ("placing the model layer by layer
-// into a buffer for transmission"): the plan is the reshard expressed as a
-// table of strided gathers, each landing in one fixed-size bucket.
+// RobustRL Section 5.2.1, step 1 (re-lay the trainer's weights out in the
+// rollout's sharding) and step 2 (fill a transfer buffer with the model, one
+// layer after another): the plan is that reshard expressed as a table of
+// strided gathers, each landing in one fixed-size bucket.
 //
 // A work item never crosses a source shard, a bucket, or `chunk_bytes` of
 // destination; items are emitted rank by rank in stream order, so the table

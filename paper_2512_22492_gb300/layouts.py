@@ -4,8 +4,8 @@ The C library knows nothing about models; a weight sync is described to it
 as a parameter manifest plus, per rollout tensor, a list of 2-D blocks of
 those parameters.  This module writes those descriptions for Qwen3 dense and
 MoE decoders, as the paper's system uses them (RobustRL Section 7.1: FSDP
-trainer, vLLM rollout with tensor parallelism; Section 5.2.1 step 1: reshard
-"to align with the sharding of the rollout").
+trainer, vLLM rollout with tensor parallelism; Section 5.2.1 step 1: the
+weights are re-laid out in the rollout's sharding).
 
 Trainer manifest: module-registration order of the Hugging Face Qwen3 model.
 Rollout tensors, per rank r of TP = t, in this order:

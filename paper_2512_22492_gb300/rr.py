@@ -377,20 +377,60 @@ def _stream(stream) -> int:
 # Hot path
 # ---------------------------------------------------------------------------
 
+def _nbytes(x):
+    """Byte size of a tensor argument, or None for a raw pointer (unchecked)."""
+    if isinstance(x, int):
+        return None
+    return int(x.numel()) * int(x.element_size())
+
+
+def _check_list(xs, n: int, min_bytes, what: str) -> None:
+    """Host arrays handed to the ABI hold exactly n pointers; tensor arguments
+    must be large enough for what the plan will write or read."""
+    if hasattr(xs, "dim") and xs.dim() == 2:
+        if xs.shape[0] != n:
+            raise ValueError(f"{what}: {xs.shape[0]} rows, plan expects {n}")
+        if min_bytes is not None and xs.shape[1] * xs.element_size() < min_bytes:
+            raise ValueError(f"{what}: rows of {xs.shape[1] * xs.element_size()} bytes, plan "
+                             f"needs {min_bytes}")
+        return
+    xs = list(xs)
+    if len(xs) != n:
+        raise ValueError(f"{what}: {len(xs)} entries, plan expects {n}")
+    for i, x in enumerate(xs):
+        need = min_bytes(i) if callable(min_bytes) else min_bytes
+        nb = _nbytes(x)
+        if nb is not None and need is not None and nb < need:
+            raise ValueError(f"{what}[{i}]: {nb} bytes, plan needs {need}")
+
+
+def _check_checksums(plan: Plan, checksums) -> None:
+    nb = _nbytes(checksums)
+    if nb is not None and nb < 8 * plan.n_buckets:
+        raise ValueError(f"checksums: {nb} bytes, plan needs {8 * plan.n_buckets}")
+
+
 def rr_pack(plan: Plan, src_shards, buckets, checksums, stream=None) -> None:
     """Reshard + cast + pack + checksum (asynchronous on `stream`)."""
+    _check_list(src_shards, plan.n_shards, plan.shard_bytes, "src_shards")
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_checksums(plan, checksums)
     _check(_lib.rr_pack(plan.handle, _ptr_array(src_shards), _ptr_array(buckets),
                         _ptr(checksums), _stream(stream)), "rr_pack")
 
 
 def rr_unpack(plan: Plan, buckets, dst, stream=None) -> None:
     """Buckets -> destination tensors (asynchronous on `stream`)."""
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst")
     _check(_lib.rr_unpack(plan.handle, _ptr_array(buckets), _ptr_array(dst), _stream(stream)),
            "rr_unpack")
 
 
 def rr_verify(plan: Plan, buckets, checksums, stream=None):
     """Recompute and compare checksums; returns (n_bad, first_bad).  Synchronous."""
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_checksums(plan, checksums)
     n_bad = ctypes.c_int64()
     first = ctypes.c_int64()
     st = _lib.rr_verify(plan.handle, _ptr_array(buckets), _ptr(checksums), ctypes.byref(n_bad),
@@ -398,3 +438,4 @@ def rr_verify(plan: Plan, buckets, checksums, stream=None):
     if st not in (RR_OK, RR_EMISMATCH):
         _check(st, "rr_verify")
     return n_bad.value, first.value
+
