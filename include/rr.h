@@ -250,6 +250,27 @@ rr_status rr_unpack(const rr_plan* plan, const void* const* buckets, void* const
 rr_status rr_verify(const rr_plan* plan, const void* const* buckets, const uint64_t* checksums,
                     int64_t* n_bad, int64_t* first_bad, cudaStream_t stream);
 
+/* Allocation-free form of rr_verify.  The paper has no counterpart: this
+ * entry point exists for callers that cannot allocate device memory when they
+ * check a pull, such as an inference engine that has reserved nearly all
+ * device memory for its weights and cache, or code running under a memory
+ * pool that refuses new cudaMalloc calls.  It takes no plan, because creating
+ * one allocates; the caller passes the buckets (host array of n_buckets device
+ * pointers, bucket_bytes each), the expected checksums (device) and host
+ * outputs as for rr_verify, and the result and blocking behaviour are those
+ * of rr_verify.
+ *   Scratch: one file-scope device array of 16384 + 4 64-bit words (128 KiB),
+ *   which every GPU that loads this library keeps until the process exits.
+ *   n_buckets above 16384 is rejected with RR_EINVAL.  The first call on a
+ *   device looks up the array's device address and sizes the grid for that
+ *   device; make that first call before any stream capture.  Each call clears
+ *   the part of the array it uses before its kernel runs; calls that overlap
+ *   on the GPU (on different streams, or from different threads) share the
+ *   array and race, so serialise them.  Calls no cudaMalloc or cudaFree. */
+rr_status rr_verify_noalloc(const void* const* buckets, int32_t n_buckets, size_t bucket_bytes,
+                            const uint64_t* checksums, int64_t* n_bad, int64_t* first_bad,
+                            cudaStream_t stream);
+
 const char* rr_status_str(rr_status status);
 const char* rr_last_error(void);
 

@@ -14,8 +14,10 @@
 // registers and flushed with one 64-bit atomic per warp per bucket change.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <climits>
 #include <cstring>
+#include <mutex>
 
 #include "rr_internal.h"
 
@@ -593,3 +595,128 @@ extern "C" rr_status rr_verify(const rr_plan* P, const void* const* buckets,
     return bad ? RR_EMISMATCH : RR_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Allocation-free verify
+//
+// For callers that must not allocate device memory at the moment they check a
+// pull: an inference engine that reserves nearly all device memory up front,
+// or a process that runs under a memory pool that refuses cudaMalloc once the
+// weights are loaded.  It needs no plan (a plan's creation allocates): the
+// caller passes the buckets, their size and the expected checksums.  The
+// per-bucket sums and counters live in one file-scope device array, which
+// every GPU that loads this library holds until the process exits.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+constexpr int32_t kStaticVerifyMaxBuckets = 16384;   // 128 KiB of sums + 4 counters
+constexpr int kStaticMaxDevices = 64;
+
+__device__ __align__(256) unsigned long long g_static_verify_scratch[kStaticVerifyMaxBuckets + 4];
+
+struct StaticVerifyDevice {
+    bool ready = false;
+    unsigned long long* scratch = nullptr;   // device address of g_static_verify_scratch
+    int32_t grid = 0;
+};
+
+std::mutex g_static_mutex;
+StaticVerifyDevice g_static_dev[kStaticMaxDevices];
+
+// Once per device, with that device current: resolve the array's device
+// address (host code may not use the symbol itself as a pointer) and size the
+// grid.  Neither step allocates.
+rr_status static_verify_setup(StaticVerifyDevice** out) {
+    int dev = -1;
+    RR_CUDA(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= kStaticMaxDevices)
+        return rr_fail(RR_EINVAL, "device %d beyond the %d devices this entry point serves", dev,
+                       kStaticMaxDevices);
+    std::lock_guard<std::mutex> lock(g_static_mutex);
+    StaticVerifyDevice& d = g_static_dev[dev];
+    if (!d.ready) {
+        void* p = nullptr;
+        RR_CUDA(cudaGetSymbolAddress(&p, g_static_verify_scratch));
+        int sms = 0, per_sm = 0;
+        RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+        RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+            &per_sm, rr_verify_kernel<kLargePtrs>, kThreads, 0));
+        d.scratch = (unsigned long long*)p;
+        d.grid = sms * (per_sm > 0 ? per_sm : 1);
+        d.ready = true;
+    }
+    *out = &d;
+    return RR_OK;
+}
+
+template <int NPTR>
+rr_status launch_static_verify(unsigned long long* scratch, int32_t grid, int32_t n_buckets,
+                               uint64_t bucket_bytes, const void* const* buckets,
+                               const uint64_t* checksums, bool table, uint64_t stride,
+                               cudaStream_t s) {
+    VerifyArgs<NPTR> a;
+    std::memset(&a, 0, sizeof a);
+    a.sums = scratch;
+    a.counters = scratch + n_buckets;
+    a.expected = (const unsigned long long*)checksums;
+    a.bucket_bytes = bucket_bytes;
+    a.chunk_bytes = std::min<uint64_t>((uint64_t)kVerifyChunk, bucket_bytes);
+    a.chunks_per_bucket = (a.bucket_bytes + a.chunk_bytes - 1) / a.chunk_bytes;
+    a.total_chunks = a.chunks_per_bucket * (uint64_t)n_buckets;
+    a.n_buckets = n_buckets;
+    if (table) {
+        for (int32_t b = 0; b < n_buckets; ++b) a.ptr[b] = buckets[b];
+    } else {
+        a.bucket_base = (const char*)buckets[0];
+        a.bucket_stride = stride;
+    }
+    rr_verify_kernel<NPTR><<<grid, kThreads, 0, s>>>(a);
+    RR_CUDA(cudaGetLastError());
+    return RR_OK;
+}
+
+}  // namespace
+
+extern "C" rr_status rr_verify_noalloc(const void* const* buckets, int32_t n_buckets,
+                                       size_t bucket_bytes, const uint64_t* checksums,
+                                       int64_t* n_bad, int64_t* first_bad, cudaStream_t stream) {
+    rr_clear_error();
+    if (n_buckets < 0 || n_buckets > kStaticVerifyMaxBuckets)
+        return rr_fail(RR_EINVAL,
+                       "rr_verify_noalloc checks at most %d buckets per call (got %d); use "
+                       "larger buckets, several calls, or rr_verify",
+                       kStaticVerifyMaxBuckets, n_buckets);
+    if (bucket_bytes < 8 || bucket_bytes % 8 != 0 || bucket_bytes > (size_t(1) << 32) - 16)
+        return rr_fail(RR_EINVAL, "bucket_bytes must be a multiple of 8 in [8, 2^32 - 16]");
+    rr_status st = check_ptrs(buckets, n_buckets, "buckets");
+    if (st) return st;
+    if (n_buckets > 0 && !aligned16(checksums))
+        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    if (n_bad) *n_bad = 0;
+    if (first_bad) *first_bad = -1;
+    if (n_buckets == 0) return RR_OK;
+    uint64_t stride = 0;
+    const bool table = !uniform(buckets, n_buckets, (int64_t)bucket_bytes, &stride);
+    if (table && n_buckets > kLargePtrs)
+        return rr_fail(RR_EINVAL, "%d separately allocated buckets exceed %d pointers", n_buckets,
+                       kLargePtrs);
+    StaticVerifyDevice* d = nullptr;
+    if ((st = static_verify_setup(&d))) return st;
+
+    // The array keeps the previous call's contents: clear the sums and counters used here.
+    RR_CUDA(cudaMemsetAsync(d->scratch, 0, (size_t(n_buckets) + 4) * sizeof(unsigned long long),
+                            stream));
+    st = (!table || n_buckets <= kSmallPtrs)
+             ? launch_static_verify<kSmallPtrs>(d->scratch, d->grid, n_buckets, bucket_bytes,
+                                                buckets, checksums, table, stride, stream)
+             : launch_static_verify<kLargePtrs>(d->scratch, d->grid, n_buckets, bucket_bytes,
+                                                buckets, checksums, table, stride, stream);
+    if (st) return st;
+    unsigned long long result[4] = {0, 0, 0, 0};   // host stack: no pinned buffer needed
+    RR_CUDA(cudaMemcpyAsync(result, d->scratch + n_buckets, sizeof result, cudaMemcpyDeviceToHost,
+                            stream));
+    RR_CUDA(cudaStreamSynchronize(stream));
+    if (n_bad) *n_bad = (int64_t)result[1];
+    if (first_bad) *first_bad = result[1] ? (int64_t)(ULLONG_MAX - result[2]) : -1;
+    return result[1] ? RR_EMISMATCH : RR_OK;
+}

@@ -130,14 +130,16 @@ _sig("rr_plan_export_unpack", [_vp, ctypes.POINTER(UnpackItem), ctypes.c_int64,
 _sig("rr_pack", [_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _vp])
 _sig("rr_unpack", [_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp])
 _sig("rr_verify", [_vp, ctypes.POINTER(_vp), _vp, _P64, _P64, _vp])
+_sig("rr_verify_noalloc", [ctypes.POINTER(_vp), ctypes.c_int32, ctypes.c_size_t, _vp, _P64, _P64,
+                           _vp])
 _sig("rr_status_str", [ctypes.c_int], ctypes.c_char_p)
 _sig("rr_last_error", [], ctypes.c_char_p)
 
 LIBRARY_PATH = _build.LIB
 EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_query",
             "rr_plan_source", "rr_plan_tensors", "rr_plan_get_stats", "rr_plan_export_pack",
-            "rr_plan_export_unpack", "rr_pack", "rr_unpack", "rr_verify", "rr_status_str",
-            "rr_last_error")
+            "rr_plan_export_unpack", "rr_pack", "rr_unpack", "rr_verify", "rr_verify_noalloc",
+            "rr_status_str", "rr_last_error")
 
 
 class RRError(RuntimeError):
@@ -439,3 +441,20 @@ def rr_verify(plan: Plan, buckets, checksums, stream=None):
         _check(st, "rr_verify")
     return n_bad.value, first.value
 
+
+def rr_verify_noalloc(buckets, n_buckets: int, bucket_bytes: int, checksums, stream=None):
+    """Allocation-free checksum check, for callers that cannot allocate device
+    memory at that moment (e.g. an inference engine that has reserved almost all
+    of it).  No plan needed; returns (n_bad, first_bad).  Synchronous; at most
+    16384 buckets; overlapping calls share one device scratch array and race."""
+    _check_list(buckets, n_buckets, bucket_bytes, "buckets")
+    nb = _nbytes(checksums)
+    if nb is not None and nb < 8 * n_buckets:
+        raise ValueError(f"checksums: {nb} bytes, need {8 * n_buckets}")
+    n_bad = ctypes.c_int64()
+    first = ctypes.c_int64()
+    st = _lib.rr_verify_noalloc(_ptr_array(buckets), n_buckets, bucket_bytes, _ptr(checksums),
+                                ctypes.byref(n_bad), ctypes.byref(first), _stream(stream))
+    if st not in (RR_OK, RR_EMISMATCH):
+        _check(st, "rr_verify_noalloc")
+    return n_bad.value, first.value
