@@ -78,6 +78,12 @@ def barrier(world):
         dist.barrier()
 
 
+def aggregate_gbs(world: int, bytes_per_replica: int, slowest_ms: float) -> float:
+    """Whole-job GB/s: every replica moved bytes_per_replica; the job took as
+    long as its slowest rank."""
+    return world * bytes_per_replica / (slowest_ms * 1e-3) / 1e9
+
+
 def max_over_ranks(x: float, world: int) -> float:
     if world == 1:
         return x
@@ -313,7 +319,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     unpack_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
     verify_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
     ms_per_step = total_ms / args.steps
-    value = world * step_bytes / (ms_per_step * 1e-3) / 1e9
+    value = aggregate_gbs(world, step_bytes, ms_per_step)
 
     # End to end through the public API with host buffers: every step copies the
     # trainer's shards from pinned host memory, syncs, and reads back the checksums.
@@ -341,7 +347,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         b.record(stream)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(a.elapsed_time(b), world) / args.steps
-        e2e = {"value": round(world * step_bytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": UNIT,
+        e2e = {"value": round(aggregate_gbs(world, step_bytes, e2e_ms), 2), "unit": UNIT,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": round(e2e_ms, 3)}
         del host_src
