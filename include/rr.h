@@ -250,6 +250,41 @@ rr_status rr_unpack(const rr_plan* plan, const void* const* buckets, void* const
 rr_status rr_verify(const rr_plan* plan, const void* const* buckets, const uint64_t* checksums,
                     int64_t* n_bad, int64_t* first_bad, cudaStream_t stream);
 
+/* Resumable sync (Section 5.2.2): when a relay fails mid-pull, the rollout
+ * keeps what it already pulled and fetches the rest elsewhere; when the trainer
+ * fails mid-pull, the partial update is cleared and the pull starts again.
+ * These calls act on buckets [first_bucket, first_bucket + n_buckets) only.
+ * The pointer arrays are the full ones (all n_buckets buckets, all tensors,
+ * as for the full calls); only the range is read or written.  A range outside
+ * [0, n_buckets) is RR_EINVAL.
+ *
+ * rr_pack_range:   writes those buckets and checksums[first .. first+n) and
+ *                  nothing else; its output equals the full rr_pack's there.
+ * rr_unpack_range: writes exactly the destination bytes that lie in those
+ *                  buckets (a tensor that straddles the range's edge is
+ *                  written in part).
+ * rr_verify_range: as rr_verify over the range; if `bad` (device, n_buckets
+ *                  bytes) is not NULL, bad[i] = 1 when bucket first+i differs,
+ *                  else 0.  *first_bad is a global bucket index.
+ * rr_clear_range:  zero-fills those buckets (the "clear partial" path: a
+ *                  cleared bucket fails verify unless its checksum is 0).
+ * All four are stream-ordered; rr_verify_range blocks like rr_verify. */
+rr_status rr_pack_range(const rr_plan* plan, int32_t first_bucket, int32_t n_buckets,
+                        const void* const* src_shards, void* const* buckets, uint64_t* checksums,
+                        cudaStream_t stream);
+rr_status rr_unpack_range(const rr_plan* plan, int32_t first_bucket, int32_t n_buckets,
+                          const void* const* buckets, void* const* dst, cudaStream_t stream);
+rr_status rr_verify_range(const rr_plan* plan, int32_t first_bucket, int32_t n_buckets,
+                          const void* const* buckets, const uint64_t* checksums, uint8_t* bad,
+                          int64_t* n_bad, int64_t* first_bad, cudaStream_t stream);
+rr_status rr_clear_range(const rr_plan* plan, int32_t first_bucket, int32_t n_buckets,
+                         void* const* buckets, cudaStream_t stream);
+
+/* Per-bucket item index of the two work tables (n_buckets + 1 entries each,
+ * either pointer may be NULL): the pack items of bucket b are
+ * [pack_first[b], pack_first[b + 1]); likewise for unpack. */
+rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32_t* unpack_first);
+
 /* Allocation-free form of rr_verify.  The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory when they
  * check a pull, such as an inference engine that has reserved nearly all

@@ -57,6 +57,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
         ["g++", "-O2", "-std=c++17", "-fPIC", "-Wall", "-c", os.path.join(CSRC, "rr_plan.cpp"),
          "-o", plan_o] + inc,
         [nvcc, "-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xptxas", "-v"] + ARCH +
+        os.environ.get("RR_EXTRA_NVCC_FLAGS", "").split() +
         ["-c", os.path.join(CSRC, "rr_device.cu"), "-o", dev_o] + inc,
     ]
     procs = [subprocess.Popen(j, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)

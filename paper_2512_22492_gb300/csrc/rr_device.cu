@@ -23,8 +23,24 @@
 
 namespace {
 
-constexpr int kThreads = 256;       // threads per block, all three kernels
-constexpr int kUnroll = 4;          // 16-byte vectors in flight per thread
+// Launch shape (overridable at build time for tuning sweeps).
+#ifndef RR_THREADS
+#define RR_THREADS 256
+#endif
+#ifndef RR_UNROLL
+#define RR_UNROLL 4
+#endif
+#ifndef RR_PACK_MIN_BLOCKS
+#define RR_PACK_MIN_BLOCKS 2
+#endif
+#ifndef RR_LD_HINT
+#define RR_LD_HINT 0
+#endif
+#ifndef RR_ST_HINT
+#define RR_ST_HINT 0
+#endif
+constexpr int kThreads = RR_THREADS;   // threads per block, all three kernels
+constexpr int kUnroll = RR_UNROLL;     // 16-byte vectors in flight per thread
 constexpr int kSmallPtrs = 64;      // pointer-table sizes of the two launch shapes
 constexpr int kLargePtrs = 3968;    // keeps the kernel parameters under 32 KB
 constexpr int64_t kVerifyChunk = 64 * 1024;
@@ -37,7 +53,9 @@ constexpr int64_t kVerifyChunk = 64 * 1024;
 template <int NPTR>
 struct PackArgs {
     const rr_pack_item* items;
-    const uint32_t* block_first;
+    const uint32_t* block_first;   // balanced per-block ranges, or NULL: split
+    uint32_t item_begin;           //   [item_begin, item_end) evenly over the grid
+    uint32_t item_end;
     unsigned long long* checksums;
     char* bucket_base;        // equally spaced buckets: base + b * stride
     uint64_t bucket_stride;   // 0: bucket b is ptr[n_shards + b]
@@ -49,7 +67,9 @@ struct PackArgs {
 template <int NPTR>
 struct UnpackArgs {
     const rr_unpack_item* items;
-    const uint32_t* block_first;
+    const uint32_t* block_first;   // as in PackArgs
+    uint32_t item_begin;
+    uint32_t item_end;
     const char* bucket_base;
     uint64_t bucket_stride;
     int32_t dst_base;         // index in ptr[] of destination tensor 0
@@ -61,7 +81,10 @@ template <int NPTR>
 struct VerifyArgs {
     unsigned long long* sums;       // [n_buckets], zeroed
     unsigned long long* counters;   // [4]: blocks done, n_bad, max(ULLONG_MAX - bad index)
-    const unsigned long long* expected;
+    const unsigned long long* expected;   // indexed by global bucket
+    uint8_t* bad;                   // optional [n_buckets]: 1 where the sum differs
+    int32_t first_bucket;           // the range checked is [first_bucket, +n_buckets)
+    int32_t pad0;
     const char* bucket_base;
     uint64_t bucket_stride;
     uint64_t bucket_bytes;
@@ -77,18 +100,36 @@ struct VerifyArgs {
 // Small device helpers
 // ---------------------------------------------------------------------------
 
+// Streaming 16-byte load of data read exactly once (read-only for the kernel).
 __device__ __forceinline__ uint4 ld_stream(const void* p) {
     uint4 r;
+#if RR_LD_HINT == 1
+    asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
+#elif RR_LD_HINT == 2
+    asm volatile("ld.global.cs.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
+#else
     asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
                  : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
                  : "l"(p));
+#endif
     return r;
 }
 
+// 16-byte store of data written exactly once.
 __device__ __forceinline__ void st_stream(void* p, uint4 v) {
+#if RR_ST_HINT == 1
+    asm volatile("st.global.cs.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+#else
     asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y),
                  "r"(v.z), "r"(v.w)
                  : "memory");
+#endif
 }
 
 // float32 bits -> value whose upper half is the bfloat16 result: round to
@@ -122,6 +163,20 @@ __device__ __forceinline__ void flush(unsigned long long* dst, unsigned long lon
     if ((threadIdx.x & 31) == 0 && acc != 0ull) atomicAdd(dst, acc);
 }
 
+// This block's item range: the plan's balanced split for a full call, an even
+// split of [begin, end) for a bucket-range call.
+__device__ __forceinline__ void block_items(const uint32_t* block_first, uint32_t begin,
+                                            uint32_t end, uint32_t* i0, uint32_t* i1) {
+    if (block_first) {
+        *i0 = block_first[blockIdx.x];
+        *i1 = block_first[blockIdx.x + 1];
+    } else {
+        const uint64_t n = end - begin;
+        *i0 = begin + (uint32_t)(n * blockIdx.x / gridDim.x);
+        *i1 = begin + (uint32_t)(n * (blockIdx.x + 1) / gridDim.x);
+    }
+}
+
 template <int NPTR>
 __device__ __forceinline__ char* bucket_of(const PackArgs<NPTR>& a, uint32_t b) {
     return a.bucket_stride ? a.bucket_base + (uint64_t)b * a.bucket_stride
@@ -139,6 +194,9 @@ __device__ __forceinline__ char* bucket_of(const PackArgs<NPTR>& a, uint32_t b) 
 template <int ES>
 __device__ __forceinline__ unsigned long long pack_vec(const char* src, char* dst,
                                                        const rr_pack_item& d) {
+    // A bf16 vector is one 16-byte load instead of two: twice as many of them
+    // keep the same bytes in flight per thread.
+    constexpr int U = ES == 4 ? kUnroll : 2 * kUnroll;
     const uint32_t vpr = d.row_len >> 3;
     const uint32_t nvec = vpr * d.n_rows;
     const uint64_t stride = (uint64_t)d.src_stride * ES;
@@ -147,10 +205,10 @@ __device__ __forceinline__ unsigned long long pack_vec(const char* src, char* ds
     uint32_t r = v / vpr, c = v - r * vpr;
     unsigned long long acc = 0;
     while (v < nvec) {
-        uint4 x[kUnroll][ES / 2];
-        uint32_t vv[kUnroll];
+        uint4 x[U][ES / 2];
+        uint32_t vv[U];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
+        for (int u = 0; u < U; ++u) {
             vv[u] = v;
             if (v < nvec) {
                 const char* p = src + r * stride + (uint64_t)c * (8 * ES);
@@ -166,7 +224,7 @@ __device__ __forceinline__ unsigned long long pack_vec(const char* src, char* ds
             }
         }
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
+        for (int u = 0; u < U; ++u) {
             if (vv[u] < nvec) {
                 uint4 o;
                 if (ES == 4) {
@@ -218,11 +276,12 @@ __device__ __forceinline__ unsigned long long pack_scalar(const char* src, char*
 }
 
 template <int NPTR>
-__global__ void __launch_bounds__(kThreads, 2) rr_pack_kernel(const __grid_constant__ PackArgs<NPTR> a) {
-    const uint32_t i1 = a.block_first[blockIdx.x + 1];
+__global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(const __grid_constant__ PackArgs<NPTR> a) {
+    uint32_t i0, i1;
+    block_items(a.block_first, a.item_begin, a.item_end, &i0, &i1);
     unsigned long long acc = 0;
     uint32_t cur = 0xFFFFFFFFu;
-    for (uint32_t it = a.block_first[blockIdx.x]; it < i1; ++it) {
+    for (uint32_t it = i0; it < i1; ++it) {
         const rr_pack_item d = a.items[it];
         if (d.bucket != cur) {
             if (cur != 0xFFFFFFFFu) flush(a.checksums + cur, acc);
@@ -255,21 +314,25 @@ __global__ void __launch_bounds__(kThreads, 2) rr_pack_kernel(const __grid_const
 
 template <int NPTR>
 __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
-    const uint32_t i1 = a.block_first[blockIdx.x + 1];
-    for (uint32_t it = a.block_first[blockIdx.x]; it < i1; ++it) {
+    uint32_t i0, i1;
+    block_items(a.block_first, a.item_begin, a.item_end, &i0, &i1);
+    for (uint32_t it = i0; it < i1; ++it) {
         const rr_unpack_item d = a.items[it];
         const char* src = (a.bucket_stride ? a.bucket_base + (uint64_t)d.bucket * a.bucket_stride
                                            : (const char*)a.ptr[d.bucket]) + d.src_off;
         char* dst = (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off;
         if (d.kind == RR_ITEM_COPY_VEC) {
+            // One 16-byte load per vector: twice the pack's depth keeps as many
+            // bytes in flight.
+            constexpr int U = 2 * kUnroll;
             const uint32_t nvec = d.nbytes >> 4;
-            for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * kUnroll) {
-                uint4 x[kUnroll];
+            for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * U) {
+                uint4 x[U];
 #pragma unroll
-                for (int u = 0; u < kUnroll; ++u)
+                for (int u = 0; u < U; ++u)
                     if (v + u * kThreads < nvec) x[u] = ld_stream(src + 16ull * (v + u * kThreads));
 #pragma unroll
-                for (int u = 0; u < kUnroll; ++u)
+                for (int u = 0; u < U; ++u)
                     if (v + u * kThreads < nvec) st_stream(dst + 16ull * (v + u * kThreads), x[u]);
             }
         } else {
@@ -290,14 +353,15 @@ __global__ void __launch_bounds__(kThreads, 4) rr_verify_kernel(const __grid_con
     unsigned long long acc = 0;
     uint32_t cur = 0xFFFFFFFFu;
     for (uint64_t ch = c0; ch < c1; ++ch) {
-        const uint32_t b = (uint32_t)(ch / a.chunks_per_bucket);
-        const uint64_t off = (ch - (uint64_t)b * a.chunks_per_bucket) * a.chunk_bytes;
+        const uint32_t bl = (uint32_t)(ch / a.chunks_per_bucket);   // index within the range
+        const uint64_t off = (ch - (uint64_t)bl * a.chunks_per_bucket) * a.chunk_bytes;
         const uint64_t len = min(a.chunk_bytes, a.bucket_bytes - off);
-        if (b != cur) {
+        if (bl != cur) {
             if (cur != 0xFFFFFFFFu) flush(a.sums + cur, acc);
-            cur = b;
+            cur = bl;
             acc = 0;
         }
+        const uint32_t b = a.first_bucket + bl;
         const char* p = (a.bucket_stride ? a.bucket_base + (uint64_t)b * a.bucket_stride
                                          : (const char*)a.ptr[b]) + off;
         const uint32_t nvec = (uint32_t)(len >> 4);
@@ -325,8 +389,11 @@ __global__ void __launch_bounds__(kThreads, 4) rr_verify_kernel(const __grid_con
     __syncthreads();
     if (!last) return;
     __threadfence();
-    for (int32_t b = threadIdx.x; b < a.n_buckets; b += kThreads) {
-        if (__ldcg(a.sums + b) != a.expected[b]) {
+    for (int32_t bl = threadIdx.x; bl < a.n_buckets; bl += kThreads) {
+        const int32_t b = a.first_bucket + bl;
+        const bool differs = __ldcg(a.sums + bl) != a.expected[b];
+        if (a.bad) a.bad[bl] = differs ? 1 : 0;
+        if (differs) {
             atomicAdd(&a.counters[1], 1ull);
             atomicMax(&a.counters[2], ULLONG_MAX - (unsigned long long)b);
         }
@@ -381,13 +448,22 @@ rr_status check_ptrs(const void* const* ptrs, int32_t n, const char* what) {
     return RR_OK;
 }
 
+// A call covers buckets [b0, b1).  The full range uses the plan's balanced
+// per-block item ranges; a sub-range splits its items evenly over the grid.
+struct Range {
+    int32_t b0, b1;
+    bool full;
+};
+
 template <int NPTR>
-rr_status launch_pack(const rr_plan* P, const void* const* src, void* const* buckets,
+rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* const* buckets,
                       uint64_t* checksums, bool table, uint64_t stride, cudaStream_t s) {
     PackArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     a.items = P->d_pack_items;
-    a.block_first = P->d_pack_block_first;
+    a.block_first = R.full ? P->d_pack_block_first : nullptr;
+    a.item_begin = P->pack_bucket_first[R.b0];
+    a.item_end = P->pack_bucket_first[R.b1];
     a.checksums = (unsigned long long*)checksums;
     a.n_shards = P->n_shards;
     for (int32_t i = 0; i < P->n_shards; ++i) a.ptr[i] = src[i];
@@ -403,12 +479,14 @@ rr_status launch_pack(const rr_plan* P, const void* const* src, void* const* buc
 }
 
 template <int NPTR>
-rr_status launch_unpack(const rr_plan* P, const void* const* buckets, void* const* dst, bool table,
-                        uint64_t stride, cudaStream_t s) {
+rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
+                        bool table, uint64_t stride, cudaStream_t s) {
     UnpackArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     a.items = P->d_unpack_items;
-    a.block_first = P->d_unpack_block_first;
+    a.block_first = R.full ? P->d_unpack_block_first : nullptr;
+    a.item_begin = P->unpack_bucket_first[R.b0];
+    a.item_end = P->unpack_bucket_first[R.b1];
     int32_t k = 0;
     if (table) {
         for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[k++] = buckets[b];
@@ -424,18 +502,22 @@ rr_status launch_unpack(const rr_plan* P, const void* const* buckets, void* cons
 }
 
 template <int NPTR>
-rr_status launch_verify(const rr_plan* P, const void* const* buckets, const uint64_t* checksums,
-                        bool table, uint64_t stride, cudaStream_t s) {
+rr_status launch_verify(const rr_plan* P, Range R, const void* const* buckets,
+                        const uint64_t* checksums, uint8_t* bad, bool table, uint64_t stride,
+                        cudaStream_t s) {
     VerifyArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
+    const int32_t n = R.b1 - R.b0;
     a.sums = P->d_verify_scratch;
-    a.counters = P->d_verify_scratch + P->n_buckets;
+    a.counters = P->d_verify_scratch + n;
     a.expected = (const unsigned long long*)checksums;
+    a.bad = bad;
+    a.first_bucket = R.b0;
     a.bucket_bytes = (uint64_t)P->bucket_bytes;
     a.chunk_bytes = (uint64_t)std::min<int64_t>(kVerifyChunk, P->bucket_bytes);
     a.chunks_per_bucket = (a.bucket_bytes + a.chunk_bytes - 1) / a.chunk_bytes;
-    a.total_chunks = a.chunks_per_bucket * (uint64_t)P->n_buckets;
-    a.n_buckets = P->n_buckets;
+    a.total_chunks = a.chunks_per_bucket * (uint64_t)n;
+    a.n_buckets = n;
     if (table) {
         for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[b] = buckets[b];
     } else {
@@ -445,6 +527,90 @@ rr_status launch_verify(const rr_plan* P, const void* const* buckets, const uint
     rr_verify_kernel<NPTR><<<P->verify_grid_blocks, kThreads, 0, s>>>(a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
+}
+
+rr_status check_range(const rr_plan* P, int32_t first, int32_t n, Range* R) {
+    if (first < 0 || n < 0 || first > P->n_buckets || n > P->n_buckets - first)
+        return rr_fail(RR_EINVAL, "bucket range [%d, %d + %d) outside [0, %d)", first, first, n,
+                       P->n_buckets);
+    *R = Range{first, first + n, first == 0 && n == P->n_buckets};
+    return RR_OK;
+}
+
+rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, void* const* buckets,
+                    uint64_t* checksums, cudaStream_t stream) {
+    rr_status st;
+    if ((st = check_ptrs(src_shards, P->n_shards, "src_shards"))) return st;
+    if ((st = check_ptrs((const void* const*)buckets, P->n_buckets, "buckets"))) return st;
+    if (R.b1 == R.b0) return RR_OK;
+    if (!aligned16(checksums)) return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    uint64_t stride = 0;
+    const bool table = !uniform((const void* const*)buckets, P->n_buckets, P->bucket_bytes, &stride);
+    const int32_t need = P->n_shards + (table ? P->n_buckets : 0);
+    if (need > kLargePtrs)
+        return rr_fail(RR_EINVAL,
+                       "%d shards + %d separately allocated buckets exceed %d pointers; allocate "
+                       "the buckets as one equally spaced block",
+                       P->n_shards, P->n_buckets, kLargePtrs);
+    RR_CUDA(cudaMemsetAsync(checksums + R.b0, 0, size_t(R.b1 - R.b0) * 8, stream));
+    if (P->pack_bucket_first[R.b0] == P->pack_bucket_first[R.b1]) return RR_OK;
+    return need <= kSmallPtrs
+               ? launch_pack<kSmallPtrs>(P, R, src_shards, buckets, checksums, table, stride, stream)
+               : launch_pack<kLargePtrs>(P, R, src_shards, buckets, checksums, table, stride, stream);
+}
+
+rr_status unpack_impl(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
+                      cudaStream_t stream) {
+    rr_status st;
+    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if (P->n_tensors > 0 && !dst) return rr_fail(RR_EINVAL, "dst array is NULL");
+    for (int32_t t = 0; t < P->n_tensors; ++t)
+        if (P->tensor_numel[t] > 0 && !aligned16(dst[t]))
+            return rr_fail(RR_EINVAL, "dst[%d] is NULL or not 16-byte aligned", t);
+    if (P->unpack_bucket_first[R.b0] == P->unpack_bucket_first[R.b1]) return RR_OK;
+    uint64_t stride = 0;
+    const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
+    const int32_t need = P->n_tensors + (table ? P->n_buckets : 0);
+    if (need <= kSmallPtrs)
+        return launch_unpack<kSmallPtrs>(P, R, buckets, dst, table, stride, stream);
+    if (need <= kLargePtrs)
+        return launch_unpack<kLargePtrs>(P, R, buckets, dst, table, stride, stream);
+    return rr_fail(RR_EINVAL, "%d tensors + %d separately allocated buckets exceed %d pointers",
+                   P->n_tensors, P->n_buckets, kLargePtrs);
+}
+
+rr_status verify_impl(const rr_plan* P, Range R, const void* const* buckets,
+                      const uint64_t* checksums, uint8_t* bad, int64_t* n_bad, int64_t* first_bad,
+                      cudaStream_t stream) {
+    rr_status st;
+    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if (R.b1 > R.b0 && !aligned16(checksums))
+        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    if (n_bad) *n_bad = 0;
+    if (first_bad) *first_bad = -1;
+    if (R.b1 == R.b0) return RR_OK;
+    uint64_t stride = 0;
+    const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
+    if (table && P->n_buckets > kLargePtrs)
+        return rr_fail(RR_EINVAL, "%d separately allocated buckets exceed %d pointers",
+                       P->n_buckets, kLargePtrs);
+
+    rr_plan* M = const_cast<rr_plan*>(P);   // the scratch area is the only mutable state
+    std::lock_guard<std::mutex> lock(M->verify_mutex);
+    const int32_t n = R.b1 - R.b0;
+    RR_CUDA(cudaMemsetAsync(P->d_verify_scratch, 0, (size_t(n) + 4) * sizeof(unsigned long long),
+                            stream));
+    st = (!table || P->n_buckets <= kSmallPtrs)
+             ? launch_verify<kSmallPtrs>(P, R, buckets, checksums, bad, table, stride, stream)
+             : launch_verify<kLargePtrs>(P, R, buckets, checksums, bad, table, stride, stream);
+    if (st) return st;
+    RR_CUDA(cudaMemcpyAsync(P->h_verify_result, P->d_verify_scratch + n,
+                            4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, stream));
+    RR_CUDA(cudaStreamSynchronize(stream));
+    const unsigned long long nb = P->h_verify_result[1];
+    if (n_bad) *n_bad = (int64_t)nb;
+    if (first_bad) *first_bad = nb ? (int64_t)(ULLONG_MAX - P->h_verify_result[2]) : -1;
+    return nb ? RR_EMISMATCH : RR_OK;
 }
 
 }  // namespace
@@ -521,23 +687,7 @@ extern "C" rr_status rr_pack(const rr_plan* P, const void* const* src_shards,
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
-    if ((st = check_ptrs(src_shards, P->n_shards, "src_shards"))) return st;
-    if ((st = check_ptrs((const void* const*)buckets, P->n_buckets, "buckets"))) return st;
-    if (P->n_buckets == 0) return RR_OK;
-    if (!aligned16(checksums)) return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
-    uint64_t stride = 0;
-    const bool table = !uniform((const void* const*)buckets, P->n_buckets, P->bucket_bytes, &stride);
-    RR_CUDA(cudaMemsetAsync(checksums, 0, size_t(P->n_buckets) * 8, stream));
-    if (P->pack_items.empty()) return RR_OK;
-    const int32_t need = P->n_shards + (table ? P->n_buckets : 0);
-    if (need <= kSmallPtrs)
-        return launch_pack<kSmallPtrs>(P, src_shards, buckets, checksums, table, stride, stream);
-    if (need <= kLargePtrs)
-        return launch_pack<kLargePtrs>(P, src_shards, buckets, checksums, table, stride, stream);
-    return rr_fail(RR_EINVAL,
-                   "%d shards + %d separately allocated buckets exceed %d pointers; allocate the "
-                   "buckets as one equally spaced block",
-                   P->n_shards, P->n_buckets, kLargePtrs);
+    return pack_impl(P, Range{0, P->n_buckets, true}, src_shards, buckets, checksums, stream);
 }
 
 extern "C" rr_status rr_unpack(const rr_plan* P, const void* const* buckets, void* const* dst,
@@ -545,19 +695,7 @@ extern "C" rr_status rr_unpack(const rr_plan* P, const void* const* buckets, voi
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
-    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
-    if (P->n_tensors > 0 && !dst) return rr_fail(RR_EINVAL, "dst array is NULL");
-    for (int32_t t = 0; t < P->n_tensors; ++t)
-        if (P->tensor_numel[t] > 0 && !aligned16(dst[t]))
-            return rr_fail(RR_EINVAL, "dst[%d] is NULL or not 16-byte aligned", t);
-    if (P->unpack_items.empty()) return RR_OK;
-    uint64_t stride = 0;
-    const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
-    const int32_t need = P->n_tensors + (table ? P->n_buckets : 0);
-    if (need <= kSmallPtrs) return launch_unpack<kSmallPtrs>(P, buckets, dst, table, stride, stream);
-    if (need <= kLargePtrs) return launch_unpack<kLargePtrs>(P, buckets, dst, table, stride, stream);
-    return rr_fail(RR_EINVAL, "%d tensors + %d separately allocated buckets exceed %d pointers",
-                   P->n_tensors, P->n_buckets, kLargePtrs);
+    return unpack_impl(P, Range{0, P->n_buckets, true}, buckets, dst, stream);
 }
 
 extern "C" rr_status rr_verify(const rr_plan* P, const void* const* buckets,
@@ -566,33 +704,58 @@ extern "C" rr_status rr_verify(const rr_plan* P, const void* const* buckets,
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
-    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
-    if (P->n_buckets > 0 && !aligned16(checksums))
-        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
-    if (n_bad) *n_bad = 0;
-    if (first_bad) *first_bad = -1;
-    if (P->n_buckets == 0) return RR_OK;
-    uint64_t stride = 0;
-    const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
-    if (table && P->n_buckets > kLargePtrs)
-        return rr_fail(RR_EINVAL, "%d separately allocated buckets exceed %d pointers",
-                       P->n_buckets, kLargePtrs);
+    return verify_impl(P, Range{0, P->n_buckets, true}, buckets, checksums, nullptr, n_bad,
+                       first_bad, stream);
+}
 
-    rr_plan* M = const_cast<rr_plan*>(P);   // the scratch area is the only mutable state
-    std::lock_guard<std::mutex> lock(M->verify_mutex);
-    RR_CUDA(cudaMemsetAsync(P->d_verify_scratch, 0,
-                            (size_t(P->n_buckets) + 4) * sizeof(unsigned long long), stream));
-    st = (!table || P->n_buckets <= kSmallPtrs)
-             ? launch_verify<kSmallPtrs>(P, buckets, checksums, table, stride, stream)
-             : launch_verify<kLargePtrs>(P, buckets, checksums, table, stride, stream);
-    if (st) return st;
-    RR_CUDA(cudaMemcpyAsync(P->h_verify_result, P->d_verify_scratch + P->n_buckets,
-                            4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, stream));
-    RR_CUDA(cudaStreamSynchronize(stream));
-    const unsigned long long bad = P->h_verify_result[1];
-    if (n_bad) *n_bad = (int64_t)bad;
-    if (first_bad) *first_bad = bad ? (int64_t)(ULLONG_MAX - P->h_verify_result[2]) : -1;
-    return bad ? RR_EMISMATCH : RR_OK;
+extern "C" rr_status rr_pack_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,
+                                   const void* const* src_shards, void* const* buckets,
+                                   uint64_t* checksums, cudaStream_t stream) {
+    rr_clear_error();
+    Range R;
+    rr_status st = check_plan(P);
+    if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
+    return pack_impl(P, R, src_shards, buckets, checksums, stream);
+}
+
+extern "C" rr_status rr_unpack_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,
+                                     const void* const* buckets, void* const* dst,
+                                     cudaStream_t stream) {
+    rr_clear_error();
+    Range R;
+    rr_status st = check_plan(P);
+    if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
+    return unpack_impl(P, R, buckets, dst, stream);
+}
+
+extern "C" rr_status rr_verify_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,
+                                     const void* const* buckets, const uint64_t* checksums,
+                                     uint8_t* bad, int64_t* n_bad, int64_t* first_bad,
+                                     cudaStream_t stream) {
+    rr_clear_error();
+    Range R;
+    rr_status st = check_plan(P);
+    if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
+    return verify_impl(P, R, buckets, checksums, bad, n_bad, first_bad, stream);
+}
+
+extern "C" rr_status rr_clear_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,
+                                    void* const* buckets, cudaStream_t stream) {
+    rr_clear_error();
+    Range R;
+    rr_status st = check_plan(P);
+    if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
+    if ((st = check_ptrs((const void* const*)buckets, P->n_buckets, "buckets"))) return st;
+    if (n_buckets == 0) return RR_OK;
+    uint64_t stride = 0;
+    if (uniform((const void* const*)buckets, P->n_buckets, P->bucket_bytes, &stride)) {
+        RR_CUDA(cudaMemset2DAsync(buckets[R.b0], stride, 0, (size_t)P->bucket_bytes,
+                                  (size_t)n_buckets, stream));
+    } else {
+        for (int32_t b = R.b0; b < R.b1; ++b)
+            RR_CUDA(cudaMemsetAsync(buckets[b], 0, (size_t)P->bucket_bytes, stream));
+    }
+    return RR_OK;
 }
 
 // ---------------------------------------------------------------------------

@@ -40,6 +40,8 @@ struct rr_plan {
     std::vector<uint32_t> pack_block_first;     // grid_blocks + 1
     std::vector<rr_unpack_item> unpack_items;
     std::vector<uint32_t> unpack_block_first;   // grid_blocks + 1
+    std::vector<uint32_t> pack_bucket_first;    // n_buckets + 1: first pack item of bucket b
+    std::vector<uint32_t> unpack_bucket_first;  // n_buckets + 1: first unpack item of bucket b
     rr_plan_stats stats{};
 
     // ---- device state (owned) -------------------------------------------

@@ -372,6 +372,17 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
         for (int32_t t = 0; t < P->n_tensors; ++t)
             if (P->tensor_rank[t] == r) b.unpack_tensor(t);
     }
+    // Both tables are sorted by bucket: index their per-bucket item ranges.
+    auto index = [&](auto& items, std::vector<uint32_t>& first) {
+        first.assign(size_t(P->n_buckets) + 1, uint32_t(items.size()));
+        size_t i = 0;
+        for (int32_t bk = 0; bk < P->n_buckets; ++bk) {
+            while (i < items.size() && int64_t(items[i].bucket) < bk) ++i;
+            first[bk] = uint32_t(i);
+        }
+    };
+    index(P->pack_items, P->pack_bucket_first);
+    index(P->unpack_items, P->unpack_bucket_first);
     partition(P->pack_items, P->grid_blocks, P->pack_block_first, pack_weight);
     partition(P->unpack_items, P->unpack_grid_blocks, P->unpack_block_first, unpack_weight);
 
@@ -516,6 +527,15 @@ rr_status rr_plan_export_unpack(const rr_plan* P, rr_unpack_item* items, int64_t
     if (n > 0) std::memcpy(items, P->unpack_items.data(), size_t(n) * sizeof(rr_unpack_item));
     if (block_first)
         std::copy(P->unpack_block_first.begin(), P->unpack_block_first.end(), block_first);
+    return RR_OK;
+}
+
+rr_status rr_plan_bucket_items(const rr_plan* P, uint32_t* pack_first, uint32_t* unpack_first) {
+    if (!P) return rr_fail(RR_EINVAL, "plan is NULL");
+    if (pack_first)
+        std::copy(P->pack_bucket_first.begin(), P->pack_bucket_first.end(), pack_first);
+    if (unpack_first)
+        std::copy(P->unpack_bucket_first.begin(), P->unpack_bucket_first.end(), unpack_first);
     return RR_OK;
 }
 

@@ -130,6 +130,14 @@ _sig("rr_plan_export_unpack", [_vp, ctypes.POINTER(UnpackItem), ctypes.c_int64,
 _sig("rr_pack", [_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _vp])
 _sig("rr_unpack", [_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp])
 _sig("rr_verify", [_vp, ctypes.POINTER(_vp), _vp, _P64, _P64, _vp])
+_sig("rr_pack_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp),
+                       ctypes.POINTER(_vp), _vp, _vp])
+_sig("rr_unpack_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp),
+                         ctypes.POINTER(_vp), _vp])
+_sig("rr_verify_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp, _vp, _P64,
+                         _P64, _vp])
+_sig("rr_clear_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp])
+_sig("rr_plan_bucket_items", [_vp, ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_uint32)])
 _sig("rr_verify_noalloc", [ctypes.POINTER(_vp), ctypes.c_int32, ctypes.c_size_t, _vp, _P64, _P64,
                            _vp])
 _sig("rr_status_str", [ctypes.c_int], ctypes.c_char_p)
@@ -138,7 +146,9 @@ _sig("rr_last_error", [], ctypes.c_char_p)
 LIBRARY_PATH = _build.LIB
 EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_query",
             "rr_plan_source", "rr_plan_tensors", "rr_plan_get_stats", "rr_plan_export_pack",
-            "rr_plan_export_unpack", "rr_pack", "rr_unpack", "rr_verify", "rr_verify_noalloc",
+            "rr_plan_export_unpack", "rr_plan_bucket_items", "rr_pack", "rr_unpack", "rr_verify",
+            "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
+            "rr_verify_noalloc",
             "rr_status_str", "rr_last_error")
 
 
@@ -284,6 +294,16 @@ class Plan:
                                           first.ctypes.data_as(ctypes.POINTER(ctypes.c_uint32))),
                "rr_plan_export_unpack")
         return items[:n], first
+
+    def bucket_items(self):
+        """Per-bucket first item of the pack and unpack tables (n_buckets + 1 each)."""
+        import numpy as np
+        pf = np.zeros(self.n_buckets + 1, np.uint32)
+        uf = np.zeros(self.n_buckets + 1, np.uint32)
+        P = ctypes.POINTER(ctypes.c_uint32)
+        _check(_lib.rr_plan_bucket_items(self._h, pf.ctypes.data_as(P), uf.ctypes.data_as(P)),
+               "rr_plan_bucket_items")
+        return pf, uf
 
     def destroy(self) -> None:
         if self._h:
@@ -440,6 +460,51 @@ def rr_verify(plan: Plan, buckets, checksums, stream=None):
     if st not in (RR_OK, RR_EMISMATCH):
         _check(st, "rr_verify")
     return n_bad.value, first.value
+
+
+def rr_pack_range(plan: Plan, first_bucket: int, n_buckets: int, src_shards, buckets, checksums,
+                  stream=None) -> None:
+    """Pack only buckets [first_bucket, first_bucket + n_buckets) (asynchronous)."""
+    _check_list(src_shards, plan.n_shards, plan.shard_bytes, "src_shards")
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_checksums(plan, checksums)
+    _check(_lib.rr_pack_range(plan.handle, first_bucket, n_buckets, _ptr_array(src_shards),
+                              _ptr_array(buckets), _ptr(checksums), _stream(stream)),
+           "rr_pack_range")
+
+
+def rr_unpack_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, dst,
+                    stream=None) -> None:
+    """Unpack only the destination bytes held by those buckets (asynchronous)."""
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst")
+    _check(_lib.rr_unpack_range(plan.handle, first_bucket, n_buckets, _ptr_array(buckets),
+                                _ptr_array(dst), _stream(stream)), "rr_unpack_range")
+
+
+def rr_verify_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, checksums, bad=None,
+                    stream=None):
+    """Verify those buckets; optional device byte array `bad` gets one flag per
+    bucket of the range.  Returns (n_bad, first_bad).  Synchronous."""
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_checksums(plan, checksums)
+    if bad is not None and _nbytes(bad) is not None and _nbytes(bad) < n_buckets:
+        raise ValueError(f"bad: {_nbytes(bad)} bytes, need {n_buckets}")
+    n_bad = ctypes.c_int64()
+    first = ctypes.c_int64()
+    st = _lib.rr_verify_range(plan.handle, first_bucket, n_buckets, _ptr_array(buckets),
+                              _ptr(checksums), None if bad is None else _ptr(bad),
+                              ctypes.byref(n_bad), ctypes.byref(first), _stream(stream))
+    if st not in (RR_OK, RR_EMISMATCH):
+        _check(st, "rr_verify_range")
+    return n_bad.value, first.value
+
+
+def rr_clear_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, stream=None) -> None:
+    """Zero-fill buckets [first_bucket, first_bucket + n_buckets) (asynchronous)."""
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check(_lib.rr_clear_range(plan.handle, first_bucket, n_buckets, _ptr_array(buckets),
+                               _stream(stream)), "rr_clear_range")
 
 
 def rr_verify_noalloc(buckets, n_buckets: int, bucket_bytes: int, checksums, stream=None):

@@ -150,3 +150,31 @@ def test_host_only_plan_refuses_to_run():
     with pytest.raises(rr.RRError) as e:
         rr.rr_pack(p, [16] * p.n_shards, [16] * p.n_buckets, 16, stream=0)
     assert e.value.status == rrmod.RR_EINVAL
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_bucket_index_and_range_interpretation(seed):
+    """Each bucket's items are a contiguous run of both tables; interpreting only
+    a bucket range's pack items reproduces the oracle's buckets of that range."""
+    desc = U.random_layout(seed)
+    L = U.to_oracle(desc)
+    p = host_plan(desc)
+    items, _ = p.export_pack()
+    uitems, _ = p.export_unpack()
+    pf, uf = p.bucket_items()
+    assert pf[0] == 0 and pf[-1] == len(items) and np.all(np.diff(pf.astype(np.int64)) >= 0)
+    assert uf[0] == 0 and uf[-1] == len(uitems) and np.all(np.diff(uf.astype(np.int64)) >= 0)
+    for b in range(p.n_buckets):
+        assert np.all(items["bucket"][pf[b]:pf[b + 1]] == b)
+        assert np.all(uitems["bucket"][uf[b]:uf[b + 1]] == b)
+    if p.n_buckets < 2:
+        return
+    rng = np.random.default_rng(seed)
+    b0 = int(rng.integers(0, p.n_buckets - 1))
+    b1 = int(rng.integers(b0 + 1, p.n_buckets + 1))
+    shards = L.host_shards(desc["seed"], desc["specials"])
+    sub = items[pf[b0]:pf[b1]].copy()
+    sub["bucket"] -= b0
+    got = U.check_and_run_pack(sub, shards, b1 - b0, p.bucket_bytes, p.shard_bytes)
+    want, _ = L.pack(oracle.Source(shards=shards), first=b0, count=b1 - b0)
+    np.testing.assert_array_equal(got, want)
