@@ -47,6 +47,8 @@ def parse():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--workload", default="qwen3-8b")
     ap.add_argument("--bucket-mib", type=int, default=0, help="override the bucket size")
+    ap.add_argument("--chunk-kib", type=int, default=0, help="plan option: KiB per work item")
+    ap.add_argument("--grid", type=int, default=0, help="plan option: persistent grid size")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-buckets", type=int, default=2,
@@ -272,7 +274,10 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     torch.cuda.set_device(local)
     stream = torch.cuda.current_stream()
     m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp)
-    plan = rr.rr_plan_create(m, s, d, bucket_bytes)
+    opts = None
+    if args.chunk_kib or args.grid:
+        opts = rr.PlanOptions(chunk_bytes=args.chunk_kib * 1024, grid_blocks=args.grid)
+    plan = rr.rr_plan_create(m, s, d, bucket_bytes, opts)
     st = plan.stats()
     buf = H.alloc(plan, poison=None)
     H.fill_with_generator(buf, m, w.seed, w.specials)
