@@ -184,7 +184,9 @@ enum {
     RR_ITEM_ZERO_VEC = 4,   /* zero fill of alignment gaps / bucket tails            */
     RR_ITEM_ZERO_SCALAR = 5,
     RR_ITEM_COPY_VEC = 6,   /* unpack: 16-byte copies                                */
-    RR_ITEM_COPY_SCALAR = 7 /* unpack: 2-byte copies                                 */
+    RR_ITEM_COPY_SCALAR = 7, /* unpack: 2-byte copies                                */
+    RR_ITEM_READ_VEC = 8,    /* unpack table: alignment gap / tail, read only by the    */
+    RR_ITEM_READ_SCALAR = 9  /*   verifying unpack (their bytes count in the checksum)  */
 };
 
 /* Pack work item: n_rows rows of row_len elements; row i starts at source
@@ -202,7 +204,8 @@ typedef struct {
 } rr_pack_item;
 
 /* Unpack work item: copy nbytes from bucket `bucket` at src_off to tensor
- * `tensor` at dst_off. */
+ * `tensor` at dst_off (READ items: bucket bytes outside every tensor; tensor
+ * and dst_off unused). */
 typedef struct {
     uint64_t dst_off;
     uint32_t src_off;
@@ -279,6 +282,21 @@ rr_status rr_verify_range(const rr_plan* plan, int32_t first_bucket, int32_t n_b
                           int64_t* n_bad, int64_t* first_bad, cudaStream_t stream);
 rr_status rr_clear_range(const rr_plan* plan, int32_t first_bucket, int32_t n_buckets,
                          void* const* buckets, cudaStream_t stream);
+
+/* Receiver side, fused: rr_unpack and rr_verify in one pass over the buckets
+ * (every bucket byte is read once, for the copy and for the checksum).
+ * Writes every destination byte of the range, as rr_unpack / rr_unpack_range
+ * would, whether or not its bucket verifies; the caller re-pulls the flagged
+ * buckets and unpacks them again (for example with this call on a range).
+ * bad, n_bad, first_bad and the return value are those of rr_verify_range.
+ * Blocks the calling thread until `stream` has finished, like rr_verify. */
+rr_status rr_unpack_verify(const rr_plan* plan, const void* const* buckets,
+                           const uint64_t* checksums, void* const* dst, uint8_t* bad,
+                           int64_t* n_bad, int64_t* first_bad, cudaStream_t stream);
+rr_status rr_unpack_verify_range(const rr_plan* plan, int32_t first_bucket, int32_t n_buckets,
+                                 const void* const* buckets, const uint64_t* checksums,
+                                 void* const* dst, uint8_t* bad, int64_t* n_bad,
+                                 int64_t* first_bad, cudaStream_t stream);
 
 /* Per-bucket item index of the two work tables (n_buckets + 1 entries each,
  * either pointer may be NULL): the pack items of bucket b are

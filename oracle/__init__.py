@@ -298,9 +298,10 @@ class Layout:
     def sync_sample(self, src: "Source", first: int, count: int) -> int:
         """One CPU weight sync restricted to buckets [first, first+count): pack
         them, unpack every tensor element that lies in them, verify them.
-        Returns the algorithmic bytes moved: pack reads the source elements and
-        writes the buckets, unpack reads and writes each element's two bytes,
-        verify reads the buckets."""
+        Returns the algorithmic bytes of that sync, counted as for the GPU path:
+        pack reads the source elements and writes the buckets; the receiver reads
+        each bucket byte once (unpack and verify) and writes each element's two
+        bytes."""
         packed, cs = self.pack(src, first, count)
         buckets = [None] * self.n_buckets
         for i in range(count):
@@ -317,13 +318,13 @@ class Layout:
                 self.unpack_elements(buckets, t, (a - t_lo) // 2, (z - t_lo) // 2)
                 es = self.params[blocks[0][0]][2]
                 moved += (z - a) // 2 * es      # pack: source bytes read
-                moved += 2 * (z - a)             # unpack: read + write
+                moved += z - a                   # unpack: tensor bytes written
         full_cs = np.zeros(self.n_buckets, np.uint64)
         full_cs[first:first + count] = cs
         n_bad, _ = self.verify(buckets, full_cs, first, count)
         if n_bad:
             raise RuntimeError("oracle verify failed on its own buckets")
-        moved += 2 * count * self.bucket_bytes   # pack writes + verify reads
+        moved += 2 * count * self.bucket_bytes   # pack writes, receiver reads
         return moved
 
     def verify(self, buckets, checksums, first: int = 0, count: Optional[int] = None):

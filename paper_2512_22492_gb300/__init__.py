@@ -8,10 +8,11 @@ a C-ABI CUDA library (``include/rr.h``, ``csrc/``) and its Python binding.
 """
 from .rr import (Block, DstLayout, DstTensor, Param, Plan, PlanOptions, RRError, SrcLayout,
                  rr_clear_range, rr_pack, rr_pack_range, rr_plan_create, rr_status_str, rr_unpack,
-                 rr_unpack_range, rr_verify, rr_verify_range)
+                 rr_unpack_range, rr_unpack_verify, rr_verify, rr_verify_range)
 from .layouts import qwen3_manifest, qwen3_rollout, qwen3_sync
 
 __all__ = ["Block", "DstLayout", "DstTensor", "Param", "Plan", "PlanOptions", "RRError",
            "SrcLayout", "rr_pack", "rr_plan_create", "rr_status_str", "rr_unpack", "rr_verify",
            "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
+           "rr_unpack_verify",
            "qwen3_manifest", "qwen3_rollout", "qwen3_sync"]

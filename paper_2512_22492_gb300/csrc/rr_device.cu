@@ -70,6 +70,14 @@ struct UnpackArgs {
     const uint32_t* block_first;   // as in PackArgs
     uint32_t item_begin;
     uint32_t item_end;
+    // Verifying unpack only (as in VerifyArgs): per-bucket sums of the range
+    // [first_bucket, first_bucket + n_buckets), counters, expected sums, flags.
+    unsigned long long* sums;
+    unsigned long long* counters;
+    const unsigned long long* expected;
+    uint8_t* bad;
+    int32_t first_bucket;
+    int32_t n_buckets;
     const char* bucket_base;
     uint64_t bucket_stride;
     int32_t dst_base;         // index in ptr[] of destination tensor 0
@@ -309,22 +317,61 @@ __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(c
 }
 
 // ---------------------------------------------------------------------------
+// Checksum comparison, run by whichever block finishes last (a ticket counter;
+// no block waits for another).  sums[i] belongs to bucket first + i.
+// ---------------------------------------------------------------------------
+
+__device__ void compare_in_last_block(unsigned long long* counters,
+                                      const unsigned long long* sums,
+                                      const unsigned long long* expected, uint8_t* bad,
+                                      int32_t first, int32_t n) {
+    __shared__ bool last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        last = atomicAdd(&counters[0], 1ull) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    for (int32_t i = threadIdx.x; i < n; i += kThreads) {
+        const int32_t b = first + i;
+        const bool differs = __ldcg(sums + i) != expected[b];
+        if (bad) bad[i] = differs ? 1 : 0;
+        if (differs) {
+            atomicAdd(&counters[1], 1ull);
+            atomicMax(&counters[2], ULLONG_MAX - (unsigned long long)b);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Unpack
 // ---------------------------------------------------------------------------
 
-template <int NPTR>
+// Copies each item's bytes from its bucket to its tensor.  With VERIFY it also
+// sums every bucket byte it reads (the gap READ items too) into the bucket's
+// checksum and compares at the end, so the buckets are read once for both.
+template <int NPTR, bool VERIFY>
 __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
+    constexpr int U = 2 * kUnroll;   // one 16-byte load per vector: twice the pack's depth
     uint32_t i0, i1;
     block_items(a.block_first, a.item_begin, a.item_end, &i0, &i1);
+    unsigned long long acc = 0;
+    uint32_t cur = 0xFFFFFFFFu;
     for (uint32_t it = i0; it < i1; ++it) {
         const rr_unpack_item d = a.items[it];
+        if (!VERIFY && d.kind >= RR_ITEM_READ_VEC) continue;
+        if (VERIFY && d.bucket != cur) {
+            if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - a.first_bucket), acc);
+            cur = d.bucket;
+            acc = 0;
+        }
         const char* src = (a.bucket_stride ? a.bucket_base + (uint64_t)d.bucket * a.bucket_stride
                                            : (const char*)a.ptr[d.bucket]) + d.src_off;
-        char* dst = (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off;
-        if (d.kind == RR_ITEM_COPY_VEC) {
-            // One 16-byte load per vector: twice the pack's depth keeps as many
-            // bytes in flight.
-            constexpr int U = 2 * kUnroll;
+        const bool copy = d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_COPY_SCALAR;
+        char* dst = copy ? (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off : nullptr;
+        if (d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_READ_VEC) {
             const uint32_t nvec = d.nbytes >> 4;
             for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * U) {
                 uint4 x[U];
@@ -332,13 +379,25 @@ __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_con
                 for (int u = 0; u < U; ++u)
                     if (v + u * kThreads < nvec) x[u] = ld_stream(src + 16ull * (v + u * kThreads));
 #pragma unroll
-                for (int u = 0; u < U; ++u)
-                    if (v + u * kThreads < nvec) st_stream(dst + 16ull * (v + u * kThreads), x[u]);
+                for (int u = 0; u < U; ++u) {
+                    if (v + u * kThreads < nvec) {
+                        if (copy) st_stream(dst + 16ull * (v + u * kThreads), x[u]);
+                        if (VERIFY) acc += words(x[u]);
+                    }
+                }
             }
         } else {
-            for (uint32_t e = threadIdx.x; e < (d.nbytes >> 1); e += kThreads)
-                *(uint16_t*)(dst + 2ull * e) = *(const uint16_t*)(src + 2ull * e);
+            for (uint32_t e = threadIdx.x; e < (d.nbytes >> 1); e += kThreads) {
+                const uint16_t h = *(const uint16_t*)(src + 2ull * e);
+                if (copy) *(uint16_t*)(dst + 2ull * e) = h;
+                if (VERIFY) acc += (unsigned long long)h << (8 * ((d.src_off + 2 * e) & 7));
+            }
         }
+    }
+    if (VERIFY) {
+        if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - a.first_bucket), acc);
+        compare_in_last_block(a.counters, a.sums, a.expected, a.bad, a.first_bucket,
+                              a.n_buckets);
     }
 }
 
@@ -379,25 +438,7 @@ __global__ void __launch_bounds__(kThreads, 4) rr_verify_kernel(const __grid_con
     }
     if (cur != 0xFFFFFFFFu) flush(a.sums + cur, acc);
 
-    // The last block to finish compares all sums (no block waits for another).
-    __shared__ bool last;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        last = atomicAdd(&a.counters[0], 1ull) == gridDim.x - 1;
-    }
-    __syncthreads();
-    if (!last) return;
-    __threadfence();
-    for (int32_t bl = threadIdx.x; bl < a.n_buckets; bl += kThreads) {
-        const int32_t b = a.first_bucket + bl;
-        const bool differs = __ldcg(a.sums + bl) != a.expected[b];
-        if (a.bad) a.bad[bl] = differs ? 1 : 0;
-        if (differs) {
-            atomicAdd(&a.counters[1], 1ull);
-            atomicMax(&a.counters[2], ULLONG_MAX - (unsigned long long)b);
-        }
-    }
+    compare_in_last_block(a.counters, a.sums, a.expected, a.bad, a.first_bucket, a.n_buckets);
 }
 
 // ---------------------------------------------------------------------------
@@ -478,15 +519,25 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
     return RR_OK;
 }
 
+// Verifying form when checksums != NULL (sums and counters in the plan's scratch).
 template <int NPTR>
 rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
-                        bool table, uint64_t stride, cudaStream_t s) {
+                        const uint64_t* checksums, uint8_t* bad, bool table, uint64_t stride,
+                        cudaStream_t s) {
     UnpackArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     a.items = P->d_unpack_items;
     a.block_first = R.full ? P->d_unpack_block_first : nullptr;
     a.item_begin = P->unpack_bucket_first[R.b0];
     a.item_end = P->unpack_bucket_first[R.b1];
+    if (checksums) {
+        a.sums = P->d_verify_scratch;
+        a.counters = P->d_verify_scratch + (R.b1 - R.b0);
+        a.expected = (const unsigned long long*)checksums;
+        a.bad = bad;
+        a.first_bucket = R.b0;
+        a.n_buckets = R.b1 - R.b0;
+    }
     int32_t k = 0;
     if (table) {
         for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[k++] = buckets[b];
@@ -496,7 +547,10 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     }
     a.dst_base = k;
     for (int32_t t = 0; t < P->n_tensors; ++t) a.ptr[k++] = dst[t];
-    rr_unpack_kernel<NPTR><<<P->unpack_grid_blocks, kThreads, 0, s>>>(a);
+    if (checksums)
+        rr_unpack_kernel<NPTR, true><<<P->unpack_grid_blocks, kThreads, 0, s>>>(a);
+    else
+        rr_unpack_kernel<NPTR, false><<<P->unpack_grid_blocks, kThreads, 0, s>>>(a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -559,24 +613,74 @@ rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, vo
                : launch_pack<kLargePtrs>(P, R, src_shards, buckets, checksums, table, stride, stream);
 }
 
-rr_status unpack_impl(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
-                      cudaStream_t stream) {
-    rr_status st;
-    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+rr_status check_dst(const rr_plan* P, void* const* dst) {
     if (P->n_tensors > 0 && !dst) return rr_fail(RR_EINVAL, "dst array is NULL");
     for (int32_t t = 0; t < P->n_tensors; ++t)
         if (P->tensor_numel[t] > 0 && !aligned16(dst[t]))
             return rr_fail(RR_EINVAL, "dst[%d] is NULL or not 16-byte aligned", t);
-    if (P->unpack_bucket_first[R.b0] == P->unpack_bucket_first[R.b1]) return RR_OK;
+    return RR_OK;
+}
+
+template <class F>
+rr_status with_unpack_shape(const rr_plan* P, const void* const* buckets, F launch) {
     uint64_t stride = 0;
     const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
     const int32_t need = P->n_tensors + (table ? P->n_buckets : 0);
-    if (need <= kSmallPtrs)
-        return launch_unpack<kSmallPtrs>(P, R, buckets, dst, table, stride, stream);
-    if (need <= kLargePtrs)
-        return launch_unpack<kLargePtrs>(P, R, buckets, dst, table, stride, stream);
-    return rr_fail(RR_EINVAL, "%d tensors + %d separately allocated buckets exceed %d pointers",
-                   P->n_tensors, P->n_buckets, kLargePtrs);
+    if (need > kLargePtrs)
+        return rr_fail(RR_EINVAL, "%d tensors + %d separately allocated buckets exceed %d pointers",
+                       P->n_tensors, P->n_buckets, kLargePtrs);
+    return launch(need <= kSmallPtrs, table, stride);
+}
+
+rr_status unpack_impl(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
+                      cudaStream_t stream) {
+    rr_status st;
+    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if ((st = check_dst(P, dst))) return st;
+    if (P->unpack_bucket_first[R.b0] == P->unpack_bucket_first[R.b1]) return RR_OK;
+    return with_unpack_shape(P, buckets, [&](bool small, bool table, uint64_t stride) {
+        return small ? launch_unpack<kSmallPtrs>(P, R, buckets, dst, nullptr, nullptr, table,
+                                                 stride, stream)
+                     : launch_unpack<kLargePtrs>(P, R, buckets, dst, nullptr, nullptr, table,
+                                                 stride, stream);
+    });
+}
+
+rr_status read_result(const rr_plan* P, int32_t n, int64_t* n_bad, int64_t* first_bad,
+                      cudaStream_t stream) {
+    RR_CUDA(cudaMemcpyAsync(P->h_verify_result, P->d_verify_scratch + n,
+                            4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, stream));
+    RR_CUDA(cudaStreamSynchronize(stream));
+    const unsigned long long nb = P->h_verify_result[1];
+    if (n_bad) *n_bad = (int64_t)nb;
+    if (first_bad) *first_bad = nb ? (int64_t)(ULLONG_MAX - P->h_verify_result[2]) : -1;
+    return nb ? RR_EMISMATCH : RR_OK;
+}
+
+rr_status unpack_verify_impl(const rr_plan* P, Range R, const void* const* buckets,
+                             const uint64_t* checksums, void* const* dst, uint8_t* bad,
+                             int64_t* n_bad, int64_t* first_bad, cudaStream_t stream) {
+    rr_status st;
+    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if ((st = check_dst(P, dst))) return st;
+    if (R.b1 > R.b0 && !aligned16(checksums))
+        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    if (n_bad) *n_bad = 0;
+    if (first_bad) *first_bad = -1;
+    if (R.b1 == R.b0) return RR_OK;
+    rr_plan* M = const_cast<rr_plan*>(P);   // the scratch area is the only mutable state
+    std::lock_guard<std::mutex> lock(M->verify_mutex);
+    const int32_t n = R.b1 - R.b0;
+    RR_CUDA(cudaMemsetAsync(P->d_verify_scratch, 0, (size_t(n) + 4) * sizeof(unsigned long long),
+                            stream));
+    st = with_unpack_shape(P, buckets, [&](bool small, bool table, uint64_t stride) {
+        return small ? launch_unpack<kSmallPtrs>(P, R, buckets, dst, checksums, bad, table, stride,
+                                                 stream)
+                     : launch_unpack<kLargePtrs>(P, R, buckets, dst, checksums, bad, table, stride,
+                                                 stream);
+    });
+    if (st) return st;
+    return read_result(P, n, n_bad, first_bad, stream);
 }
 
 rr_status verify_impl(const rr_plan* P, Range R, const void* const* buckets,
@@ -604,13 +708,7 @@ rr_status verify_impl(const rr_plan* P, Range R, const void* const* buckets,
              ? launch_verify<kSmallPtrs>(P, R, buckets, checksums, bad, table, stride, stream)
              : launch_verify<kLargePtrs>(P, R, buckets, checksums, bad, table, stride, stream);
     if (st) return st;
-    RR_CUDA(cudaMemcpyAsync(P->h_verify_result, P->d_verify_scratch + n,
-                            4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, stream));
-    RR_CUDA(cudaStreamSynchronize(stream));
-    const unsigned long long nb = P->h_verify_result[1];
-    if (n_bad) *n_bad = (int64_t)nb;
-    if (first_bad) *first_bad = nb ? (int64_t)(ULLONG_MAX - P->h_verify_result[2]) : -1;
-    return nb ? RR_EMISMATCH : RR_OK;
+    return read_result(P, n, n_bad, first_bad, stream);
 }
 
 }  // namespace
@@ -624,7 +722,7 @@ rr_status rr_device_default_grid(int32_t* pack, int32_t* unpack, int32_t* verify
     RR_CUDA(cudaGetDevice(&dev));
     RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs>, kThreads, 0));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, true>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, rr_verify_kernel<kLargePtrs>, kThreads, 0));
     *pack = sms * (p > 0 ? p : 1);
     *unpack = sms * (u > 0 ? u : 1);
@@ -737,6 +835,28 @@ extern "C" rr_status rr_verify_range(const rr_plan* P, int32_t first_bucket, int
     rr_status st = check_plan(P);
     if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
     return verify_impl(P, R, buckets, checksums, bad, n_bad, first_bad, stream);
+}
+
+extern "C" rr_status rr_unpack_verify(const rr_plan* P, const void* const* buckets,
+                                      const uint64_t* checksums, void* const* dst, uint8_t* bad,
+                                      int64_t* n_bad, int64_t* first_bad, cudaStream_t stream) {
+    rr_clear_error();
+    rr_status st = check_plan(P);
+    if (st) return st;
+    return unpack_verify_impl(P, Range{0, P->n_buckets, true}, buckets, checksums, dst, bad, n_bad,
+                              first_bad, stream);
+}
+
+extern "C" rr_status rr_unpack_verify_range(const rr_plan* P, int32_t first_bucket,
+                                            int32_t n_buckets, const void* const* buckets,
+                                            const uint64_t* checksums, void* const* dst,
+                                            uint8_t* bad, int64_t* n_bad, int64_t* first_bad,
+                                            cudaStream_t stream) {
+    rr_clear_error();
+    Range R;
+    rr_status st = check_plan(P);
+    if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
+    return unpack_verify_impl(P, R, buckets, checksums, dst, bad, n_bad, first_bad, stream);
 }
 
 extern "C" rr_status rr_clear_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,

@@ -103,6 +103,36 @@ public:
         }
     }
 
+    // Stream bytes [a, b) of rank `rank` that belong to no tensor: read (and
+    // checksummed) only by the verifying unpack.
+    void read_gap(int32_t rank, int64_t a, int64_t b) {
+        const int64_t B = P->bucket_bytes;
+        const int64_t fb = P->rank_first_bucket[rank];
+        while (a < b) {
+            const int64_t bl = a / B;
+            int64_t boff = a - bl * B;
+            int64_t len = std::min({b - a, B - boff, P->chunk_bytes});
+            int64_t h = std::min((16 - boff % 16) % 16, len);
+            if (h) {
+                emit_copy(RR_ITEM_READ_SCALAR, fb + bl, boff, -1, 0, h);
+                boff += h;
+                a += h;
+                len -= h;
+            }
+            const int64_t body = len / 16 * 16;
+            if (body) {
+                emit_copy(RR_ITEM_READ_VEC, fb + bl, boff, -1, 0, body);
+                boff += body;
+                a += body;
+                len -= body;
+            }
+            if (len) {
+                emit_copy(RR_ITEM_READ_SCALAR, fb + bl, boff, -1, 0, len);
+                a += len;
+            }
+        }
+    }
+
     int64_t pack_read = 0;
 
 private:
@@ -211,7 +241,11 @@ int64_t pack_weight(const rr_pack_item& it) {
 }
 
 int64_t unpack_weight(const rr_unpack_item& it) {
-    return (it.kind == RR_ITEM_COPY_VEC ? 2 : 4) * int64_t(it.nbytes) + kItemOverhead;
+    switch (it.kind) {
+        case RR_ITEM_COPY_VEC: return 2 * int64_t(it.nbytes) + kItemOverhead;
+        case RR_ITEM_COPY_SCALAR: return 4 * int64_t(it.nbytes) + kItemOverhead;
+        default: return int64_t(it.nbytes) + kItemOverhead;
+    }
 }
 
 // Cuts items [0, n) into `grid` contiguous ranges of roughly equal weight.
@@ -369,8 +403,14 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
         }
         const int64_t nb = P->rank_first_bucket[r + 1] - P->rank_first_bucket[r];
         b.zero_range(r, cursor, nb * P->bucket_bytes);
-        for (int32_t t = 0; t < P->n_tensors; ++t)
-            if (P->tensor_rank[t] == r) b.unpack_tensor(t);
+        cursor = 0;
+        for (int32_t t = 0; t < P->n_tensors; ++t) {
+            if (P->tensor_rank[t] != r) continue;
+            b.read_gap(r, cursor, P->tensor_off[t]);
+            b.unpack_tensor(t);
+            cursor = P->tensor_off[t] + 2 * P->tensor_numel[t];
+        }
+        b.read_gap(r, cursor, nb * P->bucket_bytes);
     }
     // Both tables are sorted by bucket: index their per-bucket item ranges.
     auto index = [&](auto& items, std::vector<uint32_t>& first) {

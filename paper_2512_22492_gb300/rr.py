@@ -136,6 +136,9 @@ _sig("rr_unpack_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp
                          ctypes.POINTER(_vp), _vp])
 _sig("rr_verify_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp, _vp, _P64,
                          _P64, _vp])
+_sig("rr_unpack_verify", [_vp, ctypes.POINTER(_vp), _vp, ctypes.POINTER(_vp), _vp, _P64, _P64, _vp])
+_sig("rr_unpack_verify_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp,
+                                ctypes.POINTER(_vp), _vp, _P64, _P64, _vp])
 _sig("rr_clear_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp])
 _sig("rr_plan_bucket_items", [_vp, ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_uint32)])
 _sig("rr_verify_noalloc", [ctypes.POINTER(_vp), ctypes.c_int32, ctypes.c_size_t, _vp, _P64, _P64,
@@ -148,6 +151,7 @@ EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_q
             "rr_plan_source", "rr_plan_tensors", "rr_plan_get_stats", "rr_plan_export_pack",
             "rr_plan_export_unpack", "rr_plan_bucket_items", "rr_pack", "rr_unpack", "rr_verify",
             "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
+            "rr_unpack_verify", "rr_unpack_verify_range",
             "rr_verify_noalloc",
             "rr_status_str", "rr_last_error")
 
@@ -497,6 +501,32 @@ def rr_verify_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, chec
                               ctypes.byref(n_bad), ctypes.byref(first), _stream(stream))
     if st not in (RR_OK, RR_EMISMATCH):
         _check(st, "rr_verify_range")
+    return n_bad.value, first.value
+
+
+def rr_unpack_verify(plan: Plan, buckets, checksums, dst, bad=None, stream=None,
+                     first_bucket: int = 0, n_buckets: Optional[int] = None):
+    """Unpack and verify in one pass over the buckets (optionally a bucket range).
+    Returns (n_bad, first_bad).  Synchronous."""
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst")
+    _check_checksums(plan, checksums)
+    n = plan.n_buckets - first_bucket if n_buckets is None else n_buckets
+    if bad is not None and _nbytes(bad) is not None and _nbytes(bad) < n:
+        raise ValueError(f"bad: {_nbytes(bad)} bytes, need {n}")
+    n_bad = ctypes.c_int64()
+    first = ctypes.c_int64()
+    badp = None if bad is None else _ptr(bad)
+    if first_bucket == 0 and n_buckets is None:
+        st = _lib.rr_unpack_verify(plan.handle, _ptr_array(buckets), _ptr(checksums),
+                                   _ptr_array(dst), badp, ctypes.byref(n_bad), ctypes.byref(first),
+                                   _stream(stream))
+    else:
+        st = _lib.rr_unpack_verify_range(plan.handle, first_bucket, n, _ptr_array(buckets),
+                                         _ptr(checksums), _ptr_array(dst), badp,
+                                         ctypes.byref(n_bad), ctypes.byref(first), _stream(stream))
+    if st not in (RR_OK, RR_EMISMATCH):
+        _check(st, "rr_unpack_verify")
     return n_bad.value, first.value
 
 

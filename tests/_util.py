@@ -13,7 +13,7 @@ import oracle
 import synth
 
 ITEM_F32_VEC, ITEM_F32_SCALAR, ITEM_BF16_VEC, ITEM_BF16_SCALAR, ITEM_ZERO_VEC, \
-    ITEM_ZERO_SCALAR, ITEM_COPY_VEC, ITEM_COPY_SCALAR = range(8)
+    ITEM_ZERO_SCALAR, ITEM_COPY_VEC, ITEM_COPY_SCALAR, ITEM_READ_VEC, ITEM_READ_SCALAR = range(10)
 
 
 def workload(name):
@@ -129,18 +129,30 @@ def check_and_run_pack(items, shards, n_buckets, bucket_bytes, shard_bytes):
 
 
 def check_and_run_unpack(items, buckets, tensor_numel):
+    """Applies unpack items; asserts their preconditions, that every tensor byte
+    is written once, and that copy + read items together read every bucket byte
+    exactly once (what the verifying unpack relies on)."""
     dst = [np.zeros(2 * n, np.uint8) for n in tensor_numel]
     hits = [np.zeros(2 * n, np.uint16) for n in tensor_numel]
+    reads = np.zeros(buckets.shape, np.uint16)
     for it in items:
         kind, b, so = int(it["kind"]), int(it["bucket"]), int(it["src_off"])
         t, do, nb = int(it["tensor"]), int(it["dst_off"]), int(it["nbytes"])
-        assert nb % 2 == 0 and so + nb <= buckets.shape[1] and do + nb <= dst[t].size
+        assert nb % 2 == 0 and so + nb <= buckets.shape[1]
+        if kind in (ITEM_COPY_VEC, ITEM_READ_VEC):
+            assert so % 16 == 0 and nb % 16 == 0
+        reads[b, so:so + nb] += 1
+        if kind in (ITEM_READ_VEC, ITEM_READ_SCALAR):
+            continue
+        assert do + nb <= dst[t].size
         if kind == ITEM_COPY_VEC:
-            assert so % 16 == 0 and do % 16 == 0 and nb % 16 == 0
+            assert do % 16 == 0
         dst[t][do:do + nb] = buckets[b, so:so + nb]
         hits[t][do:do + nb] += 1
     for h in hits:
         assert h.size == 0 or (h.min() == 1 and h.max() == 1), "dst bytes not written once"
+    assert reads.size == 0 or (reads.min() == 1 and reads.max() == 1), \
+        "bucket bytes not read exactly once by the unpack table"
     return [d.view("<u2") for d in dst]
 
 

@@ -205,3 +205,56 @@ def test_full_size_range_pack_of_one_rank():
     gen = oracle.Source(seed=w.seed, specials=w.specials)
     want, want_cs = L.pack(gen, first=fr[2] + 3, count=1)
     np.testing.assert_array_equal(H.buckets_host(buf, [fr[2] + 3])[0], want[0])
+
+
+@pytest.mark.parametrize("name,separate", [("tiny-tp4", False), ("tiny-moe-f32", True),
+                                           ("tiny", False)])
+def test_unpack_verify_equals_unpack_then_verify(name, separate):
+    desc, L, plan, buf, shards = setup(name, separate_buckets=separate)
+    H.pack(buf)
+    H.unpack(buf)
+    torch.cuda.synchronize()
+    want = [t.clone() for t in buf.dst]
+    for t in buf.dst:
+        t.fill_(0x5A5A)
+    assert rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst) == (0, -1)
+    torch.cuda.synchronize()
+    for t in range(plan.n_tensors):
+        assert torch.equal(buf.dst[t], want[t])
+    # Damage: a byte inside a tensor, and a byte in an alignment gap or tail
+    # (which no tensor holds, so only the checksum can notice it).
+    bl = H.bucket_list(buf)
+    items, _ = plan.export_unpack()
+    gaps = items[items["kind"] >= U.ITEM_READ_VEC]
+    g = gaps[len(gaps) // 2]
+    bl[int(g["bucket"])][int(g["src_off"])] ^= 0x01
+    bl[2][333] ^= 0x10
+    hit = sorted({2, int(g["bucket"])})
+    bad = torch.zeros(plan.n_buckets, dtype=torch.uint8, device="cuda")
+    got = rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst, bad)
+    assert got == rr.rr_verify(plan, buf.buckets, buf.checksums) == (len(hit), hit[0])
+    assert list(np.flatnonzero(bad.cpu().numpy())) == hit
+    # Range form over the second half only.
+    h = plan.n_buckets // 2
+    got = rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst, first_bucket=h,
+                              n_buckets=plan.n_buckets - h)
+    assert got == rr.rr_verify_range(plan, h, plan.n_buckets - h, buf.buckets, buf.checksums)
+
+
+def test_unpack_verify_full_size():
+    w = U.workload("qwen3-30b-a3b")
+    desc = U.workload_desc("qwen3-30b-a3b")
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, w.bucket_bytes)
+    buf = H.alloc(plan, poison=None)
+    H.fill_with_generator(buf, m, w.seed, w.specials)
+    H.pack(buf)
+    assert rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst) == (0, -1)
+    B = plan.bucket_bytes
+    store = buf.bucket_store.view(-1)
+    for t in range(plan.n_tensors):
+        start = plan.first_bucket_of_rank[plan.tensor_ranks[t]] * B + plan.tensor_stream_offset[t]
+        n = plan.tensor_numel[t]
+        assert torch.equal(buf.dst[t][:n], store[start:start + 2 * n].view(torch.int16))
+    buf.bucket_store[100, 12345] ^= 1
+    assert rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst) == (1, 100)
