@@ -87,13 +87,30 @@ typedef struct {
     rr_dtype dtype;     /* dtype of the trainer's copy: RR_F32 or RR_BF16          */
 } rr_param;
 
-/* Trainer side: flat FSDP-style shards. */
+/* How the trainer's parameters are cut into shards.
+ *  RR_SHARD_FLAT: one flat buffer cut into equal shards (FSDP1 FlatParameter),
+ *                 as defined at the top of this file.
+ *  RR_SHARD_ROWS: every parameter is cut on dim 0 separately (FSDP2 Shard(0),
+ *                 torch.chunk rule): with c = ceil(rows / n_shards), shard s
+ *                 holds rows [s*c, min((s+1)*c, rows)), padded to c rows.
+ *                 Within each shard the parameters' chunks follow one another
+ *                 in manifest order, each starting at a multiple of
+ *                 max(align_bytes, element size); all shards share that local
+ *                 layout and are S = (end of the last chunk rounded up to 16)
+ *                 bytes.  Padding rows are never read. */
+typedef enum { RR_SHARD_FLAT = 0, RR_SHARD_ROWS = 1 } rr_sharding;
+
+/* Trainer side. */
 typedef struct {
     int32_t n_shards;                 /* 1..65535                                      */
     int64_t align_bytes;              /* parameter start alignment, >= 1 (16 typical)  */
-    const int64_t* param_flat_offset; /* optional [n_params] explicit flat byte
-                                         offsets (each a multiple of the element size,
-                                         non-overlapping); NULL = computed as above    */
+    const int64_t* param_flat_offset; /* FLAT only, optional: [n_params] explicit flat
+                                         byte offsets (each a multiple of the element
+                                         size, non-overlapping); NULL = computed      */
+    int32_t sharding;                 /* rr_sharding; 0 = RR_SHARD_FLAT                */
+    int64_t shard_bytes;              /* FLAT only, optional: shard size S, a multiple
+                                         of 16 with n_shards * S covering every
+                                         parameter; 0 = computed                      */
 } rr_src_layout;
 
 /* A 2-D block of a parameter's matrix view. */
@@ -145,8 +162,9 @@ void rr_plan_destroy(rr_plan* plan);
 rr_status rr_plan_query(const rr_plan* plan, int32_t* n_buckets, int64_t* stream_bytes_per_rank,
                         int32_t* first_bucket_of_rank);
 
-/* Source geometry: shard size S, end of the last parameter, per-parameter flat
- * offsets ([n_params]).  Any output pointer may be NULL. */
+/* Source geometry: shard size S, end of the last parameter, and per-parameter
+ * byte offsets ([n_params]): flat offsets for RR_SHARD_FLAT, offsets within
+ * each shard for RR_SHARD_ROWS.  Any output pointer may be NULL. */
 rr_status rr_plan_source(const rr_plan* plan, int64_t* shard_bytes, int64_t* flat_bytes,
                          int64_t* param_flat_offset);
 

@@ -62,7 +62,10 @@ class _Layout(ctypes.Structure):
                 ("bucket_bytes", ctypes.c_int64),
                 ("param_offset", _P64), ("tensor_numel", _P64), ("tensor_offset", _P64),
                 ("rank_stream_bytes", _P64), ("rank_first_bucket", _P64),
-                ("flat_bytes", ctypes.c_int64), ("shard_bytes", ctypes.c_int64)]
+                ("flat_bytes", ctypes.c_int64), ("shard_bytes", ctypes.c_int64),
+                ("sharding", ctypes.c_int32), ("pad_", ctypes.c_int32),
+                ("shard_bytes_in", ctypes.c_int64), ("explicit_offset", _P64),
+                ("chunk_rows", _P64), ("param_gen_base", _P64)]
 
 
 _VALUE_FN = ctypes.CFUNCTYPE(ctypes.c_uint32, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32)
@@ -170,7 +173,9 @@ class Layout:
     """
 
     def __init__(self, params, tensors, n_shards: int, tp: int, bucket_bytes: int,
-                 align_bytes: int = 16, tensor_align: int = 256):
+                 align_bytes: int = 16, tensor_align: int = 256, sharding: str = "flat",
+                 explicit_offsets=None, shard_bytes: int = 0):
+        self.sharding = sharding
         self.params = list(params)
         self.tensors = list(tensors)
         self.n_shards, self.tp, self.bucket_bytes = n_shards, tp, bucket_bytes
@@ -196,6 +201,8 @@ class Layout:
         self.tensor_offset = np.zeros(max(1, len(self.tensors)), np.int64)
         self.rank_stream_bytes = np.zeros(tp, np.int64)
         self.rank_first_bucket = np.zeros(tp + 1, np.int64)
+        self.chunk_rows = np.zeros(max(1, len(self.params)), np.int64)
+        self.param_gen_base = np.zeros(max(1, len(self.params)), np.int64)
         L = _Layout()
         L.n_params, L.n_shards = len(self.params), n_shards
         L.params = ctypes.cast(cp, ctypes.POINTER(_Param))
@@ -204,11 +211,19 @@ class Layout:
         L.tensors = ctypes.cast(ct, ctypes.POINTER(_Tensor))
         L.tensor_align, L.bucket_bytes = tensor_align, bucket_bytes
         for name in ("param_offset", "tensor_numel", "tensor_offset", "rank_stream_bytes",
-                     "rank_first_bucket"):
+                     "rank_first_bucket", "chunk_rows", "param_gen_base"):
             setattr(L, name, getattr(self, name).ctypes.data_as(_P64))
+        L.sharding = {"flat": 0, "rows": 1}[sharding]
+        L.shard_bytes_in = shard_bytes
+        self._explicit = None
+        if explicit_offsets is not None:
+            self._explicit = np.ascontiguousarray(explicit_offsets, dtype=np.int64)
+            L.explicit_offset = self._explicit.ctypes.data_as(_P64)
         _check(lib().orc_layout_compute(ctypes.byref(L)), "layout")
         self.c = L
         self.param_offset = self.param_offset[:len(self.params)]
+        self.chunk_rows = self.chunk_rows[:len(self.params)]
+        self.param_gen_base = self.param_gen_base[:len(self.params)]
         self.tensor_numel = self.tensor_numel[:len(self.tensors)]
         self.tensor_offset = self.tensor_offset[:len(self.tensors)]
         self.flat_bytes = int(L.flat_bytes)
@@ -221,16 +236,29 @@ class Layout:
         return rows * cols
 
     def host_shards(self, seed: int, specials: bool = False) -> List[np.ndarray]:
-        """Materialise the flat source with the seeded generator and cut it into shards."""
+        """Materialise the source with the seeded generator and cut it into shards."""
         import synth
         flat = np.zeros(self.shard_bytes * self.n_shards, np.uint8)
+        S = self.shard_bytes
         for p, (_, _, es) in enumerate(self.params):
-            n = self.param_numel(p)
+            rows, cols = self.views[p]
+            base = int(self.param_gen_base[p])
             off = int(self.param_offset[p])
-            vals = synth.values_host(n, es, seed, first_idx=off // es, specials=specials)
-            flat[off:off + n * es] = vals.view(np.uint8)
-        return [flat[s * self.shard_bytes:(s + 1) * self.shard_bytes]
-                for s in range(self.n_shards)]
+            if self.sharding == "flat":
+                n = rows * cols
+                vals = synth.values_host(n, es, seed, first_idx=base, specials=specials)
+                flat[off:off + n * es] = vals.view(np.uint8)
+                continue
+            c = int(self.chunk_rows[p])
+            for s in range(self.n_shards):
+                r0, r1 = s * c, min((s + 1) * c, rows)
+                if r1 <= r0:
+                    continue
+                n = (r1 - r0) * cols
+                vals = synth.values_host(n, es, seed, first_idx=base + r0 * cols,
+                                         specials=specials)
+                flat[s * S + off:s * S + off + n * es] = vals.view(np.uint8)
+        return [flat[s * S:(s + 1) * S] for s in range(self.n_shards)]
 
     # -- reshard / pack -------------------------------------------------------
     def reshard_tensor(self, src: Source, t: int) -> np.ndarray:
@@ -351,4 +379,4 @@ def workload_layout(w, bucket_bytes: Optional[int] = None) -> Layout:
     params = qwen3.manifest(w.shape, w.src_elem_bytes)
     tensors = qwen3.rollout_tensors(w.shape, params, w.tp)
     return Layout(params, tensors, n_shards=w.n_shards, tp=w.tp,
-                  bucket_bytes=bucket_bytes or w.bucket_bytes)
+                  bucket_bytes=bucket_bytes or w.bucket_bytes, sharding=w.sharding)

@@ -19,7 +19,9 @@ output dimension.  Under TP = t, rank r takes the r-th of t equal row ranges
 of the column-parallel weights (q, k, v, gate, up, embedding, lm_head, each
 expert's gate/up) and the r-th of t equal column ranges of the row-parallel
 weights (o_proj, down_proj, each expert's down_proj); norms and the router
-are replicated on every rank.
+are replicated on every rank.  When TP exceeds the number of KV heads, each
+KV head is replicated instead: rank r takes the rows of head r * n_kv // t of
+k and of v (t / n_kv ranks per head).
 
 A block is (param index, row0, nrows, col0, ncols) on the parameter's
 [rows = d0, cols = d1 * d2 * ...] view.
@@ -96,6 +98,15 @@ def rollout_tensors(shape, params: List[Param], tp: int) -> List[Tensor]:
         n = rows // tp
         return (index[name], r * n, n, 0, cols)
 
+    def kv_slice(name, r) -> Block:
+        # TP <= n_kv: a row range of whole heads; TP > n_kv: one replicated head.
+        if tp <= shape.n_kv:
+            return row_slice(name, r)
+        assert tp % shape.n_kv == 0, f"TP={tp} is not a multiple of {shape.n_kv} KV heads"
+        rows, cols = view[name]
+        h = r * shape.n_kv // tp
+        return (index[name], h * shape.head_dim, shape.head_dim, 0, cols)
+
     def col_slice(name, r) -> Block:
         rows, cols = view[name]
         assert cols % tp == 0, f"{name}: {cols} columns do not split over TP={tp}"
@@ -110,8 +121,8 @@ def rollout_tensors(shape, params: List[Param], tp: int) -> List[Tensor]:
             a = pre + "self_attn."
             tensors += [
                 (f"layers.{i}.qkv_proj", r, [row_slice(a + "q_proj.weight", r),
-                                              row_slice(a + "k_proj.weight", r),
-                                              row_slice(a + "v_proj.weight", r)]),
+                                              kv_slice(a + "k_proj.weight", r),
+                                              kv_slice(a + "v_proj.weight", r)]),
                 (f"layers.{i}.o_proj", r, [col_slice(a + "o_proj.weight", r)]),
                 (f"layers.{i}.q_norm", r, [whole(a + "q_norm.weight")]),
                 (f"layers.{i}.k_norm", r, [whole(a + "k_norm.weight")]),

@@ -24,12 +24,25 @@
  * The paper prints no layout, byte format or checksum; the definitions below
  * are the readings this build takes, stated once here:
  *
- *  Source.  Parameters are concatenated in manifest order into one flat byte
- *  buffer; each starts at a multiple of max(align_bytes, element size); gap
- *  bytes are zero.  The total is padded up to a multiple of 16 * n_shards and
- *  cut into n_shards equal shards of S bytes: flat byte f lives in shard f / S
- *  at offset f % S.  A parameter of shape [d0, d1, ...] is viewed as a matrix
- *  [rows = d0, cols = d1 * d2 * ...] (cols = 1 for a vector).
+ *  Source, flat sharding (FSDP1-style).  Parameters are concatenated in
+ *  manifest order into one flat byte buffer; each starts at a multiple of
+ *  max(align_bytes, element size) (or at explicitly given offsets); gap bytes
+ *  are zero.  The total is padded up to a multiple of 16 * n_shards (or a
+ *  shard size S is given) and cut into n_shards equal shards of S bytes: flat
+ *  byte f lives in shard f / S at offset f % S.
+ *
+ *  Source, row sharding (FSDP2 Shard(0), the torch.chunk rule).  Each
+ *  parameter is cut on its first dimension: with c = ceil(rows / n_shards),
+ *  shard s holds rows [s*c, min((s+1)*c, rows)) padded to c rows.  In every
+ *  shard the parameters' chunks follow one another in manifest order, each
+ *  starting at a multiple of max(align_bytes, element size); S is the end of
+ *  the last chunk rounded up to 16.  Row r, column k of parameter p is in
+ *  shard r / c at offset off_p + ((r - s*c) * cols + k) * element size.
+ *
+ *  A parameter of shape [d0, d1, ...] is viewed as a matrix [rows = d0,
+ *  cols = d1 * d2 * ...] (cols = 1 for a vector).  Generated values are
+ *  indexed by the element's position in the flat layout whatever the
+ *  sharding, so one seed gives the same parameters under every sharding.
  *
  *  Destination.  A destination tensor is a list of blocks (param, row0, nrows,
  *  col0, ncols); its elements are the blocks' elements taken block by block,
@@ -91,8 +104,17 @@ typedef struct {
     int64_t* tensor_offset;     /* [n_tensors] byte offset in its rank's stream     */
     int64_t* rank_stream_bytes; /* [tp]                                             */
     int64_t* rank_first_bucket; /* [tp + 1]; rank_first_bucket[tp] = bucket count   */
-    int64_t flat_bytes;         /* end of the last parameter                        */
+    int64_t flat_bytes;         /* end of the last parameter (row sharding: of the
+                                   last chunk within a shard)                      */
     int64_t shard_bytes;        /* S                                                */
+    /* description, continued */
+    int32_t sharding;           /* 0: flat, 1: rows                                 */
+    int32_t pad_;
+    int64_t shard_bytes_in;     /* flat: explicit S, or 0                           */
+    const int64_t* explicit_offset; /* flat: explicit offsets, or NULL              */
+    /* derived, continued */
+    int64_t* chunk_rows;        /* [n_params] rows: c per parameter                 */
+    int64_t* param_gen_base;    /* [n_params] flat element index of element 0       */
 } orc_layout;
 
 /* Where source values come from: real shard buffers, or a generator that maps
@@ -117,19 +139,52 @@ int orc_layout_compute(orc_layout* L) {
         L->bucket_bytes < 8 || L->bucket_bytes % 8 != 0)
         return ORC_EINVAL;
 
-    /* Source: parameters one after another, each aligned. */
-    int64_t off = 0;
+    /* Source, flat layout first: parameters one after another, each aligned
+     * (or at the given offsets).  Generated values are indexed by it. */
+    int64_t off = 0, flat_end = 0;
     for (int32_t p = 0; p < L->n_params; ++p) {
         const orc_param* P = &L->params[p];
         if (P->rows < 0 || P->cols < 0 || (P->elem_bytes != 2 && P->elem_bytes != 4))
             return ORC_EINVAL;
         int64_t a = L->align_bytes > P->elem_bytes ? L->align_bytes : P->elem_bytes;
-        off = align_up(off, a);
-        L->param_offset[p] = off;
-        off += P->rows * P->cols * P->elem_bytes;
+        int64_t start;
+        if (L->explicit_offset) {
+            start = L->explicit_offset[p];
+            if (start < 0 || start % P->elem_bytes != 0) return ORC_EINVAL;
+        } else {
+            off = align_up(off, a);
+            start = off;
+            off += P->rows * P->cols * P->elem_bytes;
+        }
+        L->param_offset[p] = start;
+        L->param_gen_base[p] = start / P->elem_bytes;
+        int64_t end = start + P->rows * P->cols * P->elem_bytes;
+        if (end > flat_end) flat_end = end;
     }
-    L->flat_bytes = off;
-    L->shard_bytes = align_up(off, 16 * (int64_t)L->n_shards) / L->n_shards;
+    if (L->sharding == 0) {
+        L->flat_bytes = flat_end;
+        L->shard_bytes = align_up(flat_end, 16 * (int64_t)L->n_shards) / L->n_shards;
+        if (L->shard_bytes_in) {
+            if (L->shard_bytes_in % 16 != 0 || L->shard_bytes_in * L->n_shards < flat_end)
+                return ORC_EINVAL;
+            L->shard_bytes = L->shard_bytes_in;
+        }
+    } else {
+        /* Row sharding: every shard holds each parameter's chunk of c rows. */
+        if (L->explicit_offset || L->shard_bytes_in) return ORC_EINVAL;
+        int64_t local = 0;
+        for (int32_t p = 0; p < L->n_params; ++p) {
+            const orc_param* P = &L->params[p];
+            int64_t c = (P->rows + L->n_shards - 1) / L->n_shards;
+            int64_t a = L->align_bytes > P->elem_bytes ? L->align_bytes : P->elem_bytes;
+            local = align_up(local, a);
+            L->chunk_rows[p] = c;
+            L->param_offset[p] = local;
+            local += c * P->cols * P->elem_bytes;
+        }
+        L->flat_bytes = local;
+        L->shard_bytes = align_up(local, 16);
+    }
 
     /* Destination: per-rank streams. */
     for (int32_t r = 0; r < L->tp; ++r) L->rank_stream_bytes[r] = 0;
@@ -182,19 +237,30 @@ static int source_byte(const orc_layout* L, const orc_source* S, int64_t f, uint
     return ORC_OK;
 }
 
-/* Bits of the element at flat byte offset f (little-endian). */
-static int source_bits(const orc_layout* L, const orc_source* S, int64_t f, int32_t es,
+/* Bits of element e (row-major) of parameter p (little-endian). */
+static int source_bits(const orc_layout* L, const orc_source* S, int32_t p, int64_t e,
                        uint32_t* bits) {
+    const orc_param* P = &L->params[p];
+    const int32_t es = P->elem_bytes;
     if (S->shards == NULL) {
-        *bits = S->gen(S->gen_ctx, f / es, es);
+        *bits = S->gen(S->gen_ctx, L->param_gen_base[p] + e, es);
         return ORC_OK;
     }
     uint32_t v = 0;
-    for (int32_t i = 0; i < es; ++i) {
-        uint8_t byte;
-        int rc = source_byte(L, S, f + i, &byte);
-        if (rc) return rc;
-        v |= (uint32_t)byte << (8 * i);
+    if (L->sharding == 0) {
+        int64_t f = L->param_offset[p] + e * es;
+        for (int32_t i = 0; i < es; ++i) {
+            uint8_t byte;
+            int rc = source_byte(L, S, f + i, &byte);
+            if (rc) return rc;
+            v |= (uint32_t)byte << (8 * i);
+        }
+    } else {
+        int64_t row = e / P->cols;
+        int64_t s = row / L->chunk_rows[p];
+        int64_t o = L->param_offset[p] + (e - s * L->chunk_rows[p] * P->cols) * es;
+        if (s >= L->n_shards || S->shards[s] == NULL) return ORC_ESOURCE;
+        for (int32_t i = 0; i < es; ++i) v |= (uint32_t)S->shards[s][o + i] << (8 * i);
     }
     *bits = v;
     return ORC_OK;
@@ -217,9 +283,8 @@ int orc_tensor_elements(const orc_layout* L, const orc_source* S, int32_t t, int
             int64_t jj = j - base;
             int64_t row = B->row0 + jj / B->ncols;
             int64_t col = B->col0 + jj % B->ncols;
-            int64_t f = L->param_offset[B->param] + (row * P->cols + col) * P->elem_bytes;
             uint32_t bits;
-            int rc = source_bits(L, S, f, P->elem_bytes, &bits);
+            int rc = source_bits(L, S, B->param, row * P->cols + col, &bits);
             if (rc) return rc;
             out[j - j0] = cast_to_bf16(bits, P->elem_bytes);
         }

@@ -37,6 +37,24 @@ public:
 
     // ---- pack ------------------------------------------------------------
 
+    // Where element e of parameter p lives: shard, byte offset in it, and how
+    // many bytes from there on stay contiguous in that shard and in p.
+    struct Loc {
+        int64_t shard, off, room;
+    };
+    Loc loc(int32_t p, int64_t e) const {
+        const int32_t es = P->es[p];
+        if (P->sharding == RR_SHARD_FLAT) {
+            const int64_t S = P->shard_bytes;
+            const int64_t f = P->param_off[p] + e * es;
+            return {f / S, f % S, S - f % S};
+        }
+        const int64_t cols = P->cols[p], c = P->chunk_rows[p];
+        const int64_t sh = e / cols / c;
+        const int64_t end = std::min((sh + 1) * c, P->rows[p]) * cols;   // p's last element in sh
+        return {sh, P->param_off[p] + (e - sh * c * cols) * es, (end - e) * es};
+    }
+
     // Emits the items of one strided run of parameter p: n rows of l elements,
     // row i starting at parameter element first + i * st, landing contiguously
     // in rank `rank`'s stream at byte `pos0`.
@@ -44,19 +62,19 @@ public:
                   int64_t pos0) {
         if (l == 0 || n == 0) return;
         const int32_t es = P->es[p];
-        const int64_t S = P->shard_bytes, B = P->bucket_bytes;
+        const int64_t B = P->bucket_bytes;
         const int64_t fb = P->rank_first_bucket[rank];
         int64_t i = 0, c = 0;
         while (i < n) {
             const int64_t pos = pos0 + 2 * (i * l + c);
             const int64_t bl = pos / B, boff = pos - bl * B;
             const int64_t brem = (B - boff) / 2;                      // elements left in bucket
-            const int64_t f = P->param_off[p] + (first + i * st + c) * es;
-            const int64_t sh = f / S, soff = f - sh * S;
-            const int64_t srem = (S - soff) / es;                     // elements left in shard
+            const Loc at = loc(p, first + i * st + c);
+            const int64_t sh = at.shard, soff = at.off;
+            const int64_t srem = at.room / es;                        // elements left in shard
             if (c == 0 && n - i > 1 && l <= chunk_elems) {
                 int64_t k = std::min({n - i, chunk_elems / l, brem / l});
-                const int64_t room = S - soff;
+                const int64_t room = at.room;
                 const int64_t kshard = room >= l * es ? (room - l * es) / (st * es) + 1 : 0;
                 k = std::min(k, kshard);
                 if (k >= 2) {
@@ -301,7 +319,24 @@ rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_
 
     // Source offsets.
     int64_t end = 0;
-    if (src->param_flat_offset) {
+    if (src->sharding != RR_SHARD_FLAT && src->sharding != RR_SHARD_ROWS)
+        return rr_fail(RR_EINVAL, "unknown sharding %d", src->sharding);
+    P->sharding = src->sharding;
+    if (src->sharding == RR_SHARD_ROWS) {
+        if (src->param_flat_offset || src->shard_bytes)
+            return rr_fail(RR_EINVAL, "row sharding takes no explicit offsets or shard size");
+        P->chunk_rows.resize(n_params);
+        for (int32_t p = 0; p < n_params; ++p) {
+            const int64_t c = (P->rows[p] + src->n_shards - 1) / src->n_shards;
+            P->chunk_rows[p] = c;
+            end = align_up(end, std::max<int64_t>(src->align_bytes, P->es[p]));
+            P->param_off[p] = end;
+            end += c * P->cols[p] * P->es[p];
+        }
+        P->flat_bytes = end;
+        P->n_shards = src->n_shards;
+        P->shard_bytes = align_up(end, 16);
+    } else if (src->param_flat_offset) {
         std::vector<std::pair<int64_t, int64_t>> spans;
         for (int32_t p = 0; p < n_params; ++p) {
             const int64_t o = src->param_flat_offset[p];
@@ -324,9 +359,19 @@ rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_
             end += P->rows[p] * P->cols[p] * P->es[p];
         }
     }
-    P->flat_bytes = end;
-    P->n_shards = src->n_shards;
-    P->shard_bytes = align_up(end, 16 * int64_t(src->n_shards)) / src->n_shards;
+    if (src->sharding == RR_SHARD_FLAT) {
+        P->flat_bytes = end;
+        P->n_shards = src->n_shards;
+        P->shard_bytes = align_up(end, 16 * int64_t(src->n_shards)) / src->n_shards;
+        if (src->shard_bytes) {
+            if (src->shard_bytes % 16 != 0 || src->shard_bytes * src->n_shards < end)
+                return rr_fail(RR_ELAYOUT,
+                               "shard_bytes %lld: not a multiple of 16, or %d shards of it do "
+                               "not cover the %lld bytes of parameters",
+                               (long long)src->shard_bytes, src->n_shards, (long long)end);
+            P->shard_bytes = src->shard_bytes;
+        }
+    }
     if (P->shard_bytes > kMaxShardOffset) return rr_fail(RR_ELAYOUT, "shards too large");
 
     // Destination streams.

@@ -20,6 +20,8 @@ Rollout tensors, per rank r of TP = t, in this order:
                              down_e (column slices)
   norm                replicated
   lm_head             rows r of t, unless tied to the embedding
+When t exceeds the number of KV heads, k and v are not split but replicated
+by head: rank r holds KV head r * n_kv // t.
 """
 from __future__ import annotations
 
@@ -86,6 +88,17 @@ class _Slicer:
         n = rows // self.tp
         return Block(self.idx[name], r * n, n, 0, cols)
 
+    def kv_rows(self, name: str, r: int, n_heads: int, head_dim: int) -> Block:
+        """k/v rows of rank r: a row slice, or one whole replicated head when the
+        ranks outnumber the heads."""
+        if self.tp <= n_heads:
+            return self.rows(name, r)
+        if self.tp % n_heads:
+            raise ValueError(f"TP={self.tp} is not a multiple of {n_heads} KV heads")
+        _, cols = self.mat[name]
+        h = r * n_heads // self.tp
+        return Block(self.idx[name], h * head_dim, head_dim, 0, cols)
+
     def cols(self, name: str, r: int) -> Block:
         rows, cols = self.mat[name]
         if cols % self.tp:
@@ -107,9 +120,10 @@ def qwen3_rollout(shape, manifest: List[Param], tp: int = 1,
         for i in range(shape.layers):
             L = f"model.layers.{i}"
             a = f"{L}.self_attn"
-            add(f"layers.{i}.qkv_proj", [s.rows(f"{a}.q_proj.weight", r),
-                                         s.rows(f"{a}.k_proj.weight", r),
-                                         s.rows(f"{a}.v_proj.weight", r)])
+            add(f"layers.{i}.qkv_proj",
+                [s.rows(f"{a}.q_proj.weight", r),
+                 s.kv_rows(f"{a}.k_proj.weight", r, shape.n_kv, shape.head_dim),
+                 s.kv_rows(f"{a}.v_proj.weight", r, shape.n_kv, shape.head_dim)])
             add(f"layers.{i}.o_proj", [s.cols(f"{a}.o_proj.weight", r)])
             add(f"layers.{i}.q_norm", [s.whole(f"{a}.q_norm.weight")])
             add(f"layers.{i}.k_norm", [s.whole(f"{a}.k_norm.weight")])
@@ -135,7 +149,10 @@ def qwen3_rollout(shape, manifest: List[Param], tp: int = 1,
     return DstLayout(tp=tp, tensors=tensors, tensor_align_bytes=tensor_align_bytes)
 
 
-def qwen3_sync(shape, dtype: str, n_shards: int, tp: int):
-    """(manifest, source layout, destination layout) for one Qwen3 weight sync."""
+def qwen3_sync(shape, dtype: str, n_shards: int, tp: int, sharding: str = "flat"):
+    """(manifest, source layout, destination layout) for one Qwen3 weight sync.
+    sharding: "flat" (one FSDP1 FlatParameter cut evenly) or "rows" (FSDP2:
+    every parameter cut on dim 0)."""
     manifest = qwen3_manifest(shape, dtype)
-    return manifest, SrcLayout(n_shards=n_shards, align_bytes=16), qwen3_rollout(shape, manifest, tp)
+    src = SrcLayout(n_shards=n_shards, align_bytes=16, sharding=sharding)
+    return manifest, src, qwen3_rollout(shape, manifest, tp)

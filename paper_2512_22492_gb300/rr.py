@@ -41,7 +41,8 @@ class _Param(ctypes.Structure):
 
 class _SrcLayout(ctypes.Structure):
     _fields_ = [("n_shards", ctypes.c_int32), ("align_bytes", ctypes.c_int64),
-                ("param_flat_offset", ctypes.POINTER(ctypes.c_int64))]
+                ("param_flat_offset", ctypes.POINTER(ctypes.c_int64)),
+                ("sharding", ctypes.c_int32), ("shard_bytes", ctypes.c_int64)]
 
 
 class _Block(ctypes.Structure):
@@ -189,6 +190,8 @@ class SrcLayout:
     n_shards: int
     align_bytes: int = 16
     param_flat_offset: Optional[Sequence[int]] = None
+    sharding: str = "flat"    # "flat" (FSDP1 FlatParameter) or "rows" (FSDP2 dim-0 Shard)
+    shard_bytes: int = 0      # flat only: explicit shard size, 0 = computed
 
 
 @dataclass
@@ -232,9 +235,11 @@ class PlanOptions:
 class Plan:
     """Owns an rr_plan; exposes its geometry."""
 
-    def __init__(self, handle: int, n_params: int, dst: DstLayout):
+    def __init__(self, handle: int, n_params: int, dst: DstLayout, src: SrcLayout = None):
         self._h = ctypes.c_void_p(handle)
         self.n_params = n_params
+        self.sharding = src.sharding if src else "flat"
+        self.align_bytes = src.align_bytes if src else 16
         self.tp = dst.tp
         self.n_tensors = len(dst.tensors)
         self.tensor_names = [t.name for t in dst.tensors]
@@ -334,7 +339,8 @@ def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
         for d, s in enumerate(p.shape):
             cp[i].shape[d] = s
         cp[i].dtype = RR_F32 if p.dtype == "f32" else RR_BF16
-    cs = _SrcLayout(n_shards=src.n_shards, align_bytes=src.align_bytes)
+    cs = _SrcLayout(n_shards=src.n_shards, align_bytes=src.align_bytes,
+                    sharding={"flat": 0, "rows": 1}[src.sharding], shard_bytes=src.shard_bytes)
     offs = None
     if src.param_flat_offset is not None:
         offs = (ctypes.c_int64 * max(1, n))(*src.param_flat_offset)
@@ -366,7 +372,7 @@ def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
         st = _lib.rr_plan_create_ex(cp, n, ctypes.byref(cs), ctypes.byref(cd), bucket_bytes,
                                     ctypes.byref(co), ctypes.byref(out))
     _check(st, "rr_plan_create")
-    return Plan(out.value, n, dst)
+    return Plan(out.value, n, dst, src)
 
 
 # ---------------------------------------------------------------------------

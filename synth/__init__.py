@@ -67,6 +67,7 @@ class Workload:
     bucket_bytes: int
     seed: int
     specials: bool = False   # inject ~1% special bit patterns
+    sharding: str = "flat"   # "flat" (one FSDP1 FlatParameter) or "rows" (FSDP2 dim-0)
 
     @property
     def src_elem_bytes(self) -> int:
@@ -121,6 +122,24 @@ TEST_WORKLOADS = {
                              bucket_bytes=40 * 1024, seed=16),
     "tiny-moe-f32": Workload("tiny-moe-f32", TINY_MOE, "f32", n_shards=5, tp=2,
                              bucket_bytes=24 * 1024, seed=17, specials=True),
+    # FSDP2-style (each parameter cut on dim 0) trainers; uneven chunks.
+    "tiny-fsdp2": Workload("tiny-fsdp2", TINY, "f32", n_shards=3, tp=2, bucket_bytes=48 * 1024,
+                           seed=18, specials=True, sharding="rows"),
+    # TP above the KV head count: KV heads replicated over ranks.
+    "tiny-moe-kvrep": Workload("tiny-moe-kvrep", TINY_MOE, "bf16", n_shards=6, tp=4,
+                               bucket_bytes=32 * 1024, seed=19, sharding="rows"),
+    "tiny-kvrep-f32": Workload("tiny-kvrep-f32", TINY, "f32", n_shards=8, tp=8,
+                               bucket_bytes=16 * 1024, seed=20, specials=True),
+}
+
+# Full-size variants beyond the five workloads: the paper's own trainer sharding
+# (FSDP2, Section 7.1) and its rollout TP of 8.
+EXTRA_WORKLOADS = {
+    "qwen3-8b-fsdp2-tp8": Workload("qwen3-8b-fsdp2-tp8", QWEN3_8B, "f32", n_shards=8, tp=8,
+                                   bucket_bytes=128 * MiB, seed=6, sharding="rows"),
+    "qwen3-30b-a3b-fsdp2-tp8": Workload("qwen3-30b-a3b-fsdp2-tp8", QWEN3_30B_A3B, "bf16",
+                                        n_shards=8, tp=8, bucket_bytes=256 * MiB, seed=7,
+                                        sharding="rows"),
 }
 
 

@@ -17,7 +17,8 @@ ITEM_F32_VEC, ITEM_F32_SCALAR, ITEM_BF16_VEC, ITEM_BF16_SCALAR, ITEM_ZERO_VEC, \
 
 
 def workload(name):
-    return synth.WORKLOADS.get(name) or synth.TEST_WORKLOADS[name]
+    return (synth.WORKLOADS.get(name) or synth.TEST_WORKLOADS.get(name)
+            or synth.EXTRA_WORKLOADS[name])
 
 
 # ---------------------------------------------------------------------------
@@ -53,6 +54,7 @@ def random_layout(seed: int, max_params: int = 7, bucket_choices=(8, 24, 40, 64,
             blocks.append((p, r0, nr, c0, nc))
         tensors.append((f"t{t}", int(rng.integers(0, tp)), blocks))
     return dict(params=params, tensors=tensors, tp=tp,
+                sharding="rows" if rng.random() < 0.35 else "flat",
                 n_shards=int(rng.integers(1, 6)),
                 bucket_bytes=int(rng.choice(bucket_choices)),
                 align_bytes=int(rng.choice([1, 2, 4, 8, 16, 32])),
@@ -74,16 +76,18 @@ def to_oracle(desc) -> "oracle.Layout":
         return oracle.workload_layout(desc["workload"], bucket_bytes=desc["bucket_bytes"])
     return oracle.Layout(desc["params"], desc["tensors"], n_shards=desc["n_shards"],
                          tp=desc["tp"], bucket_bytes=desc["bucket_bytes"],
-                         align_bytes=desc["align_bytes"], tensor_align=desc["tensor_align"])
+                         align_bytes=desc["align_bytes"], tensor_align=desc["tensor_align"],
+                         sharding=desc.get("sharding", "flat"))
 
 
 def to_product(desc):
     import paper_2512_22492_gb300 as rr
     if desc.get("workload") is not None:
         w = desc["workload"]
-        return rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp)
+        return rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding)
     manifest = [rr.Param(n, d, "f32" if es == 4 else "bf16") for n, d, es in desc["params"]]
-    src = rr.SrcLayout(n_shards=desc["n_shards"], align_bytes=desc["align_bytes"])
+    src = rr.SrcLayout(n_shards=desc["n_shards"], align_bytes=desc["align_bytes"],
+                       sharding=desc.get("sharding", "flat"))
     dst = rr.DstLayout(tp=desc["tp"], tensor_align_bytes=desc["tensor_align"],
                        tensors=[rr.DstTensor(n, r, [rr.Block(*b) for b in blocks])
                                 for n, r, blocks in desc["tensors"]])

@@ -74,15 +74,43 @@ def fill_from_host(buf: SyncBuffers, host_shards) -> None:
     buf.flat.copy_(torch.from_numpy(host))
 
 
+def _flat_offsets(manifest, align):
+    """Flat-layout offsets: generated values are indexed by them under any sharding."""
+    offs, off = [], 0
+    for p in manifest:
+        es = 4 if p.dtype == "f32" else 2
+        a = max(align, es)
+        off = (off + a - 1) // a * a
+        offs.append(off)
+        off += (int(np.prod(p.shape)) if len(p.shape) else 1) * es
+    return offs
+
+
 def fill_with_generator(buf: SyncBuffers, manifest, seed: int, specials: bool,
                         stream: int = 0) -> None:
-    """Device generator, one launch per parameter at the library's flat offsets."""
+    """Device generator, one launch per parameter (per shard for a row-sharded
+    trainer) at the library's offsets."""
+    plan = buf.plan
     base = buf.flat.data_ptr()
-    for p, off in zip(manifest, buf.plan.param_flat_offset):
+    if plan.sharding == "flat":
+        for p, off in zip(manifest, plan.param_flat_offset):
+            es = 4 if p.dtype == "f32" else 2
+            n = int(np.prod(p.shape)) if len(p.shape) else 1
+            synth.fill_dev(base + off, n, es, seed, first_idx=off // es, specials=specials,
+                           stream=stream)
+        return
+    S = plan.shard_bytes
+    flat = _flat_offsets(manifest, plan.align_bytes)
+    for p, local, f in zip(manifest, plan.param_flat_offset, flat):
         es = 4 if p.dtype == "f32" else 2
-        n = int(np.prod(p.shape)) if len(p.shape) else 1
-        synth.fill_dev(base + off, n, es, seed, first_idx=off // es, specials=specials,
-                       stream=stream)
+        rows = p.shape[0] if len(p.shape) else 1
+        cols = int(np.prod(p.shape[1:])) if len(p.shape) > 1 else 1
+        c = -(-rows // plan.n_shards)
+        for s in range(plan.n_shards):
+            r0, r1 = s * c, min((s + 1) * c, rows)
+            if r1 > r0:
+                synth.fill_dev(base + s * S + local, (r1 - r0) * cols, es, seed,
+                               first_idx=f // es + r0 * cols, specials=specials, stream=stream)
 
 
 def bucket_list(buf: SyncBuffers):

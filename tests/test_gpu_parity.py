@@ -62,9 +62,25 @@ def full_parity(desc, separate_buckets=False, **opts):
 
 
 @pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2",
-                                  "tiny-moe-f32"])
+                                  "tiny-moe-f32", "tiny-fsdp2", "tiny-moe-kvrep",
+                                  "tiny-kvrep-f32"])
 def test_small_workloads(name):
     full_parity(U.workload_desc(name))
+
+
+@pytest.mark.parametrize("name", ["tiny-fsdp2", "tiny-moe-kvrep"])
+def test_device_generator_fill_matches_oracle_shards(name):
+    """The harness's device fill of a row-sharded trainer equals the oracle's host
+    shards byte for byte (both indexed by the flat layout)."""
+    desc = U.workload_desc(name)
+    L = U.to_oracle(desc)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"])
+    buf = H.alloc(plan, with_dst=False)
+    H.fill_with_generator(buf, m, desc["seed"], desc["specials"])
+    torch.cuda.synchronize()
+    want = np.concatenate(L.host_shards(desc["seed"], desc["specials"]))
+    np.testing.assert_array_equal(buf.flat.cpu().numpy(), want)
 
 
 @pytest.mark.parametrize("name", ["tiny", "tiny-tp4"])
@@ -186,6 +202,24 @@ def test_qwen3_8b_tp4_bucket_sweep_sampled():
     _unpack_sampled("qwen3-8b-tp4", [("layers.3.qkv_proj", 1), ("layers.20.o_proj", 2),
                                      ("layers.35.down_proj", 3), ("layers.7.gate_up_proj", 0),
                                      ("norm", 3)])
+    torch.cuda.empty_cache()
+
+
+def test_qwen3_8b_fsdp2_tp8_sampled():
+    """The paper's own trainer sharding (FSDP2) and rollout TP (8)."""
+    sampled_parity("qwen3-8b-fsdp2-tp8", n_random_buckets=2)
+    torch.cuda.empty_cache()
+    _unpack_sampled("qwen3-8b-fsdp2-tp8", [("layers.9.qkv_proj", 5), ("layers.30.down_proj", 7),
+                                           ("norm", 2)])
+    torch.cuda.empty_cache()
+
+
+def test_qwen3_30b_a3b_fsdp2_tp8_sampled():
+    """FSDP2 trainer, TP=8 rollout with 4 KV heads: each KV head on two ranks."""
+    sampled_parity("qwen3-30b-a3b-fsdp2-tp8", n_random_buckets=1)
+    torch.cuda.empty_cache()
+    _unpack_sampled("qwen3-30b-a3b-fsdp2-tp8", [("layers.1.qkv_proj", 3), ("layers.1.qkv_proj", 2),
+                                                ("layers.40.experts.w13", 6), ("norm", 7)])
     torch.cuda.empty_cache()
 
 

@@ -116,6 +116,13 @@ def _to_bf16_bits(t: torch.Tensor) -> torch.Tensor:
 def restate_rollout(shape, P, tp):
     """Per rank, the rollout tensors built the way an inference engine's loader would."""
     H = shape.hidden
+
+    def kv(t, r):
+        # Fewer KV heads than ranks: each rank loads one whole head, shared.
+        if tp <= shape.n_kv:
+            return t.chunk(tp, 0)[r]
+        return t.view(shape.n_kv, shape.head_dim, -1)[r * shape.n_kv // tp]
+
     ranks = []
     for r in range(tp):
         ts = [P["model.embed_tokens.weight"].chunk(tp, 0)[r]]
@@ -123,8 +130,8 @@ def restate_rollout(shape, P, tp):
             pre = f"model.layers.{i}."
             a = pre + "self_attn."
             ts.append(torch.cat([P[a + "q_proj.weight"].chunk(tp, 0)[r],
-                                 P[a + "k_proj.weight"].chunk(tp, 0)[r],
-                                 P[a + "v_proj.weight"].chunk(tp, 0)[r]], 0))
+                                 kv(P[a + "k_proj.weight"], r),
+                                 kv(P[a + "v_proj.weight"], r)], 0))
             ts.append(P[a + "o_proj.weight"].chunk(tp, 1)[r])
             ts.append(P[a + "q_norm.weight"])
             ts.append(P[a + "k_norm.weight"])
@@ -164,11 +171,32 @@ def restate_buckets(ranks, bucket_bytes, tensor_align=256):
     return out
 
 
-RESTATE = ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2", "tiny-moe-f32"]
+def fsdp2_shards(params, P, n, align=16):
+    """Trainer shards as FSDP2 holds them: every parameter cut on dim 0 with
+    torch.chunk, each chunk padded to the first chunk's rows; per shard the
+    chunks follow one another in manifest order at `align`-byte starts."""
+    offs, off = [], 0
+    for name, dims, es in params:
+        c = -(-dims[0] // n)
+        off = (off + max(align, es) - 1) // max(align, es) * max(align, es)
+        offs.append(off)
+        off += c * int(np.prod(dims[1:], dtype=np.int64)) * es
+    S = (off + 15) // 16 * 16
+    shards = [np.zeros(S, np.uint8) for _ in range(n)]
+    for (name, dims, es), o in zip(params, offs):
+        for s_, ch in enumerate(torch.chunk(P[name], n, dim=0)):
+            b = np.frombuffer(ch.contiguous().numpy().tobytes(), np.uint8)
+            shards[s_][o:o + b.size] = b
+    return shards
+
+
+RESTATE = ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2", "tiny-moe-f32",
+           "tiny-fsdp2", "tiny-moe-kvrep", "tiny-kvrep-f32"]
 
 
 def _workload(name):
-    return synth.WORKLOADS.get(name) or synth.TEST_WORKLOADS[name]
+    return (synth.WORKLOADS.get(name) or synth.TEST_WORKLOADS.get(name)
+            or synth.EXTRA_WORKLOADS[name])
 
 
 @pytest.mark.parametrize("name", RESTATE)
@@ -177,8 +205,15 @@ def test_oracle_matches_restatement(name):
     L = oracle.workload_layout(w)
     P = _param_tensors(L.params, _flat_offsets(L.params), w.seed, w.specials)
     ranks = restate_rollout(w.shape, P, w.tp)
-    # Per-tensor reshard, straight from the materialised shards.
-    src = oracle.Source(shards=L.host_shards(w.seed, w.specials))
+    # Per-tensor reshard, straight from trainer shards: materialised by the
+    # oracle for a flat trainer, built with torch.chunk for an FSDP2 one.
+    if w.sharding == "rows":
+        shards = fsdp2_shards(L.params, P, w.n_shards)
+        for a, b in zip(shards, L.host_shards(w.seed, w.specials)):
+            np.testing.assert_array_equal(a, b)
+    else:
+        shards = L.host_shards(w.seed, w.specials)
+    src = oracle.Source(shards=shards)
     flat_t = [t for rank in ranks for t in rank]
     order = [i for r in range(w.tp) for i, (_, rk, _) in enumerate(L.tensors) if rk == r]
     assert len(order) == len(flat_t)
@@ -199,12 +234,15 @@ def test_oracle_matches_restatement(name):
 # Invariants
 # ---------------------------------------------------------------------------
 
-@pytest.mark.parametrize("n_shards", [1, 2, 3, 7, 8, 13])
-def test_shard_count_invariance(n_shards):
+@pytest.mark.parametrize("n_shards,sharding", [(1, "flat"), (2, "flat"), (3, "flat"),
+                                               (7, "flat"), (8, "flat"), (13, "flat"),
+                                               (1, "rows"), (3, "rows"), (8, "rows"),
+                                               (13, "rows"), (300, "rows")])
+def test_shard_count_invariance(n_shards, sharding):
     w = synth.TEST_WORKLOADS["tiny-tp4"]
     ref_L = oracle.workload_layout(w.with_(n_shards=1))
     ref, ref_cs = ref_L.pack(oracle.Source(shards=ref_L.host_shards(w.seed, w.specials)))
-    L = oracle.workload_layout(w.with_(n_shards=n_shards))
+    L = oracle.workload_layout(w.with_(n_shards=n_shards, sharding=sharding))
     got, cs = L.pack(oracle.Source(shards=L.host_shards(w.seed, w.specials)))
     np.testing.assert_array_equal(got, ref)
     np.testing.assert_array_equal(cs, ref_cs)
@@ -220,7 +258,8 @@ def test_generator_mode_matches_buffer_mode():
 
 
 @pytest.mark.parametrize("name", ["qwen3-0.6b", "qwen3-8b", "qwen3-8b-tp4", "qwen3-30b-a3b",
-                                  "tiny-moe-tp2"])
+                                  "tiny-moe-tp2", "qwen3-8b-fsdp2-tp8",
+                                  "qwen3-30b-a3b-fsdp2-tp8"])
 def test_coverage_counts(name):
     """Every parameter element is read tp times if replicated, once otherwise, and
     within one rank no parameter element is read twice (metadata only: full sizes)."""
@@ -236,7 +275,9 @@ def test_coverage_counts(name):
     for p, (pname, dims, _) in enumerate(params):
         numel = int(np.prod(dims))
         replicated = len(dims) == 1 or pname.endswith("mlp.gate.weight")
-        assert area[p] == numel * (w.tp if replicated else 1), pname
+        kv = pname.endswith(("k_proj.weight", "v_proj.weight"))
+        times = w.tp if replicated else (max(1, w.tp // w.shape.n_kv) if kv else 1)
+        assert area[p] == numel * times, pname
     for (r, p), rects in per_rank.items():
         # Rectangles of one rank on one parameter must not overlap.
         for i in range(len(rects)):
@@ -293,3 +334,35 @@ def test_layout_rejects_bad_input():
         oracle.Layout(params, [("t", 1, [(0, 0, 1, 0, 4)])], 1, 1, 64)   # rank out of range
     with pytest.raises(RuntimeError):
         oracle.Layout(params, [("t", 0, [(0, 0, 1, 0, 4)])], 1, 1, 12)   # bucket % 8 != 0
+
+
+ROWS_GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "rows_sharding_worked_example.json")
+
+
+def test_rows_sharding_golden():
+    g = json.load(open(ROWS_GOLDEN))
+    params = [(p["name"], tuple(p["dims"]), p["elem_bytes"]) for p in g["params"]]
+    tensors = [(t["name"], t["rank"], [tuple(b) for b in t["blocks"]]) for t in g["tensors"]]
+    L = oracle.Layout(params, tensors, n_shards=g["n_shards"], tp=g["tp"],
+                      bucket_bytes=g["bucket_bytes"], align_bytes=g["align_bytes"],
+                      tensor_align=g["tensor_align"], sharding="rows")
+    e = g["expect"]
+    assert list(L.chunk_rows) == e["chunk_rows"]
+    assert list(L.param_offset) == e["param_offset"]
+    assert L.shard_bytes == e["shard_bytes"]
+    assert list(L.param_gen_base) == e["param_gen_base"]
+    shards = [bytearray(e["shard_bytes"]) for _ in range(g["n_shards"])]
+    for pl in g["placement"]:
+        p = g["params"][pl["param"]]
+        es = p["elem_bytes"]
+        for k in range(pl["n_elems"]):
+            v = _int(p["bits"][pl["first_elem"] + k])
+            o = pl["offset"] + k * es
+            shards[pl["shard"]][o:o + es] = v.to_bytes(es, "little")
+    src = oracle.Source(shards=[np.frombuffer(bytes(s), np.uint8) for s in shards])
+    for t, want in enumerate(e["tensors_bf16"]):
+        np.testing.assert_array_equal(L.reshard_tensor(src, t),
+                                      np.array([_int(x) for x in want], np.uint16))
+    buckets, cs = L.pack(src)
+    assert [b.tobytes().hex() for b in buckets] == e["buckets_hex"]
+    assert [int(c) for c in cs] == [_int(c) for c in e["checksums"]]
