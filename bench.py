@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--bucket-mib", type=int, default=0, help="override the bucket size")
     ap.add_argument("--chunk-kib", type=int, default=0, help="plan option: KiB per work item")
     ap.add_argument("--grid", type=int, default=0, help="plan option: persistent grid size")
+    ap.add_argument("--snapshot", action="store_true",
+                    help="also time rr_pack straight into pinned host buckets")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-buckets", type=int, default=2,
@@ -336,6 +338,40 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     unpack_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in sep)
     verify_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in sep)
 
+    # Checkpoint snapshot: rr_pack writing the buckets into pinned host memory.
+    snapshot = None
+    if args.snapshot:
+        row = (plan.bucket_bytes + 15) // 16 * 16
+        hstore = torch.empty((plan.n_buckets, row), dtype=torch.uint8, pin_memory=True)
+        hview = hstore[:, :plan.bucket_bytes]
+        hcs = torch.zeros_like(buf.checksums)
+        rr.rr_pack(plan, buf.shards, hview, hcs, stream)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        reps = 3
+        a.record(stream)
+        for _ in range(reps):
+            rr.rr_pack(plan, buf.shards, hview, hcs, stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        s_ms = a.elapsed_time(b) / reps
+        # Versus packing on the device and copying the buckets out.
+        c = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        c.record(stream)
+        for _ in range(reps):
+            H.pack(buf, stream)
+            hstore.copy_(buf.bucket_store, non_blocking=True)
+        e.record(stream)
+        torch.cuda.synchronize()
+        c_ms = c.elapsed_time(e) / reps
+        snapshot = {"pack_to_host_ms": round(s_ms, 2),
+                    "host_GB/s": round(st["pack_bytes_written"] / (s_ms * 1e-3) / 1e9, 1),
+                    "pack_then_copy_ms": round(c_ms, 2),
+                    "identical": bool(torch.equal(hcs, buf.checksums))}
+        del hstore, hview
+
     # End to end through the public API with host buffers: every step copies the
     # trainer's shards from pinned host memory, syncs, and reads back the checksums.
     e2e = None
@@ -404,6 +440,8 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         "gpu_launches": 2 * args.steps,
         "e2e": e2e,
     }
+    if snapshot:
+        line["snapshot"] = snapshot
     del buf
     torch.cuda.empty_cache()
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
