@@ -97,8 +97,12 @@ typedef struct {
  *                 in manifest order, each starting at a multiple of
  *                 max(align_bytes, element size); all shards share that local
  *                 layout and are S = (end of the last chunk rounded up to 16)
- *                 bytes.  Padding rows are never read. */
-typedef enum { RR_SHARD_FLAT = 0, RR_SHARD_ROWS = 1 } rr_sharding;
+ *                 bytes.  Padding rows are never read.
+ *  RR_SHARD_TENSORS: every parameter is its own buffer: "shard" p is
+ *                 parameter p, row-major from byte 0 (n_shards must equal the
+ *                 number of parameters).  This is how a relay re-packs from
+ *                 the rollout tensors it has loaded. */
+typedef enum { RR_SHARD_FLAT = 0, RR_SHARD_ROWS = 1, RR_SHARD_TENSORS = 2 } rr_sharding;
 
 /* Trainer side. */
 typedef struct {
@@ -164,7 +168,8 @@ rr_status rr_plan_query(const rr_plan* plan, int32_t* n_buckets, int64_t* stream
 
 /* Source geometry: shard size S, end of the last parameter, and per-parameter
  * byte offsets ([n_params]): flat offsets for RR_SHARD_FLAT, offsets within
- * each shard for RR_SHARD_ROWS.  Any output pointer may be NULL. */
+ * each shard for RR_SHARD_ROWS, 0 for RR_SHARD_TENSORS (whose S is the size of
+ * the largest parameter).  Any output pointer may be NULL. */
 rr_status rr_plan_source(const rr_plan* plan, int64_t* shard_bytes, int64_t* flat_bytes,
                          int64_t* param_flat_offset);
 

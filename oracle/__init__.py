@@ -213,7 +213,7 @@ class Layout:
         for name in ("param_offset", "tensor_numel", "tensor_offset", "rank_stream_bytes",
                      "rank_first_bucket", "chunk_rows", "param_gen_base"):
             setattr(L, name, getattr(self, name).ctypes.data_as(_P64))
-        L.sharding = {"flat": 0, "rows": 1}[sharding]
+        L.sharding = {"flat": 0, "rows": 1, "tensors": 2}[sharding]
         L.shard_bytes_in = shard_bytes
         self._explicit = None
         if explicit_offsets is not None:
@@ -238,6 +238,14 @@ class Layout:
     def host_shards(self, seed: int, specials: bool = False) -> List[np.ndarray]:
         """Materialise the source with the seeded generator and cut it into shards."""
         import synth
+        if self.sharding == "tensors":
+            out = []
+            for p, (_, _, es) in enumerate(self.params):
+                n = self.param_numel(p)
+                vals = synth.values_host(n, es, seed, first_idx=int(self.param_gen_base[p]),
+                                         specials=specials)
+                out.append(vals.view(np.uint8).copy())
+            return out
         flat = np.zeros(self.shard_bytes * self.n_shards, np.uint8)
         S = self.shard_bytes
         for p, (_, _, es) in enumerate(self.params):

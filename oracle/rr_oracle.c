@@ -39,6 +39,9 @@
  *  the last chunk rounded up to 16.  Row r, column k of parameter p is in
  *  shard r / c at offset off_p + ((r - s*c) * cols + k) * element size.
  *
+ *  Source, one buffer per parameter.  Parameter p is "shard" p, row-major
+ *  from byte 0.
+ *
  *  A parameter of shape [d0, d1, ...] is viewed as a matrix [rows = d0,
  *  cols = d1 * d2 * ...] (cols = 1 for a vector).  Generated values are
  *  indexed by the element's position in the flat layout whatever the
@@ -108,7 +111,7 @@ typedef struct {
                                    last chunk within a shard)                      */
     int64_t shard_bytes;        /* S                                                */
     /* description, continued */
-    int32_t sharding;           /* 0: flat, 1: rows                                 */
+    int32_t sharding;           /* 0: flat, 1: rows, 2: one buffer per parameter     */
     int32_t pad_;
     int64_t shard_bytes_in;     /* flat: explicit S, or 0                           */
     const int64_t* explicit_offset; /* flat: explicit offsets, or NULL              */
@@ -169,6 +172,18 @@ int orc_layout_compute(orc_layout* L) {
                 return ORC_EINVAL;
             L->shard_bytes = L->shard_bytes_in;
         }
+    } else if (L->sharding == 2) {
+        /* One buffer per parameter. */
+        if (L->explicit_offset || L->shard_bytes_in || L->n_shards != L->n_params)
+            return ORC_EINVAL;
+        int64_t biggest = 0;
+        for (int32_t p = 0; p < L->n_params; ++p) {
+            const orc_param* P = &L->params[p];
+            int64_t bytes = P->rows * P->cols * P->elem_bytes;
+            if (bytes > biggest) biggest = bytes;
+        }
+        L->flat_bytes = biggest;
+        L->shard_bytes = biggest;
     } else {
         /* Row sharding: every shard holds each parameter's chunk of c rows. */
         if (L->explicit_offset || L->shard_bytes_in) return ORC_EINVAL;
@@ -255,6 +270,9 @@ static int source_bits(const orc_layout* L, const orc_source* S, int32_t p, int6
             if (rc) return rc;
             v |= (uint32_t)byte << (8 * i);
         }
+    } else if (L->sharding == 2) {
+        if (p >= L->n_shards || S->shards[p] == NULL) return ORC_ESOURCE;
+        for (int32_t i = 0; i < es; ++i) v |= (uint32_t)S->shards[p][e * es + i] << (8 * i);
     } else {
         int64_t row = e / P->cols;
         int64_t s = row / L->chunk_rows[p];

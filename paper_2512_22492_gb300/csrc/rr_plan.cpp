@@ -49,6 +49,8 @@ public:
             const int64_t f = P->param_off[p] + e * es;
             return {f / S, f % S, S - f % S};
         }
+        if (P->sharding == RR_SHARD_TENSORS)
+            return {p, e * es, (P->rows[p] * P->cols[p] - e) * es};
         const int64_t cols = P->cols[p], c = P->chunk_rows[p];
         const int64_t sh = e / cols / c;
         const int64_t end = std::min((sh + 1) * c, P->rows[p]) * cols;   // p's last element in sh
@@ -319,10 +321,24 @@ rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_
 
     // Source offsets.
     int64_t end = 0;
-    if (src->sharding != RR_SHARD_FLAT && src->sharding != RR_SHARD_ROWS)
+    if (src->sharding != RR_SHARD_FLAT && src->sharding != RR_SHARD_ROWS &&
+        src->sharding != RR_SHARD_TENSORS)
         return rr_fail(RR_EINVAL, "unknown sharding %d", src->sharding);
     P->sharding = src->sharding;
-    if (src->sharding == RR_SHARD_ROWS) {
+    if (src->sharding == RR_SHARD_TENSORS) {
+        if (src->param_flat_offset || src->shard_bytes)
+            return rr_fail(RR_EINVAL, "per-tensor sources take no explicit offsets or shard size");
+        if (src->n_shards != n_params)
+            return rr_fail(RR_EINVAL, "per-tensor sources need n_shards (%d) == n_params (%d)",
+                           src->n_shards, n_params);
+        for (int32_t p = 0; p < n_params; ++p) {
+            P->param_off[p] = 0;
+            end = std::max(end, P->rows[p] * P->cols[p] * P->es[p]);
+        }
+        P->flat_bytes = end;
+        P->n_shards = src->n_shards;
+        P->shard_bytes = end;   // the largest parameter
+    } else if (src->sharding == RR_SHARD_ROWS) {
         if (src->param_flat_offset || src->shard_bytes)
             return rr_fail(RR_EINVAL, "row sharding takes no explicit offsets or shard size");
         P->chunk_rows.resize(n_params);

@@ -156,3 +156,108 @@ def qwen3_sync(shape, dtype: str, n_shards: int, tp: int, sharding: str = "flat"
     manifest = qwen3_manifest(shape, dtype)
     src = SrcLayout(n_shards=n_shards, align_bytes=16, sharding=sharding)
     return manifest, src, qwen3_rollout(shape, manifest, tp)
+
+
+# ---------------------------------------------------------------------------
+# Relay re-pack (Section 5.2.1, step 3): a rollout that already holds the new
+# weights serves others.  Its copy is the rollout layout in bf16 -- either the
+# buckets it pulled, or the tensors it loaded -- and the rollout it serves may
+# use another tensor-parallel degree.
+# ---------------------------------------------------------------------------
+
+def rollout_as_source(dst: DstLayout):
+    """The tensors of a rollout layout as bf16 source parameters.
+
+    Tensor t becomes parameter t of shape [sum of its blocks' rows, cols] (its
+    blocks share one column count).  Also returns, per trainer parameter, the
+    pieces that hold it: (source tensor, first row in that tensor, block)."""
+    params: List[Param] = []
+    pieces: Dict[int, List[Tuple[int, int, Block]]] = {}
+    for t, T in enumerate(dst.tensors):
+        cols = {b.ncols for b in T.blocks if b.nrows and b.ncols}
+        if len(cols) > 1:
+            raise ValueError(f"{T.name}: blocks of different widths cannot form a matrix")
+        width = cols.pop() if cols else 1
+        rows = sum(b.nrows for b in T.blocks if b.nrows and b.ncols)
+        params.append(Param(f"rank{T.rank}.{T.name}", (rows, width), "bf16"))
+        ro = 0
+        for b in T.blocks:
+            if not (b.nrows and b.ncols):
+                continue
+            pieces.setdefault(b.param, []).append((t, ro, b))
+            ro += b.nrows
+    return params, pieces
+
+
+def _translate(blk: Block, pieces) -> List[Block]:
+    """Blocks over source tensors holding `blk`'s elements in its row-major order."""
+    r0, r1 = blk.row0, blk.row0 + blk.nrows
+    c0, c1 = blk.col0, blk.col0 + blk.ncols
+    if r1 <= r0 or c1 <= c0:
+        return []
+    seen, cand = set(), []
+    for t, ro, b in pieces:
+        rect = (b.row0, b.nrows, b.col0, b.ncols)
+        if rect in seen:          # a replica (norms, router, shared KV heads): one is enough
+            continue
+        if b.row0 < r1 and r0 < b.row0 + b.nrows and b.col0 < c1 and c0 < b.col0 + b.ncols:
+            seen.add(rect)
+            cand.append((t, ro, b))
+    cuts = sorted({r0, r1} | {min(max(b.row0, r0), r1) for _, _, b in cand}
+                  | {min(max(b.row0 + b.nrows, r0), r1) for _, _, b in cand})
+    out: List[Block] = []
+    for ra, rb in zip(cuts, cuts[1:]):
+        if rb <= ra:
+            continue
+        band = sorted((x for x in cand if x[2].row0 <= ra and rb <= x[2].row0 + x[2].nrows),
+                      key=lambda x: x[2].col0)
+        spans, c = [], c0
+        for t, ro, b in band:
+            a, z = max(c, b.col0), min(c1, b.col0 + b.ncols)
+            if a > c:
+                raise ValueError("the source does not hold every element of the target")
+            if z > a:
+                spans.append((t, ro, b, a, z))
+                c = z
+        if c < c1:
+            raise ValueError("the source does not hold every element of the target")
+        if len(spans) == 1:
+            t, ro, b, a, z = spans[0]
+            out.append(Block(t, ro + ra - b.row0, rb - ra, a - b.col0, z - a))
+        else:
+            for r in range(ra, rb):        # row-parallel pieces side by side: row by row
+                for t, ro, b, a, z in spans:
+                    out.append(Block(t, ro + r - b.row0, 1, a - b.col0, z - a))
+    return out
+
+
+def relayout(source: DstLayout, target: DstLayout) -> DstLayout:
+    """`target` (blocks on trainer parameters) re-expressed on the tensors of
+    `source` (the parameters that ``rollout_as_source(source)`` returns)."""
+    _, pieces = rollout_as_source(source)
+    tensors = [DstTensor(T.name, T.rank,
+                         [nb for b in T.blocks for nb in _translate(b, pieces.get(b.param, []))])
+               for T in target.tensors]
+    return DstLayout(tp=target.tp, tensors=tensors, tensor_align_bytes=target.tensor_align_bytes)
+
+
+def qwen3_relay(shape, src_tp: int, dst_tp: int, from_plan=None):
+    """(manifest, source layout, destination layout) for a relay that holds the
+    TP=src_tp rollout image and serves a TP=dst_tp rollout.
+
+    from_plan=None: the relay re-packs from its loaded tensors (one buffer per
+    tensor, in the order of the TP=src_tp rollout layout).  from_plan=<the
+    plan that packed the image>: it re-packs straight from the buckets it
+    pulled (the buckets, in order, are the shards; bucket_bytes must be a
+    multiple of 16)."""
+    logical = qwen3_manifest(shape, "bf16")
+    src = qwen3_rollout(shape, logical, src_tp)
+    params, _ = rollout_as_source(src)
+    dst = relayout(src, qwen3_rollout(shape, logical, dst_tp))
+    if from_plan is None:
+        return params, SrcLayout(n_shards=len(params), sharding="tensors"), dst
+    B = from_plan.bucket_bytes
+    offsets = [from_plan.first_bucket_of_rank[from_plan.tensor_ranks[t]] * B
+               + from_plan.tensor_stream_offset[t] for t in range(len(params))]
+    return params, SrcLayout(n_shards=from_plan.n_buckets, param_flat_offset=offsets,
+                             shard_bytes=B), dst

@@ -190,7 +190,8 @@ class SrcLayout:
     n_shards: int
     align_bytes: int = 16
     param_flat_offset: Optional[Sequence[int]] = None
-    sharding: str = "flat"    # "flat" (FSDP1 FlatParameter) or "rows" (FSDP2 dim-0 Shard)
+    sharding: str = "flat"    # "flat" (FSDP1 FlatParameter), "rows" (FSDP2 dim-0 Shard),
+                              # or "tensors" (one buffer per parameter)
     shard_bytes: int = 0      # flat only: explicit shard size, 0 = computed
 
 
@@ -340,7 +341,8 @@ def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
             cp[i].shape[d] = s
         cp[i].dtype = RR_F32 if p.dtype == "f32" else RR_BF16
     cs = _SrcLayout(n_shards=src.n_shards, align_bytes=src.align_bytes,
-                    sharding={"flat": 0, "rows": 1}[src.sharding], shard_bytes=src.shard_bytes)
+                    sharding={"flat": 0, "rows": 1, "tensors": 2}[src.sharding],
+                    shard_bytes=src.shard_bytes)
     offs = None
     if src.param_flat_offset is not None:
         offs = (ctypes.c_int64 * max(1, n))(*src.param_flat_offset)
@@ -372,7 +374,14 @@ def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
         st = _lib.rr_plan_create_ex(cp, n, ctypes.byref(cs), ctypes.byref(cd), bucket_bytes,
                                     ctypes.byref(co), ctypes.byref(out))
     _check(st, "rr_plan_create")
-    return Plan(out.value, n, dst, src)
+    plan = Plan(out.value, n, dst, src)
+    plan.param_bytes = []
+    for p in manifest:
+        numel = 1
+        for d in p.shape:
+            numel *= d
+        plan.param_bytes.append(numel * (4 if p.dtype == "f32" else 2))
+    return plan
 
 
 # ---------------------------------------------------------------------------
@@ -442,9 +451,15 @@ def _check_checksums(plan: Plan, checksums) -> None:
         raise ValueError(f"checksums: {nb} bytes, plan needs {8 * plan.n_buckets}")
 
 
+def _shard_need(plan: Plan):
+    if plan.sharding == "tensors":
+        return lambda i: plan.param_bytes[i]
+    return plan.shard_bytes
+
+
 def rr_pack(plan: Plan, src_shards, buckets, checksums, stream=None) -> None:
     """Reshard + cast + pack + checksum (asynchronous on `stream`)."""
-    _check_list(src_shards, plan.n_shards, plan.shard_bytes, "src_shards")
+    _check_list(src_shards, plan.n_shards, _shard_need(plan), "src_shards")
     _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
     _check_checksums(plan, checksums)
     _check(_lib.rr_pack(plan.handle, _ptr_array(src_shards), _ptr_array(buckets),
@@ -475,7 +490,7 @@ def rr_verify(plan: Plan, buckets, checksums, stream=None):
 def rr_pack_range(plan: Plan, first_bucket: int, n_buckets: int, src_shards, buckets, checksums,
                   stream=None) -> None:
     """Pack only buckets [first_bucket, first_bucket + n_buckets) (asynchronous)."""
-    _check_list(src_shards, plan.n_shards, plan.shard_bytes, "src_shards")
+    _check_list(src_shards, plan.n_shards, _shard_need(plan), "src_shards")
     _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
     _check_checksums(plan, checksums)
     _check(_lib.rr_pack_range(plan.handle, first_bucket, n_buckets, _ptr_array(src_shards),
