@@ -142,12 +142,20 @@ typedef struct {
 
 typedef struct rr_plan rr_plan;
 
+/* Which kernels move the data.  RR_ENGINE_AUTO (default): the bulk-copy
+ * engine (cp.async.bulk into shared-memory stages, consumer warps cast/copy
+ * and sum) when every buffer of the call is device memory, otherwise the
+ * register path (16-byte loads and stores).  RR_ENGINE_REGISTERS: always the
+ * register path.  Both produce identical bytes. */
+typedef enum { RR_ENGINE_AUTO = 0, RR_ENGINE_REGISTERS = 1 } rr_engine;
+
 /* Tuning / inspection options for rr_plan_create_ex.  Zero means default. */
 typedef struct {
     int32_t host_only;   /* 1: build the tables on the host only and touch no GPU; such
                             a plan can be queried and exported but not executed       */
     int32_t grid_blocks; /* persistent grid size; default: SMs x resident blocks      */
     int64_t chunk_bytes; /* largest destination bytes per work item; default 32 KiB   */
+    int32_t engine;      /* rr_engine                                                 */
 } rr_plan_options;
 
 /* Compiles manifest + source layout + destination layout + bucket size into
@@ -346,6 +354,12 @@ rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32
 rr_status rr_verify_noalloc(const void* const* buckets, int32_t n_buckets, size_t bucket_bytes,
                             const uint64_t* checksums, int64_t* n_bad, int64_t* first_bad,
                             cudaStream_t stream);
+
+/* Waits for `stream`, then reports whether a kernel of this plan gave up on
+ * a wait (the bulk-copy engine bounds every wait; one that runs out marks the
+ * plan and its output is incomplete): RR_ECUDA if so (and clears the mark),
+ * RR_OK otherwise.  rr_verify and rr_unpack_verify check this themselves. */
+rr_status rr_plan_check(const rr_plan* plan, cudaStream_t stream);
 
 const char* rr_status_str(rr_status status);
 const char* rr_last_error(void);

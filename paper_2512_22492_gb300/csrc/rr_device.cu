@@ -442,6 +442,361 @@ __global__ void __launch_bounds__(kThreads, 4) rr_verify_kernel(const __grid_con
 }
 
 // ---------------------------------------------------------------------------
+// Bulk-copy engine (cp.async.bulk + mbarrier), the default for buffers in
+// device memory.  One producer lane per block turns the block's work items
+// into pieces: long contiguous or row-strided 16-byte-aligned runs are loaded
+// into a ring of shared-memory stages with cp.async.bulk (rows of a strided
+// run land back to back); ragged, misaligned and zero-fill work passes
+// through as metadata only.  Consumer warps wait for a stage, cast or copy it
+// to the destination with 16-byte stores, accumulate the checksum, and
+// release the stage.  Memory latency is hidden by the ring, not by registers.
+//
+// Every wait is bounded: a wait that runs out sets the plan's error word,
+// lets its block's loads land, and returns (the host reports it as RR_ECUDA).
+// ---------------------------------------------------------------------------
+
+constexpr int kConsumerWarps = 8;
+constexpr int kBulkThreads = 32 * (kConsumerWarps + 1);
+constexpr int kStageBytes = 32 * 1024;
+constexpr int kStages = 3;
+constexpr uint32_t kWaitLimit = 1u << 20;     // x at most kWaitHintNs each: about a second
+constexpr uint32_t kWaitHintNs = 1000;
+constexpr unsigned int kErrWaitTimeout = 1;
+
+enum : uint16_t {
+    PC_CAST = 1,      // stage holds fp32 rows -> bf16 destination
+    PC_COPY = 2,      // stage holds bf16 -> destination
+    PC_READ = 3,      // stage holds bf16 that is only summed (verifying unpack gaps)
+    PC_SCALAR = 4,    // element by element from global memory
+    PC_ZERO_VEC = 5,  // 16-byte zero stores
+    PC_ZERO_SCALAR = 6,
+    PC_END = 7
+};
+
+struct Piece {
+    const char* src;      // first source element (global)
+    char* dst;            // first destination element (global), NULL for PC_READ
+    uint64_t src_stride;  // bytes between source rows
+    uint32_t n;           // destination elements (2 bytes each)
+    uint32_t rows;        // source rows
+    uint32_t row_len;     // elements per source row
+    uint32_t sum_bucket;  // bucket the checksum contribution belongs to
+    uint32_t sum_off;     // byte offset of element 0 in that bucket
+    uint16_t kind;
+    uint16_t es;          // source element bytes
+};
+
+template <int NPTR>
+struct BulkArgs {
+    const void* items;           // rr_pack_item (MODE 0) or rr_unpack_item
+    const uint32_t* block_first; // as in PackArgs
+    uint32_t item_begin;
+    uint32_t item_end;
+    char* bucket_base;
+    uint64_t bucket_stride;
+    int32_t n_shards;            // pack: ptr[0 .. n_shards) are the shards
+    int32_t dst_base;            // unpack: index in ptr[] of destination tensor 0
+    unsigned long long* sums;    // pack: checksums by bucket; verify: range sums
+    unsigned long long* counters;
+    const unsigned long long* expected;
+    uint8_t* bad;
+    int32_t first_bucket;
+    int32_t n_buckets;
+    unsigned int* err;
+    const void* ptr[NPTR];
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned int* err) {
+    for (uint32_t it = 0; it < kWaitLimit; ++it) {
+        uint32_t done;
+        asm volatile(
+            "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; "
+            "selp.u32 %0, 1, 0, p; }"
+            : "=r"(done)
+            : "r"(bar), "r"(parity), "n"(kWaitHintNs)
+            : "memory");
+        if (done) return true;
+    }
+    atomicExch(err, kErrWaitTimeout);
+    return false;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void consumers_sync() {
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * kConsumerWarps) : "memory");
+}
+
+template <int NPTR>
+__device__ __forceinline__ char* bulk_bucket(const BulkArgs<NPTR>& a, uint32_t b, int table_base) {
+    return a.bucket_stride ? a.bucket_base + (uint64_t)b * a.bucket_stride
+                           : (char*)a.ptr[table_base + b];
+}
+
+// MODE 0: pack, 1: unpack, 2: unpack with checksum comparison.
+template <int NPTR, int MODE>
+__global__ void __launch_bounds__(kBulkThreads, 1) rr_bulk_kernel(const __grid_constant__ BulkArgs<NPTR> a) {
+    extern __shared__ __align__(128) char stage_mem[];
+    __shared__ __align__(8) uint64_t full[kStages], empty[kStages];
+    __shared__ Piece meta[kStages];
+    __shared__ bool last_block;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr bool kSum = MODE != 1;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full[s])) : "memory");
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(&empty[s])),
+                         "n"(kConsumerWarps)
+                         : "memory");
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+
+    uint32_t i0, i1;
+    block_items(a.block_first, a.item_begin, a.item_end, &i0, &i1);
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane != 0) return;
+        uint32_t count = 0;   // pieces issued
+        bool ok = true;
+        auto emit = [&](const Piece& p, bool bulk) {
+            const int s = (int)(count % kStages);
+            if (count >= (uint32_t)kStages &&
+                !mbar_wait(smem_u32(&empty[s]), ((count / kStages) - 1) & 1, a.err)) {
+                ok = false;
+                return;
+            }
+            meta[s] = p;
+            const uint32_t fb = smem_u32(&full[s]);
+            if (bulk) {
+                const uint32_t row_bytes = p.row_len * p.es;
+                asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb),
+                             "r"(row_bytes * p.rows)
+                             : "memory");
+                for (uint32_t r = 0; r < p.rows; ++r)
+                    asm volatile(
+                        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes "
+                        "[%0], [%1], %2, [%3];" ::"r"(smem_u32(stage_mem + s * kStageBytes +
+                                                               r * row_bytes)),
+                        "l"(p.src + r * p.src_stride), "r"(row_bytes), "r"(fb)
+                        : "memory");
+            } else {
+                mbar_arrive(fb);
+            }
+            ++count;
+        };
+        for (uint32_t it = i0; it < i1 && ok; ++it) {
+            Piece p;
+            p.dst = nullptr;
+            p.src_stride = 0;
+            if (MODE == 0) {
+                const rr_pack_item d = ((const rr_pack_item*)a.items)[it];
+                char* dst = bulk_bucket(a, d.bucket, a.n_shards) + d.dst_off;
+                const char* src = (const char*)a.ptr[d.src >> 48] + (d.src & 0xFFFFFFFFFFFFull);
+                p.sum_bucket = d.bucket;
+                if (d.kind == RR_ITEM_F32_VEC || d.kind == RR_ITEM_BF16_VEC) {
+                    const uint32_t es = d.kind == RR_ITEM_F32_VEC ? 4 : 2;
+                    const uint32_t L = d.row_len, R = d.n_rows;
+                    const uint64_t sstride = (uint64_t)d.src_stride * es;
+                    p.kind = es == 4 ? PC_CAST : PC_COPY;
+                    p.es = (uint16_t)es;
+                    if (R == 1 || L * es > (uint32_t)kStageBytes) {
+                        const uint32_t step = kStageBytes / es;
+                        for (uint32_t r = 0; r < R && ok; ++r)
+                            for (uint32_t e0 = 0; e0 < L && ok; e0 += step) {
+                                p.n = min(step, L - e0);
+                                p.rows = 1;
+                                p.row_len = p.n;
+                                p.src = src + r * sstride + (uint64_t)e0 * es;
+                                p.dst = dst + 2ull * ((uint64_t)r * L + e0);
+                                p.sum_off = d.dst_off + 2u * (r * L + e0);
+                                emit(p, true);
+                            }
+                    } else {
+                        const uint32_t k = kStageBytes / (L * es);
+                        for (uint32_t r0 = 0; r0 < R && ok; r0 += k) {
+                            p.rows = min(k, R - r0);
+                            p.row_len = L;
+                            p.n = p.rows * L;
+                            p.src_stride = sstride;
+                            p.src = src + r0 * sstride;
+                            p.dst = dst + 2ull * r0 * L;
+                            p.sum_off = d.dst_off + 2u * r0 * L;
+                            emit(p, true);
+                        }
+                    }
+                } else if (d.kind == RR_ITEM_ZERO_VEC || d.kind == RR_ITEM_ZERO_SCALAR) {
+                    p.kind = d.kind == RR_ITEM_ZERO_VEC ? PC_ZERO_VEC : PC_ZERO_SCALAR;
+                    p.dst = dst;
+                    p.n = d.row_len;
+                    p.rows = 1;
+                    p.row_len = d.row_len;
+                    p.es = 2;
+                    p.src = nullptr;
+                    p.sum_off = d.dst_off;
+                    emit(p, false);
+                } else {
+                    p.kind = PC_SCALAR;
+                    p.es = d.kind == RR_ITEM_F32_SCALAR ? 4 : 2;
+                    p.src = src;
+                    p.dst = dst;
+                    p.rows = d.n_rows;
+                    p.row_len = d.row_len;
+                    p.n = d.row_len * d.n_rows;
+                    p.src_stride = (uint64_t)d.src_stride * p.es;
+                    p.sum_off = d.dst_off;
+                    emit(p, false);
+                }
+            } else {
+                const rr_unpack_item d = ((const rr_unpack_item*)a.items)[it];
+                const bool read_only = d.kind == RR_ITEM_READ_VEC || d.kind == RR_ITEM_READ_SCALAR;
+                if (MODE == 1 && read_only) continue;
+                const char* src = bulk_bucket(a, d.bucket, 0) + d.src_off;
+                char* dst = read_only ? nullptr : (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off;
+                p.sum_bucket = d.bucket;
+                p.es = 2;
+                if (d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_READ_VEC) {
+                    p.kind = read_only ? PC_READ : PC_COPY;
+                    for (uint32_t o = 0; o < d.nbytes && ok; o += kStageBytes) {
+                        const uint32_t len = min((uint32_t)kStageBytes, d.nbytes - o);
+                        p.n = len / 2;
+                        p.rows = 1;
+                        p.row_len = p.n;
+                        p.src = src + o;
+                        p.dst = dst ? dst + o : nullptr;
+                        p.sum_off = d.src_off + o;
+                        emit(p, true);
+                    }
+                } else {
+                    p.kind = PC_SCALAR;
+                    p.src = src;
+                    p.dst = dst;
+                    p.n = d.nbytes / 2;
+                    p.rows = 1;
+                    p.row_len = p.n;
+                    p.sum_off = d.src_off;
+                    emit(p, false);
+                }
+            }
+        }
+        if (ok) {
+            Piece end;
+            end.kind = PC_END;
+            emit(end, false);
+        }
+        if (!ok) {
+            // Let the loads still in flight land before this block's shared memory goes away.
+            const uint32_t from = count > (uint32_t)kStages ? count - kStages : 0;
+            for (uint32_t c = from; c < count; ++c)
+                mbar_wait(smem_u32(&full[c % kStages]), (c / kStages) & 1, a.err);
+        }
+        return;
+    }
+
+    // ---------------------------------------------------------------- consumers
+    const uint32_t ct = threadIdx.x - 32;
+    constexpr uint32_t kCT = 32 * kConsumerWarps;
+    const uint32_t sum_base = MODE == 2 ? (uint32_t)a.first_bucket : 0u;
+    unsigned long long acc = 0;
+    uint32_t cur = 0xFFFFFFFFu;
+    bool ok = true;
+    for (uint32_t c = 0;; ++c) {
+        const int s = (int)(c % kStages);
+        ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&full[s]), (c / kStages) & 1, a.err));
+        if (!ok) break;
+        const Piece p = meta[s];
+        if (p.kind == PC_END) break;
+        if (kSum && p.sum_bucket != cur) {
+            if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - sum_base), acc);
+            cur = p.sum_bucket;
+            acc = 0;
+        }
+        const char* st = stage_mem + s * kStageBytes;
+        const uint32_t nvec = p.n >> 3;
+        switch (p.kind) {
+            case PC_CAST:
+#pragma unroll 4
+                for (uint32_t v = ct; v < nvec; v += kCT) {
+                    const uint4 x0 = *(const uint4*)(st + 32ull * v);
+                    const uint4 x1 = *(const uint4*)(st + 32ull * v + 16);
+                    uint4 o;
+                    o.x = cast2(x0.x, x0.y);
+                    o.y = cast2(x0.z, x0.w);
+                    o.z = cast2(x1.x, x1.y);
+                    o.w = cast2(x1.z, x1.w);
+                    st_stream(p.dst + 16ull * v, o);
+                    acc += words(o);
+                }
+                break;
+            case PC_COPY:
+            case PC_READ:
+#pragma unroll 4
+                for (uint32_t v = ct; v < nvec; v += kCT) {
+                    const uint4 x = *(const uint4*)(st + 16ull * v);
+                    if (p.kind == PC_COPY) st_stream(p.dst + 16ull * v, x);
+                    if (kSum) acc += words(x);
+                }
+                break;
+            case PC_SCALAR:
+                for (uint32_t e = ct; e < p.n; e += kCT) {
+                    const uint32_t r = e / p.row_len, cc = e - r * p.row_len;
+                    const char* q = p.src + r * p.src_stride + (uint64_t)cc * p.es;
+                    const uint16_t h = p.es == 4 ? cast1(*(const uint32_t*)q) : *(const uint16_t*)q;
+                    if (p.dst) *(uint16_t*)(p.dst + 2ull * e) = h;
+                    if (kSum) acc += (unsigned long long)h << (8 * ((p.sum_off + 2 * e) & 7));
+                }
+                break;
+            case PC_ZERO_VEC:
+                for (uint32_t v = ct; v < nvec; v += kCT)
+                    st_stream(p.dst + 16ull * v, make_uint4(0, 0, 0, 0));
+                break;
+            default:  // PC_ZERO_SCALAR
+                for (uint32_t e = ct; e < p.n; e += kCT) *(uint16_t*)(p.dst + 2ull * e) = 0;
+                break;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
+    }
+    if (kSum && cur != 0xFFFFFFFFu) flush(a.sums + (cur - sum_base), acc);
+    if (MODE != 2) return;
+    // Checksum comparison by whichever block finishes last (consumer threads only).
+    consumers_sync();
+    if (ct == 0) {
+        __threadfence();
+        last_block = atomicAdd(&a.counters[0], 1ull) == gridDim.x - 1;
+    }
+    consumers_sync();
+    if (!last_block) return;
+    __threadfence();
+    for (int32_t i = ct; i < a.n_buckets; i += kCT) {
+        const int32_t b = a.first_bucket + i;
+        const bool differs = __ldcg(a.sums + i) != a.expected[b];
+        if (a.bad) a.bad[i] = differs ? 1 : 0;
+        if (differs) {
+            atomicAdd(&a.counters[1], 1ull);
+            atomicMax(&a.counters[2], ULLONG_MAX - (unsigned long long)b);
+        }
+    }
+}
+
+constexpr int kBulkSmem = kStages * kStageBytes;
+
+template <int NPTR, int MODE>
+cudaError_t bulk_prepare() {
+    return cudaFuncSetAttribute(rr_bulk_kernel<NPTR, MODE>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, kBulkSmem);
+}
+
+// ---------------------------------------------------------------------------
 // Host helpers
 // ---------------------------------------------------------------------------
 
@@ -514,7 +869,7 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
         a.bucket_base = (char*)buckets[0];
         a.bucket_stride = stride;
     }
-    rr_pack_kernel<NPTR><<<P->grid_blocks, kThreads, 0, s>>>(a);
+    rr_pack_kernel<NPTR><<<P->reg_pack_grid, kThreads, 0, s>>>(a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -548,9 +903,9 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     a.dst_base = k;
     for (int32_t t = 0; t < P->n_tensors; ++t) a.ptr[k++] = dst[t];
     if (checksums)
-        rr_unpack_kernel<NPTR, true><<<P->unpack_grid_blocks, kThreads, 0, s>>>(a);
+        rr_unpack_kernel<NPTR, true><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
     else
-        rr_unpack_kernel<NPTR, false><<<P->unpack_grid_blocks, kThreads, 0, s>>>(a);
+        rr_unpack_kernel<NPTR, false><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -583,6 +938,85 @@ rr_status launch_verify(const rr_plan* P, Range R, const void* const* buckets,
     return RR_OK;
 }
 
+// The bulk engine reads and writes device memory only; buffers in host memory
+// (a snapshot to pinned host buckets) take the register path.  One call's
+// arrays are expected to be all device or all host memory: the first and
+// last pointer of each array are checked.
+bool device_resident(const void* p) {
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice;
+}
+
+bool all_device(const void* const* ptrs, int32_t n) {
+    return n == 0 || (device_resident(ptrs[0]) && device_resident(ptrs[n - 1]));
+}
+
+template <int NPTR, int MODE>
+rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
+                      const void* const* buckets, void* const* dst, const uint64_t* checksums,
+                      uint8_t* bad, bool table, uint64_t stride, cudaStream_t s) {
+    BulkArgs<NPTR> a;
+    std::memset(&a, 0, sizeof a);
+    a.err = P->d_error;
+    int32_t k = 0;
+    if (MODE == 0) {
+        a.items = P->d_pack_items;
+        a.block_first = R.full ? P->d_pack_block_first : nullptr;
+        a.item_begin = P->pack_bucket_first[R.b0];
+        a.item_end = P->pack_bucket_first[R.b1];
+        a.sums = (unsigned long long*)checksums;
+        a.n_shards = P->n_shards;
+        for (int32_t i = 0; i < P->n_shards; ++i) a.ptr[k++] = src_shards[i];
+    } else {
+        a.items = P->d_unpack_items;
+        a.block_first = R.full ? P->d_unpack_block_first : nullptr;
+        a.item_begin = P->unpack_bucket_first[R.b0];
+        a.item_end = P->unpack_bucket_first[R.b1];
+        if (MODE == 2) {
+            a.sums = P->d_verify_scratch;
+            a.counters = P->d_verify_scratch + (R.b1 - R.b0);
+            a.expected = (const unsigned long long*)checksums;
+            a.bad = bad;
+            a.first_bucket = R.b0;
+            a.n_buckets = R.b1 - R.b0;
+        }
+    }
+    if (table) {
+        for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[k++] = buckets[b];
+    } else {
+        a.bucket_base = (char*)buckets[0];
+        a.bucket_stride = stride;
+    }
+    if (MODE != 0) {
+        a.dst_base = k;
+        for (int32_t t = 0; t < P->n_tensors; ++t) a.ptr[k++] = dst[t];
+    }
+    RR_CUDA((bulk_prepare<NPTR, MODE>()));
+    const int32_t grid = MODE == 0 ? P->grid_blocks : P->unpack_grid_blocks;
+    rr_bulk_kernel<NPTR, MODE><<<grid, kBulkThreads, kBulkSmem, s>>>(a);
+    RR_CUDA(cudaGetLastError());
+    return RR_OK;
+}
+
+// Synchronises `stream` and reports (then clears) the plan's error word.
+rr_status read_error(const rr_plan* P, cudaStream_t stream) {
+    unsigned int* h = (unsigned int*)(P->h_verify_result + 4);
+    RR_CUDA(cudaMemcpyAsync(h, P->d_error, sizeof(unsigned int), cudaMemcpyDeviceToHost, stream));
+    RR_CUDA(cudaStreamSynchronize(stream));
+    if (*h) {
+        const unsigned int code = *h;
+        RR_CUDA(cudaMemsetAsync(P->d_error, 0, sizeof(unsigned int), stream));
+        RR_CUDA(cudaStreamSynchronize(stream));
+        return rr_fail(RR_ECUDA, "a kernel of this plan gave up waiting (code %u); its output "
+                                 "is incomplete", code);
+    }
+    return RR_OK;
+}
+
 rr_status check_range(const rr_plan* P, int32_t first, int32_t n, Range* R) {
     if (first < 0 || n < 0 || first > P->n_buckets || n > P->n_buckets - first)
         return rr_fail(RR_EINVAL, "bucket range [%d, %d + %d) outside [0, %d)", first, first, n,
@@ -608,9 +1042,18 @@ rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, vo
                        P->n_shards, P->n_buckets, kLargePtrs);
     RR_CUDA(cudaMemsetAsync(checksums + R.b0, 0, size_t(R.b1 - R.b0) * 8, stream));
     if (P->pack_bucket_first[R.b0] == P->pack_bucket_first[R.b1]) return RR_OK;
+    const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(src_shards, P->n_shards) &&
+                      all_device((const void* const*)buckets, P->n_buckets);
+    if (bulk)
+        return need <= kSmallPtrs
+                   ? launch_bulk<kSmallPtrs, 0>(P, R, src_shards, (const void* const*)buckets,
+                                                nullptr, checksums, nullptr, table, stride, stream)
+                   : launch_bulk<kLargePtrs, 0>(P, R, src_shards, (const void* const*)buckets,
+                                                nullptr, checksums, nullptr, table, stride, stream);
+    const Range Rr{R.b0, R.b1, R.full && P->engine == RR_ENGINE_REGISTERS};
     return need <= kSmallPtrs
-               ? launch_pack<kSmallPtrs>(P, R, src_shards, buckets, checksums, table, stride, stream)
-               : launch_pack<kLargePtrs>(P, R, src_shards, buckets, checksums, table, stride, stream);
+               ? launch_pack<kSmallPtrs>(P, Rr, src_shards, buckets, checksums, table, stride, stream)
+               : launch_pack<kLargePtrs>(P, Rr, src_shards, buckets, checksums, table, stride, stream);
 }
 
 rr_status check_dst(const rr_plan* P, void* const* dst) {
@@ -638,19 +1081,30 @@ rr_status unpack_impl(const rr_plan* P, Range R, const void* const* buckets, voi
     if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
     if ((st = check_dst(P, dst))) return st;
     if (P->unpack_bucket_first[R.b0] == P->unpack_bucket_first[R.b1]) return RR_OK;
+    const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
+                      all_device((const void* const*)dst, P->n_tensors);
+    const Range Rr{R.b0, R.b1, R.full && !bulk && P->engine == RR_ENGINE_REGISTERS};
     return with_unpack_shape(P, buckets, [&](bool small, bool table, uint64_t stride) {
-        return small ? launch_unpack<kSmallPtrs>(P, R, buckets, dst, nullptr, nullptr, table,
+        if (bulk)
+            return small ? launch_bulk<kSmallPtrs, 1>(P, R, nullptr, buckets, dst, nullptr, nullptr,
+                                                      table, stride, stream)
+                         : launch_bulk<kLargePtrs, 1>(P, R, nullptr, buckets, dst, nullptr, nullptr,
+                                                      table, stride, stream);
+        return small ? launch_unpack<kSmallPtrs>(P, Rr, buckets, dst, nullptr, nullptr, table,
                                                  stride, stream)
-                     : launch_unpack<kLargePtrs>(P, R, buckets, dst, nullptr, nullptr, table,
+                     : launch_unpack<kLargePtrs>(P, Rr, buckets, dst, nullptr, nullptr, table,
                                                  stride, stream);
     });
 }
+
+rr_status read_error(const rr_plan* P, cudaStream_t stream);
 
 rr_status read_result(const rr_plan* P, int32_t n, int64_t* n_bad, int64_t* first_bad,
                       cudaStream_t stream) {
     RR_CUDA(cudaMemcpyAsync(P->h_verify_result, P->d_verify_scratch + n,
                             4 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, stream));
-    RR_CUDA(cudaStreamSynchronize(stream));
+    rr_status st = read_error(P, stream);
+    if (st) return st;
     const unsigned long long nb = P->h_verify_result[1];
     if (n_bad) *n_bad = (int64_t)nb;
     if (first_bad) *first_bad = nb ? (int64_t)(ULLONG_MAX - P->h_verify_result[2]) : -1;
@@ -673,10 +1127,18 @@ rr_status unpack_verify_impl(const rr_plan* P, Range R, const void* const* bucke
     const int32_t n = R.b1 - R.b0;
     RR_CUDA(cudaMemsetAsync(P->d_verify_scratch, 0, (size_t(n) + 4) * sizeof(unsigned long long),
                             stream));
+    const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
+                      all_device((const void* const*)dst, P->n_tensors);
+    const Range Rr{R.b0, R.b1, R.full && !bulk && P->engine == RR_ENGINE_REGISTERS};
     st = with_unpack_shape(P, buckets, [&](bool small, bool table, uint64_t stride) {
-        return small ? launch_unpack<kSmallPtrs>(P, R, buckets, dst, checksums, bad, table, stride,
+        if (bulk)
+            return small ? launch_bulk<kSmallPtrs, 2>(P, R, nullptr, buckets, dst, checksums, bad,
+                                                      table, stride, stream)
+                         : launch_bulk<kLargePtrs, 2>(P, R, nullptr, buckets, dst, checksums, bad,
+                                                      table, stride, stream);
+        return small ? launch_unpack<kSmallPtrs>(P, Rr, buckets, dst, checksums, bad, table, stride,
                                                  stream)
-                     : launch_unpack<kLargePtrs>(P, R, buckets, dst, checksums, bad, table, stride,
+                     : launch_unpack<kLargePtrs>(P, Rr, buckets, dst, checksums, bad, table, stride,
                                                  stream);
     });
     if (st) return st;
@@ -717,16 +1179,20 @@ rr_status verify_impl(const rr_plan* P, Range R, const void* const* buckets,
 // Plan device state
 // ---------------------------------------------------------------------------
 
-rr_status rr_device_default_grid(int32_t* pack, int32_t* unpack, int32_t* verify) {
-    int dev = 0, sms = 0, p = 0, u = 0, v = 0;
+rr_status rr_device_default_grid(rr_grids* g) {
+    int dev = 0, sms = 0, p = 0, u = 0, v = 0, b = 0;
     RR_CUDA(cudaGetDevice(&dev));
     RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, true>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, rr_verify_kernel<kLargePtrs>, kThreads, 0));
-    *pack = sms * (p > 0 ? p : 1);
-    *unpack = sms * (u > 0 ? u : 1);
-    *verify = sms * (v > 0 ? v : 1);
+    RR_CUDA((bulk_prepare<kLargePtrs, 2>()));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, rr_bulk_kernel<kLargePtrs, 2>,
+                                                          kBulkThreads, kBulkSmem));
+    g->reg_pack = sms * (p > 0 ? p : 1);
+    g->reg_unpack = sms * (u > 0 ? u : 1);
+    g->verify = sms * (v > 0 ? v : 1);
+    g->bulk_pack = g->bulk_unpack = sms * (b > 0 ? b : 1);
     return RR_OK;
 }
 
@@ -748,8 +1214,10 @@ rr_status rr_device_upload(rr_plan* P) {
                 P->unpack_block_first.size() * sizeof(uint32_t))) != cudaSuccess ||
         (e = cudaMalloc((void**)&P->d_verify_scratch,
                         (size_t(P->n_buckets) + 4) * sizeof(unsigned long long))) != cudaSuccess ||
-        (e = cudaHostAlloc((void**)&P->h_verify_result, 4 * sizeof(unsigned long long),
-                           cudaHostAllocDefault)) != cudaSuccess)
+        (e = cudaHostAlloc((void**)&P->h_verify_result, 5 * sizeof(unsigned long long),
+                           cudaHostAllocDefault)) != cudaSuccess ||
+        (e = cudaMalloc((void**)&P->d_error, sizeof(unsigned int))) != cudaSuccess ||
+        (e = cudaMemset(P->d_error, 0, sizeof(unsigned int))) != cudaSuccess)
         return e == cudaErrorMemoryAllocation ? rr_fail(RR_ENOMEM, "device allocation failed")
                                               : cuda_fail(e, "plan upload");
     return RR_OK;
@@ -766,6 +1234,8 @@ void rr_device_release(rr_plan* P) {
     cudaFree(P->d_unpack_block_first);
     cudaFree(P->d_verify_scratch);
     cudaFreeHost(P->h_verify_result);
+    cudaFree(P->d_error);
+    P->d_error = nullptr;
     P->d_pack_items = nullptr;
     P->d_pack_block_first = nullptr;
     P->d_unpack_items = nullptr;
@@ -857,6 +1327,15 @@ extern "C" rr_status rr_unpack_verify_range(const rr_plan* P, int32_t first_buck
     rr_status st = check_plan(P);
     if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
     return unpack_verify_impl(P, R, buckets, checksums, dst, bad, n_bad, first_bad, stream);
+}
+
+extern "C" rr_status rr_plan_check(const rr_plan* P, cudaStream_t stream) {
+    rr_clear_error();
+    rr_status st = check_plan(P);
+    if (st) return st;
+    rr_plan* M = const_cast<rr_plan*>(P);   // shares the pinned result buffer with verify
+    std::lock_guard<std::mutex> lock(M->verify_mutex);
+    return read_error(P, stream);
 }
 
 extern "C" rr_status rr_clear_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,

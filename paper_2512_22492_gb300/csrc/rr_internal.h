@@ -33,9 +33,12 @@ struct rr_plan {
     int32_t n_buckets = 0;
 
     // ---- work tables ----------------------------------------------------
-    int32_t grid_blocks = 0;          // pack kernel grid
-    int32_t unpack_grid_blocks = 0;
+    int32_t grid_blocks = 0;          // pack kernel grid (the partition's block count)
+    int32_t unpack_grid_blocks = 0;   // unpack kernel grid (likewise)
     int32_t verify_grid_blocks = 0;
+    int32_t reg_pack_grid = 0;        // register-path grids when the bulk engine is the default
+    int32_t reg_unpack_grid = 0;
+    int32_t engine = RR_ENGINE_AUTO;
     int64_t chunk_bytes = 0;
     bool host_only = false;
     std::vector<rr_pack_item> pack_items;
@@ -53,7 +56,8 @@ struct rr_plan {
     rr_unpack_item* d_unpack_items = nullptr;
     uint32_t* d_unpack_block_first = nullptr;
     unsigned long long* d_verify_scratch = nullptr;  // n_buckets sums + 4 counters
-    unsigned long long* h_verify_result = nullptr;   // pinned, 4 words
+    unsigned long long* h_verify_result = nullptr;   // pinned, 5 words (4 counters + error)
+    unsigned int* d_error = nullptr;                 // set by a kernel whose wait ran out
     std::mutex verify_mutex;
 };
 
@@ -62,6 +66,9 @@ rr_status rr_fail(rr_status s, const char* fmt, ...);
 void rr_clear_error();
 
 // Device side (rr_device.cu).
-rr_status rr_device_default_grid(int32_t* pack, int32_t* unpack, int32_t* verify);
+struct rr_grids {
+    int32_t bulk_pack, bulk_unpack, reg_pack, reg_unpack, verify;
+};
+rr_status rr_device_default_grid(rr_grids* g);
 rr_status rr_device_upload(rr_plan* p);
 void rr_device_release(rr_plan* p);

@@ -62,7 +62,7 @@ class _DstLayout(ctypes.Structure):
 
 class _Options(ctypes.Structure):
     _fields_ = [("host_only", ctypes.c_int32), ("grid_blocks", ctypes.c_int32),
-                ("chunk_bytes", ctypes.c_int64)]
+                ("chunk_bytes", ctypes.c_int64), ("engine", ctypes.c_int32)]
 
 
 class _Stats(ctypes.Structure):
@@ -144,6 +144,7 @@ _sig("rr_clear_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp)
 _sig("rr_plan_bucket_items", [_vp, ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_uint32)])
 _sig("rr_verify_noalloc", [ctypes.POINTER(_vp), ctypes.c_int32, ctypes.c_size_t, _vp, _P64, _P64,
                            _vp])
+_sig("rr_plan_check", [_vp, _vp])
 _sig("rr_status_str", [ctypes.c_int], ctypes.c_char_p)
 _sig("rr_last_error", [], ctypes.c_char_p)
 
@@ -154,7 +155,7 @@ EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_q
             "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
             "rr_unpack_verify", "rr_unpack_verify_range",
             "rr_verify_noalloc",
-            "rr_status_str", "rr_last_error")
+            "rr_plan_check", "rr_status_str", "rr_last_error")
 
 
 class RRError(RuntimeError):
@@ -227,6 +228,7 @@ class PlanOptions:
     host_only: bool = False
     grid_blocks: int = 0
     chunk_bytes: int = 0
+    engine: str = "auto"      # "auto" (bulk-copy engine for device buffers) or "registers"
 
 
 # ---------------------------------------------------------------------------
@@ -370,7 +372,8 @@ def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
                                  ctypes.byref(out))
     else:
         co = _Options(host_only=int(options.host_only), grid_blocks=options.grid_blocks,
-                      chunk_bytes=options.chunk_bytes)
+                      chunk_bytes=options.chunk_bytes,
+                      engine={"auto": 0, "registers": 1}[options.engine])
         st = _lib.rr_plan_create_ex(cp, n, ctypes.byref(cs), ctypes.byref(cd), bucket_bytes,
                                     ctypes.byref(co), ctypes.byref(out))
     _check(st, "rr_plan_create")
@@ -556,6 +559,11 @@ def rr_clear_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, strea
     _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
     _check(_lib.rr_clear_range(plan.handle, first_bucket, n_buckets, _ptr_array(buckets),
                                _stream(stream)), "rr_clear_range")
+
+
+def rr_plan_check(plan: Plan, stream=None) -> None:
+    """Raise if a kernel of this plan gave up on a bounded wait (waits for `stream`)."""
+    _check(_lib.rr_plan_check(plan.handle, _stream(stream)), "rr_plan_check")
 
 
 def rr_verify_noalloc(buckets, n_buckets: int, bucket_bytes: int, checksums, stream=None):

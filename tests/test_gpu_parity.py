@@ -95,7 +95,20 @@ def test_small_chunks_and_buckets(chunk):
 
 @pytest.mark.parametrize("seed", range(24))
 def test_random_layouts(seed):
-    full_parity(U.random_layout(seed), separate_buckets=bool(seed % 2))
+    full_parity(U.random_layout(seed), separate_buckets=bool(seed % 2),
+                engine="registers" if seed % 3 == 0 else "auto")
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-moe-f32", "tiny-fsdp2"])
+def test_register_engine(name):
+    """The register path (the fallback for host-resident buffers) on device memory."""
+    full_parity(U.workload_desc(name), engine="registers")
+
+
+@pytest.mark.parametrize("chunk", [16, 1040, 65536, 1 << 20])
+def test_bulk_engine_piece_splits(chunk):
+    """Items longer than a shared-memory stage and multi-row items split into pieces."""
+    full_parity(U.workload_desc("tiny-moe-f32", bucket_bytes=256 * 1024), chunk_bytes=chunk)
 
 
 @pytest.mark.parametrize("grid", [1, 3, 1000])
@@ -106,6 +119,10 @@ def test_grid_sizes(grid):
 def test_qwen3_0_6b_full():
     """Qwen3-0.6B, 8 fp32 shards -> TP=1, 32 MiB buckets: every byte compared."""
     full_parity(U.workload_desc("qwen3-0.6b"))
+
+
+def test_qwen3_0_6b_full_register_engine():
+    full_parity(U.workload_desc("qwen3-0.6b"), engine="registers")
 
 
 def test_device_generator_matches_host():
