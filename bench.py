@@ -327,6 +327,9 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     value = aggregate_gbs(world, step_bytes, ms_per_step)
 
     # Breakdown only (not part of the step): the receiver's two separate calls.
+    for _ in range(2):
+        H.unpack(buf, stream)
+        H.verify(buf, stream)
     sep = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(3)]
     for e in sep:
         e[0].record(stream)

@@ -455,10 +455,34 @@ __global__ void __launch_bounds__(kThreads, 4) rr_verify_kernel(const __grid_con
 // lets its block's loads land, and returns (the host reports it as RR_ECUDA).
 // ---------------------------------------------------------------------------
 
-constexpr int kConsumerWarps = 8;
-constexpr int kBulkThreads = 32 * (kConsumerWarps + 1);
-constexpr int kStageBytes = 32 * 1024;
-constexpr int kStages = 3;
+// Stage ring shape per direction (build-time overridable for tuning sweeps).
+#ifndef RR_PACK_STAGE_KB
+#define RR_PACK_STAGE_KB 48
+#endif
+#ifndef RR_PACK_STAGES
+#define RR_PACK_STAGES 3
+#endif
+#ifndef RR_PACK_WARPS
+#define RR_PACK_WARPS 8
+#endif
+#ifndef RR_UNPACK_STAGE_KB
+#define RR_UNPACK_STAGE_KB 32
+#endif
+#ifndef RR_UNPACK_STAGES
+#define RR_UNPACK_STAGES 3
+#endif
+#ifndef RR_UNPACK_WARPS
+#define RR_UNPACK_WARPS 4
+#endif
+
+template <int MODE>
+struct BulkShape {
+    static constexpr int kWarps = MODE == 0 ? RR_PACK_WARPS : RR_UNPACK_WARPS;
+    static constexpr int kStageBytes = (MODE == 0 ? RR_PACK_STAGE_KB : RR_UNPACK_STAGE_KB) * 1024;
+    static constexpr int kStages = MODE == 0 ? RR_PACK_STAGES : RR_UNPACK_STAGES;
+    static constexpr int kThreads = 32 * (kWarps + 1);
+    static constexpr int kSmem = kStages * kStageBytes;
+};
 constexpr uint32_t kWaitLimit = 1u << 20;     // x at most kWaitHintNs each: about a second
 constexpr uint32_t kWaitHintNs = 1000;
 constexpr unsigned int kErrWaitTimeout = 1;
@@ -529,8 +553,9 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
+template <int kConsumerThreads>
 __device__ __forceinline__ void consumers_sync() {
-    asm volatile("bar.sync 1, %0;" ::"n"(32 * kConsumerWarps) : "memory");
+    asm volatile("bar.sync 1, %0;" ::"n"(kConsumerThreads) : "memory");
 }
 
 template <int NPTR>
@@ -541,7 +566,10 @@ __device__ __forceinline__ char* bulk_bucket(const BulkArgs<NPTR>& a, uint32_t b
 
 // MODE 0: pack, 1: unpack, 2: unpack with checksum comparison.
 template <int NPTR, int MODE>
-__global__ void __launch_bounds__(kBulkThreads, 1) rr_bulk_kernel(const __grid_constant__ BulkArgs<NPTR> a) {
+__global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(const __grid_constant__ BulkArgs<NPTR> a) {
+    constexpr int kConsumerWarps = BulkShape<MODE>::kWarps;
+    constexpr int kStageBytes = BulkShape<MODE>::kStageBytes;
+    constexpr int kStages = BulkShape<MODE>::kStages;
     extern __shared__ __align__(128) char stage_mem[];
     __shared__ __align__(8) uint64_t full[kStages], empty[kStages];
     __shared__ Piece meta[kStages];
@@ -769,12 +797,12 @@ __global__ void __launch_bounds__(kBulkThreads, 1) rr_bulk_kernel(const __grid_c
     if (kSum && cur != 0xFFFFFFFFu) flush(a.sums + (cur - sum_base), acc);
     if (MODE != 2) return;
     // Checksum comparison by whichever block finishes last (consumer threads only).
-    consumers_sync();
+    consumers_sync<kCT>();
     if (ct == 0) {
         __threadfence();
         last_block = atomicAdd(&a.counters[0], 1ull) == gridDim.x - 1;
     }
-    consumers_sync();
+    consumers_sync<kCT>();
     if (!last_block) return;
     __threadfence();
     for (int32_t i = ct; i < a.n_buckets; i += kCT) {
@@ -788,12 +816,11 @@ __global__ void __launch_bounds__(kBulkThreads, 1) rr_bulk_kernel(const __grid_c
     }
 }
 
-constexpr int kBulkSmem = kStages * kStageBytes;
-
 template <int NPTR, int MODE>
 cudaError_t bulk_prepare() {
     return cudaFuncSetAttribute(rr_bulk_kernel<NPTR, MODE>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, kBulkSmem);
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                BulkShape<MODE>::kSmem);
 }
 
 // ---------------------------------------------------------------------------
@@ -997,7 +1024,8 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
     }
     RR_CUDA((bulk_prepare<NPTR, MODE>()));
     const int32_t grid = MODE == 0 ? P->grid_blocks : P->unpack_grid_blocks;
-    rr_bulk_kernel<NPTR, MODE><<<grid, kBulkThreads, kBulkSmem, s>>>(a);
+    rr_bulk_kernel<NPTR, MODE>
+        <<<grid, BulkShape<MODE>::kThreads, BulkShape<MODE>::kSmem, s>>>(a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -1186,13 +1214,20 @@ rr_status rr_device_default_grid(rr_grids* g) {
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, true>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, rr_verify_kernel<kLargePtrs>, kThreads, 0));
+    int bp = 0;
+    RR_CUDA((bulk_prepare<kLargePtrs, 0>()));
     RR_CUDA((bulk_prepare<kLargePtrs, 2>()));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bp, rr_bulk_kernel<kLargePtrs, 0>,
+                                                          BulkShape<0>::kThreads,
+                                                          BulkShape<0>::kSmem));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, rr_bulk_kernel<kLargePtrs, 2>,
-                                                          kBulkThreads, kBulkSmem));
+                                                          BulkShape<2>::kThreads,
+                                                          BulkShape<2>::kSmem));
     g->reg_pack = sms * (p > 0 ? p : 1);
     g->reg_unpack = sms * (u > 0 ? u : 1);
     g->verify = sms * (v > 0 ? v : 1);
-    g->bulk_pack = g->bulk_unpack = sms * (b > 0 ? b : 1);
+    g->bulk_pack = sms * (bp > 0 ? bp : 1);
+    g->bulk_unpack = sms * (b > 0 ? b : 1);
     return RR_OK;
 }
 
