@@ -494,8 +494,11 @@ enum : uint16_t {
     PC_SCALAR = 4,    // element by element from global memory
     PC_ZERO_VEC = 5,  // 16-byte zero stores
     PC_ZERO_SCALAR = 6,
-    PC_END = 7
+    PC_END = 7,
+    PC_GATHER = 8     // aligned rows too short for bulk copies: 16-byte loads by consumers
 };
+
+constexpr uint32_t kMinBulkRowBytes = 1024;
 
 struct Piece {
     const char* src;      // first source element (global)
@@ -556,6 +559,56 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 template <int kConsumerThreads>
 __device__ __forceinline__ void consumers_sync() {
     asm volatile("bar.sync 1, %0;" ::"n"(kConsumerThreads) : "memory");
+}
+
+// Rows of a PC_GATHER piece: 16-byte-aligned rows of row_len (a multiple of 8)
+// elements at src_stride, landing contiguously at dst.  Thread t of NT takes
+// 8-element vectors t, t + NT, ...; four in flight per thread.
+template <int ES, int NT>
+__device__ __forceinline__ unsigned long long gather_rows(const Piece& p, uint32_t t) {
+    constexpr int U = ES == 4 ? 4 : 8;
+    const uint32_t vpr = p.row_len >> 3;
+    const uint32_t nvec = vpr * p.rows;
+    const uint32_t dq = NT / vpr, dr = NT - dq * vpr;
+    uint32_t v = t, r = v / vpr, c = v - r * vpr;
+    unsigned long long acc = 0;
+    while (v < nvec) {
+        uint4 x[U][ES / 2];
+        uint32_t vv[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            vv[u] = v;
+            if (v < nvec) {
+                const char* q = p.src + r * p.src_stride + (uint64_t)c * (8 * ES);
+                x[u][0] = ld_stream(q);
+                if (ES == 4) x[u][ES / 2 - 1] = ld_stream(q + 16);
+            }
+            v += NT;
+            c += dr;
+            r += dq;
+            if (c >= vpr) {
+                c -= vpr;
+                ++r;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (vv[u] < nvec) {
+                uint4 o;
+                if (ES == 4) {
+                    o.x = cast2(x[u][0].x, x[u][0].y);
+                    o.y = cast2(x[u][0].z, x[u][0].w);
+                    o.z = cast2(x[u][ES / 2 - 1].x, x[u][ES / 2 - 1].y);
+                    o.w = cast2(x[u][ES / 2 - 1].z, x[u][ES / 2 - 1].w);
+                } else {
+                    o = x[u][0];
+                }
+                st_stream(p.dst + 16ull * vv[u], o);
+                acc += words(o);
+            }
+        }
+    }
+    return acc;
 }
 
 template <int NPTR>
@@ -649,6 +702,18 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                                 p.sum_off = d.dst_off + 2u * (r * L + e0);
                                 emit(p, true);
                             }
+                    } else if (L * es < kMinBulkRowBytes) {
+                        // Many short rows: one bulk copy per row would make the single
+                        // producer the bottleneck.  Consumers gather them directly.
+                        p.kind = PC_GATHER;
+                        p.src = src;
+                        p.dst = dst;
+                        p.rows = R;
+                        p.row_len = L;
+                        p.n = L * R;
+                        p.src_stride = sstride;
+                        p.sum_off = d.dst_off;
+                        emit(p, false);
                     } else {
                         const uint32_t k = kStageBytes / (L * es);
                         for (uint32_t r0 = 0; r0 < R && ok; r0 += k) {
@@ -781,6 +846,14 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     const uint16_t h = p.es == 4 ? cast1(*(const uint32_t*)q) : *(const uint16_t*)q;
                     if (p.dst) *(uint16_t*)(p.dst + 2ull * e) = h;
                     if (kSum) acc += (unsigned long long)h << (8 * ((p.sum_off + 2 * e) & 7));
+                }
+                break;
+            case PC_GATHER:   // pack only
+                if constexpr (MODE == 0) {
+                    if (p.es == 4)
+                        acc += gather_rows<4, kCT>(p, ct);
+                    else
+                        acc += gather_rows<2, kCT>(p, ct);
                 }
                 break;
             case PC_ZERO_VEC:
