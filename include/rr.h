@@ -361,6 +361,13 @@ rr_status rr_verify_noalloc(const void* const* buckets, int32_t n_buckets, size_
  * RR_OK otherwise.  rr_verify and rr_unpack_verify check this themselves. */
 rr_status rr_plan_check(const rr_plan* plan, cudaStream_t stream);
 
+/* Test hook for the bounded waits: enqueues on `stream` one small kernel that
+ * waits on a barrier nothing completes.  The wait gives up after its limit
+ * (about a second) and marks the plan, so the next rr_plan_check (or
+ * rr_verify / rr_unpack_verify) reports RR_ECUDA while the CUDA context stays
+ * usable.  It touches no buffer. */
+rr_status rr_plan_selftest_wait(const rr_plan* plan, cudaStream_t stream);
+
 const char* rr_status_str(rr_status status);
 const char* rr_last_error(void);
 

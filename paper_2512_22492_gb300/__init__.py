@@ -7,12 +7,13 @@ buffer again.  This package is the on-GPU part of that route for one GB300:
 a C-ABI CUDA library (``include/rr.h``, ``csrc/``) and its Python binding.
 """
 from .rr import (Block, DstLayout, DstTensor, Param, Plan, PlanOptions, RRError, SrcLayout,
-                 rr_clear_range, rr_pack, rr_pack_range, rr_plan_create, rr_status_str, rr_unpack,
+                 rr_clear_range, rr_pack, rr_pack_range, rr_plan_check, rr_plan_create,
+                 rr_plan_selftest_wait, rr_status_str, rr_unpack,
                  rr_unpack_range, rr_unpack_verify, rr_verify, rr_verify_range)
 from .layouts import qwen3_manifest, qwen3_rollout, qwen3_sync
 
 __all__ = ["Block", "DstLayout", "DstTensor", "Param", "Plan", "PlanOptions", "RRError",
            "SrcLayout", "rr_pack", "rr_plan_create", "rr_status_str", "rr_unpack", "rr_verify",
            "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
-           "rr_unpack_verify",
+           "rr_unpack_verify", "rr_plan_check", "rr_plan_selftest_wait",
            "qwen3_manifest", "qwen3_rollout", "qwen3_sync"]

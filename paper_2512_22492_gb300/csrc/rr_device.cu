@@ -483,8 +483,9 @@ struct BulkShape {
     static constexpr int kThreads = 32 * (kWarps + 1);
     static constexpr int kSmem = kStages * kStageBytes;
 };
-constexpr uint32_t kWaitLimit = 1u << 20;     // x at most kWaitHintNs each: about a second
+constexpr uint32_t kWaitLimit = 1u << 20;        // tries, each suspending at most kWaitHintNs
 constexpr uint32_t kWaitHintNs = 1000;
+constexpr uint64_t kWaitDeadlineNs = 1000000000;  // and at most one second of wall clock
 constexpr unsigned int kErrWaitTimeout = 1;
 
 enum : uint16_t {
@@ -537,8 +538,16 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return (uint32_t)__cvta_generic_to_shared(p);
 }
 
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned int* err) {
+    const uint64_t t0 = global_ns();
     for (uint32_t it = 0; it < kWaitLimit; ++it) {
+        if ((it & 255) == 255 && global_ns() - t0 > kWaitDeadlineNs) break;
         uint32_t done;
         asm volatile(
             "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; "
@@ -887,6 +896,18 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
             atomicMax(&a.counters[2], ULLONG_MAX - (unsigned long long)b);
         }
     }
+}
+
+// Self-test of the bounded wait: waits on a barrier phase that nothing
+// completes; the wait gives up after its limit and marks the error word.
+__global__ void rr_wait_selftest_kernel(unsigned int* err) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&bar)) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) mbar_wait(smem_u32(&bar), 0, err);
 }
 
 template <int NPTR, int MODE>
@@ -1444,6 +1465,15 @@ extern "C" rr_status rr_plan_check(const rr_plan* P, cudaStream_t stream) {
     rr_plan* M = const_cast<rr_plan*>(P);   // shares the pinned result buffer with verify
     std::lock_guard<std::mutex> lock(M->verify_mutex);
     return read_error(P, stream);
+}
+
+extern "C" rr_status rr_plan_selftest_wait(const rr_plan* P, cudaStream_t stream) {
+    rr_clear_error();
+    rr_status st = check_plan(P);
+    if (st) return st;
+    rr_wait_selftest_kernel<<<1, 32, 0, stream>>>(P->d_error);
+    RR_CUDA(cudaGetLastError());
+    return RR_OK;
 }
 
 extern "C" rr_status rr_clear_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,

@@ -145,6 +145,7 @@ _sig("rr_plan_bucket_items", [_vp, ctypes.POINTER(ctypes.c_uint32), ctypes.POINT
 _sig("rr_verify_noalloc", [ctypes.POINTER(_vp), ctypes.c_int32, ctypes.c_size_t, _vp, _P64, _P64,
                            _vp])
 _sig("rr_plan_check", [_vp, _vp])
+_sig("rr_plan_selftest_wait", [_vp, _vp])
 _sig("rr_status_str", [ctypes.c_int], ctypes.c_char_p)
 _sig("rr_last_error", [], ctypes.c_char_p)
 
@@ -155,7 +156,7 @@ EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_q
             "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
             "rr_unpack_verify", "rr_unpack_verify_range",
             "rr_verify_noalloc",
-            "rr_plan_check", "rr_status_str", "rr_last_error")
+            "rr_plan_check", "rr_plan_selftest_wait", "rr_status_str", "rr_last_error")
 
 
 class RRError(RuntimeError):
@@ -564,6 +565,11 @@ def rr_clear_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, strea
 def rr_plan_check(plan: Plan, stream=None) -> None:
     """Raise if a kernel of this plan gave up on a bounded wait (waits for `stream`)."""
     _check(_lib.rr_plan_check(plan.handle, _stream(stream)), "rr_plan_check")
+
+
+def rr_plan_selftest_wait(plan: Plan, stream=None) -> None:
+    """Enqueue the bounded-wait self-test kernel (see include/rr.h)."""
+    _check(_lib.rr_plan_selftest_wait(plan.handle, _stream(stream)), "rr_plan_selftest_wait")
 
 
 def rr_verify_noalloc(buckets, n_buckets: int, bucket_bytes: int, checksums, stream=None):

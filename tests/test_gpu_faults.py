@@ -2,11 +2,13 @@
 
 Section 5.2.2 of the paper has a rollout resume or redo a pull after a relay or
 trainer failure; the checksums let it tell which buckets it holds intact.
-Every fault here is made on the host side -- bits flipped, buckets zeroed,
-swapped, or never received, buffers that do not match the plan -- and
-checked through the C ABI.  No kernel waits on anything, so none can hang.
-Also: guard bytes around every output stay untouched, two streams share one
-plan, and repeated runs give identical bits.
+Every data fault here is made on the host side -- bits flipped, buckets
+zeroed, swapped, or never received, buffers that do not match the plan -- and
+checked through the C ABI.  The only device-side waits (the bulk engine's
+barriers) are bounded; the last test makes one run out on purpose, through a
+barrier that nothing completes, and checks that the host sees the status and
+the context stays usable.  Also: guard bytes around every output stay
+untouched, two streams share one plan, and repeated runs give identical bits.
 """
 import numpy as np
 import pytest
@@ -185,3 +187,30 @@ def test_empty_layout():
     rr.rr_pack(plan, shards, [], cs)
     rr.rr_unpack(plan, [], [])
     assert rr.rr_verify(plan, [], cs) == (0, -1)
+
+
+def test_bounded_wait_reports_and_context_survives():
+    """A device wait that nothing satisfies gives up after about a second, marks
+    the plan, and the host sees RR_ECUDA; afterwards the context still works and
+    results are still exact."""
+    import time
+    desc, plan, buf = packed("tiny-tp4")
+    rr.rr_plan_check(plan)                                  # clean
+    t0 = time.time()
+    rr.rr_plan_selftest_wait(plan)
+    with pytest.raises(rr.RRError) as e:
+        rr.rr_plan_check(plan)
+    assert e.value.status == rrmod.RR_ECUDA
+    assert time.time() - t0 < 30
+    rr.rr_plan_check(plan)                                  # the mark was cleared
+    # The verifying calls report a mark left by an earlier kernel too.
+    rr.rr_plan_selftest_wait(plan)
+    with pytest.raises(rr.RRError):
+        rr.rr_verify(plan, buf.buckets, buf.checksums)
+    # And the plan keeps working, bit for bit.
+    H.pack(buf)
+    assert rr.rr_verify(plan, buf.buckets, buf.checksums) == (0, -1)
+    assert rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst) == (0, -1)
+    L = U.to_oracle(desc)
+    want, _ = L.pack(oracle.Source(seed=desc["seed"], specials=desc["specials"]))
+    np.testing.assert_array_equal(H.buckets_host(buf), want)
