@@ -82,37 +82,43 @@ _lib: Optional[ctypes.CDLL] = None
 def lib() -> ctypes.CDLL:
     global _lib
     if _lib is None:
-        L = ctypes.CDLL(build())
-        LP = ctypes.POINTER(_Layout)
-        SP = ctypes.POINTER(_Source)
-        vp = ctypes.c_void_p
-        L.orc_layout_compute.argtypes = [LP]
-        L.orc_layout_compute.restype = ctypes.c_int
-        L.orc_rne_bf16.argtypes = [ctypes.c_uint32]
-        L.orc_rne_bf16.restype = ctypes.c_uint16
-        L.orc_rne_bf16_array.argtypes = [vp, vp, ctypes.c_int64]
-        L.orc_rne_bf16_array.restype = None
-        L.orc_tensor_elements.argtypes = [LP, SP, ctypes.c_int32, ctypes.c_int64,
-                                          ctypes.c_int64, vp]
-        L.orc_tensor_elements.restype = ctypes.c_int
-        L.orc_reshard_tensor.argtypes = [LP, SP, ctypes.c_int32, vp]
-        L.orc_reshard_tensor.restype = ctypes.c_int
-        L.orc_pack_bucket.argtypes = [LP, SP, ctypes.c_int64, vp]
-        L.orc_pack_bucket.restype = ctypes.c_int
-        L.orc_pack_range.argtypes = [LP, SP, ctypes.c_int64, ctypes.c_int64, vp, vp]
-        L.orc_pack_range.restype = ctypes.c_int
-        L.orc_checksum.argtypes = [vp, ctypes.c_int64]
-        L.orc_checksum.restype = ctypes.c_uint64
-        L.orc_unpack_tensor.argtypes = [LP, ctypes.POINTER(vp), ctypes.c_int32, vp]
-        L.orc_unpack_tensor.restype = ctypes.c_int
-        L.orc_unpack_elements.argtypes = [LP, ctypes.POINTER(vp), ctypes.c_int32, ctypes.c_int64,
-                                          ctypes.c_int64, vp]
-        L.orc_unpack_elements.restype = ctypes.c_int
-        L.orc_verify.argtypes = [LP, ctypes.POINTER(vp), vp, ctypes.c_int64, ctypes.c_int64,
-                                 _P64]
-        L.orc_verify.restype = ctypes.c_int64
-        _lib = L
+        _lib = load(build())
     return _lib
+
+
+def load(path: str) -> ctypes.CDLL:
+    """Load an oracle library build and declare its functions (the mutation
+    tests load deliberately broken builds this way)."""
+    L = ctypes.CDLL(path)
+    LP = ctypes.POINTER(_Layout)
+    SP = ctypes.POINTER(_Source)
+    vp = ctypes.c_void_p
+    L.orc_layout_compute.argtypes = [LP]
+    L.orc_layout_compute.restype = ctypes.c_int
+    L.orc_rne_bf16.argtypes = [ctypes.c_uint32]
+    L.orc_rne_bf16.restype = ctypes.c_uint16
+    L.orc_rne_bf16_array.argtypes = [vp, vp, ctypes.c_int64]
+    L.orc_rne_bf16_array.restype = None
+    L.orc_tensor_elements.argtypes = [LP, SP, ctypes.c_int32, ctypes.c_int64,
+                                      ctypes.c_int64, vp]
+    L.orc_tensor_elements.restype = ctypes.c_int
+    L.orc_reshard_tensor.argtypes = [LP, SP, ctypes.c_int32, vp]
+    L.orc_reshard_tensor.restype = ctypes.c_int
+    L.orc_pack_bucket.argtypes = [LP, SP, ctypes.c_int64, vp]
+    L.orc_pack_bucket.restype = ctypes.c_int
+    L.orc_pack_range.argtypes = [LP, SP, ctypes.c_int64, ctypes.c_int64, vp, vp]
+    L.orc_pack_range.restype = ctypes.c_int
+    L.orc_checksum.argtypes = [vp, ctypes.c_int64]
+    L.orc_checksum.restype = ctypes.c_uint64
+    L.orc_unpack_tensor.argtypes = [LP, ctypes.POINTER(vp), ctypes.c_int32, vp]
+    L.orc_unpack_tensor.restype = ctypes.c_int
+    L.orc_unpack_elements.argtypes = [LP, ctypes.POINTER(vp), ctypes.c_int32, ctypes.c_int64,
+                                      ctypes.c_int64, vp]
+    L.orc_unpack_elements.restype = ctypes.c_int
+    L.orc_verify.argtypes = [LP, ctypes.POINTER(vp), vp, ctypes.c_int64, ctypes.c_int64,
+                             _P64]
+    L.orc_verify.restype = ctypes.c_int64
+    return L
 
 
 def _check(rc: int, what: str) -> None:

@@ -122,6 +122,10 @@ TEST_WORKLOADS = {
                              bucket_bytes=40 * 1024, seed=16),
     "tiny-moe-f32": Workload("tiny-moe-f32", TINY_MOE, "f32", n_shards=5, tp=2,
                              bucket_bytes=24 * 1024, seed=17, specials=True),
+    # bf16 trainer state carrying the special bit patterns (signalling NaNs must
+    # pass through a bf16 -> bf16 copy untouched).
+    "tiny-moe-bf16-specials": Workload("tiny-moe-bf16-specials", TINY_MOE, "bf16", n_shards=4,
+                                       tp=2, bucket_bytes=32 * 1024, seed=21, specials=True),
     # FSDP2-style (each parameter cut on dim 0) trainers; uneven chunks.
     "tiny-fsdp2": Workload("tiny-fsdp2", TINY, "f32", n_shards=3, tp=2, bucket_bytes=48 * 1024,
                            seed=18, specials=True, sharding="rows"),

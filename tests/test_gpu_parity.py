@@ -63,7 +63,7 @@ def full_parity(desc, separate_buckets=False, **opts):
 
 @pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2",
                                   "tiny-moe-f32", "tiny-fsdp2", "tiny-moe-kvrep",
-                                  "tiny-kvrep-f32"])
+                                  "tiny-kvrep-f32", "tiny-moe-bf16-specials"])
 def test_small_workloads(name):
     full_parity(U.workload_desc(name))
 

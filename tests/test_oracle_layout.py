@@ -191,7 +191,7 @@ def fsdp2_shards(params, P, n, align=16):
 
 
 RESTATE = ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2", "tiny-moe-f32",
-           "tiny-fsdp2", "tiny-moe-kvrep", "tiny-kvrep-f32"]
+           "tiny-fsdp2", "tiny-moe-kvrep", "tiny-kvrep-f32", "tiny-moe-bf16-specials"]
 
 
 def _workload(name):
@@ -366,3 +366,17 @@ def test_rows_sharding_golden():
     buckets, cs = L.pack(src)
     assert [b.tobytes().hex() for b in buckets] == e["buckets_hex"]
     assert [int(c) for c in cs] == [_int(c) for c in e["checksums"]]
+
+
+def test_shard_size_rule_edge():
+    """Hand-derived: one bf16 parameter of 65 elements (130 bytes) over 4 flat
+    shards.  The total rounds up to a multiple of 16 * 4 = 64 bytes: 192, so
+    S = 48 (not 32: 4 x 32 = 128 bytes would not hold byte 129).  Element 64
+    (flat bytes 128-129) is shard 128 // 48 = 2, offset 128 - 96 = 32."""
+    L = oracle.Layout([("p", (65,), 2)], [("t", 0, [(0, 64, 1, 0, 1)])], n_shards=4, tp=1,
+                      bucket_bytes=16)
+    assert L.shard_bytes == 48
+    shards = [np.zeros(48, np.uint8) for _ in range(4)]
+    shards[2][32:34] = [0x34, 0x12]
+    got = L.reshard_tensor(oracle.Source(shards=shards), 0)
+    assert list(got) == [0x1234]

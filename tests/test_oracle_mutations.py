@@ -1,0 +1,118 @@
+"""The oracle's pins catch plausible mistakes.
+
+Each case below plants one mistake in a copy of oracle/rr_oracle.c -- a
+dropped term, a wrong bit, a transposed index, a missed alignment, a wrong
+byte order -- builds that copy on its own, and runs a battery of the pins
+(hand-worked golden examples, the brute-force cast check, the PyTorch
+restatement of the layout, the numpy checksum, round trip and verify) against
+it.  Every planted mistake must make the battery fail, and the real oracle must
+pass it.  Nothing here touches a GPU.
+"""
+import os
+import subprocess
+
+import numpy as np
+import pytest
+
+import oracle
+from tests import test_oracle_cast as cast_pins
+from tests import test_oracle_layout as layout_pins
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "rr_oracle.c")
+
+# (name, text in rr_oracle.c, replacement)
+MUTATIONS = [
+    ("nan loses the quiet bit", "return (uint16_t)((b >> 16) | 0x0040u);",
+     "return (uint16_t)(b >> 16);"),
+    ("round half up, not to even", "return (uint16_t)((b + 0x7FFFu + ((b >> 16) & 1u)) >> 16);",
+     "return (uint16_t)((b + 0x8000u) >> 16);"),
+    ("wrong kept bit", "((b >> 16) & 1u)", "((b >> 15) & 1u)"),
+    ("infinity taken for a NaN", "if ((b & 0x7FFFFFFFu) > 0x7F800000u)",
+     "if ((b & 0x7FFFFFFFu) >= 0x7F800000u)"),
+    ("bf16 source rounded again", "return elem_bytes == 4 ? orc_rne_bf16(bits) : (uint16_t)bits;",
+     "return orc_rne_bf16(bits << (elem_bytes == 2 ? 16 : 0));"),
+    ("block rows and columns transposed",
+     "int64_t row = B->row0 + jj / B->ncols;\n            int64_t col = B->col0 + jj % B->ncols;",
+     "int64_t row = B->row0 + jj % B->nrows;\n            int64_t col = B->col0 + jj / B->nrows;"),
+    ("parameters not aligned", "off = align_up(off, a);", "off = off + 0 * a;"),
+    ("tensors not aligned in the stream",
+     "int64_t start = align_up(L->rank_stream_bytes[T->rank], L->tensor_align);",
+     "int64_t start = L->rank_stream_bytes[T->rank];"),
+    ("shard size ignores the shard count",
+     "L->shard_bytes = align_up(flat_end, 16 * (int64_t)L->n_shards) / L->n_shards;",
+     "L->shard_bytes = align_up(flat_end / L->n_shards, 16);"),
+    ("big-endian checksum words", "word |= (uint64_t)bytes[k + i] << (8 * i);",
+     "word |= (uint64_t)bytes[k + i] << (8 * (7 - i));"),
+    ("buckets numbered from the wrong rank",
+     "L->rank_first_bucket[r + 1] = L->rank_first_bucket[r] + nb;",
+     "L->rank_first_bucket[r + 1] = nb;"),
+    ("unpack ignores the rank's first bucket",
+     "const uint8_t* bucket = buckets[first + pos / L->bucket_bytes];",
+     "const uint8_t* bucket = buckets[pos / L->bucket_bytes];"),
+    ("verify counts the good buckets",
+     "if (orc_checksum(buckets[b], L->bucket_bytes) != checksums[b]) {",
+     "if (orc_checksum(buckets[b], L->bucket_bytes) == checksums[b]) {"),
+    ("FSDP2 chunks rounded down", "int64_t c = (P->rows + L->n_shards - 1) / L->n_shards;",
+     "int64_t c = P->rows / L->n_shards + (P->rows < L->n_shards);"),
+    ("values indexed by the in-shard offset",
+     "L->param_gen_base[p] = start / P->elem_bytes;",
+     "L->param_gen_base[p] = (start % 4096) / P->elem_bytes;"),
+    ("little-endian source bytes read reversed", "v |= (uint32_t)byte << (8 * i);",
+     "v |= (uint32_t)byte << (8 * (es - 1 - i));"),
+]
+
+
+def battery():
+    """A compact run of the pins.  Returns the name of the first that fails, or None."""
+    checks = [
+        ("golden numbers", layout_pins.test_golden_layout_numbers),
+        ("golden values", layout_pins.test_golden_values),
+        ("rows golden", layout_pins.test_rows_sharding_golden),
+        ("cast named cases", cast_pins.test_named_cases),
+        ("cast structured", cast_pins.test_structured_against_brute_force),
+        ("cast NaN", cast_pins.test_nan_properties),
+        ("checksum", layout_pins.test_checksum_against_numpy_and_linearity),
+        ("verify", layout_pins.test_verify_flags_damage),
+        ("restatement tiny-tp4", lambda: layout_pins.test_oracle_matches_restatement("tiny-tp4")),
+        ("restatement tiny-moe-tp2",
+         lambda: layout_pins.test_oracle_matches_restatement("tiny-moe-tp2")),
+        ("restatement tiny-fsdp2", lambda: layout_pins.test_oracle_matches_restatement("tiny-fsdp2")),
+        ("restatement bf16 specials",
+         lambda: layout_pins.test_oracle_matches_restatement("tiny-moe-bf16-specials")),
+        ("shard size edge", layout_pins.test_shard_size_rule_edge),
+        ("round trip", lambda: layout_pins.test_unpack_of_pack_is_reshard("tiny-tp4")),
+        ("shard invariance", lambda: layout_pins.test_shard_count_invariance(7, "flat")),
+    ]
+    for name, fn in checks:
+        try:
+            fn()
+        except Exception:        # an assertion or an oracle error code
+            return name
+    return None
+
+
+def _with_library(path):
+    saved = oracle._lib
+    oracle._lib = oracle.load(path)
+    try:
+        return battery()
+    finally:
+        oracle._lib = saved
+
+
+def test_real_oracle_passes_the_battery():
+    assert battery() is None
+
+
+@pytest.mark.parametrize("name,old,new", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_planted_mistake_is_caught(name, old, new, tmp_path):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation site not found exactly once: {name}"
+    mutant = tmp_path / "mutant.c"
+    mutant.write_text(src.replace(old, new))
+    so = tmp_path / "libmutant.so"
+    subprocess.check_call(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-o", str(so),
+                           str(mutant)])
+    failed = _with_library(str(so))
+    assert failed is not None, f"no pin catches: {name}"
