@@ -435,7 +435,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                        "GB/s": round(verify_bytes / (verify_ms * 1e-3) / 1e9, 1),
                        "frac_of_peak": round(verify_bytes / (verify_ms * 1e-3) / 1e9 / peak, 4)},
         },
-        "roofline": {"bound": "hbm", "kernel": "rr_pack_kernel", "achieved": round(pack_gbs, 1),
+        "roofline": {"bound": "hbm", "kernel": "rr_bulk_kernel (pack)", "achieved": round(pack_gbs, 1),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
                      "frac": round(pack_gbs / peak, 4), "traffic": traffic,
                      "algorithmic_bytes": pack_bytes},
