@@ -400,6 +400,8 @@ def _ptr(x) -> int:
 
 def _ptr_array(xs) -> ctypes.Array:
     """Host array of device pointers from tensors / ints, or the rows of a 2-D tensor."""
+    if isinstance(xs, Pointers):
+        return xs.array
     if hasattr(xs, "dim") and xs.dim() == 2:
         base = xs.data_ptr()
         step = xs.stride(0) * xs.element_size()
@@ -429,9 +431,21 @@ def _nbytes(x):
     return int(x.numel()) * int(x.element_size())
 
 
-def _check_list(xs, n: int, min_bytes, what: str) -> None:
+def _check_list(xs, n: int, min_bytes, what: str, plan: Optional[Plan] = None) -> None:
     """Host arrays handed to the ABI hold exactly n pointers; tensor arguments
     must be large enough for what the plan will write or read."""
+    if isinstance(xs, Pointers):
+        if xs.role != what:
+            raise ValueError(f"{what}: pointer table was built for {xs.role}")
+        if xs.n != n:
+            raise ValueError(f"{what}: {xs.n} entries, plan expects {n}")
+        if plan is not None and xs.plan is plan:
+            return                      # validated against this plan when it was built
+        for i, nb in enumerate(xs.sizes):
+            need = min_bytes(i) if callable(min_bytes) else min_bytes
+            if nb is not None and need is not None and nb < need:
+                raise ValueError(f"{what}[{i}]: {nb} bytes, plan needs {need}")
+        return
     if hasattr(xs, "dim") and xs.dim() == 2:
         if xs.shape[0] != n:
             raise ValueError(f"{what}: {xs.shape[0]} rows, plan expects {n}")
@@ -449,6 +463,46 @@ def _check_list(xs, n: int, min_bytes, what: str) -> None:
             raise ValueError(f"{what}[{i}]: {nb} bytes, plan needs {need}")
 
 
+_ROLES = ("src_shards", "buckets", "dst")
+
+
+def _role_need(plan: Plan, role: str):
+    if role == "src_shards":
+        return plan.n_shards, _shard_need(plan)
+    if role == "buckets":
+        return plan.n_buckets, plan.bucket_bytes
+    return plan.n_tensors, lambda i: 2 * plan.tensor_numel[i]
+
+
+class Pointers:
+    """A pointer table checked against a plan and marshalled once.
+
+    Pass it wherever a call takes `src_shards`, `buckets` or `dst` (the role it
+    was built for).  A list of tensors is otherwise walked on every call --
+    sizes checked, pointers gathered into a host array -- which for a rollout
+    layout of a few thousand destination tensors costs about a millisecond of
+    host time per call.  The table holds references to the tensors it was
+    built from; they must not be resized or freed while it is in use."""
+
+    def __init__(self, plan: Plan, role: str, xs):
+        if role not in _ROLES:
+            raise ValueError(f"role must be one of {_ROLES}, not {role!r}")
+        n, need = _role_need(plan, role)
+        _check_list(xs, n, need, role, plan=plan)
+        self.plan = plan
+        self.role = role
+        self.n = n
+        self.array = _ptr_array(xs)
+        if hasattr(xs, "dim") and xs.dim() == 2:
+            self.sizes = [int(xs.shape[1]) * int(xs.element_size())] * n
+        else:
+            self.sizes = [_nbytes(x) for x in xs]
+        self._keep = xs
+
+    def __len__(self) -> int:
+        return self.n
+
+
 def _check_checksums(plan: Plan, checksums) -> None:
     nb = _nbytes(checksums)
     if nb is not None and nb < 8 * plan.n_buckets:
@@ -463,8 +517,8 @@ def _shard_need(plan: Plan):
 
 def rr_pack(plan: Plan, src_shards, buckets, checksums, stream=None) -> None:
     """Reshard + cast + pack + checksum (asynchronous on `stream`)."""
-    _check_list(src_shards, plan.n_shards, _shard_need(plan), "src_shards")
-    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_list(src_shards, plan.n_shards, _shard_need(plan), "src_shards", plan=plan)
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
     _check_checksums(plan, checksums)
     _check(_lib.rr_pack(plan.handle, _ptr_array(src_shards), _ptr_array(buckets),
                         _ptr(checksums), _stream(stream)), "rr_pack")
@@ -472,15 +526,15 @@ def rr_pack(plan: Plan, src_shards, buckets, checksums, stream=None) -> None:
 
 def rr_unpack(plan: Plan, buckets, dst, stream=None) -> None:
     """Buckets -> destination tensors (asynchronous on `stream`)."""
-    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
-    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst")
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
+    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst", plan=plan)
     _check(_lib.rr_unpack(plan.handle, _ptr_array(buckets), _ptr_array(dst), _stream(stream)),
            "rr_unpack")
 
 
 def rr_verify(plan: Plan, buckets, checksums, stream=None):
     """Recompute and compare checksums; returns (n_bad, first_bad).  Synchronous."""
-    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
     _check_checksums(plan, checksums)
     n_bad = ctypes.c_int64()
     first = ctypes.c_int64()
@@ -494,8 +548,8 @@ def rr_verify(plan: Plan, buckets, checksums, stream=None):
 def rr_pack_range(plan: Plan, first_bucket: int, n_buckets: int, src_shards, buckets, checksums,
                   stream=None) -> None:
     """Pack only buckets [first_bucket, first_bucket + n_buckets) (asynchronous)."""
-    _check_list(src_shards, plan.n_shards, _shard_need(plan), "src_shards")
-    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_list(src_shards, plan.n_shards, _shard_need(plan), "src_shards", plan=plan)
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
     _check_checksums(plan, checksums)
     _check(_lib.rr_pack_range(plan.handle, first_bucket, n_buckets, _ptr_array(src_shards),
                               _ptr_array(buckets), _ptr(checksums), _stream(stream)),
@@ -505,8 +559,8 @@ def rr_pack_range(plan: Plan, first_bucket: int, n_buckets: int, src_shards, buc
 def rr_unpack_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, dst,
                     stream=None) -> None:
     """Unpack only the destination bytes held by those buckets (asynchronous)."""
-    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
-    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst")
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
+    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst", plan=plan)
     _check(_lib.rr_unpack_range(plan.handle, first_bucket, n_buckets, _ptr_array(buckets),
                                 _ptr_array(dst), _stream(stream)), "rr_unpack_range")
 
@@ -515,7 +569,7 @@ def rr_verify_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, chec
                     stream=None):
     """Verify those buckets; optional device byte array `bad` gets one flag per
     bucket of the range.  Returns (n_bad, first_bad).  Synchronous."""
-    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
     _check_checksums(plan, checksums)
     if bad is not None and _nbytes(bad) is not None and _nbytes(bad) < n_buckets:
         raise ValueError(f"bad: {_nbytes(bad)} bytes, need {n_buckets}")
@@ -533,8 +587,8 @@ def rr_unpack_verify(plan: Plan, buckets, checksums, dst, bad=None, stream=None,
                      first_bucket: int = 0, n_buckets: Optional[int] = None):
     """Unpack and verify in one pass over the buckets (optionally a bucket range).
     Returns (n_bad, first_bad).  Synchronous."""
-    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
-    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst")
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
+    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst", plan=plan)
     _check_checksums(plan, checksums)
     n = plan.n_buckets - first_bucket if n_buckets is None else n_buckets
     if bad is not None and _nbytes(bad) is not None and _nbytes(bad) < n:
@@ -557,7 +611,7 @@ def rr_unpack_verify(plan: Plan, buckets, checksums, dst, bad=None, stream=None,
 
 def rr_clear_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, stream=None) -> None:
     """Zero-fill buckets [first_bucket, first_bucket + n_buckets) (asynchronous)."""
-    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets")
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
     _check(_lib.rr_clear_range(plan.handle, first_bucket, n_buckets, _ptr_array(buckets),
                                _stream(stream)), "rr_clear_range")
 
