@@ -275,7 +275,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
 
     torch.cuda.set_device(local)
     stream = torch.cuda.current_stream()
-    m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding)
+    m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
     opts = None
     if args.chunk_kib or args.grid:
         opts = rr.PlanOptions(chunk_bytes=args.chunk_kib * 1024, grid_blocks=args.grid)
@@ -426,7 +426,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u16",
         "data": "synthetic",
         "config": {"workload": w.name, "src_dtype": w.src_dtype, "n_shards": w.n_shards,
-                   "sharding": w.sharding,
+                   "sharding": w.sharding, "expert_parallel": w.ep,
                    "tp": w.tp, "bucket_bytes": bucket_bytes, "n_buckets": plan.n_buckets,
                    "step": "rr_pack + rr_unpack_verify (unpack and checksum check fused)",
                    "step_bytes": step_bytes, "l2": "inputs > L2 (no flush needed)",

@@ -101,8 +101,23 @@ typedef struct {
  *  RR_SHARD_TENSORS: every parameter is its own buffer: "shard" p is
  *                 parameter p, row-major from byte 0 (n_shards must equal the
  *                 number of parameters).  This is how a relay re-packs from
- *                 the rollout tensors it has loaded. */
-typedef enum { RR_SHARD_FLAT = 0, RR_SHARD_ROWS = 1, RR_SHARD_TENSORS = 2 } rr_sharding;
+ *                 the rollout tensors it has loaded.
+ *  RR_SHARD_UNITS: FSDP1 with one FlatParameter per wrapped module (a
+ *                 "unit": typically one per decoder layer, plus the root
+ *                 holding what no layer wraps).  param_unit[p] names the unit
+ *                 of parameter p.  Each unit is laid out exactly like the
+ *                 RR_SHARD_FLAT buffer above, on its own: its parameters in
+ *                 manifest order from offset 0, padded to a multiple of
+ *                 16 * n_shards, cut into n_shards shards of S_u bytes.  The
+ *                 calls then take n_units * n_shards source buffers,
+ *                 unit-major: buffer u * n_shards + s is shard s of unit u.
+ *                 No explicit offsets or shard size. */
+typedef enum {
+    RR_SHARD_FLAT = 0,
+    RR_SHARD_ROWS = 1,
+    RR_SHARD_TENSORS = 2,
+    RR_SHARD_UNITS = 3
+} rr_sharding;
 
 /* Trainer side. */
 typedef struct {
@@ -115,6 +130,11 @@ typedef struct {
     int64_t shard_bytes;              /* FLAT only, optional: shard size S, a multiple
                                          of 16 with n_shards * S covering every
                                          parameter; 0 = computed                      */
+    int32_t n_units;                  /* UNITS only: number of FSDP units, >= 1;
+                                         0 for the other shardings                    */
+    const int32_t* param_unit;        /* UNITS only: [n_params] unit of each parameter,
+                                         in [0, n_units), every unit used; NULL
+                                         otherwise                                    */
 } rr_src_layout;
 
 /* A 2-D block of a parameter's matrix view. */
@@ -177,9 +197,18 @@ rr_status rr_plan_query(const rr_plan* plan, int32_t* n_buckets, int64_t* stream
 /* Source geometry: shard size S, end of the last parameter, and per-parameter
  * byte offsets ([n_params]): flat offsets for RR_SHARD_FLAT, offsets within
  * each shard for RR_SHARD_ROWS, 0 for RR_SHARD_TENSORS (whose S is the size of
- * the largest parameter).  Any output pointer may be NULL. */
+ * the largest parameter), offsets within the parameter's unit for
+ * RR_SHARD_UNITS (whose S is the largest S_u; flat_bytes is then the end of
+ * the largest unit).  Any output pointer may be NULL. */
 rr_status rr_plan_source(const rr_plan* plan, int64_t* shard_bytes, int64_t* flat_bytes,
                          int64_t* param_flat_offset);
+
+/* The source buffers the calls take: their number (the length of every
+ * src_shards array) and the bytes each must hold ([*n_buffers]).  FLAT and
+ * ROWS: n_shards buffers of S bytes; TENSORS: one per parameter, of its size;
+ * UNITS: n_units * n_shards, unit-major, each of its unit's S_u.  Pass
+ * buffer_bytes = NULL to learn the count first.  Any output pointer may be NULL. */
+rr_status rr_plan_source_buffers(const rr_plan* plan, int32_t* n_buffers, int64_t* buffer_bytes);
 
 /* Destination geometry: per tensor numel and byte offset within its rank's
  * stream ([n_tensors] each).  Any output pointer may be NULL. */

@@ -65,7 +65,9 @@ class _Layout(ctypes.Structure):
                 ("flat_bytes", ctypes.c_int64), ("shard_bytes", ctypes.c_int64),
                 ("sharding", ctypes.c_int32), ("pad_", ctypes.c_int32),
                 ("shard_bytes_in", ctypes.c_int64), ("explicit_offset", _P64),
-                ("chunk_rows", _P64), ("param_gen_base", _P64)]
+                ("chunk_rows", _P64), ("param_gen_base", _P64),
+                ("n_units", ctypes.c_int32), ("pad2_", ctypes.c_int32),
+                ("param_unit", ctypes.POINTER(ctypes.c_int32)), ("unit_shard_bytes", _P64)]
 
 
 _VALUE_FN = ctypes.CFUNCTYPE(ctypes.c_uint32, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32)
@@ -180,7 +182,8 @@ class Layout:
 
     def __init__(self, params, tensors, n_shards: int, tp: int, bucket_bytes: int,
                  align_bytes: int = 16, tensor_align: int = 256, sharding: str = "flat",
-                 explicit_offsets=None, shard_bytes: int = 0):
+                 explicit_offsets=None, shard_bytes: int = 0, units=None):
+        """units: with sharding="units", the unit of each parameter."""
         self.sharding = sharding
         self.params = list(params)
         self.tensors = list(tensors)
@@ -219,8 +222,17 @@ class Layout:
         for name in ("param_offset", "tensor_numel", "tensor_offset", "rank_stream_bytes",
                      "rank_first_bucket", "chunk_rows", "param_gen_base"):
             setattr(L, name, getattr(self, name).ctypes.data_as(_P64))
-        L.sharding = {"flat": 0, "rows": 1, "tensors": 2}[sharding]
+        L.sharding = {"flat": 0, "rows": 1, "tensors": 2, "units": 3}[sharding]
         L.shard_bytes_in = shard_bytes
+        self.units = None
+        self.unit_shard_bytes = np.zeros(0, np.int64)
+        if units is not None:
+            self.units = np.ascontiguousarray(units, dtype=np.int32)
+            n_units = int(self.units.max()) + 1 if self.units.size else 0
+            self.unit_shard_bytes = np.zeros(max(1, n_units), np.int64)
+            L.n_units = n_units
+            L.param_unit = self.units.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+            L.unit_shard_bytes = self.unit_shard_bytes.ctypes.data_as(_P64)
         self._explicit = None
         if explicit_offsets is not None:
             self._explicit = np.ascontiguousarray(explicit_offsets, dtype=np.int64)
@@ -235,6 +247,8 @@ class Layout:
         self.flat_bytes = int(L.flat_bytes)
         self.shard_bytes = int(L.shard_bytes)
         self.n_buckets = int(self.rank_first_bucket[tp])
+        if units is not None:
+            self.unit_shard_bytes = self.unit_shard_bytes[:L.n_units]
 
     # -- source ---------------------------------------------------------------
     def param_numel(self, p: int) -> int:
@@ -251,6 +265,22 @@ class Layout:
                 vals = synth.values_host(n, es, seed, first_idx=int(self.param_gen_base[p]),
                                          specials=specials)
                 out.append(vals.view(np.uint8).copy())
+            return out
+        if self.sharding == "units":
+            # Each unit: its own flat buffer, cut into n_shards shards.
+            out = []
+            for u, Su in enumerate(self.unit_shard_bytes):
+                Su = int(Su)
+                flat = np.zeros(Su * self.n_shards, np.uint8)
+                for p, (_, _, es) in enumerate(self.params):
+                    if int(self.units[p]) != u:
+                        continue
+                    n = self.param_numel(p)
+                    vals = synth.values_host(n, es, seed, first_idx=int(self.param_gen_base[p]),
+                                             specials=specials)
+                    off = int(self.param_offset[p])
+                    flat[off:off + n * es] = vals.view(np.uint8)
+                out += [flat[s * Su:(s + 1) * Su] for s in range(self.n_shards)]
             return out
         flat = np.zeros(self.shard_bytes * self.n_shards, np.uint8)
         S = self.shard_bytes
@@ -391,6 +421,7 @@ class Layout:
 def workload_layout(w, bucket_bytes: Optional[int] = None) -> Layout:
     """Oracle layout for a ``synth.Workload``."""
     params = qwen3.manifest(w.shape, w.src_elem_bytes)
-    tensors = qwen3.rollout_tensors(w.shape, params, w.tp)
+    tensors = qwen3.rollout_tensors(w.shape, params, w.tp, ep=getattr(w, "ep", False))
+    units = qwen3.layer_units(params) if w.sharding == "units" else None
     return Layout(params, tensors, n_shards=w.n_shards, tp=w.tp,
-                  bucket_bytes=bucket_bytes or w.bucket_bytes, sharding=w.sharding)
+                  bucket_bytes=bucket_bytes or w.bucket_bytes, sharding=w.sharding, units=units)

@@ -21,7 +21,13 @@ expert's gate/up) and the r-th of t equal column ranges of the row-parallel
 weights (o_proj, down_proj, each expert's down_proj); norms and the router
 are replicated on every rank.  When TP exceeds the number of KV heads, each
 KV head is replicated instead: rank r takes the rows of head r * n_kv // t of
-k and of v (t / n_kv ranks per head).
+k and of v (t / n_kv ranks per head).  Expert-parallel rollout (ep): the
+experts are not cut; rank r takes experts r*E/t .. (r+1)*E/t - 1 whole, in
+order, into its w13 and w2 (attention as above, router replicated).
+
+Per-layer FSDP1 units: each decoder layer's parameters form one unit (layer
+i is unit i + 1); the parameters outside the layers (embedding, final norm,
+lm_head) form the root unit 0.
 
 A block is (param index, row0, nrows, col0, ncols) on the parameter's
 [rows = d0, cols = d1 * d2 * ...] view.
@@ -84,7 +90,18 @@ def _view(dims) -> Tuple[int, int]:
     return rows, cols
 
 
-def rollout_tensors(shape, params: List[Param], tp: int) -> List[Tensor]:
+def layer_units(params: List[Param]) -> List[int]:
+    out = []
+    for name, _, _ in params:
+        if name.startswith("model.layers."):
+            layer = int(name[len("model.layers."):].split(".", 1)[0])
+            out.append(layer + 1)
+        else:
+            out.append(0)
+    return out
+
+
+def rollout_tensors(shape, params: List[Param], tp: int, ep: bool = False) -> List[Tensor]:
     index = {name: i for i, (name, _, _) in enumerate(params)}
     view = {name: _view(dims) for name, dims, _ in params}
 
@@ -135,10 +152,18 @@ def rollout_tensors(shape, params: List[Param], tp: int) -> List[Tensor]:
                 ex = pre + "mlp.experts."
                 w13: List[Block] = []
                 w2: List[Block] = []
-                for e in range(E):
-                    w13 += [row_slice(f"{ex}{e}.gate_proj.weight", r),
-                            row_slice(f"{ex}{e}.up_proj.weight", r)]
-                    w2.append(col_slice(f"{ex}{e}.down_proj.weight", r))
+                if ep:
+                    assert E % tp == 0, f"{E} experts do not split over {tp} ranks"
+                    per = E // tp
+                    for e in range(r * per, (r + 1) * per):
+                        w13 += [whole(f"{ex}{e}.gate_proj.weight"),
+                                whole(f"{ex}{e}.up_proj.weight")]
+                        w2.append(whole(f"{ex}{e}.down_proj.weight"))
+                else:
+                    for e in range(E):
+                        w13 += [row_slice(f"{ex}{e}.gate_proj.weight", r),
+                                row_slice(f"{ex}{e}.up_proj.weight", r)]
+                        w2.append(col_slice(f"{ex}{e}.down_proj.weight", r))
                 tensors += [
                     (f"layers.{i}.router", r, [whole(pre + "mlp.gate.weight")]),
                     (f"layers.{i}.experts.w13", r, w13),

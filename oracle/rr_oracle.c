@@ -42,6 +42,14 @@
  *  Source, one buffer per parameter.  Parameter p is "shard" p, row-major
  *  from byte 0.
  *
+ *  Source, unit sharding (FSDP1 wrapping modules separately, each with its
+ *  own FlatParameter).  Every parameter belongs to one unit; a unit is laid
+ *  out exactly like the flat source above but on its own: its parameters in
+ *  manifest order from offset 0, each aligned, the total padded to a multiple
+ *  of 16 * n_shards and cut into n_shards shards of S_u bytes.  The shard
+ *  buffers are numbered unit by unit: shard s of unit u is buffer
+ *  u * n_shards + s.
+ *
  *  A parameter of shape [d0, d1, ...] is viewed as a matrix [rows = d0,
  *  cols = d1 * d2 * ...] (cols = 1 for a vector).  Generated values are
  *  indexed by the element's position in the flat layout whatever the
@@ -118,6 +126,12 @@ typedef struct {
     /* derived, continued */
     int64_t* chunk_rows;        /* [n_params] rows: c per parameter                 */
     int64_t* param_gen_base;    /* [n_params] flat element index of element 0       */
+    /* description, continued: unit sharding (3) */
+    int32_t n_units;
+    int32_t pad2_;
+    const int32_t* param_unit;  /* [n_params] unit of each parameter                */
+    /* derived, continued */
+    int64_t* unit_shard_bytes;  /* [n_units] S_u                                    */
 } orc_layout;
 
 /* Where source values come from: real shard buffers, or a generator that maps
@@ -172,6 +186,31 @@ int orc_layout_compute(orc_layout* L) {
                 return ORC_EINVAL;
             L->shard_bytes = L->shard_bytes_in;
         }
+    } else if (L->sharding == 3) {
+        /* Units: every unit is a flat layout of its own parameters. */
+        if (L->explicit_offset || L->shard_bytes_in || L->n_units < 1 || !L->param_unit)
+            return ORC_EINVAL;
+        int64_t biggest = 0, longest = 0;
+        for (int32_t u = 0; u < L->n_units; ++u) {
+            int64_t local = 0, members = 0;
+            for (int32_t p = 0; p < L->n_params; ++p) {
+                if (L->param_unit[p] != u) continue;
+                const orc_param* P = &L->params[p];
+                int64_t a = L->align_bytes > P->elem_bytes ? L->align_bytes : P->elem_bytes;
+                local = align_up(local, a);
+                L->param_offset[p] = local;
+                local += P->rows * P->cols * P->elem_bytes;
+                ++members;
+            }
+            if (members == 0) return ORC_EINVAL;
+            L->unit_shard_bytes[u] = align_up(local, 16 * (int64_t)L->n_shards) / L->n_shards;
+            if (L->unit_shard_bytes[u] > biggest) biggest = L->unit_shard_bytes[u];
+            if (local > longest) longest = local;
+        }
+        for (int32_t p = 0; p < L->n_params; ++p)
+            if (L->param_unit[p] < 0 || L->param_unit[p] >= L->n_units) return ORC_EINVAL;
+        L->flat_bytes = longest;
+        L->shard_bytes = biggest;
     } else if (L->sharding == 2) {
         /* One buffer per parameter. */
         if (L->explicit_offset || L->shard_bytes_in || L->n_shards != L->n_params)
@@ -273,6 +312,15 @@ static int source_bits(const orc_layout* L, const orc_source* S, int32_t p, int6
     } else if (L->sharding == 2) {
         if (p >= L->n_shards || S->shards[p] == NULL) return ORC_ESOURCE;
         for (int32_t i = 0; i < es; ++i) v |= (uint32_t)S->shards[p][e * es + i] << (8 * i);
+    } else if (L->sharding == 3) {
+        const int32_t u = L->param_unit[p];
+        const int64_t Su = L->unit_shard_bytes[u];
+        for (int32_t i = 0; i < es; ++i) {
+            int64_t f = L->param_offset[p] + e * es + i;   /* byte within the unit */
+            int64_t buf = (int64_t)u * L->n_shards + f / Su;
+            if (S->shards[buf] == NULL) return ORC_ESOURCE;
+            v |= (uint32_t)S->shards[buf][f % Su] << (8 * i);
+        }
     } else {
         int64_t row = e / P->cols;
         int64_t s = row / L->chunk_rows[p];

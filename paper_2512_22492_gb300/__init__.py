@@ -12,11 +12,11 @@ from .rr import (Block, DstLayout, DstTensor, Param, Plan, PlanOptions, Pointers
                  rr_plan_selftest_wait, rr_status_str, rr_unpack,
                  rr_unpack_range, rr_unpack_verify, rr_verify, rr_verify_noalloc,
                  rr_verify_range)
-from .layouts import qwen3_manifest, qwen3_rollout, qwen3_sync
+from .layouts import qwen3_layer_units, qwen3_manifest, qwen3_rollout, qwen3_sync
 
 __all__ = ["Block", "DstLayout", "DstTensor", "Param", "Plan", "PlanOptions", "Pointers",
            "RRError",
            "SrcLayout", "rr_pack", "rr_plan_create", "rr_status_str", "rr_unpack", "rr_verify",
            "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
            "rr_unpack_verify", "rr_plan_check", "rr_plan_selftest_wait", "rr_verify_noalloc",
-           "qwen3_manifest", "qwen3_rollout", "qwen3_sync"]
+           "qwen3_layer_units", "qwen3_manifest", "qwen3_rollout", "qwen3_sync"]

@@ -13,12 +13,16 @@ struct rr_plan {
     int32_t n_params = 0;
     std::vector<int64_t> rows, cols;   // matrix view of each parameter
     std::vector<int32_t> es;           // element bytes (4 or 2)
-    std::vector<int64_t> param_off;    // flat byte offsets (FLAT) or in-shard offsets (ROWS)
+    std::vector<int64_t> param_off;    // flat byte offsets (FLAT), in-shard offsets (ROWS),
+                                       // offsets within the unit (UNITS)
     std::vector<int64_t> chunk_rows;   // ROWS: rows per shard, ceil(rows / n_shards)
     int32_t sharding = RR_SHARD_FLAT;
-    int32_t n_shards = 0;
-    int64_t shard_bytes = 0;           // S
+    int32_t n_shards = 0;              // source buffers the calls take
+    int64_t shard_bytes = 0;           // S (UNITS: the largest S_u)
     int64_t flat_bytes = 0;
+    int32_t unit_shards = 0;           // UNITS: shards per unit
+    std::vector<int32_t> unit_of;      // UNITS: unit of each parameter
+    std::vector<int64_t> unit_shard_bytes;  // UNITS: S_u
 
     // ---- destination ----------------------------------------------------
     int32_t tp = 0;

@@ -51,6 +51,12 @@ public:
         }
         if (P->sharding == RR_SHARD_TENSORS)
             return {p, e * es, (P->rows[p] * P->cols[p] - e) * es};
+        if (P->sharding == RR_SHARD_UNITS) {
+            const int32_t u = P->unit_of[p];
+            const int64_t S = P->unit_shard_bytes[u];
+            const int64_t f = P->param_off[p] + e * es;
+            return {int64_t(u) * P->unit_shards + f / S, f % S, S - f % S};
+        }
         const int64_t cols = P->cols[p], c = P->chunk_rows[p];
         const int64_t sh = e / cols / c;
         const int64_t end = std::min((sh + 1) * c, P->rows[p]) * cols;   // p's last element in sh
@@ -322,10 +328,41 @@ rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_
     // Source offsets.
     int64_t end = 0;
     if (src->sharding != RR_SHARD_FLAT && src->sharding != RR_SHARD_ROWS &&
-        src->sharding != RR_SHARD_TENSORS)
+        src->sharding != RR_SHARD_TENSORS && src->sharding != RR_SHARD_UNITS)
         return rr_fail(RR_EINVAL, "unknown sharding %d", src->sharding);
+    if (src->sharding != RR_SHARD_UNITS && (src->n_units || src->param_unit))
+        return rr_fail(RR_EINVAL, "units are given only with RR_SHARD_UNITS");
     P->sharding = src->sharding;
-    if (src->sharding == RR_SHARD_TENSORS) {
+    if (src->sharding == RR_SHARD_UNITS) {
+        if (src->param_flat_offset || src->shard_bytes)
+            return rr_fail(RR_EINVAL, "unit sharding takes no explicit offsets or shard size");
+        const int32_t U = src->n_units;
+        if (U < 1 || !src->param_unit)
+            return rr_fail(RR_EINVAL, "unit sharding needs n_units >= 1 and param_unit");
+        if (int64_t(U) * src->n_shards > 65535)
+            return rr_fail(RR_EINVAL, "n_units * n_shards must be at most 65535");
+        P->unit_shards = src->n_shards;
+        P->unit_of.assign(src->param_unit, src->param_unit + n_params);
+        std::vector<int64_t> uend(U, 0);
+        std::vector<char> used(U, 0);
+        for (int32_t p = 0; p < n_params; ++p) {   // manifest order within each unit
+            const int32_t u = P->unit_of[p];
+            if (u < 0 || u >= U) return rr_fail(RR_EINVAL, "param %d: unit %d out of range", p, u);
+            used[u] = 1;
+            uend[u] = align_up(uend[u], std::max<int64_t>(src->align_bytes, P->es[p]));
+            P->param_off[p] = uend[u];
+            uend[u] += P->rows[p] * P->cols[p] * P->es[p];
+        }
+        P->unit_shard_bytes.resize(U);
+        for (int32_t u = 0; u < U; ++u) {
+            if (!used[u]) return rr_fail(RR_EINVAL, "unit %d holds no parameter", u);
+            P->unit_shard_bytes[u] = align_up(uend[u], 16 * int64_t(src->n_shards)) / src->n_shards;
+            end = std::max(end, uend[u]);
+            P->shard_bytes = std::max(P->shard_bytes, P->unit_shard_bytes[u]);
+        }
+        P->flat_bytes = end;
+        P->n_shards = U * src->n_shards;
+    } else if (src->sharding == RR_SHARD_TENSORS) {
         if (src->param_flat_offset || src->shard_bytes)
             return rr_fail(RR_EINVAL, "per-tensor sources take no explicit offsets or shard size");
         if (src->n_shards != n_params)
@@ -601,6 +638,21 @@ rr_status rr_plan_source(const rr_plan* P, int64_t* shard_bytes, int64_t* flat_b
     if (shard_bytes) *shard_bytes = P->shard_bytes;
     if (flat_bytes) *flat_bytes = P->flat_bytes;
     if (param_flat_offset) std::copy(P->param_off.begin(), P->param_off.end(), param_flat_offset);
+    return RR_OK;
+}
+
+rr_status rr_plan_source_buffers(const rr_plan* P, int32_t* n_buffers, int64_t* buffer_bytes) {
+    if (!P) return rr_fail(RR_EINVAL, "plan is NULL");
+    if (n_buffers) *n_buffers = P->n_shards;
+    if (!buffer_bytes) return RR_OK;
+    for (int32_t i = 0; i < P->n_shards; ++i) {
+        if (P->sharding == RR_SHARD_TENSORS)
+            buffer_bytes[i] = P->rows[i] * P->cols[i] * P->es[i];
+        else if (P->sharding == RR_SHARD_UNITS)
+            buffer_bytes[i] = P->unit_shard_bytes[i / P->unit_shards];
+        else
+            buffer_bytes[i] = P->shard_bytes;
+    }
     return RR_OK;
 }
 

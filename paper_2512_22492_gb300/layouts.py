@@ -21,7 +21,14 @@ Rollout tensors, per rank r of TP = t, in this order:
   norm                replicated
   lm_head             rows r of t, unless tied to the embedding
 When t exceeds the number of KV heads, k and v are not split but replicated
-by head: rank r holds KV head r * n_kv // t.
+by head: rank r holds KV head r * n_kv // t.  With expert parallelism
+(ep=True) the experts are not sliced but dealt out whole: rank r holds
+experts [r * E / t, (r + 1) * E / t), so its w13 and w2 stack E / t full
+experts; attention stays tensor-parallel and the router replicated.
+
+Trainer sources: one flat FSDP1 FlatParameter ("flat"), FSDP2 per-parameter
+dim-0 shards ("rows"), or FSDP1 wrapping every decoder layer ("units"): unit
+0 is the root (embedding, final norm, lm_head), unit 1 + i is layer i.
 """
 from __future__ import annotations
 
@@ -107,10 +114,23 @@ class _Slicer:
         return Block(self.idx[name], 0, rows, r * n, n)
 
 
+def qwen3_layer_units(manifest: List[Param]) -> List[int]:
+    """FSDP1 units when every decoder layer is wrapped: the unit of each
+    parameter, 1 + i for layer i and 0 for the root's own parameters."""
+    units = []
+    for p in manifest:
+        parts = p.name.split(".")
+        units.append(1 + int(parts[2]) if parts[:2] == ["model", "layers"] else 0)
+    return units
+
+
 def qwen3_rollout(shape, manifest: List[Param], tp: int = 1,
-                  tensor_align_bytes: int = 256) -> DstLayout:
-    """Rollout (inference-engine) tensors for TP = tp, rank-major."""
+                  tensor_align_bytes: int = 256, ep: bool = False) -> DstLayout:
+    """Rollout (inference-engine) tensors for TP = tp, rank-major; ep=True
+    deals the experts out whole instead of slicing each one."""
     s = _Slicer(manifest, tp)
+    if ep and getattr(shape, "n_experts", 0) % tp:
+        raise ValueError(f"{shape.n_experts} experts do not divide over {tp} ranks")
     tensors: List[DstTensor] = []
     for r in range(tp):
         def add(name, blocks):
@@ -134,11 +154,19 @@ def qwen3_rollout(shape, manifest: List[Param], tp: int = 1,
                 E = shape.n_experts
                 x = f"{L}.mlp.experts"
                 add(f"layers.{i}.router", [s.whole(f"{L}.mlp.gate.weight")])
-                add(f"layers.{i}.experts.w13",
-                    [b for e in range(E) for b in (s.rows(f"{x}.{e}.gate_proj.weight", r),
-                                                   s.rows(f"{x}.{e}.up_proj.weight", r))])
-                add(f"layers.{i}.experts.w2",
-                    [s.cols(f"{x}.{e}.down_proj.weight", r) for e in range(E)])
+                if ep:
+                    mine = range(r * E // tp, (r + 1) * E // tp)
+                    add(f"layers.{i}.experts.w13",
+                        [b for e in mine for b in (s.whole(f"{x}.{e}.gate_proj.weight"),
+                                                   s.whole(f"{x}.{e}.up_proj.weight"))])
+                    add(f"layers.{i}.experts.w2",
+                        [s.whole(f"{x}.{e}.down_proj.weight") for e in mine])
+                else:
+                    add(f"layers.{i}.experts.w13",
+                        [b for e in range(E) for b in (s.rows(f"{x}.{e}.gate_proj.weight", r),
+                                                       s.rows(f"{x}.{e}.up_proj.weight", r))])
+                    add(f"layers.{i}.experts.w2",
+                        [s.cols(f"{x}.{e}.down_proj.weight", r) for e in range(E)])
             else:
                 add(f"layers.{i}.gate_up_proj", [s.rows(f"{L}.mlp.gate_proj.weight", r),
                                                  s.rows(f"{L}.mlp.up_proj.weight", r)])
@@ -149,13 +177,16 @@ def qwen3_rollout(shape, manifest: List[Param], tp: int = 1,
     return DstLayout(tp=tp, tensors=tensors, tensor_align_bytes=tensor_align_bytes)
 
 
-def qwen3_sync(shape, dtype: str, n_shards: int, tp: int, sharding: str = "flat"):
+def qwen3_sync(shape, dtype: str, n_shards: int, tp: int, sharding: str = "flat",
+               ep: bool = False):
     """(manifest, source layout, destination layout) for one Qwen3 weight sync.
-    sharding: "flat" (one FSDP1 FlatParameter cut evenly) or "rows" (FSDP2:
-    every parameter cut on dim 0)."""
+    sharding: "flat" (one FSDP1 FlatParameter cut evenly), "rows" (FSDP2:
+    every parameter cut on dim 0) or "units" (FSDP1 wrapping every decoder
+    layer); ep: expert-parallel rollout."""
     manifest = qwen3_manifest(shape, dtype)
-    src = SrcLayout(n_shards=n_shards, align_bytes=16, sharding=sharding)
-    return manifest, src, qwen3_rollout(shape, manifest, tp)
+    units = qwen3_layer_units(manifest) if sharding == "units" else None
+    src = SrcLayout(n_shards=n_shards, align_bytes=16, sharding=sharding, units=units)
+    return manifest, src, qwen3_rollout(shape, manifest, tp, ep=ep)
 
 
 # ---------------------------------------------------------------------------
@@ -241,9 +272,11 @@ def relayout(source: DstLayout, target: DstLayout) -> DstLayout:
     return DstLayout(tp=target.tp, tensors=tensors, tensor_align_bytes=target.tensor_align_bytes)
 
 
-def qwen3_relay(shape, src_tp: int, dst_tp: int, from_plan=None):
+def qwen3_relay(shape, src_tp: int, dst_tp: int, from_plan=None, src_ep: bool = False,
+                dst_ep: bool = False):
     """(manifest, source layout, destination layout) for a relay that holds the
-    TP=src_tp rollout image and serves a TP=dst_tp rollout.
+    TP=src_tp rollout image and serves a TP=dst_tp rollout (either side may
+    deal its experts out whole: src_ep / dst_ep).
 
     from_plan=None: the relay re-packs from its loaded tensors (one buffer per
     tensor, in the order of the TP=src_tp rollout layout).  from_plan=<the
@@ -251,9 +284,9 @@ def qwen3_relay(shape, src_tp: int, dst_tp: int, from_plan=None):
     pulled (the buckets, in order, are the shards; bucket_bytes must be a
     multiple of 16)."""
     logical = qwen3_manifest(shape, "bf16")
-    src = qwen3_rollout(shape, logical, src_tp)
+    src = qwen3_rollout(shape, logical, src_tp, ep=src_ep)
     params, _ = rollout_as_source(src)
-    dst = relayout(src, qwen3_rollout(shape, logical, dst_tp))
+    dst = relayout(src, qwen3_rollout(shape, logical, dst_tp, ep=dst_ep))
     if from_plan is None:
         return params, SrcLayout(n_shards=len(params), sharding="tensors"), dst
     B = from_plan.bucket_bytes

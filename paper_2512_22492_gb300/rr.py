@@ -42,7 +42,8 @@ class _Param(ctypes.Structure):
 class _SrcLayout(ctypes.Structure):
     _fields_ = [("n_shards", ctypes.c_int32), ("align_bytes", ctypes.c_int64),
                 ("param_flat_offset", ctypes.POINTER(ctypes.c_int64)),
-                ("sharding", ctypes.c_int32), ("shard_bytes", ctypes.c_int64)]
+                ("sharding", ctypes.c_int32), ("shard_bytes", ctypes.c_int64),
+                ("n_units", ctypes.c_int32), ("param_unit", ctypes.POINTER(ctypes.c_int32))]
 
 
 class _Block(ctypes.Structure):
@@ -122,6 +123,7 @@ _sig("rr_plan_create", [ctypes.POINTER(_Param), ctypes.c_int32, ctypes.POINTER(_
 _sig("rr_plan_destroy", [_vp], None)
 _sig("rr_plan_query", [_vp, _P32, _P64, _P32])
 _sig("rr_plan_source", [_vp, _P64, _P64, _P64])
+_sig("rr_plan_source_buffers", [_vp, _P32, _P64])
 _sig("rr_plan_tensors", [_vp, _P64, _P64])
 _sig("rr_plan_get_stats", [_vp, ctypes.POINTER(_Stats)])
 _sig("rr_plan_export_pack", [_vp, ctypes.POINTER(PackItem), ctypes.c_int64,
@@ -151,7 +153,8 @@ _sig("rr_last_error", [], ctypes.c_char_p)
 
 LIBRARY_PATH = _build.LIB
 EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_query",
-            "rr_plan_source", "rr_plan_tensors", "rr_plan_get_stats", "rr_plan_export_pack",
+            "rr_plan_source", "rr_plan_source_buffers", "rr_plan_tensors", "rr_plan_get_stats",
+            "rr_plan_export_pack",
             "rr_plan_export_unpack", "rr_plan_bucket_items", "rr_pack", "rr_unpack", "rr_verify",
             "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
             "rr_unpack_verify", "rr_unpack_verify_range",
@@ -193,8 +196,10 @@ class SrcLayout:
     align_bytes: int = 16
     param_flat_offset: Optional[Sequence[int]] = None
     sharding: str = "flat"    # "flat" (FSDP1 FlatParameter), "rows" (FSDP2 dim-0 Shard),
-                              # or "tensors" (one buffer per parameter)
+                              # "tensors" (one buffer per parameter), or "units" (FSDP1,
+                              # one FlatParameter per wrapped module)
     shard_bytes: int = 0      # flat only: explicit shard size, 0 = computed
+    units: Optional[Sequence[int]] = None   # units only: the unit of each parameter
 
 
 @dataclass
@@ -268,6 +273,13 @@ class Plan:
         self.shard_bytes = shard.value
         self.flat_bytes = flat.value
         self.param_flat_offset = list(offs)[:n_params]
+        nbuf = ctypes.c_int32()
+        _check(_lib.rr_plan_source_buffers(self._h, ctypes.byref(nbuf), None),
+               "rr_plan_source_buffers")
+        sizes = (ctypes.c_int64 * max(1, nbuf.value))()
+        _check(_lib.rr_plan_source_buffers(self._h, None, sizes), "rr_plan_source_buffers")
+        self.source_buffer_bytes = list(sizes)[:nbuf.value]
+        self.units = list(src.units) if src is not None and src.units is not None else None
         numel = (ctypes.c_int64 * max(1, self.n_tensors))()
         toff = (ctypes.c_int64 * max(1, self.n_tensors))()
         _check(_lib.rr_plan_tensors(self._h, numel, toff), "rr_plan_tensors")
@@ -344,12 +356,17 @@ def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
             cp[i].shape[d] = s
         cp[i].dtype = RR_F32 if p.dtype == "f32" else RR_BF16
     cs = _SrcLayout(n_shards=src.n_shards, align_bytes=src.align_bytes,
-                    sharding={"flat": 0, "rows": 1, "tensors": 2}[src.sharding],
+                    sharding={"flat": 0, "rows": 1, "tensors": 2, "units": 3}[src.sharding],
                     shard_bytes=src.shard_bytes)
     offs = None
     if src.param_flat_offset is not None:
         offs = (ctypes.c_int64 * max(1, n))(*src.param_flat_offset)
         cs.param_flat_offset = offs
+    units = None
+    if src.units is not None:
+        units = (ctypes.c_int32 * max(1, len(src.units)))(*src.units)
+        cs.n_units = max(src.units) + 1 if len(src.units) else 0
+        cs.param_unit = units
     keep = []
     ct = (_DstTensor * max(1, len(dst.tensors)))()
     for i, t in enumerate(dst.tensors):
@@ -510,8 +527,8 @@ def _check_checksums(plan: Plan, checksums) -> None:
 
 
 def _shard_need(plan: Plan):
-    if plan.sharding == "tensors":
-        return lambda i: plan.param_bytes[i]
+    if plan.sharding in ("tensors", "units"):
+        return lambda i: plan.source_buffer_bytes[i]
     return plan.shard_bytes
 
 

@@ -67,7 +67,9 @@ class Workload:
     bucket_bytes: int
     seed: int
     specials: bool = False   # inject ~1% special bit patterns
-    sharding: str = "flat"   # "flat" (one FSDP1 FlatParameter) or "rows" (FSDP2 dim-0)
+    sharding: str = "flat"   # "flat" (one FSDP1 FlatParameter), "rows" (FSDP2 dim-0), or
+                             # "units" (FSDP1, one FlatParameter per decoder layer + root)
+    ep: bool = False         # rollout experts split whole over the ranks (expert parallel)
 
     @property
     def src_elem_bytes(self) -> int:
@@ -134,6 +136,14 @@ TEST_WORKLOADS = {
                                bucket_bytes=32 * 1024, seed=19, sharding="rows"),
     "tiny-kvrep-f32": Workload("tiny-kvrep-f32", TINY, "f32", n_shards=8, tp=8,
                                bucket_bytes=16 * 1024, seed=20, specials=True),
+    # FSDP1 wrapping every decoder layer: one FlatParameter per layer plus the root's.
+    "tiny-units": Workload("tiny-units", TINY, "f32", n_shards=3, tp=2, bucket_bytes=48 * 1024,
+                           seed=22, specials=True, sharding="units"),
+    # Expert-parallel rollouts: every rank holds whole experts.
+    "tiny-moe-ep4": Workload("tiny-moe-ep4", TINY_MOE, "f32", n_shards=8, tp=4,
+                             bucket_bytes=24 * 1024, seed=23, specials=True, ep=True),
+    "tiny-moe-units-ep2": Workload("tiny-moe-units-ep2", TINY_MOE, "bf16", n_shards=5, tp=2,
+                                   bucket_bytes=32 * 1024, seed=24, sharding="units", ep=True),
 }
 
 # Full-size variants beyond the five workloads: the paper's own trainer sharding
@@ -144,6 +154,12 @@ EXTRA_WORKLOADS = {
     "qwen3-30b-a3b-fsdp2-tp8": Workload("qwen3-30b-a3b-fsdp2-tp8", QWEN3_30B_A3B, "bf16",
                                         n_shards=8, tp=8, bucket_bytes=256 * MiB, seed=7,
                                         sharding="rows"),
+    # Per-layer FSDP1 units (the common FSDP1 wrapping) and an expert-parallel rollout.
+    "qwen3-8b-units": Workload("qwen3-8b-units", QWEN3_8B, "f32", n_shards=8, tp=1,
+                               bucket_bytes=128 * MiB, seed=8, sharding="units"),
+    "qwen3-30b-a3b-fsdp2-ep8": Workload("qwen3-30b-a3b-fsdp2-ep8", QWEN3_30B_A3B, "bf16",
+                                        n_shards=8, tp=8, bucket_bytes=256 * MiB, seed=9,
+                                        sharding="rows", ep=True),
 }
 
 

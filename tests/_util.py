@@ -53,13 +53,24 @@ def random_layout(seed: int, max_params: int = 7, bucket_choices=(8, 24, 40, 64,
                 nc = int(rng.integers(0, cols - c0 + 1))
             blocks.append((p, r0, nr, c0, nc))
         tensors.append((f"t{t}", int(rng.integers(0, tp)), blocks))
-    return dict(params=params, tensors=tensors, tp=tp,
+    desc = dict(params=params, tensors=tensors, tp=tp,
                 sharding="rows" if rng.random() < 0.35 else "flat",
                 n_shards=int(rng.integers(1, 6)),
                 bucket_bytes=int(rng.choice(bucket_choices)),
                 align_bytes=int(rng.choice([1, 2, 4, 8, 16, 32])),
                 tensor_align=int(rng.choice([2, 4, 16, 256])),
                 seed=int(rng.integers(1, 1 << 20)), specials=bool(rng.random() < 0.5))
+    # Some flat trainers become per-module FSDP1 units: parameters dealt to
+    # units in scattered order, every unit used (a second stream, so the draws
+    # above stay what they were).
+    extra = np.random.default_rng(seed + 1_000_003)
+    if desc["sharding"] == "flat" and extra.random() < 0.4:
+        n_units = int(extra.integers(1, n_params + 1))
+        units = np.concatenate([np.arange(n_units),
+                                extra.integers(0, n_units, n_params - n_units)])
+        desc["sharding"] = "units"
+        desc["units"] = [int(u) for u in extra.permutation(units)]
+    return desc
 
 
 def workload_desc(name, bucket_bytes=None):
@@ -77,17 +88,17 @@ def to_oracle(desc) -> "oracle.Layout":
     return oracle.Layout(desc["params"], desc["tensors"], n_shards=desc["n_shards"],
                          tp=desc["tp"], bucket_bytes=desc["bucket_bytes"],
                          align_bytes=desc["align_bytes"], tensor_align=desc["tensor_align"],
-                         sharding=desc.get("sharding", "flat"))
+                         sharding=desc.get("sharding", "flat"), units=desc.get("units"))
 
 
 def to_product(desc):
     import paper_2512_22492_gb300 as rr
     if desc.get("workload") is not None:
         w = desc["workload"]
-        return rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding)
+        return rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
     manifest = [rr.Param(n, d, "f32" if es == 4 else "bf16") for n, d, es in desc["params"]]
     src = rr.SrcLayout(n_shards=desc["n_shards"], align_bytes=desc["align_bytes"],
-                       sharding=desc.get("sharding", "flat"))
+                       sharding=desc.get("sharding", "flat"), units=desc.get("units"))
     dst = rr.DstLayout(tp=desc["tp"], tensor_align_bytes=desc["tensor_align"],
                        tensors=[rr.DstTensor(n, r, [rr.Block(*b) for b in blocks])
                                 for n, r, blocks in desc["tensors"]])
@@ -120,7 +131,7 @@ def check_and_run_pack(items, shards, n_buckets, bucket_bytes, shard_bytes):
         if kind in (ITEM_F32_VEC, ITEM_BF16_VEC):
             assert off % 16 == 0 and L % 8 == 0 and soff % 16 == 0
             assert R == 1 or (st * es) % 16 == 0
-        assert soff + ((R - 1) * st + L) * es <= shard_bytes
+        assert soff + ((R - 1) * st + L) * es <= min(shard_bytes, len(shards[shard]))
         idx = soff + (np.arange(R, dtype=np.int64)[:, None] * st * es
                       + np.arange(L, dtype=np.int64)[None, :] * es).ravel()
         raw = np.zeros(idx.size, np.uint32)

@@ -19,7 +19,7 @@ import paper_2512_22492_gb300 as rr
 @dataclass
 class SyncBuffers:
     plan: "rr.Plan"
-    flat: torch.Tensor                 # n_shards * shard_bytes, uint8
+    flat: torch.Tensor                 # every source buffer, 16-byte starts, uint8
     shards: List[int]                  # device pointers into flat
     bucket_store: torch.Tensor         # [n_buckets, row >= bucket_bytes] uint8 (uniform layout)
     buckets: list                      # what is passed as the bucket array
@@ -35,11 +35,12 @@ def make_plan(manifest, src, dst, bucket_bytes, **opts):
 def alloc(plan, separate_buckets: bool = False, poison: Optional[int] = 0xAB,
           with_dst: bool = True, flat: Optional[torch.Tensor] = None) -> SyncBuffers:
     dev = torch.device("cuda")
+    starts = source_offsets(plan)
     if flat is None:
-        flat = torch.zeros(plan.n_shards * plan.shard_bytes, dtype=torch.uint8, device=dev)
-    assert flat.numel() == plan.n_shards * plan.shard_bytes
+        flat = torch.zeros(starts[-1], dtype=torch.uint8, device=dev)
+    assert flat.numel() == starts[-1]
     base = flat.data_ptr()
-    shards = [base + s * plan.shard_bytes for s in range(plan.n_shards)]
+    shards = [base + o for o in starts[:-1]]
     if separate_buckets:
         # Separately allocated buckets (pointer-table launch shape).
         # Shuffled so that the pointers are not equally spaced.
@@ -68,6 +69,16 @@ def alloc(plan, separate_buckets: bool = False, poison: Optional[int] = 0xAB,
     return SyncBuffers(plan, flat, shards, bucket_store, buckets, checksums, dst)
 
 
+def source_offsets(plan) -> List[int]:
+    """Byte offset of every source buffer in one allocation (each at a 16-byte
+    start), then the total.  Shards of one FlatParameter follow one another."""
+    out, off = [], 0
+    for nb in plan.source_buffer_bytes:
+        out.append(off)
+        off += (nb + 15) // 16 * 16
+    return out + [off]
+
+
 def fill_from_host(buf: SyncBuffers, host_shards) -> None:
     host = np.concatenate([np.asarray(s, np.uint8) for s in host_shards])
     assert host.size == buf.flat.numel()
@@ -92,6 +103,17 @@ def fill_with_generator(buf: SyncBuffers, manifest, seed: int, specials: bool,
     trainer) at the library's offsets."""
     plan = buf.plan
     base = buf.flat.data_ptr()
+    if plan.sharding == "units":
+        # Each unit's shards are adjacent, so the unit is one flat buffer.
+        starts = source_offsets(plan)
+        per_unit = plan.n_shards // (max(plan.units) + 1)
+        flat = _flat_offsets(manifest, plan.align_bytes)
+        for p, local, f, u in zip(manifest, plan.param_flat_offset, flat, plan.units):
+            es = 4 if p.dtype == "f32" else 2
+            n = int(np.prod(p.shape)) if len(p.shape) else 1
+            synth.fill_dev(base + starts[u * per_unit] + local, n, es, seed, first_idx=f // es,
+                           specials=specials, stream=stream)
+        return
     if plan.sharding == "flat":
         for p, off in zip(manifest, plan.param_flat_offset):
             es = 4 if p.dtype == "f32" else 2

@@ -63,15 +63,17 @@ def full_parity(desc, separate_buckets=False, **opts):
 
 @pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2",
                                   "tiny-moe-f32", "tiny-fsdp2", "tiny-moe-kvrep",
-                                  "tiny-kvrep-f32", "tiny-moe-bf16-specials"])
+                                  "tiny-kvrep-f32", "tiny-moe-bf16-specials", "tiny-units",
+                                  "tiny-moe-ep4", "tiny-moe-units-ep2"])
 def test_small_workloads(name):
     full_parity(U.workload_desc(name))
 
 
-@pytest.mark.parametrize("name", ["tiny-fsdp2", "tiny-moe-kvrep"])
+@pytest.mark.parametrize("name", ["tiny-fsdp2", "tiny-moe-kvrep", "tiny-units",
+                                  "tiny-moe-units-ep2"])
 def test_device_generator_fill_matches_oracle_shards(name):
-    """The harness's device fill of a row-sharded trainer equals the oracle's host
-    shards byte for byte (both indexed by the flat layout)."""
+    """The harness's device fill of a row-sharded or per-layer-unit trainer equals
+    the oracle's host shards byte for byte (both indexed by the flat layout)."""
     desc = U.workload_desc(name)
     L = U.to_oracle(desc)
     m, s, d = U.to_product(desc)
@@ -237,6 +239,24 @@ def test_qwen3_30b_a3b_fsdp2_tp8_sampled():
     torch.cuda.empty_cache()
     _unpack_sampled("qwen3-30b-a3b-fsdp2-tp8", [("layers.1.qkv_proj", 3), ("layers.1.qkv_proj", 2),
                                                 ("layers.40.experts.w13", 6), ("norm", 7)])
+    torch.cuda.empty_cache()
+
+
+def test_qwen3_8b_units_sampled():
+    """FSDP1 wrapping every decoder layer: 37 FlatParameters of 8 shards each."""
+    sampled_parity("qwen3-8b-units", n_random_buckets=3)
+    torch.cuda.empty_cache()
+    _unpack_sampled("qwen3-8b-units", [("embed_tokens", 0), ("layers.0.qkv_proj", 0),
+                                       ("layers.35.down_proj", 0), ("lm_head", 0)])
+    torch.cuda.empty_cache()
+
+
+def test_qwen3_30b_a3b_fsdp2_ep8_sampled():
+    """FSDP2 trainer, expert-parallel rollout over 8 ranks: 16 whole experts each."""
+    sampled_parity("qwen3-30b-a3b-fsdp2-ep8", n_random_buckets=1)
+    torch.cuda.empty_cache()
+    _unpack_sampled("qwen3-30b-a3b-fsdp2-ep8", [("layers.2.experts.w13", 5),
+                                                ("layers.47.experts.w2", 7), ("norm", 0)])
     torch.cuda.empty_cache()
 
 

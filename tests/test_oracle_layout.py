@@ -113,8 +113,9 @@ def _to_bf16_bits(t: torch.Tensor) -> torch.Tensor:
     return torch.where(nan, nan_bits, conv)
 
 
-def restate_rollout(shape, P, tp):
-    """Per rank, the rollout tensors built the way an inference engine's loader would."""
+def restate_rollout(shape, P, tp, ep=False):
+    """Per rank, the rollout tensors built the way an inference engine's loader
+    would; ep: each rank loads its own experts whole."""
     H = shape.hidden
 
     def kv(t, r):
@@ -137,7 +138,15 @@ def restate_rollout(shape, P, tp):
             ts.append(P[a + "k_norm.weight"])
             ts.append(P[pre + "input_layernorm.weight"])
             ts.append(P[pre + "post_attention_layernorm.weight"])
-            if shape.n_experts:
+            if shape.n_experts and ep:
+                ex = pre + "mlp.experts."
+                mine = torch.arange(shape.n_experts).chunk(tp)[r].tolist()
+                ts.append(P[pre + "mlp.gate.weight"])
+                ts.append(torch.stack([torch.cat([P[f"{ex}{e}.gate_proj.weight"],
+                                                  P[f"{ex}{e}.up_proj.weight"]], 0)
+                                       for e in mine]))
+                ts.append(torch.stack([P[f"{ex}{e}.down_proj.weight"] for e in mine]))
+            elif shape.n_experts:
                 ex = pre + "mlp.experts."
                 ts.append(P[pre + "mlp.gate.weight"])
                 ts.append(torch.stack([
@@ -190,8 +199,32 @@ def fsdp2_shards(params, P, n, align=16):
     return shards
 
 
+def fsdp1_unit_shards(params, P, n, align=16):
+    """Trainer shards as FSDP1 holds them when every decoder layer is wrapped:
+    one FlatParameter per layer and one for the root (embedding, final norm,
+    lm_head); each is its parameters flattened and concatenated in manifest
+    order at `align`-byte starts, zero-padded to a multiple of 16 * n bytes and
+    cut into n equal shards.  Returned unit by unit (root first, then layers)."""
+    def unit(name):
+        return 1 + int(name.split(".")[2]) if name.startswith("model.layers.") else 0
+    n_units = 1 + max(unit(name) for name, _, _ in params)
+    shards = []
+    for u in range(n_units):
+        flat = bytearray()
+        for name, dims, es in params:
+            if unit(name) != u:
+                continue
+            flat += bytes((-len(flat)) % max(align, es))
+            flat += P[name].contiguous().numpy().tobytes()
+        flat += bytes((-len(flat)) % (16 * n))
+        shards += [np.frombuffer(bytes(c.numpy().tobytes()), np.uint8).copy()
+                   for c in torch.frombuffer(bytearray(flat), dtype=torch.uint8).chunk(n)]
+    return shards
+
+
 RESTATE = ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2", "tiny-moe-f32",
-           "tiny-fsdp2", "tiny-moe-kvrep", "tiny-kvrep-f32", "tiny-moe-bf16-specials"]
+           "tiny-fsdp2", "tiny-moe-kvrep", "tiny-kvrep-f32", "tiny-moe-bf16-specials",
+           "tiny-units", "tiny-moe-ep4", "tiny-moe-units-ep2"]
 
 
 def _workload(name):
@@ -204,12 +237,15 @@ def test_oracle_matches_restatement(name):
     w = _workload(name)
     L = oracle.workload_layout(w)
     P = _param_tensors(L.params, _flat_offsets(L.params), w.seed, w.specials)
-    ranks = restate_rollout(w.shape, P, w.tp)
+    ranks = restate_rollout(w.shape, P, w.tp, ep=w.ep)
     # Per-tensor reshard, straight from trainer shards: materialised by the
-    # oracle for a flat trainer, built with torch.chunk for an FSDP2 one.
-    if w.sharding == "rows":
-        shards = fsdp2_shards(L.params, P, w.n_shards)
-        for a, b in zip(shards, L.host_shards(w.seed, w.specials)):
+    # oracle for a flat trainer, built with torch for FSDP2 and per-layer FSDP1.
+    if w.sharding in ("rows", "units"):
+        build = fsdp2_shards if w.sharding == "rows" else fsdp1_unit_shards
+        shards = build(L.params, P, w.n_shards)
+        host = L.host_shards(w.seed, w.specials)
+        assert len(shards) == len(host)
+        for a, b in zip(shards, host):
             np.testing.assert_array_equal(a, b)
     else:
         shards = L.host_shards(w.seed, w.specials)
@@ -237,7 +273,8 @@ def test_oracle_matches_restatement(name):
 @pytest.mark.parametrize("n_shards,sharding", [(1, "flat"), (2, "flat"), (3, "flat"),
                                                (7, "flat"), (8, "flat"), (13, "flat"),
                                                (1, "rows"), (3, "rows"), (8, "rows"),
-                                               (13, "rows"), (300, "rows")])
+                                               (13, "rows"), (300, "rows"),
+                                               (1, "units"), (3, "units"), (8, "units")])
 def test_shard_count_invariance(n_shards, sharding):
     w = synth.TEST_WORKLOADS["tiny-tp4"]
     ref_L = oracle.workload_layout(w.with_(n_shards=1))
@@ -259,13 +296,13 @@ def test_generator_mode_matches_buffer_mode():
 
 @pytest.mark.parametrize("name", ["qwen3-0.6b", "qwen3-8b", "qwen3-8b-tp4", "qwen3-30b-a3b",
                                   "tiny-moe-tp2", "qwen3-8b-fsdp2-tp8",
-                                  "qwen3-30b-a3b-fsdp2-tp8"])
+                                  "qwen3-30b-a3b-fsdp2-tp8", "qwen3-30b-a3b-fsdp2-ep8"])
 def test_coverage_counts(name):
     """Every parameter element is read tp times if replicated, once otherwise, and
     within one rank no parameter element is read twice (metadata only: full sizes)."""
     w = _workload(name)
     params = qwen3.manifest(w.shape, w.src_elem_bytes)
-    tensors = qwen3.rollout_tensors(w.shape, params, w.tp)
+    tensors = qwen3.rollout_tensors(w.shape, params, w.tp, ep=w.ep)
     area = np.zeros(len(params), np.int64)
     per_rank = {}
     for _, r, blocks in tensors:
@@ -380,3 +417,54 @@ def test_shard_size_rule_edge():
     shards[2][32:34] = [0x34, 0x12]
     got = L.reshard_tensor(oracle.Source(shards=shards), 0)
     assert list(got) == [0x1234]
+
+
+def test_unit_sharding_worked_example():
+    """Two FSDP1 units over 2 shards, worked by hand.
+
+    Unit 0 holds a (3 bf16) and c (5 bf16); unit 1 holds b (10 f32).
+    Unit 0: a at byte 0 (6 B); c at the next 16-byte start, 16 (10 B); the end,
+    26, pads to a multiple of 16 * 2 = 32, so S_0 = 16: a is in buffer 0 at 0,
+    c in buffer 1 at 0.  Unit 1: b at 0 (40 B) pads to 64, S_1 = 32: b's
+    elements 0..7 are buffer 2 bytes 0..31, elements 8 and 9 buffer 3 bytes 0..7."""
+    params = [("a", (3,), 2), ("b", (10,), 4), ("c", (5,), 2)]
+    tensors = [("c", 0, [(2, 0, 5, 0, 1)]), ("b", 0, [(1, 0, 10, 0, 1)])]
+    L = oracle.Layout(params, tensors, n_shards=2, tp=1, bucket_bytes=64, sharding="units",
+                      units=[0, 1, 0])
+    assert list(L.param_offset) == [0, 0, 16]
+    assert list(L.unit_shard_bytes) == [16, 32]
+    bufs = [np.zeros(16, np.uint8), np.zeros(16, np.uint8), np.zeros(32, np.uint8),
+            np.zeros(32, np.uint8)]
+    bufs[1][0:10] = np.array([0x11, 0x3F, 0x22, 0x3F, 0x33, 0x3F, 0x44, 0x3F, 0x55, 0x3F],
+                             np.uint8)                      # c = bf16 0x3F11 .. 0x3F55
+    b_vals = np.arange(1, 11, dtype=np.float32)             # b = 1.0 .. 10.0, exact in bf16
+    bufs[2][:] = b_vals[:8].view(np.uint8)
+    bufs[3][0:8] = b_vals[8:].view(np.uint8)
+    src = oracle.Source(shards=bufs)
+    assert list(L.reshard_tensor(src, 0)) == [0x3F11, 0x3F22, 0x3F33, 0x3F44, 0x3F55]
+    want_b = (b_vals.view(np.uint32) >> 16).astype(np.uint16)
+    np.testing.assert_array_equal(L.reshard_tensor(src, 1), want_b)
+
+
+def test_unit_shard_size_rule_edge():
+    """A unit whose size over the shard count truncates onto a multiple of 16.
+
+    Unit 0 holds p (25 bf16 = 50 B) over 3 shards: 50 pads to 96 (a multiple of
+    16 * 3), so S_0 = 32 and element 24 (byte 48) is buffer 1 at byte 16.  Unit
+    1 holds q (4 f32 = 16 B): 16 pads to 48, S_1 = 16, buffers 3..5."""
+    params = [("p", (25,), 2), ("q", (4,), 4)]
+    tensors = [("p", 0, [(0, 0, 25, 0, 1)]), ("q", 0, [(1, 0, 4, 0, 1)])]
+    L = oracle.Layout(params, tensors, n_shards=3, tp=1, bucket_bytes=128, sharding="units",
+                      units=[0, 1])
+    assert list(L.unit_shard_bytes) == [32, 16]
+    bufs = [np.zeros(32, np.uint8) for _ in range(3)] + [np.zeros(16, np.uint8) for _ in range(3)]
+    p_vals = np.arange(0x3F00, 0x3F00 + 25, dtype=np.uint16)
+    flat0 = np.zeros(96, np.uint8)
+    flat0[:50] = p_vals.view(np.uint8)
+    for s in range(3):
+        bufs[s][:] = flat0[32 * s:32 * (s + 1)]
+    assert bufs[1][16] == 0x18 and bufs[1][17] == 0x3F       # element 24 where it belongs
+    bufs[3][:] = np.full(4, 0xC0000000, np.uint32).view(np.uint8)   # q = -2.0 each
+    src = oracle.Source(shards=bufs)
+    np.testing.assert_array_equal(L.reshard_tensor(src, 0), p_vals)
+    assert list(L.reshard_tensor(src, 1)) == [0xC000] * 4

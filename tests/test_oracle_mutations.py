@@ -60,6 +60,14 @@ MUTATIONS = [
      "L->param_gen_base[p] = (start % 4096) / P->elem_bytes;"),
     ("little-endian source bytes read reversed", "v |= (uint32_t)byte << (8 * i);",
      "v |= (uint32_t)byte << (8 * (es - 1 - i));"),
+    ("unit buffers numbered shard-major", "int64_t buf = (int64_t)u * L->n_shards + f / Su;",
+     "int64_t buf = (f / Su) * L->n_units + u;"),
+    ("unit size not padded for the shard count",
+     "L->unit_shard_bytes[u] = align_up(local, 16 * (int64_t)L->n_shards) / L->n_shards;",
+     "L->unit_shard_bytes[u] = align_up(local / L->n_shards, 16);"),
+    ("unit parameters not aligned",
+     "                local = align_up(local, a);\n                L->param_offset[p] = local;",
+     "                L->param_offset[p] = local + 0 * a;"),
 ]
 
 
@@ -81,6 +89,10 @@ def battery():
         ("restatement bf16 specials",
          lambda: layout_pins.test_oracle_matches_restatement("tiny-moe-bf16-specials")),
         ("shard size edge", layout_pins.test_shard_size_rule_edge),
+        ("units golden", layout_pins.test_unit_sharding_worked_example),
+        ("unit shard size edge", layout_pins.test_unit_shard_size_rule_edge),
+        ("restatement tiny-units", lambda: layout_pins.test_oracle_matches_restatement("tiny-units")),
+        ("restatement EP", lambda: layout_pins.test_oracle_matches_restatement("tiny-moe-ep4")),
         ("round trip", lambda: layout_pins.test_unpack_of_pack_is_reshard("tiny-tp4")),
         ("shard invariance", lambda: layout_pins.test_shard_count_invariance(7, "flat")),
     ]

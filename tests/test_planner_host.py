@@ -37,13 +37,20 @@ def host_plan(desc, **opt):
 
 
 @pytest.mark.parametrize("name", ["tiny", "qwen3-0.6b", "qwen3-8b", "qwen3-8b-tp4",
-                                  "qwen3-30b-a3b", "tiny-moe-tp2"])
+                                  "qwen3-30b-a3b", "tiny-moe-tp2", "tiny-units",
+                                  "tiny-moe-units-ep2", "qwen3-8b-units",
+                                  "qwen3-30b-a3b-fsdp2-ep8"])
 def test_geometry_matches_oracle(name):
     desc = U.workload_desc(name)
     L = U.to_oracle(desc)
     p = host_plan(desc)
     assert p.n_buckets == L.n_buckets
     assert p.shard_bytes == L.shard_bytes and p.flat_bytes == L.flat_bytes
+    if L.sharding == "units":
+        assert p.source_buffer_bytes == [int(s) for s in L.unit_shard_bytes
+                                         for _ in range(L.n_shards)]
+    elif L.sharding != "tensors":
+        assert p.source_buffer_bytes == [L.shard_bytes] * L.n_shards
     assert p.param_flat_offset == list(L.param_offset)
     assert p.first_bucket_of_rank == list(L.rank_first_bucket)
     assert p.stream_bytes_per_rank == list(L.rank_stream_bytes)
@@ -69,7 +76,8 @@ def run_and_compare(desc, **opt):
 
 
 @pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe", "tiny-moe-tp2",
-                                  "tiny-moe-f32"])
+                                  "tiny-moe-f32", "tiny-fsdp2", "tiny-units", "tiny-moe-ep4",
+                                  "tiny-moe-units-ep2"])
 def test_tables_reproduce_oracle_workloads(name):
     run_and_compare(U.workload_desc(name))
 
@@ -142,6 +150,19 @@ def test_rejections():
     assert status(src=misaligned) == rrmod.RR_ELAYOUT
     assert status(dst=rr.DstLayout(tp=1, tensors=good.tensors, tensor_align_bytes=3)) \
         == rrmod.RR_EINVAL
+    # Per-module FSDP1 units.
+    rr.rr_plan_create(params, rr.SrcLayout(n_shards=2, sharding="units", units=[1, 0]), good, 64,
+                      opts)
+    assert status(src=rr.SrcLayout(n_shards=2, sharding="units", units=[0, 2])) \
+        == rrmod.RR_EINVAL                                   # unit 1 holds nothing
+    assert status(src=rr.SrcLayout(n_shards=2, sharding="units", units=[-1, 0])) \
+        == rrmod.RR_EINVAL                                   # unit out of range
+    assert status(src=rr.SrcLayout(n_shards=2, sharding="units")) == rrmod.RR_EINVAL
+    assert status(src=rr.SrcLayout(n_shards=2, units=[0, 0])) == rrmod.RR_EINVAL   # flat
+    assert status(src=rr.SrcLayout(n_shards=2, sharding="units", units=[0, 0],
+                                   param_flat_offset=[0, 96])) == rrmod.RR_EINVAL
+    assert status(src=rr.SrcLayout(n_shards=40000, sharding="units", units=[0, 1])) \
+        == rrmod.RR_EINVAL                                   # 80000 source buffers
 
 
 def test_host_only_plan_refuses_to_run():
