@@ -230,6 +230,9 @@ typedef struct {
     int64_t unpack_bytes_read;   /* bucket bytes read by one rr_unpack                  */
     int64_t unpack_bytes_written;/* destination bytes written by one rr_unpack          */
     int64_t verify_bytes_read;   /* bucket bytes read by one rr_verify                  */
+    int64_t n_pack_full_items;   /* items of the whole-sync pack table (see
+                                    rr_plan_export_pack_full); equals n_pack_items
+                                    when no fan-out groups were found                  */
 } rr_plan_stats;
 
 rr_status rr_plan_get_stats(const rr_plan* plan, rr_plan_stats* stats);
@@ -246,7 +249,10 @@ enum {
     RR_ITEM_COPY_VEC = 6,   /* unpack: 16-byte copies                                */
     RR_ITEM_COPY_SCALAR = 7, /* unpack: 2-byte copies                                */
     RR_ITEM_READ_VEC = 8,    /* unpack table: alignment gap / tail, read only by the    */
-    RR_ITEM_READ_SCALAR = 9  /*   verifying unpack (their bytes count in the checksum)  */
+    RR_ITEM_READ_SCALAR = 9, /*   verifying unpack (their bytes count in the checksum)  */
+    RR_ITEM_FAN_F32 = 10,    /* whole-sync table only: fan-out head (see below)         */
+    RR_ITEM_FAN_BF16 = 11,
+    RR_ITEM_FAN_DST = 12     /* one destination of the fan-out head before it           */
 };
 
 /* Pack work item: n_rows rows of row_len elements; row i starts at source
@@ -281,6 +287,24 @@ typedef struct {
  * unpack) into caller memory. */
 rr_status rr_plan_export_pack(const rr_plan* plan, rr_pack_item* items, int64_t cap,
                               uint32_t* block_first);
+
+/* The whole-sync pack table: what rr_pack runs on the bulk-copy engine when it
+ * packs every bucket.  It holds the items of rr_plan_export_pack (bucket-sorted,
+ * used by the range calls and the register path) except where several rollout
+ * ranks take narrow column slices (under 1 KiB of source per row) of the same
+ * parameter rows -- a row-parallel weight under tensor parallelism.  Those
+ * slices become fan-out groups that read each source row once:
+ *   head (RR_ITEM_FAN_F32 / RR_ITEM_FAN_BF16): n_rows rows of row_len source
+ *        elements (the slices' joint column span) at src, src_stride elements
+ *        apart; dst_off = the number of RR_ITEM_FAN_DST items that follow;
+ *   each RR_ITEM_FAN_DST: src = the slice's first column within the span,
+ *        row_len = its width, and the slice of row i goes to bucket `bucket`
+ *        at dst_off + 2 * i * row_len.
+ * Every slice is 16-byte aligned in source and destination and a multiple of 8
+ * elements wide; no destination run crosses a bucket.  The per-block ranges
+ * never separate a head from its destinations. */
+rr_status rr_plan_export_pack_full(const rr_plan* plan, rr_pack_item* items, int64_t cap,
+                                   uint32_t* block_first);
 rr_status rr_plan_export_unpack(const rr_plan* plan, rr_unpack_item* items, int64_t cap,
                                 uint32_t* block_first);
 

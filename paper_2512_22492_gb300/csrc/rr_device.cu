@@ -487,6 +487,7 @@ constexpr uint32_t kWaitLimit = 1u << 20;        // tries, each suspending at mo
 constexpr uint32_t kWaitHintNs = 1000;
 constexpr uint64_t kWaitDeadlineNs = 1000000000;  // and at most one second of wall clock
 constexpr unsigned int kErrWaitTimeout = 1;
+constexpr unsigned int kErrBadItem = 2;           // an item the engine cannot stage
 
 enum : uint16_t {
     PC_CAST = 1,      // stage holds fp32 rows -> bf16 destination
@@ -496,10 +497,12 @@ enum : uint16_t {
     PC_ZERO_VEC = 5,  // 16-byte zero stores
     PC_ZERO_SCALAR = 6,
     PC_END = 7,
-    PC_GATHER = 8     // aligned rows too short for bulk copies: 16-byte loads by consumers
+    PC_FAN = 8        // stage holds whole rows; every fan-out destination takes its slice
 };
 
 constexpr uint32_t kMinBulkRowBytes = 1024;
+constexpr int kFullArrivals = 33;   // per piece: the metadata arrival + one per producer lane
+constexpr uint32_t kMaxFanDst = 16; // fan-out destinations per head (the planner's limit)
 
 struct Piece {
     const char* src;      // first source element (global)
@@ -570,54 +573,29 @@ __device__ __forceinline__ void consumers_sync() {
     asm volatile("bar.sync 1, %0;" ::"n"(kConsumerThreads) : "memory");
 }
 
-// Rows of a PC_GATHER piece: 16-byte-aligned rows of row_len (a multiple of 8)
-// elements at src_stride, landing contiguously at dst.  Thread t of NT takes
-// 8-element vectors t, t + NT, ...; four in flight per thread.
-template <int ES, int NT>
-__device__ __forceinline__ unsigned long long gather_rows(const Piece& p, uint32_t t) {
-    constexpr int U = ES == 4 ? 4 : 8;
-    const uint32_t vpr = p.row_len >> 3;
-    const uint32_t nvec = vpr * p.rows;
-    const uint32_t dq = NT / vpr, dr = NT - dq * vpr;
-    uint32_t v = t, r = v / vpr, c = v - r * vpr;
-    unsigned long long acc = 0;
-    while (v < nvec) {
-        uint4 x[U][ES / 2];
-        uint32_t vv[U];
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            vv[u] = v;
-            if (v < nvec) {
-                const char* q = p.src + r * p.src_stride + (uint64_t)c * (8 * ES);
-                x[u][0] = ld_stream(q);
-                if (ES == 4) x[u][ES / 2 - 1] = ld_stream(q + 16);
-            }
-            v += NT;
-            c += dr;
-            r += dq;
-            if (c >= vpr) {
-                c -= vpr;
-                ++r;
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            if (vv[u] < nvec) {
-                uint4 o;
-                if (ES == 4) {
-                    o.x = cast2(x[u][0].x, x[u][0].y);
-                    o.y = cast2(x[u][0].z, x[u][0].w);
-                    o.z = cast2(x[u][ES / 2 - 1].x, x[u][ES / 2 - 1].y);
-                    o.w = cast2(x[u][ES / 2 - 1].z, x[u][ES / 2 - 1].w);
-                } else {
-                    o = x[u][0];
-                }
-                st_stream(p.dst + 16ull * vv[u], o);
-                acc += words(o);
-            }
+// Short aligned rows (16-byte aligned, row bytes a multiple of 16) gathered
+// into a stage by the whole producer warp: 16-byte cp.async copies, lane l
+// taking vectors l, l + 32, ...; the rows land back to back.  Each lane's
+// completion is one arrival on the stage's full barrier.
+__device__ __forceinline__ void gather_async(uint32_t stage, uint32_t full_bar, const char* src,
+                                             uint64_t src_stride, uint32_t rows,
+                                             uint32_t row_bytes, uint32_t lane) {
+    const uint32_t vpr = row_bytes >> 4;
+    const uint32_t nv = vpr * rows;
+    const uint32_t dq = 32 / vpr, dr = 32 - dq * vpr;
+    uint32_t r = lane / vpr, c = lane - r * vpr;
+    for (uint32_t v = lane; v < nv; v += 32) {
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(stage + 16 * v),
+                     "l"(src + r * src_stride + 16ull * c)
+                     : "memory");
+        c += dr;
+        r += dq;
+        if (c >= vpr) {
+            c -= vpr;
+            ++r;
         }
     }
-    return acc;
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(full_bar) : "memory");
 }
 
 template <int NPTR>
@@ -635,13 +613,16 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
     extern __shared__ __align__(128) char stage_mem[];
     __shared__ __align__(8) uint64_t full[kStages], empty[kStages];
     __shared__ Piece meta[kStages];
+    __shared__ rr_pack_item fan_dst[MODE == 0 ? kStages : 1][kMaxFanDst];   // PC_FAN slices
     __shared__ bool last_block;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     constexpr bool kSum = MODE != 1;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
-            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full[s])) : "memory");
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(&full[s])),
+                         "n"(kFullArrivals)
+                         : "memory");
             asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(&empty[s])),
                          "n"(kConsumerWarps)
                          : "memory");
@@ -655,30 +636,55 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
-        if (lane != 0) return;
+        // The whole warp walks the items in step (every lane decodes the same
+        // item).  Each piece takes kFullArrivals arrivals on its stage's full
+        // barrier: lane 0's plain (release) arrival after it wrote the piece's
+        // metadata, then one per lane for the data -- lane 0's carrying the
+        // byte count of its bulk copies, a gather's being its lanes' cp.async
+        // completions, plain otherwise.
+        enum { kMeta = 0, kBulk = 1, kGather = 2 };
         uint32_t count = 0;   // pieces issued
         bool ok = true;
-        auto emit = [&](const Piece& p, bool bulk) {
+        auto emit = [&](const Piece& p, int how) {
             const int s = (int)(count % kStages);
             if (count >= (uint32_t)kStages &&
-                !mbar_wait(smem_u32(&empty[s]), ((count / kStages) - 1) & 1, a.err)) {
+                !__all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&empty[s]),
+                                                   ((count / kStages) - 1) & 1, a.err))) {
                 ok = false;
                 return;
             }
-            meta[s] = p;
             const uint32_t fb = smem_u32(&full[s]);
-            if (bulk) {
-                const uint32_t row_bytes = p.row_len * p.es;
+            if constexpr (MODE == 0) {
+                // A fan-out piece carries its destination items in shared memory.
+                if (p.kind == PC_FAN && lane < p.n)
+                    fan_dst[s][lane] = ((const rr_pack_item*)a.items)[p.sum_bucket + lane];
+                __syncwarp();
+            }
+            if (lane == 0) {
+                meta[s] = p;
+                mbar_arrive(fb);
+            }
+            const uint32_t stage = smem_u32(stage_mem + s * kStageBytes);
+            const uint32_t row_bytes = p.row_len * p.es;
+            if (how == kGather) {
+                gather_async(stage, fb, p.src, p.src_stride, p.rows, row_bytes, lane);
+            } else if (how == kBulk && lane == 0) {
                 asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb),
                              "r"(row_bytes * p.rows)
                              : "memory");
-                for (uint32_t r = 0; r < p.rows; ++r)
+                if (p.rows > 1 && p.src_stride == row_bytes)   // rows back to back: one copy
                     asm volatile(
                         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes "
-                        "[%0], [%1], %2, [%3];" ::"r"(smem_u32(stage_mem + s * kStageBytes +
-                                                               r * row_bytes)),
-                        "l"(p.src + r * p.src_stride), "r"(row_bytes), "r"(fb)
+                        "[%0], [%1], %2, [%3];" ::"r"(stage),
+                        "l"(p.src), "r"(row_bytes * p.rows), "r"(fb)
                         : "memory");
+                else
+                    for (uint32_t r = 0; r < p.rows; ++r)
+                        asm volatile(
+                            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes "
+                            "[%0], [%1], %2, [%3];" ::"r"(stage + r * row_bytes),
+                            "l"(p.src + r * p.src_stride), "r"(row_bytes), "r"(fb)
+                            : "memory");
             } else {
                 mbar_arrive(fb);
             }
@@ -709,21 +715,13 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                                 p.src = src + r * sstride + (uint64_t)e0 * es;
                                 p.dst = dst + 2ull * ((uint64_t)r * L + e0);
                                 p.sum_off = d.dst_off + 2u * (r * L + e0);
-                                emit(p, true);
+                                emit(p, kBulk);
                             }
-                    } else if (L * es < kMinBulkRowBytes) {
-                        // Many short rows: one bulk copy per row would make the single
-                        // producer the bottleneck.  Consumers gather them directly.
-                        p.kind = PC_GATHER;
-                        p.src = src;
-                        p.dst = dst;
-                        p.rows = R;
-                        p.row_len = L;
-                        p.n = L * R;
-                        p.src_stride = sstride;
-                        p.sum_off = d.dst_off;
-                        emit(p, false);
                     } else {
+                        // Whole rows per stage.  Rows under kMinBulkRowBytes are gathered
+                        // by the warp's 16-byte cp.async copies (one bulk copy per short
+                        // row would leave a single issuing lane the bottleneck).
+                        const int how = L * es < kMinBulkRowBytes ? kGather : kBulk;
                         const uint32_t k = kStageBytes / (L * es);
                         for (uint32_t r0 = 0; r0 < R && ok; r0 += k) {
                             p.rows = min(k, R - r0);
@@ -733,9 +731,35 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                             p.src = src + r0 * sstride;
                             p.dst = dst + 2ull * r0 * L;
                             p.sum_off = d.dst_off + 2u * r0 * L;
-                            emit(p, true);
+                            emit(p, how);
                         }
                     }
+                } else if (d.kind == RR_ITEM_FAN_F32 || d.kind == RR_ITEM_FAN_BF16) {
+                    // Whole rows of the slices' span, staged once; the destination
+                    // items that follow the head are read by the consumers.
+                    const uint32_t es = d.kind == RR_ITEM_FAN_F32 ? 4 : 2;
+                    const uint32_t rb = d.row_len * es, R = d.n_rows, nd = d.dst_off;
+                    if (rb > (uint32_t)kStageBytes || rb % 16 != 0 || nd > kMaxFanDst) {
+                        if (lane == 0) atomicExch(a.err, kErrBadItem);
+                        ok = false;
+                        break;
+                    }
+                    const uint64_t sstride = (uint64_t)d.src_stride * es;
+                    const int how = rb < kMinBulkRowBytes ? kGather : kBulk;
+                    const uint32_t k = kStageBytes / rb;
+                    p.kind = PC_FAN;
+                    p.es = (uint16_t)es;
+                    p.row_len = d.row_len;
+                    p.src_stride = sstride;
+                    p.sum_bucket = it + 1;   // index of the first destination item
+                    p.n = nd;
+                    for (uint32_t r0 = 0; r0 < R && ok; r0 += k) {
+                        p.rows = min(k, R - r0);
+                        p.src = src + r0 * sstride;
+                        p.sum_off = r0;      // first row of this piece within the item
+                        emit(p, how);
+                    }
+                    it += nd;
                 } else if (d.kind == RR_ITEM_ZERO_VEC || d.kind == RR_ITEM_ZERO_SCALAR) {
                     p.kind = d.kind == RR_ITEM_ZERO_VEC ? PC_ZERO_VEC : PC_ZERO_SCALAR;
                     p.dst = dst;
@@ -745,7 +769,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     p.es = 2;
                     p.src = nullptr;
                     p.sum_off = d.dst_off;
-                    emit(p, false);
+                    emit(p, kMeta);
                 } else {
                     p.kind = PC_SCALAR;
                     p.es = d.kind == RR_ITEM_F32_SCALAR ? 4 : 2;
@@ -756,7 +780,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     p.n = d.row_len * d.n_rows;
                     p.src_stride = (uint64_t)d.src_stride * p.es;
                     p.sum_off = d.dst_off;
-                    emit(p, false);
+                    emit(p, kMeta);
                 }
             } else {
                 const rr_unpack_item d = ((const rr_unpack_item*)a.items)[it];
@@ -776,7 +800,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                         p.src = src + o;
                         p.dst = dst ? dst + o : nullptr;
                         p.sum_off = d.src_off + o;
-                        emit(p, true);
+                        emit(p, kBulk);
                     }
                 } else {
                     p.kind = PC_SCALAR;
@@ -786,21 +810,23 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     p.rows = 1;
                     p.row_len = p.n;
                     p.sum_off = d.src_off;
-                    emit(p, false);
+                    emit(p, kMeta);
                 }
             }
         }
         if (ok) {
             Piece end;
             end.kind = PC_END;
-            emit(end, false);
+            emit(end, kMeta);
         }
-        if (!ok) {
-            // Let the loads still in flight land before this block's shared memory goes away.
+        if (!ok && lane == 0) {
+            // Let the bulk loads still in flight land before this block's shared
+            // memory goes away.
             const uint32_t from = count > (uint32_t)kStages ? count - kStages : 0;
             for (uint32_t c = from; c < count; ++c)
                 mbar_wait(smem_u32(&full[c % kStages]), (c / kStages) & 1, a.err);
         }
+        asm volatile("cp.async.wait_all;" ::: "memory");
         return;
     }
 
@@ -817,7 +843,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
         if (!ok) break;
         const Piece p = meta[s];
         if (p.kind == PC_END) break;
-        if (kSum && p.sum_bucket != cur) {
+        if (kSum && p.kind != PC_FAN && p.sum_bucket != cur) {
             if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - sum_base), acc);
             cur = p.sum_bucket;
             acc = 0;
@@ -857,12 +883,48 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     if (kSum) acc += (unsigned long long)h << (8 * ((p.sum_off + 2 * e) & 7));
                 }
                 break;
-            case PC_GATHER:   // pack only
+            case PC_FAN:   // pack only
                 if constexpr (MODE == 0) {
-                    if (p.es == 4)
-                        acc += gather_rows<4, kCT>(p, ct);
-                    else
-                        acc += gather_rows<2, kCT>(p, ct);
+                    // Units of work: each slice's rows in q parts (q spreads the slices
+                    // over all consumer warps); one warp per unit, one sum per unit.
+                    const uint32_t nd = p.n;
+                    const uint32_t q = (kConsumerWarps + nd - 1) / nd;
+                    for (uint32_t u = warp - 1; u < nd * q; u += kConsumerWarps) {
+                        const rr_pack_item d = fan_dst[s][u / q];
+                        const uint32_t part = u % q;
+                        const uint32_t r0 = p.rows * part / q, r1 = p.rows * (part + 1) / q;
+                        const uint32_t vpr = d.row_len >> 3, nv = (r1 - r0) * vpr;
+                        const uint32_t dq = 32 / vpr, dr = 32 - dq * vpr;
+                        const char* base =
+                            st + ((uint64_t)r0 * p.row_len + (uint32_t)d.src) * p.es;
+                        char* out = bulk_bucket(a, d.bucket, a.n_shards) + d.dst_off +
+                                    2ull * (p.sum_off + r0) * d.row_len;
+                        uint32_t r = lane / vpr, c = lane - r * vpr;
+                        unsigned long long am = 0;
+                        for (uint32_t v = lane; v < nv; v += 32) {
+                            const char* q8 = base + ((uint64_t)r * p.row_len + 8u * c) * p.es;
+                            uint4 o;
+                            if (p.es == 4) {
+                                const uint4 x0 = *(const uint4*)q8;
+                                const uint4 x1 = *(const uint4*)(q8 + 16);
+                                o.x = cast2(x0.x, x0.y);
+                                o.y = cast2(x0.z, x0.w);
+                                o.z = cast2(x1.x, x1.y);
+                                o.w = cast2(x1.z, x1.w);
+                            } else {
+                                o = *(const uint4*)q8;
+                            }
+                            st_stream(out + 16ull * v, o);
+                            am += words(o);
+                            c += dr;
+                            r += dq;
+                            if (c >= vpr) {
+                                c -= vpr;
+                                ++r;
+                            }
+                        }
+                        flush(a.sums + d.bucket, am);
+                    }
                 }
                 break;
             case PC_ZERO_VEC:
@@ -1089,6 +1151,12 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         a.block_first = R.full ? P->d_pack_block_first : nullptr;
         a.item_begin = P->pack_bucket_first[R.b0];
         a.item_end = P->pack_bucket_first[R.b1];
+        if (R.full && P->d_full_items) {   // every bucket: the table with fan-out groups
+            a.items = P->d_full_items;
+            a.block_first = P->d_full_block_first;
+            a.item_begin = 0;
+            a.item_end = uint32_t(P->full_items.size());
+        }
         a.sums = (unsigned long long*)checksums;
         a.n_shards = P->n_shards;
         for (int32_t i = 0; i < P->n_shards; ++i) a.ptr[k++] = src_shards[i];
@@ -1346,7 +1414,12 @@ rr_status rr_device_upload(rr_plan* P) {
         (e = cudaHostAlloc((void**)&P->h_verify_result, 5 * sizeof(unsigned long long),
                            cudaHostAllocDefault)) != cudaSuccess ||
         (e = cudaMalloc((void**)&P->d_error, sizeof(unsigned int))) != cudaSuccess ||
-        (e = cudaMemset(P->d_error, 0, sizeof(unsigned int))) != cudaSuccess)
+        (e = cudaMemset(P->d_error, 0, sizeof(unsigned int))) != cudaSuccess ||
+        (!P->full_items.empty() &&
+         ((e = up((void**)&P->d_full_items, P->full_items.data(),
+                  P->full_items.size() * sizeof(rr_pack_item))) != cudaSuccess ||
+          (e = up((void**)&P->d_full_block_first, P->full_block_first.data(),
+                  P->full_block_first.size() * sizeof(uint32_t))) != cudaSuccess)))
         return e == cudaErrorMemoryAllocation ? rr_fail(RR_ENOMEM, "device allocation failed")
                                               : cuda_fail(e, "plan upload");
     return RR_OK;
@@ -1359,6 +1432,8 @@ void rr_device_release(rr_plan* P) {
     if (prev != P->device) cudaSetDevice(P->device);
     cudaFree(P->d_pack_items);
     cudaFree(P->d_pack_block_first);
+    cudaFree(P->d_full_items);
+    cudaFree(P->d_full_block_first);
     cudaFree(P->d_unpack_items);
     cudaFree(P->d_unpack_block_first);
     cudaFree(P->d_verify_scratch);
@@ -1367,6 +1442,8 @@ void rr_device_release(rr_plan* P) {
     P->d_error = nullptr;
     P->d_pack_items = nullptr;
     P->d_pack_block_first = nullptr;
+    P->d_full_items = nullptr;
+    P->d_full_block_first = nullptr;
     P->d_unpack_items = nullptr;
     P->d_unpack_block_first = nullptr;
     P->d_verify_scratch = nullptr;

@@ -50,6 +50,9 @@ struct rr_plan {
     std::vector<rr_unpack_item> unpack_items;
     std::vector<uint32_t> unpack_block_first;   // grid_blocks + 1
     std::vector<uint32_t> pack_bucket_first;    // n_buckets + 1: first pack item of bucket b
+    std::vector<rr_pack_item> full_items;       // whole-sync table with fan-out groups;
+                                                // empty when it would equal pack_items
+    std::vector<uint32_t> full_block_first;     // grid_blocks + 1
     std::vector<uint32_t> unpack_bucket_first;  // n_buckets + 1: first unpack item of bucket b
     rr_plan_stats stats{};
 
@@ -57,6 +60,8 @@ struct rr_plan {
     int device = -1;
     rr_pack_item* d_pack_items = nullptr;
     uint32_t* d_pack_block_first = nullptr;
+    rr_pack_item* d_full_items = nullptr;
+    uint32_t* d_full_block_first = nullptr;
     rr_unpack_item* d_unpack_items = nullptr;
     uint32_t* d_unpack_block_first = nullptr;
     unsigned long long* d_verify_scratch = nullptr;  // n_buckets sums + 4 counters

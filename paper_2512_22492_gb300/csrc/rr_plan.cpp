@@ -16,7 +16,9 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <map>
 #include <new>
+#include <tuple>
 
 #include "rr_internal.h"
 
@@ -27,13 +29,28 @@ thread_local std::string g_error;
 constexpr int64_t kDefaultChunkBytes = 32 * 1024;
 constexpr int64_t kItemOverhead = 1024;   // balancing weight of one item, in bytes
 constexpr int64_t kMaxShardOffset = (int64_t(1) << 48) - 1;
+// Fan-out groups: column slices narrower than kFanSliceBytes of source per row,
+// at most kMaxFanDst of them, over a joint span of at most kFanMaxRowBytes.
+constexpr int64_t kFanSliceBytes = 1024;
+constexpr int64_t kMaxFanDst = 16;
+constexpr int64_t kFanMaxRowBytes = 16 * 1024;
 
 int64_t align_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
 
+// One member of a fan-out group: a column slice of the group's rows that lands
+// contiguously in rank `rank`'s stream at byte `pos`.
+struct FanSlice {
+    int32_t rank;
+    int64_t pos, col0, ncols;
+};
+
 class Builder {
 public:
-    explicit Builder(rr_plan* p) : P(p), chunk_elems(p->chunk_bytes / 2) {}
+    explicit Builder(rr_plan* p) : P(p), chunk_elems(p->chunk_bytes / 2), out(&p->pack_items) {}
+
+    // Pack items go to `o` from here on (the bucket-sorted table by default).
+    void set_out(std::vector<rr_pack_item>* o) { out = o; }
 
     // ---- pack ------------------------------------------------------------
 
@@ -159,11 +176,71 @@ public:
         }
     }
 
+    // Rows [row0, row0 + nrows) of parameter p, columns [cmin, cmin + span),
+    // are cut into column slices m (sorted, adjacent) for several ranks: one
+    // fan-out head per run of rows that stays in one shard and keeps every
+    // slice inside one bucket, followed by one destination item per slice.
+    // Rows that straddle a shard or put a slice across a bucket boundary go
+    // out as plain items.
+    void fan_group(int32_t p, int64_t row0, int64_t nrows, int64_t cmin, int64_t span,
+                   const std::vector<FanSlice>& m) {
+        const int32_t es = P->es[p];
+        const int64_t C = P->cols[p], B = P->bucket_bytes;
+        // Heads are cut into stage-sized pieces by the kernel; this only bounds
+        // the balancing granularity (16 chunks of source per head).
+        const int64_t max_rows = std::max<int64_t>(1, 16 * P->chunk_bytes / (span * es));
+        int64_t i = 0;
+        while (i < nrows) {
+            const Loc at = loc(p, (row0 + i) * C + cmin);
+            int64_t k = 0;
+            if (at.room >= span * es && at.off % 16 == 0) {
+                k = std::min({nrows - i, (at.room - span * es) / (C * es) + 1, max_rows});
+                for (const FanSlice& s : m) {
+                    const int64_t boff = (s.pos + 2 * i * s.ncols) % B;
+                    k = std::min(k, (B - boff) / (2 * s.ncols));
+                }
+            }
+            if (k < 1) {
+                for (const FanSlice& s : m)
+                    pack_run(p, (row0 + i) * C + s.col0, s.ncols, 1, C, s.rank,
+                             s.pos + 2 * i * s.ncols);
+                ++i;
+                continue;
+            }
+            const int64_t fb0 = P->rank_first_bucket[m[0].rank];
+            rr_pack_item h;
+            h.src = (uint64_t(at.shard) << 48) | uint64_t(at.off);
+            h.dst_off = uint32_t(m.size());
+            h.bucket = uint32_t(fb0 + (m[0].pos + 2 * i * m[0].ncols) / B);
+            h.row_len = uint32_t(span);
+            h.n_rows = uint32_t(k);
+            h.src_stride = uint32_t(C);
+            h.kind = uint16_t(es == 4 ? RR_ITEM_FAN_F32 : RR_ITEM_FAN_BF16);
+            h.reserved = 0;
+            out->push_back(h);
+            for (const FanSlice& s : m) {
+                const int64_t at_pos = s.pos + 2 * i * s.ncols;
+                rr_pack_item d;
+                d.src = uint64_t(s.col0 - cmin);
+                d.dst_off = uint32_t(at_pos % B);
+                d.bucket = uint32_t(P->rank_first_bucket[s.rank] + at_pos / B);
+                d.row_len = uint32_t(s.ncols);
+                d.n_rows = uint32_t(k);
+                d.src_stride = 0;
+                d.kind = uint16_t(RR_ITEM_FAN_DST);
+                d.reserved = 0;
+                out->push_back(d);
+            }
+            i += k;
+        }
+    }
+
     int64_t pack_read = 0;
 
 private:
     rr_plan* P;
     int64_t chunk_elems;
+    std::vector<rr_pack_item>* out;
 
     void emit_pack(int kind, int64_t shard, int64_t soff, int64_t bucket, int64_t boff,
                    int64_t row_len, int64_t n_rows, int64_t stride) {
@@ -176,8 +253,8 @@ private:
         it.src_stride = uint32_t(stride);
         it.kind = uint16_t(kind);
         it.reserved = 0;
-        P->pack_items.push_back(it);
-        if (kind <= RR_ITEM_BF16_SCALAR)
+        out->push_back(it);
+        if (kind <= RR_ITEM_BF16_SCALAR && out == &P->pack_items)
             pack_read += row_len * n_rows * (kind <= RR_ITEM_F32_SCALAR ? 4 : 2);
     }
 
@@ -262,6 +339,9 @@ int64_t pack_weight(const rr_pack_item& it) {
         case RR_ITEM_F32_SCALAR: return 12 * n + kItemOverhead;
         case RR_ITEM_BF16_VEC: return 4 * n + kItemOverhead;
         case RR_ITEM_BF16_SCALAR: return 8 * n + kItemOverhead;
+        case RR_ITEM_FAN_F32: return 6 * n + kItemOverhead;
+        case RR_ITEM_FAN_BF16: return 4 * n + kItemOverhead;
+        case RR_ITEM_FAN_DST: return 0;
         default: return 2 * n + kItemOverhead;
     }
 }
@@ -478,8 +558,70 @@ rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_
     return RR_OK;
 }
 
+// Fan-out groups: blocks of the same parameter rows whose column slices are
+// narrow, 16-byte aligned, and tile one contiguous span.  Returns, per group,
+// its slices; marks each member block in `member` ([tensor][block] -> group).
+struct FanGroup {
+    int32_t param;
+    int64_t row0, nrows, cmin, span;
+    std::vector<FanSlice> slices;
+};
+
+std::vector<FanGroup> find_fan_groups(const rr_plan* P, const rr_dst_layout* dst,
+                                      std::vector<std::vector<int32_t>>& member) {
+    std::map<std::tuple<int32_t, int64_t, int64_t>, std::vector<std::pair<int32_t, int32_t>>> by;
+    member.assign(size_t(P->n_tensors), {});
+    for (int32_t t = 0; t < P->n_tensors; ++t) {
+        const rr_dst_tensor& T = dst->tensors[t];
+        member[t].assign(size_t(T.n_blocks), -1);
+        for (int32_t k = 0; k < T.n_blocks; ++k) {
+            const rr_block& bl = T.blocks[k];
+            if (bl.nrows > 0 && bl.ncols > 0 && bl.ncols < P->cols[bl.param])
+                by[{bl.param, bl.row0, bl.nrows}].push_back({t, k});
+        }
+    }
+    std::vector<FanGroup> groups;
+    for (auto& kv : by) {
+        auto& v = kv.second;
+        if (v.size() < 2 || int64_t(v.size()) > kMaxFanDst) continue;
+        const int32_t p = std::get<0>(kv.first);
+        const int32_t es = P->es[p];
+        const int64_t C = P->cols[p];
+        std::vector<FanSlice> s;
+        for (auto [t, k] : v) {
+            const rr_block& bl = dst->tensors[t].blocks[k];
+            int64_t pos = P->tensor_off[t];
+            for (int32_t j = 0; j < k; ++j)
+                pos += 2 * dst->tensors[t].blocks[j].nrows * dst->tensors[t].blocks[j].ncols;
+            s.push_back({P->tensor_rank[t], pos, bl.col0, bl.ncols});
+        }
+        std::vector<size_t> order(s.size());
+        for (size_t i = 0; i < order.size(); ++i) order[i] = i;
+        std::sort(order.begin(), order.end(),
+                  [&](size_t a, size_t b) { return s[a].col0 < s[b].col0; });
+        std::vector<FanSlice> m;
+        for (size_t i : order) m.push_back(s[i]);
+        const int64_t cmin = m[0].col0;
+        bool ok = (C * es) % 16 == 0;
+        for (size_t i = 0; i < m.size() && ok; ++i) {
+            ok = m[i].ncols % 8 == 0 && m[i].ncols * es < kFanSliceBytes &&
+                 ((m[i].col0 - cmin) * es) % 16 == 0 && m[i].pos % 16 == 0 &&
+                 (i == 0 || m[i].col0 == m[i - 1].col0 + m[i - 1].ncols);
+        }
+        const int64_t span = m.back().col0 + m.back().ncols - cmin;
+        if (!ok || span * es > kFanMaxRowBytes) continue;
+        const int32_t g = int32_t(groups.size());
+        for (auto [t, k] : v) member[t][k] = g;
+        groups.push_back({p, std::get<1>(kv.first), std::get<2>(kv.first), cmin, span, m});
+    }
+    return groups;
+}
+
 void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     Builder b(P);
+    std::vector<std::vector<int32_t>> member;
+    const std::vector<FanGroup> groups = find_fan_groups(P, dst, member);
+    std::vector<std::pair<size_t, size_t>> fanned;   // regular items of grouped blocks
     for (int32_t r = 0; r < P->tp; ++r) {
         int64_t cursor = 0;   // end of the previous tensor in the stream
         for (int32_t t = 0; t < P->n_tensors; ++t) {
@@ -490,11 +632,13 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
             for (int32_t k = 0; k < T.n_blocks; ++k) {
                 const rr_block& bl = T.blocks[k];
                 const int64_t C = P->cols[bl.param];
+                const size_t before = P->pack_items.size();
                 if (bl.ncols == C)   // whole rows: one contiguous run
                     b.pack_run(bl.param, bl.row0 * C, bl.nrows * bl.ncols, 1, bl.nrows * bl.ncols,
                                r, pos);
                 else
                     b.pack_run(bl.param, bl.row0 * C + bl.col0, bl.ncols, bl.nrows, C, r, pos);
+                if (member[t][k] >= 0) fanned.push_back({before, P->pack_items.size()});
                 pos += 2 * bl.nrows * bl.ncols;
             }
             cursor = pos;
@@ -524,6 +668,45 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     partition(P->pack_items, P->grid_blocks, P->pack_block_first, pack_weight);
     partition(P->unpack_items, P->unpack_grid_blocks, P->unpack_block_first, unpack_weight);
 
+    // Whole-sync table: the grouped blocks' plain items give way to fan-out groups.
+    P->full_items.clear();
+    P->full_block_first.clear();
+    if (!groups.empty()) {
+        std::vector<char> drop(P->pack_items.size(), 0);
+        for (auto [lo, hi] : fanned)
+            for (size_t i = lo; i < hi; ++i) drop[i] = 1;
+        std::vector<rr_pack_item> kept, fan;
+        for (size_t i = 0; i < P->pack_items.size(); ++i)
+            if (!drop[i]) kept.push_back(P->pack_items[i]);
+        b.set_out(&fan);
+        for (const FanGroup& g : groups) b.fan_group(g.param, g.row0, g.nrows, g.cmin, g.span, g.slices);
+        b.set_out(&P->pack_items);
+        // Spread the fan-out heads (with their destinations, and the plain items
+        // of rows that fell back) evenly through the table, so that every block
+        // of the balanced split gets its share of them.
+        std::vector<size_t> unit_start;   // fan items in runs: a head and its destinations
+        for (size_t i = 0; i < fan.size(); ++i)
+            if (fan[i].kind != RR_ITEM_FAN_DST) unit_start.push_back(i);
+        unit_start.push_back(fan.size());
+        const size_t U = unit_start.size() - 1;
+        P->full_items.reserve(kept.size() + fan.size());
+        size_t k = 0;
+        for (size_t u = 0; u < U; ++u) {
+            const size_t upto = kept.size() * u / U;
+            for (; k < upto; ++k) P->full_items.push_back(kept[k]);
+            for (size_t i = unit_start[u]; i < unit_start[u + 1]; ++i)
+                P->full_items.push_back(fan[i]);
+        }
+        for (; k < kept.size(); ++k) P->full_items.push_back(kept[k]);
+        partition(P->full_items, P->grid_blocks, P->full_block_first, pack_weight);
+        // A block never starts on a fan-out destination item.
+        auto& f = P->full_block_first;
+        for (size_t g = 1; g + 1 < f.size(); ++g) {
+            f[g] = std::max(f[g], f[g - 1]);
+            while (f[g] < P->full_items.size() && P->full_items[f[g]].kind == RR_ITEM_FAN_DST) ++f[g];
+        }
+    }
+
     rr_plan_stats& s = P->stats;
     s.n_pack_items = int64_t(P->pack_items.size());
     s.n_unpack_items = int64_t(P->unpack_items.size());
@@ -541,6 +724,8 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     s.unpack_bytes_read = dst_bytes;
     s.unpack_bytes_written = dst_bytes;
     s.verify_bytes_read = int64_t(P->n_buckets) * P->bucket_bytes;
+    s.n_pack_full_items = int64_t(P->full_items.empty() ? P->pack_items.size()
+                                                        : P->full_items.size());
 }
 
 }  // namespace
@@ -594,7 +779,8 @@ rr_status rr_plan_create_ex(const rr_param* manifest, int32_t n_params,
         }
         if (st == RR_OK) {
             build_tables(P, dst);
-            if (P->pack_items.size() >= 0xFFFFFFFFull || P->unpack_items.size() >= 0xFFFFFFFFull)
+            if (P->pack_items.size() >= 0xFFFFFFFFull || P->unpack_items.size() >= 0xFFFFFFFFull ||
+                P->full_items.size() >= 0xFFFFFFFFull)
                 st = rr_fail(RR_ELAYOUT, "too many work items; raise chunk_bytes");
         }
         if (st == RR_OK && !P->host_only) st = rr_device_upload(P);
@@ -677,6 +863,17 @@ rr_status rr_plan_export_pack(const rr_plan* P, rr_pack_item* items, int64_t cap
     if (n > 0) std::memcpy(items, P->pack_items.data(), size_t(n) * sizeof(rr_pack_item));
     if (block_first)
         std::copy(P->pack_block_first.begin(), P->pack_block_first.end(), block_first);
+    return RR_OK;
+}
+
+rr_status rr_plan_export_pack_full(const rr_plan* P, rr_pack_item* items, int64_t cap,
+                                   uint32_t* block_first) {
+    if (!P || (cap > 0 && !items)) return rr_fail(RR_EINVAL, "NULL argument");
+    if (P->full_items.empty()) return rr_plan_export_pack(P, items, cap, block_first);
+    const int64_t n = std::min<int64_t>(cap, int64_t(P->full_items.size()));
+    if (n > 0) std::memcpy(items, P->full_items.data(), size_t(n) * sizeof(rr_pack_item));
+    if (block_first)
+        std::copy(P->full_block_first.begin(), P->full_block_first.end(), block_first);
     return RR_OK;
 }
 

@@ -74,7 +74,7 @@ class _Stats(ctypes.Structure):
                 ("bucket_bytes", ctypes.c_int64),
                 ("pack_bytes_read", ctypes.c_int64), ("pack_bytes_written", ctypes.c_int64),
                 ("unpack_bytes_read", ctypes.c_int64), ("unpack_bytes_written", ctypes.c_int64),
-                ("verify_bytes_read", ctypes.c_int64)]
+                ("verify_bytes_read", ctypes.c_int64), ("n_pack_full_items", ctypes.c_int64)]
 
 
 class PackItem(ctypes.Structure):
@@ -128,6 +128,8 @@ _sig("rr_plan_tensors", [_vp, _P64, _P64])
 _sig("rr_plan_get_stats", [_vp, ctypes.POINTER(_Stats)])
 _sig("rr_plan_export_pack", [_vp, ctypes.POINTER(PackItem), ctypes.c_int64,
                              ctypes.POINTER(ctypes.c_uint32)])
+_sig("rr_plan_export_pack_full", [_vp, ctypes.POINTER(PackItem), ctypes.c_int64,
+                                  ctypes.POINTER(ctypes.c_uint32)])
 _sig("rr_plan_export_unpack", [_vp, ctypes.POINTER(UnpackItem), ctypes.c_int64,
                                ctypes.POINTER(ctypes.c_uint32)])
 _sig("rr_pack", [_vp, ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _vp])
@@ -154,7 +156,7 @@ _sig("rr_last_error", [], ctypes.c_char_p)
 LIBRARY_PATH = _build.LIB
 EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_query",
             "rr_plan_source", "rr_plan_source_buffers", "rr_plan_tensors", "rr_plan_get_stats",
-            "rr_plan_export_pack",
+            "rr_plan_export_pack", "rr_plan_export_pack_full",
             "rr_plan_export_unpack", "rr_plan_bucket_items", "rr_pack", "rr_unpack", "rr_verify",
             "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
             "rr_unpack_verify", "rr_unpack_verify_range",
@@ -306,6 +308,18 @@ class Plan:
         _check(_lib.rr_plan_export_pack(self._h, items.ctypes.data_as(ctypes.POINTER(PackItem)),
                                         n, first.ctypes.data_as(ctypes.POINTER(ctypes.c_uint32))),
                "rr_plan_export_pack")
+        return items[:n], first
+
+    def export_pack_full(self):
+        """The whole-sync pack table (fan-out groups included) and its per-block
+        first item, as rr_pack runs it on the bulk-copy engine for every bucket."""
+        import numpy as np
+        n = self.stats()["n_pack_full_items"]
+        items = np.zeros(max(1, n), dtype=PACK_ITEM_DTYPE)
+        first = np.zeros(self.stats()["grid_blocks"] + 1, dtype=np.uint32)
+        _check(_lib.rr_plan_export_pack_full(
+            self._h, items.ctypes.data_as(ctypes.POINTER(PackItem)), n,
+            first.ctypes.data_as(ctypes.POINTER(ctypes.c_uint32))), "rr_plan_export_pack_full")
         return items[:n], first
 
     def export_unpack(self):

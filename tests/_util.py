@@ -13,7 +13,8 @@ import oracle
 import synth
 
 ITEM_F32_VEC, ITEM_F32_SCALAR, ITEM_BF16_VEC, ITEM_BF16_SCALAR, ITEM_ZERO_VEC, \
-    ITEM_ZERO_SCALAR, ITEM_COPY_VEC, ITEM_COPY_SCALAR, ITEM_READ_VEC, ITEM_READ_SCALAR = range(10)
+    ITEM_ZERO_SCALAR, ITEM_COPY_VEC, ITEM_COPY_SCALAR, ITEM_READ_VEC, ITEM_READ_SCALAR, \
+    ITEM_FAN_F32, ITEM_FAN_BF16, ITEM_FAN_DST = range(13)
 
 
 def workload(name):
@@ -114,8 +115,39 @@ def check_and_run_pack(items, shards, n_buckets, bucket_bytes, shard_bytes):
     that every bucket byte is written exactly once.  Returns the buckets."""
     out = np.zeros((n_buckets, bucket_bytes), np.uint8)
     hits = np.zeros((n_buckets, bucket_bytes), np.uint16)
-    for it in items:
+    items = list(items)
+    skip = 0
+    for j, it in enumerate(items):
+        if skip:
+            skip -= 1
+            continue
         kind, b, off = int(it["kind"]), int(it["bucket"]), int(it["dst_off"])
+        assert kind != ITEM_FAN_DST, "fan-out destination without its head"
+        if kind in (ITEM_FAN_F32, ITEM_FAN_BF16):
+            es = 4 if kind == ITEM_FAN_F32 else 2
+            span, R, st = int(it["row_len"]), int(it["n_rows"]), int(it["src_stride"])
+            shard, soff = int(it["src"]) >> 48, int(it["src"]) & ((1 << 48) - 1)
+            assert soff % 16 == 0 and (span * es) % 16 == 0 and (st * es) % 16 == 0
+            assert soff + ((R - 1) * st + span) * es <= min(shard_bytes, len(shards[shard]))
+            rows = np.stack([shards[shard][soff + i * st * es:soff + (i * st + span) * es]
+                             for i in range(R)])
+            skip = off
+            covered = np.zeros(span, np.int32)
+            for d in items[j + 1:j + 1 + off]:
+                assert int(d["kind"]) == ITEM_FAN_DST and int(d["n_rows"]) == R
+                c0, w = int(d["src"]), int(d["row_len"])
+                db, doff = int(d["bucket"]), int(d["dst_off"])
+                assert w % 8 == 0 and doff % 16 == 0 and (c0 * es) % 16 == 0
+                assert 0 <= db < n_buckets and doff + 2 * R * w <= bucket_bytes
+                covered[c0:c0 + w] += 1
+                raw = np.zeros((R, w), np.uint32)
+                for k in range(es):
+                    raw |= rows[:, c0 * es + k:(c0 + w) * es:es].astype(np.uint32) << (8 * k)
+                vals = oracle.rne_bf16(raw) if es == 4 else raw.astype(np.uint16)
+                out[db, doff:doff + 2 * R * w] = vals.reshape(-1).astype("<u2").view(np.uint8)
+                hits[db, doff:doff + 2 * R * w] += 1
+            assert np.all(covered <= 1), "fan-out slices overlap"
+            continue
         L, R, st = int(it["row_len"]), int(it["n_rows"]), int(it["src_stride"])
         n = L * R
         assert 0 <= b < n_buckets and off % 2 == 0 and off + 2 * n <= bucket_bytes

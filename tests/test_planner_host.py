@@ -67,6 +67,13 @@ def run_and_compare(desc, **opt):
     U.check_partition(first, len(items))
     got = U.check_and_run_pack(items, shards, p.n_buckets, p.bucket_bytes, p.shard_bytes)
     np.testing.assert_array_equal(got, want)
+    # The whole-sync table (fan-out groups in place of narrow slices) packs the same bytes.
+    fitems, ffirst = p.export_pack_full()
+    U.check_partition(ffirst, len(fitems))
+    starts = ffirst[:-1][ffirst[:-1] < len(fitems)]
+    assert not np.any(fitems["kind"][starts] == U.ITEM_FAN_DST)
+    got = U.check_and_run_pack(fitems, shards, p.n_buckets, p.bucket_bytes, p.shard_bytes)
+    np.testing.assert_array_equal(got, want)
     uitems, ufirst = p.export_unpack()
     U.check_partition(ufirst, len(uitems))
     tensors = U.check_and_run_unpack(uitems, want, p.tensor_numel)
@@ -116,6 +123,35 @@ def test_full_size_tables_are_consistent():
     data = items["kind"] <= U.ITEM_BF16_SCALAR
     assert (n[data] * 4).sum() == st["pack_bytes_read"]
     assert np.all(items["kind"][data] == U.ITEM_F32_VEC)
+
+
+def test_fan_out_groups_on_full_size_tables():
+    """Qwen3-30B-A3B FSDP2 -> TP=8: every expert down_proj's eight 96-column slices
+    form one group per shard run of rows (metadata only)."""
+    desc = U.workload_desc("qwen3-30b-a3b-fsdp2-tp8")
+    p = host_plan(desc)
+    items, first = p.export_pack_full()
+    U.check_partition(first, len(items))
+    kind = items["kind"]
+    heads = np.flatnonzero((kind == U.ITEM_FAN_F32) | (kind == U.ITEM_FAN_BF16))
+    # One head per shard run of 256 rows, and a few more where a bucket boundary
+    # cuts a run; a row whose slice would straddle a boundary goes out as plain items.
+    assert 48 * 128 * 8 <= len(heads) < 48 * 128 * 8 + 64
+    assert np.all(items["dst_off"][heads] == 8) and np.all(items["row_len"][heads] == 768)
+    assert np.all(items["n_rows"][heads] <= 256)
+    fanned_rows = int(items["n_rows"][heads].astype(np.int64).sum())
+    assert 48 * 128 * 2048 - 64 <= fanned_rows <= 48 * 128 * 2048
+    dsts = np.flatnonzero(kind == U.ITEM_FAN_DST)
+    assert len(dsts) == 8 * len(heads) and np.all(items["row_len"][dsts] == 96)
+    # Every bucket byte is written exactly once: plain items plus fan-out slices.
+    n = items["row_len"].astype(np.int64) * items["n_rows"]
+    plain = kind < U.ITEM_FAN_F32
+    per_bucket = np.zeros(p.n_buckets, np.int64)
+    np.add.at(per_bucket, items["bucket"][plain].astype(np.int64), 2 * n[plain])
+    np.add.at(per_bucket, items["bucket"][dsts].astype(np.int64), 2 * n[dsts])
+    assert np.all(per_bucket == p.bucket_bytes)
+    starts = first[:-1][first[:-1] < len(items)]
+    assert not np.any(kind[starts] == U.ITEM_FAN_DST)
 
 
 def test_rejections():
