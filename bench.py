@@ -47,6 +47,11 @@ def parse():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--workload", default="qwen3-8b")
     ap.add_argument("--bucket-mib", type=int, default=0, help="override the bucket size")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="keep only the first N decoder layers (a small case of the same "
+                         "kernels, for profiler captures); the workload name says so")
+    ap.add_argument("--vocab", type=int, default=0,
+                    help="with --layers: a smaller vocabulary as well")
     ap.add_argument("--chunk-kib", type=int, default=0, help="plan option: KiB per work item")
     ap.add_argument("--grid", type=int, default=0, help="plan option: persistent grid size")
     ap.add_argument("--snapshot", action="store_true",
@@ -468,6 +473,11 @@ def main():
     import synth
     w = (synth.WORKLOADS.get(args.workload) or synth.TEST_WORKLOADS.get(args.workload)
          or synth.EXTRA_WORKLOADS[args.workload])
+    if args.layers:
+        import dataclasses
+        vocab = args.vocab or w.shape.vocab
+        w = w.with_(name=f"{w.name}-first{args.layers}layers-vocab{vocab}",
+                    shape=dataclasses.replace(w.shape, layers=args.layers, vocab=vocab))
     bucket_bytes = args.bucket_mib * (1 << 20) if args.bucket_mib else w.bucket_bytes
     world, rank, local = dist_setup(args)
     if args.impl == "reference":
