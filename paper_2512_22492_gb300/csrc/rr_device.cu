@@ -739,12 +739,22 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     // items that follow the head are read by the consumers.
                     const uint32_t es = d.kind == RR_ITEM_FAN_F32 ? 4 : 2;
                     const uint32_t rb = d.row_len * es, R = d.n_rows, nd = d.dst_off;
-                    if (rb > (uint32_t)kStageBytes || rb % 16 != 0 || nd > kMaxFanDst) {
+                    const uint64_t sstride = (uint64_t)d.src_stride * es;
+                    // The planner guarantees the alignments the vector paths need;
+                    // a table that breaks them is refused, not run.
+                    bool bad = rb > (uint32_t)kStageBytes || rb % 16 != 0 || nd > kMaxFanDst ||
+                               it + 1 + nd > i1 || (uintptr_t)src % 16 != 0 || sstride % 16 != 0;
+                    if (!bad && lane < nd) {
+                        const rr_pack_item f = ((const rr_pack_item*)a.items)[it + 1 + lane];
+                        bad = f.kind != RR_ITEM_FAN_DST || f.row_len % 8 != 0 ||
+                              f.dst_off % 16 != 0 || (f.src * es) % 16 != 0 ||
+                              f.src + f.row_len > d.row_len;
+                    }
+                    if (__any_sync(0xFFFFFFFFu, bad)) {
                         if (lane == 0) atomicExch(a.err, kErrBadItem);
                         ok = false;
                         break;
                     }
-                    const uint64_t sstride = (uint64_t)d.src_stride * es;
                     const int how = rb < kMinBulkRowBytes ? kGather : kBulk;
                     const uint32_t k = kStageBytes / rb;
                     p.kind = PC_FAN;

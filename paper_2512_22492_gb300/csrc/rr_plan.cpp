@@ -602,7 +602,7 @@ std::vector<FanGroup> find_fan_groups(const rr_plan* P, const rr_dst_layout* dst
         std::vector<FanSlice> m;
         for (size_t i : order) m.push_back(s[i]);
         const int64_t cmin = m[0].col0;
-        bool ok = (C * es) % 16 == 0;
+        bool ok = (C * es) % 16 == 0 && P->bucket_bytes % 16 == 0;
         for (size_t i = 0; i < m.size() && ok; ++i) {
             ok = m[i].ncols % 8 == 0 && m[i].ncols * es < kFanSliceBytes &&
                  ((m[i].col0 - cmin) * es) % 16 == 0 && m[i].pos % 16 == 0 &&

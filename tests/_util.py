@@ -74,6 +74,47 @@ def random_layout(seed: int, max_params: int = 7, bucket_choices=(8, 24, 40, 64,
     return desc
 
 
+def random_tp_layout(seed: int):
+    """Row-parallel weights cut by columns over several ranks (the planner's
+    fan-out groups), with cuts placed to hit every fallback: slice widths that
+    are or are not multiples of 8, tensor alignments that keep or break 16-byte
+    destinations, small buckets that cut through slices, flat shards that cut
+    through rows, partial row ranges, fp32 and bf16, and some whole-row
+    (replicated) blocks in between."""
+    rng = np.random.default_rng(seed + 7_000_001)
+    tp = int(rng.choice([2, 3, 4, 8]))
+    n_params = int(rng.integers(2, 6))
+    params, per_rank = [], [[] for _ in range(tp)]
+    for i in range(n_params):
+        es = int(rng.choice([2, 4]))
+        w = 8 * int(rng.integers(1, 9)) if rng.random() < 0.8 else int(rng.integers(1, 40))
+        extra = 8 * int(rng.integers(1, 3)) if rng.random() < 0.3 else 0
+        rows, cols = int(rng.integers(1, 90)), w * tp + extra
+        params.append((f"p{i}", (rows, cols), es))
+        r0 = int(rng.integers(0, rows)) if rng.random() < 0.3 else 0
+        nr = rows - r0 if rng.random() < 0.7 else int(rng.integers(1, rows - r0 + 1))
+        c_off = extra if rng.random() < 0.5 else 0
+        for r in range(tp):
+            per_rank[r].append((f"p{i}.slice", r, [(i, r0, nr, c_off + r * w, w)]))
+        if rng.random() < 0.3:
+            for r in range(tp):
+                per_rank[r].append((f"p{i}.whole", r, [(i, 0, rows, 0, cols)]))
+    tensors = []
+    for r in range(tp):
+        order = rng.permutation(len(per_rank[r]))
+        tensors += [per_rank[r][k] for k in order]
+    sharding = str(rng.choice(["flat", "flat", "rows", "units"]))
+    desc = dict(params=params, tensors=tensors, tp=tp, sharding=sharding,
+                n_shards=int(rng.integers(1, 6)),
+                bucket_bytes=int(rng.choice([64, 200, 1024, 4096, 8192, 65536])),
+                align_bytes=int(rng.choice([16, 16, 4, 32])),
+                tensor_align=int(rng.choice([256, 256, 16, 2])),
+                seed=int(rng.integers(1, 1 << 20)), specials=bool(rng.random() < 0.5))
+    if sharding == "units":
+        desc["units"] = [int(u) for u in rng.permutation(np.arange(n_params) % 2)]
+    return desc
+
+
 def workload_desc(name, bucket_bytes=None):
     w = workload(name)
     from oracle import qwen3

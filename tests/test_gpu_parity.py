@@ -101,6 +101,29 @@ def test_random_layouts(seed):
                 engine="registers" if seed % 3 == 0 else "auto")
 
 
+@pytest.mark.parametrize("seed", range(16))
+def test_random_row_parallel_layouts(seed):
+    """Fan-out groups (narrow column slices over several ranks) and their
+    fallbacks, through a full rr_pack and, on the bucket-sorted table, through
+    rr_pack_range over two ranges; the register engine on every third seed."""
+    desc = U.random_tp_layout(seed)
+    full_parity(desc, separate_buckets=bool(seed % 2),
+                engine="registers" if seed % 3 == 0 else "auto")
+    L = U.to_oracle(desc)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"])
+    buf = H.alloc(plan, with_dst=False)
+    shards = L.host_shards(desc["seed"], desc["specials"])
+    H.fill_from_host(buf, shards)
+    cut = plan.n_buckets // 3
+    for a, b in ((cut, plan.n_buckets), (0, cut)):
+        rr.rr_pack_range(plan, a, b - a, buf.shards, buf.buckets, buf.checksums)
+    torch.cuda.synchronize()
+    want, want_cs = L.pack(oracle.Source(shards=shards))
+    np.testing.assert_array_equal(H.buckets_host(buf), want)
+    np.testing.assert_array_equal(H.checksums_host(buf), want_cs)
+
+
 @pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-moe-f32", "tiny-fsdp2"])
 def test_register_engine(name):
     """The register path (the fallback for host-resident buffers) on device memory."""

@@ -99,6 +99,23 @@ def test_tables_random_layouts(seed):
     run_and_compare(U.random_layout(seed), grid_blocks=7)
 
 
+@pytest.mark.parametrize("seed", range(48))
+def test_tables_random_row_parallel_layouts(seed):
+    """Fan-out groups and all their fallbacks, through both tables."""
+    run_and_compare(U.random_tp_layout(seed), grid_blocks=5)
+
+
+def test_random_row_parallel_layouts_exercise_fan_out():
+    """The generator above does produce fan-out groups, and plain fallbacks."""
+    heads = plain_rows = 0
+    for seed in range(48):
+        p = host_plan(U.random_tp_layout(seed))
+        items, _ = p.export_pack_full()
+        heads += int(np.sum((items["kind"] == U.ITEM_FAN_F32) | (items["kind"] == U.ITEM_FAN_BF16)))
+        plain_rows += int(p.stats()["n_pack_full_items"] == p.stats()["n_pack_items"])
+    assert heads > 100 and plain_rows > 3
+
+
 def test_vector_items_dominate_on_aligned_workloads():
     p, items = run_and_compare(U.workload_desc("tiny"))
     data = items[items["kind"] <= U.ITEM_BF16_SCALAR]
