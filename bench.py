@@ -171,6 +171,28 @@ def visible_gpu_index(local_rank: int) -> int:
 # Peaks and profile summaries
 # ---------------------------------------------------------------------------
 
+def same_run_copy_gbs(stream, nbytes: int = 4 << 30, reps: int = 5) -> float:
+    """A plain device-to-device torch copy_ of nbytes (read + write counted), timed
+    with CUDA events in this run: the copy ceiling of this GPU right now."""
+    import torch
+    a = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    b = torch.empty_like(a)
+    a.fill_(1)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            b.copy_(a)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            b.copy_(a)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    del a, b
+    return 2 * nbytes / (ms * 1e-3) / 1e9
+
+
 def hbm_peak():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -422,6 +444,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         del host_src
 
     peak, peak_kind = hbm_peak()
+    copy_gbs = same_run_copy_gbs(stream)
     pack_gbs = pack_bytes / (pack_ms * 1e-3) / 1e9
     traffic = profiled_traffic(w.name) if bucket_bytes == w.bucket_bytes else None
     clocks = clk.summary()
@@ -453,7 +476,11 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         "roofline": {"bound": "hbm", "kernel": "rr_bulk_kernel (pack)", "achieved": round(pack_gbs, 1),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
                      "frac": round(pack_gbs / peak, 4), "traffic": traffic,
-                     "algorithmic_bytes": pack_bytes},
+                     "algorithmic_bytes": pack_bytes,
+                     "copy_same_run": {"GB/s": round(copy_gbs, 1),
+                                       "pack_frac": round(pack_gbs / copy_gbs, 4),
+                                       "method": "torch copy_ of 4 GiB on the device, "
+                                                 "read + write bytes"}},
         "clocks": clocks,
         "gpu_launches": 2 * args.steps,
         "e2e": e2e,

@@ -6,12 +6,20 @@
 // layer into a transfer buffer) and Section 5.2.2 (a rollout that resumes or
 // restarts a pull must know which parts of the buffer it holds intact).
 //
-// All three kernels are persistent: one launch of `grid_blocks` blocks walks
-// the whole work table, each block a contiguous, weight-balanced range of it.
-// The work is pure data movement bound by HBM bandwidth: 16-byte coalesced
-// loads and stores, several vectors in flight per thread, the cast done in
-// integer arithmetic in registers, the checksum accumulated per warp in
-// registers and flushed with one 64-bit atomic per warp per bucket change.
+// Two engines read the same work tables.  The bulk-copy engine
+// (rr_bulk_kernel, the default when every buffer is device memory) has one
+// producer warp per block stage source bytes into a shared-memory ring --
+// cp.async.bulk for long runs, the warp's 16-byte cp.async for short rows --
+// while consumer warps cast or copy from shared memory to the destination.
+// The register path (rr_pack_kernel, rr_unpack_kernel, rr_verify_kernel)
+// moves 16-byte vectors through registers; it serves host-resident buffers
+// and the standalone verify.
+//
+// Every kernel is persistent: one launch walks the whole work table, each
+// block a contiguous, weight-balanced range of it.  The work is pure data
+// movement bound by HBM bandwidth; the cast is integer arithmetic in
+// registers, and the checksum is accumulated per warp and flushed with one
+// 64-bit atomic per warp per bucket change.
 #include <cuda_runtime.h>
 
 #include <algorithm>

@@ -12,6 +12,11 @@
 // is sorted by (bucket, offset).  Items whose addresses and lengths allow it
 // are 16-byte vector items; the rest (ragged heads and tails, misaligned
 // sources, odd row lengths) are scalar items.
+//
+// A second, whole-sync table serves a full-range pack on the bulk-copy
+// engine: the same items, except that narrow column slices of the same
+// parameter rows for several ranks (row-parallel weights under tensor
+// parallelism) become fan-out groups that read each source row once.
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
