@@ -57,6 +57,8 @@ def parse():
     ap.add_argument("--snapshot", action="store_true",
                     help="also time rr_pack straight into pinned host buckets")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-next-rows", action="store_true",
+                    help="skip the resume (bucket-range) and relay re-pack timings")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-buckets", type=int, default=2,
                     help="buckets in the oracle's CPU sample")
@@ -295,6 +297,80 @@ def run_reference(args, w, bucket_bytes, world, rank):
 # GPU arm
 # ---------------------------------------------------------------------------
 
+def _event_ms(fn, stream, reps=3):
+    """Mean CUDA-event time of fn() over reps launches after one warm-up."""
+    import torch
+    fn()
+    torch.cuda.synchronize()
+    ms = []
+    for _ in range(reps):
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms.append(a.elapsed_time(b))
+    return statistics.mean(ms)
+
+
+def next_rows(rr, H, w, plan, buf, t_src, t_bkt, t_dst, stream, peak):
+    """Timings of the paths beyond the step: a resumed pull (the middle third of
+    the buckets packed and checked-unpacked again, Section 5.2.2) and a relay
+    re-pack (a rollout holding the TP=1 image serves a TP=4 one straight from
+    the buckets it pulled, Section 5.2.1).  Algorithmic bytes as for the step."""
+    import numpy as np
+    import torch
+    out = {}
+    n = plan.n_buckets // 3
+    b0 = n
+    if n:
+        items, _ = plan.export_pack()
+        sel = (items["bucket"] >= b0) & (items["bucket"] < b0 + n) & (items["kind"] <= 3)
+        es = np.where(items["kind"][sel] <= 1, 4, 2)
+        read = int((items["row_len"][sel].astype(np.int64) * items["n_rows"][sel] * es).sum())
+        wrote = n * plan.bucket_bytes
+        ms = _event_ms(lambda: rr.rr_pack_range(plan, b0, n, t_src, t_bkt, buf.checksums,
+                                                stream), stream)
+        gbs = (read + wrote) / (ms * 1e-3) / 1e9
+        out["resume_pack_range"] = {"buckets": [b0, b0 + n], "ms": round(ms, 3),
+                                    "bytes": read + wrote, "GB/s": round(gbs, 1),
+                                    "frac_of_peak": round(gbs / peak, 4)}
+        uitems, _ = plan.export_unpack()
+        usel = ((uitems["bucket"] >= b0) & (uitems["bucket"] < b0 + n)
+                & ((uitems["kind"] == 6) | (uitems["kind"] == 7)))
+        uwrote = int(uitems["nbytes"][usel].astype(np.int64).sum())
+
+        def uv():
+            n_bad, _ = rr.rr_unpack_verify(plan, t_bkt, buf.checksums, t_dst, stream=stream,
+                                           first_bucket=b0, n_buckets=n)
+            if n_bad:
+                raise RuntimeError("resumed range failed its checksums")
+        ms = _event_ms(uv, stream)
+        gbs = (wrote + uwrote) / (ms * 1e-3) / 1e9
+        out["resume_unpack_verify_range"] = {"buckets": [b0, b0 + n], "ms": round(ms, 3),
+                                             "bytes": wrote + uwrote, "GB/s": round(gbs, 1),
+                                             "frac_of_peak": round(gbs / peak, 4)}
+    if w.tp == 1 and plan.bucket_bytes % 16 == 0:
+        from paper_2512_22492_gb300 import layouts
+        m2, s2, d2 = layouts.qwen3_relay(w.shape, 1, 4, from_plan=plan)
+        relay = rr.rr_plan_create(m2, s2, d2, plan.bucket_bytes)
+        rst = relay.stats()
+        store = torch.empty((relay.n_buckets, plan.bucket_bytes), dtype=torch.uint8,
+                            device="cuda")
+        cs = torch.zeros(relay.n_buckets, dtype=torch.int64, device="cuda")
+        r_src = rr.Pointers(relay, "src_shards", buf.buckets)
+        ms = _event_ms(lambda: rr.rr_pack(relay, r_src, store, cs, stream), stream)
+        nbytes = rst["pack_bytes_read"] + rst["pack_bytes_written"]
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        out["relay_repack_tp1_to_tp4"] = {"source": "the TP=1 buckets as pulled",
+                                          "n_buckets": relay.n_buckets, "ms": round(ms, 3),
+                                          "bytes": nbytes, "GB/s": round(gbs, 1),
+                                          "frac_of_peak": round(gbs / peak, 4)}
+        del store, cs, r_src, relay
+    return out
+
+
 def run_native(args, w, bucket_bytes, world, rank, local):
     import torch
     import paper_2512_22492_gb300 as rr
@@ -444,6 +520,8 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         del host_src
 
     peak, peak_kind = hbm_peak()
+    more = None if args.no_next_rows else next_rows(rr, H, w, plan, buf, t_src, t_bkt, t_dst,
+                                                    stream, peak)
     copy_gbs = same_run_copy_gbs(stream)
     pack_gbs = pack_bytes / (pack_ms * 1e-3) / 1e9
     traffic = profiled_traffic(w.name) if bucket_bytes == w.bucket_bytes else None
@@ -487,6 +565,8 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     }
     if snapshot:
         line["snapshot"] = snapshot
+    if more:
+        line["next_rows"] = more
     del buf
     torch.cuda.empty_cache()
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
