@@ -62,8 +62,9 @@ template <int NPTR>
 struct PackArgs {
     const rr_pack_item* items;
     const uint32_t* block_first;   // balanced per-block ranges, or NULL: split
-    uint32_t item_begin;           //   [item_begin, item_end) evenly over the grid
-    uint32_t item_end;
+    uint32_t item_begin;           //   [item_begin, item_end) over the grid by
+    uint32_t item_end;             //   the items' weights (weight_prefix)
+    const unsigned long long* weight_prefix;
     unsigned long long* checksums;
     char* bucket_base;        // equally spaced buckets: base + b * stride
     uint64_t bucket_stride;   // 0: bucket b is ptr[n_shards + b]
@@ -78,6 +79,7 @@ struct UnpackArgs {
     const uint32_t* block_first;   // as in PackArgs
     uint32_t item_begin;
     uint32_t item_end;
+    const unsigned long long* weight_prefix;
     // Verifying unpack only (as in VerifyArgs): per-bucket sums of the range
     // [first_bucket, first_bucket + n_buckets), counters, expected sums, flags.
     unsigned long long* sums;
@@ -181,11 +183,34 @@ __device__ __forceinline__ void flush(unsigned long long* dst, unsigned long lon
 
 // This block's item range: the plan's balanced split for a full call, an even
 // split of [begin, end) for a bucket-range call.
-__device__ __forceinline__ void block_items(const uint32_t* block_first, uint32_t begin,
+// First item i in [lo, hi] with prefix[i] >= w (prefix is non-decreasing).
+__device__ __forceinline__ uint32_t lower_item(const unsigned long long* prefix, uint32_t lo,
+                                               uint32_t hi, unsigned long long w) {
+    while (lo < hi) {
+        const uint32_t mid = lo + (hi - lo) / 2;
+        if (prefix[mid] < w)
+            lo = mid + 1;
+        else
+            hi = mid;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ void block_items(const uint32_t* block_first,
+                                            const unsigned long long* prefix, uint32_t begin,
                                             uint32_t end, uint32_t* i0, uint32_t* i1) {
     if (block_first) {
         *i0 = block_first[blockIdx.x];
         *i1 = block_first[blockIdx.x + 1];
+    } else if (prefix) {
+        // Split points at equal shares of the range's weight; neighbouring blocks
+        // compute the same point, so the ranges tile [begin, end).
+        const unsigned long long w0 = prefix[begin], w = prefix[end] - w0;
+        *i0 = blockIdx.x == 0 ? begin
+                              : lower_item(prefix, begin, end, w0 + w * blockIdx.x / gridDim.x);
+        *i1 = blockIdx.x + 1 == gridDim.x
+                  ? end
+                  : lower_item(prefix, begin, end, w0 + w * (blockIdx.x + 1) / gridDim.x);
     } else {
         const uint64_t n = end - begin;
         *i0 = begin + (uint32_t)(n * blockIdx.x / gridDim.x);
@@ -294,7 +319,7 @@ __device__ __forceinline__ unsigned long long pack_scalar(const char* src, char*
 template <int NPTR>
 __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(const __grid_constant__ PackArgs<NPTR> a) {
     uint32_t i0, i1;
-    block_items(a.block_first, a.item_begin, a.item_end, &i0, &i1);
+    block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
     unsigned long long acc = 0;
     uint32_t cur = 0xFFFFFFFFu;
     for (uint32_t it = i0; it < i1; ++it) {
@@ -364,7 +389,7 @@ template <int NPTR, bool VERIFY>
 __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
     constexpr int U = 2 * kUnroll;   // one 16-byte load per vector: twice the pack's depth
     uint32_t i0, i1;
-    block_items(a.block_first, a.item_begin, a.item_end, &i0, &i1);
+    block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
     unsigned long long acc = 0;
     uint32_t cur = 0xFFFFFFFFu;
     for (uint32_t it = i0; it < i1; ++it) {
@@ -531,6 +556,7 @@ struct BulkArgs {
     const uint32_t* block_first; // as in PackArgs
     uint32_t item_begin;
     uint32_t item_end;
+    const unsigned long long* weight_prefix;
     char* bucket_base;
     uint64_t bucket_stride;
     int32_t n_shards;            // pack: ptr[0 .. n_shards) are the shards
@@ -640,7 +666,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
     __syncthreads();
 
     uint32_t i0, i1;
-    block_items(a.block_first, a.item_begin, a.item_end, &i0, &i1);
+    block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
@@ -1059,6 +1085,7 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
     std::memset(&a, 0, sizeof a);
     a.items = P->d_pack_items;
     a.block_first = R.full ? P->d_pack_block_first : nullptr;
+    a.weight_prefix = P->d_pack_weight_prefix;
     a.item_begin = P->pack_bucket_first[R.b0];
     a.item_end = P->pack_bucket_first[R.b1];
     a.checksums = (unsigned long long*)checksums;
@@ -1084,6 +1111,7 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     std::memset(&a, 0, sizeof a);
     a.items = P->d_unpack_items;
     a.block_first = R.full ? P->d_unpack_block_first : nullptr;
+    a.weight_prefix = P->d_unpack_weight_prefix;
     a.item_begin = P->unpack_bucket_first[R.b0];
     a.item_end = P->unpack_bucket_first[R.b1];
     if (checksums) {
@@ -1167,6 +1195,7 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
     if (MODE == 0) {
         a.items = P->d_pack_items;
         a.block_first = R.full ? P->d_pack_block_first : nullptr;
+        a.weight_prefix = P->d_pack_weight_prefix;
         a.item_begin = P->pack_bucket_first[R.b0];
         a.item_end = P->pack_bucket_first[R.b1];
         if (R.full && P->d_full_items) {   // every bucket: the table with fan-out groups
@@ -1181,6 +1210,7 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
     } else {
         a.items = P->d_unpack_items;
         a.block_first = R.full ? P->d_unpack_block_first : nullptr;
+        a.weight_prefix = P->d_unpack_weight_prefix;
         a.item_begin = P->unpack_bucket_first[R.b0];
         a.item_end = P->unpack_bucket_first[R.b1];
         if (MODE == 2) {
@@ -1433,6 +1463,10 @@ rr_status rr_device_upload(rr_plan* P) {
                            cudaHostAllocDefault)) != cudaSuccess ||
         (e = cudaMalloc((void**)&P->d_error, sizeof(unsigned int))) != cudaSuccess ||
         (e = cudaMemset(P->d_error, 0, sizeof(unsigned int))) != cudaSuccess ||
+        (e = up((void**)&P->d_pack_weight_prefix, P->pack_weight_prefix.data(),
+                P->pack_weight_prefix.size() * sizeof(unsigned long long))) != cudaSuccess ||
+        (e = up((void**)&P->d_unpack_weight_prefix, P->unpack_weight_prefix.data(),
+                P->unpack_weight_prefix.size() * sizeof(unsigned long long))) != cudaSuccess ||
         (!P->full_items.empty() &&
          ((e = up((void**)&P->d_full_items, P->full_items.data(),
                   P->full_items.size() * sizeof(rr_pack_item))) != cudaSuccess ||
@@ -1452,6 +1486,8 @@ void rr_device_release(rr_plan* P) {
     cudaFree(P->d_pack_block_first);
     cudaFree(P->d_full_items);
     cudaFree(P->d_full_block_first);
+    cudaFree(P->d_pack_weight_prefix);
+    cudaFree(P->d_unpack_weight_prefix);
     cudaFree(P->d_unpack_items);
     cudaFree(P->d_unpack_block_first);
     cudaFree(P->d_verify_scratch);
@@ -1462,6 +1498,8 @@ void rr_device_release(rr_plan* P) {
     P->d_pack_block_first = nullptr;
     P->d_full_items = nullptr;
     P->d_full_block_first = nullptr;
+    P->d_pack_weight_prefix = nullptr;
+    P->d_unpack_weight_prefix = nullptr;
     P->d_unpack_items = nullptr;
     P->d_unpack_block_first = nullptr;
     P->d_verify_scratch = nullptr;

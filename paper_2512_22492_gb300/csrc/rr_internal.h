@@ -50,6 +50,8 @@ struct rr_plan {
     std::vector<rr_unpack_item> unpack_items;
     std::vector<uint32_t> unpack_block_first;   // grid_blocks + 1
     std::vector<uint32_t> pack_bucket_first;    // n_buckets + 1: first pack item of bucket b
+    std::vector<unsigned long long> pack_weight_prefix;    // items + 1: balancing weights,
+    std::vector<unsigned long long> unpack_weight_prefix;  // summed (bucket-range calls)
     std::vector<rr_pack_item> full_items;       // whole-sync table with fan-out groups;
                                                 // empty when it would equal pack_items
     std::vector<uint32_t> full_block_first;     // grid_blocks + 1
@@ -62,6 +64,8 @@ struct rr_plan {
     uint32_t* d_pack_block_first = nullptr;
     rr_pack_item* d_full_items = nullptr;
     uint32_t* d_full_block_first = nullptr;
+    unsigned long long* d_pack_weight_prefix = nullptr;
+    unsigned long long* d_unpack_weight_prefix = nullptr;
     rr_unpack_item* d_unpack_items = nullptr;
     uint32_t* d_unpack_block_first = nullptr;
     unsigned long long* d_verify_scratch = nullptr;  // n_buckets sums + 4 counters

@@ -672,6 +672,13 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     index(P->unpack_items, P->unpack_bucket_first);
     partition(P->pack_items, P->grid_blocks, P->pack_block_first, pack_weight);
     partition(P->unpack_items, P->unpack_grid_blocks, P->unpack_block_first, unpack_weight);
+    // Summed weights: a bucket-range call splits its items over the grid by them.
+    auto prefix = [](const auto& items, std::vector<unsigned long long>& out, auto w) {
+        out.assign(items.size() + 1, 0ull);
+        for (size_t i = 0; i < items.size(); ++i) out[i + 1] = out[i] + uint64_t(w(items[i]));
+    };
+    prefix(P->pack_items, P->pack_weight_prefix, pack_weight);
+    prefix(P->unpack_items, P->unpack_weight_prefix, unpack_weight);
 
     // Whole-sync table: the grouped blocks' plain items give way to fan-out groups.
     P->full_items.clear();
