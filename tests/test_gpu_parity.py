@@ -2,11 +2,14 @@
 
 Buckets, checksums and unpacked tensors are integer / bit-pattern data, so the
 bar is exact equality (RobustRL Section 5.2.1 steps 1-2; Section 5.2.2 for
-the checksums).  Small workloads are compared in full; the full-size
-workloads (Qwen3-8B, its TP=4 bucket sweep, Qwen3-30B-A3B) on sampled
-buckets and tensors that the oracle computes one by one, plus properties that
-hold at any size (every checksum equals a word sum taken by torch; verify
-finds nothing; unpack(pack) equals the sampled tensors).
+the checksums).  Small workloads are compared in full.  The full-size
+workloads (Qwen3-8B, Qwen3-8B TP=4, Qwen3-30B-A3B) are compared on every
+bucket and checksum, the oracle running on all host cores -- at every size of
+the TP=4 bucket sweep, and for the further full-size layouts (FSDP2 -> TP=8,
+per-layer FSDP1 units, expert parallel) too.  Sampled tensors are compared
+with the oracle one by one, plus properties that hold at any size (every
+checksum equals a word sum taken by torch; verify finds nothing; every tensor
+equals its own bytes in the buckets).
 """
 import numpy as np
 import pytest
@@ -229,6 +232,49 @@ def _unpack_sampled(name, names):
         assert torch.equal(buf.dst[t][:plan.tensor_numel[t]], want), plan.tensor_names[t]
 
 
+def every_bucket_parity(name, bucket_bytes=None):
+    """Every bucket and every checksum of a full-size workload against the oracle,
+    in the launch configuration the benchmark times.  The oracle packs the
+    buckets one by one in a pool of host threads (its C calls run without the
+    interpreter lock, and it keeps no shared state); nothing is sampled."""
+    import os
+    from concurrent.futures import ThreadPoolExecutor
+    w = U.workload(name)
+    desc = U.workload_desc(name)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, bucket_bytes or w.bucket_bytes)
+    buf = H.alloc(plan, poison=0xAB, with_dst=False)
+    H.fill_with_generator(buf, m, w.seed, w.specials)
+    H.pack(buf)
+    torch.cuda.synchronize()
+    got = buf.bucket_store[:, :plan.bucket_bytes].cpu().numpy()
+    cs = H.checksums_host(buf)
+    buf = None
+    torch.cuda.empty_cache()
+    L = oracle.workload_layout(w, bucket_bytes=plan.bucket_bytes)
+    gen = oracle.Source(seed=w.seed, specials=w.specials)
+
+    def one(b):
+        want, want_cs = L.pack(gen, first=b, count=1)
+        return b if not (np.array_equal(got[b], want[0]) and cs[b] == want_cs[0]) else -1
+
+    with ThreadPoolExecutor(max_workers=os.cpu_count() or 4) as ex:
+        bad = [b for b in ex.map(one, range(plan.n_buckets)) if b >= 0]
+    assert bad == [], f"{name}: buckets differing from the oracle: {bad[:10]}"
+
+
+@pytest.mark.parametrize("name", ["qwen3-8b", "qwen3-8b-tp4", "qwen3-30b-a3b",
+                                  "qwen3-8b-fsdp2-tp8", "qwen3-30b-a3b-fsdp2-tp8",
+                                  "qwen3-8b-units", "qwen3-30b-a3b-fsdp2-ep8"])
+def test_every_bucket_full_size(name):
+    every_bucket_parity(name)
+
+
+@pytest.mark.parametrize("mib", [s >> 20 for s in synth.TP4_BUCKET_SWEEP])
+def test_every_bucket_tp4_sweep(mib):
+    every_bucket_parity("qwen3-8b-tp4", bucket_bytes=mib << 20)
+
+
 def test_qwen3_8b_sampled():
     sampled_parity("qwen3-8b", n_random_buckets=4)
     torch.cuda.empty_cache()
@@ -238,8 +284,8 @@ def test_qwen3_8b_sampled():
     torch.cuda.empty_cache()
 
 
-def test_qwen3_8b_tp4_bucket_sweep_sampled():
-    sampled_parity("qwen3-8b-tp4", bucket_sizes=synth.TP4_BUCKET_SWEEP, n_random_buckets=1)
+def test_qwen3_8b_tp4_sampled():
+    sampled_parity("qwen3-8b-tp4", n_random_buckets=1)
     torch.cuda.empty_cache()
     _unpack_sampled("qwen3-8b-tp4", [("layers.3.qkv_proj", 1), ("layers.20.o_proj", 2),
                                      ("layers.35.down_proj", 3), ("layers.7.gate_up_proj", 0),
