@@ -254,6 +254,24 @@ def oracle_time(L, src, first, count):
     return moved, time.perf_counter() - t0
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (Linux), or the architecture."""
+    import platform
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                key = line.split(":")[0].strip().lower()
+                if key in ("model name", "cpu model", "hardware"):
+                    return line.split(":", 1)[1].strip()
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return platform.machine()
+
+
 def cpu_baseline(w, bucket_bytes, n_buckets_sample):
     L, src, _keep = oracle_sample_setup(w, bucket_bytes)
     moved, dt = oracle_time(L, src, 0, n_buckets_sample)
@@ -261,7 +279,7 @@ def cpu_baseline(w, bucket_bytes, n_buckets_sample):
             "sample": f"buckets 0..{n_buckets_sample - 1} of {L.n_buckets} "
                       f"({n_buckets_sample} x {bucket_bytes >> 20} MiB): pack, unpack of their "
                       f"elements, verify; single-threaded C oracle; {moved / 1e9:.3f} GB in "
-                      f"{dt:.2f} s; host cores available {os.cpu_count()}"}
+                      f"{dt:.2f} s; 1 of {os.cpu_count()} host cores ({cpu_model()})"}
 
 
 def run_reference(args, w, bucket_bytes, world, rank):
