@@ -54,6 +54,9 @@ def parse():
                     help="with --layers: a smaller vocabulary as well")
     ap.add_argument("--chunk-kib", type=int, default=0, help="plan option: KiB per work item")
     ap.add_argument("--grid", type=int, default=0, help="plan option: persistent grid size")
+    ap.add_argument("--engine", choices=["auto", "registers"], default="auto",
+                    help="plan option: the bulk-copy engine for device buffers (auto) or the "
+                         "register path for every call")
     ap.add_argument("--snapshot", action="store_true",
                     help="also time rr_pack straight into pinned host buckets")
     ap.add_argument("--no-e2e", action="store_true")
@@ -398,8 +401,9 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     stream = torch.cuda.current_stream()
     m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
     opts = None
-    if args.chunk_kib or args.grid:
-        opts = rr.PlanOptions(chunk_bytes=args.chunk_kib * 1024, grid_blocks=args.grid)
+    if args.chunk_kib or args.grid or args.engine != "auto":
+        opts = rr.PlanOptions(chunk_bytes=args.chunk_kib * 1024, grid_blocks=args.grid,
+                              engine=args.engine)
     plan = rr.rr_plan_create(m, s, d, bucket_bytes, opts)
     st = plan.stats()
     buf = H.alloc(plan, poison=None)
@@ -542,7 +546,8 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                                                     stream, peak)
     copy_gbs = same_run_copy_gbs(stream)
     pack_gbs = pack_bytes / (pack_ms * 1e-3) / 1e9
-    traffic = profiled_traffic(w.name) if bucket_bytes == w.bucket_bytes else None
+    traffic = (profiled_traffic(w.name) if bucket_bytes == w.bucket_bytes and args.engine == "auto"
+               else None)
     clocks = clk.summary()
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
@@ -553,6 +558,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                    "sharding": w.sharding, "expert_parallel": w.ep,
                    "tp": w.tp, "bucket_bytes": bucket_bytes, "n_buckets": plan.n_buckets,
                    "step": "rr_pack + rr_unpack_verify (unpack and checksum check fused)",
+                   "engine": args.engine,
                    "step_bytes": step_bytes, "l2": "inputs > L2 (no flush needed)",
                    "parallelism": f"replicas{world}"},
         "ms_per_full_model_sync": round(pack_ms + uv_ms, 3),
@@ -569,7 +575,9 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                        "GB/s": round(verify_bytes / (verify_ms * 1e-3) / 1e9, 1),
                        "frac_of_peak": round(verify_bytes / (verify_ms * 1e-3) / 1e9 / peak, 4)},
         },
-        "roofline": {"bound": "hbm", "kernel": "rr_bulk_kernel (pack)", "achieved": round(pack_gbs, 1),
+        "roofline": {"bound": "hbm",
+                     "kernel": "rr_bulk_kernel (pack)" if args.engine == "auto" else "rr_pack_kernel",
+                     "achieved": round(pack_gbs, 1),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
                      "frac": round(pack_gbs / peak, 4), "traffic": traffic,
                      "algorithmic_bytes": pack_bytes,
