@@ -54,6 +54,8 @@ def parse():
                     help="with --layers: a smaller vocabulary as well")
     ap.add_argument("--chunk-kib", type=int, default=0, help="plan option: KiB per work item")
     ap.add_argument("--grid", type=int, default=0, help="plan option: persistent grid size")
+    ap.add_argument("--check-items", action="store_true",
+                    help="plan option: kernels check every work item's bounds")
     ap.add_argument("--engine", choices=["auto", "registers"], default="auto",
                     help="plan option: the bulk-copy engine for device buffers (auto) or the "
                          "register path for every call")
@@ -401,9 +403,9 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     stream = torch.cuda.current_stream()
     m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
     opts = None
-    if args.chunk_kib or args.grid or args.engine != "auto":
+    if args.chunk_kib or args.grid or args.engine != "auto" or args.check_items:
         opts = rr.PlanOptions(chunk_bytes=args.chunk_kib * 1024, grid_blocks=args.grid,
-                              engine=args.engine)
+                              engine=args.engine, check_items=args.check_items)
     plan = rr.rr_plan_create(m, s, d, bucket_bytes, opts)
     st = plan.stats()
     buf = H.alloc(plan, poison=None)
@@ -558,7 +560,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                    "sharding": w.sharding, "expert_parallel": w.ep,
                    "tp": w.tp, "bucket_bytes": bucket_bytes, "n_buckets": plan.n_buckets,
                    "step": "rr_pack + rr_unpack_verify (unpack and checksum check fused)",
-                   "engine": args.engine,
+                   "engine": args.engine, "check_items": args.check_items,
                    "step_bytes": step_bytes, "l2": "inputs > L2 (no flush needed)",
                    "parallelism": f"replicas{world}"},
         "ms_per_full_model_sync": round(pack_ms + uv_ms, 3),

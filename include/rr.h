@@ -176,6 +176,12 @@ typedef struct {
     int32_t grid_blocks; /* persistent grid size; default: SMs x resident blocks      */
     int64_t chunk_bytes; /* largest destination bytes per work item; default 32 KiB   */
     int32_t engine;      /* rr_engine                                                 */
+    int32_t check_items; /* 1: every kernel checks each work item against the source,
+                            bucket and tensor sizes of the plan before touching
+                            memory; an item outside them is skipped and marks the
+                            plan's error word (rr_plan_check then reports RR_ECUDA).
+                            A debugging aid in place of a memory checker; costs a
+                            little producer time                                    */
 } rr_plan_options;
 
 /* Compiles manifest + source layout + destination layout + bucket size into

@@ -52,6 +52,20 @@ constexpr int kUnroll = RR_UNROLL;     // 16-byte vectors in flight per thread
 constexpr int kSmallPtrs = 64;      // pointer-table sizes of the two launch shapes
 constexpr int kLargePtrs = 3968;    // keeps the kernel parameters under 32 KB
 constexpr int64_t kVerifyChunk = 64 * 1024;
+constexpr unsigned int kErrWaitTimeout = 1;       // plan error word: a bounded wait ran out
+constexpr unsigned int kErrBadItem = 2;           // a work item outside its buffers, refused
+
+// Sizes a kernel checks each work item against when the plan asks for it
+// (src_bytes == NULL: no checks).  An item outside them is skipped and marks
+// the plan's error word.
+struct ItemBounds {
+    const int64_t* src_bytes;     // bytes of each source buffer (pack)
+    const int64_t* tensor_bytes;  // bytes of each destination tensor (unpack)
+    int64_t bucket_bytes;
+    int32_t n_src, n_buckets;
+    int32_t n_tensors, pad;
+    unsigned int* err;
+};
 
 // ---------------------------------------------------------------------------
 // Launch arguments (passed by value in the kernel parameter space, so that a
@@ -65,6 +79,7 @@ struct PackArgs {
     uint32_t item_begin;           //   [item_begin, item_end) over the grid by
     uint32_t item_end;             //   the items' weights (weight_prefix)
     const unsigned long long* weight_prefix;
+    ItemBounds chk;
     unsigned long long* checksums;
     char* bucket_base;        // equally spaced buckets: base + b * stride
     uint64_t bucket_stride;   // 0: bucket b is ptr[n_shards + b]
@@ -80,6 +95,7 @@ struct UnpackArgs {
     uint32_t item_begin;
     uint32_t item_end;
     const unsigned long long* weight_prefix;
+    ItemBounds chk;
     // Verifying unpack only (as in VerifyArgs): per-bucket sums of the range
     // [first_bucket, first_bucket + n_buckets), counters, expected sums, flags.
     unsigned long long* sums;
@@ -179,6 +195,57 @@ __device__ __forceinline__ unsigned long long warp_sum(unsigned long long v) {
 __device__ __forceinline__ void flush(unsigned long long* dst, unsigned long long acc) {
     acc = warp_sum(acc);
     if ((threadIdx.x & 31) == 0 && acc != 0ull) atomicAdd(dst, acc);
+}
+
+// The source extent of a data item: the bytes from its first source element to
+// the end of its last row.
+__device__ __forceinline__ uint64_t src_extent(uint32_t rows, uint32_t row_len, uint32_t stride,
+                                               uint32_t es) {
+    return rows ? ((uint64_t)(rows - 1) * stride + row_len) * es : 0;
+}
+
+// Whether a pack item (or fan-out destination) lies inside the plan's buffers.
+__device__ __forceinline__ bool pack_item_in(const ItemBounds& b, const rr_pack_item& d) {
+    if (!b.src_bytes) return true;
+    const uint64_t n = (uint64_t)d.row_len * d.n_rows;
+    bool ok = d.bucket < (uint32_t)b.n_buckets;
+    if (d.kind <= RR_ITEM_BF16_SCALAR || d.kind == RR_ITEM_FAN_F32 || d.kind == RR_ITEM_FAN_BF16) {
+        const uint32_t es =
+            (d.kind <= RR_ITEM_F32_SCALAR || d.kind == RR_ITEM_FAN_F32) ? 4u : 2u;
+        const uint32_t sh = (uint32_t)(d.src >> 48);
+        const uint64_t off = d.src & 0xFFFFFFFFFFFFull;
+        ok = ok && sh < (uint32_t)b.n_src &&
+             off + src_extent(d.n_rows, d.row_len, d.src_stride, es) <= (uint64_t)b.src_bytes[sh];
+        if (d.kind <= RR_ITEM_BF16_SCALAR) ok = ok && d.dst_off + 2 * n <= (uint64_t)b.bucket_bytes;
+    } else if (d.kind == RR_ITEM_ZERO_VEC || d.kind == RR_ITEM_ZERO_SCALAR ||
+               d.kind == RR_ITEM_FAN_DST) {
+        ok = ok && d.dst_off + 2 * n <= (uint64_t)b.bucket_bytes;
+    } else {
+        ok = false;
+    }
+    return ok;
+}
+
+// As pack_item_in, called uniformly by a warp or block; its first thread marks
+// a refusal in the plan's error word.
+__device__ __forceinline__ bool pack_item_ok(const ItemBounds& b, const rr_pack_item& d) {
+    const bool ok = pack_item_in(b, d);
+    if (!ok && threadIdx.x % 32 == 0) atomicExch(b.err, kErrBadItem);
+    return ok;
+}
+
+// Whether an unpack item lies inside its bucket and (a copy) its tensor.
+__device__ __forceinline__ bool unpack_item_ok(const ItemBounds& b, const rr_unpack_item& d) {
+    if (!b.src_bytes) return true;
+    bool ok = d.bucket < (uint32_t)b.n_buckets &&
+              (uint64_t)d.src_off + d.nbytes <= (uint64_t)b.bucket_bytes;
+    if (d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_COPY_SCALAR)
+        ok = ok && d.tensor < (uint32_t)b.n_tensors &&
+             d.dst_off + d.nbytes <= (uint64_t)b.tensor_bytes[d.tensor];
+    else
+        ok = ok && (d.kind == RR_ITEM_READ_VEC || d.kind == RR_ITEM_READ_SCALAR);
+    if (!ok && threadIdx.x % 32 == 0) atomicExch(b.err, kErrBadItem);
+    return ok;
 }
 
 // This block's item range: the plan's balanced split for a full call, an even
@@ -324,6 +391,7 @@ __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(c
     uint32_t cur = 0xFFFFFFFFu;
     for (uint32_t it = i0; it < i1; ++it) {
         const rr_pack_item d = a.items[it];
+        if (!pack_item_ok(a.chk, d)) continue;
         if (d.bucket != cur) {
             if (cur != 0xFFFFFFFFu) flush(a.checksums + cur, acc);
             cur = d.bucket;
@@ -395,6 +463,7 @@ __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_con
     for (uint32_t it = i0; it < i1; ++it) {
         const rr_unpack_item d = a.items[it];
         if (!VERIFY && d.kind >= RR_ITEM_READ_VEC) continue;
+        if (!unpack_item_ok(a.chk, d)) continue;
         if (VERIFY && d.bucket != cur) {
             if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - a.first_bucket), acc);
             cur = d.bucket;
@@ -519,8 +588,6 @@ struct BulkShape {
 constexpr uint32_t kWaitLimit = 1u << 20;        // tries, each suspending at most kWaitHintNs
 constexpr uint32_t kWaitHintNs = 1000;
 constexpr uint64_t kWaitDeadlineNs = 1000000000;  // and at most one second of wall clock
-constexpr unsigned int kErrWaitTimeout = 1;
-constexpr unsigned int kErrBadItem = 2;           // an item the engine cannot stage
 
 enum : uint16_t {
     PC_CAST = 1,      // stage holds fp32 rows -> bf16 destination
@@ -557,6 +624,7 @@ struct BulkArgs {
     uint32_t item_begin;
     uint32_t item_end;
     const unsigned long long* weight_prefix;
+    ItemBounds chk;
     char* bucket_base;
     uint64_t bucket_stride;
     int32_t n_shards;            // pack: ptr[0 .. n_shards) are the shards
@@ -730,6 +798,11 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
             p.src_stride = 0;
             if (MODE == 0) {
                 const rr_pack_item d = ((const rr_pack_item*)a.items)[it];
+                if (!pack_item_ok(a.chk, d)) {
+                    if (d.kind == RR_ITEM_FAN_F32 || d.kind == RR_ITEM_FAN_BF16)
+                        it += min(d.dst_off, i1 - 1 - it);   // and its destinations
+                    continue;
+                }
                 char* dst = bulk_bucket(a, d.bucket, a.n_shards) + d.dst_off;
                 const char* src = (const char*)a.ptr[d.src >> 48] + (d.src & 0xFFFFFFFFFFFFull);
                 p.sum_bucket = d.bucket;
@@ -782,7 +855,8 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                         const rr_pack_item f = ((const rr_pack_item*)a.items)[it + 1 + lane];
                         bad = f.kind != RR_ITEM_FAN_DST || f.row_len % 8 != 0 ||
                               f.dst_off % 16 != 0 || (f.src * es) % 16 != 0 ||
-                              f.src + f.row_len > d.row_len;
+                              f.src + f.row_len > d.row_len || f.n_rows != R ||
+                              !pack_item_in(a.chk, f);
                     }
                     if (__any_sync(0xFFFFFFFFu, bad)) {
                         if (lane == 0) atomicExch(a.err, kErrBadItem);
@@ -830,6 +904,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                 const rr_unpack_item d = ((const rr_unpack_item*)a.items)[it];
                 const bool read_only = d.kind == RR_ITEM_READ_VEC || d.kind == RR_ITEM_READ_SCALAR;
                 if (MODE == 1 && read_only) continue;
+                if (!unpack_item_ok(a.chk, d)) continue;
                 const char* src = bulk_bucket(a, d.bucket, 0) + d.src_off;
                 char* dst = read_only ? nullptr : (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off;
                 p.sum_bucket = d.bucket;
@@ -1078,6 +1153,21 @@ struct Range {
     bool full;
 };
 
+// The bounds the kernels check items against, when the plan asks for checks.
+ItemBounds bounds_of(const rr_plan* P) {
+    ItemBounds b;
+    std::memset(&b, 0, sizeof b);
+    if (!P->check_items) return b;
+    b.src_bytes = P->d_src_bytes;
+    b.tensor_bytes = P->d_tensor_bytes;
+    b.bucket_bytes = P->bucket_bytes;
+    b.n_src = P->n_shards;
+    b.n_buckets = P->n_buckets;
+    b.n_tensors = P->n_tensors;
+    b.err = P->d_error;
+    return b;
+}
+
 template <int NPTR>
 rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* const* buckets,
                       uint64_t* checksums, bool table, uint64_t stride, cudaStream_t s) {
@@ -1086,6 +1176,7 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
     a.items = P->d_pack_items;
     a.block_first = R.full ? P->d_pack_block_first : nullptr;
     a.weight_prefix = P->d_pack_weight_prefix;
+    a.chk = bounds_of(P);
     a.item_begin = P->pack_bucket_first[R.b0];
     a.item_end = P->pack_bucket_first[R.b1];
     a.checksums = (unsigned long long*)checksums;
@@ -1112,6 +1203,7 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     a.items = P->d_unpack_items;
     a.block_first = R.full ? P->d_unpack_block_first : nullptr;
     a.weight_prefix = P->d_unpack_weight_prefix;
+    a.chk = bounds_of(P);
     a.item_begin = P->unpack_bucket_first[R.b0];
     a.item_end = P->unpack_bucket_first[R.b1];
     if (checksums) {
@@ -1191,6 +1283,7 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
     BulkArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     a.err = P->d_error;
+    a.chk = bounds_of(P);
     int32_t k = 0;
     if (MODE == 0) {
         a.items = P->d_pack_items;
@@ -1249,6 +1342,9 @@ rr_status read_error(const rr_plan* P, cudaStream_t stream) {
         const unsigned int code = *h;
         RR_CUDA(cudaMemsetAsync(P->d_error, 0, sizeof(unsigned int), stream));
         RR_CUDA(cudaStreamSynchronize(stream));
+        if (code == kErrBadItem)
+            return rr_fail(RR_ECUDA, "a kernel of this plan refused a work item outside the "
+                                     "plan's buffers; its output is incomplete");
         return rr_fail(RR_ECUDA, "a kernel of this plan gave up waiting (code %u); its output "
                                  "is incomplete", code);
     }
@@ -1448,6 +1544,9 @@ rr_status rr_device_upload(rr_plan* P) {
         if (e != cudaSuccess) return e;
         return bytes ? cudaMemcpy(*d, h, bytes, cudaMemcpyHostToDevice) : cudaSuccess;
     };
+    std::vector<int64_t> src_bytes(size_t(P->n_shards) + 1, 0), tensor_bytes;
+    rr_plan_source_buffers(P, nullptr, src_bytes.data());
+    for (int32_t i = 0; i < P->n_tensors; ++i) tensor_bytes.push_back(2 * P->tensor_numel[i]);
     cudaError_t e;
     if ((e = up((void**)&P->d_pack_items, P->pack_items.data(),
                 P->pack_items.size() * sizeof(rr_pack_item))) != cudaSuccess ||
@@ -1467,6 +1566,10 @@ rr_status rr_device_upload(rr_plan* P) {
                 P->pack_weight_prefix.size() * sizeof(unsigned long long))) != cudaSuccess ||
         (e = up((void**)&P->d_unpack_weight_prefix, P->unpack_weight_prefix.data(),
                 P->unpack_weight_prefix.size() * sizeof(unsigned long long))) != cudaSuccess ||
+        (P->check_items &&
+         ((e = up((void**)&P->d_src_bytes, src_bytes.data(), src_bytes.size() * 8)) != cudaSuccess ||
+          (e = up((void**)&P->d_tensor_bytes, tensor_bytes.data(), tensor_bytes.size() * 8)) !=
+              cudaSuccess)) ||
         (!P->full_items.empty() &&
          ((e = up((void**)&P->d_full_items, P->full_items.data(),
                   P->full_items.size() * sizeof(rr_pack_item))) != cudaSuccess ||
@@ -1488,6 +1591,8 @@ void rr_device_release(rr_plan* P) {
     cudaFree(P->d_full_block_first);
     cudaFree(P->d_pack_weight_prefix);
     cudaFree(P->d_unpack_weight_prefix);
+    cudaFree(P->d_src_bytes);
+    cudaFree(P->d_tensor_bytes);
     cudaFree(P->d_unpack_items);
     cudaFree(P->d_unpack_block_first);
     cudaFree(P->d_verify_scratch);
@@ -1500,6 +1605,8 @@ void rr_device_release(rr_plan* P) {
     P->d_full_block_first = nullptr;
     P->d_pack_weight_prefix = nullptr;
     P->d_unpack_weight_prefix = nullptr;
+    P->d_src_bytes = nullptr;
+    P->d_tensor_bytes = nullptr;
     P->d_unpack_items = nullptr;
     P->d_unpack_block_first = nullptr;
     P->d_verify_scratch = nullptr;

@@ -66,6 +66,9 @@ struct rr_plan {
     uint32_t* d_full_block_first = nullptr;
     unsigned long long* d_pack_weight_prefix = nullptr;
     unsigned long long* d_unpack_weight_prefix = nullptr;
+    int32_t check_items = 0;                 // kernels check every item's bounds
+    int64_t* d_src_bytes = nullptr;          // check_items: bytes of each source buffer
+    int64_t* d_tensor_bytes = nullptr;       //              and of each destination tensor
     rr_unpack_item* d_unpack_items = nullptr;
     uint32_t* d_unpack_block_first = nullptr;
     unsigned long long* d_verify_scratch = nullptr;  // n_buckets sums + 4 counters

@@ -774,6 +774,7 @@ rr_status rr_plan_create_ex(const rr_param* manifest, int32_t n_params,
                 st = rr_fail(RR_EINVAL, "chunk_bytes must be a multiple of 16 in [16, 2^30]");
         }
         if (st == RR_OK) {
+            P->check_items = opts && opts->check_items ? 1 : 0;
             P->engine = opts ? opts->engine : RR_ENGINE_AUTO;
             if (P->engine != RR_ENGINE_AUTO && P->engine != RR_ENGINE_REGISTERS)
                 st = rr_fail(RR_EINVAL, "unknown engine %d", P->engine);

@@ -63,7 +63,8 @@ class _DstLayout(ctypes.Structure):
 
 class _Options(ctypes.Structure):
     _fields_ = [("host_only", ctypes.c_int32), ("grid_blocks", ctypes.c_int32),
-                ("chunk_bytes", ctypes.c_int64), ("engine", ctypes.c_int32)]
+                ("chunk_bytes", ctypes.c_int64), ("engine", ctypes.c_int32),
+                ("check_items", ctypes.c_int32)]
 
 
 class _Stats(ctypes.Structure):
@@ -237,6 +238,7 @@ class PlanOptions:
     grid_blocks: int = 0
     chunk_bytes: int = 0
     engine: str = "auto"      # "auto" (bulk-copy engine for device buffers) or "registers"
+    check_items: bool = False  # kernels check every work item's bounds (a debugging aid)
 
 
 # ---------------------------------------------------------------------------
@@ -405,7 +407,8 @@ def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
     else:
         co = _Options(host_only=int(options.host_only), grid_blocks=options.grid_blocks,
                       chunk_bytes=options.chunk_bytes,
-                      engine={"auto": 0, "registers": 1}[options.engine])
+                      engine={"auto": 0, "registers": 1}[options.engine],
+                      check_items=int(options.check_items))
         st = _lib.rr_plan_create_ex(cp, n, ctypes.byref(cs), ctypes.byref(cd), bucket_bytes,
                                     ctypes.byref(co), ctypes.byref(out))
     _check(st, "rr_plan_create")

@@ -127,6 +127,29 @@ def test_random_row_parallel_layouts(seed):
     np.testing.assert_array_equal(H.checksums_host(buf), want_cs)
 
 
+@pytest.mark.parametrize("engine", ["auto", "registers"])
+@pytest.mark.parametrize("case", ["tiny-tp4", "tiny-moe-units-ep2", "random-7", "random-21",
+                                  "row-parallel-2", "row-parallel-9"])
+def test_item_checks_pass_on_valid_plans(case, engine):
+    """With check_items every kernel checks each work item against the plan's
+    buffers; on the plans the planner writes nothing is refused and the bytes
+    are the same."""
+    if case.startswith("random-"):
+        desc = U.random_layout(int(case.split("-")[1]))
+    elif case.startswith("row-parallel-"):
+        desc = U.random_tp_layout(int(case.split("-")[2]))
+    else:
+        desc = U.workload_desc(case)
+    full_parity(desc, engine=engine, check_items=True)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"], engine=engine, check_items=True)
+    buf = H.alloc(plan)
+    H.fill_from_host(buf, U.to_oracle(desc).host_shards(desc["seed"], desc["specials"]))
+    H.pack(buf)
+    rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst)
+    rr.rr_plan_check(plan)
+
+
 @pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-moe-f32", "tiny-fsdp2"])
 def test_register_engine(name):
     """The register path (the fallback for host-resident buffers) on device memory."""
