@@ -1621,6 +1621,7 @@ void rr_device_release(rr_plan* P) {
 
 extern "C" rr_status rr_pack(const rr_plan* P, const void* const* src_shards,
                              void* const* buckets, uint64_t* checksums, cudaStream_t stream) {
+    RR_TRACE("rr_pack");
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
@@ -1629,6 +1630,7 @@ extern "C" rr_status rr_pack(const rr_plan* P, const void* const* src_shards,
 
 extern "C" rr_status rr_unpack(const rr_plan* P, const void* const* buckets, void* const* dst,
                                cudaStream_t stream) {
+    RR_TRACE("rr_unpack");
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
@@ -1638,6 +1640,7 @@ extern "C" rr_status rr_unpack(const rr_plan* P, const void* const* buckets, voi
 extern "C" rr_status rr_verify(const rr_plan* P, const void* const* buckets,
                                const uint64_t* checksums, int64_t* n_bad, int64_t* first_bad,
                                cudaStream_t stream) {
+    RR_TRACE("rr_verify");
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
@@ -1648,6 +1651,7 @@ extern "C" rr_status rr_verify(const rr_plan* P, const void* const* buckets,
 extern "C" rr_status rr_pack_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,
                                    const void* const* src_shards, void* const* buckets,
                                    uint64_t* checksums, cudaStream_t stream) {
+    RR_TRACE("rr_pack_range");
     rr_clear_error();
     Range R;
     rr_status st = check_plan(P);
@@ -1658,6 +1662,7 @@ extern "C" rr_status rr_pack_range(const rr_plan* P, int32_t first_bucket, int32
 extern "C" rr_status rr_unpack_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,
                                      const void* const* buckets, void* const* dst,
                                      cudaStream_t stream) {
+    RR_TRACE("rr_unpack_range");
     rr_clear_error();
     Range R;
     rr_status st = check_plan(P);
@@ -1669,6 +1674,7 @@ extern "C" rr_status rr_verify_range(const rr_plan* P, int32_t first_bucket, int
                                      const void* const* buckets, const uint64_t* checksums,
                                      uint8_t* bad, int64_t* n_bad, int64_t* first_bad,
                                      cudaStream_t stream) {
+    RR_TRACE("rr_verify_range");
     rr_clear_error();
     Range R;
     rr_status st = check_plan(P);
@@ -1679,6 +1685,7 @@ extern "C" rr_status rr_verify_range(const rr_plan* P, int32_t first_bucket, int
 extern "C" rr_status rr_unpack_verify(const rr_plan* P, const void* const* buckets,
                                       const uint64_t* checksums, void* const* dst, uint8_t* bad,
                                       int64_t* n_bad, int64_t* first_bad, cudaStream_t stream) {
+    RR_TRACE("rr_unpack_verify");
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
@@ -1691,6 +1698,7 @@ extern "C" rr_status rr_unpack_verify_range(const rr_plan* P, int32_t first_buck
                                             const uint64_t* checksums, void* const* dst,
                                             uint8_t* bad, int64_t* n_bad, int64_t* first_bad,
                                             cudaStream_t stream) {
+    RR_TRACE("rr_unpack_verify_range");
     rr_clear_error();
     Range R;
     rr_status st = check_plan(P);
@@ -1699,6 +1707,7 @@ extern "C" rr_status rr_unpack_verify_range(const rr_plan* P, int32_t first_buck
 }
 
 extern "C" rr_status rr_plan_check(const rr_plan* P, cudaStream_t stream) {
+    RR_TRACE("rr_plan_check");
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
@@ -1708,6 +1717,7 @@ extern "C" rr_status rr_plan_check(const rr_plan* P, cudaStream_t stream) {
 }
 
 extern "C" rr_status rr_plan_selftest_wait(const rr_plan* P, cudaStream_t stream) {
+    RR_TRACE("rr_plan_selftest_wait");
     rr_clear_error();
     rr_status st = check_plan(P);
     if (st) return st;
@@ -1718,6 +1728,7 @@ extern "C" rr_status rr_plan_selftest_wait(const rr_plan* P, cudaStream_t stream
 
 extern "C" rr_status rr_clear_range(const rr_plan* P, int32_t first_bucket, int32_t n_buckets,
                                     void* const* buckets, cudaStream_t stream) {
+    RR_TRACE("rr_clear_range");
     rr_clear_error();
     Range R;
     rr_status st = check_plan(P);
@@ -1820,6 +1831,7 @@ rr_status launch_static_verify(unsigned long long* scratch, int32_t grid, int32_
 extern "C" rr_status rr_verify_noalloc(const void* const* buckets, int32_t n_buckets,
                                        size_t bucket_bytes, const uint64_t* checksums,
                                        int64_t* n_bad, int64_t* first_bad, cudaStream_t stream) {
+    RR_TRACE("rr_verify_noalloc");
     rr_clear_error();
     if (n_buckets < 0 || n_buckets > kStaticVerifyMaxBuckets)
         return rr_fail(RR_EINVAL,

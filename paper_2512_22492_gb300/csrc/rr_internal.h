@@ -6,7 +6,19 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "rr.h"
+
+// A scoped NVTX range named after a C-ABI call: visible on the timeline of an
+// Nsight tool attached to the process, close to free when none is.
+struct RrTraceRange {
+    explicit RrTraceRange(const char* name) { nvtxRangePushA(name); }
+    ~RrTraceRange() { nvtxRangePop(); }
+    RrTraceRange(const RrTraceRange&) = delete;
+    RrTraceRange& operator=(const RrTraceRange&) = delete;
+};
+#define RR_TRACE(name) RrTraceRange rr_trace_range_(name)
 
 struct rr_plan {
     // ---- source ---------------------------------------------------------

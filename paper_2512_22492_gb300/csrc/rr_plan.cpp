@@ -759,6 +759,7 @@ extern "C" {
 rr_status rr_plan_create_ex(const rr_param* manifest, int32_t n_params,
                             const rr_src_layout* src, const rr_dst_layout* dst,
                             size_t bucket_bytes, const rr_plan_options* opts, rr_plan** out) {
+    RR_TRACE("rr_plan_create");
     rr_clear_error();
     if (!out) return rr_fail(RR_EINVAL, "out is NULL");
     *out = nullptr;
