@@ -452,8 +452,10 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         torch.cuda.synchronize()
     barrier(world)
     total_ms = max_over_ranks(t0.elapsed_time(t1), world)
-    pack_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
-    uv_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    pack_all = [e[0].elapsed_time(e[1]) for e in evs]
+    uv_all = [e[1].elapsed_time(e[2]) for e in evs]
+    pack_ms = statistics.mean(pack_all)
+    uv_ms = statistics.mean(uv_all)
     ms_per_step = total_ms / args.steps
     value = aggregate_gbs(world, step_bytes, ms_per_step)
 
@@ -565,9 +567,11 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                    "parallelism": f"replicas{world}"},
         "ms_per_full_model_sync": round(pack_ms + uv_ms, 3),
         "ops": {
-            "pack": {"ms": round(pack_ms, 3), "bytes": pack_bytes,
+            "pack": {"ms": round(pack_ms, 3), "ms_median": round(statistics.median(pack_all), 3),
+                     "ms_best": round(min(pack_all), 3), "bytes": pack_bytes,
                      "GB/s": round(pack_gbs, 1), "frac_of_peak": round(pack_gbs / peak, 4)},
-            "unpack_verify": {"ms": round(uv_ms, 3), "bytes": uv_bytes,
+            "unpack_verify": {"ms": round(uv_ms, 3), "ms_median": round(statistics.median(uv_all), 3),
+                              "ms_best": round(min(uv_all), 3), "bytes": uv_bytes,
                               "GB/s": round(uv_bytes / (uv_ms * 1e-3) / 1e9, 1),
                               "frac_of_peak": round(uv_bytes / (uv_ms * 1e-3) / 1e9 / peak, 4)},
             "unpack": {"ms": round(unpack_ms, 3), "bytes": unpack_bytes,
