@@ -383,7 +383,7 @@ __device__ __forceinline__ unsigned long long pack_scalar(const char* src, char*
     return acc;
 }
 
-template <int NPTR>
+template <int NPTR, bool CHECK>
 __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(const __grid_constant__ PackArgs<NPTR> a) {
     uint32_t i0, i1;
     block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
@@ -391,7 +391,7 @@ __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(c
     uint32_t cur = 0xFFFFFFFFu;
     for (uint32_t it = i0; it < i1; ++it) {
         const rr_pack_item d = a.items[it];
-        if (!pack_item_ok(a.chk, d)) continue;
+        if (CHECK && !pack_item_ok(a.chk, d)) continue;
         if (d.bucket != cur) {
             if (cur != 0xFFFFFFFFu) flush(a.checksums + cur, acc);
             cur = d.bucket;
@@ -453,7 +453,7 @@ __device__ void compare_in_last_block(unsigned long long* counters,
 // Copies each item's bytes from its bucket to its tensor.  With VERIFY it also
 // sums every bucket byte it reads (the gap READ items too) into the bucket's
 // checksum and compares at the end, so the buckets are read once for both.
-template <int NPTR, bool VERIFY>
+template <int NPTR, bool VERIFY, bool CHECK>
 __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
     constexpr int U = 2 * kUnroll;   // one 16-byte load per vector: twice the pack's depth
     uint32_t i0, i1;
@@ -463,7 +463,7 @@ __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_con
     for (uint32_t it = i0; it < i1; ++it) {
         const rr_unpack_item d = a.items[it];
         if (!VERIFY && d.kind >= RR_ITEM_READ_VEC) continue;
-        if (!unpack_item_ok(a.chk, d)) continue;
+        if (CHECK && !unpack_item_ok(a.chk, d)) continue;
         if (VERIFY && d.bucket != cur) {
             if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - a.first_bucket), acc);
             cur = d.bucket;
@@ -601,7 +601,6 @@ enum : uint16_t {
 };
 
 constexpr uint32_t kMinBulkRowBytes = 1024;
-constexpr int kFullArrivals = 33;   // per piece: the metadata arrival + one per producer lane
 constexpr uint32_t kMaxFanDst = 16; // fan-out destinations per head (the planner's limit)
 
 struct Piece {
@@ -678,7 +677,10 @@ __device__ __forceinline__ void consumers_sync() {
 // Short aligned rows (16-byte aligned, row bytes a multiple of 16) gathered
 // into a stage by the whole producer warp: 16-byte cp.async copies, lane l
 // taking vectors l, l + 32, ...; the rows land back to back.  Each lane's
-// completion is one arrival on the stage's full barrier.
+// copies are tracked by the stage's full barrier: the counted form of
+// cp.async.mbarrier.arrive raises the barrier's pending count now and arrives
+// once the lane's copies have landed, so the phase cannot complete before them
+// (the caller's own arrival, after a __syncwarp, is the one the count expects).
 __device__ __forceinline__ void gather_async(uint32_t stage, uint32_t full_bar, const char* src,
                                              uint64_t src_stride, uint32_t rows,
                                              uint32_t row_bytes, uint32_t lane) {
@@ -697,7 +699,7 @@ __device__ __forceinline__ void gather_async(uint32_t stage, uint32_t full_bar, 
             ++r;
         }
     }
-    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(full_bar) : "memory");
+    asm volatile("cp.async.mbarrier.arrive.shared::cta.b64 [%0];" ::"r"(full_bar) : "memory");
 }
 
 template <int NPTR>
@@ -706,8 +708,9 @@ __device__ __forceinline__ char* bulk_bucket(const BulkArgs<NPTR>& a, uint32_t b
                            : (char*)a.ptr[table_base + b];
 }
 
-// MODE 0: pack, 1: unpack, 2: unpack with checksum comparison.
-template <int NPTR, int MODE>
+// MODE 0: pack, 1: unpack, 2: unpack with checksum comparison.  CHECK: check
+// every item against the plan's buffers first (the check_items option).
+template <int NPTR, int MODE, bool CHECK>
 __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(const __grid_constant__ BulkArgs<NPTR> a) {
     constexpr int kConsumerWarps = BulkShape<MODE>::kWarps;
     constexpr int kStageBytes = BulkShape<MODE>::kStageBytes;
@@ -722,9 +725,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
-            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(&full[s])),
-                         "n"(kFullArrivals)
-                         : "memory");
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full[s])) : "memory");
             asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(&empty[s])),
                          "n"(kConsumerWarps)
                          : "memory");
@@ -739,11 +740,10 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         // The whole warp walks the items in step (every lane decodes the same
-        // item).  Each piece takes kFullArrivals arrivals on its stage's full
-        // barrier: lane 0's plain (release) arrival after it wrote the piece's
-        // metadata, then one per lane for the data -- lane 0's carrying the
-        // byte count of its bulk copies, a gather's being its lanes' cp.async
-        // completions, plain otherwise.
+        // item).  Each piece completes its stage's full barrier with one
+        // arrival by lane 0, made after it wrote the piece's metadata: with the
+        // byte count of its bulk copies (expect_tx), or plain.  A gather's lanes
+        // have each registered their cp.async copies with the barrier first.
         enum { kMeta = 0, kBulk = 1, kGather = 2 };
         uint32_t count = 0;   // pieces issued
         bool ok = true;
@@ -760,17 +760,17 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                 // A fan-out piece carries its destination items in shared memory.
                 if (p.kind == PC_FAN && lane < p.n)
                     fan_dst[s][lane] = ((const rr_pack_item*)a.items)[p.sum_bucket + lane];
-                __syncwarp();
-            }
-            if (lane == 0) {
-                meta[s] = p;
-                mbar_arrive(fb);
             }
             const uint32_t stage = smem_u32(stage_mem + s * kStageBytes);
             const uint32_t row_bytes = p.row_len * p.es;
-            if (how == kGather) {
-                gather_async(stage, fb, p.src, p.src_stride, p.rows, row_bytes, lane);
-            } else if (how == kBulk && lane == 0) {
+            if (how == kGather) gather_async(stage, fb, p.src, p.src_stride, p.rows, row_bytes, lane);
+            __syncwarp();
+            if (lane != 0) {
+                ++count;
+                return;
+            }
+            meta[s] = p;
+            if (how == kBulk) {
                 asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb),
                              "r"(row_bytes * p.rows)
                              : "memory");
@@ -798,7 +798,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
             p.src_stride = 0;
             if (MODE == 0) {
                 const rr_pack_item d = ((const rr_pack_item*)a.items)[it];
-                if (!pack_item_ok(a.chk, d)) {
+                if (CHECK && !pack_item_ok(a.chk, d)) {
                     if (d.kind == RR_ITEM_FAN_F32 || d.kind == RR_ITEM_FAN_BF16)
                         it += min(d.dst_off, i1 - 1 - it);   // and its destinations
                     continue;
@@ -856,7 +856,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                         bad = f.kind != RR_ITEM_FAN_DST || f.row_len % 8 != 0 ||
                               f.dst_off % 16 != 0 || (f.src * es) % 16 != 0 ||
                               f.src + f.row_len > d.row_len || f.n_rows != R ||
-                              !pack_item_in(a.chk, f);
+                              (CHECK && !pack_item_in(a.chk, f));
                     }
                     if (__any_sync(0xFFFFFFFFu, bad)) {
                         if (lane == 0) atomicExch(a.err, kErrBadItem);
@@ -904,7 +904,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                 const rr_unpack_item d = ((const rr_unpack_item*)a.items)[it];
                 const bool read_only = d.kind == RR_ITEM_READ_VEC || d.kind == RR_ITEM_READ_SCALAR;
                 if (MODE == 1 && read_only) continue;
-                if (!unpack_item_ok(a.chk, d)) continue;
+                if (CHECK && !unpack_item_ok(a.chk, d)) continue;
                 const char* src = bulk_bucket(a, d.bucket, 0) + d.src_off;
                 char* dst = read_only ? nullptr : (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off;
                 p.sum_bucket = d.bucket;
@@ -1091,9 +1091,9 @@ __global__ void rr_wait_selftest_kernel(unsigned int* err) {
     if (threadIdx.x == 0) mbar_wait(smem_u32(&bar), 0, err);
 }
 
-template <int NPTR, int MODE>
+template <int NPTR, int MODE, bool CHECK = false>
 cudaError_t bulk_prepare() {
-    return cudaFuncSetAttribute(rr_bulk_kernel<NPTR, MODE>,
+    return cudaFuncSetAttribute(rr_bulk_kernel<NPTR, MODE, CHECK>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 BulkShape<MODE>::kSmem);
 }
@@ -1188,7 +1188,10 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
         a.bucket_base = (char*)buckets[0];
         a.bucket_stride = stride;
     }
-    rr_pack_kernel<NPTR><<<P->reg_pack_grid, kThreads, 0, s>>>(a);
+    if (P->check_items)
+        rr_pack_kernel<NPTR, true><<<P->reg_pack_grid, kThreads, 0, s>>>(a);
+    else
+        rr_pack_kernel<NPTR, false><<<P->reg_pack_grid, kThreads, 0, s>>>(a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -1223,10 +1226,14 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     }
     a.dst_base = k;
     for (int32_t t = 0; t < P->n_tensors; ++t) a.ptr[k++] = dst[t];
-    if (checksums)
-        rr_unpack_kernel<NPTR, true><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
+    if (checksums && P->check_items)
+        rr_unpack_kernel<NPTR, true, true><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
+    else if (checksums)
+        rr_unpack_kernel<NPTR, true, false><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
+    else if (P->check_items)
+        rr_unpack_kernel<NPTR, false, true><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
     else
-        rr_unpack_kernel<NPTR, false><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
+        rr_unpack_kernel<NPTR, false, false><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -1325,10 +1332,16 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         a.dst_base = k;
         for (int32_t t = 0; t < P->n_tensors; ++t) a.ptr[k++] = dst[t];
     }
-    RR_CUDA((bulk_prepare<NPTR, MODE>()));
     const int32_t grid = MODE == 0 ? P->grid_blocks : P->unpack_grid_blocks;
-    rr_bulk_kernel<NPTR, MODE>
-        <<<grid, BulkShape<MODE>::kThreads, BulkShape<MODE>::kSmem, s>>>(a);
+    if (P->check_items) {
+        RR_CUDA((bulk_prepare<NPTR, MODE, true>()));
+        rr_bulk_kernel<NPTR, MODE, true>
+            <<<grid, BulkShape<MODE>::kThreads, BulkShape<MODE>::kSmem, s>>>(a);
+    } else {
+        RR_CUDA((bulk_prepare<NPTR, MODE, false>()));
+        rr_bulk_kernel<NPTR, MODE, false>
+            <<<grid, BulkShape<MODE>::kThreads, BulkShape<MODE>::kSmem, s>>>(a);
+    }
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -1517,16 +1530,16 @@ rr_status rr_device_default_grid(rr_grids* g) {
     int dev = 0, sms = 0, p = 0, u = 0, v = 0, b = 0;
     RR_CUDA(cudaGetDevice(&dev));
     RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs>, kThreads, 0));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, true>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs, false>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, true, false>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, rr_verify_kernel<kLargePtrs>, kThreads, 0));
     int bp = 0;
     RR_CUDA((bulk_prepare<kLargePtrs, 0>()));
     RR_CUDA((bulk_prepare<kLargePtrs, 2>()));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bp, rr_bulk_kernel<kLargePtrs, 0>,
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bp, rr_bulk_kernel<kLargePtrs, 0, false>,
                                                           BulkShape<0>::kThreads,
                                                           BulkShape<0>::kSmem));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, rr_bulk_kernel<kLargePtrs, 2>,
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, rr_bulk_kernel<kLargePtrs, 2, false>,
                                                           BulkShape<2>::kThreads,
                                                           BulkShape<2>::kSmem));
     g->reg_pack = sms * (p > 0 ? p : 1);
