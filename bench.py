@@ -88,6 +88,13 @@ def dist_setup(args):
     return world, rank, local
 
 
+def host_memory_bytes() -> int:
+    try:
+        return os.sysconf("SC_PAGE_SIZE") * os.sysconf("SC_PHYS_PAGES")
+    except (ValueError, OSError, AttributeError):
+        return 1 << 62
+
+
 def barrier(world):
     if world > 1:
         import torch.distributed as dist
@@ -517,7 +524,15 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     # End to end through the public API with host buffers: every step copies the
     # trainer's shards from pinned host memory, syncs, and reads back the checksums.
     e2e = None
-    if not args.no_e2e:
+    local_ranks = int(os.environ.get("LOCAL_WORLD_SIZE", str(world)))
+    pinned_need = local_ranks * buf.flat.numel()
+    if not args.no_e2e and pinned_need > host_memory_bytes() // 2:
+        # Every local rank would pin its whole source on the host: refuse
+        # rather than exhaust the node's memory.
+        e2e = {"skipped": f"{local_ranks} ranks x {buf.flat.numel() / 1e9:.1f} GB of pinned "
+                          f"host memory exceed half of this host's "
+                          f"{host_memory_bytes() / 1e9:.0f} GB"}
+    elif not args.no_e2e:
         host_src = torch.empty(buf.flat.numel(), dtype=torch.uint8, pin_memory=True)
         host_src.copy_(buf.flat)
         host_cs = torch.empty(buf.checksums.numel(), dtype=torch.int64, pin_memory=True)
