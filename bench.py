@@ -54,6 +54,9 @@ def parse():
                     help="with --layers: a smaller vocabulary as well")
     ap.add_argument("--chunk-kib", type=int, default=0, help="plan option: KiB per work item")
     ap.add_argument("--grid", type=int, default=0, help="plan option: persistent grid size")
+    ap.add_argument("--sync-verify", action="store_true",
+                    help="the receiver uses the synchronous rr_unpack_verify (a host round "
+                         "trip per step) instead of rr_unpack_verify_async")
     ap.add_argument("--check-items", action="store_true",
                     help="plan option: kernels check every work item's bounds")
     ap.add_argument("--engine", choices=["auto", "registers"], default="auto",
@@ -430,17 +433,37 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     uv_bytes = st["verify_bytes_read"] + st["unpack_bytes_written"]
     step_bytes = pack_bytes + uv_bytes
 
+    # The receiver's check: stream-ordered by default, each step's {n_bad,
+    # first_bad} left in its own row of `results` and read after the timing.
+    scratch = torch.zeros(plan.n_buckets + 4, dtype=torch.int64, device="cuda")
+    n_rows = 2 * (max(3, args.warmup) + args.steps) + 8
+    results = torch.full((n_rows, 2), -7, dtype=torch.int64, device="cuda")
+    used = [0]
+
     def step(ev=None):
         if ev:
             ev[0].record(stream)
         rr.rr_pack(plan, t_src, t_bkt, buf.checksums, stream)
         if ev:
             ev[1].record(stream)
-        n_bad, _ = rr.rr_unpack_verify(plan, t_bkt, buf.checksums, t_dst, stream=stream)
+        if args.sync_verify:
+            n_bad, _ = rr.rr_unpack_verify(plan, t_bkt, buf.checksums, t_dst, stream=stream)
+            if n_bad:
+                raise RuntimeError(f"verify found {n_bad} bad buckets")
+        else:
+            row = results[used[0] % n_rows]
+            used[0] += 1
+            rr.rr_unpack_verify_async(plan, t_bkt, buf.checksums, t_dst, scratch, row,
+                                      stream=stream)
         if ev:
             ev[2].record(stream)
-        if n_bad:
-            raise RuntimeError(f"verify found {n_bad} bad buckets")
+        return None if args.sync_verify else row
+
+    def check_results():
+        torch.cuda.synchronize()
+        got = results[:min(used[0], n_rows)].cpu()
+        if used[0] and not bool(((got[:, 0] == 0) & (got[:, 1] == -1)).all()):
+            raise RuntimeError(f"verify found bad buckets: {got.tolist()}")
 
     for _ in range(max(3, args.warmup)):
         step()
@@ -465,6 +488,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     uv_ms = statistics.mean(uv_all)
     ms_per_step = total_ms / args.steps
     value = aggregate_gbs(world, step_bytes, ms_per_step)
+    check_results()
 
     # Breakdown only (not part of the step): the receiver's two separate calls.
     # rr_unpack is asynchronous, so its launches are timed back to back; rr_verify
@@ -536,12 +560,15 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         host_src = torch.empty(buf.flat.numel(), dtype=torch.uint8, pin_memory=True)
         host_src.copy_(buf.flat)
         host_cs = torch.empty(buf.checksums.numel(), dtype=torch.int64, pin_memory=True)
-        h2d, d2h = host_src.numel(), host_cs.numel() * 8 + 32
+        host_res = torch.empty(2, dtype=torch.int64, pin_memory=True)
+        h2d, d2h = host_src.numel(), host_cs.numel() * 8 + 16
 
         def e2e_step():
             buf.flat.copy_(host_src, non_blocking=True)
-            step()
+            row = step()
             host_cs.copy_(buf.checksums, non_blocking=True)
+            if row is not None:
+                host_res.copy_(row, non_blocking=True)
 
         for _ in range(2):
             e2e_step()
@@ -555,6 +582,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         b.record(stream)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(a.elapsed_time(b), world) / args.steps
+        check_results()
         e2e = {"value": round(aggregate_gbs(world, step_bytes, e2e_ms), 2), "unit": UNIT,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": round(e2e_ms, 3)}
@@ -576,7 +604,8 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         "config": {"workload": w.name, "src_dtype": w.src_dtype, "n_shards": w.n_shards,
                    "sharding": w.sharding, "expert_parallel": w.ep,
                    "tp": w.tp, "bucket_bytes": bucket_bytes, "n_buckets": plan.n_buckets,
-                   "step": "rr_pack + rr_unpack_verify (unpack and checksum check fused)",
+                   "step": "rr_pack + rr_unpack_verify" + ("" if args.sync_verify else "_async") +
+                           " (unpack and checksum check fused)",
                    "engine": args.engine, "check_items": args.check_items,
                    "step_bytes": step_bytes, "l2": "inputs > L2 (no flush needed)",
                    "parallelism": f"replicas{world}"},
@@ -607,7 +636,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                                        "method": "torch copy_ of 4 GiB on the device, "
                                                  "read + write bytes"}},
         "clocks": clocks,
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": (2 if args.sync_verify else 3) * args.steps,
         "e2e": e2e,
     }
     if snapshot:

@@ -393,6 +393,23 @@ rr_status rr_unpack_verify_range(const rr_plan* plan, int32_t first_bucket, int3
  * [pack_first[b], pack_first[b + 1]); likewise for unpack. */
 rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32_t* unpack_first);
 
+/* Stream-ordered form of rr_unpack_verify(_range), for a receiver that unpacks
+ * and checks piece after piece without waiting on the host (Sections 5.2.1 and
+ * 5.2.2: the pull completes, and a resumed pull checks what it holds).
+ *   first_bucket, n_buckets: the range (0 and the plan's count for all).
+ *   scratch: caller device memory of n_buckets + 4 uint64, 16-byte aligned;
+ *            zeroed and used by the call, free again once `result` is written.
+ *            Calls that overlap in time need distinct scratch.
+ *   result:  two int64 in device memory or pinned (mapped) host memory, 8-byte
+ *            aligned; when the call's work is done on `stream` they hold
+ *            {number of bad buckets, first bad bucket or -1}.
+ * Returns after enqueueing; argument errors come back at once.  A kernel that
+ * gave up a bounded wait is reported by rr_plan_check, not in `result`. */
+rr_status rr_unpack_verify_async(const rr_plan* plan, int32_t first_bucket, int32_t n_buckets,
+                                 const void* const* buckets, const uint64_t* checksums,
+                                 void* const* dst, uint8_t* bad, uint64_t* scratch,
+                                 int64_t* result, cudaStream_t stream);
+
 /* Allocation-free form of rr_verify.  The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory when they
  * check a pull, such as an inference engine that has reserved nearly all

@@ -10,7 +10,8 @@ from .rr import (Block, DstLayout, DstTensor, Param, Plan, PlanOptions, Pointers
                  SrcLayout,
                  rr_clear_range, rr_pack, rr_pack_range, rr_plan_check, rr_plan_create,
                  rr_plan_selftest_wait, rr_status_str, rr_unpack,
-                 rr_unpack_range, rr_unpack_verify, rr_verify, rr_verify_noalloc,
+                 rr_unpack_range, rr_unpack_verify, rr_unpack_verify_async, rr_verify,
+                 rr_verify_noalloc,
                  rr_verify_range)
 from .layouts import qwen3_layer_units, qwen3_manifest, qwen3_rollout, qwen3_sync
 
@@ -18,5 +19,5 @@ __all__ = ["Block", "DstLayout", "DstTensor", "Param", "Plan", "PlanOptions", "P
            "RRError",
            "SrcLayout", "rr_pack", "rr_plan_create", "rr_status_str", "rr_unpack", "rr_verify",
            "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
-           "rr_unpack_verify", "rr_plan_check", "rr_plan_selftest_wait", "rr_verify_noalloc",
+           "rr_unpack_verify", "rr_unpack_verify_async", "rr_plan_check", "rr_plan_selftest_wait", "rr_verify_noalloc",
            "qwen3_layer_units", "qwen3_manifest", "qwen3_rollout", "qwen3_sync"]

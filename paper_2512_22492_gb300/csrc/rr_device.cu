@@ -1151,6 +1151,7 @@ rr_status check_ptrs(const void* const* ptrs, int32_t n, const char* what) {
 struct Range {
     int32_t b0, b1;
     bool full;
+    unsigned long long* scratch;   // verify sums and counters of this call (NULL: the plan's)
 };
 
 // The bounds the kernels check items against, when the plan asks for checks.
@@ -1210,8 +1211,9 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     a.item_begin = P->unpack_bucket_first[R.b0];
     a.item_end = P->unpack_bucket_first[R.b1];
     if (checksums) {
-        a.sums = P->d_verify_scratch;
-        a.counters = P->d_verify_scratch + (R.b1 - R.b0);
+        unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
+        a.sums = sc;
+        a.counters = sc + (R.b1 - R.b0);
         a.expected = (const unsigned long long*)checksums;
         a.bad = bad;
         a.first_bucket = R.b0;
@@ -1314,8 +1316,9 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         a.item_begin = P->unpack_bucket_first[R.b0];
         a.item_end = P->unpack_bucket_first[R.b1];
         if (MODE == 2) {
-            a.sums = P->d_verify_scratch;
-            a.counters = P->d_verify_scratch + (R.b1 - R.b0);
+            unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
+            a.sums = sc;
+            a.counters = sc + (R.b1 - R.b0);
             a.expected = (const unsigned long long*)checksums;
             a.bad = bad;
             a.first_bucket = R.b0;
@@ -1458,26 +1461,18 @@ rr_status read_result(const rr_plan* P, int32_t n, int64_t* n_bad, int64_t* firs
     return nb ? RR_EMISMATCH : RR_OK;
 }
 
-rr_status unpack_verify_impl(const rr_plan* P, Range R, const void* const* buckets,
-                             const uint64_t* checksums, void* const* dst, uint8_t* bad,
-                             int64_t* n_bad, int64_t* first_bad, cudaStream_t stream) {
-    rr_status st;
-    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
-    if ((st = check_dst(P, dst))) return st;
-    if (R.b1 > R.b0 && !aligned16(checksums))
-        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
-    if (n_bad) *n_bad = 0;
-    if (first_bad) *first_bad = -1;
-    if (R.b1 == R.b0) return RR_OK;
-    rr_plan* M = const_cast<rr_plan*>(P);   // the scratch area is the only mutable state
-    std::lock_guard<std::mutex> lock(M->verify_mutex);
+// Enqueues the verifying unpack of range R: zeroes the range's sums and
+// counters (R.scratch, else the plan's) and launches the kernel.
+rr_status enqueue_unpack_verify(const rr_plan* P, Range R, const void* const* buckets,
+                                const uint64_t* checksums, void* const* dst, uint8_t* bad,
+                                cudaStream_t stream) {
     const int32_t n = R.b1 - R.b0;
-    RR_CUDA(cudaMemsetAsync(P->d_verify_scratch, 0, (size_t(n) + 4) * sizeof(unsigned long long),
-                            stream));
+    unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
+    RR_CUDA(cudaMemsetAsync(sc, 0, (size_t(n) + 4) * sizeof(unsigned long long), stream));
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
                       all_device((const void* const*)dst, P->n_tensors);
-    const Range Rr{R.b0, R.b1, R.full && !bulk && P->engine == RR_ENGINE_REGISTERS};
-    st = with_unpack_shape(P, buckets, [&](bool small, bool table, uint64_t stride) {
+    const Range Rr{R.b0, R.b1, R.full && !bulk && P->engine == RR_ENGINE_REGISTERS, R.scratch};
+    return with_unpack_shape(P, buckets, [&](bool small, bool table, uint64_t stride) {
         if (bulk)
             return small ? launch_bulk<kSmallPtrs, 2>(P, R, nullptr, buckets, dst, checksums, bad,
                                                       table, stride, stream)
@@ -1488,8 +1483,51 @@ rr_status unpack_verify_impl(const rr_plan* P, Range R, const void* const* bucke
                      : launch_unpack<kLargePtrs>(P, Rr, buckets, dst, checksums, bad, table, stride,
                                                  stream);
     });
+}
+
+rr_status check_unpack_verify_args(const rr_plan* P, Range R, const void* const* buckets,
+                                   const uint64_t* checksums, void* const* dst) {
+    rr_status st;
+    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if ((st = check_dst(P, dst))) return st;
+    if (R.b1 > R.b0 && !aligned16(checksums))
+        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    return RR_OK;
+}
+
+rr_status unpack_verify_impl(const rr_plan* P, Range R, const void* const* buckets,
+                             const uint64_t* checksums, void* const* dst, uint8_t* bad,
+                             int64_t* n_bad, int64_t* first_bad, cudaStream_t stream) {
+    rr_status st = check_unpack_verify_args(P, R, buckets, checksums, dst);
     if (st) return st;
-    return read_result(P, n, n_bad, first_bad, stream);
+    if (n_bad) *n_bad = 0;
+    if (first_bad) *first_bad = -1;
+    if (R.b1 == R.b0) return RR_OK;
+    rr_plan* M = const_cast<rr_plan*>(P);   // the scratch area is the only mutable state
+    std::lock_guard<std::mutex> lock(M->verify_mutex);
+    if ((st = enqueue_unpack_verify(P, R, buckets, checksums, dst, bad, stream))) return st;
+    return read_result(P, R.b1 - R.b0, n_bad, first_bad, stream);
+}
+
+// {n_bad, first_bad or -1} from a verifying pass's counters (NULL: an empty range).
+__global__ void rr_verify_result_kernel(const unsigned long long* counters, long long* result) {
+    const unsigned long long nb = counters ? counters[1] : 0ull;
+    result[0] = (long long)nb;
+    result[1] = nb ? (long long)(ULLONG_MAX - counters[2]) : -1ll;
+}
+
+// The device address of a result buffer: device memory, or pinned (mapped)
+// host memory; NULL for anything else (pageable host memory).
+long long* result_address(int64_t* result) {
+    cudaPointerAttributes at;
+    if (!result || (uintptr_t)result % 8 != 0 || cudaPointerGetAttributes(&at, result) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged)
+        return (long long*)result;
+    if (at.type == cudaMemoryTypeHost && at.devicePointer) return (long long*)at.devicePointer;
+    return nullptr;
 }
 
 rr_status verify_impl(const rr_plan* P, Range R, const void* const* buckets,
@@ -1717,6 +1755,32 @@ extern "C" rr_status rr_unpack_verify_range(const rr_plan* P, int32_t first_buck
     rr_status st = check_plan(P);
     if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
     return unpack_verify_impl(P, R, buckets, checksums, dst, bad, n_bad, first_bad, stream);
+}
+
+extern "C" rr_status rr_unpack_verify_async(const rr_plan* P, int32_t first_bucket,
+                                            int32_t n_buckets, const void* const* buckets,
+                                            const uint64_t* checksums, void* const* dst,
+                                            uint8_t* bad, uint64_t* scratch, int64_t* result,
+                                            cudaStream_t stream) {
+    RR_TRACE("rr_unpack_verify_async");
+    rr_clear_error();
+    Range R;
+    rr_status st = check_plan(P);
+    if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
+    if ((st = check_unpack_verify_args(P, R, buckets, checksums, dst))) return st;
+    long long* res = result_address(result);
+    if (!res)
+        return rr_fail(RR_EINVAL, "result must be 8-byte aligned device or pinned host memory");
+    if (R.b1 > R.b0) {
+        if (!aligned16(scratch)) return rr_fail(RR_EINVAL, "scratch NULL or not 16-byte aligned");
+        if (!device_resident(scratch)) return rr_fail(RR_EINVAL, "scratch must be device memory");
+        R.scratch = (unsigned long long*)scratch;
+        if ((st = enqueue_unpack_verify(P, R, buckets, checksums, dst, bad, stream))) return st;
+    }
+    rr_verify_result_kernel<<<1, 1, 0, stream>>>(R.b1 > R.b0 ? R.scratch + (R.b1 - R.b0) : nullptr,
+                                                 res);
+    RR_CUDA(cudaGetLastError());
+    return RR_OK;
 }
 
 extern "C" rr_status rr_plan_check(const rr_plan* P, cudaStream_t stream) {

@@ -146,6 +146,8 @@ _sig("rr_unpack_verify", [_vp, ctypes.POINTER(_vp), _vp, ctypes.POINTER(_vp), _v
 _sig("rr_unpack_verify_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp,
                                 ctypes.POINTER(_vp), _vp, _P64, _P64, _vp])
 _sig("rr_clear_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp])
+_sig("rr_unpack_verify_async", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp,
+                                ctypes.POINTER(_vp), _vp, _vp, _vp, _vp])
 _sig("rr_plan_bucket_items", [_vp, ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_uint32)])
 _sig("rr_verify_noalloc", [ctypes.POINTER(_vp), ctypes.c_int32, ctypes.c_size_t, _vp, _P64, _P64,
                            _vp])
@@ -160,7 +162,7 @@ EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_q
             "rr_plan_export_pack", "rr_plan_export_pack_full",
             "rr_plan_export_unpack", "rr_plan_bucket_items", "rr_pack", "rr_unpack", "rr_verify",
             "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
-            "rr_unpack_verify", "rr_unpack_verify_range",
+            "rr_unpack_verify", "rr_unpack_verify_range", "rr_unpack_verify_async",
             "rr_verify_noalloc",
             "rr_plan_check", "rr_plan_selftest_wait", "rr_status_str", "rr_last_error")
 
@@ -641,6 +643,27 @@ def rr_unpack_verify(plan: Plan, buckets, checksums, dst, bad=None, stream=None,
     if st not in (RR_OK, RR_EMISMATCH):
         _check(st, "rr_unpack_verify")
     return n_bad.value, first.value
+
+
+def rr_unpack_verify_async(plan: Plan, buckets, checksums, dst, scratch, result, bad=None,
+                           stream=None, first_bucket: int = 0,
+                           n_buckets: Optional[int] = None) -> None:
+    """Stream-ordered unpack + verify: returns after enqueueing.  `scratch` is a
+    device tensor of at least n_buckets + 4 int64 (reused only after `result`
+    is written); `result` (2 int64, device or pinned host memory) receives
+    {n_bad, first_bad or -1} when the work on `stream` is done."""
+    _check_list(buckets, plan.n_buckets, plan.bucket_bytes, "buckets", plan=plan)
+    _check_list(dst, plan.n_tensors, lambda i: 2 * plan.tensor_numel[i], "dst", plan=plan)
+    _check_checksums(plan, checksums)
+    n = plan.n_buckets - first_bucket if n_buckets is None else n_buckets
+    for what, x, need in (("scratch", scratch, 8 * (n + 4)), ("result", result, 16),
+                          ("bad", bad, n)):
+        if x is not None and _nbytes(x) is not None and _nbytes(x) < need:
+            raise ValueError(f"{what}: {_nbytes(x)} bytes, need {need}")
+    _check(_lib.rr_unpack_verify_async(plan.handle, first_bucket, n, _ptr_array(buckets),
+                                       _ptr(checksums), _ptr_array(dst),
+                                       None if bad is None else _ptr(bad), _ptr(scratch),
+                                       _ptr(result), _stream(stream)), "rr_unpack_verify_async")
 
 
 def rr_clear_range(plan: Plan, first_bucket: int, n_buckets: int, buckets, stream=None) -> None:
