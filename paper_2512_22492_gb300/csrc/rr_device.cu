@@ -1138,11 +1138,47 @@ rr_status check_plan(const rr_plan* P) {
     return RR_OK;
 }
 
-rr_status check_ptrs(const void* const* ptrs, int32_t n, const char* what) {
+// Whether a kernel of this library may touch memory at p: device (or
+// managed) memory, pinned host memory mapped for the device, or -- on a device
+// that reads pageable host memory (address translation over the CPU's page
+// tables, as on Grace) -- any host memory.  Pageable memory elsewhere would
+// fault the GPU, so it is refused.
+bool reachable(const void* p, bool pageable_ok) {
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return pageable_ok;
+    }
+    if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) return true;
+    if (at.type == cudaMemoryTypeHost) return at.devicePointer != nullptr;
+    return pageable_ok;
+}
+
+// Pointer arrays: every entry 16-byte aligned; the first and the last entry
+// reachable from the device (arrays are expected to be of one kind of memory).
+rr_status check_ptrs(bool pageable_ok, const void* const* ptrs, int32_t n, const char* what) {
     if (n > 0 && !ptrs) return rr_fail(RR_EINVAL, "%s array is NULL", what);
     for (int32_t i = 0; i < n; ++i)
         if (!aligned16(ptrs[i]))
             return rr_fail(RR_EINVAL, "%s[%d] is NULL or not 16-byte aligned", what, i);
+    for (int32_t i : {0, n - 1})
+        if (n > 0 && !reachable(ptrs[i], pageable_ok))
+            return rr_fail(RR_EINVAL,
+                           "%s[%d] is host memory this GPU cannot read (pageable); use device "
+                           "memory or pinned host memory",
+                           what, i);
+    return RR_OK;
+}
+
+// One buffer a kernel reads or writes (checksums, per-bucket flags): 16-byte
+// aligned (when `aligned` is asked) and reachable from the device.
+rr_status check_buf(bool pageable_ok, const void* p, const char* what, bool aligned = true) {
+    if (!p || (aligned && !aligned16(p)))
+        return rr_fail(RR_EINVAL, "%s NULL or not 16-byte aligned", what);
+    if (!reachable(p, pageable_ok))
+        return rr_fail(RR_EINVAL,
+                       "%s is host memory this GPU cannot read (pageable); use device memory "
+                       "or pinned host memory", what);
     return RR_OK;
 }
 
@@ -1378,10 +1414,10 @@ rr_status check_range(const rr_plan* P, int32_t first, int32_t n, Range* R) {
 rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, void* const* buckets,
                     uint64_t* checksums, cudaStream_t stream) {
     rr_status st;
-    if ((st = check_ptrs(src_shards, P->n_shards, "src_shards"))) return st;
-    if ((st = check_ptrs((const void* const*)buckets, P->n_buckets, "buckets"))) return st;
+    if ((st = check_ptrs(P->pageable_ok != 0, src_shards, P->n_shards, "src_shards"))) return st;
+    if ((st = check_ptrs(P->pageable_ok != 0, (const void* const*)buckets, P->n_buckets, "buckets"))) return st;
     if (R.b1 == R.b0) return RR_OK;
-    if (!aligned16(checksums)) return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    if ((st = check_buf(P->pageable_ok != 0, checksums, "checksums"))) return st;
     uint64_t stride = 0;
     const bool table = !uniform((const void* const*)buckets, P->n_buckets, P->bucket_bytes, &stride);
     const int32_t need = P->n_shards + (table ? P->n_buckets : 0);
@@ -1411,6 +1447,12 @@ rr_status check_dst(const rr_plan* P, void* const* dst) {
     for (int32_t t = 0; t < P->n_tensors; ++t)
         if (P->tensor_numel[t] > 0 && !aligned16(dst[t]))
             return rr_fail(RR_EINVAL, "dst[%d] is NULL or not 16-byte aligned", t);
+    for (int32_t t : {0, P->n_tensors - 1})
+        if (P->n_tensors > 0 && P->tensor_numel[t] > 0 && !reachable(dst[t], P->pageable_ok != 0))
+            return rr_fail(RR_EINVAL,
+                           "dst[%d] is host memory this GPU cannot read (pageable); use device "
+                           "memory or pinned host memory",
+                           t);
     return RR_OK;
 }
 
@@ -1428,7 +1470,7 @@ rr_status with_unpack_shape(const rr_plan* P, const void* const* buckets, F laun
 rr_status unpack_impl(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
                       cudaStream_t stream) {
     rr_status st;
-    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if ((st = check_ptrs(P->pageable_ok != 0, buckets, P->n_buckets, "buckets"))) return st;
     if ((st = check_dst(P, dst))) return st;
     if (P->unpack_bucket_first[R.b0] == P->unpack_bucket_first[R.b1]) return RR_OK;
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
@@ -1486,19 +1528,20 @@ rr_status enqueue_unpack_verify(const rr_plan* P, Range R, const void* const* bu
 }
 
 rr_status check_unpack_verify_args(const rr_plan* P, Range R, const void* const* buckets,
-                                   const uint64_t* checksums, void* const* dst) {
+                                   const uint64_t* checksums, void* const* dst,
+                                   const uint8_t* bad) {
     rr_status st;
-    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
+    if ((st = check_ptrs(P->pageable_ok != 0, buckets, P->n_buckets, "buckets"))) return st;
     if ((st = check_dst(P, dst))) return st;
-    if (R.b1 > R.b0 && !aligned16(checksums))
-        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    if (R.b1 > R.b0 && (st = check_buf(P->pageable_ok != 0, checksums, "checksums"))) return st;
+    if (R.b1 > R.b0 && bad && (st = check_buf(P->pageable_ok != 0, bad, "bad", false))) return st;
     return RR_OK;
 }
 
 rr_status unpack_verify_impl(const rr_plan* P, Range R, const void* const* buckets,
                              const uint64_t* checksums, void* const* dst, uint8_t* bad,
                              int64_t* n_bad, int64_t* first_bad, cudaStream_t stream) {
-    rr_status st = check_unpack_verify_args(P, R, buckets, checksums, dst);
+    rr_status st = check_unpack_verify_args(P, R, buckets, checksums, dst, bad);
     if (st) return st;
     if (n_bad) *n_bad = 0;
     if (first_bad) *first_bad = -1;
@@ -1534,9 +1577,9 @@ rr_status verify_impl(const rr_plan* P, Range R, const void* const* buckets,
                       const uint64_t* checksums, uint8_t* bad, int64_t* n_bad, int64_t* first_bad,
                       cudaStream_t stream) {
     rr_status st;
-    if ((st = check_ptrs(buckets, P->n_buckets, "buckets"))) return st;
-    if (R.b1 > R.b0 && !aligned16(checksums))
-        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    if ((st = check_ptrs(P->pageable_ok != 0, buckets, P->n_buckets, "buckets"))) return st;
+    if (R.b1 > R.b0 && (st = check_buf(P->pageable_ok != 0, checksums, "checksums"))) return st;
+    if (R.b1 > R.b0 && bad && (st = check_buf(P->pageable_ok != 0, bad, "bad", false))) return st;
     if (n_bad) *n_bad = 0;
     if (first_bad) *first_bad = -1;
     if (R.b1 == R.b0) return RR_OK;
@@ -1590,6 +1633,9 @@ rr_status rr_device_default_grid(rr_grids* g) {
 
 rr_status rr_device_upload(rr_plan* P) {
     RR_CUDA(cudaGetDevice(&P->device));
+    int pageable = 0;
+    RR_CUDA(cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, P->device));
+    P->pageable_ok = pageable;
     auto up = [](void** d, const void* h, size_t bytes) -> cudaError_t {
         cudaError_t e = cudaMalloc(d, bytes ? bytes : 16);
         if (e != cudaSuccess) return e;
@@ -1767,7 +1813,7 @@ extern "C" rr_status rr_unpack_verify_async(const rr_plan* P, int32_t first_buck
     Range R;
     rr_status st = check_plan(P);
     if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
-    if ((st = check_unpack_verify_args(P, R, buckets, checksums, dst))) return st;
+    if ((st = check_unpack_verify_args(P, R, buckets, checksums, dst, bad))) return st;
     long long* res = result_address(result);
     if (!res)
         return rr_fail(RR_EINVAL, "result must be 8-byte aligned device or pinned host memory");
@@ -1810,7 +1856,7 @@ extern "C" rr_status rr_clear_range(const rr_plan* P, int32_t first_bucket, int3
     Range R;
     rr_status st = check_plan(P);
     if (st || (st = check_range(P, first_bucket, n_buckets, &R))) return st;
-    if ((st = check_ptrs((const void* const*)buckets, P->n_buckets, "buckets"))) return st;
+    if ((st = check_ptrs(P->pageable_ok != 0, (const void* const*)buckets, P->n_buckets, "buckets"))) return st;
     if (n_buckets == 0) return RR_OK;
     uint64_t stride = 0;
     if (uniform((const void* const*)buckets, P->n_buckets, P->bucket_bytes, &stride)) {
@@ -1917,10 +1963,12 @@ extern "C" rr_status rr_verify_noalloc(const void* const* buckets, int32_t n_buc
                        kStaticVerifyMaxBuckets, n_buckets);
     if (bucket_bytes < 8 || bucket_bytes % 8 != 0 || bucket_bytes > (size_t(1) << 32) - 16)
         return rr_fail(RR_EINVAL, "bucket_bytes must be a multiple of 8 in [8, 2^32 - 16]");
-    rr_status st = check_ptrs(buckets, n_buckets, "buckets");
+    int dev = 0, pageable = 0;
+    RR_CUDA(cudaGetDevice(&dev));
+    RR_CUDA(cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, dev));
+    rr_status st = check_ptrs(pageable != 0, buckets, n_buckets, "buckets");
     if (st) return st;
-    if (n_buckets > 0 && !aligned16(checksums))
-        return rr_fail(RR_EINVAL, "checksums NULL or not 16-byte aligned");
+    if (n_buckets > 0 && (st = check_buf(pageable != 0, checksums, "checksums"))) return st;
     if (n_bad) *n_bad = 0;
     if (first_bad) *first_bad = -1;
     if (n_buckets == 0) return RR_OK;

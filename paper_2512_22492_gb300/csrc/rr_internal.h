@@ -79,6 +79,7 @@ struct rr_plan {
     unsigned long long* d_pack_weight_prefix = nullptr;
     unsigned long long* d_unpack_weight_prefix = nullptr;
     int32_t check_items = 0;                 // kernels check every item's bounds
+    int32_t pageable_ok = 0;                 // the device can read pageable host memory
     int64_t* d_src_bytes = nullptr;          // check_items: bytes of each source buffer
     int64_t* d_tensor_bytes = nullptr;       //              and of each destination tensor
     rr_unpack_item* d_unpack_items = nullptr;

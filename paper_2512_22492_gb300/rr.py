@@ -485,6 +485,8 @@ def _check_list(xs, n: int, min_bytes, what: str, plan: Optional[Plan] = None) -
     if hasattr(xs, "dim") and xs.dim() == 2:
         if xs.shape[0] != n:
             raise ValueError(f"{what}: {xs.shape[0]} rows, plan expects {n}")
+        if xs.shape[0] > 1 and (xs.stride(1) != 1 or xs.stride(0) < xs.shape[1]):
+            raise ValueError(f"{what}: rows must be contiguous and must not overlap")
         if min_bytes is not None and xs.shape[1] * xs.element_size() < min_bytes:
             raise ValueError(f"{what}: rows of {xs.shape[1] * xs.element_size()} bytes, plan "
                              f"needs {min_bytes}")
@@ -493,6 +495,9 @@ def _check_list(xs, n: int, min_bytes, what: str, plan: Optional[Plan] = None) -
     if len(xs) != n:
         raise ValueError(f"{what}: {len(xs)} entries, plan expects {n}")
     for i, x in enumerate(xs):
+        if hasattr(x, "is_contiguous") and not x.is_contiguous():
+            raise ValueError(f"{what}[{i}]: not contiguous (the library writes and reads its "
+                             f"bytes in order)")
         need = min_bytes(i) if callable(min_bytes) else min_bytes
         nb = _nbytes(x)
         if nb is not None and need is not None and nb < need:
@@ -540,6 +545,8 @@ class Pointers:
 
 
 def _check_checksums(plan: Plan, checksums) -> None:
+    if hasattr(checksums, "is_contiguous") and not checksums.is_contiguous():
+        raise ValueError("checksums: not contiguous")
     nb = _nbytes(checksums)
     if nb is not None and nb < 8 * plan.n_buckets:
         raise ValueError(f"checksums: {nb} bytes, plan needs {8 * plan.n_buckets}")

@@ -21,9 +21,9 @@ def host_plan(name="tiny-tp4", **kw):
 
 
 def fake_dst(plan, short=None):
-    out = [torch.empty(1, dtype=torch.bfloat16).expand(n) for n in plan.tensor_numel]
+    out = [torch.empty(n, dtype=torch.bfloat16) for n in plan.tensor_numel]
     if short is not None:
-        out[short] = torch.empty(1, dtype=torch.bfloat16).expand(plan.tensor_numel[short] - 1)
+        out[short] = torch.empty(plan.tensor_numel[short] - 1, dtype=torch.bfloat16)
     return out
 
 
@@ -103,3 +103,52 @@ def test_tables_give_the_same_bytes_as_lists():
     for t in range(plan.n_tensors):
         assert torch.equal(a.dst[t], b.dst[t])
     np.testing.assert_array_equal(H.checksums_host(a), H.checksums_host(b))
+
+
+def test_non_contiguous_buffers_are_refused():
+    """A strided view would have the library write past what it shows."""
+    plan = host_plan()
+    dst = fake_dst(plan)
+    wide = torch.empty(2 * plan.tensor_numel[0], dtype=torch.bfloat16)
+    dst[0] = wide[::2]
+    with pytest.raises(ValueError, match="not contiguous"):
+        rr.Pointers(plan, "dst", dst)
+    buckets = torch.empty(plan.bucket_bytes, plan.n_buckets, dtype=torch.uint8).t()
+    with pytest.raises(ValueError, match="contiguous"):
+        rr.rr_verify(plan, buckets, torch.empty(plan.n_buckets, dtype=torch.int64))
+    cs = torch.empty(2 * plan.n_buckets, dtype=torch.int64)[::2]
+    with pytest.raises(ValueError, match="checksums"):
+        rr.rr_verify(plan, torch.empty(plan.n_buckets, plan.bucket_bytes, dtype=torch.uint8), cs)
+
+
+def _pageable_access() -> int:
+    import ctypes
+    from paper_2512_22492_gb300 import build as B
+    from tests.test_c_abi import cudart_dir
+    rt = ctypes.CDLL(cudart_dir(B._cuda_home()) + "/libcudart.so")
+    v = ctypes.c_int(0)
+    assert rt.cudaDeviceGetAttribute(ctypes.byref(v), 88, 0) == 0   # PageableMemoryAccess
+    return v.value
+
+
+@pytest.mark.gpu
+def test_pageable_host_buffers_refused_where_unreadable():
+    """Ordinary (pageable) host memory is refused with RR_EINVAL unless this GPU
+    reads pageable host memory; nothing is launched on it either way."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    if _pageable_access():
+        pytest.skip("this GPU reads pageable host memory: nothing to refuse")
+    from tests import gpu_harness as H
+    from paper_2512_22492_gb300 import rr as rrmod
+    desc = U.workload_desc("tiny-tp4")
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"])
+    buf = H.alloc(plan)
+    host_buckets = torch.zeros(plan.n_buckets, plan.bucket_bytes, dtype=torch.uint8)
+    with pytest.raises(rr.RRError) as e:
+        rr.rr_pack(plan, buf.shards, host_buckets, buf.checksums)
+    assert e.value.status == rrmod.RR_EINVAL
+    with pytest.raises(rr.RRError) as e:
+        rr.rr_verify(plan, buf.buckets, torch.zeros(plan.n_buckets, dtype=torch.int64))
+    assert e.value.status == rrmod.RR_EINVAL
