@@ -1138,8 +1138,8 @@ rr_status check_plan(const rr_plan* P) {
     return RR_OK;
 }
 
-// Whether a kernel of this library may touch memory at p: device (or
-// managed) memory, pinned host memory mapped for the device, or -- on a device
+// Whether a kernel of this library may touch memory at p: the current GPU's
+// device (or managed) memory, pinned host memory mapped for the device, or -- on a device
 // that reads pageable host memory (address translation over the CPU's page
 // tables, as on Grace) -- any host memory.  Pageable memory elsewhere would
 // fault the GPU, so it is refused.
@@ -1149,7 +1149,11 @@ bool reachable(const void* p, bool pageable_ok) {
         cudaGetLastError();
         return pageable_ok;
     }
-    if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) return true;
+    if (at.type == cudaMemoryTypeDevice) {   // this GPU's own memory only
+        int dev = -1;
+        return cudaGetDevice(&dev) == cudaSuccess && at.device == dev;
+    }
+    if (at.type == cudaMemoryTypeManaged) return true;
     if (at.type == cudaMemoryTypeHost) return at.devicePointer != nullptr;
     return pageable_ok;
 }
@@ -1164,8 +1168,8 @@ rr_status check_ptrs(bool pageable_ok, const void* const* ptrs, int32_t n, const
     for (int32_t i : {0, n - 1})
         if (n > 0 && !reachable(ptrs[i], pageable_ok))
             return rr_fail(RR_EINVAL,
-                           "%s[%d] is host memory this GPU cannot read (pageable); use device "
-                           "memory or pinned host memory",
+                           "%s[%d] is memory this GPU cannot reach (pageable host memory, or "
+                           "another GPU's); use this GPU's memory or pinned host memory",
                            what, i);
     return RR_OK;
 }
@@ -1177,8 +1181,8 @@ rr_status check_buf(bool pageable_ok, const void* p, const char* what, bool alig
         return rr_fail(RR_EINVAL, "%s NULL or not 16-byte aligned", what);
     if (!reachable(p, pageable_ok))
         return rr_fail(RR_EINVAL,
-                       "%s is host memory this GPU cannot read (pageable); use device memory "
-                       "or pinned host memory", what);
+                       "%s is memory this GPU cannot reach (pageable host memory, or another "
+                       "GPU's); use this GPU's memory or pinned host memory", what);
     return RR_OK;
 }
 
@@ -1450,8 +1454,8 @@ rr_status check_dst(const rr_plan* P, void* const* dst) {
     for (int32_t t : {0, P->n_tensors - 1})
         if (P->n_tensors > 0 && P->tensor_numel[t] > 0 && !reachable(dst[t], P->pageable_ok != 0))
             return rr_fail(RR_EINVAL,
-                           "dst[%d] is host memory this GPU cannot read (pageable); use device "
-                           "memory or pinned host memory",
+                           "dst[%d] is memory this GPU cannot reach (pageable host memory, or "
+                           "another GPU's); use this GPU's memory or pinned host memory",
                            t);
     return RR_OK;
 }
