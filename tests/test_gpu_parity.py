@@ -162,6 +162,14 @@ def test_bulk_engine_piece_splits(chunk):
     full_parity(U.workload_desc("tiny-moe-f32", bucket_bytes=256 * 1024), chunk_bytes=chunk)
 
 
+def test_largest_bucket_size():
+    """One bucket of the largest size the ABI takes, 2^32 - 16 bytes: the tiny
+    model's stream at its start and zeros to its end, so the tail's items sit at
+    offsets just under 2^32.  Compared in full with the oracle (4 GiB)."""
+    full_parity(U.workload_desc("tiny", bucket_bytes=(1 << 32) - 16))
+    torch.cuda.empty_cache()
+
+
 @pytest.mark.parametrize("grid", [1, 3, 1000])
 def test_grid_sizes(grid):
     full_parity(U.workload_desc("tiny-moe-tp2"), grid_blocks=grid)
