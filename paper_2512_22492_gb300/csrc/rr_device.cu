@@ -1192,6 +1192,7 @@ struct Range {
     int32_t b0, b1;
     bool full;
     unsigned long long* scratch;   // verify sums and counters of this call (NULL: the plan's)
+    int32_t t_lo, t_hi;            // unpack: the destination tensors its pointer table holds
 };
 
 // The bounds the kernels check items against, when the plan asks for checks.
@@ -1266,8 +1267,8 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
         a.bucket_base = (const char*)buckets[0];
         a.bucket_stride = stride;
     }
-    a.dst_base = k;
-    for (int32_t t = 0; t < P->n_tensors; ++t) a.ptr[k++] = dst[t];
+    a.dst_base = k - R.t_lo;   // ptr[dst_base + tensor] for tensors t_lo .. t_hi
+    for (int32_t t = R.t_lo; t <= R.t_hi; ++t) a.ptr[k++] = dst[t];
     if (checksums && P->check_items)
         rr_unpack_kernel<NPTR, true, true><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
     else if (checksums)
@@ -1287,8 +1288,9 @@ rr_status launch_verify(const rr_plan* P, Range R, const void* const* buckets,
     VerifyArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     const int32_t n = R.b1 - R.b0;
-    a.sums = P->d_verify_scratch;
-    a.counters = P->d_verify_scratch + n;
+    unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
+    a.sums = sc;
+    a.counters = sc + n;
     a.expected = (const unsigned long long*)checksums;
     a.bad = bad;
     a.first_bucket = R.b0;
@@ -1372,8 +1374,8 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         a.bucket_stride = stride;
     }
     if (MODE != 0) {
-        a.dst_base = k;
-        for (int32_t t = 0; t < P->n_tensors; ++t) a.ptr[k++] = dst[t];
+        a.dst_base = k - R.t_lo;   // ptr[dst_base + tensor] for tensors t_lo .. t_hi
+        for (int32_t t = R.t_lo; t <= R.t_hi; ++t) a.ptr[k++] = dst[t];
     }
     const int32_t grid = MODE == 0 ? P->grid_blocks : P->unpack_grid_blocks;
     if (P->check_items) {
@@ -1460,15 +1462,79 @@ rr_status check_dst(const rr_plan* P, void* const* dst) {
     return RR_OK;
 }
 
-template <class F>
-rr_status with_unpack_shape(const rr_plan* P, const void* const* buckets, F launch) {
-    uint64_t stride = 0;
-    const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
-    const int32_t need = P->n_tensors + (table ? P->n_buckets : 0);
-    if (need > kLargePtrs)
-        return rr_fail(RR_EINVAL, "%d tensors + %d separately allocated buckets exceed %d pointers",
-                       P->n_tensors, P->n_buckets, kLargePtrs);
-    return launch(need <= kSmallPtrs, table, stride);
+// The sub-ranges of R that unpack launches take: runs of buckets whose
+// destination-tensor window, with the bucket pointers of a table launch, fits
+// one launch's pointer table.  Usually R itself.
+rr_status unpack_windows(const rr_plan* P, Range R, int32_t extra, std::vector<Range>* out) {
+    const int32_t cap = kLargePtrs - extra;
+    out->clear();
+    for (int32_t b = R.b0; b < R.b1;) {
+        int32_t lo = INT32_MAX, hi = -1, e = b;
+        for (; e < R.b1; ++e) {
+            const int32_t nlo = std::min(lo, P->bucket_tensor_lo[e]);
+            const int32_t nhi = std::max(hi, P->bucket_tensor_hi[e]);
+            if (nhi >= nlo && nhi - nlo + 1 > cap) break;
+            lo = nlo;
+            hi = nhi;
+        }
+        if (e == b)
+            return rr_fail(RR_EINVAL,
+                           "bucket %d writes %d destination tensors; one launch addresses at "
+                           "most %d (with %d bucket pointers)",
+                           b, P->bucket_tensor_hi[b] - P->bucket_tensor_lo[b] + 1, cap, extra);
+        if (hi < lo) lo = 0, hi = -1;   // gap and tail bytes only
+        out->push_back(Range{b, e, R.full && b == R.b0 && e == R.b1, R.scratch, lo, hi});
+        b = e;
+    }
+    return RR_OK;
+}
+
+// How one unpack-type call addresses its buffers, and the sub-ranges it is
+// launched over.
+struct UnpackShape {
+    bool table;              // buckets through the pointer table (not equally spaced)
+    uint64_t stride;         // otherwise bucket b at buckets[0] + b * stride
+    int32_t extra;           // pointer-table entries the buckets take
+    std::vector<Range> parts;
+};
+
+rr_status unpack_shape(const rr_plan* P, Range R, const void* const* buckets, UnpackShape* sh) {
+    sh->stride = 0;
+    sh->table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &sh->stride);
+    sh->extra = sh->table ? P->n_buckets : 0;
+    if (sh->extra >= kLargePtrs)
+        return rr_fail(RR_EINVAL, "%d separately allocated buckets exceed %d pointers; allocate "
+                                  "the buckets as one equally spaced block",
+                       P->n_buckets, kLargePtrs);
+    return unpack_windows(P, R, sh->extra, &sh->parts);
+}
+
+// One unpack launch (MODE 1, or 2 when checksums are given) over sub-range S,
+// on the bulk engine or the register path.
+rr_status launch_unpack_part(const rr_plan* P, const Range& S, bool bulk,
+                             const void* const* buckets, void* const* dst,
+                             const uint64_t* checksums, uint8_t* bad, const UnpackShape& sh,
+                             cudaStream_t stream) {
+    const bool small = (S.t_hi - S.t_lo + 1) + sh.extra <= kSmallPtrs;
+    if (bulk) {
+        if (checksums)
+            return small ? launch_bulk<kSmallPtrs, 2>(P, S, nullptr, buckets, dst, checksums, bad,
+                                                      sh.table, sh.stride, stream)
+                         : launch_bulk<kLargePtrs, 2>(P, S, nullptr, buckets, dst, checksums, bad,
+                                                      sh.table, sh.stride, stream);
+        return small ? launch_bulk<kSmallPtrs, 1>(P, S, nullptr, buckets, dst, nullptr, nullptr,
+                                                  sh.table, sh.stride, stream)
+                     : launch_bulk<kLargePtrs, 1>(P, S, nullptr, buckets, dst, nullptr, nullptr,
+                                                  sh.table, sh.stride, stream);
+    }
+    // The register path's balanced split is the plan's only when it was made for
+    // the register grid.
+    Range Sr = S;
+    Sr.full = S.full && P->engine == RR_ENGINE_REGISTERS;
+    return small ? launch_unpack<kSmallPtrs>(P, Sr, buckets, dst, checksums, bad, sh.table,
+                                             sh.stride, stream)
+                 : launch_unpack<kLargePtrs>(P, Sr, buckets, dst, checksums, bad, sh.table,
+                                             sh.stride, stream);
 }
 
 rr_status unpack_impl(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
@@ -1479,18 +1545,12 @@ rr_status unpack_impl(const rr_plan* P, Range R, const void* const* buckets, voi
     if (P->unpack_bucket_first[R.b0] == P->unpack_bucket_first[R.b1]) return RR_OK;
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
                       all_device((const void* const*)dst, P->n_tensors);
-    const Range Rr{R.b0, R.b1, R.full && !bulk && P->engine == RR_ENGINE_REGISTERS};
-    return with_unpack_shape(P, buckets, [&](bool small, bool table, uint64_t stride) {
-        if (bulk)
-            return small ? launch_bulk<kSmallPtrs, 1>(P, R, nullptr, buckets, dst, nullptr, nullptr,
-                                                      table, stride, stream)
-                         : launch_bulk<kLargePtrs, 1>(P, R, nullptr, buckets, dst, nullptr, nullptr,
-                                                      table, stride, stream);
-        return small ? launch_unpack<kSmallPtrs>(P, Rr, buckets, dst, nullptr, nullptr, table,
-                                                 stride, stream)
-                     : launch_unpack<kLargePtrs>(P, Rr, buckets, dst, nullptr, nullptr, table,
-                                                 stride, stream);
-    });
+    UnpackShape sh;
+    if ((st = unpack_shape(P, R, buckets, &sh))) return st;
+    for (const Range& S : sh.parts)
+        if ((st = launch_unpack_part(P, S, bulk, buckets, dst, nullptr, nullptr, sh, stream)))
+            return st;
+    return RR_OK;
 }
 
 rr_status read_error(const rr_plan* P, cudaStream_t stream);
@@ -1508,27 +1568,30 @@ rr_status read_result(const rr_plan* P, int32_t n, int64_t* n_bad, int64_t* firs
 }
 
 // Enqueues the verifying unpack of range R: zeroes the range's sums and
-// counters (R.scratch, else the plan's) and launches the kernel.
+// counters (R.scratch, else the plan's), then one fused launch -- or, when the
+// range's destination tensors need several launches, plain unpack launches
+// followed by one checksum pass over the whole range.
 rr_status enqueue_unpack_verify(const rr_plan* P, Range R, const void* const* buckets,
                                 const uint64_t* checksums, void* const* dst, uint8_t* bad,
                                 cudaStream_t stream) {
     const int32_t n = R.b1 - R.b0;
     unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
+    UnpackShape sh;
+    rr_status st = unpack_shape(P, R, buckets, &sh);
+    if (st) return st;
     RR_CUDA(cudaMemsetAsync(sc, 0, (size_t(n) + 4) * sizeof(unsigned long long), stream));
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
                       all_device((const void* const*)dst, P->n_tensors);
-    const Range Rr{R.b0, R.b1, R.full && !bulk && P->engine == RR_ENGINE_REGISTERS, R.scratch};
-    return with_unpack_shape(P, buckets, [&](bool small, bool table, uint64_t stride) {
-        if (bulk)
-            return small ? launch_bulk<kSmallPtrs, 2>(P, R, nullptr, buckets, dst, checksums, bad,
-                                                      table, stride, stream)
-                         : launch_bulk<kLargePtrs, 2>(P, R, nullptr, buckets, dst, checksums, bad,
-                                                      table, stride, stream);
-        return small ? launch_unpack<kSmallPtrs>(P, Rr, buckets, dst, checksums, bad, table, stride,
-                                                 stream)
-                     : launch_unpack<kLargePtrs>(P, Rr, buckets, dst, checksums, bad, table, stride,
-                                                 stream);
-    });
+    if (sh.parts.size() == 1)
+        return launch_unpack_part(P, sh.parts[0], bulk, buckets, dst, checksums, bad, sh, stream);
+    for (const Range& S : sh.parts)
+        if ((st = launch_unpack_part(P, S, bulk, buckets, dst, nullptr, nullptr, sh, stream)))
+            return st;
+    return (!sh.table || P->n_buckets <= kSmallPtrs)
+               ? launch_verify<kSmallPtrs>(P, R, buckets, checksums, bad, sh.table, sh.stride,
+                                           stream)
+               : launch_verify<kLargePtrs>(P, R, buckets, checksums, bad, sh.table, sh.stride,
+                                           stream);
 }
 
 rr_status check_unpack_verify_args(const rr_plan* P, Range R, const void* const* buckets,

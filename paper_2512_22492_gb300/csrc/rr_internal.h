@@ -68,6 +68,8 @@ struct rr_plan {
                                                 // empty when it would equal pack_items
     std::vector<uint32_t> full_block_first;     // grid_blocks + 1
     std::vector<uint32_t> unpack_bucket_first;  // n_buckets + 1: first unpack item of bucket b
+    std::vector<int32_t> bucket_tensor_lo;      // n_buckets: lowest / highest destination
+    std::vector<int32_t> bucket_tensor_hi;      //   tensor a bucket's unpack items write
     rr_plan_stats stats{};
 
     // ---- device state (owned) -------------------------------------------

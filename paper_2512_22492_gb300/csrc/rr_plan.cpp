@@ -18,6 +18,7 @@
 // parameter rows for several ranks (row-parallel weights under tensor
 // parallelism) become fan-out groups that read each source row once.
 #include <algorithm>
+#include <climits>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -670,6 +671,15 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     };
     index(P->pack_items, P->pack_bucket_first);
     index(P->unpack_items, P->unpack_bucket_first);
+    // Which destination tensors each bucket's unpack items write (a launch's
+    // pointer table holds only the window of tensors its buckets need).
+    P->bucket_tensor_lo.assign(size_t(P->n_buckets), INT32_MAX);
+    P->bucket_tensor_hi.assign(size_t(P->n_buckets), -1);
+    for (const rr_unpack_item& it : P->unpack_items) {
+        if (it.kind != RR_ITEM_COPY_VEC && it.kind != RR_ITEM_COPY_SCALAR) continue;
+        P->bucket_tensor_lo[it.bucket] = std::min(P->bucket_tensor_lo[it.bucket], int32_t(it.tensor));
+        P->bucket_tensor_hi[it.bucket] = std::max(P->bucket_tensor_hi[it.bucket], int32_t(it.tensor));
+    }
     partition(P->pack_items, P->grid_blocks, P->pack_block_first, pack_weight);
     partition(P->unpack_items, P->unpack_grid_blocks, P->unpack_block_first, unpack_weight);
     // Summed weights: a bucket-range call splits its items over the grid by them.

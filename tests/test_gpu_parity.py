@@ -162,6 +162,64 @@ def test_bulk_engine_piece_splits(chunk):
     full_parity(U.workload_desc("tiny-moe-f32", bucket_bytes=256 * 1024), chunk_bytes=chunk)
 
 
+def many_tensors_desc(n_tensors, bucket_bytes, tp=1):
+    """A parameter of n_tensors rows, each row its own destination tensor."""
+    return dict(params=[("p", (n_tensors, 16), 2), ("q", (5, 24), 4)],
+                tensors=[(f"t{i}", i % tp, [(0, i, 1, 0, 16)]) for i in range(n_tensors)] +
+                        [("q", 0, [(1, 0, 5, 0, 24)])],
+                tp=tp, sharding="flat", n_shards=3, bucket_bytes=bucket_bytes, align_bytes=16,
+                tensor_align=256, seed=31, specials=True)
+
+
+@pytest.mark.parametrize("engine", ["auto", "registers"])
+def test_more_destination_tensors_than_one_launch_addresses(engine):
+    """9001 destination tensors: more than one launch's pointer table holds, so
+    unpack runs as several launches over bucket ranges whose tensors fit, and
+    the verifying forms add one checksum pass.  Full calls, ranges, the async
+    form and separately allocated buckets."""
+    desc = many_tensors_desc(9000, 64 * 1024)
+    full_parity(desc, engine=engine)
+    full_parity(desc, separate_buckets=True, engine=engine)
+    L = U.to_oracle(desc)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"], engine=engine)
+    buf = H.alloc(plan)
+    shards = L.host_shards(desc["seed"], desc["specials"])
+    H.fill_from_host(buf, shards)
+    H.pack(buf)
+    H.bucket_list(buf)[20][0] ^= 0x04
+    assert rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst,
+                               first_bucket=3, n_buckets=30) == (1, 20)
+    res = torch.zeros(2, dtype=torch.int64, device="cuda")
+    scratch = torch.zeros(plan.n_buckets + 4, dtype=torch.int64, device="cuda")
+    rr.rr_unpack_verify_async(plan, buf.buckets, buf.checksums, buf.dst, scratch, res)
+    torch.cuda.synchronize()
+    assert res.cpu().tolist() == [1, 20]
+    H.bucket_list(buf)[20][0] ^= 0x04
+    for x in buf.dst:
+        x.fill_(0)
+    rr.rr_unpack_range(plan, 0, plan.n_buckets, buf.buckets, buf.dst)
+    torch.cuda.synchronize()
+    gen = oracle.Source(shards=shards)
+    for t_ in (0, 1, 4000, 8999, 9000):
+        np.testing.assert_array_equal(H.tensor_host(buf, t_), L.reshard_tensor(gen, t_))
+
+
+def test_bucket_writing_too_many_tensors_is_refused():
+    """One bucket that alone writes more tensors than a launch addresses: pack
+    works, unpack is refused with RR_EINVAL before anything is launched."""
+    desc = many_tensors_desc(8192, 2 << 20)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"])
+    buf = H.alloc(plan)
+    H.fill_from_host(buf, U.to_oracle(desc).host_shards(desc["seed"], desc["specials"]))
+    H.pack(buf)
+    assert H.verify(buf) == (0, -1)
+    with pytest.raises(rr.RRError) as e:
+        H.unpack(buf)
+    assert e.value.status == rrmod.RR_EINVAL
+
+
 def test_largest_bucket_size():
     """One bucket of the largest size the ABI takes, 2^32 - 16 bytes: the tiny
     model's stream at its start and zeros to its end, so the tail's items sit at
