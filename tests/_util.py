@@ -115,6 +115,20 @@ def random_tp_layout(seed: int):
     return desc
 
 
+def degenerate_layout(sharding: str = "flat"):
+    """Parameters with a zero dimension, empty blocks, and destination tensors
+    with no elements at all, among ordinary ones."""
+    desc = dict(params=[("a", (0, 8), 4), ("b", (3, 0), 2), ("c", (5, 16), 4), ("d", (0,), 2)],
+                tensors=[("t0", 0, [(0, 0, 0, 0, 8), (2, 1, 2, 0, 16)]),
+                         ("t1", 1, [(1, 0, 3, 0, 0)]),
+                         ("t2", 1, [(2, 0, 5, 3, 8), (3, 0, 0, 0, 1)]), ("t3", 0, [])],
+                tp=2, sharding=sharding, n_shards=3, bucket_bytes=64, align_bytes=16,
+                tensor_align=256, seed=5, specials=True)
+    if sharding == "units":
+        desc["units"] = [0, 1, 0, 1]
+    return desc
+
+
 def workload_desc(name, bucket_bytes=None):
     w = workload(name)
     from oracle import qwen3

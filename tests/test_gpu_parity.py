@@ -220,6 +220,13 @@ def test_bucket_writing_too_many_tensors_is_refused():
     assert e.value.status == rrmod.RR_EINVAL
 
 
+@pytest.mark.parametrize("sharding", ["flat", "rows", "units"])
+@pytest.mark.parametrize("engine", ["auto", "registers"])
+def test_degenerate_layout(sharding, engine):
+    """Zero-size parameters, empty blocks and empty tensors."""
+    full_parity(U.degenerate_layout(sharding), engine=engine)
+
+
 def test_largest_bucket_size():
     """One bucket of the largest size the ABI takes, 2^32 - 16 bytes: the tiny
     model's stream at its start and zeros to its end, so the tail's items sit at

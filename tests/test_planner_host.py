@@ -116,6 +116,13 @@ def test_random_row_parallel_layouts_exercise_fan_out():
     assert heads > 100 and plain_rows > 3
 
 
+@pytest.mark.parametrize("sharding", ["flat", "rows", "units"])
+def test_degenerate_layout(sharding):
+    """Zero-size parameters, empty blocks and empty tensors."""
+    p, _ = run_and_compare(U.degenerate_layout(sharding), grid_blocks=3)
+    assert p.tensor_numel == [32, 0, 40, 0]
+
+
 def test_vector_items_dominate_on_aligned_workloads():
     p, items = run_and_compare(U.workload_desc("tiny"))
     data = items[items["kind"] <= U.ITEM_BF16_SCALAR]
