@@ -82,10 +82,10 @@ struct PackArgs {
     ItemBounds chk;
     unsigned long long* checksums;
     char* bucket_base;        // equally spaced buckets: base + b * stride
-    uint64_t bucket_stride;   // 0: bucket b is ptr[n_shards + b]
+    uint64_t bucket_stride;   // 0: bucket b is ptr[n_shards + b - bucket_lo]
     int32_t n_shards;
-    int32_t pad;
-    const void* ptr[NPTR];    // shards, then (table mode) buckets
+    int32_t bucket_lo;        // table mode: the first bucket the table holds
+    const void* ptr[NPTR];    // shards, then (table mode) buckets bucket_lo, ...
 };
 
 template <int NPTR>
@@ -107,8 +107,8 @@ struct UnpackArgs {
     const char* bucket_base;
     uint64_t bucket_stride;
     int32_t dst_base;         // index in ptr[] of destination tensor 0
-    int32_t pad;
-    const void* ptr[NPTR];    // (table mode) buckets, then destination tensors
+    int32_t bucket_lo;        // table mode: the first bucket the table holds
+    const void* ptr[NPTR];    // (table mode) buckets bucket_lo, ..., then destination tensors
 };
 
 template <int NPTR>
@@ -118,7 +118,7 @@ struct VerifyArgs {
     const unsigned long long* expected;   // indexed by global bucket
     uint8_t* bad;                   // optional [n_buckets]: 1 where the sum differs
     int32_t first_bucket;           // the range checked is [first_bucket, +n_buckets)
-    int32_t pad0;
+    int32_t bucket_lo;              // table mode: the first bucket the table holds
     const char* bucket_base;
     uint64_t bucket_stride;
     uint64_t bucket_bytes;
@@ -288,7 +288,7 @@ __device__ __forceinline__ void block_items(const uint32_t* block_first,
 template <int NPTR>
 __device__ __forceinline__ char* bucket_of(const PackArgs<NPTR>& a, uint32_t b) {
     return a.bucket_stride ? a.bucket_base + (uint64_t)b * a.bucket_stride
-                           : (char*)a.ptr[a.n_shards + b];
+                           : (char*)a.ptr[a.n_shards + (b - a.bucket_lo)];
 }
 
 // ---------------------------------------------------------------------------
@@ -470,7 +470,8 @@ __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_con
             acc = 0;
         }
         const char* src = (a.bucket_stride ? a.bucket_base + (uint64_t)d.bucket * a.bucket_stride
-                                           : (const char*)a.ptr[d.bucket]) + d.src_off;
+                                           : (const char*)a.ptr[d.bucket - a.bucket_lo]) +
+                          d.src_off;
         const bool copy = d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_COPY_SCALAR;
         char* dst = copy ? (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off : nullptr;
         if (d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_READ_VEC) {
@@ -524,7 +525,7 @@ __global__ void __launch_bounds__(kThreads, 4) rr_verify_kernel(const __grid_con
         }
         const uint32_t b = a.first_bucket + bl;
         const char* p = (a.bucket_stride ? a.bucket_base + (uint64_t)b * a.bucket_stride
-                                         : (const char*)a.ptr[b]) + off;
+                                         : (const char*)a.ptr[b - a.bucket_lo]) + off;
         const uint32_t nvec = (uint32_t)(len >> 4);
         for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * kUnroll) {
             uint4 x[kUnroll];
@@ -628,6 +629,8 @@ struct BulkArgs {
     uint64_t bucket_stride;
     int32_t n_shards;            // pack: ptr[0 .. n_shards) are the shards
     int32_t dst_base;            // unpack: index in ptr[] of destination tensor 0
+    int32_t bucket_lo;           // table mode: the first bucket the table holds
+    int32_t pad_;
     unsigned long long* sums;    // pack: checksums by bucket; verify: range sums
     unsigned long long* counters;
     const unsigned long long* expected;
@@ -705,7 +708,7 @@ __device__ __forceinline__ void gather_async(uint32_t stage, uint32_t full_bar, 
 template <int NPTR>
 __device__ __forceinline__ char* bulk_bucket(const BulkArgs<NPTR>& a, uint32_t b, int table_base) {
     return a.bucket_stride ? a.bucket_base + (uint64_t)b * a.bucket_stride
-                           : (char*)a.ptr[table_base + b];
+                           : (char*)a.ptr[table_base + (b - a.bucket_lo)];
 }
 
 // MODE 0: pack, 1: unpack, 2: unpack with checksum comparison.  CHECK: check
@@ -1193,7 +1196,21 @@ struct Range {
     bool full;
     unsigned long long* scratch;   // verify sums and counters of this call (NULL: the plan's)
     int32_t t_lo, t_hi;            // unpack: the destination tensors its pointer table holds
+    int32_t sum_b0, sum_n;         // verify: the whole call's range (sums, flags, counters);
+                                   // sum_n == 0: this range itself
 };
+
+// Where range S's sums, counters and flags live in its call's scratch.
+struct SumSlot {
+    unsigned long long* sums;
+    unsigned long long* counters;
+    uint8_t* bad;
+};
+SumSlot sum_slot(const rr_plan* P, const Range& S, uint8_t* bad) {
+    unsigned long long* sc = S.scratch ? S.scratch : P->d_verify_scratch;
+    const int32_t b0 = S.sum_n ? S.sum_b0 : S.b0, n = S.sum_n ? S.sum_n : S.b1 - S.b0;
+    return {sc + (S.b0 - b0), sc + n, bad ? bad + (S.b0 - b0) : nullptr};
+}
 
 // The bounds the kernels check items against, when the plan asks for checks.
 ItemBounds bounds_of(const rr_plan* P) {
@@ -1225,7 +1242,8 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
     a.n_shards = P->n_shards;
     for (int32_t i = 0; i < P->n_shards; ++i) a.ptr[i] = src[i];
     if (table) {
-        for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[P->n_shards + b] = buckets[b];
+        a.bucket_lo = R.b0;
+        for (int32_t b = R.b0; b < R.b1; ++b) a.ptr[P->n_shards + (b - R.b0)] = buckets[b];
     } else {
         a.bucket_base = (char*)buckets[0];
         a.bucket_stride = stride;
@@ -1252,17 +1270,18 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     a.item_begin = P->unpack_bucket_first[R.b0];
     a.item_end = P->unpack_bucket_first[R.b1];
     if (checksums) {
-        unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
-        a.sums = sc;
-        a.counters = sc + (R.b1 - R.b0);
+        const SumSlot q = sum_slot(P, R, bad);
+        a.sums = q.sums;
+        a.counters = q.counters;
         a.expected = (const unsigned long long*)checksums;
-        a.bad = bad;
+        a.bad = q.bad;
         a.first_bucket = R.b0;
         a.n_buckets = R.b1 - R.b0;
     }
     int32_t k = 0;
     if (table) {
-        for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[k++] = buckets[b];
+        a.bucket_lo = R.b0;
+        for (int32_t b = R.b0; b < R.b1; ++b) a.ptr[k++] = buckets[b];
     } else {
         a.bucket_base = (const char*)buckets[0];
         a.bucket_stride = stride;
@@ -1288,11 +1307,11 @@ rr_status launch_verify(const rr_plan* P, Range R, const void* const* buckets,
     VerifyArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     const int32_t n = R.b1 - R.b0;
-    unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
-    a.sums = sc;
-    a.counters = sc + n;
+    const SumSlot q = sum_slot(P, R, bad);
+    a.sums = q.sums;
+    a.counters = q.counters;
     a.expected = (const unsigned long long*)checksums;
-    a.bad = bad;
+    a.bad = q.bad;
     a.first_bucket = R.b0;
     a.bucket_bytes = (uint64_t)P->bucket_bytes;
     a.chunk_bytes = (uint64_t)std::min<int64_t>(kVerifyChunk, P->bucket_bytes);
@@ -1300,7 +1319,8 @@ rr_status launch_verify(const rr_plan* P, Range R, const void* const* buckets,
     a.total_chunks = a.chunks_per_bucket * (uint64_t)n;
     a.n_buckets = n;
     if (table) {
-        for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[b] = buckets[b];
+        a.bucket_lo = R.b0;
+        for (int32_t b = R.b0; b < R.b1; ++b) a.ptr[b - R.b0] = buckets[b];
     } else {
         a.bucket_base = (const char*)buckets[0];
         a.bucket_stride = stride;
@@ -1358,17 +1378,18 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         a.item_begin = P->unpack_bucket_first[R.b0];
         a.item_end = P->unpack_bucket_first[R.b1];
         if (MODE == 2) {
-            unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
-            a.sums = sc;
-            a.counters = sc + (R.b1 - R.b0);
+            const SumSlot q = sum_slot(P, R, bad);
+            a.sums = q.sums;
+            a.counters = q.counters;
             a.expected = (const unsigned long long*)checksums;
-            a.bad = bad;
+            a.bad = q.bad;
             a.first_bucket = R.b0;
             a.n_buckets = R.b1 - R.b0;
         }
     }
-    if (table) {
-        for (int32_t b = 0; b < P->n_buckets; ++b) a.ptr[k++] = buckets[b];
+    if (table) {   // the range's buckets (a full-range pack: all of them, for fan-out items)
+        a.bucket_lo = R.b0;
+        for (int32_t b = R.b0; b < R.b1; ++b) a.ptr[k++] = buckets[b];
     } else {
         a.bucket_base = (char*)buckets[0];
         a.bucket_stride = stride;
@@ -1426,26 +1447,41 @@ rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, vo
     if ((st = check_buf(P->pageable_ok != 0, checksums, "checksums"))) return st;
     uint64_t stride = 0;
     const bool table = !uniform((const void* const*)buckets, P->n_buckets, P->bucket_bytes, &stride);
-    const int32_t need = P->n_shards + (table ? P->n_buckets : 0);
-    if (need > kLargePtrs)
+    // Separately allocated buckets go through the pointer table after the
+    // shards: a range with more of them than fit runs as several launches
+    // over consecutive bucket ranges (on the bucket-sorted table).
+    const int32_t cap = kLargePtrs - P->n_shards;
+    if (table && cap < 1)
         return rr_fail(RR_EINVAL,
-                       "%d shards + %d separately allocated buckets exceed %d pointers; allocate "
-                       "the buckets as one equally spaced block",
-                       P->n_shards, P->n_buckets, kLargePtrs);
+                       "%d source buffers leave no room for separately allocated buckets in one "
+                       "launch's %d pointers; allocate the buckets as one equally spaced block",
+                       P->n_shards, kLargePtrs);
     RR_CUDA(cudaMemsetAsync(checksums + R.b0, 0, size_t(R.b1 - R.b0) * 8, stream));
     if (P->pack_bucket_first[R.b0] == P->pack_bucket_first[R.b1]) return RR_OK;
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(src_shards, P->n_shards) &&
                       all_device((const void* const*)buckets, P->n_buckets);
-    if (bulk)
-        return need <= kSmallPtrs
-                   ? launch_bulk<kSmallPtrs, 0>(P, R, src_shards, (const void* const*)buckets,
-                                                nullptr, checksums, nullptr, table, stride, stream)
-                   : launch_bulk<kLargePtrs, 0>(P, R, src_shards, (const void* const*)buckets,
-                                                nullptr, checksums, nullptr, table, stride, stream);
-    const Range Rr{R.b0, R.b1, R.full && P->engine == RR_ENGINE_REGISTERS};
-    return need <= kSmallPtrs
-               ? launch_pack<kSmallPtrs>(P, Rr, src_shards, buckets, checksums, table, stride, stream)
-               : launch_pack<kLargePtrs>(P, Rr, src_shards, buckets, checksums, table, stride, stream);
+    const int32_t step = table ? cap : R.b1 - R.b0;
+    for (int32_t b = R.b0; b < R.b1; b += step) {
+        const int32_t e = std::min(R.b1, b + step);
+        const bool whole = R.full && b == R.b0 && e == R.b1;
+        const Range S{b, e, whole && (bulk || P->engine == RR_ENGINE_REGISTERS)};
+        const int32_t need = P->n_shards + (table ? e - b : 0);
+        if (P->pack_bucket_first[b] == P->pack_bucket_first[e]) continue;
+        if (bulk)
+            st = need <= kSmallPtrs
+                     ? launch_bulk<kSmallPtrs, 0>(P, S, src_shards, (const void* const*)buckets,
+                                                  nullptr, checksums, nullptr, table, stride, stream)
+                     : launch_bulk<kLargePtrs, 0>(P, S, src_shards, (const void* const*)buckets,
+                                                  nullptr, checksums, nullptr, table, stride, stream);
+        else
+            st = need <= kSmallPtrs
+                     ? launch_pack<kSmallPtrs>(P, S, src_shards, buckets, checksums, table, stride,
+                                               stream)
+                     : launch_pack<kLargePtrs>(P, S, src_shards, buckets, checksums, table, stride,
+                                               stream);
+        if (st) return st;
+    }
+    return RR_OK;
 }
 
 rr_status check_dst(const rr_plan* P, void* const* dst) {
@@ -1465,25 +1501,26 @@ rr_status check_dst(const rr_plan* P, void* const* dst) {
 // The sub-ranges of R that unpack launches take: runs of buckets whose
 // destination-tensor window, with the bucket pointers of a table launch, fits
 // one launch's pointer table.  Usually R itself.
-rr_status unpack_windows(const rr_plan* P, Range R, int32_t extra, std::vector<Range>* out) {
-    const int32_t cap = kLargePtrs - extra;
+rr_status unpack_windows(const rr_plan* P, Range R, bool table, std::vector<Range>* out) {
     out->clear();
     for (int32_t b = R.b0; b < R.b1;) {
         int32_t lo = INT32_MAX, hi = -1, e = b;
         for (; e < R.b1; ++e) {
             const int32_t nlo = std::min(lo, P->bucket_tensor_lo[e]);
             const int32_t nhi = std::max(hi, P->bucket_tensor_hi[e]);
-            if (nhi >= nlo && nhi - nlo + 1 > cap) break;
+            const int32_t need = (table ? e - b + 1 : 0) + (nhi >= nlo ? nhi - nlo + 1 : 0);
+            if (need > kLargePtrs) break;
             lo = nlo;
             hi = nhi;
         }
         if (e == b)
             return rr_fail(RR_EINVAL,
                            "bucket %d writes %d destination tensors; one launch addresses at "
-                           "most %d (with %d bucket pointers)",
-                           b, P->bucket_tensor_hi[b] - P->bucket_tensor_lo[b] + 1, cap, extra);
+                           "most %d pointers",
+                           b, P->bucket_tensor_hi[b] - P->bucket_tensor_lo[b] + 1, kLargePtrs);
         if (hi < lo) lo = 0, hi = -1;   // gap and tail bytes only
-        out->push_back(Range{b, e, R.full && b == R.b0 && e == R.b1, R.scratch, lo, hi});
+        out->push_back(Range{b, e, R.full && b == R.b0 && e == R.b1, R.scratch, lo, hi,
+                             R.b0, R.b1 - R.b0});
         b = e;
     }
     return RR_OK;
@@ -1494,19 +1531,13 @@ rr_status unpack_windows(const rr_plan* P, Range R, int32_t extra, std::vector<R
 struct UnpackShape {
     bool table;              // buckets through the pointer table (not equally spaced)
     uint64_t stride;         // otherwise bucket b at buckets[0] + b * stride
-    int32_t extra;           // pointer-table entries the buckets take
     std::vector<Range> parts;
 };
 
 rr_status unpack_shape(const rr_plan* P, Range R, const void* const* buckets, UnpackShape* sh) {
     sh->stride = 0;
     sh->table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &sh->stride);
-    sh->extra = sh->table ? P->n_buckets : 0;
-    if (sh->extra >= kLargePtrs)
-        return rr_fail(RR_EINVAL, "%d separately allocated buckets exceed %d pointers; allocate "
-                                  "the buckets as one equally spaced block",
-                       P->n_buckets, kLargePtrs);
-    return unpack_windows(P, R, sh->extra, &sh->parts);
+    return unpack_windows(P, R, sh->table, &sh->parts);
 }
 
 // One unpack launch (MODE 1, or 2 when checksums are given) over sub-range S,
@@ -1515,7 +1546,7 @@ rr_status launch_unpack_part(const rr_plan* P, const Range& S, bool bulk,
                              const void* const* buckets, void* const* dst,
                              const uint64_t* checksums, uint8_t* bad, const UnpackShape& sh,
                              cudaStream_t stream) {
-    const bool small = (S.t_hi - S.t_lo + 1) + sh.extra <= kSmallPtrs;
+    const bool small = (S.t_hi - S.t_lo + 1) + (sh.table ? S.b1 - S.b0 : 0) <= kSmallPtrs;
     if (bulk) {
         if (checksums)
             return small ? launch_bulk<kSmallPtrs, 2>(P, S, nullptr, buckets, dst, checksums, bad,
@@ -1568,9 +1599,9 @@ rr_status read_result(const rr_plan* P, int32_t n, int64_t* n_bad, int64_t* firs
 }
 
 // Enqueues the verifying unpack of range R: zeroes the range's sums and
-// counters (R.scratch, else the plan's), then one fused launch -- or, when the
-// range's destination tensors need several launches, plain unpack launches
-// followed by one checksum pass over the whole range.
+// counters (R.scratch, else the plan's), then one fused launch per sub-range
+// (usually one).  Sub-launches share the call's counters; each compares its
+// own buckets, and the "last block" ticket is reset between them.
 rr_status enqueue_unpack_verify(const rr_plan* P, Range R, const void* const* buckets,
                                 const uint64_t* checksums, void* const* dst, uint8_t* bad,
                                 cudaStream_t stream) {
@@ -1582,16 +1613,13 @@ rr_status enqueue_unpack_verify(const rr_plan* P, Range R, const void* const* bu
     RR_CUDA(cudaMemsetAsync(sc, 0, (size_t(n) + 4) * sizeof(unsigned long long), stream));
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
                       all_device((const void* const*)dst, P->n_tensors);
-    if (sh.parts.size() == 1)
-        return launch_unpack_part(P, sh.parts[0], bulk, buckets, dst, checksums, bad, sh, stream);
-    for (const Range& S : sh.parts)
-        if ((st = launch_unpack_part(P, S, bulk, buckets, dst, nullptr, nullptr, sh, stream)))
+    for (size_t i = 0; i < sh.parts.size(); ++i) {
+        if (i > 0) RR_CUDA(cudaMemsetAsync(sc + n, 0, sizeof(unsigned long long), stream));
+        if ((st = launch_unpack_part(P, sh.parts[i], bulk, buckets, dst, checksums, bad, sh,
+                                     stream)))
             return st;
-    return (!sh.table || P->n_buckets <= kSmallPtrs)
-               ? launch_verify<kSmallPtrs>(P, R, buckets, checksums, bad, sh.table, sh.stride,
-                                           stream)
-               : launch_verify<kLargePtrs>(P, R, buckets, checksums, bad, sh.table, sh.stride,
-                                           stream);
+    }
+    return RR_OK;
 }
 
 rr_status check_unpack_verify_args(const rr_plan* P, Range R, const void* const* buckets,
@@ -1652,19 +1680,25 @@ rr_status verify_impl(const rr_plan* P, Range R, const void* const* buckets,
     if (R.b1 == R.b0) return RR_OK;
     uint64_t stride = 0;
     const bool table = !uniform(buckets, P->n_buckets, P->bucket_bytes, &stride);
-    if (table && P->n_buckets > kLargePtrs)
-        return rr_fail(RR_EINVAL, "%d separately allocated buckets exceed %d pointers",
-                       P->n_buckets, kLargePtrs);
 
     rr_plan* M = const_cast<rr_plan*>(P);   // the scratch area is the only mutable state
     std::lock_guard<std::mutex> lock(M->verify_mutex);
     const int32_t n = R.b1 - R.b0;
     RR_CUDA(cudaMemsetAsync(P->d_verify_scratch, 0, (size_t(n) + 4) * sizeof(unsigned long long),
                             stream));
-    st = (!table || P->n_buckets <= kSmallPtrs)
-             ? launch_verify<kSmallPtrs>(P, R, buckets, checksums, bad, table, stride, stream)
-             : launch_verify<kLargePtrs>(P, R, buckets, checksums, bad, table, stride, stream);
-    if (st) return st;
+    // Separately allocated buckets: one launch per run of buckets that fits the
+    // pointer table, sharing the call's counters (ticket reset in between).
+    const int32_t step = table ? kLargePtrs : n;
+    for (int32_t b = R.b0; b < R.b1; b += step) {
+        const int32_t e = std::min(R.b1, b + step);
+        if (b > R.b0)
+            RR_CUDA(cudaMemsetAsync(P->d_verify_scratch + n, 0, sizeof(unsigned long long), stream));
+        const Range S{b, e, false, nullptr, 0, -1, R.b0, n};
+        st = (!table || e - b <= kSmallPtrs)
+                 ? launch_verify<kSmallPtrs>(P, S, buckets, checksums, bad, table, stride, stream)
+                 : launch_verify<kLargePtrs>(P, S, buckets, checksums, bad, table, stride, stream);
+        if (st) return st;
+    }
     return read_result(P, n, n_bad, first_bad, stream);
 }
 

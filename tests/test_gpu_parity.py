@@ -38,14 +38,8 @@ def full_parity(desc, separate_buckets=False, **opts):
     L = U.to_oracle(desc)
     m, s, d = U.to_product(desc)
     plan = H.make_plan(m, s, d, desc["bucket_bytes"], **opts)
-    if separate_buckets and plan.n_shards + plan.n_buckets > 3968:
-        # Beyond the pointer table of one launch: the library must refuse
-        # separately allocated buckets and accept one equally spaced block.
-        buf = H.alloc(plan, separate_buckets=True, with_dst=False)
-        with pytest.raises(rr.RRError) as e:
-            H.pack(buf)
-        assert e.value.status == rrmod.RR_EINVAL
-        separate_buckets = False
+    # Separately allocated buckets beyond one launch's pointer table run as
+    # several launches over bucket ranges.
     buf = H.alloc(plan, separate_buckets=separate_buckets)
     shards = L.host_shards(desc["seed"], desc["specials"])
     H.fill_from_host(buf, shards)
@@ -225,6 +219,30 @@ def test_bucket_writing_too_many_tensors_is_refused():
 def test_degenerate_layout(sharding, engine):
     """Zero-size parameters, empty blocks and empty tensors."""
     full_parity(U.degenerate_layout(sharding), engine=engine)
+
+
+@pytest.mark.parametrize("engine", ["auto", "registers"])
+def test_more_separate_buckets_than_one_launch_addresses(engine):
+    """4128 separately allocated 1 KiB buckets (with 8 source shards and the
+    tensors) exceed one launch's pointer table: pack, unpack and the verifying
+    calls run over bucket ranges; damage is still found at the right bucket."""
+    desc = U.workload_desc("tiny-tp4", bucket_bytes=1024)
+    full_parity(desc, separate_buckets=True, engine=engine)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"], engine=engine)
+    assert plan.n_buckets > 4000
+    buf = H.alloc(plan, separate_buckets=True)
+    H.fill_with_generator(buf, m, desc["seed"], desc["specials"])
+    H.pack(buf)
+    bl = H.bucket_list(buf)
+    bl[4100][8] ^= 0x01
+    bl[17][0] ^= 0x02
+    assert H.verify(buf) == (2, 17)
+    assert rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst) == (2, 17)
+    bad = torch.zeros(plan.n_buckets, dtype=torch.uint8, device="cuda")
+    assert rr.rr_verify_range(plan, 100, plan.n_buckets - 100, buf.buckets, buf.checksums,
+                              bad=bad) == (1, 4100)
+    assert list(np.flatnonzero(bad.cpu().numpy())) == [4100 - 100]
 
 
 def test_largest_bucket_size():
