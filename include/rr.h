@@ -393,6 +393,22 @@ rr_status rr_unpack_verify_range(const rr_plan* plan, int32_t first_bucket, int3
  * [pack_first[b], pack_first[b + 1]); likewise for unpack. */
 rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32_t* unpack_first);
 
+/* The verifying unpack's work units (rr_unpack_verify and its range and
+ * stream-ordered forms on the bulk-copy engine).  Each bucket's unpack items
+ * are cut into units of roughly equal weight (about 1 MiB of traffic, less on
+ * small plans, so that each block of the grid has a few dozen); a unit never
+ * spans two buckets.  A launch over buckets [b0, b1) gives block g the
+ * unit bucket_unit[b0] + g, and the rest of its units to whichever block asks
+ * next, so that blocks draining HBM at unequal rates still finish together.
+ *   *n_units: the number of units.
+ *   unit_first (NULL, or n_units + 1 entries): unit u holds unpack items
+ *     [unit_first[u], unit_first[u + 1]).
+ *   bucket_unit (NULL, or n_buckets + 1 entries): the units of bucket b are
+ *     [bucket_unit[b], bucket_unit[b + 1]).
+ * Call with both arrays NULL to learn n_units. */
+rr_status rr_plan_unpack_units(const rr_plan* plan, int32_t* n_units, uint32_t* unit_first,
+                               uint32_t* bucket_unit);
+
 /* Stream-ordered form of rr_unpack_verify(_range), for a receiver that unpacks
  * and checks piece after piece without waiting on the host (Sections 5.2.1 and
  * 5.2.2: the pull completes, and a resumed pull checks what it holds).

@@ -638,6 +638,13 @@ struct BulkArgs {
     int32_t first_bucket;
     int32_t n_buckets;
     unsigned int* err;
+    // Claimed work units (NULL: none).  block_first then holds the first item
+    // of each of n_units units (and one past the last): unit g < gridDim.x is
+    // block g's own, the rest go to whichever block asks next (atomicAdd on
+    // *claim, zero at launch).
+    unsigned long long* claim;
+    uint32_t n_units;
+    uint32_t pad2_;
     const void* ptr[NPTR];
 };
 
@@ -737,8 +744,13 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
     }
     __syncthreads();
 
-    uint32_t i0, i1;
-    block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
+    uint32_t i0 = 0, i1 = 0;
+    if (!a.claim)
+        block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
+    else if (blockIdx.x < a.n_units) {
+        i0 = a.block_first[blockIdx.x];
+        i1 = a.block_first[blockIdx.x + 1];
+    }
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
@@ -795,7 +807,27 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
             }
             ++count;
         };
-        for (uint32_t it = i0; it < i1 && ok; ++it) {
+        // Past its own range a block claims units while any are left, the next
+        // claim in flight (lane 0) while the current unit is walked.
+        unsigned long long pending = 0;
+        bool claimed = false;
+        auto next_range = [&](uint32_t* it) -> bool {
+            if (!a.claim) return false;
+            if (!claimed && lane == 0) pending = atomicAdd(a.claim, 1ull);
+            claimed = true;
+            const unsigned long long u = gridDim.x + __shfl_sync(0xFFFFFFFFu, pending, 0);
+            if (u >= a.n_units) return false;
+            if (lane == 0) pending = atomicAdd(a.claim, 1ull);
+            *it = a.block_first[u];
+            i1 = a.block_first[u + 1];
+            return true;
+        };
+        for (uint32_t it = i0; ok; ++it) {
+            if (it >= i1) {
+                bool more = true;
+                while (more && it >= i1) more = next_range(&it);
+                if (!more) break;
+            }
             Piece p;
             p.dst = nullptr;
             p.src_stride = 0;
@@ -1381,6 +1413,11 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
             const SumSlot q = sum_slot(P, R, bad);
             a.sums = q.sums;
             a.counters = q.counters;
+            // The range's work units, claimed through counters[3].
+            const uint32_t u0 = P->unpack_bucket_unit[R.b0], u1 = P->unpack_bucket_unit[R.b1];
+            a.block_first = P->d_unpack_unit_first + u0;
+            a.claim = q.counters + 3;
+            a.n_units = u1 - u0;
             a.expected = (const unsigned long long*)checksums;
             a.bad = q.bad;
             a.first_bucket = R.b0;
@@ -1601,7 +1638,8 @@ rr_status read_result(const rr_plan* P, int32_t n, int64_t* n_bad, int64_t* firs
 // Enqueues the verifying unpack of range R: zeroes the range's sums and
 // counters (R.scratch, else the plan's), then one fused launch per sub-range
 // (usually one).  Sub-launches share the call's counters; each compares its
-// own buckets, and the "last block" ticket is reset between them.
+// own buckets, and the "last block" ticket and the unit claims are reset
+// between them.
 rr_status enqueue_unpack_verify(const rr_plan* P, Range R, const void* const* buckets,
                                 const uint64_t* checksums, void* const* dst, uint8_t* bad,
                                 cudaStream_t stream) {
@@ -1614,7 +1652,10 @@ rr_status enqueue_unpack_verify(const rr_plan* P, Range R, const void* const* bu
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
                       all_device((const void* const*)dst, P->n_tensors);
     for (size_t i = 0; i < sh.parts.size(); ++i) {
-        if (i > 0) RR_CUDA(cudaMemsetAsync(sc + n, 0, sizeof(unsigned long long), stream));
+        if (i > 0) {   // a fresh "last block" ticket and unit claims
+            RR_CUDA(cudaMemsetAsync(sc + n, 0, sizeof(unsigned long long), stream));
+            RR_CUDA(cudaMemsetAsync(sc + n + 3, 0, sizeof(unsigned long long), stream));
+        }
         if ((st = launch_unpack_part(P, sh.parts[i], bulk, buckets, dst, checksums, bad, sh,
                                      stream)))
             return st;
@@ -1754,6 +1795,8 @@ rr_status rr_device_upload(rr_plan* P) {
                 P->unpack_items.size() * sizeof(rr_unpack_item))) != cudaSuccess ||
         (e = up((void**)&P->d_unpack_block_first, P->unpack_block_first.data(),
                 P->unpack_block_first.size() * sizeof(uint32_t))) != cudaSuccess ||
+        (e = up((void**)&P->d_unpack_unit_first, P->unpack_unit_first.data(),
+                P->unpack_unit_first.size() * sizeof(uint32_t))) != cudaSuccess ||
         (e = cudaMalloc((void**)&P->d_verify_scratch,
                         (size_t(P->n_buckets) + 4) * sizeof(unsigned long long))) != cudaSuccess ||
         (e = cudaHostAlloc((void**)&P->h_verify_result, 5 * sizeof(unsigned long long),
@@ -1793,6 +1836,7 @@ void rr_device_release(rr_plan* P) {
     cudaFree(P->d_tensor_bytes);
     cudaFree(P->d_unpack_items);
     cudaFree(P->d_unpack_block_first);
+    cudaFree(P->d_unpack_unit_first);
     cudaFree(P->d_verify_scratch);
     cudaFreeHost(P->h_verify_result);
     cudaFree(P->d_error);
@@ -1807,6 +1851,7 @@ void rr_device_release(rr_plan* P) {
     P->d_tensor_bytes = nullptr;
     P->d_unpack_items = nullptr;
     P->d_unpack_block_first = nullptr;
+    P->d_unpack_unit_first = nullptr;
     P->d_verify_scratch = nullptr;
     P->h_verify_result = nullptr;
     if (prev >= 0 && prev != P->device) cudaSetDevice(prev);

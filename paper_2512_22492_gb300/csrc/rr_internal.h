@@ -61,6 +61,9 @@ struct rr_plan {
     std::vector<uint32_t> pack_block_first;     // grid_blocks + 1
     std::vector<rr_unpack_item> unpack_items;
     std::vector<uint32_t> unpack_block_first;   // grid_blocks + 1
+    std::vector<uint32_t> unpack_unit_first;    // verifying unpack's claimed work units:
+                                                //   first item of each (+ 1 past the last)
+    std::vector<uint32_t> unpack_bucket_unit;   // n_buckets + 1: first unit of bucket b
     std::vector<uint32_t> pack_bucket_first;    // n_buckets + 1: first pack item of bucket b
     std::vector<unsigned long long> pack_weight_prefix;    // items + 1: balancing weights,
     std::vector<unsigned long long> unpack_weight_prefix;  // summed (bucket-range calls)
@@ -86,6 +89,7 @@ struct rr_plan {
     int64_t* d_tensor_bytes = nullptr;       //              and of each destination tensor
     rr_unpack_item* d_unpack_items = nullptr;
     uint32_t* d_unpack_block_first = nullptr;
+    uint32_t* d_unpack_unit_first = nullptr;
     unsigned long long* d_verify_scratch = nullptr;  // n_buckets sums + 4 counters
     unsigned long long* h_verify_result = nullptr;   // pinned, 5 words (4 counters + error)
     unsigned int* d_error = nullptr;                 // set by a kernel whose wait ran out

@@ -34,6 +34,8 @@ thread_local std::string g_error;
 
 constexpr int64_t kDefaultChunkBytes = 32 * 1024;
 constexpr int64_t kItemOverhead = 1024;   // balancing weight of one item, in bytes
+constexpr int64_t kUnitWeight = 1 << 20;   // largest claimed work unit of the verifying unpack
+constexpr int32_t kUnitsPerBlock = 32;     //   (weight), and the units wanted per block
 constexpr int64_t kMaxShardOffset = (int64_t(1) << 48) - 1;
 // Fan-out groups: column slices narrower than kFanSliceBytes of source per row,
 // at most kMaxFanDst of them, over a joint span of at most kFanMaxRowBytes.
@@ -375,6 +377,40 @@ void partition(const std::vector<Item>& items, int32_t grid, std::vector<uint32_
     }
 }
 
+// Work units for a kernel whose blocks claim work as they run out of it.  Each
+// bucket's items are cut into units of about kUnitWeight (a unit never spans
+// two buckets, so a bucket-range call takes a contiguous run of units):
+// first[u] is the first item of unit u, bucket_unit[b] the first unit of
+// bucket b.  Blocks drain HBM at unequal rates; small units claimed one at a
+// time let the fast blocks take more of them, and all finish together.
+template <class Item, class W>
+void bucket_units(const std::vector<Item>& items, const std::vector<uint32_t>& bucket_first,
+                  int64_t unit_weight, std::vector<uint32_t>& first,
+                  std::vector<uint32_t>& bucket_unit, W w) {
+    first.clear();
+    bucket_unit.assign(bucket_first.size(), 0);
+    for (size_t b = 0; b + 1 < bucket_first.size(); ++b) {
+        bucket_unit[b] = uint32_t(first.size());
+        const uint32_t lo = bucket_first[b], hi = bucket_first[b + 1];
+        if (lo == hi) continue;
+        int64_t total = 0;
+        for (uint32_t i = lo; i < hi; ++i) total += w(items[i]);
+        const int64_t n = std::max<int64_t>(1, (total + unit_weight - 1) / unit_weight);
+        first.push_back(lo);
+        int64_t cum = 0, k = 1;
+        for (uint32_t i = lo; i < hi && k < n; ++i) {
+            cum += w(items[i]);
+            // A cut after item i when it reaches the next share (no empty units).
+            if (cum * n >= total * k && i + 1 < hi) {
+                first.push_back(i + 1);
+                while (k < n && cum * n >= total * k) ++k;
+            }
+        }
+    }
+    bucket_unit.back() = uint32_t(first.size());
+    first.push_back(bucket_first.empty() ? 0 : bucket_first.back());
+}
+
 rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_params,
                                 const rr_src_layout* src, const rr_dst_layout* dst,
                                 size_t bucket_bytes) {
@@ -682,6 +718,17 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     }
     partition(P->pack_items, P->grid_blocks, P->pack_block_first, pack_weight);
     partition(P->unpack_items, P->unpack_grid_blocks, P->unpack_block_first, unpack_weight);
+    {
+        // About kUnitsPerBlock units per block of the grid, none above kUnitWeight
+        // (small enough to even out the finish), none below kUnitWeight / 8
+        // (each costs the producer one claim).
+        int64_t total = 0;
+        for (const rr_unpack_item& it : P->unpack_items) total += unpack_weight(it);
+        const int64_t per_block = total / (int64_t(kUnitsPerBlock) * std::max(1, P->unpack_grid_blocks));
+        const int64_t unit = std::min(kUnitWeight, std::max(kUnitWeight / 8, per_block));
+        bucket_units(P->unpack_items, P->unpack_bucket_first, unit, P->unpack_unit_first,
+                     P->unpack_bucket_unit, unpack_weight);
+    }
     // Summed weights: a bucket-range call splits its items over the grid by them.
     auto prefix = [](const auto& items, std::vector<unsigned long long>& out, auto w) {
         out.assign(items.size() + 1, 0ull);
@@ -917,6 +964,17 @@ rr_status rr_plan_bucket_items(const rr_plan* P, uint32_t* pack_first, uint32_t*
         std::copy(P->pack_bucket_first.begin(), P->pack_bucket_first.end(), pack_first);
     if (unpack_first)
         std::copy(P->unpack_bucket_first.begin(), P->unpack_bucket_first.end(), unpack_first);
+    return RR_OK;
+}
+
+rr_status rr_plan_unpack_units(const rr_plan* P, int32_t* n_units, uint32_t* unit_first,
+                               uint32_t* bucket_unit) {
+    if (!P || !n_units) return rr_fail(RR_EINVAL, "NULL argument");
+    *n_units = int32_t(P->unpack_unit_first.size()) - 1;
+    if (unit_first)
+        std::copy(P->unpack_unit_first.begin(), P->unpack_unit_first.end(), unit_first);
+    if (bucket_unit)
+        std::copy(P->unpack_bucket_unit.begin(), P->unpack_bucket_unit.end(), bucket_unit);
     return RR_OK;
 }
 

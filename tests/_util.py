@@ -262,3 +262,24 @@ def check_partition(first, n_items):
     first = np.asarray(first, np.int64)
     assert first[0] == 0 and first[-1] == n_items
     assert np.all(np.diff(first) >= 0)
+
+
+def check_units(plan, n_items):
+    """The verifying unpack's work units tile each bucket's unpack items: no
+    unit is empty or spans two buckets, and bucket b's units cover exactly its
+    items, so any bucket range is a contiguous run of whole units."""
+    first, bucket_unit = plan.unpack_units()
+    _, bucket_first = plan.bucket_items()
+    first = first.astype(np.int64)
+    bucket_unit = bucket_unit.astype(np.int64)
+    assert first[0] == 0 and first[-1] == n_items
+    assert np.all(np.diff(first) > 0)
+    assert bucket_unit[0] == 0 and bucket_unit[-1] == len(first) - 1
+    assert np.all(np.diff(bucket_unit) >= 0)
+    for b in range(plan.n_buckets):
+        lo, hi = bucket_first[b], bucket_first[b + 1]
+        u0, u1 = bucket_unit[b], bucket_unit[b + 1]
+        assert (u1 > u0) == (hi > lo)
+        if hi > lo:
+            assert first[u0] == lo and first[u1] == hi
+    return first, bucket_unit

@@ -118,3 +118,43 @@ def test_async_refuses_bad_result_and_scratch():
         rr.rr_unpack_verify_async(plan, buf.buckets, buf.checksums, buf.dst,
                                   torch.zeros(3, dtype=torch.int64, device="cuda"),
                                   torch.zeros(2, dtype=torch.int64, device="cuda"))
+
+
+@pytest.mark.parametrize("grid", [1, 3, 2048])
+def test_claimed_units_on_any_grid(grid):
+    """The verifying unpack's blocks claim work units: one block taking every
+    unit, a few blocks, and more blocks than units (most with none of their
+    own) all give the oracle's tensors and the same verdicts, for the whole
+    sync and for bucket ranges."""
+    desc, plan, buf = packed("tiny-moe-tp2", grid_blocks=grid)
+    first, bucket_unit = plan.unpack_units()
+    assert len(first) - 1 > 3 and len(first) - 1 < 2048
+    bl = H.bucket_list(buf)
+    bl[6][40] ^= 0x04
+    for t in buf.dst:
+        t.fill_(0)
+    result = torch.zeros(2, dtype=torch.int64, device="cuda")
+    bad = torch.zeros(plan.n_buckets, dtype=torch.uint8, device="cuda")
+    rr.rr_unpack_verify_async(plan, buf.buckets, buf.checksums, buf.dst, scratch_for(plan), result,
+                              bad=bad)
+    torch.cuda.synchronize()
+    assert result.cpu().tolist() == [1, 6]
+    assert list(np.flatnonzero(bad.cpu().numpy())) == [6]
+    bl[6][40] ^= 0x04                                   # undo: tensors must match the oracle
+    L = U.to_oracle(desc)
+    gen = oracle.Source(seed=desc["seed"], specials=desc["specials"])
+    for first_b, count in ((0, plan.n_buckets), (2, 5), (plan.n_buckets - 1, 1)):
+        for t in buf.dst:
+            t.fill_(0)
+        rr.rr_unpack_verify_async(plan, buf.buckets, buf.checksums, buf.dst, scratch_for(plan),
+                                  result, first_bucket=first_b, n_buckets=count)
+        torch.cuda.synchronize()
+        assert result.cpu().tolist() == [0, -1]
+        assert rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst, first_bucket=first_b,
+                                   n_buckets=count) == (0, -1)
+    for t in buf.dst:
+        t.fill_(0)
+    assert rr.rr_unpack_verify(plan, buf.buckets, buf.checksums, buf.dst) == (0, -1)
+    for t in range(plan.n_tensors):
+        np.testing.assert_array_equal(H.tensor_host(buf, t), L.reshard_tensor(gen, t))
+    rr.rr_plan_check(plan)

@@ -76,6 +76,7 @@ def run_and_compare(desc, **opt):
     np.testing.assert_array_equal(got, want)
     uitems, ufirst = p.export_unpack()
     U.check_partition(ufirst, len(uitems))
+    U.check_units(p, len(uitems))
     tensors = U.check_and_run_unpack(uitems, want, p.tensor_numel)
     for t, arr in enumerate(tensors):
         np.testing.assert_array_equal(arr, L.unpack_tensor(want, t))
@@ -147,6 +148,29 @@ def test_full_size_tables_are_consistent():
     data = items["kind"] <= U.ITEM_BF16_SCALAR
     assert (n[data] * 4).sum() == st["pack_bytes_read"]
     assert np.all(items["kind"][data] == U.ITEM_F32_VEC)
+
+
+@pytest.mark.parametrize("name", ["qwen3-0.6b", "qwen3-8b", "qwen3-30b-a3b-fsdp2-tp8"])
+def test_unpack_work_units_on_full_size_tables(name):
+    """Units of equal weight (a byte copied by vectors weighs 2, one by
+    elements 4, a read-only one 1, an item 1024 more): at most 1 MiB, or less
+    where that leaves a block of the grid fewer than 32; none heavier than
+    that plus one item, and only a bucket's last unit much lighter."""
+    p = host_plan(U.workload_desc(name))
+    items, _ = p.export_unpack()
+    first, bucket_unit = U.check_units(p, len(items))
+    nbytes = items["nbytes"].astype(np.int64)
+    per_byte = np.select([items["kind"] == U.ITEM_COPY_VEC, items["kind"] == U.ITEM_COPY_SCALAR],
+                         [2, 4], 1)
+    w = per_byte * nbytes + 1024
+    grid = p.stats()["unpack_grid_blocks"]
+    unit = min(1 << 20, max((1 << 20) // 8, int(w.sum()) // (32 * grid)))
+    unit_w = np.add.reduceat(w, first[:-1])
+    assert unit_w.max() <= unit + w.max()
+    last = np.zeros(len(unit_w), bool)
+    last[bucket_unit[1:] - 1] = True
+    assert np.all(unit_w[~last] >= unit // 2 - w.max())
+    assert len(unit_w) >= 16 * grid
 
 
 def test_fan_out_groups_on_full_size_tables():
