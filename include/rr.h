@@ -393,21 +393,34 @@ rr_status rr_unpack_verify_range(const rr_plan* plan, int32_t first_bucket, int3
  * [pack_first[b], pack_first[b + 1]); likewise for unpack. */
 rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32_t* unpack_first);
 
-/* The verifying unpack's work units (rr_unpack_verify and its range and
- * stream-ordered forms on the bulk-copy engine).  Each bucket's unpack items
- * are cut into units of roughly equal weight (about 1 MiB of traffic, less on
- * small plans, so that each block of the grid has a few dozen); a unit never
- * spans two buckets.  A launch over buckets [b0, b1) gives block g the
- * unit bucket_unit[b0] + g, and the rest of its units to whichever block asks
- * next, so that blocks draining HBM at unequal rates still finish together.
+/* Work units of the bulk-copy engine.  Blocks drain HBM at unequal rates, so
+ * a launch does not fix each block's share: block g takes the launch's unit g,
+ * then claims the next unclaimed unit (an atomic counter) until none are left,
+ * and all blocks finish together.  Each table's items are cut into units of
+ * roughly equal weight: about 1 MiB of traffic, less on small plans, so that
+ * every block of the grid has a few dozen.
+ *   which: RR_UNITS_PACK (the pack items; a unit never spans two buckets, so a
+ *     bucket range is a run of whole units), RR_UNITS_PACK_FULL (the table a
+ *     pack over every bucket runs, as rr_plan_export_pack_full gives it: with
+ *     fan-out items, a unit never starting on a fan-out destination item, or
+ *     the pack items and their units where the plan has no fan-out items),
+ *     RR_UNITS_UNPACK (the unpack items, per bucket like RR_UNITS_PACK).
  *   *n_units: the number of units.
- *   unit_first (NULL, or n_units + 1 entries): unit u holds unpack items
- *     [unit_first[u], unit_first[u + 1]).
- *   bucket_unit (NULL, or n_buckets + 1 entries): the units of bucket b are
- *     [bucket_unit[b], bucket_unit[b + 1]).
- * Call with both arrays NULL to learn n_units. */
-rr_status rr_plan_unpack_units(const rr_plan* plan, int32_t* n_units, uint32_t* unit_first,
-                               uint32_t* bucket_unit);
+ *   unit_first (NULL, or n_units + 1 entries): unit u holds items
+ *     [unit_first[u], unit_first[u + 1]) of that table.
+ *   bucket_unit (NULL, or n_buckets + 1 entries; must be NULL for
+ *     RR_UNITS_PACK_FULL): the units of bucket b are [bucket_unit[b],
+ *     bucket_unit[b + 1]).
+ * Call with both arrays NULL to learn n_units.
+ * Which launches claim: the verifying unpack always (its counter lives in the
+ * call's scratch); rr_pack and rr_unpack when one of the plan's 16 counter
+ * slots is free -- a slot is reused only after the launch that last held it
+ * has completed -- and the stream is not capturing a graph.  Otherwise the
+ * launch splits its items evenly over the grid, as a captured launch always
+ * does. */
+enum { RR_UNITS_PACK = 0, RR_UNITS_PACK_FULL = 1, RR_UNITS_UNPACK = 2 };
+rr_status rr_plan_work_units(const rr_plan* plan, int32_t which, int32_t* n_units,
+                             uint32_t* unit_first, uint32_t* bucket_unit);
 
 /* Stream-ordered form of rr_unpack_verify(_range), for a receiver that unpacks
  * and checks piece after piece without waiting on the host (Sections 5.2.1 and

@@ -644,7 +644,7 @@ struct BulkArgs {
     // *claim, zero at launch).
     unsigned long long* claim;
     uint32_t n_units;
-    uint32_t pad2_;
+    uint32_t reset_claims;       // claim is a pooled slot {counter, ticket}: zero it at the end
     const void* ptr[NPTR];
 };
 
@@ -981,6 +981,16 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                 mbar_wait(smem_u32(&full[c % kStages]), (c / kStages) & 1, a.err);
         }
         asm volatile("cp.async.wait_all;" ::: "memory");
+        if (a.claim && a.reset_claims && lane == 0) {
+            // A pooled counter goes back to zero for the slot's next launch: the
+            // last block here resets it.  Every block gets here, and only after
+            // its last claim has returned (the ticket's increment depends on it).
+            const unsigned long long t = atomicAdd(a.claim + 1, 1ull | (pending >> 63));
+            if (t == gridDim.x - 1) {
+                atomicExch(a.claim, 0ull);
+                atomicExch(a.claim + 1, 0ull);
+            }
+        }
         return;
     }
 
@@ -1379,6 +1389,38 @@ bool all_device(const void* const* ptrs, int32_t n) {
     return n == 0 || (device_resident(ptrs[0]) && device_resident(ptrs[n - 1]));
 }
 
+// A unit-claim slot for a launch on `s` that has no per-call scratch, or -1:
+// every slot's last launch still running, or `s` capturing a graph (a captured
+// launch replays whenever the graph does, so it keeps the fixed split).  The
+// caller holds claim_mutex and records claim_done[slot] after the launch.  A
+// slot is {counter, ticket}, zero when handed out: zeroed once at plan
+// creation, then by the last block of each launch that held it.
+int32_t take_claim_slot(rr_plan* M, cudaStream_t s) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &cs) != cudaSuccess) {
+        cudaGetLastError();
+        return -1;
+    }
+    if (cs != cudaStreamCaptureStatusNone) return -1;
+    // Querying an event is allowed to this thread even while another thread
+    // captures a graph.
+    cudaStreamCaptureMode mode = cudaStreamCaptureModeRelaxed;
+    cudaThreadExchangeStreamCaptureMode(&mode);
+    int32_t slot = -1;
+    for (int32_t i = 0; i < rr_plan::kClaimSlots && slot < 0; ++i) {
+        const int32_t k = (M->claim_next + i) % rr_plan::kClaimSlots;
+        if (M->claim_retired[k]) continue;
+        const cudaError_t q = cudaEventQuery(M->claim_done[k]);
+        if (q == cudaSuccess)
+            slot = k;
+        else if (q != cudaErrorNotReady)
+            cudaGetLastError();
+    }
+    cudaThreadExchangeStreamCaptureMode(&mode);
+    if (slot >= 0) M->claim_next = (slot + 1) % rr_plan::kClaimSlots;
+    return slot;
+}
+
 template <int NPTR, int MODE>
 rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
                       const void* const* buckets, void* const* dst, const uint64_t* checksums,
@@ -1436,6 +1478,29 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         for (int32_t t = R.t_lo; t <= R.t_hi; ++t) a.ptr[k++] = dst[t];
     }
     const int32_t grid = MODE == 0 ? P->grid_blocks : P->unpack_grid_blocks;
+    // Pack and plain unpack claim their units through a pooled slot when one
+    // is free; otherwise they run the fixed split set above.
+    rr_plan* M = const_cast<rr_plan*>(P);   // the claim pool is mutable state
+    std::unique_lock<std::mutex> lock(M->claim_mutex, std::defer_lock);
+    int32_t slot = -1;
+    cudaError_t e = cudaSuccess;
+    if (MODE != 2) {
+        lock.lock();
+        if ((slot = take_claim_slot(M, s)) >= 0) {
+            a.claim = P->d_claims + 2 * slot;
+            a.reset_claims = 1;
+            if (MODE == 0 && R.full && P->d_full_items) {
+                a.block_first = P->d_full_unit_first;
+                a.n_units = uint32_t(P->full_unit_first.size() - 1);
+            } else {
+                const std::vector<uint32_t>& bu =
+                    MODE == 0 ? P->pack_bucket_unit : P->unpack_bucket_unit;
+                a.block_first = (MODE == 0 ? P->d_pack_unit_first : P->d_unpack_unit_first) +
+                                bu[R.b0];
+                a.n_units = bu[R.b1] - bu[R.b0];
+            }
+        }
+    }
     if (P->check_items) {
         RR_CUDA((bulk_prepare<NPTR, MODE, true>()));
         rr_bulk_kernel<NPTR, MODE, true>
@@ -1446,6 +1511,10 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
             <<<grid, BulkShape<MODE>::kThreads, BulkShape<MODE>::kSmem, s>>>(a);
     }
     RR_CUDA(cudaGetLastError());
+    if (slot >= 0 && (e = cudaEventRecord(P->claim_done[slot], s)) != cudaSuccess) {
+        M->claim_retired[slot] = 1;   // its launch's end is unknown: never hand it out again
+        return cuda_fail(e, "cudaEventRecord");
+    }
     return RR_OK;
 }
 
@@ -1797,6 +1866,15 @@ rr_status rr_device_upload(rr_plan* P) {
                 P->unpack_block_first.size() * sizeof(uint32_t))) != cudaSuccess ||
         (e = up((void**)&P->d_unpack_unit_first, P->unpack_unit_first.data(),
                 P->unpack_unit_first.size() * sizeof(uint32_t))) != cudaSuccess ||
+        (e = up((void**)&P->d_pack_unit_first, P->pack_unit_first.data(),
+                P->pack_unit_first.size() * sizeof(uint32_t))) != cudaSuccess ||
+        (!P->full_unit_first.empty() &&
+         (e = up((void**)&P->d_full_unit_first, P->full_unit_first.data(),
+                 P->full_unit_first.size() * sizeof(uint32_t))) != cudaSuccess) ||
+        (e = cudaMalloc((void**)&P->d_claims,
+                        2 * rr_plan::kClaimSlots * sizeof(unsigned long long))) != cudaSuccess ||
+        (e = cudaMemset(P->d_claims, 0, 2 * rr_plan::kClaimSlots * sizeof(unsigned long long))) !=
+            cudaSuccess ||
         (e = cudaMalloc((void**)&P->d_verify_scratch,
                         (size_t(P->n_buckets) + 4) * sizeof(unsigned long long))) != cudaSuccess ||
         (e = cudaHostAlloc((void**)&P->h_verify_result, 5 * sizeof(unsigned long long),
@@ -1818,6 +1896,8 @@ rr_status rr_device_upload(rr_plan* P) {
                   P->full_block_first.size() * sizeof(uint32_t))) != cudaSuccess)))
         return e == cudaErrorMemoryAllocation ? rr_fail(RR_ENOMEM, "device allocation failed")
                                               : cuda_fail(e, "plan upload");
+    for (cudaEvent_t& ev : P->claim_done)
+        RR_CUDA(cudaEventCreateWithFlags(&ev, cudaEventDisableTiming));
     return RR_OK;
 }
 
@@ -1837,6 +1917,13 @@ void rr_device_release(rr_plan* P) {
     cudaFree(P->d_unpack_items);
     cudaFree(P->d_unpack_block_first);
     cudaFree(P->d_unpack_unit_first);
+    cudaFree(P->d_pack_unit_first);
+    cudaFree(P->d_full_unit_first);
+    cudaFree(P->d_claims);
+    for (cudaEvent_t& ev : P->claim_done) {
+        if (ev) cudaEventDestroy(ev);
+        ev = nullptr;
+    }
     cudaFree(P->d_verify_scratch);
     cudaFreeHost(P->h_verify_result);
     cudaFree(P->d_error);
@@ -1852,6 +1939,9 @@ void rr_device_release(rr_plan* P) {
     P->d_unpack_items = nullptr;
     P->d_unpack_block_first = nullptr;
     P->d_unpack_unit_first = nullptr;
+    P->d_pack_unit_first = nullptr;
+    P->d_full_unit_first = nullptr;
+    P->d_claims = nullptr;
     P->d_verify_scratch = nullptr;
     P->h_verify_result = nullptr;
     if (prev >= 0 && prev != P->device) cudaSetDevice(prev);

@@ -61,9 +61,13 @@ struct rr_plan {
     std::vector<uint32_t> pack_block_first;     // grid_blocks + 1
     std::vector<rr_unpack_item> unpack_items;
     std::vector<uint32_t> unpack_block_first;   // grid_blocks + 1
-    std::vector<uint32_t> unpack_unit_first;    // verifying unpack's claimed work units:
-                                                //   first item of each (+ 1 past the last)
-    std::vector<uint32_t> unpack_bucket_unit;   // n_buckets + 1: first unit of bucket b
+    // Claimed work units of the bulk-copy engine: first item of each unit (+ 1
+    // past the last); per bucket, its first unit (n_buckets + 1).
+    std::vector<uint32_t> unpack_unit_first;
+    std::vector<uint32_t> unpack_bucket_unit;
+    std::vector<uint32_t> pack_unit_first;
+    std::vector<uint32_t> pack_bucket_unit;
+    std::vector<uint32_t> full_unit_first;      // the whole-sync table's (whole launches only)
     std::vector<uint32_t> pack_bucket_first;    // n_buckets + 1: first pack item of bucket b
     std::vector<unsigned long long> pack_weight_prefix;    // items + 1: balancing weights,
     std::vector<unsigned long long> unpack_weight_prefix;  // summed (bucket-range calls)
@@ -90,6 +94,17 @@ struct rr_plan {
     rr_unpack_item* d_unpack_items = nullptr;
     uint32_t* d_unpack_block_first = nullptr;
     uint32_t* d_unpack_unit_first = nullptr;
+    uint32_t* d_pack_unit_first = nullptr;
+    uint32_t* d_full_unit_first = nullptr;
+    // Unit-claim counters of launches that have no per-call scratch (rr_pack,
+    // rr_unpack): a slot is handed to a launch only once the event recorded
+    // after its previous launch has completed; that launch left it zeroed.
+    static constexpr int kClaimSlots = 16;
+    unsigned long long* d_claims = nullptr;      // kClaimSlots x {counter, ticket}
+    cudaEvent_t claim_done[kClaimSlots] = {};
+    char claim_retired[kClaimSlots] = {};
+    int32_t claim_next = 0;
+    std::mutex claim_mutex;
     unsigned long long* d_verify_scratch = nullptr;  // n_buckets sums + 4 counters
     unsigned long long* h_verify_result = nullptr;   // pinned, 5 words (4 counters + error)
     unsigned int* d_error = nullptr;                 // set by a kernel whose wait ran out

@@ -411,6 +411,39 @@ void bucket_units(const std::vector<Item>& items, const std::vector<uint32_t>& b
     first.push_back(bucket_first.empty() ? 0 : bucket_first.back());
 }
 
+// The same for a table that a launch always takes whole (the whole-sync pack
+// table, whose fan-out groups write several buckets): equal shares of its
+// weight, a unit never starting on a fan-out destination item.
+template <class Item, class W>
+void even_units(const std::vector<Item>& items, int64_t unit_weight, std::vector<uint32_t>& first,
+                W w) {
+    first.assign(1, 0);
+    if (items.empty()) return;
+    int64_t total = 0;
+    for (const Item& it : items) total += w(it);
+    const int64_t n = std::max<int64_t>(1, (total + unit_weight - 1) / unit_weight);
+    int64_t cum = 0, k = 1;
+    for (size_t i = 0; i + 1 < items.size() && k < n; ++i) {
+        cum += w(items[i]);
+        if (cum * n >= total * k && items[i + 1].kind != RR_ITEM_FAN_DST) {
+            first.push_back(uint32_t(i + 1));
+            while (k < n && cum * n >= total * k) ++k;
+        }
+    }
+    first.push_back(uint32_t(items.size()));
+}
+
+// Claimed-unit weight for a table: about kUnitsPerBlock units per block of the
+// grid, none above kUnitWeight (small enough to even out the finish), none
+// below kUnitWeight / 8 (each costs the producer one claim).
+template <class Item, class W>
+int64_t unit_weight_for(const std::vector<Item>& items, int32_t grid, W w) {
+    int64_t total = 0;
+    for (const Item& it : items) total += w(it);
+    const int64_t per_block = total / (int64_t(kUnitsPerBlock) * std::max(1, grid));
+    return std::min(kUnitWeight, std::max(kUnitWeight / 8, per_block));
+}
+
 rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_params,
                                 const rr_src_layout* src, const rr_dst_layout* dst,
                                 size_t bucket_bytes) {
@@ -718,17 +751,12 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     }
     partition(P->pack_items, P->grid_blocks, P->pack_block_first, pack_weight);
     partition(P->unpack_items, P->unpack_grid_blocks, P->unpack_block_first, unpack_weight);
-    {
-        // About kUnitsPerBlock units per block of the grid, none above kUnitWeight
-        // (small enough to even out the finish), none below kUnitWeight / 8
-        // (each costs the producer one claim).
-        int64_t total = 0;
-        for (const rr_unpack_item& it : P->unpack_items) total += unpack_weight(it);
-        const int64_t per_block = total / (int64_t(kUnitsPerBlock) * std::max(1, P->unpack_grid_blocks));
-        const int64_t unit = std::min(kUnitWeight, std::max(kUnitWeight / 8, per_block));
-        bucket_units(P->unpack_items, P->unpack_bucket_first, unit, P->unpack_unit_first,
-                     P->unpack_bucket_unit, unpack_weight);
-    }
+    bucket_units(P->unpack_items, P->unpack_bucket_first,
+                 unit_weight_for(P->unpack_items, P->unpack_grid_blocks, unpack_weight),
+                 P->unpack_unit_first, P->unpack_bucket_unit, unpack_weight);
+    bucket_units(P->pack_items, P->pack_bucket_first,
+                 unit_weight_for(P->pack_items, P->grid_blocks, pack_weight), P->pack_unit_first,
+                 P->pack_bucket_unit, pack_weight);
     // Summed weights: a bucket-range call splits its items over the grid by them.
     auto prefix = [](const auto& items, std::vector<unsigned long long>& out, auto w) {
         out.assign(items.size() + 1, 0ull);
@@ -740,6 +768,7 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     // Whole-sync table: the grouped blocks' plain items give way to fan-out groups.
     P->full_items.clear();
     P->full_block_first.clear();
+    P->full_unit_first.clear();
     if (!groups.empty()) {
         std::vector<char> drop(P->pack_items.size(), 0);
         for (auto [lo, hi] : fanned)
@@ -774,6 +803,8 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
             f[g] = std::max(f[g], f[g - 1]);
             while (f[g] < P->full_items.size() && P->full_items[f[g]].kind == RR_ITEM_FAN_DST) ++f[g];
         }
+        even_units(P->full_items, unit_weight_for(P->full_items, P->grid_blocks, pack_weight),
+                   P->full_unit_first, pack_weight);
     }
 
     rr_plan_stats& s = P->stats;
@@ -967,14 +998,23 @@ rr_status rr_plan_bucket_items(const rr_plan* P, uint32_t* pack_first, uint32_t*
     return RR_OK;
 }
 
-rr_status rr_plan_unpack_units(const rr_plan* P, int32_t* n_units, uint32_t* unit_first,
-                               uint32_t* bucket_unit) {
+rr_status rr_plan_work_units(const rr_plan* P, int32_t which, int32_t* n_units,
+                             uint32_t* unit_first, uint32_t* bucket_unit) {
     if (!P || !n_units) return rr_fail(RR_EINVAL, "NULL argument");
-    *n_units = int32_t(P->unpack_unit_first.size()) - 1;
-    if (unit_first)
-        std::copy(P->unpack_unit_first.begin(), P->unpack_unit_first.end(), unit_first);
-    if (bucket_unit)
-        std::copy(P->unpack_bucket_unit.begin(), P->unpack_bucket_unit.end(), bucket_unit);
+    const std::vector<uint32_t>* first = nullptr;
+    const std::vector<uint32_t>* bu = nullptr;
+    switch (which) {
+        case RR_UNITS_PACK: first = &P->pack_unit_first; bu = &P->pack_bucket_unit; break;
+        case RR_UNITS_PACK_FULL:   // the table a whole-sync pack runs
+            first = P->full_items.empty() ? &P->pack_unit_first : &P->full_unit_first;
+            break;
+        case RR_UNITS_UNPACK: first = &P->unpack_unit_first; bu = &P->unpack_bucket_unit; break;
+        default: return rr_fail(RR_EINVAL, "which must be RR_UNITS_PACK, _PACK_FULL or _UNPACK");
+    }
+    if (bucket_unit && !bu) return rr_fail(RR_EINVAL, "the whole-sync table has no bucket units");
+    *n_units = first->empty() ? 0 : int32_t(first->size()) - 1;
+    if (unit_first) std::copy(first->begin(), first->end(), unit_first);
+    if (bucket_unit) std::copy(bu->begin(), bu->end(), bucket_unit);
     return RR_OK;
 }
 

@@ -149,8 +149,8 @@ _sig("rr_clear_range", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp)
 _sig("rr_unpack_verify_async", [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(_vp), _vp,
                                 ctypes.POINTER(_vp), _vp, _vp, _vp, _vp])
 _sig("rr_plan_bucket_items", [_vp, ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_uint32)])
-_sig("rr_plan_unpack_units", [_vp, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_uint32),
-                              ctypes.POINTER(ctypes.c_uint32)])
+_sig("rr_plan_work_units", [_vp, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32),
+                            ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_uint32)])
 _sig("rr_verify_noalloc", [ctypes.POINTER(_vp), ctypes.c_int32, ctypes.c_size_t, _vp, _P64, _P64,
                            _vp])
 _sig("rr_plan_check", [_vp, _vp])
@@ -162,7 +162,7 @@ LIBRARY_PATH = _build.LIB
 EXPORTED = ("rr_plan_create", "rr_plan_create_ex", "rr_plan_destroy", "rr_plan_query",
             "rr_plan_source", "rr_plan_source_buffers", "rr_plan_tensors", "rr_plan_get_stats",
             "rr_plan_export_pack", "rr_plan_export_pack_full",
-            "rr_plan_export_unpack", "rr_plan_bucket_items", "rr_plan_unpack_units", "rr_pack", "rr_unpack", "rr_verify",
+            "rr_plan_export_unpack", "rr_plan_bucket_items", "rr_plan_work_units", "rr_pack", "rr_unpack", "rr_verify",
             "rr_pack_range", "rr_unpack_range", "rr_verify_range", "rr_clear_range",
             "rr_unpack_verify", "rr_unpack_verify_range", "rr_unpack_verify_async",
             "rr_verify_noalloc",
@@ -350,18 +350,21 @@ class Plan:
                "rr_plan_bucket_items")
         return pf, uf
 
-    def unpack_units(self):
-        """The verifying unpack's work units: (first unpack item of each unit,
-        plus one past the last; first unit of each bucket, n_buckets + 1)."""
+    def work_units(self, which: str = "unpack"):
+        """The bulk-copy engine's work units of one table ("pack", "pack_full" or
+        "unpack"): (first item of each unit, plus one past the last; first unit
+        of each bucket, n_buckets + 1, or None for "pack_full")."""
         import numpy as np
+        w = {"pack": 0, "pack_full": 1, "unpack": 2}[which]
         n = ctypes.c_int32(0)
-        _check(_lib.rr_plan_unpack_units(self._h, ctypes.byref(n), None, None),
-               "rr_plan_unpack_units")
+        _check(_lib.rr_plan_work_units(self._h, w, ctypes.byref(n), None, None),
+               "rr_plan_work_units")
         first = np.zeros(n.value + 1, np.uint32)
-        bucket = np.zeros(self.n_buckets + 1, np.uint32)
+        bucket = None if which == "pack_full" else np.zeros(self.n_buckets + 1, np.uint32)
         P = ctypes.POINTER(ctypes.c_uint32)
-        _check(_lib.rr_plan_unpack_units(self._h, ctypes.byref(n), first.ctypes.data_as(P),
-                                         bucket.ctypes.data_as(P)), "rr_plan_unpack_units")
+        _check(_lib.rr_plan_work_units(self._h, w, ctypes.byref(n), first.ctypes.data_as(P),
+                                       None if bucket is None else bucket.ctypes.data_as(P)),
+               "rr_plan_work_units")
         return first, bucket
 
     def destroy(self) -> None:

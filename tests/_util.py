@@ -264,16 +264,23 @@ def check_partition(first, n_items):
     assert np.all(np.diff(first) >= 0)
 
 
-def check_units(plan, n_items):
-    """The verifying unpack's work units tile each bucket's unpack items: no
-    unit is empty or spans two buckets, and bucket b's units cover exactly its
-    items, so any bucket range is a contiguous run of whole units."""
-    first, bucket_unit = plan.unpack_units()
-    _, bucket_first = plan.bucket_items()
+def check_units(plan, n_items, which="unpack"):
+    """The bulk-copy engine's work units of one table tile its items: no unit
+    is empty; in the per-bucket tables ("pack", "unpack") no unit spans two
+    buckets and bucket b's units cover exactly its items, so any bucket range
+    is a contiguous run of whole units."""
+    first, bucket_unit = plan.work_units(which)
     first = first.astype(np.int64)
-    bucket_unit = bucket_unit.astype(np.int64)
+    if n_items == 0:
+        assert len(first) == 1 and first[0] == 0
+        return first, bucket_unit
     assert first[0] == 0 and first[-1] == n_items
     assert np.all(np.diff(first) > 0)
+    if bucket_unit is None:
+        return first, None
+    pack_first, unpack_first = plan.bucket_items()
+    bucket_first = pack_first if which == "pack" else unpack_first
+    bucket_unit = bucket_unit.astype(np.int64)
     assert bucket_unit[0] == 0 and bucket_unit[-1] == len(first) - 1
     assert np.all(np.diff(bucket_unit) >= 0)
     for b in range(plan.n_buckets):

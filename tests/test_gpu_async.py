@@ -127,7 +127,7 @@ def test_claimed_units_on_any_grid(grid):
     own) all give the oracle's tensors and the same verdicts, for the whole
     sync and for bucket ranges."""
     desc, plan, buf = packed("tiny-moe-tp2", grid_blocks=grid)
-    first, bucket_unit = plan.unpack_units()
+    first, bucket_unit = plan.work_units("unpack")
     assert len(first) - 1 > 3 and len(first) - 1 < 2048
     bl = H.bucket_list(buf)
     bl[6][40] ^= 0x04

@@ -72,6 +72,10 @@ def run_and_compare(desc, **opt):
     U.check_partition(ffirst, len(fitems))
     starts = ffirst[:-1][ffirst[:-1] < len(fitems)]
     assert not np.any(fitems["kind"][starts] == U.ITEM_FAN_DST)
+    U.check_units(p, len(items), "pack")
+    if p.stats()["n_pack_full_items"]:
+        funits, _ = U.check_units(p, len(fitems), "pack_full")
+        assert not np.any(fitems["kind"][funits[:-1]] == U.ITEM_FAN_DST)
     got = U.check_and_run_pack(fitems, shards, p.n_buckets, p.bucket_bytes, p.shard_bytes)
     np.testing.assert_array_equal(got, want)
     uitems, ufirst = p.export_unpack()
@@ -150,26 +154,52 @@ def test_full_size_tables_are_consistent():
     assert np.all(items["kind"][data] == U.ITEM_F32_VEC)
 
 
-@pytest.mark.parametrize("name", ["qwen3-0.6b", "qwen3-8b", "qwen3-30b-a3b-fsdp2-tp8"])
-def test_unpack_work_units_on_full_size_tables(name):
-    """Units of equal weight (a byte copied by vectors weighs 2, one by
-    elements 4, a read-only one 1, an item 1024 more): at most 1 MiB, or less
-    where that leaves a block of the grid fewer than 32; none heavier than
-    that plus one item, and only a bucket's last unit much lighter."""
+def unit_weights(p, which):
+    """Each unit's weight, by the planner's balancing rule (pack: 6 per fp32
+    element by vectors, 12 element by element, 4 and 8 for bf16, 2 per zero
+    element; unpack: 2 per byte copied by vectors, 4 element by element, 1 per
+    byte only read; 1024 more per item, nothing for a fan-out destination)."""
+    if which == "unpack":
+        items, _ = p.export_unpack()
+        n = items["nbytes"].astype(np.int64)
+        per = np.select([items["kind"] == U.ITEM_COPY_VEC, items["kind"] == U.ITEM_COPY_SCALAR],
+                        [2, 4], 1)
+        w = per * n + 1024
+    else:
+        items, _ = p.export_pack_full() if which == "pack_full" else p.export_pack()
+        n = items["row_len"].astype(np.int64) * items["n_rows"]
+        k = items["kind"]
+        per = np.select([k == U.ITEM_F32_VEC, k == U.ITEM_F32_SCALAR, k == U.ITEM_BF16_VEC,
+                         k == U.ITEM_BF16_SCALAR, k == U.ITEM_FAN_F32, k == U.ITEM_FAN_BF16],
+                        [6, 12, 4, 8, 6, 4], 2)
+        w = np.where(k == U.ITEM_FAN_DST, 0, per * n + 1024)
+    return items, w
+
+
+@pytest.mark.parametrize("name,which", [("qwen3-0.6b", "unpack"), ("qwen3-8b", "unpack"),
+                                        ("qwen3-30b-a3b-fsdp2-tp8", "unpack"),
+                                        ("qwen3-0.6b", "pack"), ("qwen3-8b", "pack"),
+                                        ("qwen3-30b-a3b-fsdp2-tp8", "pack_full")])
+def test_work_units_on_full_size_tables(name, which):
+    """Units of equal weight: at most 1 MiB, or less where that would leave a
+    block of the grid fewer than 32; none heavier than that plus one item (a
+    fan-out group counts as one), and only a bucket's last unit much lighter."""
     p = host_plan(U.workload_desc(name))
-    items, _ = p.export_unpack()
-    first, bucket_unit = U.check_units(p, len(items))
-    nbytes = items["nbytes"].astype(np.int64)
-    per_byte = np.select([items["kind"] == U.ITEM_COPY_VEC, items["kind"] == U.ITEM_COPY_SCALAR],
-                         [2, 4], 1)
-    w = per_byte * nbytes + 1024
-    grid = p.stats()["unpack_grid_blocks"]
+    items, w = unit_weights(p, which)
+    first, bucket_unit = U.check_units(p, len(items), which)
+    grid = p.stats()["unpack_grid_blocks" if which == "unpack" else "grid_blocks"]
     unit = min(1 << 20, max((1 << 20) // 8, int(w.sum()) // (32 * grid)))
+    heaviest = w.max()
+    if which == "pack_full":   # a fan-out head and its destinations stay together
+        heads = np.flatnonzero(w > 0)
+        heaviest = max(heaviest, int(np.add.reduceat(w, heads).max()))
     unit_w = np.add.reduceat(w, first[:-1])
-    assert unit_w.max() <= unit + w.max()
+    assert unit_w.max() <= unit + heaviest
     last = np.zeros(len(unit_w), bool)
-    last[bucket_unit[1:] - 1] = True
-    assert np.all(unit_w[~last] >= unit // 2 - w.max())
+    last[-1] = True
+    if bucket_unit is not None:
+        last[bucket_unit[1:][np.diff(bucket_unit) > 0] - 1] = True
+    assert np.all(unit_w[~last] >= unit // 2 - heaviest)
     assert len(unit_w) >= 16 * grid
 
 
