@@ -394,17 +394,20 @@ rr_status rr_unpack_verify_range(const rr_plan* plan, int32_t first_bucket, int3
 rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32_t* unpack_first);
 
 /* Work units of the bulk-copy engine.  Blocks drain HBM at unequal rates, so
- * a launch does not fix each block's share: block g takes the launch's unit g,
- * then claims the next unclaimed unit (an atomic counter) until none are left,
- * and all blocks finish together.  Each table's items are cut into units of
- * roughly equal weight: about 1 MiB of traffic, less on small plans, so that
- * every block of the grid has a few dozen.
- *   which: RR_UNITS_PACK (the pack items; a unit never spans two buckets, so a
- *     bucket range is a run of whole units), RR_UNITS_PACK_FULL (the table a
- *     pack over every bucket runs, as rr_plan_export_pack_full gives it: with
- *     fan-out items, a unit never starting on a fan-out destination item, or
- *     the pack items and their units where the plan has no fan-out items),
- *     RR_UNITS_UNPACK (the unpack items, per bucket like RR_UNITS_PACK).
+ * a launch does not fix each block's whole share: block g takes the launch's
+ * unit g, then claims the next unclaimed unit (an atomic counter) until none
+ * are left, and all blocks finish together.
+ *   which:
+ *   RR_UNITS_PACK, RR_UNITS_UNPACK: the units of a bucket-range pack, and of
+ *     every unpack and verifying unpack.  Each bucket's items are cut into
+ *     units of about 1 MiB of traffic (less on small plans, so that a block of
+ *     the grid has a few dozen), none empty, none spanning two buckets; a
+ *     range's units are the run of its buckets' units.
+ *   RR_UNITS_PACK_FULL: the units of a pack over every bucket, over the table
+ *     rr_plan_export_pack_full gives.  Units 0 .. grid - 1 are equal
+ *     contiguous shares of 70% of the table's weight, one per block; the
+ *     units after them cut the rest to the size above.  A cut never falls
+ *     before a fan-out destination item.  Units may be empty.
  *   *n_units: the number of units.
  *   unit_first (NULL, or n_units + 1 entries): unit u holds items
  *     [unit_first[u], unit_first[u + 1]) of that table.

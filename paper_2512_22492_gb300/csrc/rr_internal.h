@@ -67,7 +67,8 @@ struct rr_plan {
     std::vector<uint32_t> unpack_bucket_unit;
     std::vector<uint32_t> pack_unit_first;
     std::vector<uint32_t> pack_bucket_unit;
-    std::vector<uint32_t> full_unit_first;      // the whole-sync table's (whole launches only)
+    std::vector<uint32_t> pack_whole_unit_first;   // a pack over every bucket: own units
+                                                   //   (one per block), then claimed ones
     std::vector<uint32_t> pack_bucket_first;    // n_buckets + 1: first pack item of bucket b
     std::vector<unsigned long long> pack_weight_prefix;    // items + 1: balancing weights,
     std::vector<unsigned long long> unpack_weight_prefix;  // summed (bucket-range calls)
@@ -95,7 +96,7 @@ struct rr_plan {
     uint32_t* d_unpack_block_first = nullptr;
     uint32_t* d_unpack_unit_first = nullptr;
     uint32_t* d_pack_unit_first = nullptr;
-    uint32_t* d_full_unit_first = nullptr;
+    uint32_t* d_pack_whole_unit_first = nullptr;
     // Unit-claim counters of launches that have no per-call scratch (rr_pack,
     // rr_unpack): a slot is handed to a launch only once the event recorded
     // after its previous launch has completed; that launch left it zeroed.

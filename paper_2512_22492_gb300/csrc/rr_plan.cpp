@@ -411,26 +411,31 @@ void bucket_units(const std::vector<Item>& items, const std::vector<uint32_t>& b
     first.push_back(bucket_first.empty() ? 0 : bucket_first.back());
 }
 
-// The same for a table that a launch always takes whole (the whole-sync pack
-// table, whose fan-out groups write several buckets): equal shares of its
-// weight, a unit never starting on a fan-out destination item.
+// Units for a launch over every bucket (the table it runs is fixed): blocks
+// first drain kOwnShare of the table's weight in equal contiguous shares (unit
+// g < grid is block g's own: no claims, long runs), then claim units of about
+// unit_weight over the rest.  A cut never falls before a fan-out destination
+// item (a head and its destinations stay in one unit).
+constexpr int64_t kOwnShareNum = 7, kOwnShareDen = 10;
 template <class Item, class W>
-void even_units(const std::vector<Item>& items, int64_t unit_weight, std::vector<uint32_t>& first,
-                W w) {
-    first.assign(1, 0);
-    if (items.empty()) return;
+void whole_units(const std::vector<Item>& items, int32_t grid, int64_t unit_weight,
+                 std::vector<uint32_t>& first, W w) {
     int64_t total = 0;
     for (const Item& it : items) total += w(it);
-    const int64_t n = std::max<int64_t>(1, (total + unit_weight - 1) / unit_weight);
-    int64_t cum = 0, k = 1;
-    for (size_t i = 0; i + 1 < items.size() && k < n; ++i) {
+    const int64_t own = total * kOwnShareNum / kOwnShareDen;
+    const int64_t claimed = std::max<int64_t>(1, (total - own + unit_weight - 1) / unit_weight);
+    const int64_t U = int64_t(grid) + claimed;
+    auto target = [&](int64_t g) {   // weight before unit g
+        return g <= grid ? own * g / grid : own + (total - own) * (g - grid) / claimed;
+    };
+    first.assign(size_t(U) + 1, uint32_t(items.size()));
+    first[0] = 0;
+    int64_t cum = 0, g = 1;
+    for (size_t i = 0; i < items.size() && g < U; ++i) {
         cum += w(items[i]);
-        if (cum * n >= total * k && items[i + 1].kind != RR_ITEM_FAN_DST) {
-            first.push_back(uint32_t(i + 1));
-            while (k < n && cum * n >= total * k) ++k;
-        }
+        if (i + 1 < items.size() && items[i + 1].kind == RR_ITEM_FAN_DST) continue;
+        while (g < U && cum >= target(g)) first[size_t(g++)] = uint32_t(i + 1);
     }
-    first.push_back(uint32_t(items.size()));
 }
 
 // Claimed-unit weight for a table: about kUnitsPerBlock units per block of the
@@ -768,7 +773,6 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     // Whole-sync table: the grouped blocks' plain items give way to fan-out groups.
     P->full_items.clear();
     P->full_block_first.clear();
-    P->full_unit_first.clear();
     if (!groups.empty()) {
         std::vector<char> drop(P->pack_items.size(), 0);
         for (auto [lo, hi] : fanned)
@@ -803,9 +807,12 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
             f[g] = std::max(f[g], f[g - 1]);
             while (f[g] < P->full_items.size() && P->full_items[f[g]].kind == RR_ITEM_FAN_DST) ++f[g];
         }
-        even_units(P->full_items, unit_weight_for(P->full_items, P->grid_blocks, pack_weight),
-                   P->full_unit_first, pack_weight);
     }
+
+    // Units of a pack over every bucket.
+    const std::vector<rr_pack_item>& whole = P->full_items.empty() ? P->pack_items : P->full_items;
+    whole_units(whole, P->grid_blocks, unit_weight_for(whole, P->grid_blocks, pack_weight),
+                P->pack_whole_unit_first, pack_weight);
 
     rr_plan_stats& s = P->stats;
     s.n_pack_items = int64_t(P->pack_items.size());
@@ -1005,13 +1012,11 @@ rr_status rr_plan_work_units(const rr_plan* P, int32_t which, int32_t* n_units,
     const std::vector<uint32_t>* bu = nullptr;
     switch (which) {
         case RR_UNITS_PACK: first = &P->pack_unit_first; bu = &P->pack_bucket_unit; break;
-        case RR_UNITS_PACK_FULL:   // the table a whole-sync pack runs
-            first = P->full_items.empty() ? &P->pack_unit_first : &P->full_unit_first;
-            break;
+        case RR_UNITS_PACK_FULL: first = &P->pack_whole_unit_first; break;
         case RR_UNITS_UNPACK: first = &P->unpack_unit_first; bu = &P->unpack_bucket_unit; break;
-        default: return rr_fail(RR_EINVAL, "which must be RR_UNITS_PACK, _PACK_FULL or _UNPACK");
+        default: return rr_fail(RR_EINVAL, "which must be one of the RR_UNITS_ values");
     }
-    if (bucket_unit && !bu) return rr_fail(RR_EINVAL, "the whole-sync table has no bucket units");
+    if (bucket_unit && !bu) return rr_fail(RR_EINVAL, "the whole-sync pack's units have no bucket index");
     *n_units = first->empty() ? 0 : int32_t(first->size()) - 1;
     if (unit_first) std::copy(first->begin(), first->end(), unit_first);
     if (bucket_unit) std::copy(bu->begin(), bu->end(), bucket_unit);

@@ -351,16 +351,17 @@ class Plan:
         return pf, uf
 
     def work_units(self, which: str = "unpack"):
-        """The bulk-copy engine's work units of one table ("pack", "pack_full" or
-        "unpack"): (first item of each unit, plus one past the last; first unit
-        of each bucket, n_buckets + 1, or None for "pack_full")."""
+        """The bulk-copy engine's work units: "pack" and "unpack" (per bucket:
+        bucket-range packs, every unpack) or "pack_full" (a pack over every
+        bucket).  Returns (first item of each unit, plus one past the last;
+        first unit of each bucket, n_buckets + 1, or None for "pack_full")."""
         import numpy as np
         w = {"pack": 0, "pack_full": 1, "unpack": 2}[which]
         n = ctypes.c_int32(0)
         _check(_lib.rr_plan_work_units(self._h, w, ctypes.byref(n), None, None),
                "rr_plan_work_units")
         first = np.zeros(n.value + 1, np.uint32)
-        bucket = None if which == "pack_full" else np.zeros(self.n_buckets + 1, np.uint32)
+        bucket = None if which.endswith("_full") else np.zeros(self.n_buckets + 1, np.uint32)
         P = ctypes.POINTER(ctypes.c_uint32)
         _check(_lib.rr_plan_work_units(self._h, w, ctypes.byref(n), first.ctypes.data_as(P),
                                        None if bucket is None else bucket.ctypes.data_as(P)),

@@ -265,19 +265,24 @@ def check_partition(first, n_items):
 
 
 def check_units(plan, n_items, which="unpack"):
-    """The bulk-copy engine's work units of one table tile its items: no unit
-    is empty; in the per-bucket tables ("pack", "unpack") no unit spans two
-    buckets and bucket b's units cover exactly its items, so any bucket range
-    is a contiguous run of whole units."""
+    """The bulk-copy engine's work units of one table tile its items.  In the
+    per-bucket tables ("pack", "unpack") no unit is empty or spans two buckets
+    and bucket b's units cover exactly its items, so any bucket range is a
+    contiguous run of whole units; the whole-sync pack's ("pack_full") start
+    with one own unit per block of the grid."""
     first, bucket_unit = plan.work_units(which)
     first = first.astype(np.int64)
+    if which == "pack_full":
+        # One own unit per block, then the claimed ones; units may be empty.
+        grid = plan.stats()["grid_blocks"]
+        assert len(first) >= grid + 2
+        assert first[0] == 0 and first[-1] == n_items and np.all(np.diff(first) >= 0)
+        return first, None
     if n_items == 0:
         assert len(first) == 1 and first[0] == 0
         return first, bucket_unit
     assert first[0] == 0 and first[-1] == n_items
     assert np.all(np.diff(first) > 0)
-    if bucket_unit is None:
-        return first, None
     pack_first, unpack_first = plan.bucket_items()
     bucket_first = pack_first if which == "pack" else unpack_first
     bucket_unit = bucket_unit.astype(np.int64)

@@ -73,9 +73,9 @@ def run_and_compare(desc, **opt):
     starts = ffirst[:-1][ffirst[:-1] < len(fitems)]
     assert not np.any(fitems["kind"][starts] == U.ITEM_FAN_DST)
     U.check_units(p, len(items), "pack")
-    if p.stats()["n_pack_full_items"]:
-        funits, _ = U.check_units(p, len(fitems), "pack_full")
-        assert not np.any(fitems["kind"][funits[:-1]] == U.ITEM_FAN_DST)
+    funits, _ = U.check_units(p, len(fitems), "pack_full")
+    starts = funits[:-1][funits[:-1] < len(fitems)]
+    assert not np.any(fitems["kind"][starts] == U.ITEM_FAN_DST)
     got = U.check_and_run_pack(fitems, shards, p.n_buckets, p.bucket_bytes, p.shard_bytes)
     np.testing.assert_array_equal(got, want)
     uitems, ufirst = p.export_unpack()
@@ -159,7 +159,7 @@ def unit_weights(p, which):
     element by vectors, 12 element by element, 4 and 8 for bf16, 2 per zero
     element; unpack: 2 per byte copied by vectors, 4 element by element, 1 per
     byte only read; 1024 more per item, nothing for a fan-out destination)."""
-    if which == "unpack":
+    if which.startswith("unpack"):
         items, _ = p.export_unpack()
         n = items["nbytes"].astype(np.int64)
         per = np.select([items["kind"] == U.ITEM_COPY_VEC, items["kind"] == U.ITEM_COPY_SCALAR],
@@ -178,29 +178,45 @@ def unit_weights(p, which):
 
 @pytest.mark.parametrize("name,which", [("qwen3-0.6b", "unpack"), ("qwen3-8b", "unpack"),
                                         ("qwen3-30b-a3b-fsdp2-tp8", "unpack"),
-                                        ("qwen3-0.6b", "pack"), ("qwen3-8b", "pack"),
-                                        ("qwen3-30b-a3b-fsdp2-tp8", "pack_full")])
-def test_work_units_on_full_size_tables(name, which):
-    """Units of equal weight: at most 1 MiB, or less where that would leave a
-    block of the grid fewer than 32; none heavier than that plus one item (a
-    fan-out group counts as one), and only a bucket's last unit much lighter."""
+                                        ("qwen3-0.6b", "pack"), ("qwen3-8b", "pack")])
+def test_bucket_units_on_full_size_tables(name, which):
+    """Per-bucket units of equal weight: at most 1 MiB, or less where that would
+    leave a block of the grid fewer than 32; none heavier than that plus one
+    item, and only a bucket's last unit much lighter."""
     p = host_plan(U.workload_desc(name))
     items, w = unit_weights(p, which)
     first, bucket_unit = U.check_units(p, len(items), which)
     grid = p.stats()["unpack_grid_blocks" if which == "unpack" else "grid_blocks"]
     unit = min(1 << 20, max((1 << 20) // 8, int(w.sum()) // (32 * grid)))
-    heaviest = w.max()
-    if which == "pack_full":   # a fan-out head and its destinations stay together
-        heads = np.flatnonzero(w > 0)
-        heaviest = max(heaviest, int(np.add.reduceat(w, heads).max()))
     unit_w = np.add.reduceat(w, first[:-1])
-    assert unit_w.max() <= unit + heaviest
+    assert unit_w.max() <= unit + w.max()
     last = np.zeros(len(unit_w), bool)
-    last[-1] = True
-    if bucket_unit is not None:
-        last[bucket_unit[1:][np.diff(bucket_unit) > 0] - 1] = True
-    assert np.all(unit_w[~last] >= unit // 2 - heaviest)
+    last[bucket_unit[1:][np.diff(bucket_unit) > 0] - 1] = True
+    assert np.all(unit_w[~last] >= unit // 2 - w.max())
     assert len(unit_w) >= 16 * grid
+
+
+@pytest.mark.parametrize("name", ["qwen3-0.6b", "qwen3-8b", "qwen3-30b-a3b-fsdp2-tp8"])
+def test_whole_pack_units_on_full_size_tables(name):
+    """A pack over every bucket: one own unit per block, together 70% of the
+    weight in equal shares (to within one item, or one fan-out group), then
+    claimed units of at most the per-bucket size plus one item."""
+    which = "pack_full"
+    p = host_plan(U.workload_desc(name))
+    items, w = unit_weights(p, which)
+    first, _ = U.check_units(p, len(items), which)
+    grid = p.stats()["grid_blocks"]
+    heaviest = int(w.max())
+    if which == "pack_full":   # a fan-out head and its destinations stay together
+        heaviest = int(np.add.reduceat(w, np.flatnonzero(w > 0)).max())
+    cum = np.concatenate([[0], np.cumsum(w)])
+    unit_w = cum[first[1:]] - cum[first[:-1]]
+    total = int(cum[-1])
+    own = total * 7 // 10
+    assert abs(int(cum[first[grid]]) - own) <= heaviest
+    assert np.all(np.abs(unit_w[:grid] - own / grid) <= heaviest + 1)
+    unit = min(1 << 20, max((1 << 20) // 8, total // (32 * grid)))
+    assert unit_w[grid:].max() <= unit + heaviest
 
 
 def test_fan_out_groups_on_full_size_tables():
