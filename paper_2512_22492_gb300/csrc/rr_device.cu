@@ -1049,23 +1049,25 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                 break;
             case PC_FAN:   // pack only
                 if constexpr (MODE == 0) {
-                    // Units of work: each slice's rows in q parts (q spreads the slices
-                    // over all consumer warps); one warp per unit, one sum per unit.
+                    // Units of work: each slice's 16-byte output vectors in q parts
+                    // (q spreads the slices over all consumer warps, whatever the
+                    // number of rows staged); one warp per unit, one sum per unit.
                     const uint32_t nd = p.n;
                     const uint32_t q = (kConsumerWarps + nd - 1) / nd;
                     for (uint32_t u = warp - 1; u < nd * q; u += kConsumerWarps) {
                         const rr_pack_item d = fan_dst[s][u / q];
                         const uint32_t part = u % q;
-                        const uint32_t r0 = p.rows * part / q, r1 = p.rows * (part + 1) / q;
-                        const uint32_t vpr = d.row_len >> 3, nv = (r1 - r0) * vpr;
+                        const uint32_t vpr = d.row_len >> 3, nv_all = p.rows * vpr;
+                        const uint32_t v0 = nv_all * part / q, v1 = nv_all * (part + 1) / q;
+                        // Lane l starts at vector v0 + l (row r, vector c of the row)
+                        // and steps 32 vectors: dq rows and dr vectors at a time.
                         const uint32_t dq = 32 / vpr, dr = 32 - dq * vpr;
-                        const char* base =
-                            st + ((uint64_t)r0 * p.row_len + (uint32_t)d.src) * p.es;
+                        const char* base = st + (uint32_t)d.src * p.es;
                         char* out = bulk_bucket(a, d.bucket, a.n_shards) + d.dst_off +
-                                    2ull * (p.sum_off + r0) * d.row_len;
-                        uint32_t r = lane / vpr, c = lane - r * vpr;
+                                    2ull * p.sum_off * d.row_len;
+                        uint32_t r = (v0 + lane) / vpr, c = (v0 + lane) - r * vpr;
                         unsigned long long am = 0;
-                        for (uint32_t v = lane; v < nv; v += 32) {
+                        for (uint32_t v = v0 + lane; v < v1; v += 32) {
                             const char* q8 = base + ((uint64_t)r * p.row_len + 8u * c) * p.es;
                             uint4 o;
                             if (p.es == 4) {

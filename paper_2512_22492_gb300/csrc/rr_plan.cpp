@@ -34,14 +34,14 @@ thread_local std::string g_error;
 
 constexpr int64_t kDefaultChunkBytes = 32 * 1024;
 constexpr int64_t kItemOverhead = 1024;   // balancing weight of one item, in bytes
-constexpr int64_t kUnitWeight = 1 << 20;   // largest claimed work unit of the verifying unpack
-constexpr int32_t kUnitsPerBlock = 32;     //   (weight), and the units wanted per block
+constexpr int64_t kUnitWeight = 1 << 20;   // largest claimed work unit (weight), and the
+constexpr int32_t kUnitsPerBlock = 32;     //   units wanted per block of the grid
 constexpr int64_t kMaxShardOffset = (int64_t(1) << 48) - 1;
-// Fan-out groups: column slices narrower than kFanSliceBytes of source per row,
-// at most kMaxFanDst of them, over a joint span of at most kFanMaxRowBytes.
-constexpr int64_t kFanSliceBytes = 1024;
+// Fan-out groups: at most kMaxFanDst column slices over a joint span of at
+// most kFanMaxRowBytes of source per row (one pack stage of the bulk-copy
+// engine holds a whole row; the kernel refuses a wider head).
 constexpr int64_t kMaxFanDst = 16;
-constexpr int64_t kFanMaxRowBytes = 16 * 1024;
+constexpr int64_t kFanMaxRowBytes = 48 * 1024;
 
 int64_t align_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
@@ -684,7 +684,7 @@ std::vector<FanGroup> find_fan_groups(const rr_plan* P, const rr_dst_layout* dst
         const int64_t cmin = m[0].col0;
         bool ok = (C * es) % 16 == 0 && P->bucket_bytes % 16 == 0;
         for (size_t i = 0; i < m.size() && ok; ++i) {
-            ok = m[i].ncols % 8 == 0 && m[i].ncols * es < kFanSliceBytes &&
+            ok = m[i].ncols % 8 == 0 &&
                  ((m[i].col0 - cmin) * es) % 16 == 0 && m[i].pos % 16 == 0 &&
                  (i == 0 || m[i].col0 == m[i - 1].col0 + m[i - 1].ncols);
         }

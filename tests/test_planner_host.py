@@ -220,23 +220,31 @@ def test_whole_pack_units_on_full_size_tables(name):
 
 
 def test_fan_out_groups_on_full_size_tables():
-    """Qwen3-30B-A3B FSDP2 -> TP=8: every expert down_proj's eight 96-column slices
-    form one group per shard run of rows (metadata only)."""
+    """Qwen3-30B-A3B FSDP2 -> TP=8: every expert down_proj's eight 96-column slices,
+    and every attention o_proj's eight 512-column slices, form one group per
+    shard run of rows (metadata only)."""
     desc = U.workload_desc("qwen3-30b-a3b-fsdp2-tp8")
     p = host_plan(desc)
     items, first = p.export_pack_full()
     U.check_partition(first, len(items))
     kind = items["kind"]
     heads = np.flatnonzero((kind == U.ITEM_FAN_F32) | (kind == U.ITEM_FAN_BF16))
+    assert np.all(items["dst_off"][heads] == 8)
+    assert set(np.unique(items["row_len"][heads]).tolist()) == {768, 4096}
+    expert = heads[items["row_len"][heads] == 768]
+    o_proj = heads[items["row_len"][heads] == 4096]
     # One head per shard run of 256 rows, and a few more where a bucket boundary
     # cuts a run; a row whose slice would straddle a boundary goes out as plain items.
-    assert 48 * 128 * 8 <= len(heads) < 48 * 128 * 8 + 64
-    assert np.all(items["dst_off"][heads] == 8) and np.all(items["row_len"][heads] == 768)
-    assert np.all(items["n_rows"][heads] <= 256)
-    fanned_rows = int(items["n_rows"][heads].astype(np.int64).sum())
+    assert 48 * 128 * 8 <= len(expert) < 48 * 128 * 8 + 64
+    assert np.all(items["n_rows"][expert] <= 256)
+    fanned_rows = int(items["n_rows"][expert].astype(np.int64).sum())
     assert 48 * 128 * 2048 - 64 <= fanned_rows <= 48 * 128 * 2048
+    o_rows = int(items["n_rows"][o_proj].astype(np.int64).sum())
+    assert 48 * 2048 - 64 <= o_rows <= 48 * 2048
     dsts = np.flatnonzero(kind == U.ITEM_FAN_DST)
-    assert len(dsts) == 8 * len(heads) and np.all(items["row_len"][dsts] == 96)
+    assert len(dsts) == 8 * len(heads)
+    dst_width = items["row_len"][dsts].reshape(-1, 8)
+    assert np.all(dst_width == np.where(items["row_len"][heads] == 768, 96, 512)[:, None])
     # Every bucket byte is written exactly once: plain items plus fan-out slices.
     n = items["row_len"].astype(np.int64) * items["n_rows"]
     plain = kind < U.ITEM_FAN_F32
