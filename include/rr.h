@@ -44,17 +44,24 @@
  *
  * Memory.  Every pointer argument named "device" is CUDA device memory of
  * the device the plan was created on, owned by the caller; every device
- * pointer must be 16-byte aligned.  The plan owns its device segment tables
- * and a small verify scratch area; rr_pack and rr_unpack allocate nothing.
+ * pointer must be 16-byte aligned.  The plan owns its device segment tables,
+ * a small verify scratch area and 16 work-unit counters (rr_plan_work_units);
+ * rr_pack and rr_unpack allocate nothing.
  *
  * Errors.  Every call returns rr_status.  Argument and layout errors are
  * reported synchronously and leave outputs untouched; RR_ECUDA means a CUDA
  * call failed (rr_last_error() has the CUDA message).  rr_last_error()
  * returns a per-thread description of the most recent failure.
  *
- * Threads and streams.  A plan is immutable after creation; rr_pack and
- * rr_unpack may run on it concurrently on different streams as long as
- * their outputs are distinct.  rr_verify serialises on the plan.
+ * Threads and streams.  A plan's tables are immutable after creation; rr_pack
+ * and rr_unpack may run on it concurrently on different streams, and from
+ * different threads, as long as their outputs are distinct (each launch
+ * takes its own work-unit counter, under a lock).  rr_verify serialises on
+ * the plan.  The stream-ordered calls (rr_pack(_range), rr_unpack(_range),
+ * rr_clear_range, rr_unpack_verify_async) may be captured into a CUDA graph;
+ * the blocking ones (rr_verify(_range), rr_unpack_verify(_range),
+ * rr_plan_check) may not, and rr_unpack_verify_async takes their place in a
+ * graph.
  */
 #ifndef RR_H
 #define RR_H
@@ -414,13 +421,17 @@ rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32
  *   bucket_unit (NULL, or n_buckets + 1 entries; must be NULL for
  *     RR_UNITS_PACK_FULL): the units of bucket b are [bucket_unit[b],
  *     bucket_unit[b + 1]).
- * Call with both arrays NULL to learn n_units.
- * Which launches claim: the verifying unpack always (its counter lives in the
- * call's scratch); rr_pack and rr_unpack when one of the plan's 16 counter
- * slots is free -- a slot is reused only after the launch that last held it
- * has completed -- and the stream is not capturing a graph.  Otherwise the
- * launch splits its items evenly over the grid, as a captured launch always
- * does. */
+ * Call with both arrays NULL to learn n_units.  Host-only plans have units
+ * too.  Errors: RR_EINVAL for a NULL plan or n_units, an unknown `which`, or
+ * a bucket_unit array with RR_UNITS_PACK_FULL; nothing is written then.
+ * Which launches of the bulk-copy engine claim (the register path never
+ * does): the verifying unpack always, its counter kept in the call's scratch
+ * (the plan's for the blocking forms, the caller's for
+ * rr_unpack_verify_async); rr_pack and rr_unpack when one of the plan's 16
+ * counter slots is free -- a slot is reused only after the launch that last
+ * held it has completed -- and the stream is not capturing a graph.
+ * Otherwise the launch splits its items evenly over the grid, as a captured
+ * launch always does.  Which of these runs changes no output byte. */
 enum { RR_UNITS_PACK = 0, RR_UNITS_PACK_FULL = 1, RR_UNITS_UNPACK = 2 };
 rr_status rr_plan_work_units(const rr_plan* plan, int32_t which, int32_t* n_units,
                              uint32_t* unit_first, uint32_t* bucket_unit);

@@ -133,6 +133,17 @@ int main(int argc, char** argv) {
     CHECK(rr_plan_tensors(plan, numel, toff) == RR_OK, "tensors");
     CHECK(numel[0] == 32 && numel[1] == 8 && toff[0] == 0 && toff[1] == 256 && toff[3] == 256,
           "tensor geometry");
+    int32_t n_units = -1;
+    uint32_t unit_first[64], bucket_unit[N_BUCKETS + 1];
+    CHECK(rr_plan_work_units(plan, RR_UNITS_UNPACK, &n_units, NULL, NULL) == RR_OK &&
+              n_units >= N_BUCKETS && n_units < 64,
+          "unit count");
+    CHECK(rr_plan_work_units(plan, RR_UNITS_UNPACK, &n_units, unit_first, bucket_unit) == RR_OK &&
+              unit_first[0] == 0 && bucket_unit[0] == 0 && bucket_unit[N_BUCKETS] == (uint32_t)n_units,
+          "unit tables");
+    CHECK(rr_plan_work_units(plan, 7, &n_units, NULL, NULL) == RR_EINVAL, "unknown unit table");
+    CHECK(rr_plan_work_units(plan, RR_UNITS_PACK_FULL, &n_units, NULL, bucket_unit) == RR_EINVAL,
+          "no bucket index for the whole-sync units");
     rr_plan_stats st;
     CHECK(rr_plan_get_stats(plan, &st) == RR_OK, "stats");
     CHECK(st.pack_bytes_read == 2 * (32 * 4 + 8 * 2) && st.pack_bytes_written == 6 * BUCKET,

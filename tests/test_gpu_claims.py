@@ -9,7 +9,9 @@ every one of those paths and compare bytes with the oracle:
     sleep kernel, so that none of them can complete before the rest are
     enqueued);
   - two streams packing and unpacking their own buffers at once;
-  - the whole step captured into a CUDA graph and replayed on new inputs.
+  - the whole step captured into a CUDA graph and replayed on new inputs;
+  - a resumed pull's range calls (clear, pack, unpack, stream-ordered check)
+    captured into a CUDA graph and replayed over spoiled buckets.
 """
 import numpy as np
 import pytest
@@ -165,4 +167,64 @@ def test_step_captured_in_a_cuda_graph():
         for t in range(plan.n_tensors):
             np.testing.assert_array_equal(H.tensor_host(other, t), want_t[t])
         assert result.cpu().tolist() == [0, -1]
+    rr.rr_plan_check(plan)
+
+
+def test_range_calls_captured_in_a_cuda_graph():
+    """A resumed pull's stream-ordered calls captured once: clear buckets
+    [2, 9), pack them again, unpack them and check them; the replay restores
+    exactly the oracle's bytes for those buckets and their tensors' bytes."""
+    desc, m, plan, L, shards, want, want_cs = setup()
+    buf = H.alloc(plan)
+    H.fill_from_host(buf, shards)
+    H.pack(buf)
+    H.unpack(buf)
+    torch.cuda.synchronize()
+    first, count = 2, 7
+    scratch = torch.zeros(plan.n_buckets + 4, dtype=torch.int64, device="cuda")
+    result = torch.full((2,), 7, dtype=torch.int64, device="cuda")
+    bad = torch.full((plan.n_buckets,), 9, dtype=torch.uint8, device="cuda")
+
+    def calls():
+        rr.rr_clear_range(plan, first, count, buf.buckets)
+        rr.rr_pack_range(plan, first, count, buf.shards, buf.buckets, buf.checksums)
+        rr.rr_unpack_range(plan, first, count, buf.buckets, buf.dst)
+        rr.rr_unpack_verify_async(plan, buf.buckets, buf.checksums, buf.dst, scratch, result,
+                                  bad=bad, first_bucket=first, n_buckets=count)
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        calls()
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        calls()
+    # Spoil the range's buckets, checksums and tensors, then replay.
+    for b in range(first, first + count):
+        H.bucket_list(buf)[b].fill_(0x33)
+    buf.checksums[first:first + count].fill_(5)
+    for t in buf.dst:
+        t.fill_(0)
+    result.fill_(7)
+    bad.fill_(9)
+    g.replay()
+    torch.cuda.synchronize()
+    idx = list(range(first, first + count))
+    np.testing.assert_array_equal(H.buckets_host(buf, idx), want[first:first + count])
+    np.testing.assert_array_equal(H.checksums_host(buf)[first:first + count],
+                                  want_cs[first:first + count])
+    assert result.cpu().tolist() == [0, -1]
+    assert not bad[:count].cpu().numpy().any()
+    # The tensors' bytes held by those buckets are the oracle's; the rest stay zero.
+    _, unpack_first = plan.bucket_items()
+    items, _ = plan.export_unpack()
+    sel = items[unpack_first[first]:unpack_first[first + count]]
+    copied = sel[(sel["kind"] == U.ITEM_COPY_VEC) | (sel["kind"] == U.ITEM_COPY_SCALAR)]
+    assert len(copied) > 0
+    want_t = tensors_want(L, want, plan)
+    for it in copied:
+        t, off, nb = int(it["tensor"]), int(it["dst_off"]) // 2, int(it["nbytes"]) // 2
+        np.testing.assert_array_equal(H.tensor_host(buf, t)[off:off + nb], want_t[t][off:off + nb])
     rr.rr_plan_check(plan)
