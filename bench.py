@@ -21,6 +21,7 @@ over the slowest rank's time.
 from __future__ import annotations
 
 import argparse
+import atexit
 import hashlib
 import json
 import os
@@ -129,14 +130,25 @@ def max_over_ranks(x: float, world: int) -> float:
 # ---------------------------------------------------------------------------
 
 class ClockSampler:
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi sampling the GPU's clocks every 50 ms.
+
+    It is started before the warm-up steps (nvidia-smi takes a few hundred ms
+    to print its first row) and stopped after the last measurement.  Each row
+    carries nvidia-smi's own timestamp, so rows are assigned to the timed
+    region by when they were taken, not by when they arrived.  The summary is
+    over the timed region's rows when there are at least three; a shorter
+    region (a small workload's few ms) reports the rows of the whole window of
+    GPU work instead, and says so."""
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    MIN_ROWS = 3
 
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
-        self.rows = []
+        self.rows = []          # (seconds since the epoch, fields after the timestamp)
         self.proc = None
+        self.window = None      # (start, end) of the timed region, seconds since the epoch
 
     def __enter__(self):
         try:
@@ -146,15 +158,33 @@ class ClockSampler:
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
+            atexit.register(self.__exit__, None, None, None)   # never outlive the bench
         except OSError:
             self.proc = None
         return self
 
+    @staticmethod
+    def _when(stamp: str):
+        try:   # "2026/12/02 09:48:40.123", the box's local time
+            day, frac = (stamp.split(".") + ["0"])[:2]
+            return time.mktime(time.strptime(day, "%Y/%m/%d %H:%M:%S")) + float("0." + frac)
+        except (ValueError, OverflowError):
+            return None
+
     def _read(self):
         for line in self.proc.stdout:
             parts = [p.strip() for p in line.split(",")]
-            if len(parts) >= 9:
-                self.rows.append(parts)
+            if len(parts) >= 10:
+                self.rows.append((self._when(parts[0]), parts[1:]))
+
+    def wait_first(self, timeout: float = 3.0):
+        """Returns once nvidia-smi has printed a row (or after `timeout`)."""
+        deadline = time.time() + timeout
+        while self.proc and not self.rows and time.time() < deadline:
+            time.sleep(0.02)
+
+    def mark(self, start: float, end: float):
+        self.window = (start, end)
 
     def __exit__(self, *exc):
         if self.proc:
@@ -166,16 +196,25 @@ class ClockSampler:
             self.thread.join(timeout=2)
 
     def summary(self):
-        if not self.rows:
+        rows, where = [r for _, r in self.rows], "bench run (no timed-region marks)"
+        if self.window:
+            a, b = self.window
+            timed = [r for w, r in self.rows if w is not None and a <= w <= b]
+            if len(timed) >= self.MIN_ROWS:
+                rows, where = timed, "timed region"
+            else:
+                where = (f"warm-up to last measurement ({len(timed)} sample(s) in the "
+                         f"{1e3 * (b - a):.0f} ms timed region)")
+        if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
-        sm = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
-        mx = [float(r[2]) for r in self.rows if r[2].replace(".", "").isdigit()]
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({n for r in self.rows for n, v in zip(names, r[5:9])
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9])
                           if v.lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(self.rows)}
+                "reasons": reasons, "samples": len(rows), "window": where}
 
 
 def visible_gpu_index(local_rank: int) -> int:
@@ -468,6 +507,9 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         if used[0] and not bool(((got[:, 0] == 0) & (got[:, 1] == -1)).all()):
             raise RuntimeError(f"verify found bad buckets: {got.tolist()}")
 
+    # Clocks: sampled from before the warm-up to the last measurement.
+    clk = ClockSampler(visible_gpu_index(local)).__enter__()
+    clk.wait_first()
     for _ in range(max(3, args.warmup)):
         step()
     torch.cuda.synchronize()
@@ -483,16 +525,17 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     barrier(world)
     torch.cuda.synchronize()
-    with ClockSampler(visible_gpu_index(local)) as clk:
-        t0 = torch.cuda.Event(enable_timing=True)
-        t1 = torch.cuda.Event(enable_timing=True)
-        t0.record(stream)
-        for k in range(args.steps):
-            if flush is not None:
-                flush.fill_(k & 0xFF)
-            step(evs[k])
-        t1.record(stream)
-        torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    wall0 = time.time()
+    t0.record(stream)
+    for k in range(args.steps):
+        if flush is not None:
+            flush.fill_(k & 0xFF)
+        step(evs[k])
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clk.mark(wall0, time.time())
     barrier(world)
     pack_all = [e[0].elapsed_time(e[1]) for e in evs]
     uv_all = [e[1].elapsed_time(e[2]) for e in evs]
@@ -612,6 +655,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     pack_gbs = pack_bytes / (pack_ms * 1e-3) / 1e9
     traffic = (profiled_traffic(w.name) if bucket_bytes == w.bucket_bytes and args.engine == "auto"
                else None)
+    clk.__exit__(None, None, None)
     clocks = clk.summary()
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,

@@ -18,11 +18,15 @@ import bench  # noqa: E402
 
 FAKE = """#!/bin/sh
 # prints three samples, then idles until terminated
-echo "0, 2070, 2070, 900.00, 0x0000000000000004, Not Active, Not Active, Not Active, Active"
-echo "0, 1980, 2070, 1390.00, 0x0000000000000008, Active, Not Active, Not Active, Not Active"
-echo "0, 2070, 2070, 910.00, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active"
+echo "2026/12/02 09:00:00.100, 0, 2070, 2070, 900.00, 0x0000000000000004, Not Active, Not Active, Not Active, Active"
+echo "2026/12/02 09:00:00.150, 0, 1980, 2070, 1390.00, 0x0000000000000008, Active, Not Active, Not Active, Not Active"
+echo "2026/12/02 09:00:00.200, 0, 2070, 2070, 910.00, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active"
 exec sleep 30
 """
+
+
+def at(stamp):
+    return bench.ClockSampler._when(stamp)
 
 
 @pytest.fixture
@@ -40,9 +44,28 @@ def test_clock_sampler_reports_slowdowns(fake_smi):
         while len(clk.rows) < 3 and time.time() < deadline:
             time.sleep(0.05)
     s = clk.summary()
-    assert s["samples"] == 3
+    assert s["samples"] == 3 and s["window"].startswith("bench run")
     assert s["sm_mhz"] == 2070.0 and s["sm_max_mhz"] == 2070.0
     assert s["reasons"] == ["hw_slowdown", "sw_power_cap"]
+
+
+def test_clock_sampler_windows(fake_smi):
+    """Rows belong to the timed region by nvidia-smi's timestamps: a region
+    holding all three reports them alone; one holding fewer than three falls
+    back to every row, and says how many the region held."""
+    with bench.ClockSampler(0) as clk:
+        clk.wait_first()
+        deadline = time.time() + 10
+        while len(clk.rows) < 3 and time.time() < deadline:
+            time.sleep(0.05)
+    clk.mark(at("2026/12/02 09:00:00.050"), at("2026/12/02 09:00:00.250"))
+    s = clk.summary()
+    assert s["window"] == "timed region" and s["samples"] == 3
+    clk.mark(at("2026/12/02 09:00:00.120"), at("2026/12/02 09:00:00.160"))
+    s = clk.summary()
+    assert s["samples"] == 3 and "1 sample(s)" in s["window"]
+    assert s["reasons"] == ["hw_slowdown", "sw_power_cap"]
+    assert bench.ClockSampler._when("not a time") is None
 
 
 def test_clock_sampler_without_nvidia_smi(tmp_path, monkeypatch):
