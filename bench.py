@@ -261,22 +261,41 @@ def hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash() -> str:
-    path = os.path.join(ROOT, "paper_2512_22492_gb300", "csrc", "rr_device.cu")
-    return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
+KERNEL_SOURCES = ("include/rr.h", "paper_2512_22492_gb300/csrc/rr_device.cu",
+                  "paper_2512_22492_gb300/csrc/rr_internal.h",
+                  "paper_2512_22492_gb300/csrc/rr_plan.cpp")
+
+
+def code_only(text: str) -> str:
+    """C/C++/CUDA source with comments removed and white space collapsed, so
+    that an edit of comments alone keeps a profile's figures current."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
+def kernel_code_hash() -> str:
+    """sha256 (first 16 hex digits) of the code of the kernels, of the planner
+    that writes their work tables and of the item layouts they share: what a
+    profile's DRAM figures depend on."""
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES:
+        text = open(os.path.join(ROOT, name)).read()
+        h.update(name.encode() + b"\0" + code_only(text).encode() + b"\0")
+    return h.hexdigest()[:16]
 
 
 def profiled_traffic(workload: str):
     """DRAM bytes per pack launch from the committed ncu summary, if it was taken
-    on the current kernel source; else None."""
+    on the current code; else None."""
     path = os.path.join(ROOT, "profiles", f"rr_pack_{workload}.md")
     try:
         text = open(path).read()
     except OSError:
         return None
-    m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
+    m_hash = re.search(r"kernel_code_sha256_16:\s*([0-9a-f]+)", text)
     m_bytes = re.search(r"dram_bytes_per_launch_full:\s*([0-9]+)", text)
-    if not (m_hash and m_bytes) or m_hash.group(1) != kernel_source_hash():
+    if not (m_hash and m_bytes) or m_hash.group(1) != kernel_code_hash():
         return None
     return int(m_bytes.group(1))
 

@@ -15,9 +15,12 @@
 // moves 16-byte vectors through registers; it serves host-resident buffers
 // and the standalone verify.
 //
-// Every kernel is persistent: one launch walks the whole work table, each
-// block a contiguous, weight-balanced range of it.  The work is pure data
-// movement bound by HBM bandwidth; the cast is integer arithmetic in
+// Every kernel is persistent: one launch walks the whole work table.  On the
+// register path each block takes a contiguous, weight-balanced range of it.
+// On the bulk-copy engine blocks take work units: their own first, then the
+// next unclaimed one (an atomic counter) until none are left, so that blocks
+// draining HBM at unequal rates still finish together.  The work is pure
+// data movement bound by HBM bandwidth; the cast is integer arithmetic in
 // registers, and the checksum is accumulated per warp and flushed with one
 // 64-bit atomic per warp per bucket change.
 #include <cuda_runtime.h>

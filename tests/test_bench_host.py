@@ -83,16 +83,26 @@ def test_visible_gpu_index(monkeypatch):
 
 
 def test_profiled_traffic_needs_the_current_kernel(tmp_path, monkeypatch):
+    """The profile's traffic is reported only while the code it was taken on
+    is unchanged; a comment edit does not count as a change."""
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     (tmp_path / "profiles").mkdir()
+    (tmp_path / "include").mkdir()
     src = tmp_path / "paper_2512_22492_gb300" / "csrc"
     src.mkdir(parents=True)
-    (src / "rr_device.cu").write_text("kernel v1")
-    good = bench.kernel_source_hash()
+    for name in bench.KERNEL_SOURCES:
+        (tmp_path / name).write_text("int x; // a\n")
+    (src / "rr_device.cu").write_text("int kernel_v1(void) { return 1; }  // first\n")
+    good = bench.kernel_code_hash()
     page = tmp_path / "profiles" / "rr_pack_demo.md"
-    page.write_text(f"kernel_source_sha256_16: {good}\ndram_bytes_per_launch_full: 123\n")
+    page.write_text(f"kernel_code_sha256_16: {good}\ndram_bytes_per_launch_full: 123\n")
     assert bench.profiled_traffic("demo") == 123
-    (src / "rr_device.cu").write_text("kernel v2")      # the kernel changed since the capture
+    (src / "rr_device.cu").write_text("/* new words */ int kernel_v1(void)\n{\n  return 1;  // said\n}\n")
+    assert bench.profiled_traffic("demo") == 123        # comments and layout only
+    (src / "rr_device.cu").write_text("int kernel_v1(void) { return 2; }\n")
+    assert bench.profiled_traffic("demo") is None       # the code changed since the capture
+    (src / "rr_device.cu").write_text("int kernel_v1(void) { return 1; }\n")
+    (src / "rr_plan.cpp").write_text("int x = 1;\n")      # so did the planner's
     assert bench.profiled_traffic("demo") is None
     assert bench.profiled_traffic("other") is None
 
