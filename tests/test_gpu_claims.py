@@ -56,6 +56,8 @@ def check(plan, buf, want, want_cs, want_t):
 
 
 def test_more_launches_in_flight_than_claim_slots():
+    if not hasattr(torch.cuda, "_sleep"):
+        pytest.skip("this PyTorch has no bounded sleep kernel to hold the stream")
     desc, m, plan, L, shards, want, want_cs = setup()
     want_t = tensors_want(L, want, plan)
     first = H.alloc(plan)
