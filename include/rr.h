@@ -197,17 +197,28 @@ typedef struct {
  * 2^32 - 16.  Uses the current CUDA device.  *out is valid only on RR_OK. */
 rr_status rr_plan_create(const rr_param* manifest, int32_t n_params, const rr_src_layout* src,
                          const rr_dst_layout* dst, size_t bucket_bytes, rr_plan** out);
+/* rr_plan_create with tuning options (opts may be NULL).  The options have no
+ * counterpart in the paper; the plan they build computes the same bytes. */
 rr_status rr_plan_create_ex(const rr_param* manifest, int32_t n_params,
                             const rr_src_layout* src, const rr_dst_layout* dst,
                             size_t bucket_bytes, const rr_plan_options* opts, rr_plan** out);
+
+/* Frees the plan's device tables, scratch and events.  Section 5.2.1 reserves
+ * the transfer's memory ahead of the transfer so that it cannot run out of GPU
+ * memory mid-sync; a plan is that reservation for the work tables, held from
+ * creation until this call.  NULL is ignored.  No call of this plan may still
+ * be running on any stream. */
 void rr_plan_destroy(rr_plan* plan);
 
-/* Bucket geometry.  Any output pointer may be NULL.  stream_bytes_per_rank has
- * tp entries; first_bucket_of_rank has tp + 1 (the last is n_buckets). */
+/* Bucket geometry: the size of the transfer buffer (Section 5.2.1: a buffer
+ * reserved up front, large enough to keep the RDMA links busy), so that the
+ * caller can allocate every bucket before the first sync.  Any output pointer
+ * may be NULL.  stream_bytes_per_rank has tp entries; first_bucket_of_rank has
+ * tp + 1 (the last is n_buckets).  RR_EINVAL for a NULL plan. */
 rr_status rr_plan_query(const rr_plan* plan, int32_t* n_buckets, int64_t* stream_bytes_per_rank,
                         int32_t* first_bucket_of_rank);
 
-/* Source geometry: shard size S, end of the last parameter, and per-parameter
+/* Source geometry (the trainer's FSDP shards, Section 7.1): shard size S, end of the last parameter, and per-parameter
  * byte offsets ([n_params]): flat offsets for RR_SHARD_FLAT, offsets within
  * each shard for RR_SHARD_ROWS, 0 for RR_SHARD_TENSORS (whose S is the size of
  * the largest parameter), offsets within the parameter's unit for
@@ -216,15 +227,16 @@ rr_status rr_plan_query(const rr_plan* plan, int32_t* n_buckets, int64_t* stream
 rr_status rr_plan_source(const rr_plan* plan, int64_t* shard_bytes, int64_t* flat_bytes,
                          int64_t* param_flat_offset);
 
-/* The source buffers the calls take: their number (the length of every
+/* The source buffers the calls take (the trainer's shards, Section 7.1): their number (the length of every
  * src_shards array) and the bytes each must hold ([*n_buffers]).  FLAT and
  * ROWS: n_shards buffers of S bytes; TENSORS: one per parameter, of its size;
  * UNITS: n_units * n_shards, unit-major, each of its unit's S_u.  Pass
  * buffer_bytes = NULL to learn the count first.  Any output pointer may be NULL. */
 rr_status rr_plan_source_buffers(const rr_plan* plan, int32_t* n_buffers, int64_t* buffer_bytes);
 
-/* Destination geometry: per tensor numel and byte offset within its rank's
- * stream ([n_tensors] each).  Any output pointer may be NULL. */
+/* Destination geometry (the rollout's sharding that Section 5.2.1 step 1
+ * reshards into): per tensor numel and byte offset within its rank's stream
+ * ([n_tensors] each).  Any output pointer may be NULL. */
 rr_status rr_plan_tensors(const rr_plan* plan, int64_t* tensor_numel,
                           int64_t* tensor_stream_offset);
 
@@ -248,10 +260,12 @@ typedef struct {
                                     when no fan-out groups were found                  */
 } rr_plan_stats;
 
+/* Table sizes, grids and the algorithmic bytes each call moves.  No
+ * counterpart in the paper: it serves measurement against the HBM roofline. */
 rr_status rr_plan_get_stats(const rr_plan* plan, rr_plan_stats* stats);
 
 /* Work items of the segment tables, as the kernels read them (exported for
- * inspection and host-side tests). */
+ * inspection and host-side tests; no counterpart in the paper). */
 enum {
     RR_ITEM_F32_VEC = 0,    /* fp32 -> bf16, 8 elements per 16-byte store            */
     RR_ITEM_F32_SCALAR = 1, /* fp32 -> bf16, one element at a time (ragged/misaligned)*/
@@ -343,10 +357,20 @@ rr_status rr_unpack(const rr_plan* plan, const void* const* buckets, void* const
                     cudaStream_t stream);
 
 /* Recomputes every bucket's checksum on the GPU and compares it with
- * checksums (device, n_buckets).  Blocks the calling thread until `stream`
- * has finished the check.  *n_bad = number of mismatching buckets, *first_bad
- * = lowest such index or -1 (either pointer may be NULL).  Returns
- * RR_EMISMATCH when n_bad > 0. */
+ * checksums (device, n_buckets).  Section 5.2.2: a rollout that reconnects
+ * after a relay or trainer failure, or resumes a pull, must know which of the
+ * buckets it holds are intact before it completes its update.
+ *   buckets:   host array of n_buckets pointers (device or pinned host),
+ *              bucket_bytes each, 16-byte aligned; read only.
+ *   checksums: device (or pinned host) array of n_buckets uint64, read only.
+ *   stream:    where the check runs.  This argument extends the four-call
+ *              interface: the check is ordered after the caller's own work
+ *              (the pull that filled the buckets) without a device-wide sync.
+ * Blocks the calling thread until `stream` has finished the check.  *n_bad =
+ * number of mismatching buckets, *first_bad = lowest such index or -1 (either
+ * pointer may be NULL).  Returns RR_EMISMATCH when n_bad > 0, RR_ECUDA when a
+ * kernel of this plan gave up a bounded wait (see rr_plan_check), RR_EINVAL
+ * for bad pointers (nothing is launched then).  Serialises on the plan. */
 rr_status rr_verify(const rr_plan* plan, const void* const* buckets, const uint64_t* checksums,
                     int64_t* n_bad, int64_t* first_bad, cudaStream_t stream);
 
@@ -397,10 +421,12 @@ rr_status rr_unpack_verify_range(const rr_plan* plan, int32_t first_bucket, int3
 
 /* Per-bucket item index of the two work tables (n_buckets + 1 entries each,
  * either pointer may be NULL): the pack items of bucket b are
- * [pack_first[b], pack_first[b + 1]); likewise for unpack. */
+ * [pack_first[b], pack_first[b + 1]); likewise for unpack.  Inspection only;
+ * no counterpart in the paper. */
 rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32_t* unpack_first);
 
-/* Work units of the bulk-copy engine.  Blocks drain HBM at unequal rates, so
+/* Work units of the bulk-copy engine (inspection; no counterpart in the
+ * paper, whose reshard is plain framework kernels).  Blocks drain HBM at unequal rates, so
  * a launch does not fix each block's whole share: block g takes the launch's
  * unit g, then claims the next unclaimed unit (an atomic counter) until none
  * are left, and all blocks finish together.
@@ -464,29 +490,39 @@ rr_status rr_unpack_verify_async(const rr_plan* plan, int32_t first_bucket, int3
  * of rr_verify.
  *   Scratch: one file-scope device array of 16384 + 4 64-bit words (128 KiB),
  *   which every GPU that loads this library keeps until the process exits.
- *   n_buckets above 16384 is rejected with RR_EINVAL.  The first call on a
- *   device looks up the array's device address and sizes the grid for that
- *   device; make that first call before any stream capture.  Each call clears
- *   the part of the array it uses before its kernel runs; calls that overlap
- *   on the GPU (on different streams, or from different threads) share the
- *   array and race, so serialise them.  Calls no cudaMalloc or cudaFree. */
+ *   n_buckets above 16384 is rejected with RR_EINVAL.  Buckets that are not
+ *   equally spaced (separately allocated, passed as a pointer table in the
+ *   kernel's parameters) are limited to 3968 per call, RR_EINVAL beyond;
+ *   equally spaced buckets (one allocation cut into buckets) have only the
+ *   16384 limit.  The first call on a device sizes the grid for that device;
+ *   make that first call before any stream capture.  Every call looks up the
+ *   array's device address again (a device reset may move it).  Each call
+ *   clears the part of the array it uses before its kernel runs; calls that
+ *   overlap on the GPU (on different streams, or from different threads)
+ *   share the array and race, so serialise them.  Calls no cudaMalloc or
+ *   cudaFree. */
 rr_status rr_verify_noalloc(const void* const* buckets, int32_t n_buckets, size_t bucket_bytes,
                             const uint64_t* checksums, int64_t* n_bad, int64_t* first_bad,
                             cudaStream_t stream);
 
-/* Waits for `stream`, then reports whether a kernel of this plan gave up on
+/* Section 5.2.2: a role must know whether what it holds is whole.  Waits
+ * for `stream`, then reports whether a kernel of this plan gave up on
  * a wait (the bulk-copy engine bounds every wait; one that runs out marks the
  * plan and its output is incomplete): RR_ECUDA if so (and clears the mark),
  * RR_OK otherwise.  rr_verify and rr_unpack_verify check this themselves. */
 rr_status rr_plan_check(const rr_plan* plan, cudaStream_t stream);
 
-/* Test hook for the bounded waits: enqueues on `stream` one small kernel that
+/* Test hook for the bounded waits (no counterpart in the paper): enqueues on `stream` one small kernel that
  * waits on a barrier nothing completes.  The wait gives up after its limit
  * (about a second) and marks the plan, so the next rr_plan_check (or
  * rr_verify / rr_unpack_verify) reports RR_ECUDA while the CUDA context stays
  * usable.  It touches no buffer. */
 rr_status rr_plan_selftest_wait(const rr_plan* plan, cudaStream_t stream);
 
+/* A static description of a status code ("RR_OK", "RR_EINVAL: invalid
+ * argument", ...; "unknown rr_status" otherwise), and this thread's
+ * description of its most recent failure ("" if none).  The
+ * returned strings are owned by the library.  No counterpart in the paper. */
 const char* rr_status_str(rr_status status);
 const char* rr_last_error(void);
 

@@ -2136,36 +2136,39 @@ __device__ __align__(256) unsigned long long g_static_verify_scratch[kStaticVeri
 
 struct StaticVerifyDevice {
     bool ready = false;
-    unsigned long long* scratch = nullptr;   // device address of g_static_verify_scratch
     int32_t grid = 0;
 };
 
 std::mutex g_static_mutex;
 StaticVerifyDevice g_static_dev[kStaticMaxDevices];
 
-// Once per device, with that device current: resolve the array's device
-// address (host code may not use the symbol itself as a pointer) and size the
-// grid.  Neither step allocates.
-rr_status static_verify_setup(StaticVerifyDevice** out) {
+// With the caller's device current: the array's device address (host code may
+// not use the symbol itself as a pointer) and the grid for this device.  The
+// grid is sized once per device, on its first call.  The address is looked up
+// on every call: a device reset destroys the context that loaded this
+// library's module, the next context loads it again, and the array may then
+// sit elsewhere.  Neither step allocates.
+rr_status static_verify_setup(unsigned long long** scratch, int32_t* grid) {
     int dev = -1;
     RR_CUDA(cudaGetDevice(&dev));
     if (dev < 0 || dev >= kStaticMaxDevices)
         return rr_fail(RR_EINVAL, "device %d beyond the %d devices this entry point serves", dev,
                        kStaticMaxDevices);
+    void* p = nullptr;
+    RR_CUDA(cudaGetSymbolAddress(&p, g_static_verify_scratch));
+    if (!p) return rr_fail(RR_ECUDA, "no device address for the verify scratch array");
     std::lock_guard<std::mutex> lock(g_static_mutex);
     StaticVerifyDevice& d = g_static_dev[dev];
     if (!d.ready) {
-        void* p = nullptr;
-        RR_CUDA(cudaGetSymbolAddress(&p, g_static_verify_scratch));
         int sms = 0, per_sm = 0;
         RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
         RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
             &per_sm, rr_verify_kernel<kLargePtrs>, kThreads, 0));
-        d.scratch = (unsigned long long*)p;
         d.grid = sms * (per_sm > 0 ? per_sm : 1);
         d.ready = true;
     }
-    *out = &d;
+    *scratch = (unsigned long long*)p;
+    *grid = d.grid;
     return RR_OK;
 }
 
@@ -2223,20 +2226,21 @@ extern "C" rr_status rr_verify_noalloc(const void* const* buckets, int32_t n_buc
     if (table && n_buckets > kLargePtrs)
         return rr_fail(RR_EINVAL, "%d separately allocated buckets exceed %d pointers", n_buckets,
                        kLargePtrs);
-    StaticVerifyDevice* d = nullptr;
-    if ((st = static_verify_setup(&d))) return st;
+    unsigned long long* scratch = nullptr;
+    int32_t grid = 0;
+    if ((st = static_verify_setup(&scratch, &grid))) return st;
 
     // The array keeps the previous call's contents: clear the sums and counters used here.
-    RR_CUDA(cudaMemsetAsync(d->scratch, 0, (size_t(n_buckets) + 4) * sizeof(unsigned long long),
+    RR_CUDA(cudaMemsetAsync(scratch, 0, (size_t(n_buckets) + 4) * sizeof(unsigned long long),
                             stream));
     st = (!table || n_buckets <= kSmallPtrs)
-             ? launch_static_verify<kSmallPtrs>(d->scratch, d->grid, n_buckets, bucket_bytes,
-                                                buckets, checksums, table, stride, stream)
-             : launch_static_verify<kLargePtrs>(d->scratch, d->grid, n_buckets, bucket_bytes,
-                                                buckets, checksums, table, stride, stream);
+             ? launch_static_verify<kSmallPtrs>(scratch, grid, n_buckets, bucket_bytes, buckets,
+                                                checksums, table, stride, stream)
+             : launch_static_verify<kLargePtrs>(scratch, grid, n_buckets, bucket_bytes, buckets,
+                                                checksums, table, stride, stream);
     if (st) return st;
     unsigned long long result[4] = {0, 0, 0, 0};   // host stack: no pinned buffer needed
-    RR_CUDA(cudaMemcpyAsync(result, d->scratch + n_buckets, sizeof result, cudaMemcpyDeviceToHost,
+    RR_CUDA(cudaMemcpyAsync(result, scratch + n_buckets, sizeof result, cudaMemcpyDeviceToHost,
                             stream));
     RR_CUDA(cudaStreamSynchronize(stream));
     if (n_bad) *n_bad = (int64_t)result[1];
