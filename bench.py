@@ -1,16 +1,19 @@
 """Benchmark: one full trainer -> rollout weight sync per step on GB300.
 
 A step is the whole hot path once (RobustRL Section 5.2.1 steps 1-2 and the
-Section 5.2.2 check): rr_pack (reshard + bf16 cast + bucket pack + checksum),
-rr_unpack (buckets -> rollout tensors) and rr_verify (recompute and compare
-every checksum).  Default workload: Qwen3-8B-shaped fp32 weights in 8 flat
-FSDP-style shards -> TP=1 bf16 rollout layout with fused QKV / gate_up,
-128 MiB buckets, seeded synthetic values ~N(0, 0.02).
+Section 5.2.2 check): rr_pack (reshard + bf16 cast + bucket pack + checksum)
+and the receiver's rr_unpack_verify_async (buckets -> rollout tensors, with
+every bucket's checksum recomputed and compared in the same pass).  Default
+workload: Qwen3-8B-shaped fp32 weights in 8 flat FSDP-style shards -> TP=1
+bf16 rollout layout with fused QKV / gate_up, 128 MiB buckets, seeded
+synthetic values ~N(0, 0.02).
 
 Metric: GB/s of algorithmic bytes (every byte read once, every byte written
-once: pack = source bytes + bucket bytes, unpack = 2 x tensor bytes, verify =
-bucket bytes), plus ms per full model sync (pack + unpack).  Inputs (33 GB of
-source) are far larger than L2, so no flush is needed between steps.
+once: pack = source bytes + bucket bytes; the receiver = bucket bytes read +
+tensor bytes written), plus ms per full model sync (pack + the receiver).
+The separate rr_unpack and rr_verify are timed after the step loop as a
+breakdown.  Inputs (33 GB of source) are far larger than L2, so no flush is
+needed between steps.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
 
@@ -358,6 +361,12 @@ def cpu_baseline(w, bucket_bytes, n_buckets_sample):
                       f"{dt:.2f} s; 1 of {os.cpu_count()} host cores ({cpu_model()})"}
 
 
+def path_dtype(w) -> str:
+    """What the path computes: an fp32 source is rounded to bf16 (nearest,
+    ties to even, in integer arithmetic); a bf16 source is copied bit for bit."""
+    return "f32->bf16 (RNE)" if w.src_dtype == "f32" else "bf16 (bit copy)"
+
+
 def run_reference(args, w, bucket_bytes, world, rank):
     if rank != 0:
         return
@@ -375,7 +384,7 @@ def run_reference(args, w, bucket_bytes, world, rank):
         "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(t_total / args.steps * 1e3, 3), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "u16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": path_dtype(w), "data": "synthetic",
         "config": {"workload": w.name, "bucket_bytes": bucket_bytes,
                    "step": f"oracle sync of bucket 0 of {L.n_buckets} (bounded sample)"},
         "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
@@ -465,66 +474,100 @@ def next_rows(rr, H, w, plan, buf, t_src, t_bkt, t_dst, stream, peak):
     return out
 
 
+class BenchStep:
+    """The timed step with its buffers: one plan for workload `w`, the source
+    filled by the seeded device generator, pointer tables checked once (as a
+    caller syncing every training step would hold them), and per step rr_pack
+    followed by the receiver's verifying unpack on one stream.
+
+    The receiver's check is stream-ordered by default: each step's {n_bad,
+    first_bad} lands in its own row of `results`, read after the timing by
+    check_results().  `sync_verify` uses the blocking rr_unpack_verify instead.
+    `poison` (a byte) pre-fills buckets and tensors so that unwritten bytes
+    show; None leaves them uninitialised."""
+
+    def __init__(self, w, bucket_bytes, opts=None, sync_verify=False, n_rows=64, stream=None,
+                 poison=None):
+        import torch
+        import paper_2512_22492_gb300 as rr
+        from synth import device as D
+        self.rr, self.w, self.sync_verify = rr, w, sync_verify
+        self.stream = stream if stream is not None else torch.cuda.current_stream()
+        m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
+        self.manifest = m
+        self.plan = plan = rr.rr_plan_create(m, s, d, bucket_bytes, opts)
+        self.buf = buf = D.alloc(plan, poison=poison)
+        D.fill_with_generator(buf, m, w.seed, w.specials)
+        torch.cuda.synchronize()
+        self.t_src = rr.Pointers(plan, "src_shards", buf.shards)
+        self.t_bkt = rr.Pointers(plan, "buckets", buf.buckets)
+        self.t_dst = rr.Pointers(plan, "dst", buf.dst)
+        st = self.stats = plan.stats()
+        self.pack_bytes = st["pack_bytes_read"] + st["pack_bytes_written"]
+        self.unpack_bytes = st["unpack_bytes_read"] + st["unpack_bytes_written"]
+        self.verify_bytes = st["verify_bytes_read"]
+        # The receiver's fused pass reads every bucket byte once and writes every tensor byte.
+        self.uv_bytes = st["verify_bytes_read"] + st["unpack_bytes_written"]
+        self.step_bytes = self.pack_bytes + self.uv_bytes
+        self.scratch = torch.zeros(plan.n_buckets + 4, dtype=torch.int64, device="cuda")
+        self.n_rows = n_rows
+        self.results = torch.full((n_rows, 2), -7, dtype=torch.int64, device="cuda")
+        self.used = 0
+
+    def step(self, ev=None):
+        """Enqueues one sync; `ev` (three CUDA events) brackets pack and receiver.
+        Returns the step's result row (None with sync_verify)."""
+        rr, plan, stream = self.rr, self.plan, self.stream
+        if ev:
+            ev[0].record(stream)
+        rr.rr_pack(plan, self.t_src, self.t_bkt, self.buf.checksums, stream)
+        if ev:
+            ev[1].record(stream)
+        row = None
+        if self.sync_verify:
+            n_bad, _ = rr.rr_unpack_verify(plan, self.t_bkt, self.buf.checksums, self.t_dst,
+                                           stream=stream)
+            if n_bad:
+                raise RuntimeError(f"verify found {n_bad} bad buckets")
+        else:
+            row = self.results[self.used % self.n_rows]
+            self.used += 1
+            rr.rr_unpack_verify_async(plan, self.t_bkt, self.buf.checksums, self.t_dst,
+                                      self.scratch, row, stream=stream)
+        if ev:
+            ev[2].record(stream)
+        return row
+
+    def check_results(self):
+        """Raises unless every step so far verified clean and no kernel of the
+        plan gave up a bounded wait (which leaves its output incomplete without
+        touching the result rows; the plan's error word says so)."""
+        import torch
+        torch.cuda.synchronize()
+        got = self.results[:min(self.used, self.n_rows)].cpu()
+        if self.used and not bool(((got[:, 0] == 0) & (got[:, 1] == -1)).all()):
+            raise RuntimeError(f"verify found bad buckets: {got.tolist()}")
+        self.rr.rr_plan_check(self.plan, self.stream)
+
+
 def run_native(args, w, bucket_bytes, world, rank, local):
     import torch
     import paper_2512_22492_gb300 as rr
-    from tests import gpu_harness as H
+    from synth import device as H
 
     torch.cuda.set_device(local)
     stream = torch.cuda.current_stream()
-    m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
     opts = None
     if args.chunk_kib or args.grid or args.engine != "auto" or args.check_items:
         opts = rr.PlanOptions(chunk_bytes=args.chunk_kib * 1024, grid_blocks=args.grid,
                               engine=args.engine, check_items=args.check_items)
-    plan = rr.rr_plan_create(m, s, d, bucket_bytes, opts)
-    st = plan.stats()
-    buf = H.alloc(plan, poison=None)
-    H.fill_with_generator(buf, m, w.seed, w.specials)
-    torch.cuda.synchronize()
-    # Pointer tables checked once, as a caller syncing every training step would hold them.
-    t_src = rr.Pointers(plan, "src_shards", buf.shards)
-    t_bkt = rr.Pointers(plan, "buckets", buf.buckets)
-    t_dst = rr.Pointers(plan, "dst", buf.dst)
-
-    pack_bytes = st["pack_bytes_read"] + st["pack_bytes_written"]
-    unpack_bytes = st["unpack_bytes_read"] + st["unpack_bytes_written"]
-    verify_bytes = st["verify_bytes_read"]
-    # The receiver's fused pass reads every bucket byte once and writes every tensor byte.
-    uv_bytes = st["verify_bytes_read"] + st["unpack_bytes_written"]
-    step_bytes = pack_bytes + uv_bytes
-
-    # The receiver's check: stream-ordered by default, each step's {n_bad,
-    # first_bad} left in its own row of `results` and read after the timing.
-    scratch = torch.zeros(plan.n_buckets + 4, dtype=torch.int64, device="cuda")
-    n_rows = 2 * (max(3, args.warmup) + args.steps) + 8
-    results = torch.full((n_rows, 2), -7, dtype=torch.int64, device="cuda")
-    used = [0]
-
-    def step(ev=None):
-        if ev:
-            ev[0].record(stream)
-        rr.rr_pack(plan, t_src, t_bkt, buf.checksums, stream)
-        if ev:
-            ev[1].record(stream)
-        if args.sync_verify:
-            n_bad, _ = rr.rr_unpack_verify(plan, t_bkt, buf.checksums, t_dst, stream=stream)
-            if n_bad:
-                raise RuntimeError(f"verify found {n_bad} bad buckets")
-        else:
-            row = results[used[0] % n_rows]
-            used[0] += 1
-            rr.rr_unpack_verify_async(plan, t_bkt, buf.checksums, t_dst, scratch, row,
-                                      stream=stream)
-        if ev:
-            ev[2].record(stream)
-        return None if args.sync_verify else row
-
-    def check_results():
-        torch.cuda.synchronize()
-        got = results[:min(used[0], n_rows)].cpu()
-        if used[0] and not bool(((got[:, 0] == 0) & (got[:, 1] == -1)).all()):
-            raise RuntimeError(f"verify found bad buckets: {got.tolist()}")
+    bs = BenchStep(w, bucket_bytes, opts, sync_verify=args.sync_verify,
+                   n_rows=2 * (max(3, args.warmup) + args.steps) + 8, stream=stream)
+    plan, buf, st = bs.plan, bs.buf, bs.stats
+    t_src, t_bkt, t_dst = bs.t_src, bs.t_bkt, bs.t_dst
+    pack_bytes, unpack_bytes, verify_bytes = bs.pack_bytes, bs.unpack_bytes, bs.verify_bytes
+    uv_bytes, step_bytes = bs.uv_bytes, bs.step_bytes
+    step, check_results = bs.step, bs.check_results
 
     # Clocks: sampled from before the warm-up to the last measurement.
     clk = ClockSampler(visible_gpu_index(local)).__enter__()
@@ -679,7 +722,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u16",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": path_dtype(w),
         "data": "synthetic",
         "config": {"workload": w.name, "src_dtype": w.src_dtype, "n_shards": w.n_shards,
                    "sharding": w.sharding, "expert_parallel": w.ep,
