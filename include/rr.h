@@ -432,15 +432,19 @@ rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32
  * are left, and all blocks finish together.
  *   which:
  *   RR_UNITS_PACK, RR_UNITS_UNPACK: the units of a bucket-range pack, and of
- *     every unpack and verifying unpack.  Each bucket's items are cut into
- *     units of about 1 MiB of traffic (less on small plans, so that a block of
- *     the grid has a few dozen), none empty, none spanning two buckets; a
- *     range's units are the run of its buckets' units.
+ *     every unpack and verifying unpack (on either engine).  Each bucket's
+ *     items are cut into units of at most about 1 MiB of traffic (less on
+ *     small plans, so that a block of the grid has a few dozen), none empty,
+ *     none spanning two buckets; toward the end of the table units get
+ *     smaller (about the weight left over twice the grid, down to 64 KiB), so
+ *     that the last blocks to finish stop close together.  A range's units
+ *     are the run of its buckets' units.
  *   RR_UNITS_PACK_FULL: the units of a pack over every bucket, over the table
  *     rr_plan_export_pack_full gives.  Units 0 .. grid - 1 are equal
- *     contiguous shares of 70% of the table's weight, one per block; the
- *     units after them cut the rest to the size above.  A cut never falls
- *     before a fan-out destination item.  Units may be empty.
+ *     contiguous shares of 85% of the table's weight, one per block; the
+ *     units after them cut the rest to the sizes above, smaller toward the
+ *     end.  A cut never falls before a fan-out destination item.  Own units
+ *     may be empty.
  *   *n_units: the number of units.
  *   unit_first (NULL, or n_units + 1 entries): unit u holds items
  *     [unit_first[u], unit_first[u + 1]) of that table.
@@ -450,14 +454,15 @@ rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32
  * Call with both arrays NULL to learn n_units.  Host-only plans have units
  * too.  Errors: RR_EINVAL for a NULL plan or n_units, an unknown `which`, or
  * a bucket_unit array with RR_UNITS_PACK_FULL; nothing is written then.
- * Which launches of the bulk-copy engine claim (the register path never
- * does): the verifying unpack always, its counter kept in the call's scratch
- * (the plan's for the blocking forms, the caller's for
- * rr_unpack_verify_async); rr_pack and rr_unpack when one of the plan's 16
- * counter slots is free -- a slot is reused only after the launch that last
- * held it has completed -- and the stream is not capturing a graph.
- * Otherwise the launch splits its items evenly over the grid, as a captured
- * launch always does.  Which of these runs changes no output byte. */
+ * Which launches claim: every verifying unpack (either engine), its counter
+ * kept in the call's scratch (the plan's for the blocking forms, the
+ * caller's for rr_unpack_verify_async); rr_unpack (either engine) and rr_pack
+ * (bulk-copy engine) when one of the plan's 16 counter slots is free -- a
+ * slot is reused only after the launch that last held it has completed --
+ * and the stream is not capturing a graph.  Otherwise the launch splits its
+ * items evenly over the grid, as a captured launch always does, and the
+ * register path's pack always does.  Which of these runs changes no output
+ * byte. */
 enum { RR_UNITS_PACK = 0, RR_UNITS_PACK_FULL = 1, RR_UNITS_UNPACK = 2 };
 rr_status rr_plan_work_units(const rr_plan* plan, int32_t which, int32_t* n_units,
                              uint32_t* unit_first, uint32_t* bucket_unit);

@@ -54,8 +54,9 @@ def build(force: bool = False, verbose: bool = False) -> str:
     plan_o = os.path.join(BUILD, "rr_plan.o")
     dev_o = os.path.join(BUILD, "rr_device.o")
     jobs = [
-        ["g++", "-O2", "-std=c++17", "-fPIC", "-Wall", "-c", os.path.join(CSRC, "rr_plan.cpp"),
-         "-o", plan_o] + inc,
+        ["g++", "-O2", "-std=c++17", "-fPIC", "-Wall"] +
+        os.environ.get("RR_EXTRA_CXX_FLAGS", "").split() +
+        ["-c", os.path.join(CSRC, "rr_plan.cpp"), "-o", plan_o] + inc,
         [nvcc, "-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xptxas", "-v"] + ARCH +
         os.environ.get("RR_EXTRA_NVCC_FLAGS", "").split() +
         ["-c", os.path.join(CSRC, "rr_device.cu"), "-o", dev_o] + inc,

@@ -111,6 +111,14 @@ struct UnpackArgs {
     uint64_t bucket_stride;
     int32_t dst_base;         // index in ptr[] of destination tensor 0
     int32_t bucket_lo;        // table mode: the first bucket the table holds
+    // Claimed work units (claim NULL: none, the split above).  unit_first holds
+    // the first item of each of n_units units and one past the last; block g
+    // walks unit g, then claims the next unclaimed unit (atomicAdd on *claim,
+    // zero at launch) until none are left.
+    const uint32_t* unit_first;
+    unsigned long long* claim;
+    uint32_t n_units;
+    uint32_t reset_claims;    // claim is a pooled slot {counter, ticket}: zero it at the end
     const void* ptr[NPTR];    // (table mode) buckets bucket_lo, ..., then destination tensors
 };
 
@@ -459,44 +467,84 @@ __device__ void compare_in_last_block(unsigned long long* counters,
 template <int NPTR, bool VERIFY, bool CHECK>
 __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
     constexpr int U = 2 * kUnroll;   // one 16-byte load per vector: twice the pack's depth
-    uint32_t i0, i1;
-    block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
+    __shared__ uint32_t next_unit;
+    uint32_t i0 = 0, i1 = 0;
+    unsigned long long pending = 0;   // thread 0: the claim in flight
+    if (!a.claim) {
+        block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
+    } else {
+        if (blockIdx.x < a.n_units) {
+            i0 = a.unit_first[blockIdx.x];
+            i1 = a.unit_first[blockIdx.x + 1];
+        }
+        if (threadIdx.x == 0) pending = atomicAdd(a.claim, 1ull);   // the unit after this one
+    }
     unsigned long long acc = 0;
     uint32_t cur = 0xFFFFFFFFu;
-    for (uint32_t it = i0; it < i1; ++it) {
-        const rr_unpack_item d = a.items[it];
-        if (!VERIFY && d.kind >= RR_ITEM_READ_VEC) continue;
-        if (CHECK && !unpack_item_ok(a.chk, d)) continue;
-        if (VERIFY && d.bucket != cur) {
-            if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - a.first_bucket), acc);
-            cur = d.bucket;
-            acc = 0;
-        }
-        const char* src = (a.bucket_stride ? a.bucket_base + (uint64_t)d.bucket * a.bucket_stride
-                                           : (const char*)a.ptr[d.bucket - a.bucket_lo]) +
-                          d.src_off;
-        const bool copy = d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_COPY_SCALAR;
-        char* dst = copy ? (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off : nullptr;
-        if (d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_READ_VEC) {
-            const uint32_t nvec = d.nbytes >> 4;
-            for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * U) {
-                uint4 x[U];
+    for (;;) {
+        for (uint32_t it = i0; it < i1; ++it) {
+            const rr_unpack_item d = a.items[it];
+            if (!VERIFY && d.kind >= RR_ITEM_READ_VEC) continue;
+            if (CHECK && !unpack_item_ok(a.chk, d)) continue;
+            if (VERIFY && d.bucket != cur) {
+                if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - a.first_bucket), acc);
+                cur = d.bucket;
+                acc = 0;
+            }
+            const char* src = (a.bucket_stride ? a.bucket_base + (uint64_t)d.bucket * a.bucket_stride
+                                               : (const char*)a.ptr[d.bucket - a.bucket_lo]) +
+                              d.src_off;
+            const bool copy = d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_COPY_SCALAR;
+            char* dst = copy ? (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off : nullptr;
+            if (d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_READ_VEC) {
+                const uint32_t nvec = d.nbytes >> 4;
+                for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * U) {
+                    uint4 x[U];
 #pragma unroll
-                for (int u = 0; u < U; ++u)
-                    if (v + u * kThreads < nvec) x[u] = ld_stream(src + 16ull * (v + u * kThreads));
+                    for (int u = 0; u < U; ++u)
+                        if (v + u * kThreads < nvec) x[u] = ld_stream(src + 16ull * (v + u * kThreads));
 #pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    if (v + u * kThreads < nvec) {
-                        if (copy) st_stream(dst + 16ull * (v + u * kThreads), x[u]);
-                        if (VERIFY) acc += words(x[u]);
+                    for (int u = 0; u < U; ++u) {
+                        if (v + u * kThreads < nvec) {
+                            if (copy) st_stream(dst + 16ull * (v + u * kThreads), x[u]);
+                            if (VERIFY) acc += words(x[u]);
+                        }
                     }
                 }
+            } else {
+                for (uint32_t e = threadIdx.x; e < (d.nbytes >> 1); e += kThreads) {
+                    const uint16_t h = *(const uint16_t*)(src + 2ull * e);
+                    if (copy) *(uint16_t*)(dst + 2ull * e) = h;
+                    if (VERIFY) acc += (unsigned long long)h << (8 * ((d.src_off + 2 * e) & 7));
+                }
             }
-        } else {
-            for (uint32_t e = threadIdx.x; e < (d.nbytes >> 1); e += kThreads) {
-                const uint16_t h = *(const uint16_t*)(src + 2ull * e);
-                if (copy) *(uint16_t*)(dst + 2ull * e) = h;
-                if (VERIFY) acc += (unsigned long long)h << (8 * ((d.src_off + 2 * e) & 7));
+        }
+        if (!a.claim) break;
+        // The next unit: the claim issued when this one began (its latency hid
+        // behind the walk), then the following claim goes out at once.
+        __syncthreads();
+        if (threadIdx.x == 0)
+            next_unit = pending < (unsigned long long)(a.n_units - min(a.n_units, gridDim.x))
+                            ? gridDim.x + (uint32_t)pending
+                            : a.n_units;
+        __syncthreads();
+        const uint32_t u = next_unit;
+        if (u >= a.n_units) break;
+        if (threadIdx.x == 0) pending = atomicAdd(a.claim, 1ull);
+        i0 = a.unit_first[u];
+        i1 = a.unit_first[u + 1];
+    }
+    if (a.claim && a.reset_claims) {
+        // A pooled counter goes back to zero for the slot's next launch: the
+        // block that takes the last ticket resets it.  Every block gets here
+        // only after its last claim has returned.
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            __threadfence();
+            if (atomicAdd(a.claim + 1, 1ull) == gridDim.x - 1) {
+                __threadfence();
+                atomicExch(a.claim, 0ull);
+                atomicExch(a.claim + 1, 0ull);
             }
         }
     }
@@ -765,6 +813,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
         enum { kMeta = 0, kBulk = 1, kGather = 2 };
         uint32_t count = 0;   // pieces issued
         bool ok = true;
+        rr_pack_item fan_mine;   // fan-out head: lane l's destination item (l < its count)
         auto emit = [&](const Piece& p, int how) {
             const int s = (int)(count % kStages);
             if (count >= (uint32_t)kStages &&
@@ -775,9 +824,9 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
             }
             const uint32_t fb = smem_u32(&full[s]);
             if constexpr (MODE == 0) {
-                // A fan-out piece carries its destination items in shared memory.
-                if (p.kind == PC_FAN && lane < p.n)
-                    fan_dst[s][lane] = ((const rr_pack_item*)a.items)[p.sum_bucket + lane];
+                // A fan-out piece carries its destination items in shared memory
+                // (each lane's from registers: loaded once per head, not per piece).
+                if (p.kind == PC_FAN && lane < p.n) fan_dst[s][lane] = fan_mine;
             }
             const uint32_t stage = smem_u32(stage_mem + s * kStageBytes);
             const uint32_t row_bytes = p.row_len * p.es;
@@ -891,6 +940,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                                it + 1 + nd > i1 || (uintptr_t)src % 16 != 0 || sstride % 16 != 0;
                     if (!bad && lane < nd) {
                         const rr_pack_item f = ((const rr_pack_item*)a.items)[it + 1 + lane];
+                        fan_mine = f;
                         bad = f.kind != RR_ITEM_FAN_DST || f.row_len % 8 != 0 ||
                               f.dst_off % 16 != 0 || (f.src * es) % 16 != 0 ||
                               f.src + f.row_len > d.row_len || f.n_rows != R ||
@@ -1003,6 +1053,20 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
     const uint32_t sum_base = MODE == 2 ? (uint32_t)a.first_bucket : 0u;
     unsigned long long acc = 0;
     uint32_t cur = 0xFFFFFFFFu;
+    // Fan-out pieces: a warp serves the same slices (so the same buckets) piece
+    // after piece, up to kFanSlots of them per piece.  Each slot keeps its
+    // lane-local partial sum and bucket, and goes out only when its bucket
+    // changes, instead of one warp reduction and atomic per slice and piece.
+    constexpr uint32_t kFanUnitsMax =
+        kMaxFanDst > 2 * kConsumerWarps - 1 ? kMaxFanDst : 2 * kConsumerWarps - 1;
+    constexpr uint32_t kFanSlots = (kFanUnitsMax + kConsumerWarps - 1) / kConsumerWarps;
+    unsigned long long fan_acc[kFanSlots];
+    uint32_t fan_bucket[kFanSlots];
+#pragma unroll
+    for (uint32_t j = 0; j < kFanSlots; ++j) {
+        fan_acc[j] = 0;
+        fan_bucket[j] = 0xFFFFFFFFu;
+    }
     bool ok = true;
     for (uint32_t c = 0;; ++c) {
         const int s = (int)(c % kStages);
@@ -1054,11 +1118,23 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                 if constexpr (MODE == 0) {
                     // Units of work: each slice's 16-byte output vectors in q parts
                     // (q spreads the slices over all consumer warps, whatever the
-                    // number of rows staged); one warp per unit, one sum per unit.
+                    // number of rows staged); one warp per unit.  nd <= kMaxFanDst
+                    // (the producer refuses more), so nd * q <= kFanUnitsMax and a
+                    // warp takes at most kFanSlots units: unit j of this warp sums
+                    // into slot j.
                     const uint32_t nd = p.n;
                     const uint32_t q = (kConsumerWarps + nd - 1) / nd;
-                    for (uint32_t u = warp - 1; u < nd * q; u += kConsumerWarps) {
+#pragma unroll
+                    for (uint32_t j = 0; j < kFanSlots; ++j) {
+                        const uint32_t u = warp - 1 + j * kConsumerWarps;
+                        if (u >= nd * q) break;
                         const rr_pack_item d = fan_dst[s][u / q];
+                        if (d.bucket != fan_bucket[j]) {   // warp-uniform
+                            if (fan_bucket[j] != 0xFFFFFFFFu)
+                                flush(a.sums + fan_bucket[j], fan_acc[j]);
+                            fan_bucket[j] = d.bucket;
+                            fan_acc[j] = 0;
+                        }
                         const uint32_t part = u % q;
                         const uint32_t vpr = d.row_len >> 3, nv_all = p.rows * vpr;
                         const uint32_t v0 = nv_all * part / q, v1 = nv_all * (part + 1) / q;
@@ -1092,7 +1168,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                                 ++r;
                             }
                         }
-                        flush(a.sums + d.bucket, am);
+                        fan_acc[j] += am;
                     }
                 }
                 break;
@@ -1108,6 +1184,11 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
         if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
     }
     if (kSum && cur != 0xFFFFFFFFu) flush(a.sums + (cur - sum_base), acc);
+    if constexpr (MODE == 0) {
+#pragma unroll
+        for (uint32_t j = 0; j < kFanSlots; ++j)
+            if (fan_bucket[j] != 0xFFFFFFFFu) flush(a.sums + fan_bucket[j], fan_acc[j]);
+    }
     if (MODE != 2) return;
     // Checksum comparison by whichever block finishes last (consumer threads only).
     consumers_sync<kCT>();
@@ -1274,6 +1355,10 @@ ItemBounds bounds_of(const rr_plan* P) {
     return b;
 }
 
+int32_t take_claim_slot(rr_plan* M, cudaStream_t s);
+template <int MODE>
+void work_units(const rr_plan* P, const Range& R, const uint32_t** first, uint32_t* n);
+
 template <int NPTR>
 rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* const* buckets,
                       uint64_t* checksums, bool table, uint64_t stride, cudaStream_t s) {
@@ -1335,6 +1420,23 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     }
     a.dst_base = k - R.t_lo;   // ptr[dst_base + tensor] for tensors t_lo .. t_hi
     for (int32_t t = R.t_lo; t <= R.t_hi; ++t) a.ptr[k++] = dst[t];
+    // Claimed work units (the per-bucket units of R's buckets): the verifying
+    // form through the call's scratch counter, zeroed with its sums; the plain
+    // form through a pooled slot when one is free, else the fixed split above.
+    rr_plan* M = const_cast<rr_plan*>(P);   // the claim pool is mutable state
+    std::unique_lock<std::mutex> lock(M->claim_mutex, std::defer_lock);
+    int32_t slot = -1;
+    if (checksums) {
+        a.claim = a.counters + 3;
+        work_units<1>(P, R, &a.unit_first, &a.n_units);
+    } else {
+        lock.lock();
+        if ((slot = take_claim_slot(M, s)) >= 0) {
+            a.claim = P->d_claims + 2 * slot;
+            a.reset_claims = 1;
+            work_units<1>(P, R, &a.unit_first, &a.n_units);
+        }
+    }
     if (checksums && P->check_items)
         rr_unpack_kernel<NPTR, true, true><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
     else if (checksums)
@@ -1344,6 +1446,11 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     else
         rr_unpack_kernel<NPTR, false, false><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
     RR_CUDA(cudaGetLastError());
+    cudaError_t e;
+    if (slot >= 0 && (e = cudaEventRecord(P->claim_done[slot], s)) != cudaSuccess) {
+        M->claim_retired[slot] = 1;   // its launch's end is unknown: never hand it out again
+        return cuda_fail(e, "cudaEventRecord");
+    }
     return RR_OK;
 }
 

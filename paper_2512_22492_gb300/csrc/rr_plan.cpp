@@ -33,7 +33,24 @@ namespace {
 thread_local std::string g_error;
 
 constexpr int64_t kDefaultChunkBytes = 32 * 1024;
-constexpr int64_t kItemOverhead = 1024;   // balancing weight of one item, in bytes
+// Balancing weights (build-time overridable for tuning sweeps).
+#ifndef RR_ITEM_OVERHEAD
+#define RR_ITEM_OVERHEAD 1024
+#endif
+#ifndef RR_ZERO_WEIGHT
+#define RR_ZERO_WEIGHT 2
+#endif
+#ifndef RR_OWN_SHARE_PCT
+#define RR_OWN_SHARE_PCT 85
+#endif
+#ifndef RR_TAPER
+#define RR_TAPER 1
+#endif
+#ifndef RR_TAPER_FLOOR
+#define RR_TAPER_FLOOR (64 * 1024)
+#endif
+constexpr int64_t kItemOverhead = RR_ITEM_OVERHEAD;   // balancing weight of one item, in bytes
+constexpr int64_t kZeroWeight = RR_ZERO_WEIGHT;       // weight of one zero-filled element
 constexpr int64_t kUnitWeight = 1 << 20;   // largest claimed work unit (weight), and the
 constexpr int32_t kUnitsPerBlock = 32;     //   units wanted per block of the grid
 constexpr int64_t kMaxShardOffset = (int64_t(1) << 48) - 1;
@@ -350,7 +367,7 @@ int64_t pack_weight(const rr_pack_item& it) {
         case RR_ITEM_FAN_F32: return 6 * n + kItemOverhead;
         case RR_ITEM_FAN_BF16: return 4 * n + kItemOverhead;
         case RR_ITEM_FAN_DST: return 0;
-        default: return 2 * n + kItemOverhead;
+        default: return kZeroWeight * n + kItemOverhead;
     }
 }
 
@@ -377,33 +394,50 @@ void partition(const std::vector<Item>& items, int32_t grid, std::vector<uint32_
     }
 }
 
+// Claimed units get smaller toward the end of the table (guided
+// self-scheduling): a unit that starts with `rem` weight left before the end is
+// about rem / (2 * grid), clamped to [floor, unit_weight].  Blocks drain HBM at
+// unequal rates and stop within one unit of one another; with the last units
+// small, they stop together.
+int64_t taper_size(int64_t rem, int64_t unit_weight, int32_t grid) {
+    if (!RR_TAPER) return unit_weight;
+    const int64_t floor = std::min<int64_t>(unit_weight, RR_TAPER_FLOOR);
+    return std::max(floor, std::min(unit_weight, rem / (2 * int64_t(std::max(1, grid)))));
+}
+
 // Work units for a kernel whose blocks claim work as they run out of it.  Each
-// bucket's items are cut into units of about kUnitWeight (a unit never spans
-// two buckets, so a bucket-range call takes a contiguous run of units):
-// first[u] is the first item of unit u, bucket_unit[b] the first unit of
-// bucket b.  Blocks drain HBM at unequal rates; small units claimed one at a
-// time let the fast blocks take more of them, and all finish together.
+// bucket's items are cut into units (a unit never spans two buckets, so a
+// bucket-range call takes a contiguous run of units) of about taper_size of
+// the weight left to the table's end: first[u] is the first item of unit u,
+// bucket_unit[b] the first unit of bucket b.  Small units claimed one at a
+// time let the fast blocks take more of them, and all finish together.  Within
+// a bucket a cut falls after the item that reaches the unit's size, unless
+// less than a quarter unit would be left in the bucket; no unit is empty.
 template <class Item, class W>
 void bucket_units(const std::vector<Item>& items, const std::vector<uint32_t>& bucket_first,
-                  int64_t unit_weight, std::vector<uint32_t>& first,
+                  int64_t unit_weight, int32_t grid, std::vector<uint32_t>& first,
                   std::vector<uint32_t>& bucket_unit, W w) {
     first.clear();
     bucket_unit.assign(bucket_first.size(), 0);
+    int64_t rem = 0;   // weight from the current item to the end of the table
+    for (const Item& it : items) rem += w(it);
     for (size_t b = 0; b + 1 < bucket_first.size(); ++b) {
         bucket_unit[b] = uint32_t(first.size());
         const uint32_t lo = bucket_first[b], hi = bucket_first[b + 1];
         if (lo == hi) continue;
-        int64_t total = 0;
-        for (uint32_t i = lo; i < hi; ++i) total += w(items[i]);
-        const int64_t n = std::max<int64_t>(1, (total + unit_weight - 1) / unit_weight);
-        first.push_back(lo);
-        int64_t cum = 0, k = 1;
-        for (uint32_t i = lo; i < hi && k < n; ++i) {
-            cum += w(items[i]);
-            // A cut after item i when it reaches the next share (no empty units).
-            if (cum * n >= total * k && i + 1 < hi) {
-                first.push_back(i + 1);
-                while (k < n && cum * n >= total * k) ++k;
+        int64_t left = 0;   // weight left in this bucket
+        for (uint32_t i = lo; i < hi; ++i) left += w(items[i]);
+        uint32_t i = lo;
+        while (i < hi) {
+            first.push_back(i);
+            const int64_t size = taper_size(rem, unit_weight, grid);
+            int64_t cum = 0;
+            while (i < hi) {
+                const int64_t wi = w(items[i++]);
+                cum += wi;
+                rem -= wi;
+                left -= wi;
+                if (cum >= size && left * 4 >= size) break;
             }
         }
     }
@@ -413,29 +447,39 @@ void bucket_units(const std::vector<Item>& items, const std::vector<uint32_t>& b
 
 // Units for a launch over every bucket (the table it runs is fixed): blocks
 // first drain kOwnShare of the table's weight in equal contiguous shares (unit
-// g < grid is block g's own: no claims, long runs), then claim units of about
-// unit_weight over the rest.  A cut never falls before a fan-out destination
-// item (a head and its destinations stay in one unit).
-constexpr int64_t kOwnShareNum = 7, kOwnShareDen = 10;
+// g < grid is block g's own: no claims, long runs), then claim units of
+// taper_size over the rest.  Own units may be empty.  A cut never falls before
+// a fan-out destination item (a head and its destinations stay in one unit).
+constexpr int64_t kOwnShareNum = RR_OWN_SHARE_PCT, kOwnShareDen = 100;
 template <class Item, class W>
 void whole_units(const std::vector<Item>& items, int32_t grid, int64_t unit_weight,
                  std::vector<uint32_t>& first, W w) {
     int64_t total = 0;
     for (const Item& it : items) total += w(it);
     const int64_t own = total * kOwnShareNum / kOwnShareDen;
-    const int64_t claimed = std::max<int64_t>(1, (total - own + unit_weight - 1) / unit_weight);
-    const int64_t U = int64_t(grid) + claimed;
-    auto target = [&](int64_t g) {   // weight before unit g
-        return g <= grid ? own * g / grid : own + (total - own) * (g - grid) / claimed;
-    };
-    first.assign(size_t(U) + 1, uint32_t(items.size()));
+    first.assign(size_t(grid) + 1, uint32_t(items.size()));
     first[0] = 0;
-    int64_t cum = 0, g = 1;
-    for (size_t i = 0; i < items.size() && g < U; ++i) {
-        cum += w(items[i]);
-        if (i + 1 < items.size() && items[i + 1].kind == RR_ITEM_FAN_DST) continue;
-        while (g < U && cum >= target(g)) first[size_t(g++)] = uint32_t(i + 1);
+    int64_t cum = 0;
+    size_t i = 0;
+    // Own shares: the cut before unit g at the first item boundary reaching own * g / grid.
+    for (int64_t g = 1; g <= grid; ++g) {
+        while (i < items.size() &&
+               (cum < own * g / grid || (i < items.size() && items[i].kind == RR_ITEM_FAN_DST)))
+            cum += w(items[i++]);
+        first[size_t(g)] = uint32_t(i);
     }
+    // Claimed units over the rest, smaller toward the end.
+    while (i < items.size()) {
+        const int64_t size = taper_size(total - cum, unit_weight, grid);
+        int64_t u = 0;
+        while (i < items.size() && (u < size || items[i].kind == RR_ITEM_FAN_DST)) {
+            const int64_t wi = w(items[i++]);
+            u += wi;
+            cum += wi;
+        }
+        first.push_back(uint32_t(i));
+    }
+    if (first.size() == size_t(grid) + 1) first.push_back(uint32_t(items.size()));
 }
 
 // Claimed-unit weight for a table: about kUnitsPerBlock units per block of the
@@ -758,10 +802,11 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
     partition(P->unpack_items, P->unpack_grid_blocks, P->unpack_block_first, unpack_weight);
     bucket_units(P->unpack_items, P->unpack_bucket_first,
                  unit_weight_for(P->unpack_items, P->unpack_grid_blocks, unpack_weight),
-                 P->unpack_unit_first, P->unpack_bucket_unit, unpack_weight);
+                 P->unpack_grid_blocks, P->unpack_unit_first, P->unpack_bucket_unit,
+                 unpack_weight);
     bucket_units(P->pack_items, P->pack_bucket_first,
-                 unit_weight_for(P->pack_items, P->grid_blocks, pack_weight), P->pack_unit_first,
-                 P->pack_bucket_unit, pack_weight);
+                 unit_weight_for(P->pack_items, P->grid_blocks, pack_weight), P->grid_blocks,
+                 P->pack_unit_first, P->pack_bucket_unit, pack_weight);
     // Summed weights: a bucket-range call splits its items over the grid by them.
     auto prefix = [](const auto& items, std::vector<unsigned long long>& out, auto w) {
         out.assign(items.size() + 1, 0ull);

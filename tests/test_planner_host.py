@@ -176,31 +176,44 @@ def unit_weights(p, which):
     return items, w
 
 
+def taper(rem, unit, grid, floor=64 * 1024):
+    """The claimed-unit size for `rem` weight left before the table's end."""
+    return max(min(unit, floor), min(unit, rem // (2 * grid)))
+
+
 @pytest.mark.parametrize("name,which", [("qwen3-0.6b", "unpack"), ("qwen3-8b", "unpack"),
                                         ("qwen3-30b-a3b-fsdp2-tp8", "unpack"),
                                         ("qwen3-0.6b", "pack"), ("qwen3-8b", "pack")])
 def test_bucket_units_on_full_size_tables(name, which):
-    """Per-bucket units of equal weight: at most 1 MiB, or less where that would
-    leave a block of the grid fewer than 32; none heavier than that plus one
-    item, and only a bucket's last unit much lighter."""
+    """Per-bucket units: a unit's size is about the weight left to the table's
+    end over twice the grid, at most 1 MiB (or less where that would leave a
+    block of the grid fewer than 32) and at least 64 KiB.  A unit is cut at the
+    item reaching its size unless under a quarter of it would be left in the
+    bucket, so only a bucket's last unit is lighter; sizes shrink toward the end."""
     p = host_plan(U.workload_desc(name))
     items, w = unit_weights(p, which)
     first, bucket_unit = U.check_units(p, len(items), which)
     grid = p.stats()["unpack_grid_blocks" if which == "unpack" else "grid_blocks"]
     unit = min(1 << 20, max((1 << 20) // 8, int(w.sum()) // (32 * grid)))
-    unit_w = np.add.reduceat(w, first[:-1])
-    assert unit_w.max() <= unit + w.max()
+    cum = np.concatenate([[0], np.cumsum(w)])
+    total = int(cum[-1])
+    unit_w = cum[first[1:]] - cum[first[:-1]]
+    size = np.array([taper(total - int(cum[f]), unit, grid) for f in first[:-1]])
+    assert np.all(np.diff(size) <= 0)
+    assert size[0] == unit and size[-1] == min(unit, 64 * 1024)
+    assert np.all(unit_w <= size + size // 4 + w.max())
     last = np.zeros(len(unit_w), bool)
     last[bucket_unit[1:][np.diff(bucket_unit) > 0] - 1] = True
-    assert np.all(unit_w[~last] >= unit // 2 - w.max())
+    assert np.all(unit_w[~last] >= size[~last])
     assert len(unit_w) >= 16 * grid
 
 
 @pytest.mark.parametrize("name", ["qwen3-0.6b", "qwen3-8b", "qwen3-30b-a3b-fsdp2-tp8"])
 def test_whole_pack_units_on_full_size_tables(name):
-    """A pack over every bucket: one own unit per block, together 70% of the
+    """A pack over every bucket: one own unit per block, together 85% of the
     weight in equal shares (to within one item, or one fan-out group), then
-    claimed units of at most the per-bucket size plus one item."""
+    claimed units of the tapered size (the weight left over twice the grid,
+    within [64 KiB, the per-bucket unit size]) plus at most one item."""
     which = "pack_full"
     p = host_plan(U.workload_desc(name))
     items, w = unit_weights(p, which)
@@ -212,11 +225,14 @@ def test_whole_pack_units_on_full_size_tables(name):
     cum = np.concatenate([[0], np.cumsum(w)])
     unit_w = cum[first[1:]] - cum[first[:-1]]
     total = int(cum[-1])
-    own = total * 7 // 10
+    own = total * 85 // 100
     assert abs(int(cum[first[grid]]) - own) <= heaviest
     assert np.all(np.abs(unit_w[:grid] - own / grid) <= heaviest + 1)
     unit = min(1 << 20, max((1 << 20) // 8, total // (32 * grid)))
-    assert unit_w[grid:].max() <= unit + heaviest
+    size = np.array([taper(total - int(cum[f]), unit, grid) for f in first[grid:-1]])
+    assert np.all(unit_w[grid:] <= size + heaviest)
+    assert np.all(unit_w[grid:-1] >= size[:-1])
+    assert np.all(np.diff(size) <= 0) and size[-1] == min(unit, 64 * 1024)
 
 
 def test_fan_out_groups_on_full_size_tables():
