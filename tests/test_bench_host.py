@@ -84,7 +84,8 @@ def test_visible_gpu_index(monkeypatch):
 
 def test_profiled_traffic_needs_the_current_kernel(tmp_path, monkeypatch):
     """The profile's traffic is reported only while the code it was taken on
-    is unchanged; a comment edit does not count as a change."""
+    is unchanged (a comment edit does not count as a change), scaled from the
+    small captured case to a full launch by the ratio of algorithmic bytes."""
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     (tmp_path / "profiles").mkdir()
     (tmp_path / "include").mkdir()
@@ -95,18 +96,61 @@ def test_profiled_traffic_needs_the_current_kernel(tmp_path, monkeypatch):
     (src / "rr_device.cu").write_text("int kernel_v1(void) { return 1; }  // first\n")
     good = bench.kernel_code_hash()
     page = tmp_path / "profiles" / "rr_pack_demo.md"
-    page.write_text(f"kernel_code_sha256_16: {good}\ndram_bytes_per_launch_full: 123\n")
-    assert bench.profiled_traffic("demo") == 123
+    page.write_text(f"kernel_code_sha256_16: {good}\ndram_bytes_per_launch_small: 990\n"
+                    f"algorithmic_bytes_small: 1000\n")
+    assert bench.profiled_traffic("demo", 1000) == 990
+    assert bench.profiled_traffic("demo", 50_000) == 49_500    # scaled to the full launch
     (src / "rr_device.cu").write_text("/* new words */ int kernel_v1(void)\n{\n  return 1;  // said\n}\n")
-    assert bench.profiled_traffic("demo") == 123        # comments and layout only
+    assert bench.profiled_traffic("demo", 1000) == 990        # comments and layout only
     (src / "rr_device.cu").write_text("int kernel_v1(void) { return 2; }\n")
-    assert bench.profiled_traffic("demo") is None       # the code changed since the capture
+    assert bench.profiled_traffic("demo", 1000) is None       # the code changed since the capture
     (src / "rr_device.cu").write_text("int kernel_v1(void) { return 1; }\n")
-    (src / "rr_plan.cpp").write_text("int x = 1;\n")      # so did the planner's
-    assert bench.profiled_traffic("demo") is None
-    assert bench.profiled_traffic("other") is None
+    (src / "rr_plan.cpp").write_text("int x = 1;\n")          # so did the planner's
+    assert bench.profiled_traffic("demo", 1000) is None
+    assert bench.profiled_traffic("other", 1000) is None
+    (src / "rr_plan.cpp").write_text("int x; // a\n")
+    assert bench.profiled_traffic("demo", 1000) == 990
+    page.write_text(f"kernel_code_sha256_16: {good}\ndram_bytes_per_launch_full: 123\n")
+    assert bench.profiled_traffic("demo", 1000) is None       # full-size figures are not read
 
 
 def test_aggregate_and_host_memory():
     assert bench.aggregate_gbs(4, 1_000_000_000, 10.0) == pytest.approx(400.0)
     assert bench.host_memory_bytes() > 1 << 30
+
+
+def test_ready_runs():
+    assert bench.ready_runs([True, True, False, True]) == [(0, 2), (3, 4)]
+    assert bench.ready_runs([False, False]) == []
+    assert bench.ready_runs([]) == []
+    assert bench.ready_runs([True] * 3) == [(0, 3)]
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-fsdp2", "tiny-units"])
+def test_bucket_source_needs_cover_every_read(name):
+    """The pipelined e2e packs a bucket once the first need[b] bytes of the
+    source block have landed.  The oracle, given only those bytes (the rest
+    zero), must produce that bucket exactly as from the whole source."""
+    import numpy as np
+    import oracle
+    import paper_2512_22492_gb300 as rr
+    from synth import device as D
+    from tests import _util as U
+    desc = U.workload_desc(name)
+    L = U.to_oracle(desc)
+    m, s, d = U.to_product(desc)
+    plan = rr.rr_plan_create(m, s, d, desc["bucket_bytes"], rr.PlanOptions(host_only=1))
+    need = bench.bucket_source_needs(plan)
+    shards = L.host_shards(desc["seed"], desc["specials"])
+    starts = D.source_offsets(plan)
+    block = np.zeros(starts[-1], np.uint8)
+    for i, sh in enumerate(shards):
+        block[starts[i]:starts[i] + len(sh)] = sh
+    assert need.max() <= starts[-1] and need.min() >= 0
+    full, full_cs = L.pack(oracle.Source(shards=shards))
+    for b in range(plan.n_buckets):
+        cut = block.copy()
+        cut[need[b]:] = 0
+        part = [cut[starts[i]:starts[i] + len(sh)] for i, sh in enumerate(shards)]
+        got, cs = L.pack(oracle.Source(shards=part), first=b, count=1)
+        np.testing.assert_array_equal(got[0], full[b], err_msg=f"bucket {b}")
