@@ -114,11 +114,12 @@ struct UnpackArgs {
     // Claimed work units (claim NULL: none, the split above).  unit_first holds
     // the first item of each of n_units units and one past the last; block g
     // walks unit g, then claims the next unclaimed unit (atomicAdd on *claim,
-    // zero at launch) until none are left.
+    // zero at launch) until none are left.  claim is counters + 3.
     const uint32_t* unit_first;
     unsigned long long* claim;
     uint32_t n_units;
-    uint32_t reset_claims;    // claim is a pooled slot {counter, ticket}: zero it at the end
+    uint32_t reset_claims;    // counters are a pooled slot's: its last block leaves them zero
+    long long* result;        // verifying: {n_bad, first_bad or -1} written at the end, or NULL
     const void* ptr[NPTR];    // (table mode) buckets bucket_lo, ..., then destination tensors
 };
 
@@ -400,8 +401,12 @@ __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(c
     block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
     unsigned long long acc = 0;
     uint32_t cur = 0xFFFFFFFFu;
+    // The next item's load is in flight while the current one is moved.
+    rr_pack_item next;
+    if (i0 < i1) next = a.items[i0];
     for (uint32_t it = i0; it < i1; ++it) {
-        const rr_pack_item d = a.items[it];
+        const rr_pack_item d = next;
+        if (it + 1 < i1) next = a.items[it + 1];
         if (CHECK && !pack_item_ok(a.chk, d)) continue;
         if (d.bucket != cur) {
             if (cur != 0xFFFFFFFFu) flush(a.checksums + cur, acc);
@@ -433,10 +438,18 @@ __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(c
 // no block waits for another).  sums[i] belongs to bucket first + i.
 // ---------------------------------------------------------------------------
 
+// The last block's result: counters[1] mismatches, the lowest one's index
+// from counters[2] (which holds ULLONG_MAX - index), or -1.
+__device__ __forceinline__ void write_result(unsigned long long* counters, long long* result) {
+    const unsigned long long nb = atomicAdd(&counters[1], 0ull);
+    result[0] = (long long)nb;
+    result[1] = nb ? (long long)(ULLONG_MAX - atomicAdd(&counters[2], 0ull)) : -1ll;
+}
+
 __device__ void compare_in_last_block(unsigned long long* counters,
                                       const unsigned long long* sums,
                                       const unsigned long long* expected, uint8_t* bad,
-                                      int32_t first, int32_t n) {
+                                      int32_t first, int32_t n, long long* result = nullptr) {
     __shared__ bool last;
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -455,6 +468,10 @@ __device__ void compare_in_last_block(unsigned long long* counters,
             atomicMax(&counters[2], ULLONG_MAX - (unsigned long long)b);
         }
     }
+    if (result) {
+        __syncthreads();
+        if (threadIdx.x == 0) write_result(counters, result);
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -467,8 +484,9 @@ __device__ void compare_in_last_block(unsigned long long* counters,
 template <int NPTR, bool VERIFY, bool CHECK>
 __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
     constexpr int U = 2 * kUnroll;   // one 16-byte load per vector: twice the pack's depth
-    __shared__ uint32_t next_unit;
+    __shared__ uint32_t next_unit[2];   // the claimed unit, double-buffered by parity
     uint32_t i0 = 0, i1 = 0;
+    uint32_t walked = 0;              // units this block has walked
     unsigned long long pending = 0;   // thread 0: the claim in flight
     if (!a.claim) {
         block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
@@ -482,8 +500,12 @@ __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_con
     unsigned long long acc = 0;
     uint32_t cur = 0xFFFFFFFFu;
     for (;;) {
+        // The next item's load is in flight while the current one is moved.
+        rr_unpack_item next;
+        if (i0 < i1) next = a.items[i0];
         for (uint32_t it = i0; it < i1; ++it) {
-            const rr_unpack_item d = a.items[it];
+            const rr_unpack_item d = next;
+            if (it + 1 < i1) next = a.items[it + 1];
             if (!VERIFY && d.kind >= RR_ITEM_READ_VEC) continue;
             if (CHECK && !unpack_item_ok(a.chk, d)) continue;
             if (VERIFY && d.bucket != cur) {
@@ -521,37 +543,40 @@ __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_con
         }
         if (!a.claim) break;
         // The next unit: the claim issued when this one began (its latency hid
-        // behind the walk), then the following claim goes out at once.
-        __syncthreads();
+        // behind the walk), published by thread 0 in this unit's parity slot
+        // (the other slot may still be read by warps leaving the previous
+        // barrier), then the following claim goes out at once.  One barrier
+        // per unit.
+        const uint32_t par = walked++ & 1u;
         if (threadIdx.x == 0)
-            next_unit = pending < (unsigned long long)(a.n_units - min(a.n_units, gridDim.x))
-                            ? gridDim.x + (uint32_t)pending
-                            : a.n_units;
+            next_unit[par] = pending < (unsigned long long)(a.n_units - min(a.n_units, gridDim.x))
+                                 ? gridDim.x + (uint32_t)pending
+                                 : a.n_units;
         __syncthreads();
-        const uint32_t u = next_unit;
+        const uint32_t u = next_unit[par];
         if (u >= a.n_units) break;
         if (threadIdx.x == 0) pending = atomicAdd(a.claim, 1ull);
         i0 = a.unit_first[u];
         i1 = a.unit_first[u + 1];
     }
     if (a.claim && a.reset_claims) {
-        // A pooled counter goes back to zero for the slot's next launch: the
-        // block that takes the last ticket resets it.  Every block gets here
-        // only after its last claim has returned.
+        // A pooled slot's counters go back to zero for its next launch: the
+        // block that takes the last ticket (counters[0]) resets them.  Every
+        // block gets here only after its last claim has returned.
         __syncthreads();
         if (threadIdx.x == 0) {
             __threadfence();
-            if (atomicAdd(a.claim + 1, 1ull) == gridDim.x - 1) {
+            if (atomicAdd(&a.counters[0], 1ull) == gridDim.x - 1) {
                 __threadfence();
                 atomicExch(a.claim, 0ull);
-                atomicExch(a.claim + 1, 0ull);
+                atomicExch(&a.counters[0], 0ull);
             }
         }
     }
     if (VERIFY) {
         if (cur != 0xFFFFFFFFu) flush(a.sums + (cur - a.first_bucket), acc);
         compare_in_last_block(a.counters, a.sums, a.expected, a.bad, a.first_bucket,
-                              a.n_buckets);
+                              a.n_buckets, a.result);
     }
 }
 
@@ -671,6 +696,7 @@ struct Piece {
 template <int NPTR>
 struct BulkArgs {
     const void* items;           // rr_pack_item (MODE 0) or rr_unpack_item
+    uint32_t n_items;            // items in that table (the producer reads ahead, never past)
     const uint32_t* block_first; // as in PackArgs
     uint32_t item_begin;
     uint32_t item_end;
@@ -682,22 +708,50 @@ struct BulkArgs {
     int32_t dst_base;            // unpack: index in ptr[] of destination tensor 0
     int32_t bucket_lo;           // table mode: the first bucket the table holds
     int32_t pad_;
-    unsigned long long* sums;    // pack: checksums by bucket; verify: range sums
-    unsigned long long* counters;
+    unsigned long long* sums;    // pack: sums by global bucket; verify: range sums
+    unsigned long long* counters;// {ticket, n_bad, max(~0 - bad index), claim}
     const unsigned long long* expected;
     uint8_t* bad;
-    int32_t first_bucket;
+    int32_t first_bucket;        // the call's range [first_bucket, first_bucket + n_buckets)
     int32_t n_buckets;
     unsigned int* err;
     // Claimed work units (NULL: none).  block_first then holds the first item
     // of each of n_units units (and one past the last): unit g < gridDim.x is
     // block g's own, the rest go to whichever block asks next (atomicAdd on
-    // *claim, zero at launch).
+    // *claim = counters[3], zero at launch).
     unsigned long long* claim;
     uint32_t n_units;
-    uint32_t reset_claims;       // claim is a pooled slot {counter, ticket}: zero it at the end
+    // The launch holds a pooled slot (counters, and sums for pack and the
+    // verifying unpack): its last block leaves them zero for the slot's next
+    // launch.
+    uint32_t reset_claims;
+    unsigned long long* sums_out;  // pack through a slot: checksums[b] = sums[b] at the end
+    long long* result;             // verifying unpack: {n_bad, first_bad or -1}, or NULL
     const void* ptr[NPTR];
 };
+
+static_assert(sizeof(rr_pack_item) == 32 && sizeof(rr_unpack_item) == 32,
+              "the producer's item window moves 32-byte items as two 16-byte words");
+
+// A 32-byte work item as two 16-byte words (the window's unit of transfer).
+template <class Item>
+union ItemWords {
+    uint4 w[2];
+    Item item;
+};
+
+// Lane `src`'s two words, for every lane of the warp.
+__device__ __forceinline__ void shfl_words(const uint4& a, const uint4& b, int src, uint4& x,
+                                           uint4& y) {
+    x.x = __shfl_sync(0xFFFFFFFFu, a.x, src);
+    x.y = __shfl_sync(0xFFFFFFFFu, a.y, src);
+    x.z = __shfl_sync(0xFFFFFFFFu, a.z, src);
+    x.w = __shfl_sync(0xFFFFFFFFu, a.w, src);
+    y.x = __shfl_sync(0xFFFFFFFFu, b.x, src);
+    y.y = __shfl_sync(0xFFFFFFFFu, b.y, src);
+    y.z = __shfl_sync(0xFFFFFFFFu, b.z, src);
+    y.w = __shfl_sync(0xFFFFFFFFu, b.w, src);
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return (uint32_t)__cvta_generic_to_shared(p);
@@ -728,11 +782,6 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigne
 
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-template <int kConsumerThreads>
-__device__ __forceinline__ void consumers_sync() {
-    asm volatile("bar.sync 1, %0;" ::"n"(kConsumerThreads) : "memory");
 }
 
 // Short aligned rows (16-byte aligned, row bytes a multiple of 16) gathered
@@ -792,9 +841,14 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                          : "memory");
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        // Programmatic dependent launch: the next kernel on the stream may be
+        // scheduled now; it still waits for this grid's completion before it
+        // touches memory (its griddepcontrol.wait below).
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     }
     __syncthreads();
 
+    // The plan's tables are immutable: read them before the wait.
     uint32_t i0 = 0, i1 = 0;
     if (!a.claim)
         block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
@@ -802,6 +856,10 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
         i0 = a.block_first[blockIdx.x];
         i1 = a.block_first[blockIdx.x + 1];
     }
+    // Everything else (sources, buckets, tensors, sums, counters) may be the
+    // previous kernel's output: wait for it to complete.  A no-op when the
+    // launch did not overlap a previous kernel.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
@@ -874,17 +932,46 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
             i1 = a.block_first[u + 1];
             return true;
         };
+        // Work items pass through a window: lane l holds item win + l (one
+        // coalesced 32-byte load per lane) and item win + 32 + l is already in
+        // flight, so the walk reads an item with shuffles rather than waiting
+        // on a dependent global load for every item.  A jump (a claimed unit)
+        // reloads both halves.
+        uint32_t win = 0xFFFFFFFFu;
+        uint4 w0 = make_uint4(0, 0, 0, 0), w1 = w0, n0 = w0, n1 = w0;
+        auto load_words = [&](uint32_t i, uint4& x0, uint4& x1) {
+            if (i < a.n_items) {
+                const uint4* q = (const uint4*)((const char*)a.items + 32ull * i);
+                x0 = __ldg(q);
+                x1 = __ldg(q + 1);
+            }
+        };
+        auto window_to = [&](uint32_t at) {   // warp-uniform: win <= at < win + 32
+            if (win != 0xFFFFFFFFu && at - win < 32u) return;
+            if (win != 0xFFFFFFFFu && at - win < 64u) {
+                w0 = n0;
+                w1 = n1;
+                win += 32;
+            } else {
+                win = at;
+                load_words(win + lane, w0, w1);
+            }
+            load_words(win + 32 + lane, n0, n1);
+        };
         for (uint32_t it = i0; ok; ++it) {
             if (it >= i1) {
                 bool more = true;
                 while (more && it >= i1) more = next_range(&it);
                 if (!more) break;
             }
+            window_to(it);
             Piece p;
             p.dst = nullptr;
             p.src_stride = 0;
             if (MODE == 0) {
-                const rr_pack_item d = ((const rr_pack_item*)a.items)[it];
+                ItemWords<rr_pack_item> di;
+                shfl_words(w0, w1, (int)(it - win), di.w[0], di.w[1]);
+                const rr_pack_item d = di.item;
                 if (CHECK && !pack_item_ok(a.chk, d)) {
                     if (d.kind == RR_ITEM_FAN_F32 || d.kind == RR_ITEM_FAN_BF16)
                         it += min(d.dst_off, i1 - 1 - it);   // and its destinations
@@ -938,9 +1025,17 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     // a table that breaks them is refused, not run.
                     bool bad = rb > (uint32_t)kStageBytes || rb % 16 != 0 || nd > kMaxFanDst ||
                                it + 1 + nd > i1 || (uintptr_t)src % 16 != 0 || sstride % 16 != 0;
+                    // Lane l's destination is item it + 1 + l: in this window or
+                    // the next (it - win < 32 and nd <= kMaxFanDst).
+                    {
+                        const uint32_t k = it + 1 + min((uint32_t)lane, nd > 0 ? nd - 1 : 0u) - win;
+                        ItemWords<rr_pack_item> c, n;
+                        shfl_words(w0, w1, (int)(k & 31u), c.w[0], c.w[1]);
+                        shfl_words(n0, n1, (int)(k & 31u), n.w[0], n.w[1]);
+                        fan_mine = k < 32u ? c.item : n.item;
+                    }
                     if (!bad && lane < nd) {
-                        const rr_pack_item f = ((const rr_pack_item*)a.items)[it + 1 + lane];
-                        fan_mine = f;
+                        const rr_pack_item f = fan_mine;
                         bad = f.kind != RR_ITEM_FAN_DST || f.row_len % 8 != 0 ||
                               f.dst_off % 16 != 0 || (f.src * es) % 16 != 0 ||
                               f.src + f.row_len > d.row_len || f.n_rows != R ||
@@ -989,7 +1084,9 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     emit(p, kMeta);
                 }
             } else {
-                const rr_unpack_item d = ((const rr_unpack_item*)a.items)[it];
+                ItemWords<rr_unpack_item> di;
+                shfl_words(w0, w1, (int)(it - win), di.w[0], di.w[1]);
+                const rr_unpack_item d = di.item;
                 const bool read_only = d.kind == RR_ITEM_READ_VEC || d.kind == RR_ITEM_READ_SCALAR;
                 if (MODE == 1 && read_only) continue;
                 if (CHECK && !unpack_item_ok(a.chk, d)) continue;
@@ -1034,18 +1131,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                 mbar_wait(smem_u32(&full[c % kStages]), (c / kStages) & 1, a.err);
         }
         asm volatile("cp.async.wait_all;" ::: "memory");
-        if (a.claim && a.reset_claims && lane == 0) {
-            // A pooled counter goes back to zero for the slot's next launch: the
-            // last block here resets it.  Every block gets here, and only after
-            // its last claim has returned (the ticket's increment depends on it).
-            const unsigned long long t = atomicAdd(a.claim + 1, 1ull | (pending >> 63));
-            if (t == gridDim.x - 1) {
-                atomicExch(a.claim, 0ull);
-                atomicExch(a.claim + 1, 0ull);
-            }
-        }
-        return;
-    }
+    } else {
 
     // ---------------------------------------------------------------- consumers
     const uint32_t ct = threadIdx.x - 32;
@@ -1189,24 +1275,50 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
         for (uint32_t j = 0; j < kFanSlots; ++j)
             if (fan_bucket[j] != 0xFFFFFFFFu) flush(a.sums + fan_bucket[j], fan_acc[j]);
     }
-    if (MODE != 2) return;
-    // Checksum comparison by whichever block finishes last (consumer threads only).
-    consumers_sync<kCT>();
-    if (ct == 0) {
+    }   // consumers
+
+    // ------------------------------------------------------------- epilogue
+    // Every warp of the block is done: the producer's claims have returned and
+    // the consumers' sums are flushed.  The block that takes the last ticket
+    // finishes the launch: the verifying unpack compares the sums (and writes
+    // the result); a pack through a slot writes its checksums out of the
+    // slot's sums; a launch holding a slot leaves it zeroed.
+    if (MODE != 2 && !a.reset_claims) return;
+    __syncthreads();
+    if (threadIdx.x == 0) {
         __threadfence();
         last_block = atomicAdd(&a.counters[0], 1ull) == gridDim.x - 1;
     }
-    consumers_sync<kCT>();
+    __syncthreads();
     if (!last_block) return;
     __threadfence();
-    for (int32_t i = ct; i < a.n_buckets; i += kCT) {
-        const int32_t b = a.first_bucket + i;
-        const bool differs = __ldcg(a.sums + i) != a.expected[b];
-        if (a.bad) a.bad[i] = differs ? 1 : 0;
-        if (differs) {
-            atomicAdd(&a.counters[1], 1ull);
-            atomicMax(&a.counters[2], ULLONG_MAX - (unsigned long long)b);
+    constexpr uint32_t kBT = BulkShape<MODE>::kThreads;
+    if constexpr (MODE == 2) {
+        for (int32_t i = threadIdx.x; i < a.n_buckets; i += kBT) {
+            const int32_t b = a.first_bucket + i;
+            const unsigned long long got = __ldcg(a.sums + i);
+            const bool differs = got != a.expected[b];
+            if (a.bad) a.bad[i] = differs ? 1 : 0;
+            if (differs) {
+                atomicAdd(&a.counters[1], 1ull);
+                atomicMax(&a.counters[2], ULLONG_MAX - (unsigned long long)b);
+            }
+            if (a.reset_claims) a.sums[i] = 0;
         }
+        __syncthreads();
+        if (threadIdx.x == 0 && a.result) write_result(a.counters, a.result);
+    }
+    if constexpr (MODE == 0) {
+        if (a.sums_out)
+            for (int32_t i = threadIdx.x; i < a.n_buckets; i += kBT) {
+                const int32_t b = a.first_bucket + i;
+                a.sums_out[b] = __ldcg(a.sums + b);
+                a.sums[b] = 0;
+            }
+    }
+    if (a.reset_claims) {
+        __syncthreads();
+        if (threadIdx.x < 4) atomicExch(&a.counters[threadIdx.x], 0ull);
     }
 }
 
@@ -1392,7 +1504,7 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
 template <int NPTR>
 rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
                         const uint64_t* checksums, uint8_t* bad, bool table, uint64_t stride,
-                        cudaStream_t s) {
+                        cudaStream_t s, long long* result = nullptr) {
     UnpackArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     a.items = P->d_unpack_items;
@@ -1409,6 +1521,7 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
         a.bad = q.bad;
         a.first_bucket = R.b0;
         a.n_buckets = R.b1 - R.b0;
+        a.result = result;
     }
     int32_t k = 0;
     if (table) {
@@ -1432,7 +1545,8 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
     } else {
         lock.lock();
         if ((slot = take_claim_slot(M, s)) >= 0) {
-            a.claim = P->d_claims + 2 * slot;
+            a.counters = P->d_slots + size_t(slot) * P->slot_words() + P->n_buckets;
+            a.claim = a.counters + 3;
             a.reset_claims = 1;
             work_units<1>(P, R, &a.unit_first, &a.n_units);
         }
@@ -1550,14 +1664,45 @@ void work_units(const rr_plan* P, const Range& R, const uint32_t** first, uint32
     }
 }
 
+// How a bulk launch may use the plan's pooled slots, and what it zeroes itself.
+struct BulkOpts {
+    bool may_slot = true;                 // try a pooled slot (not for the blocking verifies)
+    unsigned long long* zero = nullptr;   // without a slot, zero these words first (pack:
+    size_t zero_words = 0;                //   the range's checksums; async verify: scratch)
+    long long* result = nullptr;          // verifying unpack: write {n_bad, first_bad} here
+};
+
+template <int NPTR, int MODE, bool CHECK>
+cudaError_t launch_bulk_kernel(int32_t grid, cudaStream_t s, const BulkArgs<NPTR>& a) {
+    cudaError_t e = bulk_prepare<NPTR, MODE, CHECK>();
+    if (e != cudaSuccess) return e;
+    // Programmatic dependent launch: this grid's blocks may be scheduled while
+    // the previous kernel on the stream drains (they wait for it to complete
+    // before touching memory), so the launch latency and prologue overlap it.
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(BulkShape<MODE>::kThreads);
+    cfg.dynamicSmemBytes = BulkShape<MODE>::kSmem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, rr_bulk_kernel<NPTR, MODE, CHECK>, a);
+}
+
 template <int NPTR, int MODE>
 rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
                       const void* const* buckets, void* const* dst, const uint64_t* checksums,
-                      uint8_t* bad, bool table, uint64_t stride, cudaStream_t s) {
+                      uint8_t* bad, bool table, uint64_t stride, cudaStream_t s,
+                      const BulkOpts& o = BulkOpts()) {
     BulkArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     a.err = P->d_error;
     a.chk = bounds_of(P);
+    a.first_bucket = R.b0;
+    a.n_buckets = R.b1 - R.b0;
     int32_t k = 0;
     if (MODE == 0) {
         a.items = P->d_pack_items;
@@ -1565,8 +1710,10 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         a.weight_prefix = P->d_pack_weight_prefix;
         a.item_begin = P->pack_bucket_first[R.b0];
         a.item_end = P->pack_bucket_first[R.b1];
+        a.n_items = uint32_t(P->pack_items.size());
         if (R.full && P->d_full_items) {   // every bucket: the table with fan-out groups
             a.items = P->d_full_items;
+            a.n_items = uint32_t(P->full_items.size());
             a.block_first = P->d_full_block_first;
             a.item_begin = 0;
             a.item_end = uint32_t(P->full_items.size());
@@ -1576,22 +1723,11 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         for (int32_t i = 0; i < P->n_shards; ++i) a.ptr[k++] = src_shards[i];
     } else {
         a.items = P->d_unpack_items;
+        a.n_items = uint32_t(P->unpack_items.size());
         a.block_first = R.full ? P->d_unpack_block_first : nullptr;
         a.weight_prefix = P->d_unpack_weight_prefix;
         a.item_begin = P->unpack_bucket_first[R.b0];
         a.item_end = P->unpack_bucket_first[R.b1];
-        if (MODE == 2) {
-            const SumSlot q = sum_slot(P, R, bad);
-            a.sums = q.sums;
-            a.counters = q.counters;
-            // The call's work units, claimed through counters[3].
-            work_units<MODE>(P, R, &a.block_first, &a.n_units);
-            a.claim = q.counters + 3;
-            a.expected = (const unsigned long long*)checksums;
-            a.bad = q.bad;
-            a.first_bucket = R.b0;
-            a.n_buckets = R.b1 - R.b0;
-        }
     }
     if (table) {   // the range's buckets (a full-range pack: all of them, for fan-out items)
         a.bucket_lo = R.b0;
@@ -1605,33 +1741,53 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         for (int32_t t = R.t_lo; t <= R.t_hi; ++t) a.ptr[k++] = dst[t];
     }
     const int32_t grid = MODE == 0 ? P->grid_blocks : P->unpack_grid_blocks;
-    // Pack and plain unpack claim their units through a pooled slot when one
-    // is free; otherwise they run the fixed split set above.
-    rr_plan* M = const_cast<rr_plan*>(P);   // the claim pool is mutable state
+    // A pooled slot when one is free: the launch claims its units through the
+    // slot's counter, and pack and the verifying unpack sum into the slot, so
+    // nothing needs zeroing first.  Otherwise pack and plain unpack run the
+    // fixed split set above, and the verifying unpack uses the call's scratch.
+    rr_plan* M = const_cast<rr_plan*>(P);   // the slot pool is mutable state
     std::unique_lock<std::mutex> lock(M->claim_mutex, std::defer_lock);
     int32_t slot = -1;
-    cudaError_t e = cudaSuccess;
-    if (MODE != 2) {
+    if (o.may_slot) {
         lock.lock();
-        if ((slot = take_claim_slot(M, s)) >= 0) {
-            a.claim = P->d_claims + 2 * slot;
-            a.reset_claims = 1;
+        slot = take_claim_slot(M, s);
+    }
+    if (slot >= 0) {
+        unsigned long long* area = P->d_slots + size_t(slot) * P->slot_words();
+        a.counters = area + P->n_buckets;
+        a.claim = a.counters + 3;
+        a.reset_claims = 1;
+        work_units<MODE>(P, R, &a.block_first, &a.n_units);
+        if (MODE == 0 && o.zero) {          // the checksums come out of the slot's sums
+            a.sums = area;
+            a.sums_out = (unsigned long long*)checksums;
+        }
+        if (MODE == 2) {
+            a.sums = area;                  // indexed from the range's first bucket
+            a.bad = bad;
+        }
+    } else {
+        if (o.zero) RR_CUDA(cudaMemsetAsync(o.zero, 0, o.zero_words * 8, s));
+        if (MODE == 2) {
+            const SumSlot q = sum_slot(P, R, bad);
+            a.sums = q.sums;
+            a.counters = q.counters;
+            a.claim = q.counters + 3;       // the call's work units, claimed through counters[3]
+            a.bad = q.bad;
             work_units<MODE>(P, R, &a.block_first, &a.n_units);
         }
     }
-    if (P->check_items) {
-        RR_CUDA((bulk_prepare<NPTR, MODE, true>()));
-        rr_bulk_kernel<NPTR, MODE, true>
-            <<<grid, BulkShape<MODE>::kThreads, BulkShape<MODE>::kSmem, s>>>(a);
-    } else {
-        RR_CUDA((bulk_prepare<NPTR, MODE, false>()));
-        rr_bulk_kernel<NPTR, MODE, false>
-            <<<grid, BulkShape<MODE>::kThreads, BulkShape<MODE>::kSmem, s>>>(a);
+    if (MODE == 2) {
+        a.expected = (const unsigned long long*)checksums;
+        a.result = o.result;
     }
-    RR_CUDA(cudaGetLastError());
-    if (slot >= 0 && (e = cudaEventRecord(P->claim_done[slot], s)) != cudaSuccess) {
+    const cudaError_t e = P->check_items ? launch_bulk_kernel<NPTR, MODE, true>(grid, s, a)
+                                         : launch_bulk_kernel<NPTR, MODE, false>(grid, s, a);
+    if (e != cudaSuccess) return cuda_fail(e, "bulk kernel launch");
+    cudaError_t er;
+    if (slot >= 0 && (er = cudaEventRecord(P->claim_done[slot], s)) != cudaSuccess) {
         M->claim_retired[slot] = 1;   // its launch's end is unknown: never hand it out again
-        return cuda_fail(e, "cudaEventRecord");
+        return cuda_fail(er, "cudaEventRecord");
     }
     return RR_OK;
 }
@@ -1680,11 +1836,21 @@ rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, vo
                        "%d source buffers leave no room for separately allocated buckets in one "
                        "launch's %d pointers; allocate the buckets as one equally spaced block",
                        P->n_shards, kLargePtrs);
-    RR_CUDA(cudaMemsetAsync(checksums + R.b0, 0, size_t(R.b1 - R.b0) * 8, stream));
-    if (P->pack_bucket_first[R.b0] == P->pack_bucket_first[R.b1]) return RR_OK;
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(src_shards, P->n_shards) &&
                       all_device((const void* const*)buckets, P->n_buckets);
     const int32_t step = table ? cap : R.b1 - R.b0;
+    const bool empty = P->pack_bucket_first[R.b0] == P->pack_bucket_first[R.b1];
+    // One bulk launch writes the range's checksums itself (out of a pooled
+    // slot's sums, or after zeroing them when no slot is free); otherwise they
+    // are zeroed here and every launch adds into them.
+    BulkOpts o;
+    if (bulk && !empty && step >= R.b1 - R.b0) {
+        o.zero = (unsigned long long*)checksums + R.b0;
+        o.zero_words = size_t(R.b1 - R.b0);
+    } else {
+        RR_CUDA(cudaMemsetAsync(checksums + R.b0, 0, size_t(R.b1 - R.b0) * 8, stream));
+    }
+    if (empty) return RR_OK;
     for (int32_t b = R.b0; b < R.b1; b += step) {
         const int32_t e = std::min(R.b1, b + step);
         const bool whole = R.full && b == R.b0 && e == R.b1;
@@ -1694,9 +1860,11 @@ rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, vo
         if (bulk)
             st = need <= kSmallPtrs
                      ? launch_bulk<kSmallPtrs, 0>(P, S, src_shards, (const void* const*)buckets,
-                                                  nullptr, checksums, nullptr, table, stride, stream)
+                                                  nullptr, checksums, nullptr, table, stride, stream,
+                                                  o)
                      : launch_bulk<kLargePtrs, 0>(P, S, src_shards, (const void* const*)buckets,
-                                                  nullptr, checksums, nullptr, table, stride, stream);
+                                                  nullptr, checksums, nullptr, table, stride, stream,
+                                                  o);
         else
             st = need <= kSmallPtrs
                      ? launch_pack<kSmallPtrs>(P, S, src_shards, buckets, checksums, table, stride,
@@ -1769,14 +1937,14 @@ rr_status unpack_shape(const rr_plan* P, Range R, const void* const* buckets, Un
 rr_status launch_unpack_part(const rr_plan* P, const Range& S, bool bulk,
                              const void* const* buckets, void* const* dst,
                              const uint64_t* checksums, uint8_t* bad, const UnpackShape& sh,
-                             cudaStream_t stream) {
+                             cudaStream_t stream, const BulkOpts& o = BulkOpts()) {
     const bool small = (S.t_hi - S.t_lo + 1) + (sh.table ? S.b1 - S.b0 : 0) <= kSmallPtrs;
     if (bulk) {
         if (checksums)
             return small ? launch_bulk<kSmallPtrs, 2>(P, S, nullptr, buckets, dst, checksums, bad,
-                                                      sh.table, sh.stride, stream)
+                                                      sh.table, sh.stride, stream, o)
                          : launch_bulk<kLargePtrs, 2>(P, S, nullptr, buckets, dst, checksums, bad,
-                                                      sh.table, sh.stride, stream);
+                                                      sh.table, sh.stride, stream, o);
         return small ? launch_bulk<kSmallPtrs, 1>(P, S, nullptr, buckets, dst, nullptr, nullptr,
                                                   sh.table, sh.stride, stream)
                      : launch_bulk<kLargePtrs, 1>(P, S, nullptr, buckets, dst, nullptr, nullptr,
@@ -1787,9 +1955,9 @@ rr_status launch_unpack_part(const rr_plan* P, const Range& S, bool bulk,
     Range Sr = S;
     Sr.full = S.full && P->engine == RR_ENGINE_REGISTERS;
     return small ? launch_unpack<kSmallPtrs>(P, Sr, buckets, dst, checksums, bad, sh.table,
-                                             sh.stride, stream)
+                                             sh.stride, stream, o.result)
                  : launch_unpack<kLargePtrs>(P, Sr, buckets, dst, checksums, bad, sh.table,
-                                             sh.stride, stream);
+                                             sh.stride, stream, o.result);
 }
 
 rr_status unpack_impl(const rr_plan* P, Range R, const void* const* buckets, void* const* dst,
@@ -1822,29 +1990,43 @@ rr_status read_result(const rr_plan* P, int32_t n, int64_t* n_bad, int64_t* firs
     return nb ? RR_EMISMATCH : RR_OK;
 }
 
-// Enqueues the verifying unpack of range R: zeroes the range's sums and
-// counters (R.scratch, else the plan's), then one fused launch per sub-range
-// (usually one).  Sub-launches share the call's counters; each compares its
-// own buckets, and the "last block" ticket and the unit claims are reset
-// between them.
+// Enqueues the verifying unpack of range R.  The stream-ordered form (R has
+// the caller's scratch) in one bulk launch sums into a pooled slot when one is
+// free, zeroing nothing first; otherwise the range's sums and counters
+// (R.scratch, else the plan's) are zeroed, then one fused launch per sub-range
+// (usually one) runs.  Sub-launches share the call's counters; each compares
+// its own buckets, and the "last block" ticket and the unit claims are reset
+// between them.  `result` (device address or NULL) receives {n_bad,
+// first_bad} from the last launch's last block.
 rr_status enqueue_unpack_verify(const rr_plan* P, Range R, const void* const* buckets,
                                 const uint64_t* checksums, void* const* dst, uint8_t* bad,
-                                cudaStream_t stream) {
+                                cudaStream_t stream, long long* result = nullptr) {
     const int32_t n = R.b1 - R.b0;
     unsigned long long* sc = R.scratch ? R.scratch : P->d_verify_scratch;
     UnpackShape sh;
     rr_status st = unpack_shape(P, R, buckets, &sh);
     if (st) return st;
-    RR_CUDA(cudaMemsetAsync(sc, 0, (size_t(n) + 4) * sizeof(unsigned long long), stream));
     const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(buckets, P->n_buckets) &&
                       all_device((const void* const*)dst, P->n_tensors);
+    if (bulk && R.scratch && sh.parts.size() == 1) {
+        BulkOpts o;
+        o.zero = sc;
+        o.zero_words = size_t(n) + 4;
+        o.result = result;
+        return launch_unpack_part(P, sh.parts[0], bulk, buckets, dst, checksums, bad, sh, stream,
+                                  o);
+    }
+    RR_CUDA(cudaMemsetAsync(sc, 0, (size_t(n) + 4) * sizeof(unsigned long long), stream));
     for (size_t i = 0; i < sh.parts.size(); ++i) {
         if (i > 0) {   // a fresh "last block" ticket and unit claims
             RR_CUDA(cudaMemsetAsync(sc + n, 0, sizeof(unsigned long long), stream));
             RR_CUDA(cudaMemsetAsync(sc + n + 3, 0, sizeof(unsigned long long), stream));
         }
+        BulkOpts o;
+        o.may_slot = false;
+        o.result = i + 1 == sh.parts.size() ? result : nullptr;
         if ((st = launch_unpack_part(P, sh.parts[i], bulk, buckets, dst, checksums, bad, sh,
-                                     stream)))
+                                     stream, o)))
             return st;
     }
     return RR_OK;
@@ -1988,10 +2170,10 @@ rr_status rr_device_upload(rr_plan* P) {
                 P->pack_unit_first.size() * sizeof(uint32_t))) != cudaSuccess ||
         (e = up((void**)&P->d_pack_whole_unit_first, P->pack_whole_unit_first.data(),
                 P->pack_whole_unit_first.size() * sizeof(uint32_t))) != cudaSuccess ||
-        (e = cudaMalloc((void**)&P->d_claims,
-                        2 * rr_plan::kClaimSlots * sizeof(unsigned long long))) != cudaSuccess ||
-        (e = cudaMemset(P->d_claims, 0, 2 * rr_plan::kClaimSlots * sizeof(unsigned long long))) !=
-            cudaSuccess ||
+        (e = cudaMalloc((void**)&P->d_slots, rr_plan::kClaimSlots * P->slot_words() *
+                                                 sizeof(unsigned long long))) != cudaSuccess ||
+        (e = cudaMemset(P->d_slots, 0, rr_plan::kClaimSlots * P->slot_words() *
+                                           sizeof(unsigned long long))) != cudaSuccess ||
         (e = cudaMalloc((void**)&P->d_verify_scratch,
                         (size_t(P->n_buckets) + 4) * sizeof(unsigned long long))) != cudaSuccess ||
         (e = cudaHostAlloc((void**)&P->h_verify_result, 5 * sizeof(unsigned long long),
@@ -2036,7 +2218,7 @@ void rr_device_release(rr_plan* P) {
     cudaFree(P->d_unpack_unit_first);
     cudaFree(P->d_pack_unit_first);
     cudaFree(P->d_pack_whole_unit_first);
-    cudaFree(P->d_claims);
+    cudaFree(P->d_slots);
     for (cudaEvent_t& ev : P->claim_done) {
         if (ev) cudaEventDestroy(ev);
         ev = nullptr;
@@ -2058,7 +2240,7 @@ void rr_device_release(rr_plan* P) {
     P->d_unpack_unit_first = nullptr;
     P->d_pack_unit_first = nullptr;
     P->d_pack_whole_unit_first = nullptr;
-    P->d_claims = nullptr;
+    P->d_slots = nullptr;
     P->d_verify_scratch = nullptr;
     P->h_verify_result = nullptr;
     if (prev >= 0 && prev != P->device) cudaSetDevice(prev);
@@ -2174,10 +2356,10 @@ extern "C" rr_status rr_unpack_verify_async(const rr_plan* P, int32_t first_buck
         if (!aligned16(scratch)) return rr_fail(RR_EINVAL, "scratch NULL or not 16-byte aligned");
         if (!device_resident(scratch)) return rr_fail(RR_EINVAL, "scratch must be device memory");
         R.scratch = (unsigned long long*)scratch;
-        if ((st = enqueue_unpack_verify(P, R, buckets, checksums, dst, bad, stream))) return st;
+        // The launch's last block writes the result.
+        return enqueue_unpack_verify(P, R, buckets, checksums, dst, bad, stream, res);
     }
-    rr_verify_result_kernel<<<1, 1, 0, stream>>>(R.b1 > R.b0 ? R.scratch + (R.b1 - R.b0) : nullptr,
-                                                 res);
+    rr_verify_result_kernel<<<1, 1, 0, stream>>>(nullptr, res);   // an empty range
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }

@@ -97,11 +97,14 @@ struct rr_plan {
     uint32_t* d_unpack_unit_first = nullptr;
     uint32_t* d_pack_unit_first = nullptr;
     uint32_t* d_pack_whole_unit_first = nullptr;
-    // Unit-claim counters of launches that have no per-call scratch (rr_pack,
-    // rr_unpack): a slot is handed to a launch only once the event recorded
-    // after its previous launch has completed; that launch left it zeroed.
+    // Pooled scratch of launches that need no per-call scratch: a slot is
+    // handed to a launch only once the event recorded after its previous
+    // launch has completed, and that launch's last block left it zeroed.  Slot
+    // k is slot_words() words at d_slots + k * slot_words(): per-bucket sums
+    // [n_buckets], then counters {ticket, n_bad, max(~0 - bad index), claim}.
     static constexpr int kClaimSlots = 16;
-    unsigned long long* d_claims = nullptr;      // kClaimSlots x {counter, ticket}
+    unsigned long long* d_slots = nullptr;
+    size_t slot_words() const { return size_t(n_buckets) + 4; }
     cudaEvent_t claim_done[kClaimSlots] = {};
     char claim_retired[kClaimSlots] = {};
     int32_t claim_next = 0;

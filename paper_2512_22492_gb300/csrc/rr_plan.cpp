@@ -49,6 +49,12 @@ constexpr int64_t kDefaultChunkBytes = 32 * 1024;
 #ifndef RR_TAPER_FLOOR
 #define RR_TAPER_FLOOR (64 * 1024)
 #endif
+#ifndef RR_FAN_HEAD_CHUNKS
+#define RR_FAN_HEAD_CHUNKS 16
+#endif
+#ifndef RR_FAN_END_PCT
+#define RR_FAN_END_PCT 80
+#endif
 constexpr int64_t kItemOverhead = RR_ITEM_OVERHEAD;   // balancing weight of one item, in bytes
 constexpr int64_t kZeroWeight = RR_ZERO_WEIGHT;       // weight of one zero-filled element
 constexpr int64_t kUnitWeight = 1 << 20;   // largest claimed work unit (weight), and the
@@ -212,8 +218,9 @@ public:
         const int32_t es = P->es[p];
         const int64_t C = P->cols[p], B = P->bucket_bytes;
         // Heads are cut into stage-sized pieces by the kernel; this only bounds
-        // the balancing granularity (16 chunks of source per head).
-        const int64_t max_rows = std::max<int64_t>(1, 16 * P->chunk_bytes / (span * es));
+        // the balancing granularity (RR_FAN_HEAD_CHUNKS chunks of source per head).
+        const int64_t max_rows =
+            std::max<int64_t>(1, RR_FAN_HEAD_CHUNKS * P->chunk_bytes / (span * es));
         int64_t i = 0;
         while (i < nrows) {
             const Loc at = loc(p, (row0 + i) * C + cmin);
@@ -829,17 +836,28 @@ void build_tables(rr_plan* P, const rr_dst_layout* dst) {
         for (const FanGroup& g : groups) b.fan_group(g.param, g.row0, g.nrows, g.cmin, g.span, g.slices);
         b.set_out(&P->pack_items);
         // Spread the fan-out heads (with their destinations, and the plain items
-        // of rows that fell back) evenly through the table, so that every block
-        // of the balanced split gets its share of them.
+        // of rows that fell back) evenly through the first part of the table,
+        // so that every block's own share gets its part of them and the heads
+        // are done by RR_FAN_END_PCT of the table's weight: a head cannot be
+        // split, and the claimed units at the end should all be small.
         std::vector<size_t> unit_start;   // fan items in runs: a head and its destinations
         for (size_t i = 0; i < fan.size(); ++i)
             if (fan[i].kind != RR_ITEM_FAN_DST) unit_start.push_back(i);
         unit_start.push_back(fan.size());
         const size_t U = unit_start.size() - 1;
+        int64_t w_kept = 0, w_fan = 0;
+        for (const rr_pack_item& it : kept) w_kept += pack_weight(it);
+        for (const rr_pack_item& it : fan) w_fan += pack_weight(it);
+        // The plain items the heads are spread over: the first `span_kept` of them.
+        const int64_t room = (w_kept + w_fan) * RR_FAN_END_PCT / 100 - w_fan;
+        const size_t span_kept =
+            w_kept <= 0 || room <= 0
+                ? 0
+                : std::min(kept.size(), size_t(double(kept.size()) * double(room) / double(w_kept)));
         P->full_items.reserve(kept.size() + fan.size());
         size_t k = 0;
         for (size_t u = 0; u < U; ++u) {
-            const size_t upto = kept.size() * u / U;
+            const size_t upto = span_kept * u / U;
             for (; k < upto; ++k) P->full_items.push_back(kept[k]);
             for (size_t i = unit_start[u]; i < unit_start[u + 1]; ++i)
                 P->full_items.push_back(fan[i]);
