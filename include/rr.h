@@ -181,7 +181,7 @@ typedef struct {
     int32_t host_only;   /* 1: build the tables on the host only and touch no GPU; such
                             a plan can be queried and exported but not executed       */
     int32_t grid_blocks; /* persistent grid size; default: SMs x resident blocks      */
-    int64_t chunk_bytes; /* largest destination bytes per work item; default 32 KiB   */
+    int64_t chunk_bytes; /* largest destination bytes per work item; default 64 KiB   */
     int32_t engine;      /* rr_engine                                                 */
     int32_t check_items; /* 1: every kernel checks each work item against the source,
                             bucket and tensor sizes of the plan before touching
@@ -456,11 +456,14 @@ rr_status rr_plan_bucket_items(const rr_plan* plan, uint32_t* pack_first, uint32
  * a bucket_unit array with RR_UNITS_PACK_FULL; nothing is written then.
  * Which launches claim: every verifying unpack (either engine), its counter
  * kept in the call's scratch (the plan's for the blocking forms, the
- * caller's for rr_unpack_verify_async); rr_unpack (either engine) and rr_pack
- * (bulk-copy engine) when one of the plan's 16 counter slots is free -- a
- * slot is reused only after the launch that last held it has completed --
- * and the stream is not capturing a graph.  Otherwise the launch splits its
- * items evenly over the grid, as a captured launch always does, and the
+ * caller's for rr_unpack_verify_async) or in a pooled slot; rr_unpack (either
+ * engine) and rr_pack (bulk-copy engine) when they get one of the plan's 16
+ * pooled slots.  A slot is free once the launch that last held it has
+ * completed; when none is, a launch takes the slot handed out longest ago if
+ * that slot's launch ran on the same stream, and the stream waits on the GPU
+ * for that launch (which it would anyway).  A launch gets no slot when every
+ * slot is held by another stream's launch still in flight, or when its stream
+ * is capturing a graph; it then splits its items evenly over the grid, as the
  * register path's pack always does.  Which of these runs changes no output
  * byte. */
 enum { RR_UNITS_PACK = 0, RR_UNITS_PACK_FULL = 1, RR_UNITS_UNPACK = 2 };

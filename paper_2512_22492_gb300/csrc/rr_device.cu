@@ -1615,11 +1615,14 @@ bool all_device(const void* const* ptrs, int32_t n) {
     return n == 0 || (device_resident(ptrs[0]) && device_resident(ptrs[n - 1]));
 }
 
-// A unit-claim slot for a launch on `s` that has no per-call scratch, or -1:
-// every slot's last launch still running, or `s` capturing a graph (a captured
-// launch replays whenever the graph does, so it keeps the fixed split).  The
-// caller holds claim_mutex and records claim_done[slot] after the launch.  A
-// slot is {counter, ticket}, zero when handed out: zeroed once at plan
+// A pooled slot for a launch on `s`, or -1.  A slot whose last launch has
+// completed is free.  When none is, the slot handed out longest ago is taken
+// if its last launch ran on `s` itself: `s` then waits (on the GPU) for that
+// launch's event, which costs nothing since the stream runs its work in order
+// anyway.  Otherwise (every slot held by another stream's launch in flight, or
+// `s` capturing a graph -- a captured launch replays whenever the graph does)
+// there is none.  The caller holds claim_mutex and records claim_done[slot]
+// after the launch.  A slot is all zero when handed out: zeroed once at plan
 // creation, then by the last block of each launch that held it.
 int32_t take_claim_slot(rr_plan* M, cudaStream_t s) {
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
@@ -1642,8 +1645,19 @@ int32_t take_claim_slot(rr_plan* M, cudaStream_t s) {
         else if (q != cudaErrorNotReady)
             cudaGetLastError();
     }
+    for (int32_t i = 0; i < rr_plan::kClaimSlots && slot < 0; ++i) {
+        const int32_t k = (M->claim_next + i) % rr_plan::kClaimSlots;
+        if (M->claim_retired[k] || M->claim_stream[k] != s) continue;
+        if (cudaStreamWaitEvent(s, M->claim_done[k], 0) == cudaSuccess)
+            slot = k;
+        else
+            cudaGetLastError();
+    }
     cudaThreadExchangeStreamCaptureMode(&mode);
-    if (slot >= 0) M->claim_next = (slot + 1) % rr_plan::kClaimSlots;
+    if (slot >= 0) {
+        M->claim_next = (slot + 1) % rr_plan::kClaimSlots;
+        M->claim_stream[slot] = s;
+    }
     return slot;
 }
 

@@ -106,6 +106,7 @@ struct rr_plan {
     unsigned long long* d_slots = nullptr;
     size_t slot_words() const { return size_t(n_buckets) + 4; }
     cudaEvent_t claim_done[kClaimSlots] = {};
+    cudaStream_t claim_stream[kClaimSlots] = {};   // the stream of the slot's last launch
     char claim_retired[kClaimSlots] = {};
     int32_t claim_next = 0;
     std::mutex claim_mutex;

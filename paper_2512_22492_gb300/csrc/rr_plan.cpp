@@ -32,7 +32,7 @@ namespace {
 
 thread_local std::string g_error;
 
-constexpr int64_t kDefaultChunkBytes = 32 * 1024;
+constexpr int64_t kDefaultChunkBytes = 64 * 1024;
 // Balancing weights (build-time overridable for tuning sweeps).
 #ifndef RR_ITEM_OVERHEAD
 #define RR_ITEM_OVERHEAD 1024
@@ -50,7 +50,7 @@ constexpr int64_t kDefaultChunkBytes = 32 * 1024;
 #define RR_TAPER_FLOOR (64 * 1024)
 #endif
 #ifndef RR_FAN_HEAD_CHUNKS
-#define RR_FAN_HEAD_CHUNKS 16
+#define RR_FAN_HEAD_CHUNKS 32
 #endif
 #ifndef RR_FAN_END_PCT
 #define RR_FAN_END_PCT 80

@@ -1,13 +1,17 @@
 """Work units claimed at run time by the bulk-copy engine's blocks.
 
-rr_pack and rr_unpack take a claim counter from a pool of 16 per plan; a slot
-is handed out again only after the launch that last held it has completed,
-and a launch that finds none free, or that is being captured into a CUDA
-graph, splits its items evenly over the grid instead.  These tests drive
-every one of those paths and compare bytes with the oracle:
-  - more launches in flight than slots (the stream held back by a bounded
-    sleep kernel, so that none of them can complete before the rest are
-    enqueued);
+rr_pack and rr_unpack take a slot (a claim counter, and for pack its sums)
+from a pool of 16 per plan.  A slot is free once the launch that last held
+it has completed.  When none is, a launch takes the slot handed out longest
+ago if that slot's launch ran on its own stream, and waits on the GPU for it.
+A launch finds no slot when every slot is held by another stream's launch
+still in flight, or when it is being captured into a CUDA graph.  It then
+zeroes its checksums first and splits its items evenly over the grid.  These
+tests drive every one of those paths and compare bytes with the oracle:
+  - more launches in flight on one stream than slots (the stream held back by
+    a bounded sleep kernel, so that none of them can complete before the rest
+    are enqueued), and meanwhile a second stream's launches, which find every
+    slot held;
   - two streams packing and unpacking their own buffers at once;
   - the whole step captured into a CUDA graph and replayed on new inputs;
   - a resumed pull's range calls (clear, pack, unpack, stream-ordered check)
@@ -63,14 +67,19 @@ def test_more_launches_in_flight_than_claim_slots():
     first = H.alloc(plan)
     H.fill_from_host(first, shards)
     bufs = [H.alloc(plan, flat=first.flat) for _ in range(24)]
+    side = [H.alloc(plan, flat=first.flat) for _ in range(2)]
+    other = torch.cuda.Stream()
     torch.cuda.synchronize()
     torch.cuda._sleep(SLEEP_CYCLES)            # nothing below can complete until it ends
-    for b in bufs:
+    for b in bufs:                             # past 16, each waits for the oldest slot
         rr.rr_pack(plan, b.shards, b.buckets, b.checksums)
     for b in bufs:
         rr.rr_unpack(plan, b.buckets, b.dst)
+    for b in side:                             # every slot held by the first stream: none
+        rr.rr_pack(plan, b.shards, b.buckets, b.checksums, stream=other)
+        rr.rr_unpack(plan, b.buckets, b.dst, stream=other)
     torch.cuda.synchronize()
-    for b in bufs:
+    for b in bufs + side:
         check(plan, b, want, want_cs, want_t)
     # The pool is whole again: later launches claim as usual.
     for b in bufs[:3]:
