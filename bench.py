@@ -955,7 +955,9 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                                        "method": "torch copy_ of 4 GiB on the device, "
                                                  "read + write bytes"}},
         "clocks": clocks,
-        "gpu_launches": (2 if args.sync_verify else 3) * args.steps,
+        # Per step: the pack kernel and the verifying unpack kernel, which
+        # writes its own result (bench launches hold a pooled slot each).
+        "gpu_launches": 2 * args.steps,
         "e2e": e2e,
     }
     if snapshot:
