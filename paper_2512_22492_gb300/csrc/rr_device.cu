@@ -178,6 +178,11 @@ __device__ __forceinline__ void st_stream(void* p, uint4 v) {
 #endif
 }
 
+// 8-byte store of data written exactly once.
+__device__ __forceinline__ void st_stream8(void* p, uint32_t x, uint32_t y) {
+    asm volatile("st.global.v2.u32 [%0], {%1, %2};" ::"l"(p), "r"(x), "r"(y) : "memory");
+}
+
 // float32 bits -> value whose upper half is the bfloat16 result: round to
 // nearest even by adding 0x7FFF plus the lowest kept bit; a NaN instead
 // keeps its upper half with the quiet bit set (no rounding, so it can never
@@ -363,6 +368,50 @@ __device__ __forceinline__ unsigned long long pack_vec(const char* src, char* ds
     return acc;
 }
 
+// fp32 vector item with its source in host memory: vectors of 4 elements, one
+// 16-byte load and one 8-byte store each, so that a warp's load instruction
+// covers 512 contiguous source bytes.  Over NVLink-C2C a load instruction that
+// uses half of every 32-byte sector it touches (the two 16-byte halves of an
+// 8-element vector, loaded by two instructions) moves each sector twice: with
+// 8-element vectors the pack read pinned host memory at half the link's rate.
+// The destination is 16-byte aligned, so each store is one whole checksum word.
+__device__ __forceinline__ unsigned long long pack_vec_f32_narrow(const char* src, char* dst,
+                                                                  const rr_pack_item& d) {
+    constexpr int U = 2 * kUnroll;
+    const uint32_t vpr = d.row_len >> 2;
+    const uint32_t nvec = vpr * d.n_rows;
+    const uint64_t stride = (uint64_t)d.src_stride * 4;
+    const uint32_t dq = kThreads / vpr, dr = kThreads - dq * vpr;
+    uint32_t v = threadIdx.x;
+    uint32_t r = v / vpr, c = v - r * vpr;
+    unsigned long long acc = 0;
+    while (v < nvec) {
+        uint4 x[U];
+        uint32_t vv[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            vv[u] = v;
+            if (v < nvec) x[u] = ld_stream(src + r * stride + (uint64_t)c * 16);
+            v += kThreads;
+            c += dr;
+            r += dq;
+            if (c >= vpr) {
+                c -= vpr;
+                ++r;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (vv[u] < nvec) {
+                const uint32_t lo = cast2(x[u].x, x[u].y), hi = cast2(x[u].z, x[u].w);
+                st_stream8(dst + (uint64_t)vv[u] * 8, lo, hi);
+                acc += (unsigned long long)hi << 32 | lo;
+            }
+        }
+    }
+    return acc;
+}
+
 // Scalar item: any alignment and row length; one element per thread-step.
 // Each element's checksum contribution is its bits shifted to its byte
 // position within the 64-bit word it lands in.
@@ -395,7 +444,8 @@ __device__ __forceinline__ unsigned long long pack_scalar(const char* src, char*
     return acc;
 }
 
-template <int NPTR, bool CHECK>
+// HOST_SRC: the source is in host memory (fp32 vectors of 4 elements).
+template <int NPTR, bool CHECK, bool HOST_SRC>
 __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(const __grid_constant__ PackArgs<NPTR> a) {
     uint32_t i0, i1;
     block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
@@ -416,7 +466,9 @@ __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(c
         char* dst = bucket_of(a, d.bucket) + d.dst_off;
         const char* src = (const char*)a.ptr[d.src >> 48] + (d.src & 0xFFFFFFFFFFFFull);
         switch (d.kind) {
-            case RR_ITEM_F32_VEC: acc += pack_vec<4>(src, dst, d); break;
+            case RR_ITEM_F32_VEC:
+                acc += HOST_SRC ? pack_vec_f32_narrow(src, dst, d) : pack_vec<4>(src, dst, d);
+                break;
             case RR_ITEM_BF16_VEC: acc += pack_vec<2>(src, dst, d); break;
             case RR_ITEM_F32_SCALAR: acc += pack_scalar<4>(src, dst, d); break;
             case RR_ITEM_BF16_SCALAR: acc += pack_scalar<2>(src, dst, d); break;
@@ -1473,7 +1525,8 @@ void work_units(const rr_plan* P, const Range& R, const uint32_t** first, uint32
 
 template <int NPTR>
 rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* const* buckets,
-                      uint64_t* checksums, bool table, uint64_t stride, cudaStream_t s) {
+                      uint64_t* checksums, bool table, uint64_t stride, bool host_src,
+                      cudaStream_t s) {
     PackArgs<NPTR> a;
     std::memset(&a, 0, sizeof a);
     a.items = P->d_pack_items;
@@ -1492,10 +1545,15 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
         a.bucket_base = (char*)buckets[0];
         a.bucket_stride = stride;
     }
-    if (P->check_items)
-        rr_pack_kernel<NPTR, true><<<P->reg_pack_grid, kThreads, 0, s>>>(a);
+    const int g = P->reg_pack_grid;
+    if (P->check_items && host_src)
+        rr_pack_kernel<NPTR, true, true><<<g, kThreads, 0, s>>>(a);
+    else if (P->check_items)
+        rr_pack_kernel<NPTR, true, false><<<g, kThreads, 0, s>>>(a);
+    else if (host_src)
+        rr_pack_kernel<NPTR, false, true><<<g, kThreads, 0, s>>>(a);
     else
-        rr_pack_kernel<NPTR, false><<<P->reg_pack_grid, kThreads, 0, s>>>(a);
+        rr_pack_kernel<NPTR, false, false><<<g, kThreads, 0, s>>>(a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -1850,7 +1908,8 @@ rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, vo
                        "%d source buffers leave no room for separately allocated buckets in one "
                        "launch's %d pointers; allocate the buckets as one equally spaced block",
                        P->n_shards, kLargePtrs);
-    const bool bulk = P->engine == RR_ENGINE_AUTO && all_device(src_shards, P->n_shards) &&
+    const bool src_device = all_device(src_shards, P->n_shards);
+    const bool bulk = P->engine == RR_ENGINE_AUTO && src_device &&
                       all_device((const void* const*)buckets, P->n_buckets);
     const int32_t step = table ? cap : R.b1 - R.b0;
     const bool empty = P->pack_bucket_first[R.b0] == P->pack_bucket_first[R.b1];
@@ -1882,9 +1941,9 @@ rr_status pack_impl(const rr_plan* P, Range R, const void* const* src_shards, vo
         else
             st = need <= kSmallPtrs
                      ? launch_pack<kSmallPtrs>(P, S, src_shards, buckets, checksums, table, stride,
-                                               stream)
+                                               !src_device, stream)
                      : launch_pack<kLargePtrs>(P, S, src_shards, buckets, checksums, table, stride,
-                                               stream);
+                                               !src_device, stream);
         if (st) return st;
     }
     return RR_OK;
@@ -2136,7 +2195,7 @@ rr_status rr_device_default_grid(rr_grids* g) {
     int dev = 0, sms = 0, p = 0, u = 0, v = 0, b = 0;
     RR_CUDA(cudaGetDevice(&dev));
     RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs, false>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs, false, false>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, true, false>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, rr_verify_kernel<kLargePtrs>, kThreads, 0));
     int bp = 0;
