@@ -50,7 +50,17 @@ namespace {
 #ifndef RR_ST_HINT
 #define RR_ST_HINT 0
 #endif
-constexpr int kThreads = RR_THREADS;   // threads per block, all three kernels
+// The verifying register-path unpack has a shape of its own (measured on GB300:
+// with 256-thread blocks it ran Qwen3-0.6B at 0.78 of the copy ceiling, with
+// 128-thread blocks and 16 vectors in flight per thread at 0.99; the plain
+// unpack and the pack run best at 256).
+#ifndef RR_VUNPACK_THREADS
+#define RR_VUNPACK_THREADS 128
+#endif
+#ifndef RR_VUNPACK_VECS
+#define RR_VUNPACK_VECS 16
+#endif
+constexpr int kThreads = RR_THREADS;   // threads per block: pack, plain unpack, verify
 constexpr int kUnroll = RR_UNROLL;     // 16-byte vectors in flight per thread
 constexpr int kSmallPtrs = 64;      // pointer-table sizes of the two launch shapes
 constexpr int kLargePtrs = 3968;    // keeps the kernel parameters under 32 KB
@@ -511,7 +521,7 @@ __device__ void compare_in_last_block(unsigned long long* counters,
     __syncthreads();
     if (!last) return;
     __threadfence();
-    for (int32_t i = threadIdx.x; i < n; i += kThreads) {
+    for (int32_t i = threadIdx.x; i < n; i += blockDim.x) {
         const int32_t b = first + i;
         const bool differs = __ldcg(sums + i) != expected[b];
         if (bad) bad[i] = differs ? 1 : 0;
@@ -530,12 +540,21 @@ __device__ void compare_in_last_block(unsigned long long* counters,
 // Unpack
 // ---------------------------------------------------------------------------
 
+// Launch shape of rr_unpack_kernel: threads per block and 16-byte vectors in
+// flight per thread (plain: twice the pack's depth, one load per vector).
+template <bool VERIFY>
+struct RegUnpackShape {
+    static constexpr int kBlock = VERIFY ? RR_VUNPACK_THREADS : kThreads;
+    static constexpr int kVecs = VERIFY ? RR_VUNPACK_VECS : 2 * kUnroll;
+};
+
 // Copies each item's bytes from its bucket to its tensor.  With VERIFY it also
 // sums every bucket byte it reads (the gap READ items too) into the bucket's
 // checksum and compares at the end, so the buckets are read once for both.
 template <int NPTR, bool VERIFY, bool CHECK>
-__global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
-    constexpr int U = 2 * kUnroll;   // one 16-byte load per vector: twice the pack's depth
+__global__ void __launch_bounds__(RegUnpackShape<VERIFY>::kBlock, 4) rr_unpack_kernel(const __grid_constant__ UnpackArgs<NPTR> a) {
+    constexpr int T = RegUnpackShape<VERIFY>::kBlock;
+    constexpr int U = RegUnpackShape<VERIFY>::kVecs;
     __shared__ uint32_t next_unit[2];   // the claimed unit, double-buffered by parity
     uint32_t i0 = 0, i1 = 0;
     uint32_t walked = 0;              // units this block has walked
@@ -572,21 +591,21 @@ __global__ void __launch_bounds__(kThreads, 4) rr_unpack_kernel(const __grid_con
             char* dst = copy ? (char*)a.ptr[a.dst_base + d.tensor] + d.dst_off : nullptr;
             if (d.kind == RR_ITEM_COPY_VEC || d.kind == RR_ITEM_READ_VEC) {
                 const uint32_t nvec = d.nbytes >> 4;
-                for (uint32_t v = threadIdx.x; v < nvec; v += kThreads * U) {
+                for (uint32_t v = threadIdx.x; v < nvec; v += T * U) {
                     uint4 x[U];
 #pragma unroll
                     for (int u = 0; u < U; ++u)
-                        if (v + u * kThreads < nvec) x[u] = ld_stream(src + 16ull * (v + u * kThreads));
+                        if (v + u * T < nvec) x[u] = ld_stream(src + 16ull * (v + u * T));
 #pragma unroll
                     for (int u = 0; u < U; ++u) {
-                        if (v + u * kThreads < nvec) {
-                            if (copy) st_stream(dst + 16ull * (v + u * kThreads), x[u]);
+                        if (v + u * T < nvec) {
+                            if (copy) st_stream(dst + 16ull * (v + u * T), x[u]);
                             if (VERIFY) acc += words(x[u]);
                         }
                     }
                 }
             } else {
-                for (uint32_t e = threadIdx.x; e < (d.nbytes >> 1); e += kThreads) {
+                for (uint32_t e = threadIdx.x; e < (d.nbytes >> 1); e += T) {
                     const uint16_t h = *(const uint16_t*)(src + 2ull * e);
                     if (copy) *(uint16_t*)(dst + 2ull * e) = h;
                     if (VERIFY) acc += (unsigned long long)h << (8 * ((d.src_off + 2 * e) & 7));
@@ -1609,10 +1628,11 @@ rr_status launch_unpack(const rr_plan* P, Range R, const void* const* buckets, v
             work_units<1>(P, R, &a.unit_first, &a.n_units);
         }
     }
+    constexpr int VT = RegUnpackShape<true>::kBlock;
     if (checksums && P->check_items)
-        rr_unpack_kernel<NPTR, true, true><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
+        rr_unpack_kernel<NPTR, true, true><<<P->reg_vunpack_grid, VT, 0, s>>>(a);
     else if (checksums)
-        rr_unpack_kernel<NPTR, true, false><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
+        rr_unpack_kernel<NPTR, true, false><<<P->reg_vunpack_grid, VT, 0, s>>>(a);
     else if (P->check_items)
         rr_unpack_kernel<NPTR, false, true><<<P->reg_unpack_grid, kThreads, 0, s>>>(a);
     else
@@ -2192,11 +2212,13 @@ rr_status verify_impl(const rr_plan* P, Range R, const void* const* buckets,
 // ---------------------------------------------------------------------------
 
 rr_status rr_device_default_grid(rr_grids* g) {
-    int dev = 0, sms = 0, p = 0, u = 0, v = 0, b = 0;
+    int dev = 0, sms = 0, p = 0, u = 0, vu = 0, v = 0, b = 0;
     RR_CUDA(cudaGetDevice(&dev));
     RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs, false, false>, kThreads, 0));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, true, false>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, false, false>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &vu, rr_unpack_kernel<kLargePtrs, true, false>, RegUnpackShape<true>::kBlock, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, rr_verify_kernel<kLargePtrs>, kThreads, 0));
     int bp = 0;
     RR_CUDA((bulk_prepare<kLargePtrs, 0>()));
@@ -2209,6 +2231,7 @@ rr_status rr_device_default_grid(rr_grids* g) {
                                                           BulkShape<2>::kSmem));
     g->reg_pack = sms * (p > 0 ? p : 1);
     g->reg_unpack = sms * (u > 0 ? u : 1);
+    g->reg_vunpack = sms * (vu > 0 ? vu : 1);
     g->verify = sms * (v > 0 ? v : 1);
     g->bulk_pack = sms * (bp > 0 ? bp : 1);
     g->bulk_unpack = sms * (b > 0 ? b : 1);

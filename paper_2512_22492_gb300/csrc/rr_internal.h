@@ -54,6 +54,7 @@ struct rr_plan {
     int32_t verify_grid_blocks = 0;
     int32_t reg_pack_grid = 0;        // register-path grids when the bulk engine is the default
     int32_t reg_unpack_grid = 0;
+    int32_t reg_vunpack_grid = 0;     // the register path's verifying unpack (its own block size)
     int32_t engine = RR_ENGINE_AUTO;
     int64_t chunk_bytes = 0;
     bool host_only = false;
@@ -122,7 +123,7 @@ void rr_clear_error();
 
 // Device side (rr_device.cu).
 struct rr_grids {
-    int32_t bulk_pack, bulk_unpack, reg_pack, reg_unpack, verify;
+    int32_t bulk_pack, bulk_unpack, reg_pack, reg_unpack, verify, reg_vunpack;
 };
 rr_status rr_device_default_grid(rr_grids* g);
 rr_status rr_device_upload(rr_plan* p);

@@ -937,17 +937,18 @@ rr_status rr_plan_create_ex(const rr_param* manifest, int32_t n_params,
             P->engine = opts ? opts->engine : RR_ENGINE_AUTO;
             if (P->engine != RR_ENGINE_AUTO && P->engine != RR_ENGINE_REGISTERS)
                 st = rr_fail(RR_EINVAL, "unknown engine %d", P->engine);
-            rr_grids g{152 * 2, 152 * 2, 152 * 2, 152 * 4, 152 * 4};
+            rr_grids g{152 * 2, 152 * 2, 152 * 2, 152 * 4, 152 * 4, 152 * 4};
             if (st == RR_OK && !P->host_only) st = rr_device_default_grid(&g);
             const bool bulk = P->engine == RR_ENGINE_AUTO;
             P->grid_blocks = bulk ? g.bulk_pack : g.reg_pack;
             P->unpack_grid_blocks = bulk ? g.bulk_unpack : g.reg_unpack;
             P->reg_pack_grid = g.reg_pack;
             P->reg_unpack_grid = g.reg_unpack;
+            P->reg_vunpack_grid = g.reg_vunpack;
             P->verify_grid_blocks = g.verify;
             if (opts && opts->grid_blocks > 0)
                 P->grid_blocks = P->unpack_grid_blocks = P->verify_grid_blocks = P->reg_pack_grid =
-                    P->reg_unpack_grid = opts->grid_blocks;
+                    P->reg_unpack_grid = P->reg_vunpack_grid = opts->grid_blocks;
         }
         if (st == RR_OK) {
             build_tables(P, dst);
