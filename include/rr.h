@@ -44,7 +44,10 @@
  *
  * Memory.  Every pointer argument named "device" is CUDA device memory of
  * the device the plan was created on, owned by the caller; every device
- * pointer must be 16-byte aligned.  The plan owns its device segment tables,
+ * pointer must be 16-byte aligned.  Where a call says so, a buffer may
+ * instead be host memory this GPU reads (pinned, or any host memory on a
+ * device with pageable memory access, as on Grace); memory it cannot reach
+ * is refused with RR_EINVAL before anything is launched.  The plan owns its device segment tables,
  * a small verify scratch area and 16 work-unit counters (rr_plan_work_units);
  * rr_pack and rr_unpack allocate nothing.
  *
@@ -338,20 +341,30 @@ rr_status rr_plan_export_unpack(const rr_plan* plan, rr_unpack_item* items, int6
 /* Reshard + cast + pack + checksum, fused in one persistent kernel launch
  * (Section 5.2.1 steps 1-2: the resharded model fills a transfer buffer; the
  * checksums serve the reconnect cases of Section 5.2.2).
- *   src_shards: host array of n_shards device pointers, S bytes each.
- *   buckets:    host array of n_buckets device pointers, bucket_bytes each;
- *               equally spaced pointers (one allocation cut into buckets)
- *               lift the limit on how many buckets a launch can address.
+ *   src_shards: host array of n_shards pointers, S bytes each: device
+ *               memory, or host memory this GPU reads (pinned; any host
+ *               memory where the device has pageable memory access).  A
+ *               host-memory source is read by the pack's own loads over the
+ *               host link, with nothing copied to the device first; its fp32
+ *               vectors are 4 elements wide, so that every warp load uses
+ *               whole 32-byte sectors of host memory.
+ *   buckets:    host array of n_buckets pointers, bucket_bytes each (device
+ *               memory, or host memory as above: a snapshot); equally spaced
+ *               pointers (one allocation cut into buckets) lift the limit on
+ *               how many buckets a launch can address.
  *   checksums:  device array of n_buckets uint64, overwritten.
- * Stream-ordered and asynchronous: returns after enqueueing a memset of the
- * checksums and one kernel on `stream`. */
+ * Any host-memory array runs the call on the register path.  Stream-ordered
+ * and asynchronous: returns after enqueueing one kernel on `stream`, preceded
+ * by a memset of the checksums unless the launch holds a pooled work-unit
+ * slot (the bulk-copy engine outside graph capture). */
 rr_status rr_pack(const rr_plan* plan, const void* const* src_shards, void* const* buckets,
                   uint64_t* checksums, cudaStream_t stream);
 
 /* Buckets -> rollout tensors (Section 5.2.1: the receiving rollout completes
  * its weight update from what it pulled).
- *   buckets: host array of n_buckets device pointers;
- *   dst:     host array of n_tensors device pointers, numel * 2 bytes each.
+ *   buckets: host array of n_buckets pointers (device memory, or host memory
+ *            this GPU reads: restoring a snapshot);
+ *   dst:     host array of n_tensors pointers, numel * 2 bytes each.
  * Stream-ordered and asynchronous (one kernel launch). */
 rr_status rr_unpack(const rr_plan* plan, const void* const* buckets, void* const* dst,
                     cudaStream_t stream);
