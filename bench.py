@@ -376,6 +376,32 @@ def cpu_baseline(w, bucket_bytes, n_buckets_sample):
                       f"{dt:.2f} s; 1 of {os.cpu_count()} host cores ({cpu_model()})"}
 
 
+def workload_config(w, bucket_bytes: int, n_buckets: int, pack_read: int, dst_bytes: int,
+                    world: int) -> dict:
+    """The JSON line's `config`: the workload alone, the same on both arms.
+    Its byte counts are the step's algorithmic bytes: pack reads `pack_read`
+    source bytes and writes every bucket byte; the receiver reads every bucket
+    byte and writes `dst_bytes` of tensors."""
+    buckets = n_buckets * bucket_bytes
+    step_bytes = pack_read + 2 * buckets + dst_bytes
+    resident = pack_read + buckets + dst_bytes
+    return {"workload": w.name, "src_dtype": w.src_dtype, "n_shards": w.n_shards,
+            "sharding": w.sharding, "expert_parallel": w.ep, "tp": w.tp,
+            "bucket_bytes": bucket_bytes, "n_buckets": n_buckets, "step_bytes": step_bytes,
+            "l2": ("inputs > L2 (no flush needed)" if resident >= 4 * L2_BYTES else
+                   "L2 flushed between steps (512 MiB write outside the step's events)"),
+            "parallelism": f"replicas{world}"}
+
+
+def oracle_config(L, w, bucket_bytes: int, world: int) -> dict:
+    """workload_config from the oracle's own layout: every destination element
+    reads one source element of its parameter's width and writes 2 bytes."""
+    pack_read = sum(nr * nc * L.params[p][2]
+                    for _, _, blocks in L.tensors for p, _, nr, _, nc in blocks)
+    dst_bytes = 2 * int(sum(L.tensor_numel[:len(L.tensors)]))
+    return workload_config(w, bucket_bytes, int(L.n_buckets), int(pack_read), dst_bytes, world)
+
+
 def path_dtype(w) -> str:
     """What the path computes: an fp32 source is rounded to bf16 (nearest,
     ties to even, in integer arithmetic); a bf16 source is copied bit for bit."""
@@ -400,8 +426,9 @@ def run_reference(args, w, bucket_bytes, world, rank):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(t_total / args.steps * 1e3, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": path_dtype(w), "data": "synthetic",
-        "config": {"workload": w.name, "bucket_bytes": bucket_bytes,
-                   "step": f"oracle sync of bucket 0 of {L.n_buckets} (bounded sample)"},
+        "config": oracle_config(L, w, bucket_bytes, args.gpus),
+        "path": {"step": f"oracle sync of bucket 0 of {L.n_buckets} per step (a bounded "
+                         f"sample of the workload)"},
         "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"bucket 0 of {L.n_buckets} ({bucket_bytes >> 20} MiB): "
                                    "pack, unpack of its elements, verify per step"},
@@ -827,10 +854,11 @@ def run_native(args, w, bucket_bytes, world, rank, local):
     # Inputs smaller than a few L2 sizes would be served from L2 on the next
     # step: flush it between steps (a 512 MiB write outside the step's events)
     # and take the step time from those events.
-    resident = buf.flat.numel() + plan.n_buckets * plan.bucket_bytes + sum(
-        2 * n for n in plan.tensor_numel)
+    config = workload_config(w, bucket_bytes, plan.n_buckets, st["pack_bytes_read"],
+                             st["unpack_bytes_written"], world)
+    assert config["step_bytes"] == step_bytes
     flush = None
-    if resident < 4 * L2_BYTES:
+    if config["l2"].startswith("L2 flushed"):
         flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     barrier(world)
@@ -1037,16 +1065,10 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": path_dtype(w),
         "data": "synthetic",
-        "config": {"workload": w.name, "src_dtype": w.src_dtype, "n_shards": w.n_shards,
-                   "sharding": w.sharding, "expert_parallel": w.ep,
-                   "tp": w.tp, "bucket_bytes": bucket_bytes, "n_buckets": plan.n_buckets,
-                   "step": "rr_pack + rr_unpack_verify" + ("" if args.sync_verify else "_async") +
-                           " (unpack and checksum check fused)",
-                   "engine": args.engine, "check_items": args.check_items,
-                   "step_bytes": step_bytes,
-                   "l2": ("inputs > L2 (no flush needed)" if resident >= 4 * L2_BYTES else
-                          "L2 flushed between steps (512 MiB write outside the step's events)"),
-                   "parallelism": f"replicas{world}"},
+        "config": config,
+        "path": {"step": "rr_pack + rr_unpack_verify" + ("" if args.sync_verify else "_async") +
+                         " (unpack and checksum check fused)",
+                 "engine": args.engine, "check_items": args.check_items},
         "ms_per_full_model_sync": round(pack_ms + uv_ms, 3),
         "ops": {
             "pack": {"ms": round(pack_ms, 3), "ms_median": round(statistics.median(pack_all), 3),

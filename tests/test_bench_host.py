@@ -154,3 +154,23 @@ def test_bucket_source_needs_cover_every_read(name):
         part = [cut[starts[i]:starts[i] + len(sh)] for i, sh in enumerate(shards)]
         got, cs = L.pack(oracle.Source(shards=part), first=b, count=1)
         np.testing.assert_array_equal(got[0], full[b], err_msg=f"bucket {b}")
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-tied", "tiny-moe-kvrep", "tiny-units",
+                                  "qwen3-0.6b", "qwen3-8b", "qwen3-8b-tp4", "qwen3-30b-a3b",
+                                  "qwen3-8b-fsdp2-tp8", "qwen3-30b-a3b-fsdp2-ep8"])
+def test_both_arms_print_one_config(name):
+    """The reference arm's config, from the oracle's layout, equals the native
+    arm's, from the plan's byte counts (a host-only plan: no GPU)."""
+    import oracle
+    import paper_2512_22492_gb300 as rr
+    from tests import _util as U
+    w = U.workload(name)
+    m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
+    plan = rr.rr_plan_create(m, s, d, w.bucket_bytes, rr.PlanOptions(host_only=True))
+    st = plan.stats()
+    native = bench.workload_config(w, w.bucket_bytes, plan.n_buckets, st["pack_bytes_read"],
+                                   st["unpack_bytes_written"], 2)
+    assert native["step_bytes"] == (st["pack_bytes_read"] + st["pack_bytes_written"] +
+                                    st["verify_bytes_read"] + st["unpack_bytes_written"])
+    assert bench.oracle_config(oracle.workload_layout(w), w, w.bucket_bytes, 2) == native
