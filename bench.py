@@ -15,6 +15,12 @@ The separate rr_unpack and rr_verify are timed after the step loop as a
 breakdown.  Inputs (33 GB of source) are far larger than L2, so no flush is
 needed between steps.
 
+End to end (`e2e`): the same step with the trainer's shards in pinned host
+memory, by two routes, both timed and the faster reported -- the copy
+engines bringing the source over in pieces while the buckets whose sources
+have landed are packed, or the pack reading the pinned shards itself over
+NVLink-C2C.
+
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
 
 Under torchrun each rank runs an independent replica on its own GPU (the
