@@ -598,6 +598,37 @@ class BenchStep:
         self.rr.rr_plan_check(self.plan, self.stream)
 
 
+# Pointers one launch carries in its kernel parameters (include/rr.h: a launch
+# addresses at most 3968 buckets or destination tensors).
+LAUNCH_POINTERS = 3968
+
+
+def receiver_launches(plan) -> int:
+    """Kernel launches of one verifying unpack over every bucket (equally spaced
+    buckets): one, unless the buckets' destination tensors exceed one launch's
+    pointer table; the call then runs over consecutive bucket ranges whose
+    tensor windows fit, one launch each (the rule of include/rr.h), counted
+    here from the exported unpack table."""
+    import numpy as np
+    items, _ = plan.export_unpack()
+    copy = items[(items["kind"] == 6) | (items["kind"] == 7)]
+    lo = np.full(plan.n_buckets, np.iinfo(np.int64).max, np.int64)
+    hi = np.full(plan.n_buckets, -1, np.int64)
+    np.minimum.at(lo, copy["bucket"].astype(np.int64), copy["tensor"].astype(np.int64))
+    np.maximum.at(hi, copy["bucket"].astype(np.int64), copy["tensor"].astype(np.int64))
+    n, b = 0, 0
+    while b < plan.n_buckets:
+        wlo, whi, e = np.iinfo(np.int64).max, -1, b
+        while e < plan.n_buckets:
+            nlo, nhi = min(wlo, lo[e]), max(whi, hi[e])
+            if (nhi - nlo + 1 if nhi >= nlo else 0) > LAUNCH_POINTERS:
+                break
+            wlo, whi, e = nlo, nhi, e + 1
+        n += 1
+        b = max(e, b + 1)
+    return n
+
+
 def bucket_source_needs(plan) -> "np.ndarray":
     """Per bucket: how many leading bytes of the source block (every source
     buffer one after another at 16-byte starts, as synth.device lays them out)
@@ -1102,9 +1133,10 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                                        "method": "torch copy_ of 4 GiB on the device, "
                                                  "read + write bytes"}},
         "clocks": clocks,
-        # Per step: the pack kernel and the verifying unpack kernel, which
-        # writes its own result (bench launches hold a pooled slot each).
-        "gpu_launches": 2 * args.steps,
+        # Per step: the pack kernel and the verifying unpack, which writes its
+        # own result (bench launches hold a pooled slot each): one kernel, or
+        # one per bucket range where the tensors exceed one launch's table.
+        "gpu_launches": (1 + receiver_launches(plan)) * args.steps,
         "e2e": e2e,
     }
     if snapshot:

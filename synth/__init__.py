@@ -1,7 +1,8 @@
 """Seeded synthetic inputs for the weight-sync path: workload shapes and values.
 
 Input generation only.  This module holds none of the method's arithmetic: it
-names the model shapes of the five workloads (plus scaled-down test shapes)
+names the model shapes of the five workloads (plus full-size variants and
+scaled-down test shapes)
 and draws parameter values from a counter-based generator that is defined
 once and implemented twice, on the host (``synth_host.c``) and on the device
 (``synth_dev.cu``).  Both the oracle and the CUDA path take their inputs from
@@ -85,6 +86,8 @@ QWEN3_0_6B = ModelShape("qwen3-0.6b", layers=28, hidden=1024, n_q=16, n_kv=8, he
                         intermediate=3072, vocab=151936, tied=True)
 QWEN3_8B = ModelShape("qwen3-8b", layers=36, hidden=4096, n_q=32, n_kv=8, head_dim=128,
                       intermediate=12288, vocab=151936, tied=False)
+QWEN3_32B = ModelShape("qwen3-32b", layers=64, hidden=5120, n_q=64, n_kv=8, head_dim=128,
+                       intermediate=25600, vocab=151936, tied=False)
 QWEN3_30B_A3B = ModelShape("qwen3-30b-a3b", layers=48, hidden=2048, n_q=32, n_kv=4,
                            head_dim=128, intermediate=0, vocab=151936, tied=False,
                            n_experts=128, moe_intermediate=768)
@@ -160,6 +163,11 @@ EXTRA_WORKLOADS = {
     "qwen3-30b-a3b-fsdp2-ep8": Workload("qwen3-30b-a3b-fsdp2-ep8", QWEN3_30B_A3B, "bf16",
                                         n_shards=8, tp=8, bucket_bytes=256 * MiB, seed=9,
                                         sharding="rows", ep=True),
+    # The paper's Qwen3-32B with its FSDP2 trainer and TP=8 rollout: the largest
+    # of its models whose whole sync fits one GPU (131 GB of fp32 source, 67 GB
+    # of buckets and 66 GB of rollout tensors: 245 GiB).
+    "qwen3-32b-fsdp2-tp8": Workload("qwen3-32b-fsdp2-tp8", QWEN3_32B, "f32", n_shards=8, tp=8,
+                                    bucket_bytes=128 * MiB, seed=10, sharding="rows"),
 }
 
 

@@ -174,3 +174,17 @@ def test_both_arms_print_one_config(name):
     assert native["step_bytes"] == (st["pack_bytes_read"] + st["pack_bytes_written"] +
                                     st["verify_bytes_read"] + st["unpack_bytes_written"])
     assert bench.oracle_config(oracle.workload_layout(w), w, w.bucket_bytes, 2) == native
+
+
+@pytest.mark.parametrize("name,want", [("qwen3-8b", 1), ("qwen3-30b-a3b-fsdp2-tp8", 1),
+                                       ("qwen3-32b-fsdp2-tp8", 2)])
+def test_receiver_launch_count(name, want):
+    """The verifying unpack's launches per full call: one while every
+    destination tensor fits one launch's pointer table (3480 tensors for
+    30B-A3B at TP=8), two bucket ranges for Qwen3-32B at TP=8 (4120)."""
+    import paper_2512_22492_gb300 as rr
+    from tests import _util as U
+    w = U.workload(name)
+    m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
+    plan = rr.rr_plan_create(m, s, d, w.bucket_bytes, rr.PlanOptions(host_only=True))
+    assert bench.receiver_launches(plan) == want
