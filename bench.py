@@ -80,7 +80,7 @@ def parse():
     ap.add_argument("--e2e-route", choices=["auto", "copy", "direct"], default="auto",
                     help="e2e source route: copy engines, the pack reading pinned host "
                          "memory directly, or both timed and the faster reported (auto)")
-    ap.add_argument("--e2e-direct-pieces", type=int, default=8,
+    ap.add_argument("--e2e-direct-pieces", type=int, default=16,
                     help="bucket ranges of the direct e2e route (the receiver follows each)")
     ap.add_argument("--no-next-rows", action="store_true",
                     help="skip the resume (bucket-range) and relay re-pack timings")
@@ -777,7 +777,7 @@ class DirectE2E:
     the checksums and the result rows read back to pinned host memory, and the
     step's stream waits for the receiver, so events on it bracket everything."""
 
-    def __init__(self, bs, host_src, pieces: int = 8, ring_steps: int = 64):
+    def __init__(self, bs, host_src, pieces: int = 16, ring_steps: int = 64):
         import torch
         from synth import device as D
         self.bs = bs
@@ -798,8 +798,8 @@ class DirectE2E:
         self.scratch = torch.zeros(nb + 4, dtype=torch.int64, device="cuda")
         self.host_cs = torch.empty(bs.buf.checksums.numel(), dtype=torch.int64, pin_memory=True)
         self.host_res = torch.empty((self.n_ranges, 2), dtype=torch.int64, pin_memory=True)
-        lo, _hi = torch.cuda.Stream.priority_range()
-        self.recv = torch.cuda.Stream(priority=lo)
+        _least, greatest = torch.cuda.Stream.priority_range()   # lower number: higher priority
+        self.recv = torch.cuda.Stream(priority=greatest)
         self.received = torch.cuda.Event()     # after the last step's receiver and read-back
         self.received.record(self.recv)
         self.used = 0
