@@ -314,7 +314,7 @@ typedef struct {
 
 /* Copies up to cap items (and, if block_first is not NULL, the per-block item
  * ranges: grid_blocks + 1 entries for pack, unpack_grid_blocks + 1 for
- * unpack) into caller memory. */
+ * unpack) into caller memory.  No counterpart in the paper (inspection). */
 rr_status rr_plan_export_pack(const rr_plan* plan, rr_pack_item* items, int64_t cap,
                               uint32_t* block_first);
 
@@ -419,6 +419,8 @@ rr_status rr_clear_range(const rr_plan* plan, int32_t first_bucket, int32_t n_bu
 
 /* Receiver side, fused: rr_unpack and rr_verify in one pass over the buckets
  * (every bucket byte is read once, for the copy and for the checksum).
+ * Sections 5.2.1 and 5.2.2: the rollout completes its update from what it
+ * pulled, and must know which of the buckets it holds are intact.
  * Writes every destination byte of the range, as rr_unpack / rr_unpack_range
  * would, whether or not its bucket verifies; the caller re-pulls the flagged
  * buckets and unpacks them again (for example with this call on a range).
