@@ -77,9 +77,11 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-pieces", type=int, default=16,
                     help="pieces the e2e source copy is cut into (the pack follows each)")
-    ap.add_argument("--e2e-route", choices=["auto", "copy", "direct"], default="auto",
+    ap.add_argument("--e2e-route", choices=["auto", "copy", "direct", "pageable"],
+                    default="auto",
                     help="e2e source route: copy engines, the pack reading pinned host "
-                         "memory directly, or both timed and the faster reported (auto)")
+                         "memory directly, the same from pageable host memory, or all "
+                         "timed and the fastest reported (auto)")
     ap.add_argument("--e2e-direct-pieces", type=int, default=16,
                     help="bucket ranges of the direct e2e route (the receiver follows each)")
     ap.add_argument("--no-next-rows", action="store_true",
@@ -1076,6 +1078,25 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                 "how": "rr_pack_range reads the pinned host shards (register path over "
                        "NVLink-C2C); the receiver overlaps on a second stream"}
             del de
+        refused = {}
+        if args.e2e_route in ("auto", "pageable") and 2 * pinned_need <= host_memory_bytes() // 2:
+            # The direct route from ordinary (pageable) host memory: a GPU that
+            # reads it through the CPU's page tables (Grace) needs no pinning;
+            # elsewhere the library refuses it before launching anything.
+            pageable = torch.empty(buf.flat.numel(), dtype=torch.uint8)
+            pageable.copy_(buf.flat)
+            try:
+                de = DirectE2E(bs, pageable, pieces=args.e2e_direct_pieces)
+                ms = time_e2e(de, args.steps, world, stream)
+                routes["direct_pageable"] = {
+                    "ms_per_step": round(ms, 3), "h2d_bytes_per_step": de.h2d_bytes,
+                    "d2h_bytes_per_step": de.d2h_bytes, "bucket_ranges_per_step": de.n_ranges,
+                    "link_GB/s": round(de.h2d_bytes / (ms * 1e-3) / 1e9, 1),
+                    "how": "as direct, from pageable (unpinned) host memory"}
+                del de
+            except rr.RRError as exc:
+                refused["direct_pageable"] = str(exc).splitlines()[0]
+            del pageable
         best = min(routes, key=lambda k: routes[k]["ms_per_step"])
         e2e_ms = routes[best]["ms_per_step"]
         e2e = {"value": round(aggregate_gbs(world, step_bytes, e2e_ms), 2), "unit": UNIT,
@@ -1083,6 +1104,8 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                "d2h_bytes_per_step": routes[best]["d2h_bytes_per_step"],
                "ms_per_step": e2e_ms, "route": best, "pipelined": True,
                "routes": routes}
+        if refused:
+            e2e["refused_routes"] = refused
         if "copy_engine" in routes:
             ceil_ms = routes["copy_engine"]["h2d_ceiling"]["ms"]
             e2e["h2d_ceiling_frac"] = round(ceil_ms / e2e_ms, 4)

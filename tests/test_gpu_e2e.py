@@ -1,9 +1,10 @@
-"""The benchmark's two end-to-end routes, run as bench.py runs them, against the oracle.
+"""The benchmark's end-to-end routes, run as bench.py runs them, against the oracle.
 
 The trainer's shards sit in pinned host memory.  The copy-engine route
 (bench.PipelinedE2E) copies them to the device in pieces and packs each run of
 buckets as its sources land; the direct route (bench.DirectE2E) packs straight
-from host memory, the pack's loads crossing NVLink-C2C.  Both hand each bucket
+from host memory, the pack's loads crossing NVLink-C2C, from pinned memory or,
+where the GPU reads it, from ordinary pageable memory.  Each hands every bucket
 range to the stream-ordered verifying unpack and read the checksums and result
 rows back to the host (RobustRL Section 5.2.1: the rollout completes its update
 from what it pulled; Section 5.2.2: it must know that what it holds is whole).
@@ -55,14 +56,19 @@ SAMPLED = ["embed_tokens", "layers.0.qkv_proj", "layers.13.o_proj", "layers.27.d
            "layers.27.post_attention_layernorm", "norm"]
 
 
-@pytest.mark.parametrize("route", ["copy_engine", "direct"])
+@pytest.mark.parametrize("route", ["copy_engine", "direct", "direct_pageable"])
 def test_e2e_route(route, oracle_image):
     import bench
+    if route == "direct_pageable":
+        from tests.test_pointers import _pageable_access
+        if not _pageable_access():
+            pytest.skip("this GPU does not read pageable host memory")
     L, gen, want, want_cs = oracle_image
     w = synth.WORKLOADS["qwen3-0.6b"]
     bs = bench.BenchStep(w, w.bucket_bytes, poison=0xAB)
     plan, buf = bs.plan, bs.buf
-    host = torch.empty(buf.flat.numel(), dtype=torch.uint8, pin_memory=True)
+    host = torch.empty(buf.flat.numel(), dtype=torch.uint8,
+                       pin_memory=route != "direct_pageable")
     host.copy_(buf.flat)
     buf.flat.fill_(0x5A)                     # only the host copy holds the weights now
     torch.cuda.synchronize()
