@@ -1,4 +1,5 @@
-"""rr_pack reading the trainer's shards from pinned host memory.
+"""rr_pack reading the trainer's shards from host memory (pinned, or pageable
+where the GPU reads it).
 
 A trainer that keeps its master weights in host RAM (offloaded optimizer
 state) hands the pack host pointers: on GB300 the pack's own loads read them
@@ -130,3 +131,27 @@ def test_qwen3_0_6b_from_host():
     for t in sorted({0, 1, plan.n_tensors // 2, plan.n_tensors - 1}):
         np.testing.assert_array_equal(H.tensor_host(buf, t), L.unpack_tensor(want, t),
                                       err_msg=plan.tensor_names[t])
+
+
+@pytest.mark.parametrize("name", ["tiny-tp4", "tiny-moe-kvrep", "qwen3-0.6b"])
+def test_pageable_host_source(name):
+    """On a GPU that reads pageable host memory (Grace, through address
+    translation) the trainer's shards need not be pinned: ordinary host
+    memory is read by the same kernel, with the same bytes."""
+    from tests.test_pointers import _pageable_access
+    if not _pageable_access():
+        pytest.skip("this GPU does not read pageable host memory (the call refuses it)")
+    desc = U.workload_desc(name)
+    L = U.to_oracle(desc)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"])
+    shards = L.host_shards(desc["seed"], desc["specials"])
+    flat = torch.from_numpy(np.concatenate([np.asarray(x, np.uint8) for x in shards]))
+    assert not flat.is_pinned()
+    buf = H.alloc(plan, flat=flat)
+    H.pack(buf)
+    torch.cuda.synchronize()
+    rr.rr_plan_check(plan)
+    want, want_cs = oracle_pack(L, shards, parallel=name == "qwen3-0.6b")
+    np.testing.assert_array_equal(H.buckets_host(buf), want)
+    np.testing.assert_array_equal(H.checksums_host(buf), want_cs)
