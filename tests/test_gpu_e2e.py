@@ -96,3 +96,37 @@ def test_e2e_route(route, oracle_image):
         t = L.tensor_index(name, 0)
         got = buf.dst[t][:plan.tensor_numel[t]].cpu().numpy().view(np.uint16)
         np.testing.assert_array_equal(got, L.reshard_tensor(gen, t), err_msg=name)
+
+
+@pytest.mark.parametrize("route", ["copy_engine", "direct", "direct_pageable"])
+def test_e2e_route_tp4_special_values(route):
+    """The same routes on the tiny TP=4 workload with special values (RNE ties,
+    subnormals, infinities, NaNs): four ranks' streams, every bucket, checksum
+    and tensor against the oracle."""
+    import bench
+    if route == "direct_pageable":
+        from tests.test_pointers import _pageable_access
+        if not _pageable_access():
+            pytest.skip("this GPU does not read pageable host memory")
+    w = synth.TEST_WORKLOADS["tiny-tp4"]
+    L = oracle.workload_layout(w)
+    gen = oracle.Source(seed=w.seed, specials=w.specials)
+    want, want_cs = L.pack(gen)
+    bs = bench.BenchStep(w, w.bucket_bytes, poison=0xAB)
+    plan, buf = bs.plan, bs.buf
+    host = torch.empty(buf.flat.numel(), dtype=torch.uint8,
+                       pin_memory=route != "direct_pageable")
+    host.copy_(buf.flat)
+    buf.flat.fill_(0x5A)
+    torch.cuda.synchronize()
+    e2e = (bench.PipelinedE2E(bs, host, pieces=4) if route == "copy_engine"
+           else bench.DirectE2E(bs, host, pieces=4))
+    for _ in range(2):
+        e2e.step()
+    e2e.check()
+    np.testing.assert_array_equal(buf.bucket_store[:, :plan.bucket_bytes].cpu().numpy(), want)
+    np.testing.assert_array_equal(e2e.host_cs.numpy().view(np.uint64)[:plan.n_buckets], want_cs)
+    for t in range(plan.n_tensors):
+        np.testing.assert_array_equal(
+            buf.dst[t][:plan.tensor_numel[t]].cpu().numpy().view(np.uint16),
+            L.unpack_tensor(want, t), err_msg=f"{plan.tensor_names[t]} rank {plan.tensor_ranks[t]}")
