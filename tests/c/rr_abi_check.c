@@ -14,8 +14,9 @@
  *     272 stream bytes in buckets of 128 bytes: 3 per rank, 6 in all.
  *
  * Without arguments only host-side calls run (a host-only plan); with "gpu"
- * the plan runs: pack, verify, unpack, and verify again after one byte of one
- * bucket is damaged.  Exit status 0 means every check passed.
+ * the plan runs: pack, verify, unpack, pack again from a source in pinned
+ * host memory, and verify again after one byte of one bucket is damaged.
+ * Exit status 0 means every check passed.
  */
 #include <stdint.h>
 #include <stdio.h>
@@ -203,6 +204,29 @@ int main(int argc, char** argv) {
     CUDA(cudaMemcpy(t_b0, d_dst + 256 * 1, 16, cudaMemcpyDeviceToHost));
     CHECK(memcmp(t_a1, want[3], 64) == 0 && memcmp(t_b0, want[2] + 0, 16) == 0,
           "unpacked tensors");
+
+    /* The same pack with the source left in pinned host memory: the pack's own
+     * loads read it over the host link; the bytes are the same. */
+    uint8_t* h_flat = NULL;
+    uint8_t* d_buckets2 = NULL;
+    uint64_t* d_sums2 = NULL;
+    CUDA(cudaMallocHost((void**)&h_flat, sizeof host_flat));
+    memcpy(h_flat, host_flat, sizeof host_flat);
+    CUDA(cudaMalloc((void**)&d_buckets2, N_BUCKETS * BUCKET));
+    CUDA(cudaMalloc((void**)&d_sums2, N_BUCKETS * sizeof(uint64_t)));
+    CUDA(cudaMemset(d_buckets2, 0xAB, N_BUCKETS * BUCKET));
+    const void* h_shards[2] = {h_flat, h_flat + S};
+    void* bucket_ptrs2[N_BUCKETS];
+    for (int b = 0; b < N_BUCKETS; ++b) bucket_ptrs2[b] = d_buckets2 + b * BUCKET;
+    CHECK(rr_pack(plan, h_shards, bucket_ptrs2, d_sums2, 0) == RR_OK, "pack from host memory");
+    CUDA(cudaDeviceSynchronize());
+    CUDA(cudaMemcpy(got, d_buckets2, sizeof got, cudaMemcpyDeviceToHost));
+    CUDA(cudaMemcpy(got_sums, d_sums2, sizeof got_sums, cudaMemcpyDeviceToHost));
+    CHECK(memcmp(got, want, sizeof got) == 0, "bucket bytes, host source");
+    CHECK(memcmp(got_sums, want_sums, sizeof got_sums) == 0, "checksums, host source");
+    cudaFreeHost(h_flat);
+    cudaFree(d_buckets2);
+    cudaFree(d_sums2);
 
     CUDA(cudaMemset(d_buckets + 4 * BUCKET + 7, 0x5A, 1));   /* one damaged byte */
     CHECK(rr_verify(plan, (const void* const*)bucket_ptrs, d_sums, &n_bad, &first_bad, 0) ==
