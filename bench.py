@@ -999,10 +999,34 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                                     "restore_frac": round(h2d_ms / r_ms, 4),
                                     "method": "copy of the pinned snapshot's bucket block host -> "
                                               "device, mean of 2 after one warm-up"}}
+        del hstore, hview
+        # The same into ordinary (pageable) host memory, where the GPU reaches it
+        # through the CPU's page tables (Grace); elsewhere the call is refused.
+        pstore = torch.empty((plan.n_buckets, row), dtype=torch.uint8)
+        pstore.fill_(0)
+        pview = pstore[:, :plan.bucket_bytes]
+        pcs = torch.zeros_like(buf.checksums)
+        try:
+            p_ms = _event_ms(lambda: rr.rr_pack(plan, t_src, pview, pcs, stream), stream)
+            n_bad, _ = rr.rr_unpack_verify(plan, pview, pcs, t_dst, stream=stream)
+            if n_bad:
+                raise RuntimeError(f"pageable snapshot restore: {n_bad} bad buckets")
+            pr_ms = _event_ms(lambda: rr.rr_unpack_verify(plan, pview, pcs, t_dst,
+                                                          stream=stream), stream)
+            snapshot["pageable"] = {
+                "pack_to_host_ms": round(p_ms, 2),
+                "host_GB/s": round(st["pack_bytes_written"] / (p_ms * 1e-3) / 1e9, 1),
+                "identical": bool(torch.equal(pcs, buf.checksums)),
+                "restore_ms": round(pr_ms, 2),
+                "restore_link_GB/s": round(st["verify_bytes_read"] / (pr_ms * 1e-3) / 1e9, 1),
+                "how": "snapshot into and restore from unpinned host memory (mean of 3 "
+                       "after one warm-up)"}
+        except rr.RRError as exc:
+            snapshot["pageable"] = {"refused": str(exc).splitlines()[0]}
+        del pstore, pview
         # The device buckets were overwritten by the ceiling copy: pack them again.
         rr.rr_pack(plan, t_src, t_bkt, buf.checksums, stream)
         torch.cuda.synchronize()
-        del hstore, hview
 
     # End to end through the public API with host buffers: every step copies the
     # trainer's shards from pinned host memory, syncs, and reads back the checksums.

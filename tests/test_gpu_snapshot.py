@@ -31,9 +31,9 @@ def _cuda():
     yield
 
 
-def host_buckets(plan):
+def host_buckets(plan, pinned=True):
     row = (plan.bucket_bytes + 15) // 16 * 16
-    store = torch.empty((plan.n_buckets, row), dtype=torch.uint8, pin_memory=True)
+    store = torch.empty((plan.n_buckets, row), dtype=torch.uint8, pin_memory=pinned)
     store.fill_(0xAB)
     return store, store[:, :plan.bucket_bytes]
 
@@ -48,8 +48,16 @@ def oracle_pack(L, desc):
             np.concatenate([p[1] for p in parts]).astype(np.uint64))
 
 
+@pytest.mark.parametrize("where", ["pinned", "pageable"])
 @pytest.mark.parametrize("name", ["tiny-tp4", "tiny-moe-kvrep", "qwen3-0.6b"])
-def test_snapshot_to_host_and_restore(name):
+def test_snapshot_to_host_and_restore(name, where):
+    """`pageable`: the snapshot goes into ordinary host memory, which a GPU that
+    reads and writes pageable memory through the CPU's page tables (Grace)
+    reaches without pinning."""
+    if where == "pageable":
+        from tests.test_pointers import _pageable_access
+        if not _pageable_access():
+            pytest.skip("this GPU does not reach pageable host memory")
     desc = U.workload_desc(name)
     L = U.to_oracle(desc)
     m, s, d = U.to_product(desc)
@@ -57,7 +65,7 @@ def test_snapshot_to_host_and_restore(name):
     assert L.n_buckets == plan.n_buckets
     dev = H.alloc(plan, with_dst=False)
     H.fill_with_generator(dev, m, desc["seed"], desc["specials"])
-    store, view = host_buckets(plan)
+    store, view = host_buckets(plan, pinned=where == "pinned")
     cs = torch.zeros(plan.n_buckets, dtype=torch.int64, device="cuda")
     rr.rr_pack(plan, dev.shards, view, cs)                     # straight into host memory
     H.pack(dev)                                                # and on the device
