@@ -67,7 +67,8 @@ class _Layout(ctypes.Structure):
                 ("shard_bytes_in", ctypes.c_int64), ("explicit_offset", _P64),
                 ("chunk_rows", _P64), ("param_gen_base", _P64),
                 ("n_units", ctypes.c_int32), ("pad2_", ctypes.c_int32),
-                ("param_unit", ctypes.POINTER(ctypes.c_int32)), ("unit_shard_bytes", _P64)]
+                ("param_unit", ctypes.POINTER(ctypes.c_int32)), ("unit_shard_bytes", _P64),
+                ("dst_dtype", ctypes.c_int32), ("pad3_", ctypes.c_int32)]
 
 
 _VALUE_FN = ctypes.CFUNCTYPE(ctypes.c_uint32, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32)
@@ -101,6 +102,8 @@ def load(path: str) -> ctypes.CDLL:
     L.orc_rne_bf16.restype = ctypes.c_uint16
     L.orc_rne_bf16_array.argtypes = [vp, vp, ctypes.c_int64]
     L.orc_rne_bf16_array.restype = None
+    L.orc_rne_f16_array.argtypes = [vp, vp, ctypes.c_int64]
+    L.orc_rne_f16_array.restype = None
     L.orc_tensor_elements.argtypes = [LP, SP, ctypes.c_int32, ctypes.c_int64,
                                       ctypes.c_int64, vp]
     L.orc_tensor_elements.restype = ctypes.c_int
@@ -137,6 +140,14 @@ def rne_bf16(bits: np.ndarray) -> np.ndarray:
     a = np.ascontiguousarray(bits, dtype=np.uint32)
     out = np.empty(a.shape, dtype=np.uint16)
     lib().orc_rne_bf16_array(a.ctypes.data, out.ctypes.data, a.size)
+    return out
+
+
+def rne_f16(bits: np.ndarray) -> np.ndarray:
+    """float32 bit patterns (uint32) -> IEEE binary16 bit patterns (uint16)."""
+    a = np.ascontiguousarray(bits, dtype=np.uint32)
+    out = np.empty(a.shape, dtype=np.uint16)
+    lib().orc_rne_f16_array(a.ctypes.data, out.ctypes.data, a.size)
     return out
 
 
@@ -182,8 +193,10 @@ class Layout:
 
     def __init__(self, params, tensors, n_shards: int, tp: int, bucket_bytes: int,
                  align_bytes: int = 16, tensor_align: int = 256, sharding: str = "flat",
-                 explicit_offsets=None, shard_bytes: int = 0, units=None):
-        """units: with sharding="units", the unit of each parameter."""
+                 explicit_offsets=None, shard_bytes: int = 0, units=None,
+                 dst_dtype: str = "bf16"):
+        """units: with sharding="units", the unit of each parameter.
+        dst_dtype: the rollout's 16-bit element type, "bf16" or "f16"."""
         self.sharding = sharding
         self.params = list(params)
         self.tensors = list(tensors)
@@ -223,6 +236,8 @@ class Layout:
                      "rank_first_bucket", "chunk_rows", "param_gen_base"):
             setattr(L, name, getattr(self, name).ctypes.data_as(_P64))
         L.sharding = {"flat": 0, "rows": 1, "tensors": 2, "units": 3}[sharding]
+        self.dst_dtype = dst_dtype
+        L.dst_dtype = {"bf16": 0, "f16": 1}[dst_dtype]
         L.shard_bytes_in = shard_bytes
         self.units = None
         self.unit_shard_bytes = np.zeros(0, np.int64)
@@ -424,4 +439,5 @@ def workload_layout(w, bucket_bytes: Optional[int] = None) -> Layout:
     tensors = qwen3.rollout_tensors(w.shape, params, w.tp, ep=getattr(w, "ep", False))
     units = qwen3.layer_units(params) if w.sharding == "units" else None
     return Layout(params, tensors, n_shards=w.n_shards, tp=w.tp,
-                  bucket_bytes=bucket_bytes or w.bucket_bytes, sharding=w.sharding, units=units)
+                  bucket_bytes=bucket_bytes or w.bucket_bytes, sharding=w.sharding, units=units,
+                  dst_dtype=getattr(w, "dst_dtype", "bf16"))

@@ -66,6 +66,17 @@
  *  (so +-0 and subnormals are kept, overflow carries into +-inf and +-inf map
  *  to themselves).  A bfloat16 source is copied bit for bit.
  *
+ *  Cast to float16 instead (the rollout's 16-bit weights as IEEE binary16;
+ *  Section 7.4 calls the transferred model FP16).  A float32 value is rounded
+ *  to the nearest binary16 value, ties to the even significand: binary16
+ *  values are the multiples of 2^(E - 10) in the binade [2^E, 2^(E+1)) for
+ *  E = -14 .. 15, and the multiples of 2^-24 below 2^-14 (subnormals, kept);
+ *  a value that rounds to 2^16 or more is an infinity.  +-0 and +-inf map to
+ *  themselves.  A NaN keeps its sign and its top payload bits with the quiet
+ *  bit forced: sign | 0x7E00 | ((b >> 13) & 0x01FF), never an infinity.  A
+ *  bfloat16 source is first widened exactly (its bits shifted up by 16) and
+ *  then rounded the same way.
+ *
  *  Stream and buckets.  Each rollout rank r has a byte stream holding its
  *  destination tensors in the given order, each starting at the next multiple
  *  of tensor_align; elements are little-endian.  The stream is cut every
@@ -132,6 +143,9 @@ typedef struct {
     const int32_t* param_unit;  /* [n_params] unit of each parameter                */
     /* derived, continued */
     int64_t* unit_shard_bytes;  /* [n_units] S_u                                    */
+    /* description, continued: destination element type */
+    int32_t dst_dtype;          /* 0: bfloat16, 1: float16                          */
+    int32_t pad3_;
 } orc_layout;
 
 /* Where source values come from: real shard buffers, or a generator that maps
@@ -278,7 +292,54 @@ void orc_rne_bf16_array(const uint32_t* in, uint16_t* out, int64_t n) {
     for (int64_t i = 0; i < n; ++i) out[i] = orc_rne_bf16(in[i]);
 }
 
-static uint16_t cast_to_bf16(uint32_t bits, int32_t elem_bytes) {
+/* Nearest integer to v / 2^sh, ties to even (sh >= 1). */
+static uint64_t round_shift(uint64_t v, int32_t sh) {
+    if (sh > 40) return 0; /* v < 2^24: below half of one unit */
+    uint64_t q = v >> sh;
+    uint64_t r = v - (q << sh);
+    uint64_t half = 1ull << (sh - 1);
+    if (r > half || (r == half && (q & 1u))) q += 1;
+    return q;
+}
+
+uint16_t orc_rne_f16(uint32_t b) {
+    const uint16_t sign = (uint16_t)((b >> 16) & 0x8000u);
+    const uint32_t mag = b & 0x7FFFFFFFu;
+    if (mag > 0x7F800000u) return (uint16_t)(sign | 0x7E00u | ((mag >> 13) & 0x01FFu));
+    if (mag == 0x7F800000u) return (uint16_t)(sign | 0x7C00u);
+    /* |x| = sig * 2^(e - 150), sig the significand with its leading bit */
+    int32_t e = (int32_t)(mag >> 23);
+    uint64_t sig = mag & 0x7FFFFFu;
+    if (e == 0)
+        e = 1; /* float32 subnormal */
+    else
+        sig |= 0x800000u;
+    uint32_t h;
+    if (mag >= 0x38800000u) {
+        /* |x| >= 2^-14: the binade of |x| is 2^E with E = e - 127; binary16
+         * spacing there is 2^(E - 10), so n = |x| / 2^(E - 10) = sig / 2^13,
+         * an integer in [2^10, 2^11] after rounding.  The value n * 2^(E - 10)
+         * is encoded as exponent field E + 15 and mantissa n - 2^10, i.e.
+         * ((E + 14) << 10) + n; n = 2^11 carries into the next binade. */
+        const int32_t E = e - 127;
+        const uint64_t n = round_shift(sig, 13);
+        const int64_t bits = ((int64_t)(E + 14) << 10) + (int64_t)n;
+        h = bits >= 0x7C00 ? 0x7C00u : (uint32_t)bits;
+    } else {
+        /* |x| < 2^-14: the multiples of 2^-24; n = |x| / 2^-24 = sig * 2^(e - 126),
+         * at most 2^10 (which is 2^-14, the smallest normal, encoded as n). */
+        h = (uint32_t)round_shift(sig, 126 - e);
+    }
+    return (uint16_t)(sign | h);
+}
+
+void orc_rne_f16_array(const uint32_t* in, uint16_t* out, int64_t n) {
+    for (int64_t i = 0; i < n; ++i) out[i] = orc_rne_f16(in[i]);
+}
+
+/* The 16-bit destination element for source bits of elem_bytes. */
+static uint16_t cast_to_dst(uint32_t bits, int32_t elem_bytes, int32_t dst_dtype) {
+    if (dst_dtype == 1) return orc_rne_f16(elem_bytes == 4 ? bits : bits << 16);
     return elem_bytes == 4 ? orc_rne_bf16(bits) : (uint16_t)bits;
 }
 
@@ -352,7 +413,7 @@ int orc_tensor_elements(const orc_layout* L, const orc_source* S, int32_t t, int
             uint32_t bits;
             int rc = source_bits(L, S, B->param, row * P->cols + col, &bits);
             if (rc) return rc;
-            out[j - j0] = cast_to_bf16(bits, P->elem_bytes);
+            out[j - j0] = cast_to_dst(bits, P->elem_bytes, L->dst_dtype);
         }
         base += n;
     }

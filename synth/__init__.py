@@ -71,6 +71,7 @@ class Workload:
     sharding: str = "flat"   # "flat" (one FSDP1 FlatParameter), "rows" (FSDP2 dim-0), or
                              # "units" (FSDP1, one FlatParameter per decoder layer + root)
     ep: bool = False         # rollout experts split whole over the ranks (expert parallel)
+    dst_dtype: str = "bf16"  # the rollout's 16-bit element type: "bf16" or "f16"
 
     @property
     def src_elem_bytes(self) -> int:

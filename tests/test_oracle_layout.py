@@ -113,9 +113,23 @@ def _to_bf16_bits(t: torch.Tensor) -> torch.Tensor:
     return torch.where(nan, nan_bits, conv)
 
 
-def restate_rollout(shape, P, tp, ep=False):
+def _to_f16_bits(t: torch.Tensor) -> torch.Tensor:
+    """fp32 (or bf16, widened exactly) bit patterns -> IEEE binary16 bit
+    patterns: PyTorch's conversion for numbers, the stated NaN rule for NaNs."""
+    u = t.to(torch.int64) & (0xFFFF if t.dtype == torch.int16 else 0xFFFFFFFF)
+    if t.dtype == torch.int16:
+        u = u << 16
+    f = u.to(torch.int32).view(torch.float32)
+    conv = f.to(torch.float16).view(torch.int16)
+    nan = (u & 0x7FFFFFFF) > 0x7F800000
+    nan_bits = (((u >> 16) & 0x8000) | 0x7E00 | ((u >> 13) & 0x1FF)).to(torch.int32).to(torch.int16)
+    return torch.where(nan, nan_bits, conv)
+
+
+def restate_rollout(shape, P, tp, ep=False, dst_dtype="bf16"):
     """Per rank, the rollout tensors built the way an inference engine's loader
-    would; ep: each rank loads its own experts whole."""
+    would; ep: each rank loads its own experts whole; dst_dtype: the rollout's
+    16-bit type."""
     H = shape.hidden
 
     def kv(t, r):
@@ -164,7 +178,8 @@ def restate_rollout(shape, P, tp, ep=False):
         if not shape.tied:
             ts.append(P["lm_head.weight"].chunk(tp, 0)[r])
         assert all(t.shape[-1] in (H, t.shape[-1]) for t in ts)
-        ranks.append([_to_bf16_bits(t.contiguous()) for t in ts])
+        cast = _to_f16_bits if dst_dtype == "f16" else _to_bf16_bits
+        ranks.append([cast(t.contiguous()) for t in ts])
     return ranks
 
 
@@ -261,6 +276,35 @@ def test_oracle_matches_restatement(name):
     want_b = restate_buckets(ranks, w.bucket_bytes)
     buckets, cs = L.pack(src)
     assert buckets.shape[0] == len(want_b)
+    for b, wb in enumerate(want_b):
+        assert buckets[b].tobytes() == wb, f"bucket {b}"
+        assert int(cs[b]) == int(np.frombuffer(wb, "<u8").sum(dtype=np.uint64))
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-tp4", "tiny-moe-bf16-specials", "tiny-fsdp2",
+                                  "tiny-kvrep-f32"])
+def test_oracle_matches_restatement_f16(name):
+    """The same restatement for a float16 rollout: PyTorch's float16 conversion
+    of the loader-built tensors (the stated NaN rule for NaNs), then the same
+    stream and buckets."""
+    w = _workload(name).with_(dst_dtype="f16")
+    L = oracle.workload_layout(w)
+    assert L.dst_dtype == "f16"
+    P = _param_tensors(L.params, _flat_offsets(L.params), w.seed, w.specials)
+    ranks = restate_rollout(w.shape, P, w.tp, ep=w.ep, dst_dtype="f16")
+    if w.sharding == "rows":
+        shards = fsdp2_shards(L.params, P, w.n_shards)
+    else:
+        shards = L.host_shards(w.seed, w.specials)
+    src = oracle.Source(shards=shards)
+    flat_t = [t for rank in ranks for t in rank]
+    order = [i for r in range(w.tp) for i, (_, rk, _) in enumerate(L.tensors) if rk == r]
+    for t_idx, want in zip(order, flat_t):
+        np.testing.assert_array_equal(L.reshard_tensor(src, t_idx),
+                                      want.reshape(-1).numpy().view(np.uint16),
+                                      err_msg=L.tensors[t_idx][0])
+    want_b = restate_buckets(ranks, w.bucket_bytes)
+    buckets, cs = L.pack(src)
     for b, wb in enumerate(want_b):
         assert buckets[b].tobytes() == wb, f"bucket {b}"
         assert int(cs[b]) == int(np.frombuffer(wb, "<u8").sum(dtype=np.uint64))

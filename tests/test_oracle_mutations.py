@@ -68,6 +68,21 @@ MUTATIONS = [
     ("unit parameters not aligned",
      "                local = align_up(local, a);\n                L->param_offset[p] = local;",
      "                L->param_offset[p] = local + 0 * a;"),
+    ("f16: NaN loses the quiet bit",
+     "return (uint16_t)(sign | 0x7E00u | ((mag >> 13) & 0x01FFu));",
+     "return (uint16_t)(sign | 0x7C00u | ((mag >> 13) & 0x01FFu));"),
+    ("f16: rounding half up, not to even",
+     "if (r > half || (r == half && (q & 1u))) q += 1;", "if (r >= half) q += 1;"),
+    ("f16: overflow saturates to the largest finite",
+     "h = bits >= 0x7C00 ? 0x7C00u : (uint32_t)bits;",
+     "h = bits >= 0x7C00 ? 0x7BFFu : (uint32_t)bits;"),
+    ("f16: subnormal spacing off by one", "h = (uint32_t)round_shift(sig, 126 - e);",
+     "h = (uint32_t)round_shift(sig, 127 - e);"),
+    ("f16: exponent bias off by one", "const int64_t bits = ((int64_t)(E + 14) << 10) + (int64_t)n;",
+     "const int64_t bits = ((int64_t)(E + 15) << 10) + (int64_t)n;"),
+    ("f16: bf16 source not widened",
+     "if (dst_dtype == 1) return orc_rne_f16(elem_bytes == 4 ? bits : bits << 16);",
+     "if (dst_dtype == 1) return orc_rne_f16(bits);"),
 ]
 
 
@@ -80,6 +95,10 @@ def battery():
         ("cast named cases", cast_pins.test_named_cases),
         ("cast structured", cast_pins.test_structured_against_brute_force),
         ("cast NaN", cast_pins.test_nan_properties),
+        ("f16 named cases", cast_pins.test_f16_named_cases),
+        ("f16 ties", cast_pins.test_f16_ties_against_brute_force_and_numpy),
+        ("f16 NaN", cast_pins.test_f16_nan_properties),
+        ("f16 from bf16", cast_pins.test_f16_from_every_bfloat16_pattern),
         ("checksum", layout_pins.test_checksum_against_numpy_and_linearity),
         ("verify", layout_pins.test_verify_flags_damage),
         ("restatement tiny-tp4", lambda: layout_pins.test_oracle_matches_restatement("tiny-tp4")),
