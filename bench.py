@@ -57,6 +57,8 @@ def parse():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--workload", default="qwen3-8b")
     ap.add_argument("--bucket-mib", type=int, default=0, help="override the bucket size")
+    ap.add_argument("--dst-dtype", choices=["bf16", "f16"], default="bf16",
+                    help="the rollout's 16-bit element type")
     ap.add_argument("--layers", type=int, default=0,
                     help="keep only the first N decoder layers (a small case of the same "
                          "kernels, for profiler captures); the workload name says so")
@@ -393,7 +395,8 @@ def workload_config(w, bucket_bytes: int, n_buckets: int, pack_read: int, dst_by
     buckets = n_buckets * bucket_bytes
     step_bytes = pack_read + 2 * buckets + dst_bytes
     resident = pack_read + buckets + dst_bytes
-    return {"workload": w.name, "src_dtype": w.src_dtype, "n_shards": w.n_shards,
+    return {"workload": w.name, "src_dtype": w.src_dtype,
+            "dst_dtype": getattr(w, "dst_dtype", "bf16"), "n_shards": w.n_shards,
             "sharding": w.sharding, "expert_parallel": w.ep, "tp": w.tp,
             "bucket_bytes": bucket_bytes, "n_buckets": n_buckets, "step_bytes": step_bytes,
             "l2": ("inputs > L2 (no flush needed)" if resident >= 4 * L2_BYTES else
@@ -412,7 +415,10 @@ def oracle_config(L, w, bucket_bytes: int, world: int) -> dict:
 
 def path_dtype(w) -> str:
     """What the path computes: an fp32 source is rounded to bf16 (nearest,
-    ties to even, in integer arithmetic); a bf16 source is copied bit for bit."""
+    ties to even, in integer arithmetic); a bf16 source is copied bit for bit.
+    For a float16 rollout either source is rounded to IEEE binary16."""
+    if getattr(w, "dst_dtype", "bf16") == "f16":
+        return "f32->f16 (RNE)" if w.src_dtype == "f32" else "bf16->f16 (RNE)"
     return "f32->bf16 (RNE)" if w.src_dtype == "f32" else "bf16 (bit copy)"
 
 
@@ -543,7 +549,8 @@ class BenchStep:
         from synth import device as D
         self.rr, self.w, self.sync_verify = rr, w, sync_verify
         self.stream = stream if stream is not None else torch.cuda.current_stream()
-        m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
+        m, s, d = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep,
+                                dst_dtype=w.dst_dtype)
         self.manifest = m
         self.plan = plan = rr.rr_plan_create(m, s, d, bucket_bytes, opts)
         self.buf = buf = D.alloc(plan, poison=poison)
@@ -1208,6 +1215,8 @@ def main():
         vocab = args.vocab or w.shape.vocab
         w = w.with_(name=f"{w.name}-first{args.layers}layers-vocab{vocab}",
                     shape=dataclasses.replace(w.shape, layers=args.layers, vocab=vocab))
+    if args.dst_dtype != "bf16":
+        w = w.with_(name=f"{w.name}-{args.dst_dtype}", dst_dtype=args.dst_dtype)
     bucket_bytes = args.bucket_mib * (1 << 20) if args.bucket_mib else w.bucket_bytes
     world, rank, local = dist_setup(args)
     if args.impl == "reference":

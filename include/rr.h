@@ -162,12 +162,22 @@ typedef struct {
     const rr_block* blocks;
 } rr_dst_tensor;
 
+/* The rollout's 16-bit element type.  bfloat16 is the default (zero); a
+ * float16 rollout takes IEEE binary16 (Section 7.4 counts the transferred
+ * model as FP16): round to nearest, ties to even, subnormals kept, overflow to
+ * +-inf, and a NaN kept as a quiet NaN with its sign and top payload bits
+ * (sign | 0x7E00 | ((b >> 13) & 0x1FF) for float32 bits b).  A bfloat16
+ * source is widened exactly and rounded the same way. */
+typedef enum { RR_DST_BF16 = 0, RR_DST_F16 = 1 } rr_dst_dtype;
+
 /* Rollout side. */
 typedef struct {
     int32_t tp;                   /* number of destination ranks (tensor parallel)     */
     int32_t n_tensors;
     const rr_dst_tensor* tensors; /* order within a rank = order in its stream         */
     int64_t tensor_align_bytes;   /* power of two >= 2; 256 typical                    */
+    int32_t dtype;                /* rr_dst_dtype; 0 (bfloat16) by default             */
+    int32_t reserved;             /* 0                                                 */
 } rr_dst_layout;
 
 typedef struct rr_plan rr_plan;

@@ -209,6 +209,55 @@ __device__ __forceinline__ uint32_t cast2(uint32_t a, uint32_t b) {
 
 __device__ __forceinline__ uint16_t cast1(uint32_t a) { return uint16_t(round_hi(a) >> 16); }
 
+// float32 bits -> IEEE binary16 bits.  Numbers take the hardware conversion,
+// cvt.rn (round to nearest, ties to even; subnormals kept, overflow to +-inf);
+// a NaN is replaced by the quiet NaN that keeps its sign and top payload bits,
+// whatever NaN the conversion gives.
+__device__ __forceinline__ bool is_nan32(uint32_t x) { return (x & 0x7FFFFFFFu) > 0x7F800000u; }
+
+__device__ __forceinline__ uint32_t nan_f16(uint32_t x) {
+    return ((x >> 16) & 0x8000u) | 0x7E00u | ((x >> 13) & 0x01FFu);
+}
+
+// Two float32 -> two binary16 packed little-endian in one word (a low).
+__device__ __forceinline__ uint32_t cast2_f16(uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(__uint_as_float(b)), "f"(__uint_as_float(a)));
+    if (is_nan32(a)) r = (r & 0xFFFF0000u) | nan_f16(a);
+    if (is_nan32(b)) r = (r & 0x0000FFFFu) | (nan_f16(b) << 16);
+    return r;
+}
+
+__device__ __forceinline__ uint16_t cast1_f16(uint32_t a) {
+    uint16_t h;
+    asm("cvt.rn.f16.f32 %0, %1;" : "=h"(h) : "f"(__uint_as_float(a)));
+    return is_nan32(a) ? uint16_t(nan_f16(a)) : h;
+}
+
+// The destination element type of a pack: bfloat16 (F16 false: a float32
+// source is rounded, a bfloat16 one copied) or float16 (a bfloat16 source is
+// widened exactly, then rounded like a float32 one).
+template <bool F16>
+struct DstCast {
+    static __device__ __forceinline__ uint32_t f32x2(uint32_t a, uint32_t b) {
+        return F16 ? cast2_f16(a, b) : cast2(a, b);
+    }
+    static __device__ __forceinline__ uint16_t f32(uint32_t a) {
+        return F16 ? cast1_f16(a) : cast1(a);
+    }
+    // Two bfloat16 packed in a word.
+    static __device__ __forceinline__ uint32_t bf16x2(uint32_t w) {
+        return F16 ? cast2_f16(w << 16, w & 0xFFFF0000u) : w;
+    }
+    static __device__ __forceinline__ uint16_t bf16(uint16_t h) {
+        return F16 ? cast1_f16(uint32_t(h) << 16) : h;
+    }
+    static __device__ __forceinline__ uint4 bf16x8(uint4 v) {
+        if (!F16) return v;
+        return make_uint4(bf16x2(v.x), bf16x2(v.y), bf16x2(v.z), bf16x2(v.w));
+    }
+};
+
 __device__ __forceinline__ unsigned long long words(uint4 v) {
     return ((unsigned long long)v.y << 32 | v.x) + ((unsigned long long)v.w << 32 | v.z);
 }
@@ -326,9 +375,10 @@ __device__ __forceinline__ char* bucket_of(const PackArgs<NPTR>& a, uint32_t b) 
 // aligned source rows and destination.  One "vector" is 8 elements: 32 (fp32)
 // or 16 (bf16) source bytes, 16 destination bytes.  Thread t handles vectors
 // t, t + T, t + 2T, ...; (row, vector-in-row) is advanced incrementally.
-template <int ES>
+template <int ES, bool F16>
 __device__ __forceinline__ unsigned long long pack_vec(const char* src, char* dst,
                                                        const rr_pack_item& d) {
+    using D = DstCast<F16>;
     // A bf16 vector is one 16-byte load instead of two: twice as many of them
     // keep the same bytes in flight per thread.
     constexpr int U = ES == 4 ? kUnroll : 2 * kUnroll;
@@ -363,12 +413,12 @@ __device__ __forceinline__ unsigned long long pack_vec(const char* src, char* ds
             if (vv[u] < nvec) {
                 uint4 o;
                 if (ES == 4) {
-                    o.x = cast2(x[u][0].x, x[u][0].y);
-                    o.y = cast2(x[u][0].z, x[u][0].w);
-                    o.z = cast2(x[u][ES / 2 - 1].x, x[u][ES / 2 - 1].y);
-                    o.w = cast2(x[u][ES / 2 - 1].z, x[u][ES / 2 - 1].w);
+                    o.x = D::f32x2(x[u][0].x, x[u][0].y);
+                    o.y = D::f32x2(x[u][0].z, x[u][0].w);
+                    o.z = D::f32x2(x[u][ES / 2 - 1].x, x[u][ES / 2 - 1].y);
+                    o.w = D::f32x2(x[u][ES / 2 - 1].z, x[u][ES / 2 - 1].w);
                 } else {
-                    o = x[u][0];
+                    o = D::bf16x8(x[u][0]);
                 }
                 st_stream(dst + (uint64_t)vv[u] * 16, o);
                 acc += words(o);
@@ -385,8 +435,10 @@ __device__ __forceinline__ unsigned long long pack_vec(const char* src, char* ds
 // 8-element vector, loaded by two instructions) moves each sector twice: with
 // 8-element vectors the pack read pinned host memory at half the link's rate.
 // The destination is 16-byte aligned, so each store is one whole checksum word.
+template <bool F16>
 __device__ __forceinline__ unsigned long long pack_vec_f32_narrow(const char* src, char* dst,
                                                                   const rr_pack_item& d) {
+    using D = DstCast<F16>;
     constexpr int U = 2 * kUnroll;
     const uint32_t vpr = d.row_len >> 2;
     const uint32_t nvec = vpr * d.n_rows;
@@ -413,7 +465,7 @@ __device__ __forceinline__ unsigned long long pack_vec_f32_narrow(const char* sr
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             if (vv[u] < nvec) {
-                const uint32_t lo = cast2(x[u].x, x[u].y), hi = cast2(x[u].z, x[u].w);
+                const uint32_t lo = D::f32x2(x[u].x, x[u].y), hi = D::f32x2(x[u].z, x[u].w);
                 st_stream8(dst + (uint64_t)vv[u] * 8, lo, hi);
                 acc += (unsigned long long)hi << 32 | lo;
             }
@@ -425,9 +477,10 @@ __device__ __forceinline__ unsigned long long pack_vec_f32_narrow(const char* sr
 // Scalar item: any alignment and row length; one element per thread-step.
 // Each element's checksum contribution is its bits shifted to its byte
 // position within the 64-bit word it lands in.
-template <int ES>
+template <int ES, bool F16>
 __device__ __forceinline__ unsigned long long pack_scalar(const char* src, char* dst,
                                                           const rr_pack_item& d) {
+    using D = DstCast<F16>;
     const uint32_t L = d.row_len;
     const uint32_t n = L * d.n_rows;
     const uint64_t stride = (uint64_t)d.src_stride * ES;
@@ -439,9 +492,9 @@ __device__ __forceinline__ unsigned long long pack_scalar(const char* src, char*
         const char* p = src + r * stride + (uint64_t)c * ES;
         uint16_t h;
         if (ES == 4)
-            h = cast1(*(const uint32_t*)p);
+            h = D::f32(*(const uint32_t*)p);
         else
-            h = *(const uint16_t*)p;
+            h = D::bf16(*(const uint16_t*)p);
         *(uint16_t*)(dst + 2ull * e) = h;
         acc += (unsigned long long)h << (8 * ((d.dst_off + 2 * e) & 7));
         c += dr;
@@ -455,7 +508,8 @@ __device__ __forceinline__ unsigned long long pack_scalar(const char* src, char*
 }
 
 // HOST_SRC: the source is in host memory (fp32 vectors of 4 elements).
-template <int NPTR, bool CHECK, bool HOST_SRC>
+// F16: the rollout's elements are float16 (else bfloat16).
+template <int NPTR, bool CHECK, bool HOST_SRC, bool F16>
 __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(const __grid_constant__ PackArgs<NPTR> a) {
     uint32_t i0, i1;
     block_items(a.block_first, a.weight_prefix, a.item_begin, a.item_end, &i0, &i1);
@@ -477,11 +531,12 @@ __global__ void __launch_bounds__(kThreads, RR_PACK_MIN_BLOCKS) rr_pack_kernel(c
         const char* src = (const char*)a.ptr[d.src >> 48] + (d.src & 0xFFFFFFFFFFFFull);
         switch (d.kind) {
             case RR_ITEM_F32_VEC:
-                acc += HOST_SRC ? pack_vec_f32_narrow(src, dst, d) : pack_vec<4>(src, dst, d);
+                acc += HOST_SRC ? pack_vec_f32_narrow<F16>(src, dst, d)
+                                : pack_vec<4, F16>(src, dst, d);
                 break;
-            case RR_ITEM_BF16_VEC: acc += pack_vec<2>(src, dst, d); break;
-            case RR_ITEM_F32_SCALAR: acc += pack_scalar<4>(src, dst, d); break;
-            case RR_ITEM_BF16_SCALAR: acc += pack_scalar<2>(src, dst, d); break;
+            case RR_ITEM_BF16_VEC: acc += pack_vec<2, F16>(src, dst, d); break;
+            case RR_ITEM_F32_SCALAR: acc += pack_scalar<4, F16>(src, dst, d); break;
+            case RR_ITEM_BF16_SCALAR: acc += pack_scalar<2, F16>(src, dst, d); break;
             case RR_ITEM_ZERO_VEC:
                 for (uint32_t v = threadIdx.x; v < (d.row_len >> 3); v += kThreads)
                     st_stream(dst + 16ull * v, make_uint4(0, 0, 0, 0));
@@ -890,9 +945,12 @@ __device__ __forceinline__ char* bulk_bucket(const BulkArgs<NPTR>& a, uint32_t b
 }
 
 // MODE 0: pack, 1: unpack, 2: unpack with checksum comparison.  CHECK: check
-// every item against the plan's buffers first (the check_items option).
-template <int NPTR, int MODE, bool CHECK>
+// every item against the plan's buffers first (the check_items option).  F16
+// (pack only): the rollout's elements are float16, else bfloat16.
+template <int NPTR, int MODE, bool CHECK, bool F16>
 __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(const __grid_constant__ BulkArgs<NPTR> a) {
+    static_assert(MODE == 0 || !F16, "the destination type matters to the pack only");
+    using D = DstCast<F16>;
     constexpr int kConsumerWarps = BulkShape<MODE>::kWarps;
     constexpr int kStageBytes = BulkShape<MODE>::kStageBytes;
     constexpr int kStages = BulkShape<MODE>::kStages;
@@ -1245,10 +1303,10 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                     const uint4 x0 = *(const uint4*)(st + 32ull * v);
                     const uint4 x1 = *(const uint4*)(st + 32ull * v + 16);
                     uint4 o;
-                    o.x = cast2(x0.x, x0.y);
-                    o.y = cast2(x0.z, x0.w);
-                    o.z = cast2(x1.x, x1.y);
-                    o.w = cast2(x1.z, x1.w);
+                    o.x = D::f32x2(x0.x, x0.y);
+                    o.y = D::f32x2(x0.z, x0.w);
+                    o.z = D::f32x2(x1.x, x1.y);
+                    o.w = D::f32x2(x1.z, x1.w);
                     st_stream(p.dst + 16ull * v, o);
                     acc += words(o);
                 }
@@ -1257,7 +1315,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
             case PC_READ:
 #pragma unroll 4
                 for (uint32_t v = ct; v < nvec; v += kCT) {
-                    const uint4 x = *(const uint4*)(st + 16ull * v);
+                    const uint4 x = D::bf16x8(*(const uint4*)(st + 16ull * v));
                     if (p.kind == PC_COPY) st_stream(p.dst + 16ull * v, x);
                     if (kSum) acc += words(x);
                 }
@@ -1266,7 +1324,8 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                 for (uint32_t e = ct; e < p.n; e += kCT) {
                     const uint32_t r = e / p.row_len, cc = e - r * p.row_len;
                     const char* q = p.src + r * p.src_stride + (uint64_t)cc * p.es;
-                    const uint16_t h = p.es == 4 ? cast1(*(const uint32_t*)q) : *(const uint16_t*)q;
+                    const uint16_t h = p.es == 4 ? D::f32(*(const uint32_t*)q)
+                                                 : D::bf16(*(const uint16_t*)q);
                     if (p.dst) *(uint16_t*)(p.dst + 2ull * e) = h;
                     if (kSum) acc += (unsigned long long)h << (8 * ((p.sum_off + 2 * e) & 7));
                 }
@@ -1309,12 +1368,12 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1) rr_bulk_kernel(c
                             if (p.es == 4) {
                                 const uint4 x0 = *(const uint4*)q8;
                                 const uint4 x1 = *(const uint4*)(q8 + 16);
-                                o.x = cast2(x0.x, x0.y);
-                                o.y = cast2(x0.z, x0.w);
-                                o.z = cast2(x1.x, x1.y);
-                                o.w = cast2(x1.z, x1.w);
+                                o.x = D::f32x2(x0.x, x0.y);
+                                o.y = D::f32x2(x0.z, x0.w);
+                                o.z = D::f32x2(x1.x, x1.y);
+                                o.w = D::f32x2(x1.z, x1.w);
                             } else {
-                                o = *(const uint4*)q8;
+                                o = D::bf16x8(*(const uint4*)q8);
                             }
                             st_stream(out + 16ull * v, o);
                             am += words(o);
@@ -1405,9 +1464,9 @@ __global__ void rr_wait_selftest_kernel(unsigned int* err) {
     if (threadIdx.x == 0) mbar_wait(smem_u32(&bar), 0, err);
 }
 
-template <int NPTR, int MODE, bool CHECK = false>
+template <int NPTR, int MODE, bool CHECK = false, bool F16 = false>
 cudaError_t bulk_prepare() {
-    return cudaFuncSetAttribute(rr_bulk_kernel<NPTR, MODE, CHECK>,
+    return cudaFuncSetAttribute(rr_bulk_kernel<NPTR, MODE, CHECK, F16>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 BulkShape<MODE>::kSmem);
 }
@@ -1542,6 +1601,20 @@ int32_t take_claim_slot(rr_plan* M, cudaStream_t s);
 template <int MODE>
 void work_units(const rr_plan* P, const Range& R, const uint32_t** first, uint32_t* n);
 
+// The register-path pack instantiation for a launch: item checks, a source in
+// host memory, and the destination type.
+template <int NPTR, bool F16>
+void pack_kernel_for(bool check, bool host_src, int g, cudaStream_t s, const PackArgs<NPTR>& a) {
+    if (check && host_src)
+        rr_pack_kernel<NPTR, true, true, F16><<<g, kThreads, 0, s>>>(a);
+    else if (check)
+        rr_pack_kernel<NPTR, true, false, F16><<<g, kThreads, 0, s>>>(a);
+    else if (host_src)
+        rr_pack_kernel<NPTR, false, true, F16><<<g, kThreads, 0, s>>>(a);
+    else
+        rr_pack_kernel<NPTR, false, false, F16><<<g, kThreads, 0, s>>>(a);
+}
+
 template <int NPTR>
 rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* const* buckets,
                       uint64_t* checksums, bool table, uint64_t stride, bool host_src,
@@ -1564,15 +1637,10 @@ rr_status launch_pack(const rr_plan* P, Range R, const void* const* src, void* c
         a.bucket_base = (char*)buckets[0];
         a.bucket_stride = stride;
     }
-    const int g = P->reg_pack_grid;
-    if (P->check_items && host_src)
-        rr_pack_kernel<NPTR, true, true><<<g, kThreads, 0, s>>>(a);
-    else if (P->check_items)
-        rr_pack_kernel<NPTR, true, false><<<g, kThreads, 0, s>>>(a);
-    else if (host_src)
-        rr_pack_kernel<NPTR, false, true><<<g, kThreads, 0, s>>>(a);
+    if (P->dst_f16)
+        pack_kernel_for<NPTR, true>(P->check_items != 0, host_src, P->reg_pack_grid, s, a);
     else
-        rr_pack_kernel<NPTR, false, false><<<g, kThreads, 0, s>>>(a);
+        pack_kernel_for<NPTR, false>(P->check_items != 0, host_src, P->reg_pack_grid, s, a);
     RR_CUDA(cudaGetLastError());
     return RR_OK;
 }
@@ -1764,9 +1832,9 @@ struct BulkOpts {
     long long* result = nullptr;          // verifying unpack: write {n_bad, first_bad} here
 };
 
-template <int NPTR, int MODE, bool CHECK>
+template <int NPTR, int MODE, bool CHECK, bool F16>
 cudaError_t launch_bulk_kernel(int32_t grid, cudaStream_t s, const BulkArgs<NPTR>& a) {
-    cudaError_t e = bulk_prepare<NPTR, MODE, CHECK>();
+    cudaError_t e = bulk_prepare<NPTR, MODE, CHECK, F16>();
     if (e != cudaSuccess) return e;
     // Programmatic dependent launch: this grid's blocks may be scheduled while
     // the previous kernel on the stream drains (they wait for it to complete
@@ -1781,7 +1849,7 @@ cudaError_t launch_bulk_kernel(int32_t grid, cudaStream_t s, const BulkArgs<NPTR
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, rr_bulk_kernel<NPTR, MODE, CHECK>, a);
+    return cudaLaunchKernelEx(&cfg, rr_bulk_kernel<NPTR, MODE, CHECK, F16>, a);
 }
 
 template <int NPTR, int MODE>
@@ -1873,8 +1941,14 @@ rr_status launch_bulk(const rr_plan* P, Range R, const void* const* src_shards,
         a.expected = (const unsigned long long*)checksums;
         a.result = o.result;
     }
-    const cudaError_t e = P->check_items ? launch_bulk_kernel<NPTR, MODE, true>(grid, s, a)
-                                         : launch_bulk_kernel<NPTR, MODE, false>(grid, s, a);
+    // The float16 instantiations exist for the pack only (F16 = MODE == 0 there).
+    constexpr bool kF16 = MODE == 0;
+    const cudaError_t e =
+        MODE == 0 && P->dst_f16
+            ? (P->check_items ? launch_bulk_kernel<NPTR, MODE, true, kF16>(grid, s, a)
+                              : launch_bulk_kernel<NPTR, MODE, false, kF16>(grid, s, a))
+            : (P->check_items ? launch_bulk_kernel<NPTR, MODE, true, false>(grid, s, a)
+                              : launch_bulk_kernel<NPTR, MODE, false, false>(grid, s, a));
     if (e != cudaSuccess) return cuda_fail(e, "bulk kernel launch");
     cudaError_t er;
     if (slot >= 0 && (er = cudaEventRecord(P->claim_done[slot], s)) != cudaSuccess) {
@@ -2215,7 +2289,7 @@ rr_status rr_device_default_grid(rr_grids* g) {
     int dev = 0, sms = 0, p = 0, u = 0, vu = 0, v = 0, b = 0;
     RR_CUDA(cudaGetDevice(&dev));
     RR_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs, false, false>, kThreads, 0));
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&p, rr_pack_kernel<kLargePtrs, false, false, false>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&u, rr_unpack_kernel<kLargePtrs, false, false>, kThreads, 0));
     RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
         &vu, rr_unpack_kernel<kLargePtrs, true, false>, RegUnpackShape<true>::kBlock, 0));
@@ -2223,10 +2297,10 @@ rr_status rr_device_default_grid(rr_grids* g) {
     int bp = 0;
     RR_CUDA((bulk_prepare<kLargePtrs, 0>()));
     RR_CUDA((bulk_prepare<kLargePtrs, 2>()));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bp, rr_bulk_kernel<kLargePtrs, 0, false>,
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bp, rr_bulk_kernel<kLargePtrs, 0, false, false>,
                                                           BulkShape<0>::kThreads,
                                                           BulkShape<0>::kSmem));
-    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, rr_bulk_kernel<kLargePtrs, 2, false>,
+    RR_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, rr_bulk_kernel<kLargePtrs, 2, false, false>,
                                                           BulkShape<2>::kThreads,
                                                           BulkShape<2>::kSmem));
     g->reg_pack = sms * (p > 0 ? p : 1);

@@ -56,6 +56,7 @@ struct rr_plan {
     int32_t reg_unpack_grid = 0;
     int32_t reg_vunpack_grid = 0;     // the register path's verifying unpack (its own block size)
     int32_t engine = RR_ENGINE_AUTO;
+    int32_t dst_f16 = 0;              // the rollout's elements are float16 (else bfloat16)
     int64_t chunk_bytes = 0;
     bool host_only = false;
     std::vector<rr_pack_item> pack_items;

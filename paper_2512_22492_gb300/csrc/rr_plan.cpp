@@ -515,6 +515,8 @@ rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_
         return rr_fail(RR_EINVAL, "bad destination tensor list");
     if (!is_pow2(dst->tensor_align_bytes) || dst->tensor_align_bytes < 2)
         return rr_fail(RR_EINVAL, "tensor_align_bytes must be a power of two >= 2");
+    if (dst->dtype != RR_DST_BF16 && dst->dtype != RR_DST_F16)
+        return rr_fail(RR_EINVAL, "unknown destination dtype %d", dst->dtype);
 
     P->n_params = n_params;
     P->rows.resize(n_params);
@@ -639,6 +641,7 @@ rr_status validate_and_describe(rr_plan* P, const rr_param* manifest, int32_t n_
     if (P->shard_bytes > kMaxShardOffset) return rr_fail(RR_ELAYOUT, "shards too large");
 
     // Destination streams.
+    P->dst_f16 = dst->dtype == RR_DST_F16 ? 1 : 0;
     P->tp = dst->tp;
     P->n_tensors = dst->n_tensors;
     P->tensor_align = dst->tensor_align_bytes;

@@ -178,15 +178,18 @@ def qwen3_rollout(shape, manifest: List[Param], tp: int = 1,
 
 
 def qwen3_sync(shape, dtype: str, n_shards: int, tp: int, sharding: str = "flat",
-               ep: bool = False):
+               ep: bool = False, dst_dtype: str = "bf16"):
     """(manifest, source layout, destination layout) for one Qwen3 weight sync.
     sharding: "flat" (one FSDP1 FlatParameter cut evenly), "rows" (FSDP2:
     every parameter cut on dim 0) or "units" (FSDP1 wrapping every decoder
-    layer); ep: expert-parallel rollout."""
+    layer); ep: expert-parallel rollout; dst_dtype: the rollout's 16-bit
+    element type, "bf16" or "f16"."""
     manifest = qwen3_manifest(shape, dtype)
     units = qwen3_layer_units(manifest) if sharding == "units" else None
     src = SrcLayout(n_shards=n_shards, align_bytes=16, sharding=sharding, units=units)
-    return manifest, src, qwen3_rollout(shape, manifest, tp, ep=ep)
+    dst = qwen3_rollout(shape, manifest, tp, ep=ep)
+    dst.dtype = dst_dtype
+    return manifest, src, dst
 
 
 # ---------------------------------------------------------------------------

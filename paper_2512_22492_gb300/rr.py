@@ -58,7 +58,11 @@ class _DstTensor(ctypes.Structure):
 
 class _DstLayout(ctypes.Structure):
     _fields_ = [("tp", ctypes.c_int32), ("n_tensors", ctypes.c_int32),
-                ("tensors", ctypes.POINTER(_DstTensor)), ("tensor_align_bytes", ctypes.c_int64)]
+                ("tensors", ctypes.POINTER(_DstTensor)), ("tensor_align_bytes", ctypes.c_int64),
+                ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+_DST_DTYPES = {"bf16": 0, "f16": 1}
 
 
 class _Options(ctypes.Structure):
@@ -234,6 +238,7 @@ class DstLayout:
     tp: int
     tensors: List[DstTensor]
     tensor_align_bytes: int = 256
+    dtype: str = "bf16"      # the rollout's 16-bit element type: "bf16" or "f16"
 
 
 @dataclass
@@ -255,6 +260,7 @@ class Plan:
     def __init__(self, handle: int, n_params: int, dst: DstLayout, src: SrcLayout = None):
         self._h = ctypes.c_void_p(handle)
         self.n_params = n_params
+        self.dst_dtype = dst.dtype
         self.sharding = src.sharding if src else "flat"
         self.align_bytes = src.align_bytes if src else 16
         self.tp = dst.tp
@@ -419,9 +425,12 @@ def rr_plan_create(manifest: Sequence[Param], src: SrcLayout, dst: DstLayout,
         ct[i].numel = t.size()
         ct[i].n_blocks = len(t.blocks)
         ct[i].blocks = ctypes.cast(cb, ctypes.POINTER(_Block))
+    if dst.dtype not in _DST_DTYPES:
+        raise ValueError(f"destination dtype must be one of {sorted(_DST_DTYPES)}, "
+                         f"not {dst.dtype!r}")
     cd = _DstLayout(tp=dst.tp, n_tensors=len(dst.tensors),
                     tensors=ctypes.cast(ct, ctypes.POINTER(_DstTensor)),
-                    tensor_align_bytes=dst.tensor_align_bytes)
+                    tensor_align_bytes=dst.tensor_align_bytes, dtype=_DST_DTYPES[dst.dtype])
     out = ctypes.c_void_p()
     if options is None:
         st = _lib.rr_plan_create(cp, n, ctypes.byref(cs), ctypes.byref(cd), bucket_bytes,

@@ -129,8 +129,10 @@ def degenerate_layout(sharding: str = "flat"):
     return desc
 
 
-def workload_desc(name, bucket_bytes=None):
+def workload_desc(name, bucket_bytes=None, dst_dtype=None):
     w = workload(name)
+    if dst_dtype is not None:
+        w = w.with_(dst_dtype=dst_dtype)
     from oracle import qwen3
     params = qwen3.manifest(w.shape, w.src_elem_bytes)
     return dict(params=params, tensors=None, workload=w, tp=w.tp, n_shards=w.n_shards,
@@ -144,20 +146,23 @@ def to_oracle(desc) -> "oracle.Layout":
     return oracle.Layout(desc["params"], desc["tensors"], n_shards=desc["n_shards"],
                          tp=desc["tp"], bucket_bytes=desc["bucket_bytes"],
                          align_bytes=desc["align_bytes"], tensor_align=desc["tensor_align"],
-                         sharding=desc.get("sharding", "flat"), units=desc.get("units"))
+                         sharding=desc.get("sharding", "flat"), units=desc.get("units"),
+                         dst_dtype=desc.get("dst_dtype", "bf16"))
 
 
 def to_product(desc):
     import paper_2512_22492_gb300 as rr
     if desc.get("workload") is not None:
         w = desc["workload"]
-        return rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep)
+        return rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep,
+                             dst_dtype=w.dst_dtype)
     manifest = [rr.Param(n, d, "f32" if es == 4 else "bf16") for n, d, es in desc["params"]]
     src = rr.SrcLayout(n_shards=desc["n_shards"], align_bytes=desc["align_bytes"],
                        sharding=desc.get("sharding", "flat"), units=desc.get("units"))
     dst = rr.DstLayout(tp=desc["tp"], tensor_align_bytes=desc["tensor_align"],
                        tensors=[rr.DstTensor(n, r, [rr.Block(*b) for b in blocks])
-                                for n, r, blocks in desc["tensors"]])
+                                for n, r, blocks in desc["tensors"]],
+                       dtype=desc.get("dst_dtype", "bf16"))
     return manifest, src, dst
 
 

@@ -96,7 +96,7 @@ int main(int argc, char** argv) {
     rr_block blocks[4] = {{0, 0, 4, 0, 8}, {1, 0, 8, 0, 1}, {0, 0, 4, 8, 8}, {1, 0, 8, 0, 1}};
     rr_dst_tensor tensors[4] = {{"a", 0, 32, 1, &blocks[0]}, {"b", 0, 8, 1, &blocks[1]},
                                 {"a", 1, 32, 1, &blocks[2]}, {"b", 1, 8, 1, &blocks[3]}};
-    rr_dst_layout dst = {2, 4, tensors, 256};
+    rr_dst_layout dst = {2, 4, tensors, 256, RR_DST_BF16, 0};
     rr_plan_options opt;
     memset(&opt, 0, sizeof opt);
     opt.host_only = !gpu;
@@ -109,9 +109,12 @@ int main(int argc, char** argv) {
           "error text");
     rr_block off_end = {0, 3, 2, 0, 8};
     rr_dst_tensor t_bad = {"x", 0, 16, 1, &off_end};
-    rr_dst_layout d_bad = {1, 1, &t_bad, 256};
+    rr_dst_layout d_bad = {1, 1, &t_bad, 256, RR_DST_BF16, 0};
     CHECK(rr_plan_create_ex(man, 2, &src, &d_bad, 128, &opt, &bad) == RR_ELAYOUT,
           "rows past the parameter refused");
+    rr_dst_layout d_type = {2, 4, tensors, 256, 7, 0};
+    CHECK(rr_plan_create_ex(man, 2, &src, &d_type, 128, &opt, &bad) == RR_EINVAL,
+          "unknown destination dtype refused");
 
     rr_plan* plan = NULL;
     CHECK(rr_plan_create_ex(man, 2, &src, &dst, BUCKET, &opt, &plan) == RR_OK, "plan");

@@ -1,4 +1,5 @@
-"""Every float32 bit pattern through the pack kernels, against the oracle's cast.
+"""Every float32 bit pattern through the pack kernels, against the oracle's cast
+(to bfloat16, and to float16 for a float16 rollout).
 
 The source is one fp32 parameter of 2^32 elements ([65536, 65536], 16 GiB)
 whose element i holds the bit pattern i, in 7 flat shards (so shard cuts fall
@@ -49,10 +50,12 @@ def plan_of(desc, **opts):
     return H.make_plan(m, s, d, desc["bucket_bytes"], **opts)
 
 
-def test_every_float32_pattern():
+@pytest.mark.parametrize("dst", ["bf16", "f16"])
+def test_every_float32_pattern(dst):
     desc = dict(params=[("w", (65536, 65536), 4)], tensors=[("w", 0, [(0, 0, 65536, 0, 65536)])],
                 tp=1, sharding="flat", n_shards=7, bucket_bytes=BUCKET, align_bytes=16,
-                tensor_align=256, seed=1, specials=False)
+                tensor_align=256, seed=1, specials=False, dst_dtype=dst)
+    cast = oracle.rne_f16 if dst == "f16" else oracle.rne_bf16
     auto = plan_of(desc)
     regs = plan_of(desc, engine="registers")
     assert auto.n_buckets == regs.n_buckets == N * 2 // BUCKET
@@ -79,7 +82,7 @@ def test_every_float32_pattern():
 
     def one(c):
         pats = np.arange(CHUNK, dtype=np.uint32) + np.uint32(c * CHUNK)
-        want = oracle.rne_bf16(pats).view(np.uint8)
+        want = cast(pats).view(np.uint8)
         b, off = divmod(c * CHUNK * 2, BUCKET)
         for name, buf in runs.items():
             got = buf.bucket_store[b, off:off + CHUNK * 2].cpu().numpy()
@@ -99,13 +102,15 @@ def test_every_float32_pattern():
         np.testing.assert_array_equal(H.checksums_host(buf), want_cs, err_msg=name)
 
 
+@pytest.mark.parametrize("dst", ["bf16", "f16"])
 @pytest.mark.parametrize("where", ["bulk", "registers", "host source"])
-def test_every_bfloat16_pattern(where):
-    """bf16 -> bf16 is a bit copy, NaN payloads included: all 2^16 patterns, in
-    3 flat shards and 8 KiB buckets, against the oracle's pack."""
+def test_every_bfloat16_pattern(where, dst):
+    """bf16 -> bf16 is a bit copy, NaN payloads included; bf16 -> f16 widens and
+    rounds: all 2^16 patterns, in 3 flat shards and 8 KiB buckets, against the
+    oracle's pack."""
     desc = dict(params=[("v", (256, 256), 2)], tensors=[("v", 0, [(0, 0, 256, 0, 256)])],
                 tp=1, sharding="flat", n_shards=3, bucket_bytes=8192, align_bytes=16,
-                tensor_align=256, seed=1, specials=False)
+                tensor_align=256, seed=1, specials=False, dst_dtype=dst)
     plan = plan_of(desc, engine="registers" if where == "registers" else "auto")
     L = U.to_oracle(desc)
     starts = H.source_offsets(plan)
@@ -122,5 +127,9 @@ def test_every_bfloat16_pattern(where):
     want, want_cs = L.pack(oracle.Source(shards=shards))
     np.testing.assert_array_equal(H.buckets_host(buf), want)
     np.testing.assert_array_equal(H.checksums_host(buf), want_cs)
-    np.testing.assert_array_equal(want.reshape(-1)[:1 << 17].view(np.uint16),
-                                  np.arange(1 << 16, dtype=np.uint16))
+    stream = want.reshape(-1)[:1 << 17].view(np.uint16)
+    patterns = np.arange(1 << 16, dtype=np.uint32)
+    if dst == "bf16":
+        np.testing.assert_array_equal(stream, patterns.astype(np.uint16))
+    else:
+        np.testing.assert_array_equal(stream, oracle.rne_f16(patterns << 16))
