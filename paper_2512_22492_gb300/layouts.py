@@ -285,7 +285,11 @@ def qwen3_relay(shape, src_tp: int, dst_tp: int, from_plan=None, src_ep: bool = 
     tensor, in the order of the TP=src_tp rollout layout).  from_plan=<the
     plan that packed the image>: it re-packs straight from the buckets it
     pulled (the buckets, in order, are the shards; bucket_bytes must be a
-    multiple of 16)."""
+    multiple of 16).
+
+    A relay copies 16-bit elements bit for bit, so the same layout serves a
+    bfloat16 and a float16 image alike: its manifest reads the elements as
+    bf16 and its destination keeps the default type (no cast)."""
     logical = qwen3_manifest(shape, "bf16")
     src = qwen3_rollout(shape, logical, src_tp, ep=src_ep)
     params, _ = rollout_as_source(src)
