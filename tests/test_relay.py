@@ -22,7 +22,11 @@ PAIRS = [(4, 4), (4, 2), (2, 4), (4, 1), (1, 4), (2, 1)]
 
 def trainer_image(name, src_tp, src_ep=False):
     """The oracle's trainer source, its TP=src_tp rollout tensors and buckets."""
-    w = U.workload(name).with_(tp=src_tp, ep=src_ep)
+    return trainer_image_of(U.workload(name), src_tp, src_ep)
+
+
+def trainer_image_of(w, src_tp, src_ep=False):
+    w = w.with_(tp=src_tp, ep=src_ep)
     L = oracle.workload_layout(w)
     src = oracle.Source(shards=L.host_shards(w.seed, w.specials))
     tensors = [L.reshard_tensor(src, t) for t in range(len(L.tensors))]
@@ -138,3 +142,27 @@ def test_relay_expert_parallel_on_gpu(src_tp, src_ep, dst_tp, dst_ep):
     torch.cuda.synchronize()
     np.testing.assert_array_equal(out.cpu().numpy(), want)
     np.testing.assert_array_equal(cs.cpu().numpy().view(np.uint64), want_cs)
+
+
+@pytest.mark.parametrize("src_tp,dst_tp", [(4, 2), (1, 4)])
+def test_relay_of_a_float16_image(src_tp, dst_tp):
+    """A float16 rollout relays like a bf16 one: the relay copies the 16-bit
+    elements, so re-packing the TP=src_tp float16 image (from its tensors and
+    from its buckets) gives the oracle's float16 pack of the TP=dst_tp layout."""
+    w0 = U.workload("tiny-moe-f32").with_(dst_dtype="f16")
+    w, src, tensors, buckets = trainer_image_of(w0, src_tp)
+    B = 16 * 1024
+    want, _ = expected(w, src, dst_tp, B)
+    m, s, d = layouts.qwen3_relay(w.shape, src_tp, dst_tp)
+    plan = rr.rr_plan_create(m, s, d, B, rr.PlanOptions(host_only=True))
+    items, _ = plan.export_pack()
+    got = U.check_and_run_pack(items, [t.view(np.uint8) for t in tensors], plan.n_buckets, B,
+                               plan.shard_bytes)
+    np.testing.assert_array_equal(got, want)
+    m0, s0, d0 = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, src_tp, dst_dtype="f16")
+    src_plan = rr.rr_plan_create(m0, s0, d0, w.bucket_bytes, rr.PlanOptions(host_only=True))
+    m, s, d = layouts.qwen3_relay(w.shape, src_tp, dst_tp, from_plan=src_plan)
+    plan = rr.rr_plan_create(m, s, d, B, rr.PlanOptions(host_only=True))
+    items, _ = plan.export_pack()
+    got = U.check_and_run_pack(items, [b for b in buckets], plan.n_buckets, B, plan.shard_bytes)
+    np.testing.assert_array_equal(got, want)
