@@ -7,7 +7,8 @@ against the oracle bit for bit.
   patterns (widened, then rounded), TP=4, FSDP2 rows, KV replication, per-layer
   units, expert parallel;
 * random ragged layouts and random row-parallel layouts (the fan-out groups);
-* the pack from pinned host memory;
+* the pack from pinned host memory; bucket ranges into separately allocated
+  buckets;
 * full-size Qwen3-8B and Qwen3-30B-A3B: sampled buckets against the oracle,
   every checksum against torch's word sum, sampled tensors against the
   oracle's reshard.
@@ -96,9 +97,9 @@ def test_item_checks_f16():
 
 
 def test_a_bf16_plan_and_an_f16_plan_differ_only_in_the_cast():
-    """Same layout, both element types: identical geometry, and every bucket
-    element of the f16 plan is the f16 rounding of what the bf16 plan's source
-    element was (checked through the oracle on the same shards)."""
+    """Same layout, both element types: the same buckets, stream offsets,
+    tensor sizes and algorithmic bytes (the element values are checked against
+    the oracle by the tests above)."""
     desc = U.workload_desc("tiny-tp4")
     m, s, d = U.to_product(desc)
     m2, s2, d2 = U.to_product(f16(desc))
@@ -139,3 +140,24 @@ def test_full_size_f16_sampled(name, names):
                                       err_msg=nm)
     buf = None
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("engine", ["auto", "registers"])
+def test_ranges_and_separate_buckets_f16(engine):
+    """rr_pack_range over three ranges (last first) into separately allocated
+    buckets (the pointer-table launch shape), float16 destination."""
+    desc = f16(U.workload_desc("tiny-tp4"))
+    L = U.to_oracle(desc)
+    m, s, d = U.to_product(desc)
+    plan = H.make_plan(m, s, d, desc["bucket_bytes"], engine=engine)
+    shards = L.host_shards(desc["seed"], desc["specials"])
+    buf = H.alloc(plan, separate_buckets=True, with_dst=False)
+    H.fill_from_host(buf, shards)
+    n = plan.n_buckets
+    cuts = [0, n // 3, 2 * n // 3, n]
+    for a, b in reversed(list(zip(cuts[:-1], cuts[1:]))):
+        rr.rr_pack_range(plan, a, b - a, buf.shards, buf.buckets, buf.checksums)
+    torch.cuda.synchronize()
+    want, want_cs = L.pack(oracle.Source(shards=shards))
+    np.testing.assert_array_equal(H.buckets_host(buf), want)
+    np.testing.assert_array_equal(H.checksums_host(buf), want_cs)
