@@ -219,10 +219,17 @@ __device__ __forceinline__ uint32_t nan_f16(uint32_t x) {
     return ((x >> 16) & 0x8000u) | 0x7E00u | ((x >> 13) & 0x01FFu);
 }
 
-// Two float32 -> two binary16 packed little-endian in one word (a low).
-__device__ __forceinline__ uint32_t cast2_f16(uint32_t a, uint32_t b) {
+// Two float32 -> two binary16 packed little-endian in one word (a low), by the
+// conversion alone (numbers only).
+__device__ __forceinline__ uint32_t cvt_f16x2(uint32_t a, uint32_t b) {
     uint32_t r;
     asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(__uint_as_float(b)), "f"(__uint_as_float(a)));
+    return r;
+}
+
+// The same with NaNs replaced by the stated rule.
+__device__ __forceinline__ uint32_t cast2_f16(uint32_t a, uint32_t b) {
+    uint32_t r = cvt_f16x2(a, b);
     if (is_nan32(a)) r = (r & 0xFFFF0000u) | nan_f16(a);
     if (is_nan32(b)) r = (r & 0x0000FFFFu) | (nan_f16(b) << 16);
     return r;
@@ -254,7 +261,16 @@ struct DstCast {
     }
     static __device__ __forceinline__ uint4 bf16x8(uint4 v) {
         if (!F16) return v;
-        return make_uint4(bf16x2(v.x), bf16x2(v.y), bf16x2(v.z), bf16x2(v.w));
+        // One test for the eight elements: a bfloat16 is a NaN when its
+        // magnitude exceeds 0x7F80.  Without one, the conversions need no patch.
+        const uint32_t m = __vmaxu2(__vmaxu2(v.x & 0x7FFF7FFFu, v.y & 0x7FFF7FFFu),
+                                    __vmaxu2(v.z & 0x7FFF7FFFu, v.w & 0x7FFF7FFFu));
+        if (__vcmpgtu2(m, 0x7F807F80u) != 0)
+            return make_uint4(bf16x2(v.x), bf16x2(v.y), bf16x2(v.z), bf16x2(v.w));
+        return make_uint4(cvt_f16x2(v.x << 16, v.x & 0xFFFF0000u),
+                          cvt_f16x2(v.y << 16, v.y & 0xFFFF0000u),
+                          cvt_f16x2(v.z << 16, v.z & 0xFFFF0000u),
+                          cvt_f16x2(v.w << 16, v.w & 0xFFFF0000u));
     }
 };
 
