@@ -22,7 +22,7 @@
  *   (5) unpack: buckets back to the rollout's tensors; (6) verify.
  *
  * The paper prints no layout, byte format or checksum; the definitions below
- * are the readings this build takes, stated once here:
+ * are the readings taken here, stated once:
  *
  *  Source, flat sharding (FSDP1-style).  Parameters are concatenated in
  *  manifest order into one flat byte buffer; each starts at a multiple of

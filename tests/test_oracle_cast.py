@@ -1,7 +1,7 @@
 """Pins for the oracle's float32 -> bfloat16 round-to-nearest-even cast.
 
 The cast itself is implied by the paper (Section 7.4: the rollout holds
-16-bit weights); the rounding mode and the NaN rule are this build's reading.
+16-bit weights); the rounding mode and the NaN rule are the reading taken here.
 The oracle uses a bit trick; these tests check it against things other than
 that trick:
 
