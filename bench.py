@@ -185,7 +185,7 @@ class ClockSampler:
 
     @staticmethod
     def _when(stamp: str):
-        try:   # "2026/12/02 09:48:40.123", the box's local time
+        try:   # "2026/12/02 09:48:40.123", the host's local time
             day, frac = (stamp.split(".") + ["0"])[:2]
             return time.mktime(time.strptime(day, "%Y/%m/%d %H:%M:%S")) + float("0." + frac)
         except (ValueError, OverflowError):
@@ -1079,7 +1079,7 @@ def run_native(args, w, bucket_bytes, world, rank, local):
         # Two routes for the source, both through the public API and both timed:
         # copy engines (the source copied into HBM in pieces, each piece packed
         # as it lands) and direct (the pack reads the pinned shards itself).
-        # Which is faster depends on the box: where the copy engines run below
+        # Which is faster depends on the machine: where the copy engines run below
         # the link, the SMs' own loads still reach it.  The line reports the
         # faster and carries both.
         host_src = torch.empty(buf.flat.numel(), dtype=torch.uint8, pin_memory=True)

@@ -200,7 +200,7 @@ typedef struct {
                             bucket and tensor sizes of the plan before touching
                             memory; an item outside them is skipped and marks the
                             plan's error word (rr_plan_check then reports RR_ECUDA).
-                            A debugging aid in place of a memory checker; costs a
+                            A debugging aid in place of a memory-checking tool; costs a
                             little producer time                                    */
 } rr_plan_options;
 
