@@ -353,3 +353,40 @@ def test_bucket_index_and_range_interpretation(seed):
     got = U.check_and_run_pack(sub, shards, b1 - b0, p.bucket_bytes, p.shard_bytes)
     want, _ = L.pack(oracle.Source(shards=shards), first=b0, count=b1 - b0)
     np.testing.assert_array_equal(got, want)
+
+
+@pytest.mark.parametrize("case", ["tiny-tp4", "tiny-moe-bf16-specials", "qwen3-8b-fsdp2-tp8",
+                                  "random-3", "row-parallel-5"])
+def test_float16_rollout_changes_only_the_cast(case):
+    """A float16 destination is the same plan as a bf16 one but for the cast the
+    kernels apply: every work table, per-block range, work unit and count is
+    identical."""
+    if case.startswith("random-"):
+        desc = U.random_layout(int(case.split("-")[1]))
+    elif case.startswith("row-parallel-"):
+        desc = U.random_tp_layout(int(case.split("-")[2]))
+    else:
+        desc = U.workload_desc(case)
+    plans = []
+    for dtype in ("bf16", "f16"):
+        d16 = dict(desc)
+        if d16.get("workload") is not None:
+            d16["workload"] = d16["workload"].with_(dst_dtype=dtype)
+        else:
+            d16["dst_dtype"] = dtype
+        m, s, d = U.to_product(d16)
+        assert d.dtype == dtype
+        plans.append(rr.rr_plan_create(m, s, d, desc["bucket_bytes"],
+                                       rr.PlanOptions(host_only=True)))
+    a, b = plans
+    assert a.dst_dtype == "bf16" and b.dst_dtype == "f16"
+    assert a.stats() == b.stats()
+    for export in ("export_pack", "export_pack_full", "export_unpack"):
+        ia, fa = getattr(a, export)()
+        ib, fb = getattr(b, export)()
+        np.testing.assert_array_equal(ia, ib, err_msg=export)
+        np.testing.assert_array_equal(fa, fb, err_msg=export)
+    for which in ("pack", "unpack", "pack_full"):
+        ua, ub = a.work_units(which), b.work_units(which)
+        for x, y in zip(ua, ub):
+            np.testing.assert_array_equal(x, y, err_msg=which)
