@@ -475,9 +475,10 @@ def _event_ms(fn, stream, reps=3):
 
 def next_rows(rr, H, w, plan, buf, t_src, t_bkt, t_dst, stream, peak):
     """Timings of the paths beyond the step: a resumed pull (the middle third of
-    the buckets packed and checked-unpacked again, Section 5.2.2) and a relay
+    the buckets packed and checked-unpacked again, Section 5.2.2), a relay
     re-pack (a rollout holding the TP=1 image serves a TP=4 one straight from
-    the buckets it pulled, Section 5.2.1).  Algorithmic bytes as for the step."""
+    the buckets it pulled, Section 5.2.1), and the pack for a float16 rollout.
+    Algorithmic bytes as for the step."""
     import numpy as np
     import torch
     out = {}
@@ -527,6 +528,28 @@ def next_rows(rr, H, w, plan, buf, t_src, t_bkt, t_dst, stream, peak):
                                           "bytes": nbytes, "GB/s": round(gbs, 1),
                                           "frac_of_peak": round(gbs / peak, 4)}
         del store, cs, r_src, relay
+    if getattr(w, "dst_dtype", "bf16") == "bf16":
+        # The same sync for a float16 rollout (Section 7.4 counts the transferred
+        # model as FP16): the same tables and bytes, the float16 cast.  Its pack
+        # overwrites the step's buckets, which nothing reads after this.
+        m2, s2, d2 = rr.qwen3_sync(w.shape, w.src_dtype, w.n_shards, w.tp, w.sharding, ep=w.ep,
+                                   dst_dtype="f16")
+        p16 = rr.rr_plan_create(m2, s2, d2, plan.bucket_bytes)
+        cs16 = torch.zeros_like(buf.checksums)
+        t16_src = rr.Pointers(p16, "src_shards", buf.shards)
+        t16_bkt = rr.Pointers(p16, "buckets", buf.buckets)
+        ms = _event_ms(lambda: rr.rr_pack(p16, t16_src, t16_bkt, cs16, stream), stream)
+        n_bad, _ = rr.rr_verify(p16, t16_bkt, cs16, stream)
+        if n_bad:
+            raise RuntimeError("float16 pack: its buckets do not match its checksums")
+        st16 = p16.stats()
+        nbytes = st16["pack_bytes_read"] + st16["pack_bytes_written"]
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        out["float16_rollout_pack"] = {"dtype": "f32->f16 (RNE)" if w.src_dtype == "f32"
+                                       else "bf16->f16 (RNE)", "ms": round(ms, 3),
+                                       "bytes": nbytes, "GB/s": round(gbs, 1),
+                                       "frac_of_peak": round(gbs / peak, 4)}
+        del p16, cs16, t16_src, t16_bkt
     return out
 
 
