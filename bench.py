@@ -15,11 +15,11 @@ The separate rr_unpack and rr_verify are timed after the step loop as a
 breakdown.  Inputs (33 GB of source) are far larger than L2, so no flush is
 needed between steps.
 
-End to end (`e2e`): the same step with the trainer's shards in pinned host
-memory, by two routes, both timed and the faster reported -- the copy
-engines bringing the source over in pieces while the buckets whose sources
-have landed are packed, or the pack reading the pinned shards itself over
-NVLink-C2C.
+End to end (`e2e`): the same step with the trainer's shards in host memory,
+by three routes, all timed and the fastest reported -- the copy engines
+bringing the source over in pieces while the buckets whose sources have
+landed are packed, the pack reading the pinned shards itself over
+NVLink-C2C, or the same from ordinary pageable memory where the GPU reads it.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
 
@@ -1099,12 +1099,12 @@ def run_native(args, w, bucket_bytes, world, rank, local):
                "ms_per_step": round(e2e_ms, 3), "pipelined": False}
         del host_src
     elif not args.no_e2e:
-        # Two routes for the source, both through the public API and both timed:
+        # Routes for the source, all through the public API and all timed:
         # copy engines (the source copied into HBM in pieces, each piece packed
-        # as it lands) and direct (the pack reads the pinned shards itself).
-        # Which is faster depends on the machine: where the copy engines run below
-        # the link, the SMs' own loads still reach it.  The line reports the
-        # faster and carries both.
+        # as it lands), direct (the pack reads the pinned shards itself) and
+        # direct from pageable memory (below).  Which is fastest depends on the
+        # machine: where the copy engines run below the link, the SMs' own
+        # loads still reach it.  The line reports the fastest and carries all.
         host_src = torch.empty(buf.flat.numel(), dtype=torch.uint8, pin_memory=True)
         host_src.copy_(buf.flat)
         routes = {}
