@@ -115,6 +115,90 @@ def random_tp_layout(seed: int):
     return desc
 
 
+def random_medium_layout(seed: int, max_elems: int = 6 << 20):
+    """Odd shapes at the scale where a bucket holds many work items: parameters
+    of up to about 1500 x 3000 elements (at most ``max_elems`` in all), buckets
+    of 64 KiB to 4 MiB.  Each parameter reaches the rollout ranks in one of the
+    ways a TP rollout cuts a model: rows split over the ranks (column-parallel;
+    long contiguous runs), columns split over the ranks (row-parallel; one
+    slice per rank in every row, wide or narrow), replicated whole, or fused
+    with the next parameter into one tensor (like qkv or gate_up), rows split.
+    Row counts that do not divide by TP give the last rank the remainder."""
+    rng = np.random.default_rng(seed + 9_000_011)
+    tp = int(rng.choice([1, 2, 3, 4, 8]))
+    n_params = int(rng.integers(3, 9))
+    hows = [str(h) for h in rng.choice(["rows", "cols", "whole", "fused"], size=n_params,
+                                       p=[0.3, 0.4, 0.15, 0.15])]
+    shapes = []
+    for i in range(n_params):
+        es = int(rng.choice([2, 4, 4]))
+        if hows[i] == "cols" and tp > 1:
+            # mostly 8-element multiples over a 16-byte aligned row (fan-out
+            # groups), sometimes an odd width or a ragged remainder (fallbacks)
+            w = 8 * int(rng.integers(1, 400)) if rng.random() < 0.75 else int(rng.integers(1, 900))
+            extra = 8 * int(rng.integers(1, 4)) if rng.random() < 0.3 else 0
+            dims = (int(rng.integers(1, 1500)), w * tp + extra)
+        elif rng.random() < 0.2:
+            dims = (int(rng.integers(1, 5000)),)
+        else:
+            dims = (int(rng.integers(1, 1500)), int(rng.integers(1, 3000)))
+        shapes.append([dims, es])
+    total = sum(int(np.prod(d)) for d, _ in shapes)
+    if total > max_elems:                     # shrink rows until the layout fits
+        f = max_elems / total
+        for s in shapes:
+            d = s[0]
+            s[0] = (max(1, int(d[0] * f)),) + tuple(d[1:])
+    params = [(f"p{i}", tuple(d), es) for i, (d, es) in enumerate(shapes)]
+
+    def row_split(rows):
+        h = rows // tp
+        return [(r * h, (rows - r * h) if r == tp - 1 else h) for r in range(tp)]
+
+    tensors, i = [[] for _ in range(tp)], 0
+    while i < n_params:
+        dims = params[i][1]
+        rows = dims[0]
+        cols = int(np.prod(dims[1:])) if len(dims) > 1 else 1
+        how = hows[i]
+        if how == "cols" and cols >= tp:
+            w = cols // tp
+            c_off = 8 * int(rng.integers(0, (cols - w * tp) // 8 + 1))
+            for r in range(tp):
+                tensors[r].append((f"p{i}.cols", r, [(i, 0, rows, c_off + r * w, w)]))
+        elif how == "whole" or (how == "cols" and cols < tp):
+            for r in range(tp):
+                tensors[r].append((f"p{i}.whole", r, [(i, 0, rows, 0, cols)]))
+        elif how == "fused" and i + 1 < n_params:
+            j = i + 1
+            cj = int(np.prod(params[j][1][1:])) if len(params[j][1]) > 1 else 1
+            for r, ((a0, an), (b0, bn)) in enumerate(zip(row_split(rows),
+                                                          row_split(params[j][1][0]))):
+                tensors[r].append((f"p{i}+p{j}", r, [(i, a0, an, 0, cols), (j, b0, bn, 0, cj)]))
+            i += 1
+        else:
+            for r, (r0, nr) in enumerate(row_split(rows)):
+                tensors[r].append((f"p{i}.rows", r, [(i, r0, nr, 0, cols)]))
+        i += 1
+    flat_tensors = []
+    for r in range(tp):
+        order = rng.permutation(len(tensors[r])) if rng.random() < 0.5 else range(len(tensors[r]))
+        flat_tensors += [tensors[r][k] for k in order]
+    sharding = str(rng.choice(["flat", "flat", "rows", "units"]))
+    desc = dict(params=params, tensors=flat_tensors, tp=tp, sharding=sharding,
+                n_shards=int(rng.integers(1, 9)),
+                bucket_bytes=int(rng.choice([1 << 16, (1 << 16) + 8, 1 << 18, 1 << 20,
+                                             (3 << 20) + 16, 4 << 20])),
+                align_bytes=int(rng.choice([16, 16, 16, 4, 32])),
+                tensor_align=int(rng.choice([256, 256, 16, 2])),
+                seed=int(rng.integers(1, 1 << 20)), specials=bool(rng.random() < 0.5))
+    if sharding == "units":
+        n_units = int(rng.integers(1, n_params + 1))
+        units = np.concatenate([np.arange(n_units), rng.integers(0, n_units, n_params - n_units)])
+        desc["units"] = [int(u) for u in rng.permutation(units)]
+    return desc
+
+
 def degenerate_layout(sharding: str = "flat"):
     """Parameters with a zero dimension, empty blocks, and destination tensors
     with no elements at all, among ordinary ones."""

@@ -121,6 +121,30 @@ def test_random_row_parallel_layouts_exercise_fan_out():
     assert heads > 100 and plain_rows > 3
 
 
+@pytest.mark.parametrize("seed", range(6))
+def test_tables_medium_layouts(seed):
+    """Medium random layouts (many items per bucket, wide and narrow
+    row-parallel slices, fused blocks) through both tables."""
+    run_and_compare(U.random_medium_layout(seed), grid_blocks=11)
+
+
+def test_medium_layouts_reach_every_item_kind():
+    """The first 40 medium seeds (the GPU parity cases) produce fan-out groups,
+    buckets of many items, every TP degree and every sharding."""
+    heads = many = 0
+    tps, shardings = set(), set()
+    for seed in range(40):
+        desc = U.random_medium_layout(seed)
+        p = host_plan(desc)
+        items, _ = p.export_pack_full()
+        heads += int(np.sum((items["kind"] == U.ITEM_FAN_F32) | (items["kind"] == U.ITEM_FAN_BF16)))
+        many += int(len(items) > 8 * max(1, p.n_buckets))
+        tps.add(desc["tp"])
+        shardings.add(desc["sharding"])
+    assert heads >= 50 and many >= 5
+    assert tps == {1, 2, 3, 4, 8} and shardings == {"flat", "rows", "units"}
+
+
 @pytest.mark.parametrize("sharding", ["flat", "rows", "units"])
 def test_degenerate_layout(sharding):
     """Zero-size parameters, empty blocks and empty tensors."""
