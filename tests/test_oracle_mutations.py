@@ -68,6 +68,25 @@ MUTATIONS = [
     ("unit parameters not aligned",
      "                local = align_up(local, a);\n                L->param_offset[p] = local;",
      "                L->param_offset[p] = local + 0 * a;"),
+    ("block column offset dropped", "int64_t col = B->col0 + jj % B->ncols;",
+     "int64_t col = jj % B->ncols;"),
+    ("rows strided by the block width, not the parameter's",
+     "source_bits(L, S, B->param, row * P->cols + col, &bits);",
+     "source_bits(L, S, B->param, row * B->ncols + col, &bits);"),
+    ("FSDP2 chunk read from the shard's start, not the parameter's",
+     "int64_t o = L->param_offset[p] + (e - s * L->chunk_rows[p] * P->cols) * es;",
+     "int64_t o = (e - s * L->chunk_rows[p] * P->cols) * es;"),
+    ("flat byte read from the shard before", "*out = S->shards[s][f % L->shard_bytes];",
+     "*out = S->shards[s > 0 ? s - 1 : 0][f % L->shard_bytes];"),
+    ("checksum drops the last word", "for (int64_t k = 0; k + 8 <= n; k += 8) {",
+     "for (int64_t k = 0; k + 16 <= n; k += 8) {"),
+    ("bucket gaps and tail not zero", "memset(out, 0, (size_t)L->bucket_bytes);",
+     "memset(out, 0xFF, (size_t)L->bucket_bytes);"),
+    ("unpack reads big-endian elements",
+     "out[j - j0] = (uint16_t)(bucket[o] | (bucket[o + 1] << 8));",
+     "out[j - j0] = (uint16_t)(bucket[o + 1] | (bucket[o] << 8));"),
+    ("verify reports the last bad bucket, not the first", "if (bad == 0) *first_bad = b;",
+     "*first_bad = b;"),
     ("f16: NaN loses the quiet bit",
      "return (uint16_t)(sign | 0x7E00u | ((mag >> 13) & 0x01FFu));",
      "return (uint16_t)(sign | 0x7C00u | ((mag >> 13) & 0x01FFu));"),
