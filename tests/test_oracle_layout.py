@@ -3,6 +3,9 @@ unpack and verify (RobustRL Section 5.2.1 steps 1-2 and Section 5.2.2).
 
 The paper prints no worked example for this path, so the oracle is pinned by:
 * a hand-worked example (tests/golden/layout_worked_example.json);
+* hand-derived Qwen3 manifests and rollout tensor lists
+  (tests/golden/qwen3_rollout_worked_example.json): registration order, fused
+  orders, TP row and column cuts, KV replication, expert parallel, units;
 * a PyTorch restatement of the rollout layout (vLLM-style cat/chunk/stack on
   whole parameter tensors, then byte-level concatenation into streams and
   buckets) on scaled-down workloads of every family;
@@ -405,6 +408,31 @@ def test_verify_flags_damage():
     swapped = buckets.copy()
     swapped[[2, 3]] = swapped[[3, 2]]
     assert L.verify(swapped, cs) == (2, 2)
+
+
+QWEN3_GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "qwen3_rollout_worked_example.json")
+
+
+def test_qwen3_layout_worked_example():
+    """The oracle's Qwen3 manifest, FSDP1 units and rollout tensors (Section 7.1:
+    a verl FSDP trainer, a vLLM TP rollout) against the hand-derived lists.
+    Looked up through ``oracle.qwen3`` at call time."""
+    g = json.load(open(QWEN3_GOLDEN))
+    base = None
+    for case in g["cases"]:
+        shape = synth.ModelShape("golden", **case["shape"])
+        params = oracle.qwen3.manifest(shape, 4)
+        tensors = oracle.qwen3.rollout_tensors(shape, params, case["tp"], ep=case["ep"])
+        got = [[n, r, [list(b) for b in bl]] for n, r, bl in tensors]
+        if "manifest" in case:
+            assert [[n, list(d)] for n, d, _ in params] == case["manifest"], case["name"]
+            assert oracle.qwen3.layer_units(params) == case["units"], case["name"]
+            assert got == case["tensors"], case["name"]
+            base = case["tensors"]
+        else:                                # expert parallel: only w13 and w2 change
+            want = {(n, r): bl for n, r, bl in case["tensors_differing_from_tp"]}
+            expect = [[n, r, want.get((n, r), bl)] for n, r, bl in base]
+            assert got == expect, case["name"]
 
 
 def test_layout_rejects_bad_input():

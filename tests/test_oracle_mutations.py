@@ -5,9 +5,12 @@ dropped term, a wrong bit, a transposed index, a missed alignment, a wrong
 byte order -- builds that copy on its own, and runs a battery of the pins
 (hand-worked golden examples, the brute-force cast check, the PyTorch
 restatement of the layout, the numpy checksum, round trip and verify) against
-it.  Every planted mistake must make the battery fail, and the real oracle must
-pass it.  Nothing here touches a GPU.
+it.  The same is done with mistakes planted in a copy of oracle/qwen3.py (the
+oracle's Qwen3 manifest and rollout layout), loaded in place of the real
+module.  Every planted mistake must make the battery fail, and the real oracle
+must pass it.  Nothing here touches a GPU.
 """
+import importlib.util
 import os
 import subprocess
 
@@ -20,6 +23,7 @@ from tests import test_oracle_layout as layout_pins
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 SRC = os.path.join(ROOT, "oracle", "rr_oracle.c")
+QWEN3_SRC = os.path.join(ROOT, "oracle", "qwen3.py")
 
 # (name, text in rr_oracle.c, replacement)
 MUTATIONS = [
@@ -105,6 +109,63 @@ MUTATIONS = [
 ]
 
 
+# (name, text in qwen3.py, replacement)
+QWEN3_MUTATIONS = [
+    ("qkv fused as [q; v; k]",
+     'kv_slice(a + "k_proj.weight", r),\n                                              '
+     'kv_slice(a + "v_proj.weight", r)]',
+     'kv_slice(a + "v_proj.weight", r),\n                                              '
+     'kv_slice(a + "k_proj.weight", r)]'),
+    ("gate_up fused as [up; gate]",
+     'row_slice(m + "gate_proj.weight", r),\n                                                      '
+     'row_slice(m + "up_proj.weight", r)]',
+     'row_slice(m + "up_proj.weight", r),\n                                                      '
+     'row_slice(m + "gate_proj.weight", r)]'),
+    ("w13 stacked as [up; gate]",
+     'w13 += [row_slice(f"{ex}{e}.gate_proj.weight", r),\n                                '
+     'row_slice(f"{ex}{e}.up_proj.weight", r)]',
+     'w13 += [row_slice(f"{ex}{e}.up_proj.weight", r),\n                                '
+     'row_slice(f"{ex}{e}.gate_proj.weight", r)]'),
+    ("o_proj cut by rows", '[col_slice(a + "o_proj.weight", r)]',
+     '[row_slice(a + "o_proj.weight", r)]'),
+    ("expert down_proj cut by rows", 'w2.append(col_slice(f"{ex}{e}.down_proj.weight", r))',
+     'w2.append(row_slice(f"{ex}{e}.down_proj.weight", r))'),
+    ("column slices all start at column 0", "return (index[name], 0, rows, r * n, n)",
+     "return (index[name], 0, rows, 0, n)"),
+    ("row slices in reverse rank order", "return (index[name], r * n, n, 0, cols)",
+     "return (index[name], (tp - 1 - r) * n, n, 0, cols)"),
+    ("KV heads shared round-robin", "h = r * shape.n_kv // tp", "h = r % shape.n_kv"),
+    ("experts dealt round-robin under EP", "for e in range(r * per, (r + 1) * per):",
+     "for e in range(r, E, tp):"),
+    ("layer i put in unit i, with the root", "out.append(layer + 1)", "out.append(layer)"),
+    ("router registered after the experts",
+     '            out.append((pre + "mlp.gate.weight", (E, H), elem_bytes))\n'
+     '            for e in range(E):\n'
+     '                ep = pre + f"mlp.experts.{e}."\n'
+     '                out += [\n'
+     '                    (ep + "gate_proj.weight", (Im, H), elem_bytes),\n'
+     '                    (ep + "up_proj.weight", (Im, H), elem_bytes),\n'
+     '                    (ep + "down_proj.weight", (H, Im), elem_bytes),\n'
+     '                ]\n',
+     '            for e in range(E):\n'
+     '                ep = pre + f"mlp.experts.{e}."\n'
+     '                out += [\n'
+     '                    (ep + "gate_proj.weight", (Im, H), elem_bytes),\n'
+     '                    (ep + "up_proj.weight", (Im, H), elem_bytes),\n'
+     '                    (ep + "down_proj.weight", (H, Im), elem_bytes),\n'
+     '                ]\n'
+     '            out.append((pre + "mlp.gate.weight", (E, H), elem_bytes))\n'),
+    ("down_proj registered before up_proj",
+     '                (pre + "mlp.up_proj.weight", (I, H), elem_bytes),\n'
+     '                (pre + "mlp.down_proj.weight", (H, I), elem_bytes),\n',
+     '                (pre + "mlp.down_proj.weight", (H, I), elem_bytes),\n'
+     '                (pre + "mlp.up_proj.weight", (I, H), elem_bytes),\n'),
+    ("o_proj registered as [Q, hidden]", '(pre + "self_attn.o_proj.weight", (H, Q), elem_bytes)',
+     '(pre + "self_attn.o_proj.weight", (Q, H), elem_bytes)'),
+    ("tied models keep lm_head", "    if not shape.tied:\n        out.append",
+     "    if True:\n        out.append"),
+]
+
 def battery():
     """A compact run of the pins.  Returns the name of the first that fails, or None."""
     checks = [
@@ -131,6 +192,9 @@ def battery():
         ("unit shard size edge", layout_pins.test_unit_shard_size_rule_edge),
         ("restatement tiny-units", lambda: layout_pins.test_oracle_matches_restatement("tiny-units")),
         ("restatement EP", lambda: layout_pins.test_oracle_matches_restatement("tiny-moe-ep4")),
+        ("restatement KV replication",
+         lambda: layout_pins.test_oracle_matches_restatement("tiny-moe-kvrep")),
+        ("qwen3 golden", layout_pins.test_qwen3_layout_worked_example),
         ("round trip", lambda: layout_pins.test_unpack_of_pack_is_reshard("tiny-tp4")),
         ("shard invariance", lambda: layout_pins.test_shard_count_invariance(7, "flat")),
     ]
@@ -151,6 +215,18 @@ def _with_library(path):
         oracle._lib = saved
 
 
+def _with_qwen3(path):
+    spec = importlib.util.spec_from_file_location("oracle_qwen3_mutant", path)
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    saved = oracle.qwen3
+    oracle.qwen3 = mod
+    try:
+        return battery()
+    finally:
+        oracle.qwen3 = saved
+
+
 def test_real_oracle_passes_the_battery():
     assert battery() is None
 
@@ -165,4 +241,14 @@ def test_planted_mistake_is_caught(name, old, new, tmp_path):
     subprocess.check_call(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-o", str(so),
                            str(mutant)])
     failed = _with_library(str(so))
+    assert failed is not None, f"no pin catches: {name}"
+
+
+@pytest.mark.parametrize("name,old,new", QWEN3_MUTATIONS, ids=[m[0] for m in QWEN3_MUTATIONS])
+def test_planted_layout_mistake_is_caught(name, old, new, tmp_path):
+    src = open(QWEN3_SRC).read()
+    assert src.count(old) == 1, f"mutation site not found exactly once: {name}"
+    mutant = tmp_path / "qwen3_mutant.py"
+    mutant.write_text(src.replace(old, new))
+    failed = _with_qwen3(str(mutant))
     assert failed is not None, f"no pin catches: {name}"
