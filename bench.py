@@ -475,17 +475,19 @@ def _event_ms(fn, stream, reps=3):
 
 def next_rows(rr, H, w, plan, buf, t_src, t_bkt, t_dst, stream, peak):
     """Timings of the paths beyond the step: a resumed pull (the middle third of
-    the buckets packed and checked-unpacked again, Section 5.2.2), a relay
+    the buckets packed and checked-unpacked again, Section 5.2.2; with TP > 1,
+    also one rank's buckets packed again), a relay
     re-pack (a rollout holding the TP=1 image serves a TP=4 one straight from
     the buckets it pulled, Section 5.2.1), and the pack for a float16 rollout.
     Algorithmic bytes as for the step."""
     import numpy as np
     import torch
     out = {}
-    n = plan.n_buckets // 3
-    b0 = n
-    if n:
-        items, _ = plan.export_pack()
+    items, _ = plan.export_pack()
+
+    def pack_range(b0, n):
+        # Algorithmic bytes of a range pack: its items' source reads and its
+        # whole buckets written.
         sel = (items["bucket"] >= b0) & (items["bucket"] < b0 + n) & (items["kind"] <= 3)
         es = np.where(items["kind"][sel] <= 1, 4, 2)
         read = int((items["row_len"][sel].astype(np.int64) * items["n_rows"][sel] * es).sum())
@@ -493,9 +495,13 @@ def next_rows(rr, H, w, plan, buf, t_src, t_bkt, t_dst, stream, peak):
         ms = _event_ms(lambda: rr.rr_pack_range(plan, b0, n, t_src, t_bkt, buf.checksums,
                                                 stream), stream)
         gbs = (read + wrote) / (ms * 1e-3) / 1e9
-        out["resume_pack_range"] = {"buckets": [b0, b0 + n], "ms": round(ms, 3),
-                                    "bytes": read + wrote, "GB/s": round(gbs, 1),
-                                    "frac_of_peak": round(gbs / peak, 4)}
+        return {"buckets": [b0, b0 + n], "ms": round(ms, 3), "bytes": read + wrote,
+                "GB/s": round(gbs, 1), "frac_of_peak": round(gbs / peak, 4)}, wrote
+
+    n = plan.n_buckets // 3
+    b0 = n
+    if n:
+        out["resume_pack_range"], wrote = pack_range(b0, n)
         uitems, _ = plan.export_unpack()
         usel = ((uitems["bucket"] >= b0) & (uitems["bucket"] < b0 + n)
                 & ((uitems["kind"] == 6) | (uitems["kind"] == 7)))
@@ -511,6 +517,14 @@ def next_rows(rr, H, w, plan, buf, t_src, t_bkt, t_dst, stream, peak):
         out["resume_unpack_verify_range"] = {"buckets": [b0, b0 + n], "ms": round(ms, 3),
                                              "bytes": wrote + uwrote, "GB/s": round(gbs, 1),
                                              "frac_of_peak": round(gbs / peak, 4)}
+    if plan.tp > 1:
+        # A rollout rank that reconnects pulls its own buckets only (Section
+        # 5.2.2): rank tp/2's whole range.
+        r = plan.tp // 2
+        fb = list(plan.first_bucket_of_rank) + [plan.n_buckets]
+        if fb[r + 1] > fb[r]:
+            row, _ = pack_range(fb[r], fb[r + 1] - fb[r])
+            out["resume_one_rank_pack_range"] = {"rank": r, **row}
     if w.tp == 1 and plan.bucket_bytes % 16 == 0:
         from paper_2512_22492_gb300 import layouts
         m2, s2, d2 = layouts.qwen3_relay(w.shape, 1, 4, from_plan=plan)
